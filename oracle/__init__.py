@@ -1,0 +1,230 @@
+"""CPU oracle for the TSS / TRE hot path (ctypes wrapper around tre_oracle.cpp).
+
+TEST INFRASTRUCTURE ONLY: the slow, plain reference the CUDA library is
+checked against. Only tests/, __graft_entry__.smoke() and the CPU-baseline
+leg of bench.py may import this package. It shares no code with the library.
+
+Functions take and return numpy arrays laid out [window][model] (row-major).
+Pins: every function here is checked in tests/test_oracle_*.py against values
+the paper prints (Sec. II-B, Fig. 1 pair), hand-derived traces, closed forms,
+brute force on tiny inputs and invariants; see those files for which pin
+covers which step.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+import subprocess
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "tre_oracle.cpp")
+_OUT = os.path.join(_HERE, "_build", "liboracle.so")
+
+CRIT, NOM, SURP, IDLE = 0, 1, 2, 3
+RESCUE, REBALANCE = 1, 2
+
+MOVE_DTYPE = np.dtype([("window", np.int32), ("recv", np.int32), ("donor", np.int32),
+                       ("kind", np.int32), ("seq", np.int32)])
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle with plain IEEE arithmetic (no contraction, no fast-math)."""
+    if force or not os.path.exists(_OUT) or os.path.getmtime(_OUT) < os.path.getmtime(_SRC):
+        os.makedirs(os.path.dirname(_OUT), exist_ok=True)
+        tmp = _OUT + f".tmp{os.getpid()}"
+        subprocess.run(["g++", "-O2", "-std=c++17", "-ffp-contract=off", "-fno-fast-math",
+                        "-fPIC", "-shared", _SRC, "-o", tmp], check=True)
+        os.replace(tmp, _OUT)
+    return _OUT
+
+
+_lib = None
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        _lib = C.CDLL(build())
+        assert _lib.orc_move_size() == MOVE_DTYPE.itemsize
+    return _lib
+
+
+def _p(a):
+    return None if a is None else a.ctypes.data_as(C.c_void_p)
+
+
+def _i32(a):
+    return np.ascontiguousarray(a, dtype=np.int32)
+
+
+def _req_cols(req):
+    return [_i32(req[k]) for k in ("model", "t_arr_ms", "t_start_ms", "t_first_ms",
+                                   "t_end_ms", "L_in", "L_out")]
+
+
+def reduce_requests(req, M, window_ms, K):
+    """Per-window prompt (P) and decode (D) token counts and running (A) /
+    waiting (W) gauges from request records. Returns (P, D, A, W, drops[3])."""
+    cols = _req_cols(req)
+    n = len(cols[0])
+    P, D, A, W = (np.zeros((K, M), np.int32) for _ in range(4))
+    drops = np.zeros(3, np.int64)
+    rc = lib().orc_reduce_requests(C.c_int32(M), C.c_int32(window_ms), C.c_int32(K),
+                                   C.c_int64(n), *[_p(c) for c in cols],
+                                   _p(P), _p(D), _p(A), _p(W), _p(drops))
+    if rc:
+        raise ValueError("oracle: bad arguments")
+    return P, D, A, W, drops
+
+
+def slo_counts_requests(req, M, window_ms, K, slo_ttft_ms):
+    cols = _req_cols(req)
+    n_arr, n_met = np.zeros((K, M), np.int32), np.zeros((K, M), np.int32)
+    rc = lib().orc_slo_counts_requests(C.c_int32(M), C.c_int32(window_ms), C.c_int32(K),
+                                       C.c_int64(len(cols[0])), *[_p(c) for c in cols],
+                                       _p(_i32(slo_ttft_ms)), _p(n_arr), _p(n_met))
+    if rc:
+        raise ValueError("oracle: bad arguments")
+    return n_arr, n_met
+
+
+def reduce_events(ev, M, window_ms, K):
+    model, req = _i32(ev["model"]), _i32(ev["req"])
+    t_s = np.ascontiguousarray(ev["t_s"], dtype=np.float32)
+    phase = np.ascontiguousarray(ev["phase"], dtype=np.uint8)
+    rm, rta = _i32(ev["req_model"]), _i32(ev["req_t_arr_ms"])
+    P, D, A, W = (np.zeros((K, M), np.int32) for _ in range(4))
+    drops = np.zeros(3, np.int64)
+    rc = lib().orc_reduce_events(C.c_int32(M), C.c_int32(window_ms), C.c_int32(K),
+                                 C.c_int64(len(model)), _p(model), _p(req), _p(t_s), _p(phase),
+                                 C.c_int64(len(rm)), _p(rm), _p(rta),
+                                 _p(P), _p(D), _p(A), _p(W), _p(drops))
+    if rc:
+        raise ValueError("oracle: bad arguments")
+    return P, D, A, W, drops
+
+
+def slo_counts_events(ev, M, window_ms, K, slo_ttft_ms):
+    rm, rta, rtt = _i32(ev["req_model"]), _i32(ev["req_t_arr_ms"]), _i32(ev["req_ttft_ms"])
+    n_arr, n_met = np.zeros((K, M), np.int32), np.zeros((K, M), np.int32)
+    rc = lib().orc_slo_counts_events(C.c_int32(M), C.c_int32(window_ms), C.c_int32(K),
+                                     C.c_int64(len(rm)), _p(rm), _p(rta), _p(rtt),
+                                     _p(_i32(slo_ttft_ms)), _p(n_arr), _p(n_met))
+    if rc:
+        raise ValueError("oracle: bad arguments")
+    return n_arr, n_met
+
+
+def _suffix(dtype):
+    dtype = np.dtype(dtype)
+    if dtype == np.float32:
+        return "f32"
+    if dtype == np.float64:
+        return "f64"
+    raise ValueError(dtype)
+
+
+def _prof(profile, M, dtype):
+    return {k: np.ascontiguousarray(np.broadcast_to(np.asarray(profile[k], dtype=dtype), (M,)))
+            for k in ("w_p", "w_q", "alpha", "theta", "tau_crit", "tau_surplus")}
+
+
+def score(P, D, A, W, profile, window_ms, dtype=np.float64, carry=None):
+    """Eq. 1 raw TSS -> EMA -> Eq. 2 Z -> region. Returns (S, Z, cls, recv).
+    carry: optional dict {"S": [M], "init": [M] uint8} updated in place."""
+    K, M = P.shape
+    pr = _prof(profile, M, dtype)
+    S = np.zeros((K, M), dtype)
+    Z = np.zeros((K, M), dtype)
+    cls = np.zeros((K, M), np.uint8)
+    recv = np.zeros(K, np.int32)
+    f = getattr(lib(), "orc_score_" + _suffix(dtype))
+    rc = f(C.c_int32(M), C.c_int32(window_ms), C.c_int32(K),
+           *[_p(_i32(a)) for a in (P, D, A, W)],
+           *[_p(pr[k]) for k in ("w_p", "w_q", "alpha", "theta", "tau_crit", "tau_surplus")],
+           _p(carry["S"]) if carry else None, _p(carry["init"]) if carry else None,
+           _p(S), _p(Z), _p(cls), _p(recv))
+    if rc:
+        raise ValueError("oracle: bad arguments")
+    return S, Z, cls, recv
+
+
+def calibrate(S, cls, n_arr, n_met, ok_frac=0.95, reliability=0.95):
+    """theta per model (Sec. III-B). Returns (theta[M], n_degenerate)."""
+    K, M = S.shape
+    theta = np.zeros(M, S.dtype)
+    deg = np.zeros(1, np.int64)
+    f = getattr(lib(), "orc_calibrate_" + _suffix(S.dtype))
+    rc = f(C.c_int32(M), C.c_int32(K), _p(np.ascontiguousarray(S)),
+           _p(np.ascontiguousarray(cls, np.uint8)), _p(_i32(n_arr)), _p(_i32(n_met)),
+           C.c_double(ok_frac), C.c_double(reliability), _p(theta), _p(deg))
+    if rc:
+        raise ValueError("oracle: bad arguments")
+    return theta, int(deg[0])
+
+
+def select_moves(Z, cls, tau_crit, tau_surplus, window_ms, budget, r0, r_min, footprint,
+                 fast_ms=5000, slow_ms=10000, pacing_cap=1, cap=None):
+    """Open-loop TRE move selection. Returns (moves structured array, r_final, status)."""
+    K, M = Z.shape
+    dtype = Z.dtype
+    tc = np.ascontiguousarray(np.broadcast_to(np.asarray(tau_crit, dtype), (M,)))
+    ts = np.ascontiguousarray(np.broadcast_to(np.asarray(tau_surplus, dtype), (M,)))
+    r = _i32(r0).copy()
+    if cap is None:
+        cap = 1024
+    while True:
+        moves = np.zeros(cap, MOVE_DTYPE)
+        n = np.zeros(1, np.int64)
+        rr = r.copy()
+        f = getattr(lib(), "orc_select_" + _suffix(dtype))
+        rc = f(C.c_int32(M), C.c_int32(window_ms), C.c_int32(K), _p(np.ascontiguousarray(Z)),
+               _p(np.ascontiguousarray(cls, np.uint8)), _p(tc), _p(ts), C.c_int64(budget),
+               _p(_i32(r_min)), _p(_i32(footprint)), C.c_int32(fast_ms), C.c_int32(slow_ms),
+               C.c_int32(pacing_cap), _p(rr), _p(moves), C.c_int64(cap), _p(n))
+        if rc == 1:
+            raise ValueError("oracle: bad arguments")
+        if rc == 4:
+            cap = int(n[0])
+            continue
+        return moves[: int(n[0])], rr, rc
+
+
+def pipeline_requests(req, M, window_ms, K, profile, slo_ttft_ms, dtype, ok_frac=0.95,
+                      reliability=0.95):
+    """Reduce -> score (S) -> calibrate theta -> score (Z, class, receiver)."""
+    P, D, A, W, drops = reduce_requests(req, M, window_ms, K)
+    n_arr, n_met = slo_counts_requests(req, M, window_ms, K, slo_ttft_ms)
+    S, _, cls, _ = score(P, D, A, W, profile, window_ms, dtype)
+    theta, deg = calibrate(S, cls, n_arr, n_met, ok_frac, reliability)
+    prof = dict(profile)
+    prof["theta"] = theta
+    S, Z, cls, recv = score(P, D, A, W, prof, window_ms, dtype)
+    return {"P": P, "D": D, "A": A, "W": W, "drops": drops, "n_arr": n_arr, "n_met": n_met,
+            "S": S, "Z": Z, "cls": cls, "recv": recv, "theta": theta, "degenerate": deg}
+
+
+def sweep(traces, M, duration_ms, window_ms_list, tau_crit_list, pacing_list, w_p, w_q,
+          tau_surplus, alpha_list, slo_ttft_ms, budget, r0, r_min, footprint, fast_ms=5000,
+          slow_ms=10000, dtype=np.float32, ok_frac=0.95, reliability=0.95, series_hook=None):
+    """Open-loop sweep: for every trace and window length, reduce the records at
+    that window length directly, calibrate theta, score; then run the move
+    selection for every (rescue threshold, pacing cap) setting."""
+    out = {"series": [], "instances": []}
+    for ti, req in enumerate(traces):
+        for wi, win in enumerate(window_ms_list):
+            K = duration_ms // int(win)
+            prof = {"w_p": w_p, "w_q": w_q, "alpha": alpha_list[wi], "theta": 1.0,
+                    "tau_crit": tau_crit_list[0], "tau_surplus": tau_surplus}
+            s = pipeline_requests(req, M, int(win), K, prof, slo_ttft_ms, dtype, ok_frac,
+                                  reliability)
+            s["trace"], s["window_ms"], s["K"] = ti, int(win), K
+            out["series"].append(s if series_hook is None else series_hook(s))
+            for tau in tau_crit_list:
+                for cap in pacing_list:
+                    mv, rf, _ = select_moves(s["Z"], s["cls"], tau, tau_surplus, int(win), budget,
+                                             r0, r_min, footprint, fast_ms, slow_ms, int(cap))
+                    out["instances"].append({"moves": mv, "r_final": rf})
+    return out

@@ -1,0 +1,510 @@
+// CPU oracle for the Token Service Share (TSS) signal and TRE move selection.
+//
+// TEST INFRASTRUCTURE ONLY. This file is the slow, plain reference that the
+// CUDA library is checked against. Only the tests, the smoke check and the
+// CPU-baseline leg of the benchmark may load it; the library never does, and
+// it shares no code, header, table or helper with the library.
+//
+// Every step follows the paper's definitions in the paper's order, with the
+// readings listed below where the paper is silent. Floating-point expressions
+// are evaluated one IEEE operation at a time in the caller's precision T
+// (float or double); build with -ffp-contract=off so no multiply-add is fused.
+//
+// Readings (the paper does not fix these):
+//  * time base: all times are integer milliseconds; window k covers
+//    [k*win, (k+1)*win), windows start at t = 0 (Eq. 1 "window of width Delta").
+//  * prompt tokens of a request are all counted at its first-token time; decode
+//    token j (0 <= j < L_out) is emitted at t_first + floor(j*(t_end-t_first)/(L_out-1))
+//    (a single decode token is at t_first). Counters become window deltas
+//    (Sec. V-B).
+//  * running (A) and waiting (W) counts are gauges read at the last millisecond
+//    of each window: running on [t_start, t_end), waiting on [t_arr, t_start)
+//    (Sec. III-A, Sec. V-B).
+//  * the demand denominator is floored at one request (Sec. II-B: the raw
+//    inverse sits "under the signal's floor"); a window with no tokens and no
+//    requests is IDLE.
+//  * EMA: S = alpha*raw + (1-alpha)*S_prev, started at the first non-idle window
+//    and held through idle windows (Sec. III-B).
+//  * regions: critical if Z < tau_crit, surplus if Z > tau_surplus, else nominal
+//    (Sec. III-B); idle windows form their own class.
+//  * theta: the smallest smoothed TSS value s such that, among calibration
+//    windows with S >= s, the healthy fraction reaches the reliability target
+//    (Sec. III-B "smallest smoothed TSS that achieves target SLO reliability").
+//  * control ticks: a window ends a fast (slow) tick when a multiple of
+//    fast_ms (slow_ms) falls in (k*win, (k+1)*win] (Sec. IV-B, Sec. V-B).
+//  * rescue, rebalance and bounded transfer as in Sec. IV-B/IV-C, Eq. 3.
+
+#include <algorithm>
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <utility>
+#include <vector>
+
+namespace {
+
+constexpr uint8_t kCrit = 0, kNom = 1, kSurp = 2, kIdle = 3;
+constexpr int kRescue = 1, kRebalance = 2;
+
+struct Move {          // one released donor replica (or pool draw) of a transition
+  int32_t window, recv, donor, kind, seq;
+};
+
+// window of a non-negative millisecond time, clamped to [0, K]
+int64_t win_of(int64_t t, int64_t win, int64_t K) {
+  int64_t b = t / win;
+  return b > K ? K : b;
+}
+
+// --------------------------------------------------------------------------
+// Window reduction of request records (Eq. 1 inputs, Sec. V-B).
+// drops[0] = arrival outside [0, K*win), drops[1] = bad model id,
+// drops[2] = times out of order or bad lengths.
+// --------------------------------------------------------------------------
+int reduce_requests(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* model,
+                    const int32_t* t_arr, const int32_t* t_start, const int32_t* t_first,
+                    const int32_t* t_end, const int32_t* L_in, const int32_t* L_out,
+                    int32_t* P, int32_t* D, int32_t* A, int32_t* W, int64_t* drops) {
+  if (M < 1 || win < 1 || K < 0 || n < 0) return 1;
+  const int64_t span = (int64_t)K * win;
+  std::vector<uint32_t> p((size_t)K * M, 0), d((size_t)K * M, 0);
+  std::vector<int64_t> dA((size_t)(K + 1) * M, 0), dW((size_t)(K + 1) * M, 0);
+  for (int64_t i = 0; i < n; ++i) {
+    const int64_t m = model[i];
+    if (m < 0 || m >= M) { drops[1]++; continue; }
+    const int64_t ta = t_arr[i], ts = t_start[i], tf = t_first[i], te = t_end[i];
+    if (ta < 0 || ta >= span) { drops[0]++; continue; }
+    if (!(ta <= ts && ts <= tf && tf <= te) || L_in[i] < 0 || L_out[i] < 1) {
+      drops[2]++;
+      continue;
+    }
+    // prompt tokens, all at the first-token time
+    if (tf < span) p[(size_t)(tf / win) * M + m] += (uint32_t)L_in[i];
+    // decode tokens, one at a time at their emission times
+    const int64_t L = L_out[i], dur = te - tf;
+    for (int64_t j = 0; j < L; ++j) {
+      const int64_t tj = (L == 1) ? tf : tf + (j * dur) / (L - 1);
+      if (tj < span) d[(size_t)(tj / win) * M + m] += 1u;
+    }
+    // gauges: +1 where a state begins, -1 where it ends (window of the
+    // transition time); the running sum over windows is the gauge value at
+    // each window's last millisecond
+    dW[(size_t)win_of(ta, win, K) * M + m] += 1;
+    dW[(size_t)win_of(ts, win, K) * M + m] -= 1;
+    dA[(size_t)win_of(ts, win, K) * M + m] += 1;
+    dA[(size_t)win_of(te, win, K) * M + m] -= 1;
+  }
+  for (int64_t m = 0; m < M; ++m) {
+    int64_t a = 0, w = 0;
+    for (int64_t k = 0; k < K; ++k) {
+      a += dA[(size_t)k * M + m];
+      w += dW[(size_t)k * M + m];
+      A[(size_t)k * M + m] = (int32_t)a;
+      W[(size_t)k * M + m] = (int32_t)w;
+    }
+  }
+  for (size_t x = 0; x < (size_t)K * M; ++x) {
+    P[x] = (int32_t)p[x];
+    D[x] = (int32_t)d[x];
+  }
+  return 0;
+}
+
+// Calibration counts of request records: arrivals per (arrival window, model)
+// and how many of them met the TTFT bound of their model's SLO class.
+int slo_counts_requests(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* model,
+                        const int32_t* t_arr, const int32_t* t_start, const int32_t* t_first,
+                        const int32_t* t_end, const int32_t* L_in, const int32_t* L_out,
+                        const int32_t* slo_ttft_ms, int32_t* n_arr, int32_t* n_met) {
+  if (M < 1 || win < 1 || K < 0 || n < 0) return 1;
+  const int64_t span = (int64_t)K * win;
+  for (size_t x = 0; x < (size_t)K * M; ++x) n_arr[x] = n_met[x] = 0;
+  for (int64_t i = 0; i < n; ++i) {
+    const int64_t m = model[i];
+    if (m < 0 || m >= M) continue;
+    const int64_t ta = t_arr[i], ts = t_start[i], tf = t_first[i], te = t_end[i];
+    if (ta < 0 || ta >= span) continue;
+    if (!(ta <= ts && ts <= tf && tf <= te) || L_in[i] < 0 || L_out[i] < 1) continue;
+    const size_t x = (size_t)(ta / win) * M + m;
+    n_arr[x] += 1;
+    if (tf - ta <= slo_ttft_ms[m]) n_met[x] += 1;
+  }
+  return 0;
+}
+
+// --------------------------------------------------------------------------
+// Window reduction of token-level events (one record per emitted token).
+// --------------------------------------------------------------------------
+int reduce_events(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* model,
+                  const int32_t* req, const float* t_s, const uint8_t* phase, int64_t n_req,
+                  const int32_t* req_model, const int32_t* req_t_arr, int32_t* P, int32_t* D,
+                  int32_t* A, int32_t* W, int64_t* drops) {
+  if (M < 1 || win < 1 || K < 0 || n < 0 || n_req < 0) return 1;
+  const double span = (double)((int64_t)K * win);
+  std::vector<uint32_t> p((size_t)K * M, 0), d((size_t)K * M, 0);
+  std::vector<int64_t> first((size_t)n_req, INT64_MAX), last((size_t)n_req, -1);
+  for (int64_t i = 0; i < n; ++i) {
+    const int64_t m = model[i], r = req[i];
+    if (m < 0 || m >= M || r < 0 || r >= n_req || req_model[r] != m) { drops[1]++; continue; }
+    // exact millisecond tick of the float timestamp: the product of a float
+    // and 1000 is exact in double
+    const double ms = std::floor((double)t_s[i] * 1000.0);
+    if (!(ms >= 0.0 && ms < span)) { drops[0]++; continue; }
+    if (phase[i] > 1) { drops[2]++; continue; }
+    const int64_t t = (int64_t)ms;
+    const size_t x = (size_t)(t / win) * M + m;
+    if (phase[i] == 0) p[x] += 1u; else d[x] += 1u;
+    if (t < first[r]) first[r] = t;
+    if (t > last[r]) last[r] = t;
+  }
+  std::vector<int64_t> dA((size_t)(K + 1) * M, 0), dW((size_t)(K + 1) * M, 0);
+  for (int64_t r = 0; r < n_req; ++r) {
+    if (last[r] < 0) continue;                       // no valid event
+    const int64_t m = req_model[r], ta = req_t_arr[r];
+    if (!(ta >= 0 && ta <= first[r])) { drops[2]++; continue; }
+    dW[(size_t)win_of(ta, win, K) * M + m] += 1;
+    dW[(size_t)win_of(first[r], win, K) * M + m] -= 1;
+    dA[(size_t)win_of(first[r], win, K) * M + m] += 1;
+    dA[(size_t)win_of(last[r], win, K) * M + m] -= 1;
+  }
+  for (int64_t m = 0; m < M; ++m) {
+    int64_t a = 0, w = 0;
+    for (int64_t k = 0; k < K; ++k) {
+      a += dA[(size_t)k * M + m];
+      w += dW[(size_t)k * M + m];
+      A[(size_t)k * M + m] = (int32_t)a;
+      W[(size_t)k * M + m] = (int32_t)w;
+    }
+  }
+  for (size_t x = 0; x < (size_t)K * M; ++x) {
+    P[x] = (int32_t)p[x];
+    D[x] = (int32_t)d[x];
+  }
+  return 0;
+}
+
+int slo_counts_events(int32_t M, int32_t win, int32_t K, int64_t n_req, const int32_t* req_model,
+                      const int32_t* req_t_arr, const int32_t* req_ttft,
+                      const int32_t* slo_ttft_ms, int32_t* n_arr, int32_t* n_met) {
+  if (M < 1 || win < 1 || K < 0 || n_req < 0) return 1;
+  const int64_t span = (int64_t)K * win;
+  for (size_t x = 0; x < (size_t)K * M; ++x) n_arr[x] = n_met[x] = 0;
+  for (int64_t r = 0; r < n_req; ++r) {
+    const int64_t m = req_model[r], ta = req_t_arr[r];
+    if (m < 0 || m >= M || ta < 0 || ta >= span) continue;
+    const size_t x = (size_t)(ta / win) * M + m;
+    n_arr[x] += 1;
+    if (req_ttft[r] <= slo_ttft_ms[m]) n_met[x] += 1;
+  }
+  return 0;
+}
+
+// --------------------------------------------------------------------------
+// Eq. 1 (raw TSS), EMA smoothing, Eq. 2 (Z = S / theta) and the regions.
+// S_carry / init_carry (may be null) hold the smoothing state across calls.
+// recv (may be null): per window, the Eq. 3 receiver argmin Z over non-idle
+// models (lowest index on ties), -1 if every model is idle.
+// --------------------------------------------------------------------------
+template <class T>
+int score(int32_t M, int32_t win, int32_t K, const int32_t* P, const int32_t* D,
+          const int32_t* A, const int32_t* W, const T* w_p, const T* w_q, const T* alpha,
+          const T* theta, const T* tau_crit, const T* tau_surplus, T* S_carry,
+          uint8_t* init_carry, T* S_out, T* Z_out, uint8_t* cls_out, int32_t* recv) {
+  if (M < 1 || win < 1 || K < 0) return 1;
+  const T dt = (T)win / (T)1000;                     // window length in seconds
+  for (int64_t m = 0; m < M; ++m) {
+    T S = S_carry ? S_carry[m] : (T)0;
+    bool init = init_carry ? init_carry[m] != 0 : false;
+    if (!init) S = (T)0;
+    const T a = alpha[m];
+    const T b = (T)1 - a;
+    for (int64_t k = 0; k < K; ++k) {
+      const size_t x = (size_t)k * M + m;
+      const bool idle = P[x] == 0 && D[x] == 0 && A[x] == 0 && W[x] == 0;
+      if (!idle) {
+        const T r_pre = (T)P[x] / dt;                  // prefill token rate
+        const T r_dec = (T)D[x] / dt;                  // decode token rate
+        const T svc = w_p[m] * r_pre;
+        const T num = svc + r_dec;
+        const T qw = w_q[m] * (T)W[x];
+        T den = (T)A[x] + qw;
+        if (den < (T)1) den = (T)1;                    // demand floor of one request
+        const T raw = num / den;
+        if (!init) {
+          S = raw;
+          init = true;
+        } else {
+          const T x1 = a * raw;
+          const T x2 = b * S;
+          S = x1 + x2;
+        }
+      }
+      const T Z = S / theta[m];
+      S_out[x] = S;
+      Z_out[x] = Z;
+      uint8_t c;
+      if (idle) c = kIdle;
+      else if (Z < tau_crit[m]) c = kCrit;
+      else if (Z > tau_surplus[m]) c = kSurp;
+      else c = kNom;
+      cls_out[x] = c;
+    }
+    if (S_carry) S_carry[m] = S;
+    if (init_carry) init_carry[m] = init ? 1 : 0;
+  }
+  if (recv) {
+    for (int64_t k = 0; k < K; ++k) {
+      int32_t best = -1;
+      for (int64_t m = 0; m < M; ++m) {
+        const size_t x = (size_t)k * M + m;
+        if (cls_out[x] == kIdle) continue;
+        if (best < 0 || Z_out[x] < Z_out[(size_t)k * M + best]) best = (int32_t)m;
+      }
+      recv[k] = best;
+    }
+  }
+  return 0;
+}
+
+// --------------------------------------------------------------------------
+// theta calibration (Sec. III-B): per model, among windows that had at least
+// one arrival, are not idle and have S > 0, find the smallest S value s such
+// that the windows with S >= s are healthy in at least a `reliability`
+// fraction. A window is healthy when at least `ok_frac` of its arrivals met
+// the TTFT bound. Falls back to max S (no s qualifies) or 1 (no candidate),
+// counting the model in *degenerate.
+// --------------------------------------------------------------------------
+template <class T>
+int calibrate(int32_t M, int32_t K, const T* S, const uint8_t* cls, const int32_t* n_arr,
+              const int32_t* n_met, double ok_frac, double reliability, T* theta,
+              int64_t* degenerate) {
+  if (M < 1 || K < 0) return 1;
+  for (int64_t m = 0; m < M; ++m) {
+    std::vector<std::pair<T, int>> cand;
+    for (int64_t k = 0; k < K; ++k) {
+      const size_t x = (size_t)k * M + m;
+      if (cls[x] == kIdle || n_arr[x] < 1 || !(S[x] > (T)0)) continue;
+      const int healthy = (double)n_met[x] >= ok_frac * (double)n_arr[x] ? 1 : 0;
+      cand.push_back({S[x], healthy});
+    }
+    if (cand.empty()) {
+      theta[m] = (T)1;
+      (*degenerate)++;
+      continue;
+    }
+    std::sort(cand.begin(), cand.end(),
+              [](const std::pair<T, int>& u, const std::pair<T, int>& v) { return u.first > v.first; });
+    int64_t H = 0, C = 0;
+    bool found = false;
+    T best = (T)0;
+    size_t i = 0;
+    while (i < cand.size()) {                // one step per distinct value, descending
+      const T s = cand[i].first;
+      while (i < cand.size() && cand[i].first == s) {
+        C += 1;
+        H += cand[i].second;
+        ++i;
+      }
+      if ((double)H >= reliability * (double)C) {
+        best = s;
+        found = true;
+      }
+    }
+    if (found) {
+      theta[m] = best;
+    } else {
+      theta[m] = cand.front().first;
+      (*degenerate)++;
+    }
+  }
+  return 0;
+}
+
+// --------------------------------------------------------------------------
+// TRE move selection (Sec. IV-B dual-speed control, Eq. 3, Sec. IV-C bounded
+// pairwise transfer), open loop over a scored trace. Z and the idle class come
+// from the scored windows; the critical/surplus regions are re-derived here
+// from the given thresholds so one scored series serves many settings.
+// r (in/out) holds routable replicas; the idle pool is budget - sum(g*r).
+// Emits one Move per released donor replica, or one with donor = -1 for a
+// transition served from the idle pool. Returns 4 if more than `cap` moves.
+// --------------------------------------------------------------------------
+template <class T>
+struct Walk {
+  int32_t M;
+  const T* Zk;                 // Z of the current window
+  const uint8_t* ck;           // class of the current window (only kIdle is used)
+  const T* tau_crit;
+  const T* tau_surplus;
+  const int32_t* r_min;
+  const int32_t* g;
+
+  uint8_t region(int32_t m) const {
+    if (ck[m] == kIdle) return kIdle;
+    if (Zk[m] < tau_crit[m]) return kCrit;
+    if (Zk[m] > tau_surplus[m]) return kSurp;
+    return kNom;
+  }
+  // donor preference: idle models (lowest index), then surplus by Z
+  // descending, then nominal by Z descending (nominal only above the
+  // receiver's Z when `nom_above` is set); never critical, never the receiver,
+  // never below the replica floor.
+  int32_t pick_donor(const std::vector<int64_t>& r, int32_t recv, bool nom_above) const {
+    for (int32_t m = 0; m < M; ++m)
+      if (m != recv && region(m) == kIdle && r[m] > r_min[m]) return m;
+    int32_t best = -1;
+    for (int32_t m = 0; m < M; ++m)
+      if (m != recv && region(m) == kSurp && r[m] > r_min[m] && (best < 0 || Zk[m] > Zk[best]))
+        best = m;
+    if (best >= 0) return best;
+    for (int32_t m = 0; m < M; ++m) {
+      if (m == recv || region(m) != kNom || r[m] <= r_min[m]) continue;
+      if (nom_above && !(Zk[m] > Zk[recv])) continue;
+      if (best < 0 || Zk[m] > Zk[best]) best = m;
+    }
+    return best;
+  }
+};
+
+template <class T>
+int select_moves(int32_t M, int32_t win, int32_t K, const T* Z, const uint8_t* cls,
+                 const T* tau_crit, const T* tau_surplus, int64_t budget, const int32_t* r_min,
+                 const int32_t* footprint, int32_t fast_ms, int32_t slow_ms, int32_t pacing_cap,
+                 int32_t* r_inout, Move* moves, int64_t cap, int64_t* n_moves) {
+  if (M < 1 || win < 1 || K < 0 || fast_ms < 1 || slow_ms < 1 || pacing_cap < 0) return 1;
+  std::vector<int64_t> r(M);
+  int64_t used = 0;
+  for (int32_t m = 0; m < M; ++m) {
+    if (r_inout[m] < 0 || footprint[m] < 1 || r_min[m] < 0) return 1;
+    r[m] = r_inout[m];
+    used += (int64_t)footprint[m] * r[m];
+  }
+  if (used > budget) return 1;
+  int64_t free_pool = budget - used;
+  int64_t nm = 0;
+  Walk<T> wk{M, nullptr, nullptr, tau_crit, tau_surplus, r_min, footprint};
+  auto emit = [&](int64_t k, int32_t recv, int32_t donor, int kind, int seq) {
+    if (nm < cap) moves[nm] = Move{(int32_t)k, recv, donor, kind, seq};
+    ++nm;
+  };
+  for (int64_t k = 0; k < K; ++k) {
+    const int64_t lo = k * (int64_t)win, hi = (k + 1) * (int64_t)win;
+    const bool fast = hi / fast_ms > lo / fast_ms;
+    const bool slow = hi / slow_ms > lo / slow_ms;
+    if (!fast && !slow) continue;
+    wk.Zk = Z + (size_t)k * M;
+    wk.ck = cls + (size_t)k * M;
+    int32_t recv = -1;
+    int kind = 0;
+    bool nom_above = false;
+    if (fast) {                                  // rescue: lowest Z among critical models
+      for (int32_t m = 0; m < M; ++m)
+        if (wk.region(m) == kCrit && (recv < 0 || wk.Zk[m] < wk.Zk[recv])) recv = m;
+      if (recv >= 0) kind = kRescue;
+    }
+    if (kind == 0 && slow) {                     // rebalance: Eq. 3 over non-idle models
+      for (int32_t m = 0; m < M; ++m)
+        if (wk.region(m) != kIdle && (recv < 0 || wk.Zk[m] < wk.Zk[recv])) recv = m;
+      if (recv >= 0 && wk.Zk[recv] < (T)1) {
+        kind = kRebalance;
+        nom_above = true;
+      }
+    }
+    if (kind == 0) continue;
+    for (int32_t seq = 0; seq < pacing_cap; ++seq) {
+      const int64_t need = footprint[recv];
+      if (free_pool >= need) {                   // idle capacity first
+        free_pool -= need;
+        r[recv] += 1;
+        emit(k, recv, -1, kind, seq);
+        continue;
+      }
+      // release donors one replica at a time until the receiver's footprint
+      // fits; abandon the transition if the eligible donors cannot cover it
+      std::vector<int64_t> rr = r;
+      int64_t f = free_pool;
+      std::vector<int32_t> rel;
+      bool ok = true;
+      while (f < need) {
+        const int32_t d = wk.pick_donor(rr, recv, nom_above);
+        if (d < 0) { ok = false; break; }
+        rr[d] -= 1;
+        f += footprint[d];
+        rel.push_back(d);
+      }
+      if (!ok) break;
+      r = rr;
+      free_pool = f - need;
+      r[recv] += 1;
+      for (int32_t d : rel) emit(k, recv, d, kind, seq);
+    }
+  }
+  for (int32_t m = 0; m < M; ++m) r_inout[m] = (int32_t)r[m];
+  *n_moves = nm;
+  return nm > cap ? 4 : 0;
+}
+
+}  // namespace
+
+extern "C" {
+
+int orc_reduce_requests(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* model,
+                        const int32_t* t_arr, const int32_t* t_start, const int32_t* t_first,
+                        const int32_t* t_end, const int32_t* L_in, const int32_t* L_out,
+                        int32_t* P, int32_t* D, int32_t* A, int32_t* W, int64_t* drops) {
+  return reduce_requests(M, win, K, n, model, t_arr, t_start, t_first, t_end, L_in, L_out, P, D,
+                         A, W, drops);
+}
+
+int orc_slo_counts_requests(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* model,
+                            const int32_t* t_arr, const int32_t* t_start, const int32_t* t_first,
+                            const int32_t* t_end, const int32_t* L_in, const int32_t* L_out,
+                            const int32_t* slo, int32_t* n_arr, int32_t* n_met) {
+  return slo_counts_requests(M, win, K, n, model, t_arr, t_start, t_first, t_end, L_in, L_out,
+                             slo, n_arr, n_met);
+}
+
+int orc_reduce_events(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* model,
+                      const int32_t* req, const float* t_s, const uint8_t* phase, int64_t n_req,
+                      const int32_t* req_model, const int32_t* req_t_arr, int32_t* P, int32_t* D,
+                      int32_t* A, int32_t* W, int64_t* drops) {
+  return reduce_events(M, win, K, n, model, req, t_s, phase, n_req, req_model, req_t_arr, P, D,
+                       A, W, drops);
+}
+
+int orc_slo_counts_events(int32_t M, int32_t win, int32_t K, int64_t n_req,
+                          const int32_t* req_model, const int32_t* req_t_arr,
+                          const int32_t* req_ttft, const int32_t* slo, int32_t* n_arr,
+                          int32_t* n_met) {
+  return slo_counts_events(M, win, K, n_req, req_model, req_t_arr, req_ttft, slo, n_arr, n_met);
+}
+
+#define ORC_TYPED(SUF, T)                                                                          \
+  int orc_score_##SUF(int32_t M, int32_t win, int32_t K, const int32_t* P, const int32_t* D,      \
+                      const int32_t* A, const int32_t* W, const T* w_p, const T* w_q,             \
+                      const T* alpha, const T* theta, const T* tau_crit, const T* tau_surplus,    \
+                      T* S_carry, uint8_t* init_carry, T* S, T* Z, uint8_t* cls, int32_t* recv) { \
+    return score<T>(M, win, K, P, D, A, W, w_p, w_q, alpha, theta, tau_crit, tau_surplus,         \
+                    S_carry, init_carry, S, Z, cls, recv);                                         \
+  }                                                                                                \
+  int orc_calibrate_##SUF(int32_t M, int32_t K, const T* S, const uint8_t* cls,                   \
+                          const int32_t* n_arr, const int32_t* n_met, double ok_frac,             \
+                          double reliability, T* theta, int64_t* degenerate) {                    \
+    return calibrate<T>(M, K, S, cls, n_arr, n_met, ok_frac, reliability, theta, degenerate);     \
+  }                                                                                                \
+  int orc_select_##SUF(int32_t M, int32_t win, int32_t K, const T* Z, const uint8_t* cls,         \
+                       const T* tau_crit, const T* tau_surplus, int64_t budget,                   \
+                       const int32_t* r_min, const int32_t* footprint, int32_t fast_ms,           \
+                       int32_t slow_ms, int32_t pacing_cap, int32_t* r_inout, void* moves,        \
+                       int64_t cap, int64_t* n_moves) {                                            \
+    return select_moves<T>(M, win, K, Z, cls, tau_crit, tau_surplus, budget, r_min, footprint,    \
+                           fast_ms, slow_ms, pacing_cap, r_inout, static_cast<Move*>(moves), cap, \
+                           n_moves);                                                               \
+  }
+
+ORC_TYPED(f32, float)
+ORC_TYPED(f64, double)
+
+int orc_move_size(void) { return (int)sizeof(Move); }
+
+}  // extern "C"
