@@ -1,0 +1,336 @@
+#!/usr/bin/env python
+"""Benchmark: the open-loop TSS + TRE sweep on one batch of synthetic telemetry.
+
+A step is one tre_sweep call: 7 synthetic one-hour traces of ~1M request
+records each (8 models, diurnal load, a 10x burst), reduced at 100 ms and
+aggregated exactly to 0.5 / 1 / 2 s windows, theta calibrated for each of the
+28 (trace, window) series, scored, and the TRE controller run for all 256
+settings (4 window lengths x 8 rescue thresholds x 8 pacing caps) -- 1792
+controller instances. Inputs stay resident in HBM for the device-timed value;
+the e2e number copies the records in from pinned host memory and the results
+out every step.
+
+Prints one JSON line (rank 0). `--impl reference` times the CPU oracle on a
+bounded sample of the same workload instead.
+"""
+import argparse
+import ctypes as C
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import tracegen  # noqa: E402
+
+METRIC = "telemetry events/sec and model-windows/sec through TSS+selection; % of HBM peak"
+UNIT = "events/s"
+WORKLOAD = "sweep: 7 traces x 1M requests (8 models, 1 h), 4 window lengths x 8 rescue thresholds x 8 pacing caps"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=300)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--scale", type=float, default=1.0, help="request-count scale (1.0 = full)")
+    ap.add_argument("--e2e-steps", type=int, default=20)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def alphas(windows):
+    return [min(1.0, w / 5000.0) for w in windows]
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu):
+        self.gpu = gpu
+        self.proc = None
+        self.t0 = self.t1 = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def mark(self, begin):
+        if begin:
+            self.t0 = time.time()
+        else:
+            self.t1 = time.time()
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.15)
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            out = ""
+        rows = [r.split(", ") for r in out.strip().splitlines() if r.count(",") >= 8]
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = set()
+        for r in rows:
+            for i, n in enumerate(names):
+                if r[5 + i].strip().lower() == "active":
+                    reasons.add(n)
+        # samples are taken every 100 ms through warm-up and the timed loop; the
+        # loaded ones are those at or above the median of the run
+        load = [s for s in sm if s >= statistics.median(sm)] if sm else []
+        return {"sm_mhz": statistics.median(load) if load else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def run_reference(args):
+    """The CPU oracle, as it stands, on a bounded sample: one trace of the
+    workload with all window lengths and all 64 controller settings."""
+    import oracle
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    sw = tracegen.sweep_workload(scale=args.scale, n_traces=1)
+    n_rec = len(sw["traces"][0]["model"])
+
+    def step():
+        oracle.sweep(sw["traces"], sw["M"], sw["duration_ms"], sw["window_ms"], sw["tau_crit"],
+                     sw["pacing_cap"], sw["w_p"], sw["w_q"], sw["tau_surplus"],
+                     alphas(sw["window_ms"]), sw["slo_ttft_ms"], sw["budget"], sw["r0"],
+                     sw["r_min"], sw["footprint"], dtype=np.float32)
+
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    dt = time.perf_counter() - t0
+    v = n_rec * args.steps / dt
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic",
+        "config": {"workload": WORKLOAD, "sample": "1 of 7 traces, all 4 window lengths, all 64 settings"},
+        "cpu_baseline": {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": "1 trace (~1M records), 4 window lengths, 64 settings per step"},
+        "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}))
+
+
+def cpu_baseline(scale):
+    import oracle
+    sw = tracegen.sweep_workload(scale=scale, n_traces=1)
+    n_rec = len(sw["traces"][0]["model"])
+    t0 = time.perf_counter()
+    oracle.sweep(sw["traces"], sw["M"], sw["duration_ms"], sw["window_ms"], sw["tau_crit"],
+                 sw["pacing_cap"], sw["w_p"], sw["w_q"], sw["tau_surplus"],
+                 alphas(sw["window_ms"]), sw["slo_ttft_ms"], sw["budget"], sw["r0"], sw["r_min"],
+                 sw["footprint"], dtype=np.float32)
+    dt = time.perf_counter() - t0
+    return {"value": n_rec / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"1 of the 7 traces ({n_rec} records), all 4 window lengths, all 64 settings; {dt:.1f} s"}
+
+
+def phase_bytes(sw, n_records_per_trace, M):
+    """Algorithmic bytes per launch of each phase (what the method must read and
+    write once): see the design doc, 'Roofline'."""
+    K = [sw["duration_ms"] // int(w) for w in sw["window_ms"]]
+    Kb = min(K) and sw["duration_ms"] // int(min(sw["window_ms"]))
+    n_series = len(sw["traces"]) * len(K)
+    mw = sum(K) * len(sw["traces"]) * M
+    return {
+        # records in (7 int32 columns) + P, D, A and W diffs, SLO counts out at the base grid
+        "reduce": float(np.mean(n_records_per_trace)) * 28 + Kb * M * 24,
+        # counts in, S + idle flag out, per series (average over series)
+        "score": mw * (16 + 4 + 1) / n_series,
+        # S + class + SLO counts in per series
+        "calibrate": mw * (4 + 1 + 8) / n_series,
+        "normalize": mw * (4 + 1 + 4 + 1) / n_series,
+    }
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        return run_reference(args)
+    import torch
+    import torch.distributed as dist
+
+    import paper_2609_29160_gb300 as tre
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl")
+    lib = tre.load()
+    lib.tre_trace_enable.argtypes = [C.c_int]
+
+    class Trace(C.Structure):
+        _fields_ = [("n_phases", C.c_int32), ("name", C.c_char_p * 9), ("ms", C.c_double * 9),
+                    ("calls", C.c_int64 * 9), ("launches", C.c_int64 * 9)]
+    lib.tre_trace_collect.argtypes = [C.POINTER(Trace)]
+
+    # each rank sweeps its own 7 traces (independent problems: weak scaling)
+    sw = tracegen.sweep_workload(scale=args.scale, seed0=100 + 7 * rank)
+    M = sw["M"]
+    win = sw["window_ms"]
+    al = alphas(win)
+    n_rec = [len(t["model"]) for t in sw["traces"]]
+    total_rec = int(sum(n_rec))
+    K = [sw["duration_ms"] // int(w) for w in win]
+    model_windows = sum(K) * len(sw["traces"]) * M
+    n_inst = len(sw["traces"]) * len(win) * len(sw["tau_crit"]) * len(sw["pacing_cap"])
+    moves_cap = 512
+    dev_traces = [{k: torch.as_tensor(v).cuda() for k, v in t.items()} for t in sw["traces"]]
+    stream = torch.cuda.current_stream()
+
+    def step(traces, ws=None):
+        return tre.tre_sweep(traces, M, sw["duration_ms"], win, al, sw["tau_crit"],
+                             sw["pacing_cap"], sw["w_p"], sw["w_q"], sw["tau_surplus"],
+                             sw["slo_ttft_ms"], sw["budget"], sw["r0"], sw["r_min"],
+                             sw["footprint"], dtype="f32", moves_cap=moves_cap, ws=ws)
+
+    out = step(dev_traces)
+    ws = out["ws"]
+    for _ in range(args.warmup):
+        out = step(dev_traces, ws)
+    torch.cuda.synchronize()
+
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    lib.tre_trace_enable(1)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks.mark(True)
+    ev0.record(stream)
+    for _ in range(args.steps):
+        out = step(dev_traces, ws)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    clocks.mark(False)
+    if world > 1:
+        dist.barrier()
+    ms = ev0.elapsed_time(ev1)
+    tr = Trace()
+    lib.tre_trace_collect(C.byref(tr))
+    lib.tre_trace_enable(0)
+    clk = clocks.stop()
+    if world > 1:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    ms_step = ms / args.steps
+    value = total_rec * world * args.steps / (ms / 1e3)
+    mw_s = model_windows * world * args.steps / (ms / 1e3)
+    phases = {tr.name[i].decode(): {"ms": tr.ms[i], "calls": tr.calls[i],
+                                    "launches": tr.launches[i]} for i in range(tr.n_phases)}
+    launches = int(sum(p["launches"] for p in phases.values()))
+
+    # dominant kernel phase and its roofline
+    hbm, peak_kind = peaks()
+    pb = phase_bytes(sw, n_rec, M)
+    dom = max(phases, key=lambda k: phases[k]["ms"])
+    share = phases[dom]["ms"] / max(ms, 1e-9)
+    if dom in pb and phases[dom]["calls"]:
+        per_launch_ms = phases[dom]["ms"] / phases[dom]["calls"]
+        achieved = pb[dom] / (per_launch_ms / 1e3) / 1e9
+        roof = {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                "frac": achieved / hbm, "traffic": None, "share_of_step": share,
+                "peak_kind": peak_kind}
+    else:
+        roof = {"bound": "latency", "kernel": dom, "achieved": None, "peak": hbm, "unit": "GB/s",
+                "frac": None, "traffic": None, "share_of_step": share, "peak_kind": peak_kind}
+    # whole-step view against HBM: algorithmic bytes of the full sweep per step
+    step_bytes = total_rec * 28 + model_windows * (16 + 4 + 4 + 1)
+    whole = {"algorithmic_bytes": step_bytes, "achieved_gbs": step_bytes / (ms_step / 1e3) / 1e9,
+             "frac": step_bytes / (ms_step / 1e3) / 1e9 / hbm}
+
+    # end to end: records in from pinned host memory, results out, every step
+    host = [{k: v.cpu().pin_memory() for k, v in t.items()} for t in dev_traces]
+    h2d = sum(v.numel() * v.element_size() for t in host for v in t.values())
+    res_host = {"n_moves": torch.empty(n_inst, dtype=torch.int64).pin_memory(),
+                "r_final": torch.empty((n_inst, M), dtype=torch.int32).pin_memory(),
+                "theta": torch.empty((len(sw["traces"]) * len(win), M),
+                                     dtype=torch.float32).pin_memory()}
+    d2h = sum(v.numel() * v.element_size() for v in res_host.values())
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.e2e_steps):
+        for d, h in zip(dev_traces, host):
+            for k in d:
+                d[k].copy_(h[k], non_blocking=True)
+        o = step(dev_traces, ws)
+        for k in res_host:
+            res_host[k].copy_(o[k], non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1) / args.e2e_steps
+    if world > 1:
+        t = torch.tensor([e2e_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+    e2e = {"value": total_rec * world / (e2e_ms / 1e3), "unit": UNIT,
+           "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+           "ms_per_step": e2e_ms}
+
+    base = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        base = cpu_baseline(args.scale)
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic",
+            "config": {"workload": WORKLOAD, "records_per_step": total_rec * world,
+                       "model_windows_per_step": model_windows * world,
+                       "controller_instances": n_inst * world, "scale": args.scale,
+                       "l2": "inputs larger than L2 (7 x 28 B x ~1M records = 196 MB per step)",
+                       "parallelism": f"independent sweeps per GPU x{world}"},
+            "model_windows_per_s": mw_s,
+            "roofline": roof, "step_roofline": whole, "phases_ms_per_step": {
+                k: p["ms"] / args.steps for k, p in phases.items() if p["calls"]},
+            "gpu_launches": launches, "clocks": clk, "e2e": e2e, "cpu_baseline": base,
+        }
+        print(json.dumps(line))
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

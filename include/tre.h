@@ -1,0 +1,282 @@
+/*
+ * tre.h -- C ABI of the GB300 Token Service Share / TRE library (libtre.so).
+ *
+ * The library computes, in batch over request telemetry, the control signal and
+ * the capacity moves of "Cross-Model Autoscaling for Shared LLM Serving"
+ * (arXiv 2609.29160):
+ *   - per-(window, model) prompt/decode token counts and running/waiting gauges
+ *     (the inputs of Eq. 1, collected as in Sec. V-B),
+ *   - raw Token Service Share (Eq. 1), its exponential smoothing (Sec. III-B),
+ *     Z = TSS / theta (Eq. 2) and the critical / nominal / surplus regions,
+ *   - the SLO calibration of the healthy boundary theta (Sec. III-B),
+ *   - the open-loop rescue / rebalance move selection with bounded pairwise
+ *     transfer under a fixed replica budget (Sec. IV-B, Eq. 3, Sec. IV-C),
+ *   - and a batched sweep of all of the above over many traces and settings.
+ *
+ * Conventions (every entry point):
+ *   - Array arguments are DEVICE pointers owned by the caller, unless a field
+ *     says "host". The library allocates nothing and keeps no state; scratch
+ *     memory comes in through `ws`.
+ *   - Workspace query: call with ws == NULL; the required size is written to
+ *     *ws_bytes and TRE_OK is returned without touching the device. With
+ *     ws != NULL, *ws_bytes must be at least that size (else TRE_ENOMEM). `ws`
+ *     must be 256-byte aligned.
+ *   - Work is enqueued on `stream` (NULL = legacy default stream) and is
+ *     asynchronous. Argument errors are detected on the host before anything
+ *     is enqueued and returned as TRE_EINVAL. Launch failures return TRE_ECUDA.
+ *   - Data problems never trap: malformed records are dropped and counted in
+ *     the device-resident `tre_diag` (added to, never reset by the library:
+ *     zero it before the first call), valid after the stream is synchronised.
+ *   - Layout of every per-window array is row-major [n_windows][n_models].
+ *   - Floating-point results are computed in the profile's dtype with one
+ *     correctly rounded IEEE operation per step and no fused multiply-add, in
+ *     the same order as the sequential definitions; results are reproducible
+ *     bit for bit.
+ * Limits: 1 <= n_models <= 1024; window_ms >= 1; n_windows * window_ms < 2^31.
+ */
+#ifndef TRE_H
+#define TRE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* tre_stream; /* a cudaStream_t */
+
+typedef enum {
+  TRE_OK = 0,
+  TRE_EINVAL = 1,    /* bad argument (host-side check, nothing enqueued) */
+  TRE_ENOMEM = 2,    /* workspace smaller than the queried size */
+  TRE_ECUDA = 3,     /* a CUDA launch or runtime call failed */
+  TRE_EOVERFLOW = 4, /* move list longer than its capacity (reported in diag.err) */
+  TRE_ETIMEOUT = 5   /* reserved: a bounded device wait gave up (reported in diag.err) */
+} tre_status;
+
+typedef enum { TRE_F32 = 0, TRE_F64 = 1 } tre_dtype;
+
+/* Region of a model in a window (Sec. III-B): Z < tau_crit critical, Z > tau_surplus
+ * surplus, otherwise nominal. A window with no tokens and no running or waiting
+ * request is IDLE: never a receiver, the first donor candidate. */
+enum { TRE_CRIT = 0, TRE_NOM = 1, TRE_SURP = 2, TRE_IDLE = 3 };
+/* Kind of a move: fast-loop rescue or slow-loop rebalance (Sec. IV-B). */
+enum { TRE_RESCUE = 1, TRE_REBALANCE = 2 };
+
+/* Window grid: window k covers [k*window_ms, (k+1)*window_ms) milliseconds. */
+typedef struct {
+  int32_t n_models;
+  int32_t window_ms;
+  int32_t n_windows;
+} tre_grid;
+
+/* Request records, structure of arrays (device, int32, length n). Times in ms.
+ * A record is valid when 0 <= model < n_models, 0 <= t_arr < n_windows*window_ms,
+ * t_arr <= t_start <= t_first <= t_end, L_in >= 0 and L_out >= 1. Prompt tokens
+ * count at t_first; decode token j is emitted at
+ * t_first + floor(j*(t_end-t_first)/(L_out-1)) (at t_first when L_out == 1). */
+typedef struct {
+  int64_t n;
+  const int32_t *model, *t_arr_ms, *t_start_ms, *t_first_ms, *t_end_ms, *L_in, *L_out;
+} tre_requests;
+
+/* Token-level events (device, length n): one record per emitted token, phase 0 =
+ * prompt (prefill), 1 = decode; t_s in float seconds (tick = floor(t_s*1000) ms,
+ * exact). The request table (device, length n_req) gives each request's model,
+ * arrival ms and TTFT ms. An event is valid when its model matches
+ * req_model[req], its tick lies inside the grid and phase <= 1. A request runs
+ * from its first to its last valid event and waits from t_arr to its first. */
+typedef struct {
+  int64_t n;
+  const int32_t *model, *req;
+  const float* t_s;
+  const uint8_t* phase;
+  int64_t n_req;
+  const int32_t *req_model, *req_t_arr_ms, *req_ttft_ms;
+} tre_events;
+
+/* Per-window counts (device, int32, [n_windows][n_models] each):
+ * P prompt tokens, D decode tokens, A running and W waiting requests read at
+ * the last millisecond of the window. Counts wrap modulo 2^32. */
+typedef struct {
+  int32_t *P, *D, *A, *W;
+} tre_counts;
+
+/* Control profile (Sec. III-B, Sec. V-B): six scalars per model, device arrays
+ * of length n_models in `dtype`. */
+typedef struct {
+  tre_dtype dtype;
+  const void *w_p, *w_q, *alpha, *theta, *tau_crit, *tau_surplus;
+} tre_profile;
+
+/* Controller (Sec. IV-B, IV-C): fixed budget in footprint units, per-model
+ * replica floor and footprint (device int32 [n_models]), cadences of the fast
+ * (rescue) and slow (rebalance) loops in ms, and the pacing cap: the most
+ * transitions per control tick (the paper's rule is 1). */
+typedef struct {
+  int64_t budget;
+  const int32_t *r_min, *footprint;
+  int32_t fast_ms, slow_ms, pacing_cap;
+} tre_ctrl;
+
+/* One move. A transition activates one receiver replica; it is served from the
+ * idle pool (donor = -1) or by releasing donor replicas, one entry per released
+ * replica, all with the same (window, seq). */
+typedef struct {
+  int32_t window;
+  int16_t recv, donor;
+  uint8_t kind, seq;
+  uint16_t reserved;
+} tre_move;
+
+/* Device-resident diagnostics (accumulated). */
+typedef struct {
+  unsigned long long dropped_range; /* record time outside the grid */
+  unsigned long long dropped_model; /* model id out of range / event-request mismatch */
+  unsigned long long dropped_order; /* times out of order, bad lengths, bad phase */
+  unsigned long long degenerate_calib; /* models whose theta fell back */
+  unsigned long long ema_resolved;  /* smoothing segments re-run to exactness */
+  int32_t err;                      /* last data-dependent error status, 0 if none */
+  int32_t reserved;
+} tre_diag;
+
+/*
+ * tss_window_reduce -- window telemetry (Sec. III-A Eq. 1 inputs; Sec. V-B:
+ * counters become window deltas, running/waiting counts are the demand).
+ * Exactly one of `req` / `ev` is non-NULL (host pointer to the descriptor).
+ * Writes out.P, out.D, out.A, out.W (all four required).
+ */
+tre_status tss_window_reduce(const tre_grid* grid, const tre_requests* req, const tre_events* ev,
+                             tre_counts out, void* ws, size_t* ws_bytes, tre_diag* diag,
+                             tre_stream stream);
+
+/*
+ * tss_score -- Eq. 1 raw TSS = (w_p*P/dt + D/dt) / max(A + w_q*W, 1) with dt the
+ * window length in seconds; smoothing S = alpha*raw + (1-alpha)*S_prev started at
+ * a model's first non-idle window and held through idle ones (Sec. III-B);
+ * Z = S / theta (Eq. 2); region per window.
+ * S_carry (dtype[n_models]) and init_carry (uint8[n_models]) carry the smoothing
+ * state in and out across calls on consecutive window ranges; both NULL = fresh.
+ * S_out, Z_out (dtype), cls_out (uint8) are [n_windows][n_models] and required.
+ * recv_out (int32[n_windows], may be NULL): the Eq. 3 receiver argmin Z over
+ * non-idle models, lowest index on ties, -1 if all idle.
+ */
+tre_status tss_score(const tre_grid* grid, const tre_counts* in, const tre_profile* prof,
+                     void* S_carry, uint8_t* init_carry, void* S_out, void* Z_out,
+                     uint8_t* cls_out, int32_t* recv_out, void* ws, size_t* ws_bytes,
+                     tre_diag* diag, tre_stream stream);
+
+/*
+ * tss_calibrate -- healthy boundary theta (Sec. III-B: the smallest smoothed TSS
+ * that achieves the target SLO reliability). Calibration windows have at least
+ * one arrival, are not idle and have S > 0. A window is healthy when at least
+ * ok_frac of the requests arriving in it met the TTFT bound slo_ttft_ms[model]
+ * (device int32[n_models]). theta[m] is the smallest S value s for which the
+ * windows with S >= s are healthy in at least a `reliability` fraction; if none
+ * qualifies theta = max S, if there is no calibration window theta = 1 (both
+ * counted in diag.degenerate_calib). S uses w_p, w_q, alpha of `prof` (theta
+ * and thresholds are ignored). Exactly one of req / ev non-NULL; `in` holds the
+ * counts of the same telemetry. theta_out: dtype[n_models] on the device.
+ */
+tre_status tss_calibrate(const tre_grid* grid, const tre_requests* req, const tre_events* ev,
+                         const tre_counts* in, const tre_profile* prof, const int32_t* slo_ttft_ms,
+                         double ok_frac, double reliability, void* theta_out, void* ws,
+                         size_t* ws_bytes, tre_diag* diag, tre_stream stream);
+
+/*
+ * tre_select_moves -- open-loop TRE controller over a scored trace (Sec. IV-B,
+ * Eq. 3, Sec. IV-C). A window ends a fast (slow) tick when a multiple of
+ * fast_ms (slow_ms) falls in (k*window_ms, (k+1)*window_ms]. At a fast tick with
+ * a critical model: rescue the critical model with the lowest Z. Otherwise at a
+ * slow tick: rebalance toward argmin Z over non-idle models if its Z < 1. Up to
+ * pacing_cap transitions per tick toward that receiver; each takes the idle
+ * pool if it covers the receiver's footprint, else releases donor replicas in
+ * the order idle models (by index), surplus by Z descending, nominal by Z
+ * descending (in rebalance only nominal models with Z above the receiver's);
+ * never a critical model, never below its floor; an uncoverable transition
+ * releases nothing and ends the tick. Regions are re-derived from Z with the
+ * profile's thresholds; only the IDLE class is taken from cls.
+ * r_inout (device int32[n_models]): routable replicas in, final replicas out;
+ * the idle pool is budget - sum(footprint*r). moves: device tre_move[moves_cap];
+ * n_moves_out (device int64[1]): number of moves produced; when it exceeds
+ * moves_cap only the first moves_cap are written and diag.err = TRE_EOVERFLOW.
+ */
+tre_status tre_select_moves(const tre_grid* grid, const void* Z, const uint8_t* cls,
+                            const tre_profile* prof, const tre_ctrl* ctrl, int32_t* r_inout,
+                            tre_move* moves, int64_t moves_cap, int64_t* n_moves_out, void* ws,
+                            size_t* ws_bytes, tre_diag* diag, tre_stream stream);
+
+/* Sweep description. Host fields are read during the call only. */
+typedef struct {
+  int32_t n_models;
+  int32_t duration_ms;               /* every window length divides it */
+  int32_t n_traces;
+  const tre_requests* traces;        /* host array [n_traces] of device column sets */
+  int32_t n_win;
+  const int32_t* window_ms;          /* host [n_win]; each a multiple of the smallest */
+  const double* alpha;               /* host [n_win]: smoothing weight per window length */
+  int32_t n_tau;
+  const double* tau_crit;            /* host [n_tau] rescue thresholds */
+  int32_t n_cap;
+  const int32_t* pacing_cap;         /* host [n_cap] */
+  tre_dtype dtype;
+  const void *w_p, *w_q, *tau_surplus; /* device [n_models] of dtype */
+  const int32_t* slo_ttft_ms;        /* device [n_models] */
+  double ok_frac, reliability;
+  tre_ctrl ctrl;                     /* budget, floors, footprints, cadences (pacing_cap unused) */
+  const int32_t* r0;                 /* device [n_models] initial replicas */
+} tre_sweep_spec;
+
+/* Sweep outputs (device). Series s = trace*n_win + w has K_s = duration_ms /
+ * window_ms[w] windows; per-window arrays concatenate the series in that order
+ * (series s starts at element n_models * sum_{s'<s} K_s'). Instance
+ * i = (s*n_tau + t)*n_cap + c. Optional arrays may be NULL. */
+typedef struct {
+  int32_t *P, *D, *A, *W; /* optional counts */
+  void *S, *Z;            /* optional dtype */
+  uint8_t* cls;           /* optional: regions with tau_crit[0] */
+  void* theta;            /* required: dtype [n_series][n_models] */
+  tre_move* moves;        /* required: [n_instances][moves_cap] */
+  int64_t moves_cap;
+  int64_t* n_moves;       /* required: [n_instances] */
+  int32_t* r_final;       /* required: [n_instances][n_models] */
+} tre_sweep_out;
+
+/*
+ * tre_sweep -- the open-loop sweep: for every trace and window length, the
+ * window reduction, calibration of theta, scoring, and then the move selection
+ * for every (rescue threshold, pacing cap) setting (controller cadences of
+ * Sec. IV-B, bounded transfer of Sec. IV-C). Equivalent, bit for bit, to calling
+ * the four entry points above per (trace, window length, setting).
+ */
+tre_status tre_sweep(const tre_sweep_spec* spec, const tre_sweep_out* out, void* ws,
+                     size_t* ws_bytes, tre_diag* diag, tre_stream stream);
+
+/* Kernel-phase tracing (host side, not thread safe). While enabled, every
+ * kernel phase an entry point enqueues is bracketed by a pair of CUDA events
+ * recorded on the call's stream, so phases can be timed on the device inside
+ * a caller's timed region. tre_trace_collect synchronises the recorded events,
+ * returns per-phase device milliseconds and kernel-launch counts accumulated
+ * since tracing was enabled (or since the last collect), and starts over.
+ * Phases: reduce, gauge_scan, aggregate, score, receiver, slo_counts,
+ * calibrate, normalize, select. No counterpart in the paper (instrumentation). */
+#define TRE_TRACE_PHASES 9
+typedef struct {
+  int32_t n_phases;
+  const char* name[TRE_TRACE_PHASES];
+  double ms[TRE_TRACE_PHASES];
+  int64_t calls[TRE_TRACE_PHASES];
+  int64_t launches[TRE_TRACE_PHASES];
+} tre_trace;
+void tre_trace_enable(int on);
+tre_status tre_trace_collect(tre_trace* out);
+
+/* Human-readable name of a status. */
+const char* tre_status_str(tre_status s);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TRE_H */

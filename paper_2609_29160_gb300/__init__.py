@@ -1,0 +1,378 @@
+"""GB300 Token Service Share / TRE library: thin Python binding of libtre.so.
+
+Functions here carry the names of the C ABI in include/tre.h and only marshal
+arguments: torch CUDA tensors become device pointers, the current torch stream
+becomes the launch stream, and workspaces are allocated with torch. Every step
+of the computation runs in the library's CUDA kernels; there is no fallback, and
+loading fails loudly when the compiled library is missing.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+
+import numpy as np
+
+from . import _build
+
+CRIT, NOM, SURP, IDLE = 0, 1, 2, 3
+RESCUE, REBALANCE = 1, 2
+F32, F64 = 0, 1
+STATUS = {0: "ok", 1: "invalid argument", 2: "workspace too small", 3: "CUDA error",
+          4: "move list overflow", 5: "device wait timed out"}
+
+
+class TreError(RuntimeError):
+    def __init__(self, fn, code):
+        super().__init__(f"{fn}: {STATUS.get(code, code)} ({code})")
+        self.code = code
+
+
+class Grid(C.Structure):
+    _fields_ = [("n_models", C.c_int32), ("window_ms", C.c_int32), ("n_windows", C.c_int32)]
+
+
+class Requests(C.Structure):
+    _fields_ = [("n", C.c_int64)] + [(k, C.c_void_p) for k in (
+        "model", "t_arr_ms", "t_start_ms", "t_first_ms", "t_end_ms", "L_in", "L_out")]
+
+
+class Events(C.Structure):
+    _fields_ = [("n", C.c_int64), ("model", C.c_void_p), ("req", C.c_void_p),
+                ("t_s", C.c_void_p), ("phase", C.c_void_p), ("n_req", C.c_int64),
+                ("req_model", C.c_void_p), ("req_t_arr_ms", C.c_void_p),
+                ("req_ttft_ms", C.c_void_p)]
+
+
+class Counts(C.Structure):
+    _fields_ = [(k, C.c_void_p) for k in ("P", "D", "A", "W")]
+
+
+class Profile(C.Structure):
+    _fields_ = [("dtype", C.c_int)] + [(k, C.c_void_p) for k in (
+        "w_p", "w_q", "alpha", "theta", "tau_crit", "tau_surplus")]
+
+
+class Ctrl(C.Structure):
+    _fields_ = [("budget", C.c_int64), ("r_min", C.c_void_p), ("footprint", C.c_void_p),
+                ("fast_ms", C.c_int32), ("slow_ms", C.c_int32), ("pacing_cap", C.c_int32)]
+
+
+class Diag(C.Structure):
+    _fields_ = [("dropped_range", C.c_uint64), ("dropped_model", C.c_uint64),
+                ("dropped_order", C.c_uint64), ("degenerate_calib", C.c_uint64),
+                ("ema_resolved", C.c_uint64), ("err", C.c_int32), ("reserved", C.c_int32)]
+
+
+class SweepSpec(C.Structure):
+    _fields_ = [("n_models", C.c_int32), ("duration_ms", C.c_int32), ("n_traces", C.c_int32),
+                ("traces", C.POINTER(Requests)), ("n_win", C.c_int32),
+                ("window_ms", C.POINTER(C.c_int32)), ("alpha", C.POINTER(C.c_double)),
+                ("n_tau", C.c_int32), ("tau_crit", C.POINTER(C.c_double)), ("n_cap", C.c_int32),
+                ("pacing_cap", C.POINTER(C.c_int32)), ("dtype", C.c_int),
+                ("w_p", C.c_void_p), ("w_q", C.c_void_p), ("tau_surplus", C.c_void_p),
+                ("slo_ttft_ms", C.c_void_p), ("ok_frac", C.c_double),
+                ("reliability", C.c_double), ("ctrl", Ctrl), ("r0", C.c_void_p)]
+
+
+class SweepOut(C.Structure):
+    _fields_ = [(k, C.c_void_p) for k in ("P", "D", "A", "W", "S", "Z", "cls", "theta", "moves")] + [
+        ("moves_cap", C.c_int64), ("n_moves", C.c_void_p), ("r_final", C.c_void_p)]
+
+
+MOVE_DTYPE = np.dtype([("window", np.int32), ("recv", np.int16), ("donor", np.int16),
+                       ("kind", np.uint8), ("seq", np.uint8), ("reserved", np.uint16)])
+DIAG_BYTES = C.sizeof(Diag)
+
+_lib = None
+EXPORTS = ("tss_window_reduce", "tss_score", "tss_calibrate", "tre_select_moves", "tre_sweep",
+           "tre_status_str")
+
+
+def library_path():
+    return _build.LIB
+
+
+def load(build_if_missing: bool = True):
+    """Load libtre.so (building it in-tree first if asked). Raises if absent."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = _build.LIB
+    if build_if_missing:
+        path = _build.build()
+    if not os.path.exists(path):
+        raise RuntimeError(f"libtre.so not built ({path}); run __graft_entry__.build()")
+    lib = C.CDLL(path)
+    P = C.c_void_p
+    lib.tss_window_reduce.argtypes = [C.POINTER(Grid), C.POINTER(Requests), C.POINTER(Events),
+                                      Counts, P, C.POINTER(C.c_size_t), P, P]
+    lib.tss_score.argtypes = [C.POINTER(Grid), C.POINTER(Counts), C.POINTER(Profile), P, P, P, P,
+                              P, P, P, C.POINTER(C.c_size_t), P, P]
+    lib.tss_calibrate.argtypes = [C.POINTER(Grid), C.POINTER(Requests), C.POINTER(Events),
+                                  C.POINTER(Counts), C.POINTER(Profile), P, C.c_double,
+                                  C.c_double, P, P, C.POINTER(C.c_size_t), P, P]
+    lib.tre_select_moves.argtypes = [C.POINTER(Grid), P, P, C.POINTER(Profile), C.POINTER(Ctrl),
+                                     P, P, C.c_int64, P, P, C.POINTER(C.c_size_t), P, P]
+    lib.tre_sweep.argtypes = [C.POINTER(SweepSpec), C.POINTER(SweepOut), P,
+                              C.POINTER(C.c_size_t), P, P]
+    for f in ("tss_window_reduce", "tss_score", "tss_calibrate", "tre_select_moves", "tre_sweep"):
+        getattr(lib, f).restype = C.c_int
+    lib.tre_status_str.argtypes = [C.c_int]
+    lib.tre_status_str.restype = C.c_char_p
+    _lib = lib
+    return lib
+
+
+# ---------------------------------------------------------------------------
+# torch plumbing
+# ---------------------------------------------------------------------------
+def _torch():
+    import torch
+    return torch
+
+
+def _ptr(t):
+    return None if t is None else C.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    torch = _torch()
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return C.c_void_p(s.cuda_stream)
+
+
+def _check(fn, code):
+    if code != 0:
+        raise TreError(fn, code)
+
+
+def _dt(dtype):
+    torch = _torch()
+    if dtype in (torch.float32, np.float32, "f32", F32):
+        return F32, torch.float32
+    if dtype in (torch.float64, np.float64, "f64", F64):
+        return F64, torch.float64
+    raise ValueError(dtype)
+
+
+def new_diag(device="cuda"):
+    """Zeroed device-resident tre_diag."""
+    torch = _torch()
+    return torch.zeros(DIAG_BYTES, dtype=torch.uint8, device=device)
+
+
+def read_diag(diag):
+    raw = diag.cpu().numpy().tobytes()
+    d = Diag.from_buffer_copy(raw)
+    return {k: getattr(d, k) for k, _ in Diag._fields_ if k != "reserved"}
+
+
+def _workspace(fn, call):
+    """Query the workspace size (ws=NULL), allocate it with torch, then call."""
+    torch = _torch()
+    size = C.c_size_t(0)
+    _check(fn, call(None, C.byref(size)))
+    ws = torch.empty(max(int(size.value), 256), dtype=torch.uint8, device="cuda")
+    _check(fn, call(_ptr(ws), C.byref(size)))
+    return ws
+
+
+def requests_struct(req):
+    """tre_requests from a dict of int32 CUDA tensors (keeps no reference)."""
+    keys = ("model", "t_arr_ms", "t_start_ms", "t_first_ms", "t_end_ms", "L_in", "L_out")
+    n = int(req["model"].numel())
+    return Requests(n, *[req[k].data_ptr() if n else None for k in keys])
+
+
+def events_struct(ev):
+    n, nr = int(ev["model"].numel()), int(ev["req_model"].numel())
+    return Events(n, ev["model"].data_ptr() if n else None, ev["req"].data_ptr() if n else None,
+                  ev["t_s"].data_ptr() if n else None, ev["phase"].data_ptr() if n else None, nr,
+                  ev["req_model"].data_ptr() if nr else None,
+                  ev["req_t_arr_ms"].data_ptr() if nr else None,
+                  ev["req_ttft_ms"].data_ptr() if nr else None)
+
+
+def _counts(c):
+    return Counts(*[c[k].data_ptr() for k in ("P", "D", "A", "W")])
+
+
+def _profile(prof, M, tdt, code):
+    torch = _torch()
+    out = {}
+    for k in ("w_p", "w_q", "alpha", "theta", "tau_crit", "tau_surplus"):
+        v = prof.get(k)
+        if v is None:
+            out[k] = None
+            continue
+        t = v if torch.is_tensor(v) else torch.as_tensor(np.broadcast_to(np.asarray(v), (M,)).copy())
+        out[k] = t.to(device="cuda", dtype=tdt).contiguous()
+    st = Profile(code, *[out[k].data_ptr() if out[k] is not None else None
+                         for k in ("w_p", "w_q", "alpha", "theta", "tau_crit", "tau_surplus")])
+    return st, out
+
+
+# ---------------------------------------------------------------------------
+# entry points
+# ---------------------------------------------------------------------------
+def tss_window_reduce(M, window_ms, K, requests=None, events=None, diag=None, stream=None,
+                      out=None):
+    """Per-window P, D, A, W ([K][M] int32 CUDA tensors) from request records or
+    token events (dicts of CUDA tensors)."""
+    torch = _torch()
+    lib = load()
+    g = Grid(M, window_ms, K)
+    if out is None:
+        out = {k: torch.empty((K, M), dtype=torch.int32, device="cuda") for k in "PDAW"}
+    diag = new_diag() if diag is None else diag
+    rq = requests_struct(requests) if requests is not None else None
+    ev = events_struct(events) if events is not None else None
+    cs = _counts(out)
+    s = _stream(stream)
+    _workspace("tss_window_reduce", lambda ws, n: lib.tss_window_reduce(
+        C.byref(g), C.byref(rq) if rq else None, C.byref(ev) if ev else None, cs, ws, n,
+        _ptr(diag), s))
+    return out
+
+
+def tss_score(counts, profile, window_ms, dtype="f32", carry=None, recv=True, diag=None,
+              stream=None):
+    """Eq. 1 -> EMA -> Eq. 2 -> regions. Returns dict S, Z, cls (and recv)."""
+    torch = _torch()
+    lib = load()
+    K, M = counts["P"].shape
+    code, tdt = _dt(dtype)
+    g = Grid(M, window_ms, K)
+    pst, keep = _profile(profile, M, tdt, code)
+    S = torch.empty((K, M), dtype=tdt, device="cuda")
+    Z = torch.empty((K, M), dtype=tdt, device="cuda")
+    cls = torch.empty((K, M), dtype=torch.uint8, device="cuda")
+    rv = torch.empty(K, dtype=torch.int32, device="cuda") if recv else None
+    diag = new_diag() if diag is None else diag
+    cs = _counts(counts)
+    s = _stream(stream)
+    _workspace("tss_score", lambda ws, n: lib.tss_score(
+        C.byref(g), C.byref(cs), C.byref(pst), _ptr(carry["S"]) if carry else None,
+        _ptr(carry["init"]) if carry else None, _ptr(S), _ptr(Z), _ptr(cls), _ptr(rv), ws, n,
+        _ptr(diag), s))
+    return {"S": S, "Z": Z, "cls": cls, "recv": rv}
+
+
+def tss_calibrate(counts, profile, window_ms, slo_ttft_ms, requests=None, events=None,
+                  dtype="f32", ok_frac=0.95, reliability=0.95, diag=None, stream=None):
+    """theta per model (CUDA tensor of dtype)."""
+    torch = _torch()
+    lib = load()
+    K, M = counts["P"].shape
+    code, tdt = _dt(dtype)
+    g = Grid(M, window_ms, K)
+    pst, keep = _profile(profile, M, tdt, code)
+    slo = torch.as_tensor(np.asarray(slo_ttft_ms, np.int32)).cuda() \
+        if not torch.is_tensor(slo_ttft_ms) else slo_ttft_ms
+    theta = torch.empty(M, dtype=tdt, device="cuda")
+    diag = new_diag() if diag is None else diag
+    rq = requests_struct(requests) if requests is not None else None
+    ev = events_struct(events) if events is not None else None
+    cs = _counts(counts)
+    s = _stream(stream)
+    _workspace("tss_calibrate", lambda ws, n: lib.tss_calibrate(
+        C.byref(g), C.byref(rq) if rq else None, C.byref(ev) if ev else None, C.byref(cs),
+        C.byref(pst), _ptr(slo), C.c_double(ok_frac), C.c_double(reliability), _ptr(theta), ws,
+        n, _ptr(diag), s))
+    return theta
+
+
+def tre_select_moves(Z, cls, profile, window_ms, budget, r0, r_min, footprint, fast_ms=5000,
+                     slow_ms=10000, pacing_cap=1, moves_cap=4096, diag=None, stream=None):
+    """Open-loop move selection. Returns (moves [n] structured numpy, r_final
+    CUDA tensor, n_moves int, diag)."""
+    torch = _torch()
+    lib = load()
+    K, M = Z.shape
+    code, tdt = _dt(Z.dtype)
+    g = Grid(M, window_ms, K)
+    pst, keep = _profile(profile, M, tdt, code)
+    dev = lambda a: (a if torch.is_tensor(a) else torch.as_tensor(np.asarray(a, np.int32))).to(
+        device="cuda", dtype=torch.int32).contiguous()
+    r = dev(r0).clone()
+    rmin, fp = dev(r_min), dev(footprint)
+    ctrl = Ctrl(int(budget), rmin.data_ptr(), fp.data_ptr(), fast_ms, slow_ms, pacing_cap)
+    moves = torch.zeros(max(moves_cap, 1) * MOVE_DTYPE.itemsize, dtype=torch.uint8, device="cuda")
+    nmv = torch.zeros(1, dtype=torch.int64, device="cuda")
+    diag = new_diag() if diag is None else diag
+    s = _stream(stream)
+    _workspace("tre_select_moves", lambda ws, n: lib.tre_select_moves(
+        C.byref(g), _ptr(Z), _ptr(cls), C.byref(pst), C.byref(ctrl), _ptr(r), _ptr(moves),
+        C.c_int64(moves_cap), _ptr(nmv), ws, n, _ptr(diag), s))
+    n = int(nmv.item())
+    mv = np.frombuffer(moves.cpu().numpy().tobytes(), dtype=MOVE_DTYPE)[: min(n, moves_cap)]
+    return mv, r, n, diag
+
+
+def tre_sweep(traces, M, duration_ms, window_ms, alpha, tau_crit, pacing_cap, w_p, w_q,
+              tau_surplus, slo_ttft_ms, budget, r0, r_min, footprint, fast_ms=5000,
+              slow_ms=10000, dtype="f32", ok_frac=0.95, reliability=0.95, moves_cap=256,
+              want_counts=False, want_S=False, diag=None, stream=None, ws=None):
+    """Batched open-loop sweep. `traces`: list of dicts of int32 CUDA tensors.
+    Returns a dict of CUDA tensors (theta, Z, cls, moves, n_moves, r_final, ...)."""
+    torch = _torch()
+    lib = load()
+    code, tdt = _dt(dtype)
+    win = np.asarray(window_ms, np.int32)
+    n_series = len(traces) * len(win)
+    K = [duration_ms // int(w) for w in win]
+    total = sum(K[i % len(win)] * M for i in range(n_series))
+    n_inst = n_series * len(tau_crit) * len(pacing_cap)
+    f = lambda v: torch.as_tensor(np.broadcast_to(np.asarray(v), (M,)).copy()).to(
+        device="cuda", dtype=tdt)
+    i32 = lambda v: torch.as_tensor(np.asarray(v, np.int32)).cuda()
+    keep = {"w_p": f(w_p), "w_q": f(w_q), "ts": f(tau_surplus), "slo": i32(slo_ttft_ms),
+            "r0": i32(r0), "rmin": i32(r_min), "fp": i32(footprint)}
+    out = {"theta": torch.empty((n_series, M), dtype=tdt, device="cuda"),
+           "Z": torch.empty(total, dtype=tdt, device="cuda"),
+           "cls": torch.empty(total, dtype=torch.uint8, device="cuda"),
+           "moves": torch.zeros(n_inst * max(moves_cap, 1) * MOVE_DTYPE.itemsize,
+                                dtype=torch.uint8, device="cuda"),
+           "n_moves": torch.zeros(n_inst, dtype=torch.int64, device="cuda"),
+           "r_final": torch.empty((n_inst, M), dtype=torch.int32, device="cuda")}
+    if want_counts:
+        for k in "PDAW":
+            out[k] = torch.empty(total, dtype=torch.int32, device="cuda")
+    if want_S:
+        out["S"] = torch.empty(total, dtype=tdt, device="cuda")
+    tr = (Requests * len(traces))(*[requests_struct(t) for t in traces])
+    wins = (C.c_int32 * len(win))(*[int(x) for x in win])
+    alph = (C.c_double * len(win))(*[float(a) for a in alpha])
+    taus = (C.c_double * len(tau_crit))(*[float(t) for t in tau_crit])
+    caps = (C.c_int32 * len(pacing_cap))(*[int(c) for c in pacing_cap])
+    ctrl = Ctrl(int(budget), keep["rmin"].data_ptr(), keep["fp"].data_ptr(), fast_ms, slow_ms, 0)
+    spec = SweepSpec(M, duration_ms, len(traces), tr, len(win), wins, alph, len(tau_crit), taus,
+                     len(pacing_cap), caps, code, keep["w_p"].data_ptr(), keep["w_q"].data_ptr(),
+                     keep["ts"].data_ptr(), keep["slo"].data_ptr(), ok_frac, reliability, ctrl,
+                     keep["r0"].data_ptr())
+    so = SweepOut(*[out[k].data_ptr() if k in out else None
+                    for k in ("P", "D", "A", "W", "S", "Z", "cls", "theta", "moves")],
+                  moves_cap, out["n_moves"].data_ptr(), out["r_final"].data_ptr())
+    diag = new_diag() if diag is None else diag
+    s = _stream(stream)
+    if ws is None:
+        ws = _workspace("tre_sweep", lambda w, n: lib.tre_sweep(C.byref(spec), C.byref(so), w, n,
+                                                                _ptr(diag), s))
+    else:
+        n = C.c_size_t(ws.numel())
+        _check("tre_sweep", lib.tre_sweep(C.byref(spec), C.byref(so), _ptr(ws), C.byref(n),
+                                          _ptr(diag), s))
+    out["ws"] = ws
+    out["diag"] = diag
+    out["K"] = K
+    out["_keep"] = (keep, tr)
+    return out
+
+
+def sweep_moves(out, n_inst, moves_cap):
+    """Host view of the sweep's move lists: list of structured arrays per instance."""
+    raw = np.frombuffer(out["moves"].cpu().numpy().tobytes(), dtype=MOVE_DTYPE)
+    raw = raw.reshape(n_inst, max(moves_cap, 1))
+    n = out["n_moves"].cpu().numpy()
+    return [raw[i, : min(int(n[i]), moves_cap)] for i in range(n_inst)]

@@ -1,0 +1,515 @@
+// C ABI of the library: argument checks, workspace layout and the launch order
+// of each entry point. Every array argument is a device pointer owned by the
+// caller; nothing here allocates.
+#include <algorithm>
+#include <cstring>
+#include <vector>
+
+#include "internal.h"
+
+using namespace tre;
+
+namespace {
+
+bool grid_ok(const tre_grid* g) {
+  return g && g->n_models >= 1 && g->n_models <= 1024 && g->window_ms >= 1 && g->n_windows >= 0 &&
+         (int64_t)g->n_windows * g->window_ms < (int64_t)2147483647;
+}
+
+bool req_ok(const tre_requests* r) {
+  if (!r || r->n < 0) return false;
+  if (r->n == 0) return true;
+  return r->model && r->t_arr_ms && r->t_start_ms && r->t_first_ms && r->t_end_ms && r->L_in &&
+         r->L_out;
+}
+
+bool ev_ok(const tre_events* e) {
+  if (!e || e->n < 0 || e->n_req < 0) return false;
+  if (e->n > 0 && !(e->model && e->req && e->t_s && e->phase)) return false;
+  if ((e->n > 0 || e->n_req > 0) && !(e->req_model && e->req_t_arr_ms && e->req_ttft_ms))
+    return false;
+  return true;
+}
+
+bool counts_ok(const tre_counts* c) { return c && c->P && c->D && c->A && c->W; }
+
+bool prof_ok(const tre_profile* p, bool need_theta_tau) {
+  if (!p || (p->dtype != TRE_F32 && p->dtype != TRE_F64)) return false;
+  if (!(p->w_p && p->w_q && p->alpha)) return false;
+  if (need_theta_tau && !(p->theta && p->tau_crit && p->tau_surplus)) return false;
+  return true;
+}
+
+ReqCols cols_of(const tre_requests* r) {
+  return ReqCols{r->model, r->t_arr_ms, r->t_start_ms, r->t_first_ms, r->t_end_ms, r->L_in,
+                 r->L_out, r->n};
+}
+
+EvCols cols_of(const tre_events* e) {
+  return EvCols{e->model, e->req, e->t_s, e->phase, e->n, e->n_req, e->req_model,
+                e->req_t_arr_ms, e->req_ttft_ms};
+}
+
+// Workspace protocol shared by every entry point: with ws == NULL report the
+// size, else check it.
+tre_status ws_check(const Arena& a, void* ws, size_t* ws_bytes, bool& query) {
+  query = ws == nullptr;
+  if (query) {
+    *ws_bytes = a.off ? a.off : 256;
+    return TRE_OK;
+  }
+  if (reinterpret_cast<uintptr_t>(ws) & 255) return TRE_EINVAL;
+  if (*ws_bytes < a.off) return TRE_ENOMEM;
+  return TRE_OK;
+}
+
+tre_status cuda_status(cudaError_t e) { return e == cudaSuccess ? TRE_OK : TRE_ECUDA; }
+
+// ---- phase tracing ----------------------------------------------------------
+enum Phase { kReduce, kScan, kAggregate, kScore, kReceiver, kSlo, kCalibrate, kNormalize,
+             kSelect };
+const char* const kPhaseName[TRE_TRACE_PHASES] = {"reduce", "gauge_scan", "aggregate", "score",
+                                                  "receiver", "slo_counts", "calibrate",
+                                                  "normalize", "select"};
+struct TraceRec {
+  int phase, launches;
+  cudaEvent_t a, b;
+};
+struct Tracer {
+  bool on = false;
+  std::vector<cudaEvent_t> pool;
+  size_t used = 0;
+  std::vector<TraceRec> recs;
+  cudaEvent_t next() {
+    if (used == pool.size()) {
+      cudaEvent_t e;
+      if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+      pool.push_back(e);
+    }
+    return pool[used++];
+  }
+};
+Tracer g_trace;
+
+// brackets the launches of one phase with events when tracing is on
+struct Scope {
+  TraceRec rec{};
+  cudaStream_t s;
+  bool live = false;
+  Scope(int phase, int launches, cudaStream_t st) : s(st) {
+    if (!g_trace.on) return;
+    rec.phase = phase;
+    rec.launches = launches;
+    rec.a = g_trace.next();
+    rec.b = g_trace.next();
+    if (!rec.a || !rec.b) return;
+    live = cudaEventRecord(rec.a, s) == cudaSuccess;
+  }
+  ~Scope() {
+    if (live && cudaEventRecord(rec.b, s) == cudaSuccess) g_trace.recs.push_back(rec);
+  }
+};
+
+template <class T> T to_t(double v) { return (T)v; }
+
+// ---- tss_score --------------------------------------------------------------
+template <class T>
+tre_status score_typed(const tre_grid* g, const tre_counts* in, const tre_profile* p,
+                       void* S_carry, uint8_t* init_carry, void* S_out, void* Z_out,
+                       uint8_t* cls_out, int32_t* recv_out, void* ws, size_t* ws_bytes,
+                       tre_diag* diag, cudaStream_t s) {
+  const int M = g->n_models, K = g->n_windows;
+  Arena a(ws);
+  ScoreWs<T> w;
+  score_ws_layout<T>(a, M, K, w);
+  bool query;
+  tre_status st = ws_check(a, ws, ws_bytes, query);
+  if (st != TRE_OK || query) return st;
+  cudaError_t e;
+  {
+    Scope sc(kScore, 5, s);
+    e = launch_score<T>(
+      M, g->window_ms, K, in->P, in->D, in->A, in->W, static_cast<const T*>(p->w_p),
+      static_cast<const T*>(p->w_q), static_cast<const T*>(p->alpha),
+      static_cast<const T*>(p->theta), static_cast<const T*>(p->tau_crit),
+      static_cast<const T*>(p->tau_surplus), static_cast<T*>(S_carry), init_carry,
+      static_cast<T*>(S_out), static_cast<T*>(Z_out), cls_out, w, diag, s);
+  }
+  if (!e && recv_out) {
+    Scope sc(kReceiver, 1, s);
+    e = launch_receiver<T>(M, K, static_cast<const T*>(Z_out), cls_out, recv_out, s);
+  }
+  return cuda_status(e);
+}
+
+// ---- tss_calibrate ----------------------------------------------------------
+template <class T>
+tre_status calibrate_typed(const tre_grid* g, const tre_requests* req, const tre_events* ev,
+                           const tre_counts* in, const tre_profile* p, const int32_t* slo_ms,
+                           double ok_frac, double rel, void* theta, void* ws, size_t* ws_bytes,
+                           tre_diag* diag, cudaStream_t s) {
+  const int M = g->n_models, K = g->n_windows;
+  Arena a(ws);
+  unsigned long long* slo = a.take<unsigned long long>((size_t)K * M);
+  T* S = a.take<T>((size_t)K * M);
+  uint8_t* cls = a.take<uint8_t>((size_t)K * M);
+  ScoreWs<T> sw;
+  score_ws_layout<T>(a, M, K, sw);
+  CalibWs<T> cw;
+  calib_ws_layout<T>(a, M, K, cw);
+  bool query;
+  tre_status st = ws_check(a, ws, ws_bytes, query);
+  if (st != TRE_OK || query) return st;
+  cudaError_t e;
+  {
+    Scope sc(kSlo, 1, s);
+    e = req ? launch_slo_requests(cols_of(req), M, g->window_ms, K, slo, slo_ms, s)
+            : launch_slo_events(cols_of(ev), M, g->window_ms, K, slo, slo_ms, s);
+  }
+  if (!e) {
+    Scope sc(kScore, 5, s);
+    e = launch_score<T>(M, g->window_ms, K, in->P, in->D, in->A, in->W,
+                        static_cast<const T*>(p->w_p), static_cast<const T*>(p->w_q),
+                        static_cast<const T*>(p->alpha), nullptr, nullptr, nullptr, nullptr,
+                        nullptr, S, nullptr, cls, sw, diag, s);
+  }
+  if (!e) {
+    Scope sc(kCalibrate, 3, s);
+    e = launch_calibrate<T>(M, K, S, cls, slo, ok_frac, rel, static_cast<T*>(theta), cw, diag, s);
+  }
+  return cuda_status(e);
+}
+
+// ---- tre_select_moves -------------------------------------------------------
+template <class T>
+tre_status select_typed(const tre_grid* g, const void* Z, const uint8_t* cls,
+                        const tre_profile* p, const tre_ctrl* c, int32_t* r_inout, tre_move* moves,
+                        int64_t cap, int64_t* n_moves, void* ws, size_t* ws_bytes, tre_diag* diag,
+                        cudaStream_t s) {
+  Arena a(ws);
+  bool query;
+  tre_status st = ws_check(a, ws, ws_bytes, query);
+  if (st != TRE_OK || query) return st;
+  WalkBatch<T> b;
+  std::memset(&b, 0, sizeof(b));
+  b.M = g->n_models;
+  b.n_inst = 1;
+  b.n_series = 1;
+  b.n_tau = 1;
+  b.n_cap = 1;
+  b.series_off[0] = 0;
+  b.series_K[0] = g->n_windows;
+  b.series_win[0] = g->window_ms;
+  b.cap_list[0] = c->pacing_cap;
+  b.Z = static_cast<const T*>(Z);
+  b.cls = cls;
+  b.tau_crit = static_cast<const T*>(p->tau_crit);
+  b.tau_surp = static_cast<const T*>(p->tau_surplus);
+  b.budget = c->budget;
+  b.r_min = c->r_min;
+  b.footprint = c->footprint;
+  b.r0 = r_inout;
+  b.fast_ms = c->fast_ms;
+  b.slow_ms = c->slow_ms;
+  b.r_out = r_inout;
+  b.moves = moves;
+  b.moves_cap = cap;
+  b.n_moves = n_moves;
+  b.diag = diag;
+  Scope sc(kSelect, 1, s);
+  return cuda_status(launch_walk<T>(b, s));
+}
+
+// ---- tre_sweep --------------------------------------------------------------
+struct SweepPlan {
+  int M, n_series, base_win, Kb;
+  std::vector<int> K, q;           // per window length
+  std::vector<int64_t> off;        // per series element offset
+  int64_t total;                   // sum over series of K*M
+  int Kmax;
+};
+
+bool sweep_plan(const tre_sweep_spec* sp, SweepPlan& pl) {
+  if (!sp || sp->n_models < 1 || sp->n_models > 1024 || sp->duration_ms < 1) return false;
+  if (sp->n_traces < 1 || !sp->traces || sp->n_win < 1 || !sp->window_ms || !sp->alpha) return false;
+  if (sp->n_tau < 1 || sp->n_tau > kMaxTau || !sp->tau_crit) return false;
+  if (sp->n_cap < 1 || sp->n_cap > kMaxCap || !sp->pacing_cap) return false;
+  if ((int64_t)sp->n_traces * sp->n_win > kMaxSeries) return false;
+  if (sp->dtype != TRE_F32 && sp->dtype != TRE_F64) return false;
+  if (!(sp->w_p && sp->w_q && sp->tau_surplus && sp->slo_ttft_ms && sp->r0)) return false;
+  if (!(sp->ctrl.r_min && sp->ctrl.footprint) || sp->ctrl.fast_ms < 1 || sp->ctrl.slow_ms < 1)
+    return false;
+  for (int c = 0; c < sp->n_cap; ++c)
+    if (sp->pacing_cap[c] < 0 || sp->pacing_cap[c] > 255) return false;
+  for (int t = 0; t < sp->n_traces; ++t)
+    if (!req_ok(&sp->traces[t])) return false;
+  pl.M = sp->n_models;
+  pl.base_win = *std::min_element(sp->window_ms, sp->window_ms + sp->n_win);
+  if (pl.base_win < 1 || sp->duration_ms % pl.base_win) return false;
+  pl.Kb = sp->duration_ms / pl.base_win;
+  pl.K.resize(sp->n_win);
+  pl.q.resize(sp->n_win);
+  pl.Kmax = 0;
+  for (int w = 0; w < sp->n_win; ++w) {
+    const int win = sp->window_ms[w];
+    if (win < 1 || win % pl.base_win || sp->duration_ms % win) return false;
+    pl.q[w] = win / pl.base_win;
+    pl.K[w] = sp->duration_ms / win;
+    pl.Kmax = std::max(pl.Kmax, pl.K[w]);
+  }
+  pl.n_series = sp->n_traces * sp->n_win;
+  pl.off.resize(pl.n_series);
+  int64_t o = 0;
+  for (int s = 0; s < pl.n_series; ++s) {
+    pl.off[s] = o;
+    o += (int64_t)pl.K[s % sp->n_win] * pl.M;
+  }
+  pl.total = o;
+  return true;
+}
+
+template <class T>
+tre_status sweep_typed(const tre_sweep_spec* sp, const SweepPlan& pl, const tre_sweep_out* out,
+                       void* ws, size_t* ws_bytes, tre_diag* diag, cudaStream_t s) {
+  const int M = pl.M;
+  Arena a(ws);
+  const size_t nb = (size_t)pl.Kb * M;
+  int32_t* Pb = a.take<int32_t>(nb);
+  int32_t* Db = a.take<int32_t>(nb);
+  int32_t* Ab = a.take<int32_t>(nb);
+  int32_t* Wb = a.take<int32_t>(nb);
+  unsigned long long* slob = a.take<unsigned long long>(nb);
+  ReduceWs rw;
+  reduce_ws_layout(a, M, pl.Kb, 0, rw);
+  const size_t tot = (size_t)pl.total;
+  int32_t* P = out->P ? out->P : a.take<int32_t>(tot);
+  int32_t* D = out->D ? out->D : a.take<int32_t>(tot);
+  int32_t* A = out->A ? out->A : a.take<int32_t>(tot);
+  int32_t* W = out->W ? out->W : a.take<int32_t>(tot);
+  T* S = out->S ? static_cast<T*>(out->S) : a.take<T>(tot);
+  T* Z = out->Z ? static_cast<T*>(out->Z) : a.take<T>(tot);
+  uint8_t* cls = out->cls ? out->cls : a.take<uint8_t>(tot);
+  uint8_t* idle = a.take<uint8_t>(tot);
+  unsigned long long* slo = a.take<unsigned long long>(tot);
+  ScoreWs<T> sw;
+  score_ws_layout<T>(a, M, pl.Kmax, sw);
+  CalibWs<T> cw;
+  calib_ws_layout<T>(a, M, pl.Kmax, cw);
+  bool query;
+  tre_status st = ws_check(a, ws, ws_bytes, query);
+  if (st != TRE_OK || query) return st;
+
+  T* theta = static_cast<T*>(out->theta);
+  cudaError_t e = cudaSuccess;
+  for (int t = 0; t < sp->n_traces && !e; ++t) {
+    {
+      Scope sc(kReduce, 1, s);
+      e = launch_reduce_requests(cols_of(&sp->traces[t]), M, pl.base_win, pl.Kb, Pb, Db, rw,
+                                 slob, sp->slo_ttft_ms, diag, s);
+    }
+    if (!e) {
+      Scope sc(kScan, 3, s);
+      e = launch_gauge_scan(M, pl.Kb, rw, Ab, Wb, s);
+    }
+    for (int w = 0; w < sp->n_win && !e; ++w) {
+      const int si = t * sp->n_win + w;
+      const size_t o = (size_t)pl.off[si];
+      Scope sc(kAggregate, 1, s);
+      e = launch_aggregate(M, pl.K[w], pl.q[w], Pb, Db, Ab, Wb, slob, P + o, D + o, A + o, W + o,
+                           slo + o, s);
+    }
+  }
+  for (int si = 0; si < pl.n_series && !e; ++si) {
+    const int w = si % sp->n_win;
+    const size_t o = (size_t)pl.off[si];
+    const int K = pl.K[w];
+    {
+      Scope sc(kScore, 5, s);
+      e = launch_score_alpha<T>(M, sp->window_ms[w], K, P + o, D + o, A + o, W + o,
+                                static_cast<const T*>(sp->w_p), static_cast<const T*>(sp->w_q),
+                                to_t<T>(sp->alpha[w]), S + o, idle + o, sw, diag, s);
+    }
+    if (!e) {
+      Scope sc(kCalibrate, 3, s);
+      e = launch_calibrate<T>(M, K, S + o, idle + o, slo + o, sp->ok_frac, sp->reliability,
+                              theta + (size_t)si * M, cw, diag, s);
+    }
+    if (!e) {
+      Scope sc(kNormalize, 1, s);
+      e = launch_normalize<T>(M, K, S + o, idle + o, theta + (size_t)si * M, nullptr,
+                              to_t<T>(sp->tau_crit[0]), static_cast<const T*>(sp->tau_surplus),
+                              Z + o, cls + o, s);
+    }
+  }
+  if (e) return TRE_ECUDA;
+  WalkBatch<T> b;
+  std::memset(&b, 0, sizeof(b));
+  b.M = M;
+  b.n_series = pl.n_series;
+  b.n_tau = sp->n_tau;
+  b.n_cap = sp->n_cap;
+  b.n_inst = pl.n_series * sp->n_tau * sp->n_cap;
+  for (int si = 0; si < pl.n_series; ++si) {
+    b.series_off[si] = pl.off[si];
+    b.series_K[si] = pl.K[si % sp->n_win];
+    b.series_win[si] = sp->window_ms[si % sp->n_win];
+  }
+  for (int t = 0; t < sp->n_tau; ++t) b.tau_list[t] = to_t<T>(sp->tau_crit[t]);
+  for (int c = 0; c < sp->n_cap; ++c) b.cap_list[c] = sp->pacing_cap[c];
+  b.Z = Z;
+  b.cls = idle;
+  b.tau_crit = nullptr;
+  b.tau_surp = static_cast<const T*>(sp->tau_surplus);
+  b.budget = sp->ctrl.budget;
+  b.r_min = sp->ctrl.r_min;
+  b.footprint = sp->ctrl.footprint;
+  b.r0 = sp->r0;
+  b.fast_ms = sp->ctrl.fast_ms;
+  b.slow_ms = sp->ctrl.slow_ms;
+  b.r_out = out->r_final;
+  b.moves = out->moves;
+  b.moves_cap = out->moves_cap;
+  b.n_moves = out->n_moves;
+  b.diag = diag;
+  Scope sc(kSelect, 1, s);
+  return cuda_status(launch_walk<T>(b, s));
+}
+
+}  // namespace
+
+extern "C" {
+
+void tre_trace_enable(int on) {
+  g_trace.on = on != 0;
+  g_trace.recs.clear();
+  g_trace.used = 0;
+}
+
+tre_status tre_trace_collect(tre_trace* out) {
+  if (!out) return TRE_EINVAL;
+  std::memset(out, 0, sizeof(*out));
+  out->n_phases = TRE_TRACE_PHASES;
+  for (int i = 0; i < TRE_TRACE_PHASES; ++i) out->name[i] = kPhaseName[i];
+  tre_status st = TRE_OK;
+  for (const TraceRec& r : g_trace.recs) {
+    float ms = 0.f;
+    if (cudaEventSynchronize(r.b) != cudaSuccess || cudaEventElapsedTime(&ms, r.a, r.b)) {
+      st = TRE_ECUDA;
+      continue;
+    }
+    out->ms[r.phase] += ms;
+    out->calls[r.phase] += 1;
+    out->launches[r.phase] += r.launches;
+  }
+  g_trace.recs.clear();
+  g_trace.used = 0;
+  return st;
+}
+
+const char* tre_status_str(tre_status s) {
+  switch (s) {
+    case TRE_OK: return "ok";
+    case TRE_EINVAL: return "invalid argument";
+    case TRE_ENOMEM: return "workspace too small";
+    case TRE_ECUDA: return "CUDA error";
+    case TRE_EOVERFLOW: return "move list overflow";
+    case TRE_ETIMEOUT: return "device wait timed out";
+  }
+  return "unknown status";
+}
+
+tre_status tss_window_reduce(const tre_grid* grid, const tre_requests* req, const tre_events* ev,
+                             tre_counts out, void* ws, size_t* ws_bytes, tre_diag* diag,
+                             tre_stream stream) {
+  if (!grid_ok(grid) || !ws_bytes || (!req) == (!ev)) return TRE_EINVAL;
+  if (req ? !req_ok(req) : !ev_ok(ev)) return TRE_EINVAL;
+  if (!counts_ok(&out)) return TRE_EINVAL;
+  if (ws && !diag) return TRE_EINVAL;
+  const int M = grid->n_models, K = grid->n_windows;
+  Arena a(ws);
+  ReduceWs w;
+  reduce_ws_layout(a, M, K, ev ? ev->n_req : 0, w);
+  bool query;
+  tre_status st = ws_check(a, ws, ws_bytes, query);
+  if (st != TRE_OK || query) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e;
+  {
+    Scope sc(kReduce, req ? 1 : 3, s);
+    e = req ? launch_reduce_requests(cols_of(req), M, grid->window_ms, K, out.P, out.D, w,
+                                     nullptr, nullptr, diag, s)
+            : launch_reduce_events(cols_of(ev), M, grid->window_ms, K, out.P, out.D, w, diag, s);
+  }
+  if (!e) {
+    Scope sc(kScan, 3, s);
+    e = launch_gauge_scan(M, K, w, out.A, out.W, s);
+  }
+  return cuda_status(e);
+}
+
+tre_status tss_score(const tre_grid* grid, const tre_counts* in, const tre_profile* prof,
+                     void* S_carry, uint8_t* init_carry, void* S_out, void* Z_out,
+                     uint8_t* cls_out, int32_t* recv_out, void* ws, size_t* ws_bytes,
+                     tre_diag* diag, tre_stream stream) {
+  if (!grid_ok(grid) || !ws_bytes || !counts_ok(in) || !prof_ok(prof, true)) return TRE_EINVAL;
+  if (!S_out || !Z_out || !cls_out || (!S_carry) != (!init_carry)) return TRE_EINVAL;
+  if (ws && !diag) return TRE_EINVAL;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (prof->dtype == TRE_F32)
+    return score_typed<float>(grid, in, prof, S_carry, init_carry, S_out, Z_out, cls_out,
+                              recv_out, ws, ws_bytes, diag, s);
+  return score_typed<double>(grid, in, prof, S_carry, init_carry, S_out, Z_out, cls_out, recv_out,
+                             ws, ws_bytes, diag, s);
+}
+
+tre_status tss_calibrate(const tre_grid* grid, const tre_requests* req, const tre_events* ev,
+                         const tre_counts* in, const tre_profile* prof, const int32_t* slo_ttft_ms,
+                         double ok_frac, double reliability, void* theta_out, void* ws,
+                         size_t* ws_bytes, tre_diag* diag, tre_stream stream) {
+  if (!grid_ok(grid) || !ws_bytes || (!req) == (!ev) || !counts_ok(in) || !prof_ok(prof, false))
+    return TRE_EINVAL;
+  if (req ? !req_ok(req) : !ev_ok(ev)) return TRE_EINVAL;
+  if (!slo_ttft_ms || !theta_out) return TRE_EINVAL;
+  if (ws && !diag) return TRE_EINVAL;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (prof->dtype == TRE_F32)
+    return calibrate_typed<float>(grid, req, ev, in, prof, slo_ttft_ms, ok_frac, reliability,
+                                  theta_out, ws, ws_bytes, diag, s);
+  return calibrate_typed<double>(grid, req, ev, in, prof, slo_ttft_ms, ok_frac, reliability,
+                                 theta_out, ws, ws_bytes, diag, s);
+}
+
+tre_status tre_select_moves(const tre_grid* grid, const void* Z, const uint8_t* cls,
+                            const tre_profile* prof, const tre_ctrl* ctrl, int32_t* r_inout,
+                            tre_move* moves, int64_t moves_cap, int64_t* n_moves_out, void* ws,
+                            size_t* ws_bytes, tre_diag* diag, tre_stream stream) {
+  if (!grid_ok(grid) || !ws_bytes || !Z || !cls || !prof || !ctrl || !r_inout || !n_moves_out)
+    return TRE_EINVAL;
+  if (prof->dtype != TRE_F32 && prof->dtype != TRE_F64) return TRE_EINVAL;
+  if (!prof->tau_crit || !prof->tau_surplus || !ctrl->r_min || !ctrl->footprint) return TRE_EINVAL;
+  if (ctrl->fast_ms < 1 || ctrl->slow_ms < 1 || ctrl->pacing_cap < 0 || ctrl->pacing_cap > 255)
+    return TRE_EINVAL;
+  if (moves_cap < 0 || (moves_cap > 0 && !moves)) return TRE_EINVAL;
+  if (ws && !diag) return TRE_EINVAL;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (prof->dtype == TRE_F32)
+    return select_typed<float>(grid, Z, cls, prof, ctrl, r_inout, moves, moves_cap, n_moves_out,
+                               ws, ws_bytes, diag, s);
+  return select_typed<double>(grid, Z, cls, prof, ctrl, r_inout, moves, moves_cap, n_moves_out,
+                              ws, ws_bytes, diag, s);
+}
+
+tre_status tre_sweep(const tre_sweep_spec* spec, const tre_sweep_out* out, void* ws,
+                     size_t* ws_bytes, tre_diag* diag, tre_stream stream) {
+  SweepPlan pl;
+  if (!ws_bytes || !sweep_plan(spec, pl) || !out) return TRE_EINVAL;
+  if (!out->theta || !out->n_moves || !out->r_final || out->moves_cap < 0 ||
+      (out->moves_cap > 0 && !out->moves))
+    return TRE_EINVAL;
+  if (ws && !diag) return TRE_EINVAL;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (spec->dtype == TRE_F32) return sweep_typed<float>(spec, pl, out, ws, ws_bytes, diag, s);
+  return sweep_typed<double>(spec, pl, out, ws, ws_bytes, diag, s);
+}
+
+}  // extern "C"

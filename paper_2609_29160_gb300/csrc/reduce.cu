@@ -1,0 +1,539 @@
+// Window reduction of request telemetry: the inputs of Eq. 1 (Sec. III-A)
+// collected as window deltas of prompt/decode token counters plus running and
+// waiting gauges (Sec. V-B).
+//
+// Request records are sorted by arrival in practice, so the records of one CTA
+// touch a short run of windows: the CTA accumulates into a shared-memory copy
+// of those rows and flushes them once; targets outside the staged rows (long
+// queue waits, unsorted input) go straight to global atomics. All arithmetic is
+// integer and all atomics are integer adds, so the result does not depend on
+// the order of the records.
+#include <algorithm>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace tre {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kStageBytes = 48 * 1024;
+constexpr int kSpill = 32;  // staged rows beyond the CTA's arrival range
+
+__device__ __forceinline__ int64_t win_clamp(int64_t t, int win, int K) {
+  if (t < 0) return 0;
+  const int64_t b = t / win;
+  return b > K ? K : b;
+}
+
+template <class V>
+__device__ __forceinline__ void stage_add(V* s, V* g, int64_t k, int64_t k_lo, int used, int M,
+                                          int m, V v) {
+  const int64_t rel = k - k_lo;
+  if (rel >= 0 && rel < used) atomicAdd(&s[rel * M + m], v);
+  else atomicAdd(&g[k * M + m], v);
+}
+
+// --------------------------------------------------------------------------
+// request records -> P, D, gauge diffs, optional packed SLO counts
+// --------------------------------------------------------------------------
+template <bool SLO>
+__global__ void __launch_bounds__(kThreads)
+k_reduce_requests(ReqCols r, int M, int win, int K, int64_t per_cta, int rows,
+                  int32_t* __restrict__ P, int32_t* __restrict__ D, int32_t* __restrict__ dA,
+                  int32_t* __restrict__ dW, unsigned long long* __restrict__ slo,
+                  const int32_t* __restrict__ slo_ms, tre_diag* diag) {
+  extern __shared__ unsigned long long smem[];
+  const int64_t i0 = (int64_t)blockIdx.x * per_cta;
+  const int64_t i1 = min(r.n, i0 + per_cta);
+  if (i0 >= i1) return;
+  const int64_t span = (int64_t)K * win;
+  const int64_t k_lo = win_clamp(r.t_arr[i0], win, K);
+  const int64_t k_hi = win_clamp(r.t_arr[i1 - 1], win, K);
+  const int64_t need = (k_hi >= k_lo ? k_hi - k_lo + 1 : 1) + kSpill;
+  const int used = (int)min64(rows, need);
+  const int cells = used * M;
+  unsigned long long* sS = smem;
+  int32_t* sP = reinterpret_cast<int32_t*>(smem + (SLO ? (size_t)rows * M : 0));
+  int32_t* sD = sP + (size_t)rows * M;
+  int32_t* sA = sD + (size_t)rows * M;
+  int32_t* sW = sA + (size_t)rows * M;
+  for (int c = threadIdx.x; c < cells; c += kThreads) {
+    sP[c] = 0; sD[c] = 0; sA[c] = 0; sW[c] = 0;
+    if (SLO) sS[c] = 0;
+  }
+  __syncthreads();
+
+  unsigned long long n_range = 0, n_model = 0, n_order = 0;
+  for (int64_t i = i0 + threadIdx.x; i < i1; i += kThreads) {
+    const int m = r.model[i];
+    const int64_t ta = r.t_arr[i], ts = r.t_start[i], tf = r.t_first[i], te = r.t_end[i];
+    const int32_t L_in = r.L_in[i], L = r.L_out[i];
+    if (m < 0 || m >= M) { ++n_model; continue; }
+    if (ta < 0 || ta >= span) { ++n_range; continue; }
+    if (!(ta <= ts && ts <= tf && tf <= te) || L_in < 0 || L < 1) { ++n_order; continue; }
+
+    if (tf < span) {
+      const int64_t kf = tf / win;
+      // prompt tokens, all at the first-token time
+      if (L_in) stage_add<int32_t>(sP, P, kf, k_lo, used, M, m, L_in);
+      // decode tokens: N(T) = tokens emitted before T; D[k] = N((k+1)w) - N(kw)
+      const int64_t ke_raw = te / win;
+      if (L == 1 || ke_raw == kf) {
+        stage_add<int32_t>(sD, D, kf, k_lo, used, M, m, L);
+      } else {
+        const unsigned long long dur = (unsigned long long)(te - tf);
+        const unsigned long long Lm1 = (unsigned long long)(L - 1);
+        const int64_t ke = min64(ke_raw, K - 1);
+        // N(T) = ceil((T - tf) * (L-1) / dur) for tf < T <= te, stepped by whole windows
+        unsigned long long q, rem, qs, rs;
+        divmod((unsigned long long)((kf + 1) * win - tf) * Lm1, (uint32_t)dur, q, rem);
+        divmod((unsigned long long)win * Lm1, (uint32_t)dur, qs, rs);
+        unsigned long long prevN = 0;
+        for (int64_t k = kf; k <= ke; ++k) {
+          unsigned long long N;
+          if ((k + 1) * win > te) {
+            N = (unsigned long long)L;
+          } else {
+            N = q + (rem != 0);
+            q += qs;
+            rem += rs;
+            if (rem >= dur) { rem -= dur; q += 1; }
+          }
+          const int32_t cnt = (int32_t)(N - prevN);
+          if (cnt) stage_add<int32_t>(sD, D, k, k_lo, used, M, m, cnt);
+          prevN = N;
+        }
+      }
+    }
+    // gauges: +1 where the state begins, -1 where it ends
+    const int64_t ba = win_clamp(ta, win, K), bs = win_clamp(ts, win, K), be = win_clamp(te, win, K);
+    if (ba != bs) {
+      stage_add<int32_t>(sW, dW, ba, k_lo, used, M, m, 1);
+      stage_add<int32_t>(sW, dW, bs, k_lo, used, M, m, -1);
+    }
+    if (bs != be) {
+      stage_add<int32_t>(sA, dA, bs, k_lo, used, M, m, 1);
+      stage_add<int32_t>(sA, dA, be, k_lo, used, M, m, -1);
+    }
+    if (SLO) {
+      const unsigned long long met = (tf - ta <= (int64_t)slo_ms[m]) ? 1ull : 0ull;
+      stage_add<unsigned long long>(sS, slo, ba, k_lo, used, M, m, 1ull + (met << 32));
+    }
+  }
+  __syncthreads();
+  for (int c = threadIdx.x; c < cells; c += kThreads) {
+    const int64_t k = k_lo + c / M;
+    const int m = c % M;
+    const size_t g = (size_t)k * M + m;
+    if (k < K) {
+      if (sP[c]) atomicAdd(&P[g], sP[c]);
+      if (sD[c]) atomicAdd(&D[g], sD[c]);
+      if (SLO && sS[c]) atomicAdd(&slo[g], sS[c]);
+    }
+    if (k <= K) {
+      if (sA[c]) atomicAdd(&dA[g], sA[c]);
+      if (sW[c]) atomicAdd(&dW[g], sW[c]);
+    }
+  }
+  warp_add_counter(&diag->dropped_range, n_range);
+  warp_add_counter(&diag->dropped_model, n_model);
+  warp_add_counter(&diag->dropped_order, n_order);
+}
+
+// SLO counts alone (for calibration from records whose counts exist already)
+__global__ void __launch_bounds__(kThreads)
+k_slo_requests(ReqCols r, int M, int win, int K, unsigned long long* __restrict__ slo,
+               const int32_t* __restrict__ slo_ms) {
+  const int64_t span = (int64_t)K * win;
+  for (int64_t i = (int64_t)blockIdx.x * kThreads + threadIdx.x; i < r.n;
+       i += (int64_t)gridDim.x * kThreads) {
+    const int m = r.model[i];
+    const int64_t ta = r.t_arr[i], ts = r.t_start[i], tf = r.t_first[i], te = r.t_end[i];
+    if (m < 0 || m >= M || ta < 0 || ta >= span) continue;
+    if (!(ta <= ts && ts <= tf && tf <= te) || r.L_in[i] < 0 || r.L_out[i] < 1) continue;
+    const unsigned long long met = (tf - ta <= (int64_t)slo_ms[m]) ? 1ull : 0ull;
+    atomicAdd(&slo[(size_t)(ta / win) * M + m], 1ull + (met << 32));
+  }
+}
+
+// --------------------------------------------------------------------------
+// token events -> P, D and per-request first/last tick
+// --------------------------------------------------------------------------
+
+// exact floor(t * 1000) of a float seconds value, as integer arithmetic on its
+// significand; returns false for NaN, infinities and negative values (a
+// negative zero is tick 0)
+__device__ __forceinline__ bool ms_tick(float t, int64_t span, int64_t& tick) {
+  const uint32_t b = __float_as_uint(t);
+  if ((b & 0x7fffffffu) == 0) { tick = 0; return span > 0; }
+  if (b >> 31) return false;
+  const uint32_t ex = (b >> 23) & 0xffu;
+  if (ex == 0xffu) return false;
+  const unsigned long long mant = ex ? ((b & 0x7fffffu) | 0x800000u) : (b & 0x7fffffu);
+  const int e = (ex ? (int)ex : 1) - 150;  // t = mant * 2^e
+  const unsigned long long prod = mant * 1000ull;
+  unsigned long long v;
+  if (e >= 0) {
+    if (e > 29) return false;                 // beyond any int32 millisecond
+    v = prod << e;
+  } else {
+    v = (-e >= 64) ? 0ull : (prod >> (-e));
+  }
+  if ((long long)v >= span) return false;
+  tick = (int64_t)v;
+  return true;
+}
+
+__global__ void __launch_bounds__(kThreads)
+k_reduce_events(EvCols e, int M, int win, int K, int64_t per_cta, int rows,
+                int32_t* __restrict__ P, int32_t* __restrict__ D, int32_t* __restrict__ first,
+                int32_t* __restrict__ last, tre_diag* diag) {
+  extern __shared__ unsigned long long smem[];
+  const int64_t i0 = (int64_t)blockIdx.x * per_cta;
+  const int64_t i1 = min(e.n, i0 + per_cta);
+  if (i0 >= i1) return;
+  const int64_t span = (int64_t)K * win;
+  int64_t t0, t1;
+  const int64_t k_lo = ms_tick(e.t_s[i0], span, t0) ? t0 / win : 0;
+  const int64_t k_hi = ms_tick(e.t_s[i1 - 1], span, t1) ? t1 / win : K;
+  const int64_t need = (k_hi >= k_lo ? k_hi - k_lo + 1 : 1) + kSpill;
+  const int used = (int)min64(rows, need);
+  const int cells = used * M;
+  int32_t* sP = reinterpret_cast<int32_t*>(smem);
+  int32_t* sD = sP + (size_t)rows * M;
+  for (int c = threadIdx.x; c < cells; c += kThreads) { sP[c] = 0; sD[c] = 0; }
+  __syncthreads();
+
+  const unsigned full = 0xffffffffu;
+  const int lane = threadIdx.x & 31;
+  unsigned long long n_range = 0, n_model = 0, n_order = 0;
+  for (int64_t base = i0; base < i1; base += kThreads) {
+    const int64_t i = base + threadIdx.x;
+    bool ok = false;
+    int64_t tick = 0;
+    int rq = 0;
+    if (i < i1) {
+      const int m = e.model[i];
+      rq = e.req[i];
+      const float ts = e.t_s[i];
+      const uint8_t ph = e.phase[i];
+      if (m < 0 || m >= M || rq < 0 || rq >= e.n_req || e.req_model[rq] != m) {
+        ++n_model;
+      } else if (!ms_tick(ts, span, tick)) {
+        ++n_range;
+      } else if (ph > 1) {
+        ++n_order;
+      } else {
+        ok = true;
+        const int64_t k = tick / win;
+        stage_add<int32_t>(ph == 0 ? sP : sD, ph == 0 ? P : D, k, k_lo, used, M, m, 1);
+      }
+    }
+    // first / last tick per request, one atomic per run of equal request ids
+    const unsigned active = __ballot_sync(full, ok);
+    if (ok) {
+      const unsigned grp = __match_any_sync(active, rq);
+      const int t32 = (int)tick;
+      const int mn = __reduce_min_sync(grp, t32);
+      const int mx = __reduce_max_sync(grp, t32);
+      if (lane == __ffs(grp) - 1) {
+        atomicMin(&first[rq], mn);
+        atomicMax(&last[rq], mx);
+      }
+    }
+  }
+  __syncthreads();
+  for (int c = threadIdx.x; c < cells; c += kThreads) {
+    const int64_t k = k_lo + c / M;
+    if (k >= K) continue;
+    const size_t g = (size_t)k * M + (c % M);
+    if (sP[c]) atomicAdd(&P[g], sP[c]);
+    if (sD[c]) atomicAdd(&D[g], sD[c]);
+  }
+  warp_add_counter(&diag->dropped_range, n_range);
+  warp_add_counter(&diag->dropped_model, n_model);
+  warp_add_counter(&diag->dropped_order, n_order);
+}
+
+__global__ void k_fill_first_last(int32_t* first, int32_t* last, int64_t n) {
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    first[i] = 0x7fffffff;
+    last[i] = -1;
+  }
+}
+
+// per request with at least one valid event: waiting on [t_arr, first),
+// running on [first, last)
+__global__ void __launch_bounds__(kThreads)
+k_event_gauges(EvCols e, int M, int win, int K, const int32_t* __restrict__ first,
+               const int32_t* __restrict__ last, int32_t* __restrict__ dA,
+               int32_t* __restrict__ dW, tre_diag* diag) {
+  unsigned long long n_order = 0;
+  for (int64_t r = (int64_t)blockIdx.x * kThreads + threadIdx.x; r < e.n_req;
+       r += (int64_t)gridDim.x * kThreads) {
+    const int64_t lt = last[r];
+    if (lt < 0) continue;
+    const int64_t ft = first[r];
+    const int m = e.req_model[r];
+    const int64_t ta = e.req_t_arr[r];
+    if (!(ta >= 0 && ta <= ft)) { ++n_order; continue; }
+    const int64_t ba = win_clamp(ta, win, K), bf = win_clamp(ft, win, K), bl = win_clamp(lt, win, K);
+    if (ba != bf) {
+      atomicAdd(&dW[ba * M + m], 1);
+      atomicAdd(&dW[bf * M + m], -1);
+    }
+    if (bf != bl) {
+      atomicAdd(&dA[bf * M + m], 1);
+      atomicAdd(&dA[bl * M + m], -1);
+    }
+  }
+  warp_add_counter(&diag->dropped_order, n_order);
+}
+
+__global__ void __launch_bounds__(kThreads)
+k_slo_events(EvCols e, int M, int win, int K, unsigned long long* __restrict__ slo,
+             const int32_t* __restrict__ slo_ms) {
+  const int64_t span = (int64_t)K * win;
+  for (int64_t r = (int64_t)blockIdx.x * kThreads + threadIdx.x; r < e.n_req;
+       r += (int64_t)gridDim.x * kThreads) {
+    const int m = e.req_model[r];
+    const int64_t ta = e.req_t_arr[r];
+    if (m < 0 || m >= M || ta < 0 || ta >= span) continue;
+    const unsigned long long met = (e.req_ttft[r] <= slo_ms[m]) ? 1ull : 0ull;
+    atomicAdd(&slo[(size_t)(ta / win) * M + m], 1ull + (met << 32));
+  }
+}
+
+// --------------------------------------------------------------------------
+// gauge scan: inclusive prefix over windows of the diff arrays, per model.
+// Segment = (chunk of rows, model); adjacent threads take adjacent models so
+// each row is read coalesced.
+// --------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads)
+k_scan_partials(int M, int K, int L, int n_chunks, const int32_t* __restrict__ dA,
+                const int32_t* __restrict__ dW, int32_t* __restrict__ pA,
+                int32_t* __restrict__ pW) {
+  const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+  if (t >= (int64_t)n_chunks * M) return;
+  const int m = (int)(t % M);
+  const int c = (int)(t / M);
+  const int64_t r0 = (int64_t)c * L, r1 = min64(r0 + L, K);
+  int32_t a = 0, w = 0;
+  for (int64_t k = r0; k < r1; ++k) {
+    a += dA[k * M + m];
+    w += dW[k * M + m];
+  }
+  pA[t] = a;
+  pW[t] = w;
+}
+
+// exclusive scan over chunks, one warp per model (n_chunks <= 1024)
+__global__ void k_scan_chunks(int M, int n_chunks, int32_t* __restrict__ pA,
+                              int32_t* __restrict__ pW) {
+  const int m = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
+  if (m >= M) return;
+  const int lane = threadIdx.x & 31;
+  const int per = (n_chunks + 31) / 32;
+  const int c0 = lane * per, c1 = min(n_chunks, c0 + per);
+  int32_t sa = 0, sw = 0;
+  for (int c = c0; c < c1; ++c) { sa += pA[(size_t)c * M + m]; sw += pW[(size_t)c * M + m]; }
+  int32_t ia = sa, iw = sw;
+  for (int o = 1; o < 32; o <<= 1) {
+    const int32_t xa = __shfl_up_sync(0xffffffffu, ia, o);
+    const int32_t xw = __shfl_up_sync(0xffffffffu, iw, o);
+    if (lane >= o) { ia += xa; iw += xw; }
+  }
+  int32_t ea = ia - sa, ew = iw - sw;
+  for (int c = c0; c < c1; ++c) {
+    const size_t x = (size_t)c * M + m;
+    const int32_t va = pA[x], vw = pW[x];
+    pA[x] = ea;
+    pW[x] = ew;
+    ea += va;
+    ew += vw;
+  }
+}
+
+__global__ void __launch_bounds__(kThreads)
+k_scan_apply(int M, int K, int L, int n_chunks, const int32_t* __restrict__ dA,
+             const int32_t* __restrict__ dW, const int32_t* __restrict__ pA,
+             const int32_t* __restrict__ pW, int32_t* __restrict__ A, int32_t* __restrict__ W) {
+  const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+  if (t >= (int64_t)n_chunks * M) return;
+  const int m = (int)(t % M);
+  const int c = (int)(t / M);
+  const int64_t r0 = (int64_t)c * L, r1 = min64(r0 + L, K);
+  int32_t a = pA[t], w = pW[t];
+  for (int64_t k = r0; k < r1; ++k) {
+    a += dA[k * M + m];
+    w += dW[k * M + m];
+    A[k * M + m] = a;
+    W[k * M + m] = w;
+  }
+}
+
+// exact coarsening: counts add over q base windows, gauges are read at the
+// last base window of each coarse window
+__global__ void __launch_bounds__(kThreads)
+k_aggregate(int M, int Kq, int q, const int32_t* __restrict__ P, const int32_t* __restrict__ D,
+            const int32_t* __restrict__ A, const int32_t* __restrict__ W,
+            const unsigned long long* __restrict__ slo, int32_t* __restrict__ Pq,
+            int32_t* __restrict__ Dq, int32_t* __restrict__ Aq, int32_t* __restrict__ Wq,
+            unsigned long long* __restrict__ sloq) {
+  const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+  if (t >= (int64_t)Kq * M) return;
+  const int m = (int)(t % M);
+  const int64_t k = t / M;
+  int32_t p = 0, d = 0;
+  unsigned long long s = 0;
+  for (int j = 0; j < q; ++j) {
+    const size_t x = (size_t)(k * q + j) * M + m;
+    p += P[x];
+    d += D[x];
+    if (slo) s += slo[x];
+  }
+  const size_t last = (size_t)(k * q + q - 1) * M + m;
+  Pq[t] = p;
+  Dq[t] = d;
+  Aq[t] = A[last];
+  Wq[t] = W[last];
+  if (sloq) sloq[t] = s;
+}
+
+int num_sms() {
+  static int n = 0;
+  if (!n) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 1;
+  }
+  return n;
+}
+
+int64_t per_cta_records(int64_t n, int lo, int hi) {
+  int64_t per = (n + (int64_t)num_sms() * 4 - 1) / ((int64_t)num_sms() * 4);
+  per = std::max<int64_t>(lo, std::min<int64_t>(hi, per));
+  return (per + kThreads - 1) / kThreads * kThreads;
+}
+
+unsigned grid_for(int64_t work, int per_thread = 1) {
+  const int64_t b = (work + (int64_t)kThreads * per_thread - 1) / ((int64_t)kThreads * per_thread);
+  return (unsigned)std::max<int64_t>(1, std::min<int64_t>(b, (int64_t)num_sms() * 16));
+}
+
+int scan_chunk_rows(int K) {
+  int L = (K + 1023) / 1024;
+  return L < 16 ? 16 : L;
+}
+
+}  // namespace
+
+void reduce_ws_layout(Arena& a, int M, int K, int64_t n_req, ReduceWs& w) {
+  const size_t cells = (size_t)(K + 1) * M;
+  w.dA = a.take<int32_t>(cells);
+  w.dW = a.take<int32_t>(cells);
+  w.first = n_req > 0 ? a.take<int32_t>((size_t)n_req) : nullptr;
+  w.last = n_req > 0 ? a.take<int32_t>((size_t)n_req) : nullptr;
+  const int L = scan_chunk_rows(K);
+  const int n_chunks = (K + L - 1) / L;
+  w.partA = a.take<int32_t>((size_t)std::max(n_chunks, 1) * M);
+  w.partW = a.take<int32_t>((size_t)std::max(n_chunks, 1) * M);
+}
+
+cudaError_t launch_reduce_requests(const ReqCols& r, int M, int win, int K, int32_t* P,
+                                   int32_t* D, ReduceWs& w, unsigned long long* slo,
+                                   const int32_t* slo_ms, tre_diag* diag, cudaStream_t s) {
+  const size_t cells = (size_t)K * M;
+  cudaError_t e;
+  if ((e = cudaMemsetAsync(P, 0, cells * sizeof(int32_t), s))) return e;
+  if ((e = cudaMemsetAsync(D, 0, cells * sizeof(int32_t), s))) return e;
+  if ((e = cudaMemsetAsync(w.dA, 0, (cells + M) * sizeof(int32_t), s))) return e;
+  if ((e = cudaMemsetAsync(w.dW, 0, (cells + M) * sizeof(int32_t), s))) return e;
+  if (slo && (e = cudaMemsetAsync(slo, 0, cells * sizeof(unsigned long long), s))) return e;
+  if (r.n == 0) return cudaSuccess;
+  const int cell_bytes = 16 + (slo ? 8 : 0);
+  const int rows = std::max(1, kStageBytes / (cell_bytes * M));
+  const int64_t per = per_cta_records(r.n, 1024, 8192);
+  const unsigned grid = (unsigned)((r.n + per - 1) / per);
+  const size_t smem = (size_t)rows * M * cell_bytes;
+  if (slo)
+    k_reduce_requests<true><<<grid, kThreads, smem, s>>>(r, M, win, K, per, rows, P, D, w.dA,
+                                                          w.dW, slo, slo_ms, diag);
+  else
+    k_reduce_requests<false><<<grid, kThreads, smem, s>>>(r, M, win, K, per, rows, P, D, w.dA,
+                                                           w.dW, nullptr, nullptr, diag);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_slo_requests(const ReqCols& r, int M, int win, int K,
+                                unsigned long long* slo, const int32_t* slo_ms, cudaStream_t s) {
+  cudaError_t e = cudaMemsetAsync(slo, 0, (size_t)K * M * sizeof(unsigned long long), s);
+  if (e || r.n == 0) return e;
+  k_slo_requests<<<grid_for(r.n, 4), kThreads, 0, s>>>(r, M, win, K, slo, slo_ms);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_reduce_events(const EvCols& ev, int M, int win, int K, int32_t* P, int32_t* D,
+                                 ReduceWs& w, tre_diag* diag, cudaStream_t s) {
+  const size_t cells = (size_t)K * M;
+  cudaError_t e;
+  if ((e = cudaMemsetAsync(P, 0, cells * sizeof(int32_t), s))) return e;
+  if ((e = cudaMemsetAsync(D, 0, cells * sizeof(int32_t), s))) return e;
+  if ((e = cudaMemsetAsync(w.dA, 0, (cells + M) * sizeof(int32_t), s))) return e;
+  if ((e = cudaMemsetAsync(w.dW, 0, (cells + M) * sizeof(int32_t), s))) return e;
+  if (ev.n_req > 0) {
+    k_fill_first_last<<<grid_for(ev.n_req, 4), kThreads, 0, s>>>(w.first, w.last, ev.n_req);
+    if ((e = cudaGetLastError())) return e;
+  }
+  if (ev.n > 0) {
+    const int rows = std::max(1, kStageBytes / (8 * M));
+    const int64_t per = per_cta_records(ev.n, 2048, 16384);
+    const unsigned grid = (unsigned)((ev.n + per - 1) / per);
+    k_reduce_events<<<grid, kThreads, (size_t)rows * M * 8, s>>>(ev, M, win, K, per, rows, P, D,
+                                                                 w.first, w.last, diag);
+    if ((e = cudaGetLastError())) return e;
+  }
+  if (ev.n_req > 0) {
+    k_event_gauges<<<grid_for(ev.n_req, 4), kThreads, 0, s>>>(ev, M, win, K, w.first, w.last,
+                                                               w.dA, w.dW, diag);
+    if ((e = cudaGetLastError())) return e;
+  }
+  return cudaSuccess;
+}
+
+cudaError_t launch_slo_events(const EvCols& ev, int M, int win, int K, unsigned long long* slo,
+                              const int32_t* slo_ms, cudaStream_t s) {
+  cudaError_t e = cudaMemsetAsync(slo, 0, (size_t)K * M * sizeof(unsigned long long), s);
+  if (e || ev.n_req == 0) return e;
+  k_slo_events<<<grid_for(ev.n_req, 4), kThreads, 0, s>>>(ev, M, win, K, slo, slo_ms);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gauge_scan(int M, int K, ReduceWs& w, int32_t* A, int32_t* W,
+                              cudaStream_t s) {
+  if (K == 0) return cudaSuccess;
+  const int L = scan_chunk_rows(K);
+  const int n_chunks = (K + L - 1) / L;
+  const int64_t segs = (int64_t)n_chunks * M;
+  const unsigned g = (unsigned)((segs + kThreads - 1) / kThreads);
+  k_scan_partials<<<g, kThreads, 0, s>>>(M, K, L, n_chunks, w.dA, w.dW, w.partA, w.partW);
+  k_scan_chunks<<<(M + 3) / 4, 128, 0, s>>>(M, n_chunks, w.partA, w.partW);
+  k_scan_apply<<<g, kThreads, 0, s>>>(M, K, L, n_chunks, w.dA, w.dW, w.partA, w.partW, A, W);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_aggregate(int M, int Kq, int q, const int32_t* P, const int32_t* D,
+                             const int32_t* A, const int32_t* W, const unsigned long long* slo,
+                             int32_t* Pq, int32_t* Dq, int32_t* Aq, int32_t* Wq,
+                             unsigned long long* sloq, cudaStream_t s) {
+  const int64_t n = (int64_t)Kq * M;
+  if (n == 0) return cudaSuccess;
+  k_aggregate<<<(unsigned)((n + kThreads - 1) / kThreads), kThreads, 0, s>>>(
+      M, Kq, q, P, D, A, W, slo, Pq, Dq, Aq, Wq, sloq);
+  return cudaGetLastError();
+}
+
+}  // namespace tre

@@ -1,0 +1,368 @@
+"""GPU parity: the CUDA library (called through the C ABI) against the CPU oracle
+on the same seeded inputs. Integers, decisions and -- because the library
+evaluates every floating-point step in the definition's order with one IEEE
+rounding each -- the floating-point outputs too are compared bit for bit."""
+import numpy as np
+import pytest
+
+import oracle
+import tracegen
+
+pytestmark = pytest.mark.gpu
+
+REQ_KEYS = ("model", "t_arr_ms", "t_start_ms", "t_first_ms", "t_end_ms", "L_in", "L_out")
+
+
+@pytest.fixture(scope="module")
+def tre():
+    import torch
+    import paper_2609_29160_gb300 as lib
+    lib.load()
+    torch.cuda.set_device(0)
+    return lib
+
+
+def _cuda(d):
+    import torch
+    return {k: torch.as_tensor(np.ascontiguousarray(v)).cuda() for k, v in d.items()}
+
+
+def _np(t):
+    return t.detach().cpu().numpy()
+
+
+def _adversarial(rng, n, M, win, K):
+    """Records on window boundaries, L_out = 1, zero-length spans, requests past
+    the end, bad model ids, order violations, shuffled order."""
+    span = K * win
+    t_arr = rng.integers(-win, span + 2 * win, n)
+    t_arr = np.where(rng.random(n) < 0.2, (t_arr // win) * win, t_arr)
+    wait = rng.integers(0, 8 * win, n) * (rng.random(n) < 0.6)
+    pre = rng.integers(0, 3 * win, n) * (rng.random(n) < 0.8)
+    dec = rng.integers(0, 12 * win, n) * (rng.random(n) < 0.9)
+    L_out = np.where(rng.random(n) < 0.15, 1, rng.integers(1, 600, n))
+    t_start = t_arr + wait
+    t_first = t_start + pre
+    t_end = np.where(L_out == 1, t_first, t_first + dec)
+    t_end = np.where(rng.random(n) < 0.05, (t_end // win) * win, t_end)
+    model = rng.integers(0, M, n)
+    model = np.where(rng.random(n) < 0.03, rng.choice([-1, M, M + 5], n), model)
+    bad = rng.random(n) < 0.03
+    t_start = np.where(bad, t_arr - 1, t_start)
+    L_in = np.where(rng.random(n) < 0.01, -3, rng.integers(0, 4000, n))
+    L_out = np.where(rng.random(n) < 0.01, 0, L_out)
+    return {"model": model.astype(np.int32), "t_arr_ms": t_arr.astype(np.int32),
+            "t_start_ms": t_start.astype(np.int32), "t_first_ms": t_first.astype(np.int32),
+            "t_end_ms": t_end.astype(np.int32), "L_in": L_in.astype(np.int32),
+            "L_out": L_out.astype(np.int32)}
+
+
+def _check_reduce(tre, req, M, win, K):
+    P, D, A, W, drops = oracle.reduce_requests(req, M, win, K)
+    diag = tre.new_diag()
+    c = tre.tss_window_reduce(M, win, K, requests=_cuda(req), diag=diag)
+    for k, ref in zip("PDAW", (P, D, A, W)):
+        np.testing.assert_array_equal(_np(c[k]), ref, err_msg=k)
+    d = tre.read_diag(diag)
+    assert [d["dropped_range"], d["dropped_model"], d["dropped_order"]] == drops.tolist()
+    return c
+
+
+@pytest.mark.parametrize("name,scale", [("tiny", 1.0), ("mid", 0.05), ("hetero", 0.01)])
+def test_reduce_requests_generated(tre, name, scale):
+    w = tracegen.workload(name, scale=scale)
+    _check_reduce(tre, w["requests"], w["M"], w["window_ms"], w["K"])
+
+
+@pytest.mark.parametrize("seed,M,win,K", [(1, 3, 1000, 50), (2, 8, 100, 700), (3, 17, 7, 333),
+                                          (4, 64, 250, 40), (5, 1, 1, 5000)])
+def test_reduce_requests_adversarial(tre, seed, M, win, K):
+    rng = np.random.default_rng(seed)
+    req = _adversarial(rng, 20000, M, win, K)
+    _check_reduce(tre, req, M, win, K)
+    # the same records shuffled give the same result
+    perm = rng.permutation(len(req["model"]))
+    _check_reduce(tre, {k: v[perm] for k, v in req.items()}, M, win, K)
+
+
+def test_reduce_empty_and_zero_windows(tre):
+    req = {k: np.zeros(0, np.int32) for k in REQ_KEYS}
+    _check_reduce(tre, req, 4, 1000, 10)
+
+
+def _events_case(seed, scale=0.002):
+    w = tracegen.workload("stream", scale=scale, seed=seed)
+    return w
+
+
+def test_reduce_events(tre):
+    w = _events_case(4)
+    ev, M, win, K = w["events"], w["M"], w["window_ms"], w["K"]
+    P, D, A, W, drops = oracle.reduce_events(ev, M, win, K)
+    diag = tre.new_diag()
+    c = tre.tss_window_reduce(M, win, K, events=_cuda(ev), diag=diag)
+    for k, ref in zip("PDAW", (P, D, A, W)):
+        np.testing.assert_array_equal(_np(c[k]), ref, err_msg=k)
+    d = tre.read_diag(diag)
+    assert [d["dropped_range"], d["dropped_model"], d["dropped_order"]] == drops.tolist()
+
+
+def test_reduce_events_shuffled_and_corrupt(tre):
+    w = _events_case(5)
+    ev = {k: v.copy() for k, v in w["events"].items()}
+    M, win, K = w["M"], w["window_ms"], w["K"]
+    rng = np.random.default_rng(0)
+    n = len(ev["model"])
+    idx = rng.choice(n, n // 50, replace=False)
+    ev["t_s"][idx[: len(idx) // 4]] = np.float32(-1.0)
+    ev["t_s"][idx[len(idx) // 4: len(idx) // 2]] = np.float32(np.nan)
+    ev["phase"][idx[len(idx) // 2: 3 * len(idx) // 4]] = 7
+    ev["model"][idx[3 * len(idx) // 4:]] = (ev["model"][idx[3 * len(idx) // 4:]] + 1) % M
+    ev["t_s"][idx[:5]] = np.float32(-0.0)
+    ev["req_t_arr_ms"][rng.choice(len(ev["req_model"]), 20)] = 10 ** 9
+    perm = rng.permutation(n)
+    ev = {k: (v[perm] if len(v) == n else v) for k, v in ev.items()}
+    P, D, A, W, drops = oracle.reduce_events(ev, M, win, K)
+    diag = tre.new_diag()
+    c = tre.tss_window_reduce(M, win, K, events=_cuda(ev), diag=diag)
+    for k, ref in zip("PDAW", (P, D, A, W)):
+        np.testing.assert_array_equal(_np(c[k]), ref, err_msg=k)
+    d = tre.read_diag(diag)
+    assert [d["dropped_range"], d["dropped_model"], d["dropped_order"]] == drops.tolist()
+
+
+def _score_inputs(rng, K, M, idle_frac=0.2):
+    cnt = {}
+    for k, hi in (("P", 5000), ("D", 800), ("A", 30), ("W", 60)):
+        cnt[k] = rng.integers(0, hi, (K, M)).astype(np.int32)
+    idle = rng.random((K, M)) < idle_frac
+    runs = rng.random(K) < 0.01               # long all-idle stretches
+    idle |= np.repeat(runs, M).reshape(K, M)
+    idle[: K // 20, M // 2:] = True           # some models start late
+    for k in cnt:
+        cnt[k][idle] = 0
+    return cnt
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f64"])
+@pytest.mark.parametrize("K,M,win,alpha", [(600, 3, 1000, 0.2), (36000, 8, 100, 0.02),
+                                           (43200, 16, 500, 0.1), (5000, 64, 100, 0.02),
+                                           (3000, 5, 2000, 0.4), (257, 2, 100, 1.0)])
+def test_score_bit_exact(tre, dtype, K, M, win, alpha):
+    rng = np.random.default_rng(K + M)
+    cnt = _score_inputs(rng, K, M)
+    npdt = np.float32 if dtype == "f32" else np.float64
+    prof = {"w_p": rng.uniform(0.1, 0.3, M), "w_q": rng.uniform(1.0, 3.0, M),
+            "alpha": np.full(M, alpha), "theta": rng.uniform(5, 50, M),
+            "tau_crit": np.full(M, 0.8), "tau_surplus": np.full(M, 1.2)}
+    S, Z, cls, recv = oracle.score(cnt["P"], cnt["D"], cnt["A"], cnt["W"], prof, win, npdt)
+    diag = tre.new_diag()
+    out = tre.tss_score(_cuda(cnt), prof, win, dtype=dtype, diag=diag)
+    np.testing.assert_array_equal(_np(out["S"]), S)
+    np.testing.assert_array_equal(_np(out["Z"]), Z)
+    np.testing.assert_array_equal(_np(out["cls"]), cls)
+    np.testing.assert_array_equal(_np(out["recv"]), recv)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f64"])
+def test_score_carry_across_calls(tre, dtype):
+    import torch
+    rng = np.random.default_rng(9)
+    K, M, win = 20000, 6, 100
+    cnt = _score_inputs(rng, K, M)
+    npdt = np.float32 if dtype == "f32" else np.float64
+    prof = {"w_p": 0.2, "w_q": 2.0, "alpha": 0.05, "theta": 10.0, "tau_crit": 0.8,
+            "tau_surplus": 1.2}
+    S, Z, cls, _ = oracle.score(cnt["P"], cnt["D"], cnt["A"], cnt["W"], prof, win, npdt)
+    tdt = torch.float32 if dtype == "f32" else torch.float64
+    carry = {"S": torch.zeros(M, dtype=tdt, device="cuda"),
+             "init": torch.zeros(M, dtype=torch.uint8, device="cuda")}
+    parts = []
+    for a, b in ((0, 7777), (7777, 7778), (7778, K)):
+        sub = _cuda({k: v[a:b] for k, v in cnt.items()})
+        parts.append(tre.tss_score(sub, prof, win, dtype=dtype, carry=carry))
+    np.testing.assert_array_equal(np.concatenate([_np(p["S"]) for p in parts]), S)
+    np.testing.assert_array_equal(np.concatenate([_np(p["cls"]) for p in parts]), cls)
+
+
+def test_score_is_deterministic(tre):
+    rng = np.random.default_rng(5)
+    cnt = _cuda(_score_inputs(rng, 50000, 8))
+    prof = {"w_p": 0.2, "w_q": 2.0, "alpha": 0.02, "theta": 10.0, "tau_crit": 0.8,
+            "tau_surplus": 1.2}
+    a = tre.tss_score(cnt, prof, 100)
+    b = tre.tss_score(cnt, prof, 100)
+    for k in ("S", "Z", "cls", "recv"):
+        assert (a[k] == b[k]).all()
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f64"])
+@pytest.mark.parametrize("name,scale", [("tiny", 1.0), ("mid", 0.05), ("hetero", 0.005)])
+def test_pipeline_requests(tre, dtype, name, scale):
+    w = tracegen.workload(name, scale=scale)
+    M, win, K = w["M"], w["window_ms"], w["K"]
+    npdt = np.float32 if dtype == "f32" else np.float64
+    prof = tracegen.default_profile(M, win)
+    o = oracle.pipeline_requests(w["requests"], M, win, K, prof, w["slo_ttft_ms"], npdt)
+    req = _cuda(w["requests"])
+    c = tre.tss_window_reduce(M, win, K, requests=req)
+    diag = tre.new_diag()
+    theta = tre.tss_calibrate(c, prof, win, w["slo_ttft_ms"], requests=req, dtype=dtype,
+                              diag=diag)
+    np.testing.assert_array_equal(_np(theta), o["theta"])
+    assert tre.read_diag(diag)["degenerate_calib"] == o["degenerate"]
+    sc = tre.tss_score(c, dict(prof, theta=theta), win, dtype=dtype)
+    for k in ("S", "Z", "cls", "recv"):
+        np.testing.assert_array_equal(_np(sc[k]), o[k], err_msg=k)
+    for cap in (1, 3):
+        for tc in (0.6, 0.9):
+            p2 = dict(prof, theta=theta, tau_crit=np.full(M, tc))
+            mv, rf, n, _ = tre.tre_select_moves(sc["Z"], sc["cls"], p2, win, w["budget"],
+                                                w["r0"], w["r_min"], w["footprint"],
+                                                pacing_cap=cap)
+            om, orf, _ = oracle.select_moves(o["Z"], o["cls"], tc, 1.2, win, w["budget"],
+                                             w["r0"], w["r_min"], w["footprint"], pacing_cap=cap)
+            assert n == len(om)
+            np.testing.assert_array_equal(_np(rf), orf)
+            got = np.stack([mv[f].astype(np.int32) for f in ("window", "recv", "donor", "kind",
+                                                               "seq")], 1) if n else np.zeros((0, 5))
+            ref = np.stack([om[f] for f in ("window", "recv", "donor", "kind", "seq")], 1) \
+                if n else np.zeros((0, 5))
+            np.testing.assert_array_equal(got, ref)
+
+
+def test_calibrate_events(tre):
+    w = _events_case(6)
+    ev, M, win, K = w["events"], w["M"], w["window_ms"], w["K"]
+    prof = tracegen.default_profile(M, win)
+    P, D, A, W, _ = oracle.reduce_events(ev, M, win, K)
+    n_arr, n_met = oracle.slo_counts_events(ev, M, win, K, w["slo_ttft_ms"])
+    S, _, cls, _ = oracle.score(P, D, A, W, prof, win, np.float32)
+    theta, deg = oracle.calibrate(S, cls, n_arr, n_met)
+    evc = _cuda(ev)
+    c = tre.tss_window_reduce(M, win, K, events=evc)
+    diag = tre.new_diag()
+    th = tre.tss_calibrate(c, prof, win, w["slo_ttft_ms"], events=evc, dtype="f32", diag=diag)
+    np.testing.assert_array_equal(_np(th), theta)
+    assert tre.read_diag(diag)["degenerate_calib"] == deg
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f64"])
+def test_calibrate_adversarial_ties(tre, dtype):
+    """Few distinct S levels (many exact ties), idle and zero-S windows, rho 1."""
+    import torch
+    rng = np.random.default_rng(3)
+    K, M, win = 3000, 5, 1000
+    cnt = _score_inputs(rng, K, M, idle_frac=0.3)
+    cnt["P"] = (cnt["P"] // 1000 * 1000).astype(np.int32)
+    cnt["D"] = (cnt["D"] // 200 * 200).astype(np.int32)
+    cnt["A"] = np.where(cnt["A"] > 0, 4, 0).astype(np.int32)
+    cnt["W"] = np.zeros_like(cnt["W"])
+    prof = {"w_p": 0.25, "w_q": 2.0, "alpha": 1.0, "theta": 1.0, "tau_crit": 0.8,
+            "tau_surplus": 1.2}
+    npdt = np.float32 if dtype == "f32" else np.float64
+    S, _, cls, _ = oracle.score(cnt["P"], cnt["D"], cnt["A"], cnt["W"], prof, win, npdt)
+    # arrivals: one request per window at a random ms; met with probability rising in S
+    req = {k: [] for k in REQ_KEYS}
+    for k in range(K):
+        for m in range(M):
+            if rng.random() < 0.7:
+                ta = k * win + int(rng.integers(0, win))
+                ok = rng.random() < min(1.0, 0.3 + S[k, m] / (S.max() + 1e-9))
+                tf = ta + (100 if ok else 5000)
+                for key, v in zip(REQ_KEYS, (m, ta, ta, tf, tf, 1, 1)):
+                    req[key].append(v)
+    req = {k: np.array(v, np.int32) for k, v in req.items()}
+    slo = np.full(M, 1000, np.int32)
+    n_arr, n_met = oracle.slo_counts_requests(req, M, win, K, slo)
+    for rho in (0.5, 0.95, 1.0):
+        theta, deg = oracle.calibrate(S, cls, n_arr, n_met, 0.95, rho)
+        diag = tre.new_diag()
+        th = tre.tss_calibrate(_cuda(cnt), prof, win, slo, requests=_cuda(req), dtype=dtype,
+                               ok_frac=0.95, reliability=rho, diag=diag)
+        np.testing.assert_array_equal(_np(th), theta)
+        assert tre.read_diag(diag)["degenerate_calib"] == deg
+
+
+def test_select_heterogeneous_footprints_and_overflow(tre):
+    import torch
+    rng = np.random.default_rng(12)
+    K, M, win = 3000, 6, 1000
+    Z = rng.choice(np.array([0.3, 0.6, 0.85, 0.95, 1.0, 1.1, 1.3, 2.0]), (K, M)).astype(np.float32)
+    cls = np.where(rng.random((K, M)) < 0.1, oracle.IDLE, oracle.NOM).astype(np.uint8)
+    g = np.array([1, 2, 3, 1, 2, 1], np.int32)
+    r0 = np.array([3, 2, 2, 4, 1, 3], np.int32)
+    budget = int((g * r0).sum()) + 2
+    r_min = np.array([1, 1, 0, 2, 0, 1], np.int32)
+    prof = {"w_p": 0.2, "w_q": 2.0, "alpha": 0.2, "theta": 1.0, "tau_crit": 0.8,
+            "tau_surplus": 1.2}
+    om, orf, _ = oracle.select_moves(Z, cls, 0.8, 1.2, win, budget, r0, r_min, g, 5000, 10000, 3)
+    Zc, Cc = torch.as_tensor(Z).cuda(), torch.as_tensor(cls).cuda()
+    mv, rf, n, diag = tre.tre_select_moves(Zc, Cc, prof, win, budget, r0, r_min, g, pacing_cap=3,
+                                           moves_cap=len(om) + 5)
+    assert n == len(om)
+    np.testing.assert_array_equal(_np(rf), orf)
+    for a, b in zip(mv, om):
+        assert (int(a["window"]), int(a["recv"]), int(a["donor"]), int(a["kind"]),
+                int(a["seq"])) == tuple(int(x) for x in b)
+    assert tre.read_diag(diag)["err"] == 0
+    # overflow: only the first `cap` moves are written, the count is the full one
+    mv, rf, n, diag = tre.tre_select_moves(Zc, Cc, prof, win, budget, r0, r_min, g, pacing_cap=3,
+                                           moves_cap=7)
+    assert n == len(om) and len(mv) == 7
+    assert tre.read_diag(diag)["err"] == 4
+    np.testing.assert_array_equal(_np(rf), orf)
+
+
+def _sweep_case(scale, n_traces, duration_s):
+    sw = tracegen.sweep_workload(scale=scale, n_traces=n_traces, duration_s=duration_s)
+    alpha = [min(1.0, w / 5000.0) for w in sw["window_ms"]]
+    return sw, alpha
+
+
+def _run_sweep_both(tre, sw, alpha, moves_cap, dtype="f32"):
+    M = sw["M"]
+    npdt = np.float32 if dtype == "f32" else np.float64
+    ref = oracle.sweep(sw["traces"], M, sw["duration_ms"], sw["window_ms"], sw["tau_crit"],
+                       sw["pacing_cap"], sw["w_p"], sw["w_q"], sw["tau_surplus"], alpha,
+                       sw["slo_ttft_ms"], sw["budget"], sw["r0"], sw["r_min"], sw["footprint"],
+                       dtype=npdt)
+    out = tre.tre_sweep([_cuda(t) for t in sw["traces"]], M, sw["duration_ms"], sw["window_ms"],
+                        alpha, sw["tau_crit"], sw["pacing_cap"], sw["w_p"], sw["w_q"],
+                        sw["tau_surplus"], sw["slo_ttft_ms"], sw["budget"], sw["r0"],
+                        sw["r_min"], sw["footprint"], dtype=dtype, moves_cap=moves_cap,
+                        want_counts=True, want_S=True)
+    return ref, out
+
+
+def _compare_sweep(tre, sw, ref, out, moves_cap):
+    M = sw["M"]
+    off = 0
+    theta = _np(out["theta"])
+    for si, s in enumerate(ref["series"]):
+        n = s["K"] * M
+        for k in ("P", "D", "A", "W", "S", "Z"):
+            np.testing.assert_array_equal(_np(out[k][off: off + n]).reshape(s["K"], M), s[k],
+                                          err_msg=f"series {si} {k}")
+        np.testing.assert_array_equal(theta[si], s["theta"], err_msg=f"theta {si}")
+        off += n
+    n_inst = len(ref["instances"])
+    moves = tre.sweep_moves(out, n_inst, moves_cap)
+    rf = _np(out["r_final"])
+    for i, inst in enumerate(ref["instances"]):
+        np.testing.assert_array_equal(rf[i], inst["r_final"], err_msg=f"instance {i}")
+        got = moves[i]
+        om = inst["moves"]
+        assert int(_np(out["n_moves"])[i]) == len(om), f"instance {i}"
+        assert len(got) == min(len(om), moves_cap)
+        for a, b in zip(got, om):
+            assert (int(a["window"]), int(a["recv"]), int(a["donor"]), int(a["kind"]),
+                    int(a["seq"])) == tuple(int(x) for x in b), f"instance {i}"
+
+
+def test_sweep_small(tre):
+    sw, alpha = _sweep_case(0.02, 2, 600.0)
+    sw["tau_crit"] = sw["tau_crit"][::3]
+    sw["pacing_cap"] = sw["pacing_cap"][::3]
+    ref, out = _run_sweep_both(tre, sw, alpha, moves_cap=512)
+    _compare_sweep(tre, sw, ref, out, 512)

@@ -1,0 +1,111 @@
+"""The C-ABI library builds for sm_103a, loads, and exports every entry point
+that include/tre.h declares; host-side argument checks answer without a GPU
+(no compute call is made here)."""
+import ctypes as C
+import os
+import re
+
+import pytest
+
+import paper_2609_29160_gb300 as tre
+from tests.conftest import ROOT
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "tre.h")).read()
+    return sorted(set(re.findall(r"^(?:tre_status|const char\*)\s+(\w+)\s*\(", src, re.M)))
+
+
+def test_header_declares_the_five_entry_points():
+    names = _declared()
+    for n in ("tss_window_reduce", "tss_score", "tss_calibrate", "tre_select_moves", "tre_sweep",
+              "tre_status_str"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol():
+    lib = tre.load()
+    for name in _declared():
+        assert hasattr(lib, name), name
+
+
+def test_struct_layouts_match_header_sizes():
+    # sizes fixed by the header's field lists on LP64
+    assert C.sizeof(tre.Grid) == 12
+    assert C.sizeof(tre.Requests) == 8 + 7 * 8
+    assert C.sizeof(tre.Diag) == 5 * 8 + 8
+    assert tre.MOVE_DTYPE.itemsize == 12
+
+
+def test_status_strings():
+    lib = tre.load()
+    assert lib.tre_status_str(0) == b"ok"
+    assert lib.tre_status_str(4) == b"move list overflow"
+
+
+def test_argument_errors_are_reported_on_the_host():
+    lib = tre.load()
+    g = tre.Grid(0, 1000, 10)           # no models
+    n = C.c_size_t(0)
+    rq = tre.Requests(0)
+    cs = tre.Counts(1, 1, 1, 1)
+    assert lib.tss_window_reduce(C.byref(g), C.byref(rq), None, cs, None, C.byref(n), None,
+                                 None) == 1
+    g = tre.Grid(3, 1000, 10)
+    # both and neither telemetry descriptor
+    ev = tre.Events(0)
+    assert lib.tss_window_reduce(C.byref(g), C.byref(rq), C.byref(ev), cs, None, C.byref(n),
+                                 None, None) == 1
+    assert lib.tss_window_reduce(C.byref(g), None, None, cs, None, C.byref(n), None, None) == 1
+    # a workspace query needs no device
+    assert lib.tss_window_reduce(C.byref(g), C.byref(rq), None, cs, None, C.byref(n), None,
+                                 None) == 0
+    assert n.value > 0
+    # records present but a column missing
+    rq2 = tre.Requests(5, 1, 1, 1, 1, 1, 1, None)
+    assert lib.tss_window_reduce(C.byref(g), C.byref(rq2), None, cs, None, C.byref(n), None,
+                                 None) == 1
+    # window grid beyond int32 milliseconds
+    big = tre.Grid(3, 1_000_000, 10_000)
+    assert lib.tss_window_reduce(C.byref(big), C.byref(rq), None, cs, None, C.byref(n), None,
+                                 None) == 1
+
+
+def test_workspace_too_small_is_enomem():
+    lib = tre.load()
+    g = tre.Grid(4, 100, 1000)
+    cs = tre.Counts(1, 1, 1, 1)
+    prof = tre.Profile(0, 8, 8, 8, 8, 8, 8)
+    n = C.c_size_t(0)
+    assert lib.tss_score(C.byref(g), C.byref(cs), C.byref(prof), None, None, 8, 8, 8, None, None,
+                         C.byref(n), None, None) == 0
+    need = n.value
+    small = C.c_size_t(need - 1)
+    assert lib.tss_score(C.byref(g), C.byref(cs), C.byref(prof), None, None, 8, 8, 8, None,
+                         C.c_void_p(4096), C.byref(small), C.c_void_p(8), None) == 2
+
+
+def test_select_and_sweep_argument_checks():
+    lib = tre.load()
+    g = tre.Grid(3, 1000, 100)
+    prof = tre.Profile(0, 8, 8, 8, 8, 8, 8)
+    n = C.c_size_t(0)
+    bad = tre.Ctrl(8, 8, 8, 5000, 10000, 300)     # pacing cap beyond one byte of seq
+    assert lib.tre_select_moves(C.byref(g), 8, 8, C.byref(prof), C.byref(bad), 8, 8, 10, 8, None,
+                                C.byref(n), None, None) == 1
+    ok = tre.Ctrl(8, 8, 8, 5000, 10000, 1)
+    assert lib.tre_select_moves(C.byref(g), 8, 8, C.byref(prof), C.byref(ok), 8, 8, 10, 8, None,
+                                C.byref(n), None, None) == 0
+    # sweep window lengths that do not nest
+    tr = (tre.Requests * 1)(tre.Requests(0))
+    wins = (C.c_int32 * 2)(300, 500)
+    al = (C.c_double * 2)(0.1, 0.1)
+    tau = (C.c_double * 1)(0.8)
+    cap = (C.c_int32 * 1)(1)
+    spec = tre.SweepSpec(3, 3000, 1, tr, 2, wins, al, 1, tau, 1, cap, 0, 8, 8, 8, 8, 0.95, 0.95,
+                         tre.Ctrl(8, 8, 8, 5000, 10000, 0), 8)
+    so = tre.SweepOut(None, None, None, None, None, None, None, 8, 8, 4, 8, 8)
+    assert lib.tre_sweep(C.byref(spec), C.byref(so), None, C.byref(n), None, None) == 1
+    wins2 = (C.c_int32 * 2)(500, 1000)
+    spec.window_ms = wins2
+    assert lib.tre_sweep(C.byref(spec), C.byref(so), None, C.byref(n), None, None) == 0
