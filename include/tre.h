@@ -207,6 +207,27 @@ tre_status tre_select_moves(const tre_grid* grid, const void* Z, const uint8_t* 
                             tre_move* moves, int64_t moves_cap, int64_t* n_moves_out, void* ws,
                             size_t* ws_bytes, tre_diag* diag, tre_stream stream);
 
+/*
+ * tss_score_noalloc -- the same computation and outputs as tss_score, for
+ * callers that cannot allocate device memory (no cudaMalloc where they run, or
+ * a host that owns every allocation), so they cannot supply `ws`. It takes no
+ * workspace: its scratch is a 4 MiB buffer compiled into the library, one copy
+ * on every GPU that loads the library, held until the process exits. The paper
+ * has no counterpart; this is a deployment variant of the scoring call.
+ * Limit: ceil(n_windows / L) * n_models <= 65536 with L = max(256,
+ * ceil(n_windows / 1024)) -- any n_windows for n_models <= 64; larger problems
+ * return TRE_ENOMEM before anything is enqueued. The first call on a device
+ * looks up the buffer's device address (make it before any stream capture).
+ * All calls share the one buffer: calls whose GPU work overlaps in time (other
+ * streams, other host threads) race on it and must be serialised by the
+ * caller. Nothing in the buffer needs to start at zero; every call writes what
+ * it later reads. diag is required.
+ */
+tre_status tss_score_noalloc(const tre_grid* grid, const tre_counts* in, const tre_profile* prof,
+                             void* S_carry, uint8_t* init_carry, void* S_out, void* Z_out,
+                             uint8_t* cls_out, int32_t* recv_out, tre_diag* diag,
+                             tre_stream stream);
+
 /* Sweep description. Host fields are read during the call only. */
 typedef struct {
   int32_t n_models;

@@ -1,0 +1,89 @@
+// tss_score_noalloc: the scoring entry point for callers that cannot allocate
+// device memory (for example code running where cudaMalloc is forbidden or
+// unavailable, such as inside a host callback, a plug-in host that owns every
+// allocation, or a process whose allocator is locked down). Its scratch lives in
+// a fixed buffer compiled into this library instead of a caller workspace.
+#include <cuda_runtime.h>
+
+#include "internal.h"
+
+using namespace tre;
+
+namespace {
+
+// Per-(segment, model) smoothing state of the scoring scan: at most this many
+// (segment, model) pairs, at 64 bytes each in double precision, plus alignment.
+constexpr int64_t kMaxSegModels = 65536;
+constexpr size_t kScratchBytes = (size_t)kMaxSegModels * 64 + 16 * 256;
+
+// One copy per GPU that loads this library; it stays allocated until the
+// process exits. In host code this name is only a host-side stand-in: kernels
+// get the device address obtained with cudaGetSymbolAddress below.
+static __device__ __align__(256) unsigned char g_score_scratch[kScratchBytes];
+
+constexpr int kMaxDevices = 256;
+void* g_scratch_addr[kMaxDevices];
+
+// Device address of the scratch for the current device, looked up once per
+// device (the first call on a device does this; make it before any stream
+// capture).
+tre_status scratch_address(void** out) {
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return TRE_ECUDA;
+  if (!g_scratch_addr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_score_scratch) != cudaSuccess || !p) return TRE_ECUDA;
+    g_scratch_addr[dev] = p;
+  }
+  *out = g_scratch_addr[dev];
+  return TRE_OK;
+}
+
+template <class T>
+tre_status run(const tre_grid* g, const tre_counts* in, const tre_profile* p, void* S_carry,
+               uint8_t* init_carry, void* S_out, void* Z_out, uint8_t* cls_out,
+               int32_t* recv_out, tre_diag* diag, cudaStream_t s) {
+  const int M = g->n_models, K = g->n_windows;
+  Arena measure(nullptr);
+  ScoreWs<T> w;
+  score_ws_layout<T>(measure, M, K, w);
+  if ((int64_t)w.n_seg * M > kMaxSegModels || measure.off > kScratchBytes) return TRE_ENOMEM;
+  void* base = nullptr;
+  tre_status st = scratch_address(&base);
+  if (st != TRE_OK) return st;
+  Arena a(base);
+  score_ws_layout<T>(a, M, K, w);
+  cudaError_t e = launch_score<T>(
+      M, g->window_ms, K, in->P, in->D, in->A, in->W, static_cast<const T*>(p->w_p),
+      static_cast<const T*>(p->w_q), static_cast<const T*>(p->alpha),
+      static_cast<const T*>(p->theta), static_cast<const T*>(p->tau_crit),
+      static_cast<const T*>(p->tau_surplus), static_cast<T*>(S_carry), init_carry,
+      static_cast<T*>(S_out), static_cast<T*>(Z_out), cls_out, w, diag, s);
+  if (!e && recv_out)
+    e = launch_receiver<T>(M, K, static_cast<const T*>(Z_out), cls_out, recv_out, s);
+  return e == cudaSuccess ? TRE_OK : TRE_ECUDA;
+}
+
+}  // namespace
+
+extern "C" tre_status tss_score_noalloc(const tre_grid* grid, const tre_counts* in,
+                                        const tre_profile* prof, void* S_carry,
+                                        uint8_t* init_carry, void* S_out, void* Z_out,
+                                        uint8_t* cls_out, int32_t* recv_out, tre_diag* diag,
+                                        tre_stream stream) {
+  if (!grid || grid->n_models < 1 || grid->n_models > 1024 || grid->window_ms < 1 ||
+      grid->n_windows < 0 || (int64_t)grid->n_windows * grid->window_ms >= (int64_t)2147483647)
+    return TRE_EINVAL;
+  if (!in || !in->P || !in->D || !in->A || !in->W || !prof || !diag) return TRE_EINVAL;
+  if (prof->dtype != TRE_F32 && prof->dtype != TRE_F64) return TRE_EINVAL;
+  if (!prof->w_p || !prof->w_q || !prof->alpha || !prof->theta || !prof->tau_crit ||
+      !prof->tau_surplus)
+    return TRE_EINVAL;
+  if (!S_out || !Z_out || !cls_out || (!S_carry) != (!init_carry)) return TRE_EINVAL;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (prof->dtype == TRE_F32)
+    return run<float>(grid, in, prof, S_carry, init_carry, S_out, Z_out, cls_out, recv_out, diag,
+                      s);
+  return run<double>(grid, in, prof, S_carry, init_carry, S_out, Z_out, cls_out, recv_out, diag,
+                     s);
+}
