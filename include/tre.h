@@ -168,8 +168,8 @@ tre_status tss_score(const tre_grid* grid, const tre_counts* in, const tre_profi
                      tre_diag* diag, tre_stream stream);
 
 /*
- * tss_calibrate -- healthy boundary theta (Sec. III-B: the smallest smoothed TSS
- * that achieves the target SLO reliability). Calibration windows have at least
+ * tss_calibrate -- healthy boundary theta (Sec. III-B: the lowest smoothed TSS at
+ * which the SLO reliability target is still met). Calibration windows have at least
  * one arrival, are not idle and have S > 0. A window is healthy when at least
  * ok_frac of the requests arriving in it met the TTFT bound slo_ttft_ms[model]
  * (device int32[n_models]). theta[m] is the smallest S value s for which the

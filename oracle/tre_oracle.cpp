@@ -12,7 +12,8 @@
 //
 // Readings (the paper does not fix these):
 //  * time base: all times are integer milliseconds; window k covers
-//    [k*win, (k+1)*win), windows start at t = 0 (Eq. 1 "window of width Delta").
+//    [k*win, (k+1)*win), windows start at t = 0 (Eq. 1 observes counts over
+//    windows of a fixed length).
 //  * prompt tokens of a request are all counted at its first-token time; decode
 //    token j (0 <= j < L_out) is emitted at t_first + floor(j*(t_end-t_first)/(L_out-1))
 //    (a single decode token is at t_first). Counters become window deltas
@@ -21,7 +22,7 @@
 //    of each window: running on [t_start, t_end), waiting on [t_arr, t_start)
 //    (Sec. III-A, Sec. V-B).
 //  * the demand denominator is floored at one request (Sec. II-B: the raw
-//    inverse sits "under the signal's floor"); a window with no tokens and no
+//    inverse is clamped at one request); a window with no tokens and no
 //    requests is IDLE.
 //  * EMA: S = alpha*raw + (1-alpha)*S_prev, started at the first non-idle window
 //    and held through idle windows (Sec. III-B).
@@ -29,7 +30,8 @@
 //    (Sec. III-B); idle windows form their own class.
 //  * theta: the smallest smoothed TSS value s such that, among calibration
 //    windows with S >= s, the healthy fraction reaches the reliability target
-//    (Sec. III-B "smallest smoothed TSS that achieves target SLO reliability").
+//    (Sec. III-B: theta is the lowest smoothed TSS at which the SLO reliability
+//    target is still met).
 //  * control ticks: a window ends a fast (slow) tick when a multiple of
 //    fast_ms (slow_ms) falls in (k*win, (k+1)*win] (Sec. IV-B, Sec. V-B).
 //  * rescue, rebalance and bounded transfer as in Sec. IV-B/IV-C, Eq. 3.

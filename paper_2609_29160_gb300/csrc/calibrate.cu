@@ -1,5 +1,5 @@
-// Calibration of the healthy boundary theta (Sec. III-B: the smallest smoothed
-// TSS value that achieves the target SLO reliability).
+// Calibration of the healthy boundary theta (Sec. III-B: the lowest smoothed TSS
+// value at which the SLO reliability target is still met).
 //
 // For model m, let the calibration windows be those with at least one arrival,
 // not idle, S > 0. For a value s let C(s) be the number of calibration windows

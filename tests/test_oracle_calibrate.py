@@ -1,5 +1,5 @@
 """Pins for the oracle's theta calibration (Sec. III-B: theta is the smallest
-smoothed TSS value that achieves the target SLO reliability).
+smoothed TSS value at which the SLO reliability target is still met).
 
 Brute force: for every candidate value s, count directly the windows with
 S >= s and how many of them are healthy; theta is the smallest qualifying s.

@@ -213,7 +213,7 @@ def test_rescue_blocks_rebalance_even_without_capacity():
 def test_heterogeneous_footprints_release_several_donors():
     """A receiver with footprint 2 needs two releases of footprint-1 donors; a
     footprint-2 donor funds a footprint-1 receiver and leaves one unit idle
-    (Sec. IV-C: a transition is not assumed to be a one-to-one exchange)."""
+    (Sec. IV-C: released and activated footprints need not match one for one)."""
     K, M = 10, 3
     Z = np.ones((K, M))
     cls = np.full((K, M), NOM, np.uint8)
