@@ -211,12 +211,12 @@ tre_status tre_select_moves(const tre_grid* grid, const void* Z, const uint8_t* 
  * tss_score_noalloc -- the same computation and outputs as tss_score, for
  * callers that cannot allocate device memory (no cudaMalloc where they run, or
  * a host that owns every allocation), so they cannot supply `ws`. It takes no
- * workspace: its scratch is a 4 MiB buffer compiled into the library, one copy
- * on every GPU that loads the library, held until the process exits. The paper
- * has no counterpart; this is a deployment variant of the scoring call.
- * Limit: ceil(n_windows / L) * n_models <= 65536 with L = max(256,
- * ceil(n_windows / 1024)) -- any n_windows for n_models <= 64; larger problems
- * return TRE_ENOMEM before anything is enqueued. The first call on a device
+ * workspace: its scratch is a 12 MiB buffer compiled into the library, one
+ * copy on every GPU that loads the library, held until the process exits. The
+ * paper has no counterpart; this is a deployment variant of the scoring call.
+ * Limit: n_windows * n_models <= 1048576 (for example 36000 windows x 8 models
+ * or 16384 x 64); larger problems return TRE_ENOMEM before anything is
+ * enqueued. The first call on a device
  * looks up the buffer's device address (make it before any stream capture).
  * All calls share the one buffer: calls whose GPU work overlaps in time (other
  * streams, other host threads) race on it and must be serialised by the

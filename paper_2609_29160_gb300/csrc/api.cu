@@ -113,27 +113,42 @@ struct Scope {
 template <class T> T to_t(double v) { return (T)v; }
 
 // ---- tss_score --------------------------------------------------------------
+// one-series table over a whole grid (per-model alpha comes from the profile)
+template <class T> SeriesTable<T> single_series(const tre_grid* g) {
+  SeriesTable<T> t;
+  std::memset(&t, 0, sizeof(t));
+  t.n = 1;
+  t.M = g->n_models;
+  t.off[0] = 0;
+  t.K[0] = g->n_windows;
+  t.win[0] = g->window_ms;
+  t.alpha[0] = (T)0.01;  // alpha is per model on the device: size segments for slow smoothing
+  series_segments(t);
+  return t;
+}
+
 template <class T>
 tre_status score_typed(const tre_grid* g, const tre_counts* in, const tre_profile* p,
                        void* S_carry, uint8_t* init_carry, void* S_out, void* Z_out,
                        uint8_t* cls_out, int32_t* recv_out, void* ws, size_t* ws_bytes,
                        tre_diag* diag, cudaStream_t s) {
   const int M = g->n_models, K = g->n_windows;
+  SeriesTable<T> tab = single_series<T>(g);
   Arena a(ws);
   ScoreWs<T> w;
-  score_ws_layout<T>(a, M, K, w);
+  score_ws_layout<T>(a, M, (int64_t)K * M, tab.seg_base[1], w);
   bool query;
   tre_status st = ws_check(a, ws, ws_bytes, query);
   if (st != TRE_OK || query) return st;
   cudaError_t e;
   {
-    Scope sc(kScore, 5, s);
-    e = launch_score<T>(
-      M, g->window_ms, K, in->P, in->D, in->A, in->W, static_cast<const T*>(p->w_p),
-      static_cast<const T*>(p->w_q), static_cast<const T*>(p->alpha),
-      static_cast<const T*>(p->theta), static_cast<const T*>(p->tau_crit),
-      static_cast<const T*>(p->tau_surplus), static_cast<T*>(S_carry), init_carry,
-      static_cast<T*>(S_out), static_cast<T*>(Z_out), cls_out, w, diag, s);
+    Scope sc(kScore, 6, s);
+    e = launch_score<T>(tab, in->P, in->D, in->A, in->W, static_cast<const T*>(p->w_p),
+                        static_cast<const T*>(p->w_q), static_cast<const T*>(p->alpha),
+                        static_cast<const T*>(p->theta), static_cast<const T*>(p->tau_crit),
+                        static_cast<const T*>(p->tau_surplus), static_cast<T*>(S_carry),
+                        init_carry, static_cast<T*>(S_out), static_cast<T*>(Z_out), cls_out, w,
+                        diag, s);
   }
   if (!e && recv_out) {
     Scope sc(kReceiver, 1, s);
@@ -149,14 +164,15 @@ tre_status calibrate_typed(const tre_grid* g, const tre_requests* req, const tre
                            double ok_frac, double rel, void* theta, void* ws, size_t* ws_bytes,
                            tre_diag* diag, cudaStream_t s) {
   const int M = g->n_models, K = g->n_windows;
+  SeriesTable<T> tab = single_series<T>(g);
   Arena a(ws);
   unsigned long long* slo = a.take<unsigned long long>((size_t)K * M);
   T* S = a.take<T>((size_t)K * M);
   uint8_t* cls = a.take<uint8_t>((size_t)K * M);
   ScoreWs<T> sw;
-  score_ws_layout<T>(a, M, K, sw);
+  score_ws_layout<T>(a, M, (int64_t)K * M, tab.seg_base[1], sw);
   CalibWs<T> cw;
-  calib_ws_layout<T>(a, M, K, cw);
+  calib_ws_layout<T>(a, (int64_t)K * M, cw);
   bool query;
   tre_status st = ws_check(a, ws, ws_bytes, query);
   if (st != TRE_OK || query) return st;
@@ -167,15 +183,14 @@ tre_status calibrate_typed(const tre_grid* g, const tre_requests* req, const tre
             : launch_slo_events(cols_of(ev), M, g->window_ms, K, slo, slo_ms, s);
   }
   if (!e) {
-    Scope sc(kScore, 5, s);
-    e = launch_score<T>(M, g->window_ms, K, in->P, in->D, in->A, in->W,
-                        static_cast<const T*>(p->w_p), static_cast<const T*>(p->w_q),
-                        static_cast<const T*>(p->alpha), nullptr, nullptr, nullptr, nullptr,
-                        nullptr, S, nullptr, cls, sw, diag, s);
+    Scope sc(kScore, 6, s);
+    e = launch_score<T>(tab, in->P, in->D, in->A, in->W, static_cast<const T*>(p->w_p),
+                        static_cast<const T*>(p->w_q), static_cast<const T*>(p->alpha), nullptr,
+                        nullptr, nullptr, nullptr, nullptr, S, nullptr, cls, sw, diag, s);
   }
   if (!e) {
     Scope sc(kCalibrate, 3, s);
-    e = launch_calibrate<T>(M, K, S, cls, slo, ok_frac, rel, static_cast<T*>(theta), cw, diag, s);
+    e = launch_calibrate<T>(tab, S, cls, slo, ok_frac, rel, static_cast<T*>(theta), cw, diag, s);
   }
   return cuda_status(e);
 }
@@ -186,10 +201,6 @@ tre_status select_typed(const tre_grid* g, const void* Z, const uint8_t* cls,
                         const tre_profile* p, const tre_ctrl* c, int32_t* r_inout, tre_move* moves,
                         int64_t cap, int64_t* n_moves, void* ws, size_t* ws_bytes, tre_diag* diag,
                         cudaStream_t s) {
-  Arena a(ws);
-  bool query;
-  tre_status st = ws_check(a, ws, ws_bytes, query);
-  if (st != TRE_OK || query) return st;
   WalkBatch<T> b;
   std::memset(&b, 0, sizeof(b));
   b.M = g->n_models;
@@ -216,8 +227,14 @@ tre_status select_typed(const tre_grid* g, const void* Z, const uint8_t* cls,
   b.moves_cap = cap;
   b.n_moves = n_moves;
   b.diag = diag;
-  Scope sc(kSelect, 1, s);
-  return cuda_status(launch_walk<T>(b, s));
+  Arena a(ws);
+  WalkWs w;
+  walk_ws_layout<T>(a, b, w);
+  bool query;
+  tre_status st = ws_check(a, ws, ws_bytes, query);
+  if (st != TRE_OK || query) return st;
+  Scope sc(kSelect, 2, s);
+  return cuda_status(launch_walk<T>(b, w, s));
 }
 
 // ---- tre_sweep --------------------------------------------------------------
@@ -231,7 +248,9 @@ struct SweepPlan {
 
 bool sweep_plan(const tre_sweep_spec* sp, SweepPlan& pl) {
   if (!sp || sp->n_models < 1 || sp->n_models > 1024 || sp->duration_ms < 1) return false;
-  if (sp->n_traces < 1 || !sp->traces || sp->n_win < 1 || !sp->window_ms || !sp->alpha) return false;
+  if (sp->n_traces < 1 || !sp->traces || sp->n_win < 1 || sp->n_win > 16 || !sp->window_ms ||
+      !sp->alpha)
+    return false;
   if (sp->n_tau < 1 || sp->n_tau > kMaxTau || !sp->tau_crit) return false;
   if (sp->n_cap < 1 || sp->n_cap > kMaxCap || !sp->pacing_cap) return false;
   if ((int64_t)sp->n_traces * sp->n_win > kMaxSeries) return false;
@@ -272,15 +291,42 @@ template <class T>
 tre_status sweep_typed(const tre_sweep_spec* sp, const SweepPlan& pl, const tre_sweep_out* out,
                        void* ws, size_t* ws_bytes, tre_diag* diag, cudaStream_t s) {
   const int M = pl.M;
+  const int NT = sp->n_traces;
+  // series table: series si = trace * n_win + w
+  SeriesTable<T> tab;
+  std::memset(&tab, 0, sizeof(tab));
+  tab.n = pl.n_series;
+  tab.M = M;
+  for (int si = 0; si < pl.n_series; ++si) {
+    const int w = si % sp->n_win;
+    tab.off[si] = pl.off[si];
+    tab.K[si] = pl.K[w];
+    tab.win[si] = sp->window_ms[w];
+    tab.alpha[si] = to_t<T>(sp->alpha[w]);
+  }
+  const int n_seg = series_segments(tab);
+  AggPlan ag;
+  std::memset(&ag, 0, sizeof(ag));
+  ag.n_traces = NT;
+  ag.n_win = sp->n_win;
+  ag.M = M;
+  ag.Kb = pl.Kb;
+  for (int w = 0; w < sp->n_win; ++w) {
+    ag.q[w] = pl.q[w];
+    ag.Kq[w] = pl.K[w];
+  }
+  for (int t = 0; t < NT; ++t)
+    for (int w = 0; w < sp->n_win; ++w) ag.out_off[t][w] = pl.off[t * sp->n_win + w];
+
   Arena a(ws);
-  const size_t nb = (size_t)pl.Kb * M;
+  const size_t nb = (size_t)pl.Kb * M * NT;
   int32_t* Pb = a.take<int32_t>(nb);
   int32_t* Db = a.take<int32_t>(nb);
   int32_t* Ab = a.take<int32_t>(nb);
   int32_t* Wb = a.take<int32_t>(nb);
   unsigned long long* slob = a.take<unsigned long long>(nb);
   ReduceWs rw;
-  reduce_ws_layout(a, M, pl.Kb, 0, rw);
+  reduce_ws_layout(a, M, pl.Kb, NT, 0, rw);
   const size_t tot = (size_t)pl.total;
   int32_t* P = out->P ? out->P : a.take<int32_t>(tot);
   int32_t* D = out->D ? out->D : a.take<int32_t>(tot);
@@ -288,60 +334,12 @@ tre_status sweep_typed(const tre_sweep_spec* sp, const SweepPlan& pl, const tre_
   int32_t* W = out->W ? out->W : a.take<int32_t>(tot);
   T* S = out->S ? static_cast<T*>(out->S) : a.take<T>(tot);
   T* Z = out->Z ? static_cast<T*>(out->Z) : a.take<T>(tot);
-  uint8_t* cls = out->cls ? out->cls : a.take<uint8_t>(tot);
   uint8_t* idle = a.take<uint8_t>(tot);
   unsigned long long* slo = a.take<unsigned long long>(tot);
   ScoreWs<T> sw;
-  score_ws_layout<T>(a, M, pl.Kmax, sw);
+  score_ws_layout<T>(a, M, (int64_t)tot, n_seg, sw);
   CalibWs<T> cw;
-  calib_ws_layout<T>(a, M, pl.Kmax, cw);
-  bool query;
-  tre_status st = ws_check(a, ws, ws_bytes, query);
-  if (st != TRE_OK || query) return st;
-
-  T* theta = static_cast<T*>(out->theta);
-  cudaError_t e = cudaSuccess;
-  for (int t = 0; t < sp->n_traces && !e; ++t) {
-    {
-      Scope sc(kReduce, 1, s);
-      e = launch_reduce_requests(cols_of(&sp->traces[t]), M, pl.base_win, pl.Kb, Pb, Db, rw,
-                                 slob, sp->slo_ttft_ms, diag, s);
-    }
-    if (!e) {
-      Scope sc(kScan, 3, s);
-      e = launch_gauge_scan(M, pl.Kb, rw, Ab, Wb, s);
-    }
-    for (int w = 0; w < sp->n_win && !e; ++w) {
-      const int si = t * sp->n_win + w;
-      const size_t o = (size_t)pl.off[si];
-      Scope sc(kAggregate, 1, s);
-      e = launch_aggregate(M, pl.K[w], pl.q[w], Pb, Db, Ab, Wb, slob, P + o, D + o, A + o, W + o,
-                           slo + o, s);
-    }
-  }
-  for (int si = 0; si < pl.n_series && !e; ++si) {
-    const int w = si % sp->n_win;
-    const size_t o = (size_t)pl.off[si];
-    const int K = pl.K[w];
-    {
-      Scope sc(kScore, 5, s);
-      e = launch_score_alpha<T>(M, sp->window_ms[w], K, P + o, D + o, A + o, W + o,
-                                static_cast<const T*>(sp->w_p), static_cast<const T*>(sp->w_q),
-                                to_t<T>(sp->alpha[w]), S + o, idle + o, sw, diag, s);
-    }
-    if (!e) {
-      Scope sc(kCalibrate, 3, s);
-      e = launch_calibrate<T>(M, K, S + o, idle + o, slo + o, sp->ok_frac, sp->reliability,
-                              theta + (size_t)si * M, cw, diag, s);
-    }
-    if (!e) {
-      Scope sc(kNormalize, 1, s);
-      e = launch_normalize<T>(M, K, S + o, idle + o, theta + (size_t)si * M, nullptr,
-                              to_t<T>(sp->tau_crit[0]), static_cast<const T*>(sp->tau_surplus),
-                              Z + o, cls + o, s);
-    }
-  }
-  if (e) return TRE_ECUDA;
+  calib_ws_layout<T>(a, (int64_t)tot, cw);
   WalkBatch<T> b;
   std::memset(&b, 0, sizeof(b));
   b.M = M;
@@ -371,8 +369,47 @@ tre_status sweep_typed(const tre_sweep_spec* sp, const SweepPlan& pl, const tre_
   b.moves_cap = out->moves_cap;
   b.n_moves = out->n_moves;
   b.diag = diag;
-  Scope sc(kSelect, 1, s);
-  return cuda_status(launch_walk<T>(b, s));
+  WalkWs wk;
+  walk_ws_layout<T>(a, b, wk);
+  bool query;
+  tre_status st = ws_check(a, ws, ws_bytes, query);
+  if (st != TRE_OK || query) return st;
+
+  T* theta = static_cast<T*>(out->theta);
+  std::vector<ReqCols> cols(NT);
+  for (int t = 0; t < NT; ++t) cols[t] = cols_of(&sp->traces[t]);
+  cudaError_t e;
+  {
+    Scope sc(kReduce, 1, s);
+    e = launch_reduce_requests(cols.data(), NT, M, pl.base_win, pl.Kb, Pb, Db, rw, slob,
+                               sp->slo_ttft_ms, diag, s);
+  }
+  if (!e) {
+    Scope sc(kScan, 3, s);
+    e = launch_gauge_scan(M, pl.Kb, rw, Ab, Wb, s);
+  }
+  if (!e) {
+    Scope sc(kAggregate, 1, s);
+    e = launch_aggregate(ag, Pb, Db, Ab, Wb, slob, P, D, A, W, slo, s);
+  }
+  if (!e) {
+    Scope sc(kScore, 6, s);
+    e = launch_score<T>(tab, P, D, A, W, static_cast<const T*>(sp->w_p),
+                        static_cast<const T*>(sp->w_q), nullptr, nullptr, nullptr, nullptr,
+                        nullptr, nullptr, S, nullptr, idle, sw, diag, s);
+  }
+  if (!e) {
+    Scope sc(kCalibrate, 3, s);
+    e = launch_calibrate<T>(tab, S, idle, slo, sp->ok_frac, sp->reliability, theta, cw, diag, s);
+  }
+  if (!e) {
+    Scope sc(kNormalize, 1, s);
+    e = launch_normalize<T>(tab, S, idle, theta, nullptr, to_t<T>(sp->tau_crit[0]),
+                            static_cast<const T*>(sp->tau_surplus), Z, out->cls, s);
+  }
+  if (e) return TRE_ECUDA;
+  Scope sc(kSelect, 2, s);
+  return cuda_status(launch_walk<T>(b, wk, s));
 }
 
 }  // namespace
@@ -428,7 +465,7 @@ tre_status tss_window_reduce(const tre_grid* grid, const tre_requests* req, cons
   const int M = grid->n_models, K = grid->n_windows;
   Arena a(ws);
   ReduceWs w;
-  reduce_ws_layout(a, M, K, ev ? ev->n_req : 0, w);
+  reduce_ws_layout(a, M, K, 1, ev ? ev->n_req : 0, w);
   bool query;
   tre_status st = ws_check(a, ws, ws_bytes, query);
   if (st != TRE_OK || query) return st;
@@ -436,8 +473,9 @@ tre_status tss_window_reduce(const tre_grid* grid, const tre_requests* req, cons
   cudaError_t e;
   {
     Scope sc(kReduce, req ? 1 : 3, s);
-    e = req ? launch_reduce_requests(cols_of(req), M, grid->window_ms, K, out.P, out.D, w,
-                                     nullptr, nullptr, diag, s)
+    const ReqCols rc = req ? cols_of(req) : ReqCols{};
+    e = req ? launch_reduce_requests(&rc, 1, M, grid->window_ms, K, out.P, out.D, w, nullptr,
+                                     nullptr, diag, s)
             : launch_reduce_events(cols_of(ev), M, grid->window_ms, K, out.P, out.D, w, diag, s);
   }
   if (!e) {

@@ -1,21 +1,23 @@
 // Calibration of the healthy boundary theta (Sec. III-B: the lowest smoothed TSS
-// value at which the SLO reliability target is still met).
+// value at which the SLO reliability target is still met), for a batch of
+// series at once.
 //
 // For model m, let the calibration windows be those with at least one arrival,
 // not idle, S > 0. For a value s let C(s) be the number of calibration windows
 // with S >= s and H(s) the healthy ones among them. theta is the smallest S
 // value s with H(s) >= reliability * C(s).
 //
-// Instead of sorting, each model's (S, healthy) pairs are packed into unsigned
-// keys (the bit pattern of a positive float orders like the float) and theta is
-// found by a radix descent over 8-bit digits: at each level a histogram of
-// counts, healthy counts and the smallest key per bucket; buckets are visited
-// from the smallest values up. A bucket whose smallest value already satisfies
-// the condition gives theta (nothing below it did). A bucket that could contain
-// a qualifying value -- the bound that adds only its healthy windows passes --
-// is refined one digit further; if the refinement finds nothing the scan
-// resumes above it. All counts are exact integers and every comparison is the
-// same double expression the definition uses, so theta is exact.
+// Instead of sorting, each (series, model) packs its (S, healthy) pairs into
+// unsigned keys (the bit pattern of a positive float orders like the float)
+// and one CTA finds theta by a descent over the key range: the current range
+// is split linearly into buckets; a histogram gives per bucket the count, the
+// healthy count and the smallest key; per bucket, in parallel, the exact test
+// at its smallest value (everything at or above it included) and an upper
+// bound for any value inside it (only its healthy windows added). The lowest
+// bucket that passes either gives theta directly (its smallest value
+// qualifies and nothing below did) or is refined; a refinement that finds
+// nothing resumes with the buckets above it. Counts are exact integers and the
+// final test is the definition's double expression, so theta is exact.
 #include <algorithm>
 
 #include "common.cuh"
@@ -25,17 +27,23 @@ namespace tre {
 namespace {
 
 constexpr int kThrTable = 4096;
-constexpr int kSearchThreads = 1024;
+constexpr int kNB = 512;            // buckets per level = threads per CTA
+constexpr int kWarps = kNB / 32;
 
 template <class T> struct KeyOf;
 template <> struct KeyOf<float> {
   using U = uint32_t;
-  static constexpr int kBits = 31;  // key bits of a non-negative float
+  static constexpr int kLevels = 4;   // 31 key bits, >= 9 bits resolved per level
 };
 template <> struct KeyOf<double> {
   using U = unsigned long long;
-  static constexpr int kBits = 63;
+  static constexpr int kLevels = 7;   // 63 key bits
 };
+
+__device__ __forceinline__ float value_of(uint32_t k) { return __uint_as_float(k); }
+__device__ __forceinline__ double value_of(unsigned long long k) {
+  return __longlong_as_double((long long)k);
+}
 
 // thr[a] = smallest integer n with (double)n >= ok_frac * (double)a
 __global__ void k_thr(double ok_frac, int32_t* thr) {
@@ -55,198 +63,249 @@ __device__ __forceinline__ bool healthy(uint32_t n_arr, uint32_t n_met, const in
   return (double)n_met >= ok_frac * (double)n_arr;
 }
 
-// [K][M] S, cls, packed SLO counts -> [M][K] packed keys (0 = not a calibration window)
+// [K][M] S, class, packed SLO counts of every series -> [M][K] packed keys
+// (0 = not a calibration window) at the series' element offset
 template <class T>
-__global__ void k_pack(int M, int K, const T* __restrict__ S, const uint8_t* __restrict__ cls,
-                       const unsigned long long* __restrict__ slo, const int32_t* __restrict__ thr,
-                       double ok_frac, typename KeyOf<T>::U* __restrict__ keys) {
+__global__ void k_pack(const __grid_constant__ SeriesTable<T> tab, const T* __restrict__ S,
+                       const uint8_t* __restrict__ cls, const unsigned long long* __restrict__ slo,
+                       const int32_t* __restrict__ thr, double ok_frac,
+                       typename KeyOf<T>::U* __restrict__ keys) {
   using U = typename KeyOf<T>::U;
   __shared__ U tile[32][33];
+  const int s = blockIdx.z;
+  const int M = tab.M, K = tab.K[s];
   const int k0 = blockIdx.x * 32, m0 = blockIdx.y * 32;
+  if (k0 >= K) return;
+  const size_t off = (size_t)tab.off[s];
   for (int j = threadIdx.y; j < 32; j += blockDim.y) {
     const int k = k0 + j, m = m0 + threadIdx.x;
     U v = 0;
     if (k < K && m < M) {
-      const size_t x = (size_t)k * M + m;
+      const size_t x = off + (size_t)k * M + m;
       const unsigned long long c = slo[x];
       const uint32_t n_arr = (uint32_t)c, n_met = (uint32_t)(c >> 32);
-      const T s = S[x];
-      if (cls[x] != kIdle && n_arr >= 1 && s > (T)0)
-        v = ((U)key_of(s) << 1) | (U)(healthy(n_arr, n_met, thr, ok_frac) ? 1 : 0);
+      const T sv = S[x];
+      if (cls[x] != kIdle && n_arr >= 1 && sv > (T)0)
+        v = ((U)key_of(sv) << 1) | (U)(healthy(n_arr, n_met, thr, ok_frac) ? 1 : 0);
     }
     tile[j][threadIdx.x] = v;
   }
   __syncthreads();
   for (int j = threadIdx.y; j < 32; j += blockDim.y) {
     const int m = m0 + j, k = k0 + threadIdx.x;
-    if (m < M && k < K) keys[(size_t)m * K + k] = tile[threadIdx.x][j];
+    if (m < M && k < K) keys[off + (size_t)m * K + k] = tile[threadIdx.x][j];
   }
 }
 
-template <class T>
-__global__ void __launch_bounds__(kSearchThreads)
-k_search(int M, int K, const typename KeyOf<T>::U* __restrict__ keys, double reliability,
-         T* theta, tre_diag* diag) {
-  using U = typename KeyOf<T>::U;
-  constexpr int NB = 256;
-  constexpr int NL = (KeyOf<T>::kBits + 7) / 8;
-  __shared__ int32_t cnt[NL][NB], hl[NL][NB];
-  __shared__ int64_t tot_c[NL], tot_h[NL];
-  __shared__ U mn[NL][NB];
-  __shared__ int64_t cab[NL], hab[NL];
-  __shared__ U prefix[NL];
-  __shared__ int pos[NL];
-  __shared__ int level, action, act_b;
-  __shared__ U max_key;
-  __shared__ U result;
-  const int m = blockIdx.x;
-  const U* mk = keys + (size_t)m * K;
+// exclusive suffix sums over the block: out = sum of v over threads > tid
+__device__ __forceinline__ int64_t block_suffix(int64_t v, int64_t* red) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x / 32;
+  // inclusive suffix within the warp (lanes above)
+  int64_t inc = v;
+  for (int o = 1; o < 32; o <<= 1) {
+    const int64_t x = __shfl_down_sync(0xffffffffu, inc, o);
+    if (lane + o < 32) inc += x;
+  }
+  if (lane == 0) red[wid] = inc;
+  __syncthreads();
+  int64_t above = 0;
+  for (int w = wid + 1; w < kWarps; ++w) above += red[w];
+  __syncthreads();
+  return inc - v + above;
+}
 
-  auto lo_bit = [](int l) { return max(0, KeyOf<T>::kBits - 8 * (l + 1)); };
+__device__ __forceinline__ int block_min(int v, int* red) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x / 32;
+  v = __reduce_min_sync(0xffffffffu, v);
+  if (lane == 0) red[wid] = v;
+  __syncthreads();
+  int r = 0x7fffffff;
+  for (int w = 0; w < kWarps; ++w) r = min(r, red[w]);
+  __syncthreads();
+  return r;
+}
+
+template <class T>
+__global__ void __launch_bounds__(kNB)
+k_search(const __grid_constant__ SeriesTable<T> tab, const typename KeyOf<T>::U* __restrict__ keys,
+         double reliability, T* theta, tre_diag* diag) {
+  using U = typename KeyOf<T>::U;
+  constexpr int NL = KeyOf<T>::kLevels;
+  __shared__ int32_t cnt[NL][kNB], hl[NL][kNB];
+  __shared__ U mn[NL][kNB];
+  __shared__ U lo_s[NL], hi_s[NL];
+  __shared__ int shift_s[NL], pos_s[NL];
+  __shared__ int64_t cab_s[NL], hab_s[NL];
+  __shared__ int64_t red64[kWarps];
+  __shared__ int red32[kWarps];
+  __shared__ U kmin_s, kmax_s;
+  __shared__ unsigned long long ncand_s;
+  const int M = tab.M;
+  const int s = blockIdx.x / M, m = blockIdx.x % M;
+  const int K = tab.K[s];
+  const U* mk = keys + (size_t)tab.off[s] + (size_t)m * K;
+  const int tid = threadIdx.x, lane = tid & 31;
+
+  // range of candidate keys
+  if (tid == 0) {
+    kmin_s = ~(U)0;
+    kmax_s = 0;
+    ncand_s = 0;
+  }
+  __syncthreads();
+  U lmin = ~(U)0, lmax = 0;
+  unsigned long long lc = 0;
+  for (int i = tid; i < K; i += kNB) {
+    const U p = mk[i];
+    if (!p) continue;
+    const U key = p >> 1;
+    lmin = key < lmin ? key : lmin;
+    lmax = key > lmax ? key : lmax;
+    ++lc;
+  }
+  if (lc) {
+    atomicMin(&kmin_s, lmin);
+    atomicMax(&kmax_s, lmax);
+    atomicAdd(&ncand_s, lc);
+  }
+  __syncthreads();
+  const size_t out = (size_t)s * M + m;
+  if (ncand_s == 0) {
+    if (tid == 0) {
+      theta[out] = (T)1;
+      atomicAdd(&diag->degenerate_calib, 1ull);
+    }
+    return;
+  }
+
+  // histogram of the keys in [lo, hi] of level l, bucket (key - lo) >> shift
   auto build = [&](int l) {
-    for (int b = threadIdx.x; b < NB; b += blockDim.x) {
-      cnt[l][b] = 0;
-      hl[l][b] = 0;
-      mn[l][b] = ~(U)0;
-    }
+    cnt[l][tid] = 0;
+    hl[l][tid] = 0;
+    mn[l][tid] = ~(U)0;
     __syncthreads();
-    const int lo = lo_bit(l);
-    const int hi = KeyOf<T>::kBits - 8 * l;   // bits [lo, hi) are this level's digit
-    const U pre = prefix[l];
-    U local_max = 0;
-    for (int64_t i = threadIdx.x; i < K; i += blockDim.x) {
-      const U p = mk[i];
-      if (!p) continue;
+    const U lo = lo_s[l], hi = hi_s[l];
+    const int sh = shift_s[l];
+    for (int i0 = 0; i0 < K; i0 += kNB) {
+      const int i = i0 + tid;
+      const U p = i < K ? mk[i] : (U)0;
       const U key = p >> 1;
-      if (l == 0) local_max = key > local_max ? key : local_max;
-      if (hi < KeyOf<T>::kBits && (key >> hi) != pre) continue;
-      const int b = (int)((key >> lo) & (U)(NB - 1));
-      atomicAdd(&cnt[l][b], 1);
-      if (p & 1) atomicAdd(&hl[l][b], 1);
-      atomicMin(&mn[l][b], key);
-    }
-    if (l == 0 && local_max) atomicMax(&max_key, local_max);
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      int64_t tc = 0, th = 0;
-      for (int b = 0; b < NB; ++b) {
-        tc += cnt[l][b];
-        th += hl[l][b];
+      const bool in = p != 0 && key >= lo && key <= hi;
+      const int b = in ? (int)((key - lo) >> sh) : -1;
+      const unsigned act = __ballot_sync(0xffffffffu, in);
+      if (in) {
+        const unsigned grp = __match_any_sync(act, b);
+        const unsigned hgrp = __ballot_sync(grp, (p & 1) != 0);
+        if (lane == __ffs(grp) - 1) {
+          atomicAdd(&cnt[l][b], __popc(grp));
+          if (hgrp) atomicAdd(&hl[l][b], __popc(hgrp));
+        }
+        if (key < mn[l][b]) atomicMin(&mn[l][b], key);
       }
-      tot_c[l] = tc;
-      tot_h[l] = th;
-      pos[l] = 0;
     }
     __syncthreads();
   };
 
-  if (threadIdx.x == 0) {
-    level = 0;
-    prefix[0] = 0;
-    cab[0] = 0;
-    hab[0] = 0;
-    max_key = 0;
-  }
+  // level 0 covers [kmin, kmax]
+  auto set_range = [&](int l, U lo, U hi, int64_t ca, int64_t ha) {
+    int sh = 0;
+    while (sh < 63 && ((hi - lo) >> sh) >= (U)kNB) ++sh;
+    lo_s[l] = lo;
+    hi_s[l] = hi;
+    shift_s[l] = sh;
+    pos_s[l] = 0;
+    cab_s[l] = ca;
+    hab_s[l] = ha;
+  };
+  if (tid == 0) set_range(0, kmin_s, kmax_s, 0, 0);
   __syncthreads();
   build(0);
-  // action: 0 = descend into act_b, 1 = found, 2 = pop, 3 = none at all
+  int l = 0;
   while (true) {
-    if (threadIdx.x == 0) {
-      const int l = level;
-      action = 2;
-      int64_t run_c = 0, run_h = 0;  // windows in buckets below b
-      for (int b = 0; b < pos[l]; ++b) {
-        run_c += cnt[l][b];
-        run_h += hl[l][b];
+    // per bucket: windows above it (inside this range and above the range)
+    const int64_t c_above = block_suffix(cnt[l][tid], red64) + cab_s[l];
+    const int64_t h_above = block_suffix(hl[l][tid], red64) + hab_s[l];
+    const int32_t c = cnt[l][tid], h = hl[l][tid];
+    int cand = 0x7fffffff;
+    int kind = 0;   // 1 = its smallest value qualifies, 2 = may contain one
+    if (c > 0 && tid >= pos_s[l]) {
+      if ((double)(h_above + h) >= reliability * (double)(c_above + c)) {
+        kind = 1;
+      } else if (shift_s[l] > 0 &&
+                 (double)(h_above + h + 1) >= reliability * (double)(c_above + h)) {
+        // a value inside the bucket adds at most its healthy windows to those
+        // above; one window of slack keeps the bound valid under rounding
+        kind = 2;
       }
-      for (int b = pos[l]; b < NB; ++b) {
-        run_c += cnt[l][b];
-        run_h += hl[l][b];
-        if (!cnt[l][b]) continue;
-        // windows of this range in buckets above b, plus everything above the range
-        const int64_t Ca = cab[l] + tot_c[l] - run_c, Ha = hab[l] + tot_h[l] - run_h;
-        const int64_t C = Ca + cnt[l][b], H = Ha + hl[l][b];
-        if ((double)H >= reliability * (double)C) {
-          action = 1;
-          result = mn[l][b];
-          break;
-        }
-        // a value inside the bucket has at most its healthy windows on top of
-        // those above; one window of slack keeps the bound valid under rounding
-        if (l + 1 < NL &&
-            (double)(Ha + hl[l][b] + 1) >= reliability * (double)(Ca + hl[l][b])) {
-          action = 0;
-          act_b = b;
-          pos[l] = b + 1;
-          cab[l + 1] = Ca;
-          hab[l + 1] = Ha;
-          prefix[l + 1] = (prefix[l] << 8) | (U)b;
-          level = l + 1;
-          break;
-        }
-      }
-      if (action == 2) {
-        if (l == 0) action = 3;
-        else level = l - 1;
-      }
+      if (kind) cand = tid;
     }
-    __syncthreads();
-    const int a = action;
-    if (a == 0) {
-      build(level);
-      continue;
-    }
-    if (a == 2) {
+    const int b = block_min(cand, red32);
+    if (b == 0x7fffffff) {
+      // nothing in this range: resume the parent range above the refined bucket
+      if (l == 0) {
+        if (tid == 0) {
+          theta[out] = value_of(kmax_s);
+          atomicAdd(&diag->degenerate_calib, 1ull);
+        }
+        return;
+      }
+      --l;
       __syncthreads();
       continue;
     }
-    if (threadIdx.x == 0) {
-      T th;
-      if (a == 1) {
-        th = [&] { U k = result; T v; memcpy(&v, &k, sizeof(T)); return v; }();
-      } else if (max_key) {
-        U k = max_key;
-        memcpy(&th, &k, sizeof(T));
-        atomicAdd(&diag->degenerate_calib, 1ull);
-      } else {
-        th = (T)1;
-        atomicAdd(&diag->degenerate_calib, 1ull);
-      }
-      theta[m] = th;
+    if (tid == b) red32[0] = kind;
+    __syncthreads();
+    const int kb = red32[0];
+    if (kb == 1) {
+      if (tid == 0) theta[out] = value_of(mn[l][b]);
+      return;
     }
-    break;
+    // refine bucket b
+    if (tid == b) {
+      const U lo = lo_s[l] + ((U)b << shift_s[l]);
+      const U hi = lo + (((U)1 << shift_s[l]) - 1);
+      pos_s[l] = b + 1;
+      set_range(l + 1, lo, hi, c_above, h_above);
+    }
+    __syncthreads();
+    ++l;
+    build(l);
   }
 }
 
 }  // namespace
 
-template <class T> void calib_ws_layout(Arena& a, int M, int K, CalibWs<T>& w) {
-  w.keys = a.take<typename KeyOf<T>::U>((size_t)M * std::max(K, 1));
+template <class T> void calib_ws_layout(Arena& a, int64_t elems, CalibWs<T>& w) {
+  w.keys = a.take<typename KeyOf<T>::U>((size_t)std::max<int64_t>(elems, 1));
   w.thr = a.take<int32_t>(kThrTable);
 }
 
 template <class T>
-cudaError_t launch_calibrate(int M, int K, const T* S, const uint8_t* cls,
+cudaError_t launch_calibrate(const SeriesTable<T>& tab, const T* S, const uint8_t* cls,
                              const unsigned long long* slo, double ok_frac, double reliability,
                              T* theta, CalibWs<T>& w, tre_diag* diag, cudaStream_t s) {
   using U = typename KeyOf<T>::U;
   k_thr<<<kThrTable / 256, 256, 0, s>>>(ok_frac, w.thr);
-  if (K > 0) {
-    dim3 g((K + 31) / 32, (M + 31) / 32), b(32, 8);
-    k_pack<T><<<g, b, 0, s>>>(M, K, S, cls, slo, w.thr, ok_frac, static_cast<U*>(w.keys));
+  int Kmax = 0;
+  for (int i = 0; i < tab.n; ++i) Kmax = std::max(Kmax, tab.K[i]);
+  if (Kmax > 0) {
+    dim3 g((Kmax + 31) / 32, (tab.M + 31) / 32, tab.n), b(32, 8);
+    k_pack<T><<<g, b, 0, s>>>(tab, S, cls, slo, w.thr, ok_frac, static_cast<U*>(w.keys));
   }
-  k_search<T><<<M, kSearchThreads, 0, s>>>(M, K, static_cast<const U*>(w.keys), reliability,
-                                           theta, diag);
+  k_search<T><<<tab.n * tab.M, kNB, 0, s>>>(tab, static_cast<const U*>(w.keys), reliability,
+                                            theta, diag);
   return cudaGetLastError();
 }
 
-template void calib_ws_layout<float>(Arena&, int, int, CalibWs<float>&);
-template void calib_ws_layout<double>(Arena&, int, int, CalibWs<double>&);
-template cudaError_t launch_calibrate<float>(int, int, const float*, const uint8_t*,
-                                             const unsigned long long*, double, double, float*,
-                                             CalibWs<float>&, tre_diag*, cudaStream_t);
-template cudaError_t launch_calibrate<double>(int, int, const double*, const uint8_t*,
-                                              const unsigned long long*, double, double, double*,
-                                              CalibWs<double>&, tre_diag*, cudaStream_t);
+template void calib_ws_layout<float>(Arena&, int64_t, CalibWs<float>&);
+template void calib_ws_layout<double>(Arena&, int64_t, CalibWs<double>&);
+template cudaError_t launch_calibrate<float>(const SeriesTable<float>&, const float*,
+                                             const uint8_t*, const unsigned long long*, double,
+                                             double, float*, CalibWs<float>&, tre_diag*,
+                                             cudaStream_t);
+template cudaError_t launch_calibrate<double>(const SeriesTable<double>&, const double*,
+                                              const uint8_t*, const unsigned long long*, double,
+                                              double, double*, CalibWs<double>&, tre_diag*,
+                                              cudaStream_t);
 
 }  // namespace tre

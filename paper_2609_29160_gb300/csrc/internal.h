@@ -37,18 +37,22 @@ struct EvCols {
 };
 
 // ---- reduce.cu ------------------------------------------------------------
-// Reduction scratch: diff arrays [K+1][M] for the gauges, per-request first and
-// last event ticks, scan partials.
+// Reduction scratch for a batch of traces on one grid: diff arrays
+// [trace][K+1][M] for the gauges, per-request first and last event ticks, scan
+// partials [trace][chunk][M].
 struct ReduceWs {
   int32_t *dA, *dW;
   int32_t *first, *last;       // events only, [n_req]
-  int32_t *partA, *partW;      // [n_chunks][M]
+  int32_t *partA, *partW;
+  int n_traces;
 };
-void reduce_ws_layout(Arena& a, int M, int K, int64_t n_req, ReduceWs& w);
-// slo (may be null): packed per-(window, model) arrivals (low 32 bits) and
-// arrivals that met the TTFT bound (high 32 bits), added to.
-cudaError_t launch_reduce_requests(const ReqCols& r, int M, int win, int K, int32_t* P,
-                                   int32_t* D, ReduceWs& w, unsigned long long* slo,
+void reduce_ws_layout(Arena& a, int M, int K, int n_traces, int64_t n_req, ReduceWs& w);
+// Request records of n_traces traces (host array of column sets) on one grid;
+// trace t writes P, D (and the packed SLO counts when slo != null) at element
+// offset t*K*M. slo packs per-(window, model) arrivals (low 32 bits) and the
+// arrivals that met the TTFT bound (high 32 bits).
+cudaError_t launch_reduce_requests(const ReqCols* traces, int n_traces, int M, int win, int K,
+                                   int32_t* P, int32_t* D, ReduceWs& w, unsigned long long* slo,
                                    const int32_t* slo_ms, tre_diag* diag, cudaStream_t s);
 cudaError_t launch_reduce_events(const EvCols& e, int M, int win, int K, int32_t* P, int32_t* D,
                                  ReduceWs& w, tre_diag* diag, cudaStream_t s);
@@ -56,63 +60,84 @@ cudaError_t launch_slo_requests(const ReqCols& r, int M, int win, int K,
                                 unsigned long long* slo, const int32_t* slo_ms, cudaStream_t s);
 cudaError_t launch_slo_events(const EvCols& e, int M, int win, int K, unsigned long long* slo,
                               const int32_t* slo_ms, cudaStream_t s);
-// inclusive scan of the diff arrays over windows -> A, W
+// inclusive scan of the diff arrays over windows -> A, W (trace t at t*K*M)
 cudaError_t launch_gauge_scan(int M, int K, ReduceWs& w, int32_t* A, int32_t* W, cudaStream_t s);
-// exact aggregation of a base grid to a coarser one (q base windows per window)
-cudaError_t launch_aggregate(int M, int Kq, int q, const int32_t* P, const int32_t* D,
+// exact coarsening of every trace's base grid to every window length: counts
+// add over q base windows, gauges are read at the last base window
+struct AggPlan {
+  int n_traces, n_win, M, Kb;
+  int32_t q[16], Kq[16];
+  int64_t out_off[64][16];      // element offset of (trace, window length) in the outputs
+};
+cudaError_t launch_aggregate(const AggPlan& plan, const int32_t* P, const int32_t* D,
                              const int32_t* A, const int32_t* W, const unsigned long long* slo,
                              int32_t* Pq, int32_t* Dq, int32_t* Aq, int32_t* Wq,
                              unsigned long long* sloq, cudaStream_t s);
 
+// ---- series tables ----------------------------------------------------------
+// A batch of series (one per (trace, window length) in a sweep, one for the
+// single-trace entry points) laid out back to back: series s occupies elements
+// [off[s], off[s] + K[s]*M) of every per-window array. Passed by value.
+constexpr int kMaxSeries = 64, kMaxTau = 32, kMaxCap = 32;
+template <class T> struct SeriesTable {
+  int n, M;
+  int64_t off[kMaxSeries];
+  int32_t K[kMaxSeries];
+  int32_t win[kMaxSeries];
+  T alpha[kMaxSeries];            // per series, used when the per-model alpha is null
+  int32_t seg_len[kMaxSeries];    // smoothing segment length of the series
+  int32_t seg_base[kMaxSeries + 1];  // prefix sum of segments per series
+};
+// fill seg_len / seg_base from K (returns the total segment count)
+template <class T> int series_segments(SeriesTable<T>& t);
+
 // ---- score.cu -------------------------------------------------------------
 template <class T> struct ScoreWs {
-  T *sum_m, *sum_c, *sum_ci;   // per-segment affine summaries [n_seg][M]
+  T* raw;                      // Eq. 1 value per element (idle windows hold junk)
+  T *sum_m, *sum_c, *sum_ci;   // per-(segment, model) affine summaries
   int32_t* sum_h;
-  T* start_S;                  // start state used by the stored trajectory [n_seg][M]
+  T* start_S;                  // start state of the stored trajectory
   int32_t* start_init;
-  T *end_S, *end_S2;           // end states (double buffered) [n_seg][M]
+  T *end_S, *end_S2;           // end states (double buffered)
   int32_t *end_init, *end_init2;
-  int n_seg, seg_len;
+  int cap_seg;                 // segments the arrays hold (per model)
 };
-template <class T> void score_ws_layout(Arena& a, int M, int K, ScoreWs<T>& w);
-// profile arrays are device pointers of T; theta may be null (Z not written)
+template <class T> void score_ws_layout(Arena& a, int M, int64_t elems, int n_seg, ScoreWs<T>& w);
+// Eq. 1, smoothing and (when theta is given) Z and regions for every series
+// of the table. Profile arrays are device [M]; alpha may be null (then the
+// table's per-series value is used); theta null = S only (cls = IDLE / NOM).
+// The carries (device [M], may be null) apply to a one-series table.
 template <class T>
-cudaError_t launch_score(int M, int win, int K, const int32_t* P, const int32_t* D,
+cudaError_t launch_score(const SeriesTable<T>& tab, const int32_t* P, const int32_t* D,
                          const int32_t* A, const int32_t* W, const T* w_p, const T* w_q,
                          const T* alpha, const T* theta, const T* tau_crit, const T* tau_surp,
                          T* S_carry, uint8_t* init_carry, T* S, T* Z, uint8_t* cls,
                          ScoreWs<T>& w, tre_diag* diag, cudaStream_t s);
-// same, with one alpha value for all models given on the host
+// Z = S / theta[series][m] and regions for every series (tau_crit device [M] or
+// one value for all)
 template <class T>
-cudaError_t launch_score_alpha(int M, int win, int K, const int32_t* P, const int32_t* D,
-                               const int32_t* A, const int32_t* W, const T* w_p, const T* w_q,
-                               T alpha, T* S, uint8_t* cls, ScoreWs<T>& w, tre_diag* diag,
-                               cudaStream_t s);
-// Z = S / theta and regions (tau arrays device, or one host value when the
-// pointer is null)
-template <class T>
-cudaError_t launch_normalize(int M, int K, const T* S, const uint8_t* idle_cls, const T* theta,
-                             const T* tau_crit, T tau_crit_v, const T* tau_surp, T* Z,
-                             uint8_t* cls, cudaStream_t s);
+cudaError_t launch_normalize(const SeriesTable<T>& tab, const T* S, const uint8_t* idle_cls,
+                             const T* theta, const T* tau_crit, T tau_crit_v, const T* tau_surp,
+                             T* Z, uint8_t* cls, cudaStream_t s);
 template <class T>
 cudaError_t launch_receiver(int M, int K, const T* Z, const uint8_t* cls, int32_t* recv,
                             cudaStream_t s);
 
 // ---- calibrate.cu ---------------------------------------------------------
 template <class T> struct CalibWs {
-  void* keys;                  // [M][K] packed keys (u32 for float, u64 for double)
+  void* keys;                  // packed keys, same element offsets as the series
   int32_t* thr;                // healthy threshold table
 };
-template <class T> void calib_ws_layout(Arena& a, int M, int K, CalibWs<T>& w);
+template <class T> void calib_ws_layout(Arena& a, int64_t elems, CalibWs<T>& w);
+// theta[s*M + m] for every series of the table
 template <class T>
-cudaError_t launch_calibrate(int M, int K, const T* S, const uint8_t* cls,
+cudaError_t launch_calibrate(const SeriesTable<T>& tab, const T* S, const uint8_t* cls,
                              const unsigned long long* slo, double ok_frac, double reliability,
                              T* theta, CalibWs<T>& w, tre_diag* diag, cudaStream_t s);
 
 // ---- select.cu ------------------------------------------------------------
 // One controller instance per (series, tau, cap). The small per-series tables
 // travel by value in the kernel parameters.
-constexpr int kMaxSeries = 64, kMaxTau = 32, kMaxCap = 32;
 template <class T> struct WalkBatch {
   int M, n_inst, n_series, n_tau, n_cap;
   int64_t series_off[kMaxSeries];  // element offset of each series in Z / cls
@@ -132,7 +157,15 @@ template <class T> struct WalkBatch {
   int64_t moves_cap;
   int64_t* n_moves;                // [n_inst]
   tre_diag* diag;
+  int32_t ent_base[kMaxSeries + 1];  // tick entries (fast then slow) per series, prefix
 };
-template <class T> cudaError_t launch_walk(const WalkBatch<T>& b, cudaStream_t s);
+// per-(series, tau, tick) receiver and per-model donor ranks
+struct WalkWs {
+  int16_t* recv;
+  uint16_t* rank;
+};
+// lays out the tick tables and fills b.ent_base
+template <class T> void walk_ws_layout(Arena& a, WalkBatch<T>& b, WalkWs& w);
+template <class T> cudaError_t launch_walk(const WalkBatch<T>& b, WalkWs& w, cudaStream_t s);
 
 }  // namespace tre

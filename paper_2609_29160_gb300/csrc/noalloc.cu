@@ -5,16 +5,20 @@
 // a fixed buffer compiled into this library instead of a caller workspace.
 #include <cuda_runtime.h>
 
+#include <cstring>
+
 #include "internal.h"
 
 using namespace tre;
 
 namespace {
 
-// Per-(segment, model) smoothing state of the scoring scan: at most this many
-// (segment, model) pairs, at 64 bytes each in double precision, plus alignment.
-constexpr int64_t kMaxSegModels = 65536;
-constexpr size_t kScratchBytes = (size_t)kMaxSegModels * 64 + 16 * 256;
+// Scratch of one scoring call: the Eq. 1 value of every (window, model) and the
+// per-(segment, model) smoothing state, in double precision at most
+// 8 * K*M + 64 * segments*M bytes plus alignment.
+constexpr int64_t kMaxElems = 1 << 20;        // K * M
+constexpr int64_t kMaxSegModels = 65536;      // segments * M
+constexpr size_t kScratchBytes = (size_t)kMaxElems * 8 + (size_t)kMaxSegModels * 64 + 16 * 256;
 
 // One copy per GPU that loads this library; it stays allocated until the
 // process exits. In host code this name is only a host-side stand-in: kernels
@@ -44,17 +48,27 @@ tre_status run(const tre_grid* g, const tre_counts* in, const tre_profile* p, vo
                uint8_t* init_carry, void* S_out, void* Z_out, uint8_t* cls_out,
                int32_t* recv_out, tre_diag* diag, cudaStream_t s) {
   const int M = g->n_models, K = g->n_windows;
+  SeriesTable<T> tab;
+  memset(&tab, 0, sizeof(tab));
+  tab.n = 1;
+  tab.M = M;
+  tab.K[0] = K;
+  tab.win[0] = g->window_ms;
+  tab.alpha[0] = (T)0.01;  // alpha is per model on the device: size segments for slow smoothing
+  const int n_seg = series_segments(tab);
+  const int64_t elems = (int64_t)K * M;
   Arena measure(nullptr);
   ScoreWs<T> w;
-  score_ws_layout<T>(measure, M, K, w);
-  if ((int64_t)w.n_seg * M > kMaxSegModels || measure.off > kScratchBytes) return TRE_ENOMEM;
+  score_ws_layout<T>(measure, M, elems, n_seg, w);
+  if (elems > kMaxElems || (int64_t)n_seg * M > kMaxSegModels || measure.off > kScratchBytes)
+    return TRE_ENOMEM;
   void* base = nullptr;
   tre_status st = scratch_address(&base);
   if (st != TRE_OK) return st;
   Arena a(base);
-  score_ws_layout<T>(a, M, K, w);
+  score_ws_layout<T>(a, M, elems, n_seg, w);
   cudaError_t e = launch_score<T>(
-      M, g->window_ms, K, in->P, in->D, in->A, in->W, static_cast<const T*>(p->w_p),
+      tab, in->P, in->D, in->A, in->W, static_cast<const T*>(p->w_p),
       static_cast<const T*>(p->w_q), static_cast<const T*>(p->alpha),
       static_cast<const T*>(p->theta), static_cast<const T*>(p->tau_crit),
       static_cast<const T*>(p->tau_surplus), static_cast<T*>(S_carry), init_carry,

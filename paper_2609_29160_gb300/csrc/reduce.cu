@@ -35,16 +35,35 @@ __device__ __forceinline__ void stage_add(V* s, V* g, int64_t k, int64_t k_lo, i
 }
 
 // --------------------------------------------------------------------------
-// request records -> P, D, gauge diffs, optional packed SLO counts
+// request records -> P, D, gauge diffs, optional packed SLO counts, for a
+// batch of traces on one grid (CTAs [cta_base[t], cta_base[t+1]) take trace t)
 // --------------------------------------------------------------------------
+constexpr int kMaxTraces = 64;
+struct ReqBatch {
+  int n;
+  ReqCols cols[kMaxTraces];
+  int64_t per_cta[kMaxTraces];
+  int32_t cta_base[kMaxTraces + 1];
+};
+
 template <bool SLO>
 __global__ void __launch_bounds__(kThreads)
-k_reduce_requests(ReqCols r, int M, int win, int K, int64_t per_cta, int rows,
-                  int32_t* __restrict__ P, int32_t* __restrict__ D, int32_t* __restrict__ dA,
-                  int32_t* __restrict__ dW, unsigned long long* __restrict__ slo,
+k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int win, int K, int rows,
+                  int32_t* __restrict__ P0, int32_t* __restrict__ D0, int32_t* __restrict__ dA0,
+                  int32_t* __restrict__ dW0, unsigned long long* __restrict__ slo0,
                   const int32_t* __restrict__ slo_ms, tre_diag* diag) {
   extern __shared__ unsigned long long smem[];
-  const int64_t i0 = (int64_t)blockIdx.x * per_cta;
+  int t = 0;
+  while (t + 1 < bt.n && bt.cta_base[t + 1] <= (int)blockIdx.x) ++t;
+  const ReqCols& r = bt.cols[t];
+  const int64_t per_cta = bt.per_cta[t];
+  const size_t cells0 = (size_t)K * M, cells1 = (size_t)(K + 1) * M;
+  int32_t* P = P0 + t * cells0;
+  int32_t* D = D0 + t * cells0;
+  int32_t* dA = dA0 + t * cells1;
+  int32_t* dW = dW0 + t * cells1;
+  unsigned long long* slo = SLO ? slo0 + t * cells0 : nullptr;
+  const int64_t i0 = (int64_t)(blockIdx.x - bt.cta_base[t]) * per_cta;
   const int64_t i1 = min(r.n, i0 + per_cta);
   if (i0 >= i1) return;
   const int64_t span = (int64_t)K * win;
@@ -317,6 +336,10 @@ k_scan_partials(int M, int K, int L, int n_chunks, const int32_t* __restrict__ d
                 int32_t* __restrict__ pW) {
   const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
   if (t >= (int64_t)n_chunks * M) return;
+  dA += (size_t)blockIdx.y * (K + 1) * M;
+  dW += (size_t)blockIdx.y * (K + 1) * M;
+  pA += (size_t)blockIdx.y * n_chunks * M;
+  pW += (size_t)blockIdx.y * n_chunks * M;
   const int m = (int)(t % M);
   const int c = (int)(t / M);
   const int64_t r0 = (int64_t)c * L, r1 = min64(r0 + L, K);
@@ -334,6 +357,8 @@ __global__ void k_scan_chunks(int M, int n_chunks, int32_t* __restrict__ pA,
                               int32_t* __restrict__ pW) {
   const int m = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
   if (m >= M) return;
+  pA += (size_t)blockIdx.y * n_chunks * M;
+  pW += (size_t)blockIdx.y * n_chunks * M;
   const int lane = threadIdx.x & 31;
   const int per = (n_chunks + 31) / 32;
   const int c0 = lane * per, c1 = min(n_chunks, c0 + per);
@@ -362,6 +387,12 @@ k_scan_apply(int M, int K, int L, int n_chunks, const int32_t* __restrict__ dA,
              const int32_t* __restrict__ pW, int32_t* __restrict__ A, int32_t* __restrict__ W) {
   const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
   if (t >= (int64_t)n_chunks * M) return;
+  dA += (size_t)blockIdx.y * (K + 1) * M;
+  dW += (size_t)blockIdx.y * (K + 1) * M;
+  pA += (size_t)blockIdx.y * n_chunks * M;
+  pW += (size_t)blockIdx.y * n_chunks * M;
+  A += (size_t)blockIdx.y * K * M;
+  W += (size_t)blockIdx.y * K * M;
   const int m = (int)(t % M);
   const int c = (int)(t / M);
   const int64_t r0 = (int64_t)c * L, r1 = min64(r0 + L, K);
@@ -375,31 +406,38 @@ k_scan_apply(int M, int K, int L, int n_chunks, const int32_t* __restrict__ dA,
 }
 
 // exact coarsening: counts add over q base windows, gauges are read at the
-// last base window of each coarse window
+// last base window of each coarse window (blockIdx.y = window length,
+// blockIdx.z = trace)
 __global__ void __launch_bounds__(kThreads)
-k_aggregate(int M, int Kq, int q, const int32_t* __restrict__ P, const int32_t* __restrict__ D,
-            const int32_t* __restrict__ A, const int32_t* __restrict__ W,
-            const unsigned long long* __restrict__ slo, int32_t* __restrict__ Pq,
-            int32_t* __restrict__ Dq, int32_t* __restrict__ Aq, int32_t* __restrict__ Wq,
-            unsigned long long* __restrict__ sloq) {
-  const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
-  if (t >= (int64_t)Kq * M) return;
-  const int m = (int)(t % M);
-  const int64_t k = t / M;
-  int32_t p = 0, d = 0;
-  unsigned long long s = 0;
-  for (int j = 0; j < q; ++j) {
-    const size_t x = (size_t)(k * q + j) * M + m;
-    p += P[x];
-    d += D[x];
-    if (slo) s += slo[x];
+k_aggregate(const __grid_constant__ AggPlan pl, const int32_t* __restrict__ P,
+            const int32_t* __restrict__ D, const int32_t* __restrict__ A,
+            const int32_t* __restrict__ W, const unsigned long long* __restrict__ slo,
+            int32_t* __restrict__ Pq, int32_t* __restrict__ Dq, int32_t* __restrict__ Aq,
+            int32_t* __restrict__ Wq, unsigned long long* __restrict__ sloq) {
+  const int w = blockIdx.y, tr = blockIdx.z;
+  const int M = pl.M, q = pl.q[w];
+  const int64_t n = (int64_t)pl.Kq[w] * M;
+  const size_t in0 = (size_t)tr * pl.Kb * M;
+  const size_t o0 = (size_t)pl.out_off[tr][w];
+  for (int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x; t < n;
+       t += (int64_t)gridDim.x * kThreads) {
+    const int m = (int)(t % M);
+    const int64_t k = t / M;
+    int32_t p = 0, d = 0;
+    unsigned long long sl = 0;
+    for (int j = 0; j < q; ++j) {
+      const size_t x = in0 + (size_t)(k * q + j) * M + m;
+      p += P[x];
+      d += D[x];
+      if (slo) sl += slo[x];
+    }
+    const size_t last = in0 + (size_t)(k * q + q - 1) * M + m;
+    Pq[o0 + t] = p;
+    Dq[o0 + t] = d;
+    Aq[o0 + t] = A[last];
+    Wq[o0 + t] = W[last];
+    if (sloq) sloq[o0 + t] = sl;
   }
-  const size_t last = (size_t)(k * q + q - 1) * M + m;
-  Pq[t] = p;
-  Dq[t] = d;
-  Aq[t] = A[last];
-  Wq[t] = W[last];
-  if (sloq) sloq[t] = s;
 }
 
 int num_sms() {
@@ -431,40 +469,55 @@ int scan_chunk_rows(int K) {
 
 }  // namespace
 
-void reduce_ws_layout(Arena& a, int M, int K, int64_t n_req, ReduceWs& w) {
-  const size_t cells = (size_t)(K + 1) * M;
+void reduce_ws_layout(Arena& a, int M, int K, int n_traces, int64_t n_req, ReduceWs& w) {
+  const size_t cells = (size_t)(K + 1) * M * n_traces;
+  w.n_traces = n_traces;
   w.dA = a.take<int32_t>(cells);
   w.dW = a.take<int32_t>(cells);
   w.first = n_req > 0 ? a.take<int32_t>((size_t)n_req) : nullptr;
   w.last = n_req > 0 ? a.take<int32_t>((size_t)n_req) : nullptr;
   const int L = scan_chunk_rows(K);
   const int n_chunks = (K + L - 1) / L;
-  w.partA = a.take<int32_t>((size_t)std::max(n_chunks, 1) * M);
-  w.partW = a.take<int32_t>((size_t)std::max(n_chunks, 1) * M);
+  w.partA = a.take<int32_t>((size_t)std::max(n_chunks, 1) * M * n_traces);
+  w.partW = a.take<int32_t>((size_t)std::max(n_chunks, 1) * M * n_traces);
 }
 
-cudaError_t launch_reduce_requests(const ReqCols& r, int M, int win, int K, int32_t* P,
-                                   int32_t* D, ReduceWs& w, unsigned long long* slo,
+cudaError_t launch_reduce_requests(const ReqCols* traces, int n_traces, int M, int win, int K,
+                                   int32_t* P, int32_t* D, ReduceWs& w, unsigned long long* slo,
                                    const int32_t* slo_ms, tre_diag* diag, cudaStream_t s) {
-  const size_t cells = (size_t)K * M;
+  if (n_traces < 1 || n_traces > kMaxTraces || n_traces > w.n_traces)
+    return cudaErrorInvalidValue;
+  const size_t cells = (size_t)K * M * n_traces;
   cudaError_t e;
   if ((e = cudaMemsetAsync(P, 0, cells * sizeof(int32_t), s))) return e;
   if ((e = cudaMemsetAsync(D, 0, cells * sizeof(int32_t), s))) return e;
-  if ((e = cudaMemsetAsync(w.dA, 0, (cells + M) * sizeof(int32_t), s))) return e;
-  if ((e = cudaMemsetAsync(w.dW, 0, (cells + M) * sizeof(int32_t), s))) return e;
+  if ((e = cudaMemsetAsync(w.dA, 0, (cells + (size_t)M * n_traces) * sizeof(int32_t), s))) return e;
+  if ((e = cudaMemsetAsync(w.dW, 0, (cells + (size_t)M * n_traces) * sizeof(int32_t), s))) return e;
   if (slo && (e = cudaMemsetAsync(slo, 0, cells * sizeof(unsigned long long), s))) return e;
-  if (r.n == 0) return cudaSuccess;
+  ReqBatch bt;
+  bt.n = n_traces;
+  int64_t total_n = 0;
+  for (int t = 0; t < n_traces; ++t) total_n += traces[t].n;
+  int ctas = 0;
+  for (int t = 0; t < n_traces; ++t) {
+    bt.cols[t] = traces[t];
+    // records per CTA sized on the whole batch so the grid fills the GPU
+    const int64_t per = per_cta_records(std::max<int64_t>(total_n / n_traces, 1), 1024, 8192);
+    bt.per_cta[t] = per;
+    bt.cta_base[t] = ctas;
+    ctas += (int)((traces[t].n + per - 1) / per);
+  }
+  bt.cta_base[n_traces] = ctas;
+  if (ctas == 0) return cudaSuccess;
   const int cell_bytes = 16 + (slo ? 8 : 0);
   const int rows = std::max(1, kStageBytes / (cell_bytes * M));
-  const int64_t per = per_cta_records(r.n, 1024, 8192);
-  const unsigned grid = (unsigned)((r.n + per - 1) / per);
   const size_t smem = (size_t)rows * M * cell_bytes;
   if (slo)
-    k_reduce_requests<true><<<grid, kThreads, smem, s>>>(r, M, win, K, per, rows, P, D, w.dA,
-                                                          w.dW, slo, slo_ms, diag);
+    k_reduce_requests<true><<<ctas, kThreads, smem, s>>>(bt, M, win, K, rows, P, D, w.dA, w.dW,
+                                                         slo, slo_ms, diag);
   else
-    k_reduce_requests<false><<<grid, kThreads, smem, s>>>(r, M, win, K, per, rows, P, D, w.dA,
-                                                           w.dW, nullptr, nullptr, diag);
+    k_reduce_requests<false><<<ctas, kThreads, smem, s>>>(bt, M, win, K, rows, P, D, w.dA, w.dW,
+                                                          nullptr, nullptr, diag);
   return cudaGetLastError();
 }
 
@@ -518,21 +571,22 @@ cudaError_t launch_gauge_scan(int M, int K, ReduceWs& w, int32_t* A, int32_t* W,
   const int L = scan_chunk_rows(K);
   const int n_chunks = (K + L - 1) / L;
   const int64_t segs = (int64_t)n_chunks * M;
-  const unsigned g = (unsigned)((segs + kThreads - 1) / kThreads);
+  dim3 g((unsigned)((segs + kThreads - 1) / kThreads), w.n_traces);
   k_scan_partials<<<g, kThreads, 0, s>>>(M, K, L, n_chunks, w.dA, w.dW, w.partA, w.partW);
-  k_scan_chunks<<<(M + 3) / 4, 128, 0, s>>>(M, n_chunks, w.partA, w.partW);
+  k_scan_chunks<<<dim3((M + 3) / 4, w.n_traces), 128, 0, s>>>(M, n_chunks, w.partA, w.partW);
   k_scan_apply<<<g, kThreads, 0, s>>>(M, K, L, n_chunks, w.dA, w.dW, w.partA, w.partW, A, W);
   return cudaGetLastError();
 }
 
-cudaError_t launch_aggregate(int M, int Kq, int q, const int32_t* P, const int32_t* D,
+cudaError_t launch_aggregate(const AggPlan& pl, const int32_t* P, const int32_t* D,
                              const int32_t* A, const int32_t* W, const unsigned long long* slo,
                              int32_t* Pq, int32_t* Dq, int32_t* Aq, int32_t* Wq,
                              unsigned long long* sloq, cudaStream_t s) {
-  const int64_t n = (int64_t)Kq * M;
-  if (n == 0) return cudaSuccess;
-  k_aggregate<<<(unsigned)((n + kThreads - 1) / kThreads), kThreads, 0, s>>>(
-      M, Kq, q, P, D, A, W, slo, Pq, Dq, Aq, Wq, sloq);
+  int64_t mx = 0;
+  for (int w = 0; w < pl.n_win; ++w) mx = std::max<int64_t>(mx, (int64_t)pl.Kq[w] * pl.M);
+  if (mx == 0) return cudaSuccess;
+  dim3 g(grid_for(mx), pl.n_win, pl.n_traces);
+  k_aggregate<<<g, kThreads, 0, s>>>(pl, P, D, A, W, slo, Pq, Dq, Aq, Wq, sloq);
   return cudaGetLastError();
 }
 

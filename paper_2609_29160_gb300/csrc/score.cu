@@ -1,8 +1,9 @@
 // Raw TSS (Eq. 1), exponential smoothing (Sec. III-B), Z = TSS / theta (Eq. 2),
-// regions, and the per-window Eq. 3 receiver.
+// regions, and the per-window Eq. 3 receiver -- for a batch of series at once.
 //
-// The smoothing S_k = alpha*raw_k + (1-alpha)*S_{k-1} is a sequential chain per
-// model. To spread it over the GPU and still return exactly the values of the
+// Eq. 1 is evaluated for every (window, model) in one fully parallel pass. The
+// smoothing S_k = alpha*raw_k + (1-alpha)*S_{k-1} is a sequential chain per
+// model; to spread it over the GPU and still return exactly the values of the
 // sequential definition (one rounding per operation, in order):
 //   1. each segment of windows computes its affine summary (approximate);
 //   2. a per-model scan of the summaries gives every segment an approximate
@@ -25,6 +26,7 @@ namespace tre {
 namespace {
 
 constexpr int kThreads = 256;
+constexpr int kBatch = 16;  // windows loaded ahead in the sequential chains
 
 template <class T> __device__ __forceinline__ T sub_rn(T a, T b);
 template <> __device__ __forceinline__ float sub_rn<float>(float a, float b) { return __fsub_rn(a, b); }
@@ -37,19 +39,27 @@ __device__ __forceinline__ bool same_bits(double a, double b) {
   return __double_as_longlong(a) == __double_as_longlong(b);
 }
 
+struct Counts {
+  const int32_t *P, *D, *A, *W;
+};
+
+// series of a global segment index (the table has at most 64 entries)
+template <class T> __device__ __forceinline__ int series_of_seg(const SeriesTable<T>& t, int seg) {
+  int s = 0;
+  while (s + 1 < t.n && t.seg_base[s + 1] <= seg) ++s;
+  return s;
+}
+
 template <class T> struct ModelParams {
-  T wp, wq, a, b, th, tc, ts;
+  T a, b, th, tc, ts;
 };
 
 template <class T>
-__device__ __forceinline__ ModelParams<T> load_params(const T* w_p, const T* w_q, const T* alpha,
-                                                      T alpha_v, const T* theta,
-                                                      const T* tau_crit, const T* tau_surp,
-                                                      int m) {
+__device__ __forceinline__ ModelParams<T> load_params(const SeriesTable<T>& t, int s, int m,
+                                                      const T* alpha, const T* theta,
+                                                      const T* tau_crit, const T* tau_surp) {
   ModelParams<T> p;
-  p.wp = w_p[m];
-  p.wq = w_q[m];
-  p.a = alpha ? alpha[m] : alpha_v;
+  p.a = alpha ? alpha[m] : t.alpha[s];
   p.b = sub_rn<T>((T)1, p.a);
   p.th = theta ? theta[m] : (T)1;
   p.tc = tau_crit ? tau_crit[m] : (T)0;
@@ -57,65 +67,74 @@ __device__ __forceinline__ ModelParams<T> load_params(const T* w_p, const T* w_q
   return p;
 }
 
-// Eq. 1 for one (window, model); returns false for an idle window
+// ---- pass 0: Eq. 1 for every (window, model); idle windows marked ---------
 template <class T>
-__device__ __forceinline__ bool raw_tss(int32_t p, int32_t d, int32_t a, int32_t w,
-                                        const ModelParams<T>& q, T dt, T& raw) {
-  if ((p | d | a | w) == 0) return false;
-  const T r_pre = div_rn(from_i32<T>(p), dt);
-  const T r_dec = div_rn(from_i32<T>(d), dt);
-  const T num = add_rn(mul_rn(q.wp, r_pre), r_dec);
-  T den = add_rn(from_i32<T>(a), mul_rn(q.wq, from_i32<T>(w)));
-  if (den < (T)1) den = (T)1;
-  raw = div_rn(num, den);
-  return true;
-}
-
-template <class T>
-__device__ __forceinline__ void ema_step(T& S, int& init, T raw, const ModelParams<T>& q) {
-  if (!init) {
-    S = raw;
-    init = 1;
-  } else {
-    S = add_rn(mul_rn(q.a, raw), mul_rn(q.b, S));
+__global__ void __launch_bounds__(kThreads)
+k_raw(const __grid_constant__ SeriesTable<T> tab, Counts c, const T* __restrict__ w_p,
+      const T* __restrict__ w_q, T* __restrict__ raw, uint8_t* __restrict__ cls) {
+  const int s = blockIdx.y;
+  const int M = tab.M;
+  const int64_t n = (int64_t)tab.K[s] * M;
+  const T dt = div_rn((T)tab.win[s], (T)1000);      // window length in seconds
+  for (int64_t i = (int64_t)blockIdx.x * kThreads + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * kThreads) {
+    const size_t x = (size_t)(tab.off[s] + i);
+    const int m = (int)(i % M);
+    const int32_t p = c.P[x], d = c.D[x], a = c.A[x], w = c.W[x];
+    if ((p | d | a | w) == 0) {
+      cls[x] = kIdle;
+      continue;
+    }
+    const T r_pre = div_rn(from_i32<T>(p), dt);
+    const T r_dec = div_rn(from_i32<T>(d), dt);
+    const T num = add_rn(mul_rn(w_p[m], r_pre), r_dec);
+    T den = add_rn(from_i32<T>(a), mul_rn(w_q[m], from_i32<T>(w)));
+    if (den < (T)1) den = (T)1;                       // demand floor of one request
+    raw[x] = div_rn(num, den);
+    cls[x] = kNom;
   }
 }
-
-template <class T>
-__device__ __forceinline__ uint8_t region(bool idle, T Z, const ModelParams<T>& q, bool classify) {
-  if (idle) return kIdle;
-  if (!classify) return kNom;
-  if (Z < q.tc) return kCrit;
-  if (Z > q.ts) return kSurp;
-  return kNom;
-}
-
-struct Counts {
-  const int32_t *P, *D, *A, *W;
-};
 
 // ---- pass 1: affine summary of each segment -------------------------------
 template <class T>
 __global__ void __launch_bounds__(kThreads)
-k_summary(int M, int K, int L, int n_seg, Counts c, const T* w_p, const T* w_q, const T* alpha,
-          T alpha_v, T dt, T* sm, T* sc, T* sci, int32_t* sh) {
+k_summary(const __grid_constant__ SeriesTable<T> tab, const T* __restrict__ raw,
+          const uint8_t* __restrict__ cls, const T* __restrict__ alpha, T* sm, T* sc, T* sci,
+          int32_t* sh) {
+  const int M = tab.M;
   const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
-  if (t >= (int64_t)n_seg * M) return;
+  if (t >= (int64_t)tab.seg_base[tab.n] * M) return;
   const int m = (int)(t % M);
-  const int s = (int)(t / M);
-  const ModelParams<T> q = load_params<T>(w_p, w_q, alpha, alpha_v, nullptr, nullptr, nullptr, m);
+  const int seg = (int)(t / M);
+  const int s = series_of_seg(tab, seg);
+  const int L = tab.seg_len[s];
+  const int64_t k0 = (int64_t)(seg - tab.seg_base[s]) * L, k1 = min64(k0 + L, tab.K[s]);
+  const T a = alpha ? alpha[m] : tab.alpha[s];
+  const T b = sub_rn<T>((T)1, a);
+  const size_t base = (size_t)tab.off[s] + m;
   T mm = (T)1, cc = (T)0, ci = (T)0;
   int h = 0;
-  const int64_t k0 = (int64_t)s * L, k1 = min64(k0 + L, K);
-  for (int64_t k = k0; k < k1; ++k) {
-    const size_t x = (size_t)k * M + m;
-    T raw;
-    if (!raw_tss<T>(c.P[x], c.D[x], c.A[x], c.W[x], q, dt, raw)) continue;
-    const T ar = q.a * raw;
-    ci = h ? ci * q.b + ar : raw;
-    cc = cc * q.b + ar;
-    mm = mm * q.b;
-    h = 1;
+  for (int64_t k = k0; k < k1; k += kBatch) {
+    T r[kBatch];
+    uint8_t c[kBatch];
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) {
+      c[j] = kIdle;
+      if (k + j < k1) {
+        const size_t x = base + (size_t)(k + j) * M;
+        c[j] = cls[x];
+        r[j] = raw[x];
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) {
+      if (c[j] == kIdle) continue;
+      const T ar = a * r[j];
+      ci = h ? ci * b + ar : r[j];
+      cc = cc * b + ar;
+      mm = mm * b;
+      h = 1;
+    }
   }
   sm[t] = mm;
   sc[t] = cc;
@@ -145,19 +164,23 @@ template <class T> __device__ __forceinline__ void apply(const Sum<T>& u, T& S, 
   init = 1;
 }
 
-// ---- pass 2: per-model exclusive scan of summaries -> approximate starts ----
+// ---- pass 2: per-(series, model) exclusive scan -> approximate starts ------
 template <class T>
-__global__ void k_starts(int M, int n_seg, const T* sm, const T* sc, const T* sci,
-                         const int32_t* sh, const T* S_carry, const uint8_t* init_carry,
-                         T* start_S, int32_t* start_init) {
-  const int m = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
-  if (m >= M) return;
+__global__ void k_starts(const __grid_constant__ SeriesTable<T> tab, const T* sm, const T* sc,
+                         const T* sci, const int32_t* sh, const T* S_carry,
+                         const uint8_t* init_carry, T* start_S, int32_t* start_init) {
+  const int M = tab.M;
+  const int w = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
+  if (w >= tab.n * M) return;
+  const int s = w / M, m = w % M;
   const int lane = threadIdx.x & 31;
+  const int n_seg = tab.seg_base[s + 1] - tab.seg_base[s];
   const int per = (n_seg + 31) / 32;
   const int s0 = lane * per, s1 = min(n_seg, s0 + per);
+  const size_t g0 = (size_t)tab.seg_base[s] * M + m;
   Sum<T> agg{(T)1, (T)0, (T)0, 0};
-  for (int s = s0; s < s1; ++s) {
-    const size_t x = (size_t)s * M + m;
+  for (int q = s0; q < s1; ++q) {
+    const size_t x = g0 + (size_t)q * M;
     agg = combine(agg, Sum<T>{sm[x], sc[x], sci[x], sh[x]});
   }
   Sum<T> inc = agg;
@@ -178,40 +201,60 @@ __global__ void k_starts(int M, int n_seg, const T* sm, const T* sc, const T* sc
   int init = (init_carry && init_carry[m]) ? 1 : 0;
   T S = init ? S_carry[m] : (T)0;
   apply(exc, S, init);
-  for (int s = s0; s < s1; ++s) {
-    const size_t x = (size_t)s * M + m;
+  for (int q = s0; q < s1; ++q) {
+    const size_t x = g0 + (size_t)q * M;
     start_S[x] = S;
     start_init[x] = init;
     apply(Sum<T>{sm[x], sc[x], sci[x], sh[x]}, S, init);
   }
 }
 
-// Run segment (s, m) exactly from (S, init) over windows [k0, k1), writing S,
-// Z and the region. With `verify`, stop at the first window whose new S equals
-// the stored one (same init state): from there the stored trajectory is the
-// one this start produces. Returns true if it stopped early.
+// Run windows [k0, k1) of model m exactly from (S, init), writing S and, with
+// `with_z`, Z and the region (idle windows keep their class). With `verify`,
+// stop at the first window whose new S equals the stored one with the same
+// init state: from there the stored trajectory is the one this start produces.
+// Returns true if it stopped early.
 template <class T>
-__device__ __forceinline__ bool run_segment(int M, int m, int64_t k0, int64_t k1, Counts c,
-                                            const ModelParams<T>& q, T dt, T& S, int& init,
-                                            bool verify, int stored_init, T* S_out, T* Z_out,
-                                            uint8_t* cls_out, bool with_z) {
-  for (int64_t k = k0; k < k1; ++k) {
-    const size_t x = (size_t)k * M + m;
-    T raw;
-    const bool active = raw_tss<T>(c.P[x], c.D[x], c.A[x], c.W[x], q, dt, raw);
-    if (active) {
-      ema_step<T>(S, init, raw, q);
-      stored_init = 1;
+__device__ __forceinline__ bool run_segment(size_t base, int M, int64_t k0, int64_t k1,
+                                            const T* __restrict__ raw, const ModelParams<T>& q,
+                                            T& S, int& init, bool verify, int stored_init,
+                                            T* S_out, T* Z_out, uint8_t* cls, bool with_z) {
+  for (int64_t k = k0; k < k1; k += kBatch) {
+    T r[kBatch], old[kBatch];
+    uint8_t c[kBatch];
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) {
+      c[j] = kIdle;
+      if (k + j < k1) {
+        const size_t x = base + (size_t)(k + j) * M;
+        c[j] = cls[x];
+        r[j] = raw[x];
+        if (verify) old[j] = S_out[x];
+      }
     }
-    if (verify && init == stored_init && same_bits(S, S_out[x])) return true;
-    const T Sv = init ? S : (T)0;
-    S_out[x] = Sv;
-    T Z = (T)0;
-    if (with_z) {
-      Z = div_rn(Sv, q.th);
-      Z_out[x] = Z;
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) {
+      if (k + j >= k1) break;
+      const bool active = c[j] != kIdle;
+      if (active) {
+        if (!init) {
+          S = r[j];
+          init = 1;
+        } else {
+          S = add_rn(mul_rn(q.a, r[j]), mul_rn(q.b, S));
+        }
+        stored_init = 1;
+      }
+      if (verify && init == stored_init && same_bits(S, old[j])) return true;
+      const size_t x = base + (size_t)(k + j) * M;
+      const T Sv = init ? S : (T)0;
+      S_out[x] = Sv;
+      if (with_z) {
+        const T Z = div_rn(Sv, q.th);
+        Z_out[x] = Z;
+        if (active) cls[x] = Z < q.tc ? kCrit : (Z > q.ts ? kSurp : kNom);
+      }
     }
-    cls_out[x] = region<T>(!active, Z, q, with_z);
   }
   return false;
 }
@@ -219,19 +262,21 @@ __device__ __forceinline__ bool run_segment(int M, int m, int64_t k0, int64_t k1
 // ---- pass 3: run every segment from its approximate start -------------------
 template <class T>
 __global__ void __launch_bounds__(kThreads)
-k_run(int M, int K, int L, int n_seg, Counts c, const T* w_p, const T* w_q, const T* alpha,
-      T alpha_v, const T* theta, const T* tau_crit, const T* tau_surp, T dt,
-      const T* start_S, const int32_t* start_init, T* end_S, int32_t* end_init, T* S_out,
-      T* Z_out, uint8_t* cls_out) {
+k_run(const __grid_constant__ SeriesTable<T> tab, const T* __restrict__ raw, const T* alpha,
+      const T* theta, const T* tau_crit, const T* tau_surp, const T* start_S,
+      const int32_t* start_init, T* end_S, int32_t* end_init, T* S_out, T* Z_out, uint8_t* cls) {
+  const int M = tab.M;
   const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
-  if (t >= (int64_t)n_seg * M) return;
+  if (t >= (int64_t)tab.seg_base[tab.n] * M) return;
   const int m = (int)(t % M);
-  const int s = (int)(t / M);
-  const ModelParams<T> q = load_params<T>(w_p, w_q, alpha, alpha_v, theta, tau_crit, tau_surp, m);
+  const int seg = (int)(t / M);
+  const int s = series_of_seg(tab, seg);
+  const ModelParams<T> q = load_params(tab, s, m, alpha, theta, tau_crit, tau_surp);
+  const int L = tab.seg_len[s];
+  const int64_t k0 = (int64_t)(seg - tab.seg_base[s]) * L, k1 = min64(k0 + L, tab.K[s]);
   T S = start_S[t];
   int init = start_init[t];
-  const int64_t k0 = (int64_t)s * L, k1 = min64(k0 + L, K);
-  run_segment<T>(M, m, k0, k1, c, q, dt, S, init, false, 0, S_out, Z_out, cls_out,
+  run_segment<T>((size_t)tab.off[s] + m, M, k0, k1, raw, q, S, init, false, 0, S_out, Z_out, cls,
                  theta != nullptr);
   end_S[t] = S;
   end_init[t] = init;
@@ -240,29 +285,31 @@ k_run(int M, int K, int L, int n_seg, Counts c, const T* w_p, const T* w_q, cons
 // ---- pass 4: parallel verification from the predecessor's computed end ------
 template <class T>
 __global__ void __launch_bounds__(kThreads)
-k_verify(int M, int K, int L, int n_seg, Counts c, const T* w_p, const T* w_q, const T* alpha,
-         T alpha_v, const T* theta, const T* tau_crit, const T* tau_surp, T dt, T* start_S,
-         int32_t* start_init, const T* end_S, const int32_t* end_init, T* end_S2,
-         int32_t* end_init2, T* S_out, T* Z_out, uint8_t* cls_out, tre_diag* diag) {
+k_verify(const __grid_constant__ SeriesTable<T> tab, const T* __restrict__ raw, const T* alpha,
+         const T* theta, const T* tau_crit, const T* tau_surp, T* start_S, int32_t* start_init,
+         const T* end_S, const int32_t* end_init, T* end_S2, int32_t* end_init2, T* S_out,
+         T* Z_out, uint8_t* cls, tre_diag* diag) {
+  const int M = tab.M;
   const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
-  if (t >= (int64_t)n_seg * M) return;
+  if (t >= (int64_t)tab.seg_base[tab.n] * M) return;
   const int m = (int)(t % M);
-  const int s = (int)(t / M);
+  const int seg = (int)(t / M);
+  const int s = series_of_seg(tab, seg);
   T eS = end_S[t];
   int eI = end_init[t];
-  if (s > 0) {
+  if (seg > tab.seg_base[s]) {
     const size_t p = t - M;
     T S = end_S[p];
     int init = end_init[p];
     if (init != start_init[t] || !same_bits(S, start_S[t])) {
-      const ModelParams<T> q =
-          load_params<T>(w_p, w_q, alpha, alpha_v, theta, tau_crit, tau_surp, m);
-      const int64_t k0 = (int64_t)s * L, k1 = min64(k0 + L, K);
+      const ModelParams<T> q = load_params(tab, s, m, alpha, theta, tau_crit, tau_surp);
+      const int L = tab.seg_len[s];
+      const int64_t k0 = (int64_t)(seg - tab.seg_base[s]) * L, k1 = min64(k0 + L, tab.K[s]);
       const int stored_init = start_init[t];
       start_S[t] = S;
       start_init[t] = init;
-      const bool met = run_segment<T>(M, m, k0, k1, c, q, dt, S, init, true, stored_init, S_out,
-                                      Z_out, cls_out, theta != nullptr);
+      const bool met = run_segment<T>((size_t)tab.off[s] + m, M, k0, k1, raw, q, S, init, true,
+                                      stored_init, S_out, Z_out, cls, theta != nullptr);
       if (!met) {
         eS = S;
         eI = init;
@@ -274,57 +321,85 @@ k_verify(int M, int K, int L, int n_seg, Counts c, const T* w_p, const T* w_q, c
   end_init2[t] = eI;
 }
 
-// ---- pass 5: in-order repair, one thread per model ---------------------------
+// ---- pass 5: in-order repair, one thread per (series, model) ---------------
 template <class T>
-__global__ void k_resolve(int M, int K, int L, int n_seg, Counts c, const T* w_p, const T* w_q,
-                          const T* alpha, T alpha_v, const T* theta, const T* tau_crit,
-                          const T* tau_surp, T dt, const T* start_S, const int32_t* start_init,
-                          const T* end_S, const int32_t* end_init, T* S_out, T* Z_out,
-                          uint8_t* cls_out, T* S_carry, uint8_t* init_carry, tre_diag* diag) {
-  const int m = blockIdx.x * blockDim.x + threadIdx.x;
-  if (m >= M) return;
-  const ModelParams<T> q = load_params<T>(w_p, w_q, alpha, alpha_v, theta, tau_crit, tau_surp, m);
-  T S = end_S[m];
-  int init = end_init[m];
-  for (int s = 1; s < n_seg; ++s) {
-    const size_t x = (size_t)s * M + m;
-    if (init == start_init[x] && same_bits(S, start_S[x])) {
-      S = end_S[x];
-      init = end_init[x];
-      continue;
+__global__ void k_resolve(const __grid_constant__ SeriesTable<T> tab, const T* __restrict__ raw,
+                          const T* alpha, const T* theta, const T* tau_crit, const T* tau_surp,
+                          const T* start_S, const int32_t* start_init, const T* end_S,
+                          const int32_t* end_init, T* S_out, T* Z_out, uint8_t* cls,
+                          T* S_carry, uint8_t* init_carry, tre_diag* diag) {
+  const int M = tab.M;
+  const int w = blockIdx.x * blockDim.x + threadIdx.x;
+  if (w >= tab.n * M) return;
+  const int s = w / M, m = w % M;
+  const int n_seg = tab.seg_base[s + 1] - tab.seg_base[s];
+  if (n_seg == 0) return;
+  const ModelParams<T> q = load_params(tab, s, m, alpha, theta, tau_crit, tau_surp);
+  const int L = tab.seg_len[s];
+  const size_t g0 = (size_t)tab.seg_base[s] * M + m;
+  T S = end_S[g0];
+  int init = end_init[g0];
+  for (int q0 = 1; q0 < n_seg; q0 += kBatch) {
+    // load the boundary states of a batch of segments ahead of the checks
+    T bS[kBatch], bE[kBatch];
+    int bI[kBatch], bEI[kBatch];
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) {
+      if (q0 + j < n_seg) {
+        const size_t x = g0 + (size_t)(q0 + j) * M;
+        bS[j] = start_S[x];
+        bI[j] = start_init[x];
+        bE[j] = end_S[x];
+        bEI[j] = end_init[x];
+      }
     }
-    const int64_t k0 = (int64_t)s * L, k1 = min64(k0 + L, K);
-    const bool met = run_segment<T>(M, m, k0, k1, c, q, dt, S, init, true, start_init[x], S_out,
-                                    Z_out, cls_out, theta != nullptr);
-    if (met) {
-      S = end_S[x];
-      init = end_init[x];
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) {
+      const int qq = q0 + j;
+      if (qq >= n_seg) break;
+      if (init == bI[j] && same_bits(S, bS[j])) {
+        S = bE[j];
+        init = bEI[j];
+        continue;
+      }
+      const int64_t k0 = (int64_t)qq * L, k1 = min64(k0 + L, tab.K[s]);
+      const bool met = run_segment<T>((size_t)tab.off[s] + m, M, k0, k1, raw, q, S, init, true,
+                                      bI[j], S_out, Z_out, cls, theta != nullptr);
+      if (met) {
+        S = bE[j];
+        init = bEI[j];
+      }
+      atomicAdd(&diag->ema_resolved, 1ull);
     }
-    atomicAdd(&diag->ema_resolved, 1ull);
   }
-  if (S_carry && n_seg > 0) {
+  if (S_carry) {
     S_carry[m] = S;
     init_carry[m] = (uint8_t)init;
   }
 }
 
-// ---- Z and regions from S (one threshold for every model optional) ---------
+// ---- Z and regions from S for every series ---------------------------------
 template <class T>
 __global__ void __launch_bounds__(kThreads)
-k_normalize(int M, int64_t n, const T* S, const uint8_t* idle_cls, const T* theta,
-            const T* tau_crit, T tau_crit_v, const T* tau_surp, T* Z, uint8_t* cls) {
-  for (int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x; t < n;
-       t += (int64_t)gridDim.x * kThreads) {
-    const int m = (int)(t % M);
-    const T z = div_rn(S[t], theta[m]);
-    if (Z) Z[t] = z;
+k_normalize(const __grid_constant__ SeriesTable<T> tab, const T* S, const uint8_t* idle_cls,
+            const T* theta, const T* tau_crit, T tau_crit_v, const T* tau_surp, T* Z,
+            uint8_t* cls) {
+  const int s = blockIdx.y;
+  const int M = tab.M;
+  const int64_t n = (int64_t)tab.K[s] * M;
+  for (int64_t i = (int64_t)blockIdx.x * kThreads + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * kThreads) {
+    const size_t x = (size_t)(tab.off[s] + i);
+    const int m = (int)(i % M);
+    const T z = div_rn(S[x], theta[(size_t)s * M + m]);
+    if (Z) Z[x] = z;
     if (cls) {
       uint8_t c;
-      if (idle_cls[t] == kIdle) c = kIdle;
+      if (idle_cls[x] == kIdle) c = kIdle;
       else if (z < (tau_crit ? tau_crit[m] : tau_crit_v)) c = kCrit;
       else if (z > tau_surp[m]) c = kSurp;
       else c = kNom;
-      cls[t] = c;
+      cls[x] = c;
     }
   }
 }
@@ -351,49 +426,43 @@ __global__ void k_receiver(int M, int K, const T* Z, const uint8_t* cls, int32_t
   if (lane == 0) recv[k] = best;
 }
 
-int seg_len_for(int K) {
-  const int L = (K + 1023) / 1024;
-  return L < 256 ? 256 : L;
+template <class T> int64_t max_elems(const SeriesTable<T>& t) {
+  int64_t mx = 0;
+  for (int s = 0; s < t.n; ++s) mx = std::max<int64_t>(mx, (int64_t)t.K[s] * t.M);
+  return mx;
 }
 
-template <class T>
-cudaError_t score_impl(int M, int win, int K, const int32_t* P, const int32_t* D, const int32_t* A,
-                       const int32_t* W, const T* w_p, const T* w_q, const T* alpha, T alpha_v,
-                       const T* theta, const T* tau_crit, const T* tau_surp, T* S_carry,
-                       uint8_t* init_carry, T* S, T* Z, uint8_t* cls, ScoreWs<T>& w,
-                       tre_diag* diag, cudaStream_t s) {
-  if (K == 0) return cudaSuccess;
-  const T dt = (T)win / (T)1000;
-  // segmenting of this call; never more segments than the workspace was laid
-  // out for (the count grows with K)
-  const int L = seg_len_for(K), n = (K + L - 1) / L;
-  if (n > w.n_seg) return cudaErrorInvalidValue;
-  const int64_t segs = (int64_t)n * M;
-  const unsigned g = (unsigned)((segs + kThreads - 1) / kThreads);
-  const Counts c{P, D, A, W};
-  k_summary<T><<<g, kThreads, 0, s>>>(M, K, L, n, c, w_p, w_q, alpha, alpha_v, dt, w.sum_m,
-                                      w.sum_c, w.sum_ci, w.sum_h);
-  k_starts<T><<<(M + 3) / 4, 128, 0, s>>>(M, n, w.sum_m, w.sum_c, w.sum_ci, w.sum_h, S_carry,
-                                          init_carry, w.start_S, w.start_init);
-  k_run<T><<<g, kThreads, 0, s>>>(M, K, L, n, c, w_p, w_q, alpha, alpha_v, theta, tau_crit,
-                                  tau_surp, dt, w.start_S, w.start_init, w.end_S, w.end_init, S,
-                                  Z, cls);
-  k_verify<T><<<g, kThreads, 0, s>>>(M, K, L, n, c, w_p, w_q, alpha, alpha_v, theta, tau_crit,
-                                     tau_surp, dt, w.start_S, w.start_init, w.end_S, w.end_init,
-                                     w.end_S2, w.end_init2, S, Z, cls, diag);
-  k_resolve<T><<<(M + 63) / 64, 64, 0, s>>>(M, K, L, n, c, w_p, w_q, alpha, alpha_v, theta,
-                                            tau_crit, tau_surp, dt, w.start_S, w.start_init,
-                                            w.end_S2, w.end_init2, S, Z, cls, S_carry,
-                                            init_carry, diag);
-  return cudaGetLastError();
+unsigned blocks_for(int64_t n, int cap) {
+  int64_t b = (n + kThreads - 1) / kThreads;
+  return (unsigned)std::max<int64_t>(1, std::min<int64_t>(b, cap));
 }
 
 }  // namespace
 
-template <class T> void score_ws_layout(Arena& a, int M, int K, ScoreWs<T>& w) {
-  w.seg_len = seg_len_for(K);
-  w.n_seg = (K + w.seg_len - 1) / w.seg_len;
-  const size_t n = (size_t)std::max(w.n_seg, 1) * M;
+template <class T> int series_segments(SeriesTable<T>& t) {
+  int total = 0;
+  for (int s = 0; s < t.n; ++s) {
+    const int K = t.K[s];
+    // Two trajectories of the smoothing that start a few dozen ulps apart meet
+    // after about 4 / alpha windows; segments about twice that long let the
+    // verification pass meet the stored trajectory inside one segment.
+    const double a = (double)t.alpha[s];
+    int base = 64;
+    while (base < 512 && !(a > 0 && (double)base * a >= 8.0)) base *= 2;
+    int L = (K + 1023) / 1024;
+    L = L < base ? base : L;
+    t.seg_len[s] = L;
+    t.seg_base[s] = total;
+    total += (K + L - 1) / L;
+  }
+  t.seg_base[t.n] = total;
+  return total;
+}
+
+template <class T> void score_ws_layout(Arena& a, int M, int64_t elems, int n_seg, ScoreWs<T>& w) {
+  w.raw = a.take<T>((size_t)std::max<int64_t>(elems, 1));
+  w.cap_seg = std::max(n_seg, 1);
+  const size_t n = (size_t)w.cap_seg * M;
   w.sum_m = a.take<T>(n);
   w.sum_c = a.take<T>(n);
   w.sum_ci = a.take<T>(n);
@@ -407,34 +476,45 @@ template <class T> void score_ws_layout(Arena& a, int M, int K, ScoreWs<T>& w) {
 }
 
 template <class T>
-cudaError_t launch_score(int M, int win, int K, const int32_t* P, const int32_t* D,
+cudaError_t launch_score(const SeriesTable<T>& tab, const int32_t* P, const int32_t* D,
                          const int32_t* A, const int32_t* W, const T* w_p, const T* w_q,
                          const T* alpha, const T* theta, const T* tau_crit, const T* tau_surp,
                          T* S_carry, uint8_t* init_carry, T* S, T* Z, uint8_t* cls,
                          ScoreWs<T>& w, tre_diag* diag, cudaStream_t s) {
-  return score_impl<T>(M, win, K, P, D, A, W, w_p, w_q, alpha, (T)0, theta, tau_crit, tau_surp,
-                       S_carry, init_carry, S, Z, cls, w, diag, s);
+  const int M = tab.M;
+  const int n_seg = tab.seg_base[tab.n];
+  if (n_seg > w.cap_seg) return cudaErrorInvalidValue;
+  const int64_t mx = max_elems(tab);
+  if (mx == 0) return cudaSuccess;
+  const Counts c{P, D, A, W};
+  dim3 ge(blocks_for(mx, 2048), tab.n);
+  k_raw<T><<<ge, kThreads, 0, s>>>(tab, c, w_p, w_q, w.raw, cls);
+  const int64_t segs = (int64_t)n_seg * M;
+  const unsigned g = (unsigned)((segs + kThreads - 1) / kThreads);
+  k_summary<T><<<g, kThreads, 0, s>>>(tab, w.raw, cls, alpha, w.sum_m, w.sum_c, w.sum_ci, w.sum_h);
+  const int warps = tab.n * M;
+  k_starts<T><<<(warps + 3) / 4, 128, 0, s>>>(tab, w.sum_m, w.sum_c, w.sum_ci, w.sum_h, S_carry,
+                                              init_carry, w.start_S, w.start_init);
+  k_run<T><<<g, kThreads, 0, s>>>(tab, w.raw, alpha, theta, tau_crit, tau_surp, w.start_S,
+                                  w.start_init, w.end_S, w.end_init, S, Z, cls);
+  k_verify<T><<<g, kThreads, 0, s>>>(tab, w.raw, alpha, theta, tau_crit, tau_surp, w.start_S,
+                                     w.start_init, w.end_S, w.end_init, w.end_S2, w.end_init2, S,
+                                     Z, cls, diag);
+  k_resolve<T><<<(warps + 63) / 64, 64, 0, s>>>(tab, w.raw, alpha, theta, tau_crit, tau_surp,
+                                                w.start_S, w.start_init, w.end_S2, w.end_init2,
+                                                S, Z, cls, S_carry, init_carry, diag);
+  return cudaGetLastError();
 }
 
 template <class T>
-cudaError_t launch_score_alpha(int M, int win, int K, const int32_t* P, const int32_t* D,
-                               const int32_t* A, const int32_t* W, const T* w_p, const T* w_q,
-                               T alpha, T* S, uint8_t* cls, ScoreWs<T>& w, tre_diag* diag,
-                               cudaStream_t s) {
-  return score_impl<T>(M, win, K, P, D, A, W, w_p, w_q, nullptr, alpha, nullptr, nullptr, nullptr,
-                       nullptr, nullptr, S, nullptr, cls, w, diag, s);
-}
-
-template <class T>
-cudaError_t launch_normalize(int M, int K, const T* S, const uint8_t* idle_cls, const T* theta,
-                             const T* tau_crit, T tau_crit_v, const T* tau_surp, T* Z,
-                             uint8_t* cls, cudaStream_t s) {
-  const int64_t n = (int64_t)K * M;
-  if (n == 0) return cudaSuccess;
-  int64_t b = (n + kThreads - 1) / kThreads;
-  if (b > 152 * 32) b = 152 * 32;
-  k_normalize<T><<<(unsigned)b, kThreads, 0, s>>>(M, n, S, idle_cls, theta, tau_crit, tau_crit_v,
-                                                  tau_surp, Z, cls);
+cudaError_t launch_normalize(const SeriesTable<T>& tab, const T* S, const uint8_t* idle_cls,
+                             const T* theta, const T* tau_crit, T tau_crit_v, const T* tau_surp,
+                             T* Z, uint8_t* cls, cudaStream_t s) {
+  const int64_t mx = max_elems(tab);
+  if (mx == 0) return cudaSuccess;
+  dim3 g(blocks_for(mx, 1024), tab.n);
+  k_normalize<T><<<g, kThreads, 0, s>>>(tab, S, idle_cls, theta, tau_crit, tau_crit_v, tau_surp,
+                                        Z, cls);
   return cudaGetLastError();
 }
 
@@ -447,17 +527,15 @@ cudaError_t launch_receiver(int M, int K, const T* Z, const uint8_t* cls, int32_
 }
 
 #define TRE_INST(T)                                                                               \
-  template void score_ws_layout<T>(Arena&, int, int, ScoreWs<T>&);                                \
-  template cudaError_t launch_score<T>(int, int, int, const int32_t*, const int32_t*,              \
+  template int series_segments<T>(SeriesTable<T>&);                                               \
+  template void score_ws_layout<T>(Arena&, int, int64_t, int, ScoreWs<T>&);                       \
+  template cudaError_t launch_score<T>(const SeriesTable<T>&, const int32_t*, const int32_t*,      \
                                        const int32_t*, const int32_t*, const T*, const T*,         \
                                        const T*, const T*, const T*, const T*, T*, uint8_t*, T*,   \
                                        T*, uint8_t*, ScoreWs<T>&, tre_diag*, cudaStream_t);        \
-  template cudaError_t launch_score_alpha<T>(int, int, int, const int32_t*, const int32_t*,        \
-                                             const int32_t*, const int32_t*, const T*, const T*,   \
-                                             T, T*, uint8_t*, ScoreWs<T>&, tre_diag*,              \
-                                             cudaStream_t);                                        \
-  template cudaError_t launch_normalize<T>(int, int, const T*, const uint8_t*, const T*,           \
-                                           const T*, T, const T*, T*, uint8_t*, cudaStream_t);     \
+  template cudaError_t launch_normalize<T>(const SeriesTable<T>&, const T*, const uint8_t*,        \
+                                           const T*, const T*, T, const T*, T*, uint8_t*,          \
+                                           cudaStream_t);                                          \
   template cudaError_t launch_receiver<T>(int, int, const T*, const uint8_t*, int32_t*,            \
                                           cudaStream_t);
 TRE_INST(float)

@@ -1,11 +1,19 @@
 // Open-loop TRE move selection (Sec. IV-B dual-speed control, Eq. 3 receiver,
 // Sec. IV-C bounded pairwise transfer under a fixed budget).
 //
-// One warp runs one controller instance serially over its control ticks; the
-// models are spread over the lanes (models m = lane + 32*j, j < MPL) with their
-// replica counts in registers. Receiver and donor choices are warp arg-min /
-// arg-max reductions with the lowest model index winning ties. Only the windows
-// that end a fast or slow tick are visited.
+// Everything that does not depend on the replica state is computed first, in
+// parallel, for every (series, rescue threshold, control tick):
+//   - at each fast tick: whether any model is critical, the rescue receiver
+//     (lowest Z among critical models, lowest index on ties) and every model's
+//     rank in the rescue donor order;
+//   - at each slow tick: the Eq. 3 receiver over non-idle models, whether its
+//     Z is below 1, and every model's rank in the rebalance donor order.
+// Donor order: idle models by index, then surplus by Z descending, then
+// nominal by Z descending (in rebalance only those above the receiver's Z);
+// critical models and the receiver get no rank.
+// The serial part -- one warp per controller instance walking its ticks with
+// the replica counts in registers (models m = lane + 32*j) -- then only picks,
+// per released replica, the lowest-ranked model still above its floor.
 #include <algorithm>
 
 #include "common.cuh"
@@ -15,37 +23,118 @@ namespace tre {
 namespace {
 
 constexpr int kWarpsPerBlock = 4;
+constexpr uint16_t kNoRank = 0xffff;
 
-// candidate ordering: smaller `grp` first, then larger `z` (when by_z),
-// then smaller index
-template <class T> struct Cand {
-  int grp;   // INT_MAX = none
-  T z;
-  int m;
-};
-
-template <class T> __device__ __forceinline__ bool better(const Cand<T>& a, const Cand<T>& b,
-                                                          bool hi_z) {
-  if (a.grp != b.grp) return a.grp < b.grp;
-  if (a.grp == 0x7fffffff) return false;
-  if (a.z != b.z) return hi_z ? (a.z > b.z) : (a.z < b.z);
-  return a.m < b.m;
+__device__ __forceinline__ int64_t tick_window(int64_t j, int64_t cadence, int64_t win) {
+  // window whose right edge passes the j-th multiple of the cadence (j >= 1)
+  return (j * cadence + win - 1) / win - 1;
 }
 
-template <class T> __device__ __forceinline__ Cand<T> warp_best(Cand<T> c, bool hi_z) {
-  for (int o = 16; o > 0; o >>= 1) {
-    Cand<T> x;
-    x.grp = __shfl_xor_sync(0xffffffffu, c.grp, o);
-    x.z = __shfl_xor_sync(0xffffffffu, c.z, o);
-    x.m = __shfl_xor_sync(0xffffffffu, c.m, o);
-    if (better(x, c, hi_z)) c = x;
+template <class T>
+__device__ __forceinline__ uint8_t region_of(uint8_t c, T z, T tc, T ts) {
+  if (c == kIdle) return kIdle;
+  if (z < tc) return kCrit;
+  if (z > ts) return kSurp;
+  return kNom;
+}
+
+// One thread per (series, tau, tick entry, model). Entries [0, nf) of a series
+// are its fast ticks, [nf, nf + ns) its slow ticks.
+template <class T>
+__global__ void __launch_bounds__(256)
+k_tick_rank(const __grid_constant__ WalkBatch<T> b, int16_t* recv_out, uint16_t* rank) {
+  const int M = b.M;
+  const int64_t gid = (int64_t)blockIdx.x * 256 + threadIdx.x;
+  const int64_t total_ent = (int64_t)b.ent_base[b.n_series] * b.n_tau;
+  if (gid >= total_ent * M) return;
+  const int m = (int)(gid % M);
+  const int64_t e = gid / M;                       // entry over (series, tau, tick)
+  int s = 0;
+  while (s + 1 < b.n_series && (int64_t)b.ent_base[s + 1] * b.n_tau <= e) ++s;
+  const int64_t local = e - (int64_t)b.ent_base[s] * b.n_tau;
+  const int n_ent = b.ent_base[s + 1] - b.ent_base[s];
+  const int ti = (int)(local / n_ent);
+  const int j = (int)(local % n_ent);
+  const int64_t win = b.series_win[s];
+  const int64_t K = b.series_K[s];
+  const int64_t nf = K * win / b.fast_ms;
+  const bool fast = j < nf;
+  const int64_t k =
+      fast ? tick_window(j + 1, b.fast_ms, win) : tick_window(j - nf + 1, b.slow_ms, win);
+  const T* Zk = b.Z + b.series_off[s] + (size_t)k * M;
+  const uint8_t* Ck = b.cls + b.series_off[s] + (size_t)k * M;
+  const bool tau_dev = b.tau_crit != nullptr;
+  const T tau_v = b.tau_list[tau_dev ? 0 : ti];
+  auto reg = [&](int q) {
+    return region_of(Ck[q], Zk[q], tau_dev ? b.tau_crit[q] : tau_v, b.tau_surp[q]);
+  };
+  // receiver: rescue -> lowest Z among critical; rebalance -> lowest Z among non-idle
+  int recv = -1;
+  T zr = (T)0;
+  for (int q = 0; q < M; ++q) {
+    const uint8_t rg = reg(q);
+    const bool cand = fast ? rg == kCrit : rg != kIdle;
+    if (cand && (recv < 0 || Zk[q] < zr)) {
+      recv = q;
+      zr = Zk[q];
+    }
   }
-  return c;
+  const bool act = recv >= 0 && (fast || zr < (T)1);
+  // donor group of model q, -1 = not a donor at this tick
+  auto group = [&](int q, uint8_t rg) -> int {
+    if (q == recv || rg == kCrit) return -1;
+    if (rg == kIdle) return 0;
+    if (rg == kSurp) return 1;
+    if (!fast && !(Zk[q] > zr)) return -1;       // rebalance: nominal donors above the receiver
+    return 2;
+  };
+  const int gm = act ? group(m, reg(m)) : -1;
+  uint16_t r = kNoRank;
+  if (gm >= 0) {
+    const T zm = Zk[m];
+    int before = 0;
+    for (int q = 0; q < M; ++q) {
+      if (q == m) continue;
+      const int gq = group(q, reg(q));
+      if (gq < 0) continue;
+      bool prec;
+      if (gq != gm) prec = gq < gm;
+      else if (gq == 0) prec = q < m;
+      else prec = Zk[q] > zm || (Zk[q] == zm && q < m);
+      before += prec;
+    }
+    r = (uint16_t)before;
+  }
+  const size_t row = (size_t)b.ent_base[s] * b.n_tau + (size_t)ti * n_ent + j;
+  rank[row * M + m] = r;
+  if (m == 0) recv_out[row] = (int16_t)(act ? recv : -1);
+}
+
+template <int MPL>
+__device__ __forceinline__ int lane_of_min_rank(const uint16_t (&rk)[MPL], const int (&r)[MPL],
+                                                const int (&rmin)[MPL], int lane, int M,
+                                                int& model) {
+  uint32_t best = 0xffffffffu;
+  int bj = 0;
+#pragma unroll
+  for (int j = 0; j < MPL; ++j) {
+    const bool ok = lane + 32 * j < M && rk[j] != kNoRank && r[j] > rmin[j];
+    if (ok && rk[j] < best) {
+      best = rk[j];
+      bj = j;
+    }
+  }
+  const uint32_t wmin = __reduce_min_sync(0xffffffffu, best);
+  if (wmin == 0xffffffffu) return -1;
+  const unsigned who = __ballot_sync(0xffffffffu, best == wmin);
+  const int src = __ffs(who) - 1;            // ranks are distinct within a tick
+  model = src + 32 * __shfl_sync(0xffffffffu, bj, src);
+  return src;
 }
 
 template <class T, int MPL>
 __global__ void __launch_bounds__(kWarpsPerBlock * 32)
-k_walk(const __grid_constant__ WalkBatch<T> b) {
+k_walk(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab, const uint16_t* rank) {
   const int inst = blockIdx.x * kWarpsPerBlock + threadIdx.x / 32;
   if (inst >= b.n_inst) return;
   const int lane = threadIdx.x & 31;
@@ -53,19 +142,21 @@ k_walk(const __grid_constant__ WalkBatch<T> b) {
   const int ci = inst % b.n_cap;
   const int ti = (inst / b.n_cap) % b.n_tau;
   const int si = inst / (b.n_cap * b.n_tau);
-  const int64_t off = b.series_off[si];
   const int K = b.series_K[si];
   const int64_t win = b.series_win[si];
-  const T* Zs = b.Z + off;
-  const uint8_t* Cs = b.cls + off;
   const int Kp = b.cap_list[ci];
-  const T tau_v = b.tau_crit ? (T)0 : b.tau_list[ti];
   const int64_t cap = b.moves_cap;
   tre_move* mv = b.moves + (size_t)inst * cap;
+  const int n_ent = b.ent_base[si + 1] - b.ent_base[si];
+  const size_t row0 = (size_t)b.ent_base[si] * b.n_tau + (size_t)ti * n_ent;
+  const int16_t* rv_tab = recv_tab + row0;
+  const uint16_t* rk0 = rank + row0 * M;
+  const int64_t F = b.fast_ms, Sl = b.slow_ms;
+  const int64_t nf = (int64_t)K * win / F;
 
   int r[MPL], rmin[MPL], g[MPL];
-  T tc[MPL], ts[MPL];
   int64_t used = 0;
+  bool bad = false;
 #pragma unroll
   for (int j = 0; j < MPL; ++j) {
     const int m = lane + 32 * j;
@@ -73,20 +164,14 @@ k_walk(const __grid_constant__ WalkBatch<T> b) {
       r[j] = b.r0[m];
       rmin[j] = b.r_min[m];
       g[j] = b.footprint[m];
-      tc[j] = b.tau_crit ? b.tau_crit[m] : tau_v;
-      ts[j] = b.tau_surp[m];
       used += (int64_t)g[j] * r[j];
+      if (r[j] < 0 || g[j] < 1 || rmin[j] < 0) bad = true;
     } else {
-      r[j] = 0; rmin[j] = 0; g[j] = 0; tc[j] = (T)0; ts[j] = (T)0;
+      r[j] = 0; rmin[j] = 0; g[j] = 0;
     }
   }
   for (int o = 16; o > 0; o >>= 1) used += __shfl_xor_sync(0xffffffffu, used, o);
   int64_t free_pool = b.budget - used;
-  int64_t nm = 0;
-  bool bad = false;
-#pragma unroll
-  for (int j = 0; j < MPL; ++j)
-    if (lane + 32 * j < M && (r[j] < 0 || g[j] < 1 || rmin[j] < 0)) bad = true;
   // an inconsistent controller state (negative replicas or floors, footprint
   // below one, replicas beyond the budget) produces no moves
   if (__any_sync(0xffffffffu, bad) || free_pool < 0) {
@@ -99,65 +184,32 @@ k_walk(const __grid_constant__ WalkBatch<T> b) {
     }
     return;
   }
-
-  const int64_t F = b.fast_ms, Sl = b.slow_ms;
+  int64_t nm = 0;
   int64_t jf = 1, js = 1;
   while (true) {
-    // next window that ends a fast / slow tick: smallest k with (k+1)*win >= j*cadence
-    const int64_t kf = (jf * F + win - 1) / win - 1;
-    const int64_t ks = (js * Sl + win - 1) / win - 1;
+    const int64_t kf = tick_window(jf, F, win);
+    const int64_t ks = tick_window(js, Sl, win);
     const int64_t k = kf < ks ? kf : ks;
     if (k >= K) break;
     const bool fast = kf == k, slow = ks == k;
-    while ((jf * F + win - 1) / win - 1 <= k) ++jf;
-    while ((js * Sl + win - 1) / win - 1 <= k) ++js;
-
-    T z[MPL];
-    uint8_t reg[MPL];
-#pragma unroll
-    for (int j = 0; j < MPL; ++j) {
-      const int m = lane + 32 * j;
-      if (m < M) {
-        const size_t x = (size_t)k * M + m;
-        z[j] = Zs[x];
-        if (Cs[x] == kIdle) reg[j] = kIdle;
-        else if (z[j] < tc[j]) reg[j] = kCrit;
-        else if (z[j] > ts[j]) reg[j] = kSurp;
-        else reg[j] = kNom;
-      } else {
-        z[j] = (T)0;
-        reg[j] = 0xff;
-      }
-    }
-    int kind = 0;
-    Cand<T> rc{0x7fffffff, (T)0, 0};
+    const int64_t ef = jf - 1, es = nf + js - 1;   // entries of this tick
+    while (tick_window(jf, F, win) <= k) ++jf;
+    while (tick_window(js, Sl, win) <= k) ++js;
+    int recv = -1, kind = 0;
+    int64_t ent = -1;
     if (fast) {
-#pragma unroll
-      for (int j = 0; j < MPL; ++j) {
-        const Cand<T> c{reg[j] == kCrit ? 0 : 0x7fffffff, z[j], lane + 32 * j};
-        if (better(c, rc, false)) rc = c;
-      }
-      rc = warp_best(rc, false);
-      if (rc.grp == 0) kind = TRE_RESCUE;
+      const int rv = rv_tab[ef];
+      if (rv >= 0) { recv = rv; ent = ef; kind = TRE_RESCUE; }
     }
-    bool nom_above = false;
     if (!kind && slow) {
-      rc = Cand<T>{0x7fffffff, (T)0, 0};
-#pragma unroll
-      for (int j = 0; j < MPL; ++j) {
-        const bool ok = reg[j] != kIdle && reg[j] != 0xff;
-        const Cand<T> c{ok ? 0 : 0x7fffffff, z[j], lane + 32 * j};
-        if (better(c, rc, false)) rc = c;
-      }
-      rc = warp_best(rc, false);
-      if (rc.grp == 0 && rc.z < (T)1) {
-        kind = TRE_REBALANCE;
-        nom_above = true;
-      }
+      const int rv = rv_tab[es];
+      if (rv >= 0) { recv = rv; ent = es; kind = TRE_REBALANCE; }
     }
     if (!kind) continue;
-    const int recv = rc.m;
-    const T zr = rc.z;
+    uint16_t rk[MPL];
+#pragma unroll
+    for (int j = 0; j < MPL; ++j)
+      rk[j] = lane + 32 * j < M ? rk0[(size_t)ent * M + lane + 32 * j] : kNoRank;
     int g_own = 0;
 #pragma unroll
     for (int j = 0; j < MPL; ++j)
@@ -174,6 +226,8 @@ k_walk(const __grid_constant__ WalkBatch<T> b) {
         ++nm;
         continue;
       }
+      // release donor replicas one at a time until the receiver's footprint
+      // fits; an uncoverable transition releases nothing and ends the tick
       int rr[MPL];
 #pragma unroll
       for (int j = 0; j < MPL; ++j) rr[j] = r[j];
@@ -181,35 +235,21 @@ k_walk(const __grid_constant__ WalkBatch<T> b) {
       const int64_t nm0 = nm;
       bool ok = true;
       while (f < need) {
-        Cand<T> dc{0x7fffffff, (T)0, 0};
-#pragma unroll
-        for (int j = 0; j < MPL; ++j) {
-          const int m = lane + 32 * j;
-          if (m == recv || reg[j] == kCrit || reg[j] == 0xff || rr[j] <= rmin[j]) continue;
-          int grp;
-          if (reg[j] == kIdle) grp = 0;
-          else if (reg[j] == kSurp) grp = 1;
-          else if (!nom_above || z[j] > zr) grp = 2;
-          else continue;
-          // idle donors go by index only
-          const Cand<T> c{grp, grp == 0 ? (T)0 : z[j], m};
-          if (better(c, dc, true)) dc = c;
-        }
-        dc = warp_best(dc, true);
-        if (dc.grp == 0x7fffffff) { ok = false; break; }
-        const int d = dc.m;
+        int d = -1;
+        const int src = lane_of_min_rank<MPL>(rk, rr, rmin, lane, M, d);
+        if (src < 0) { ok = false; break; }
         int gd = 0;
 #pragma unroll
         for (int j = 0; j < MPL; ++j)
           if (lane + 32 * j == d) { rr[j] -= 1; gd = g[j]; }
-        gd = __shfl_sync(0xffffffffu, gd, d & 31);
+        gd = __shfl_sync(0xffffffffu, gd, src);
         f += gd;
         if (lane == 0 && nm < cap)
           mv[nm] = tre_move{(int32_t)k, (int16_t)recv, (int16_t)d, (uint8_t)kind, (uint8_t)seq, 0};
         ++nm;
       }
       if (!ok) {
-        nm = nm0;   // an uncoverable transition releases nothing
+        nm = nm0;
         break;
       }
 #pragma unroll
@@ -233,21 +273,40 @@ k_walk(const __grid_constant__ WalkBatch<T> b) {
 
 }  // namespace
 
-template <class T> cudaError_t launch_walk(const WalkBatch<T>& b, cudaStream_t s) {
+template <class T> void walk_ws_layout(Arena& a, WalkBatch<T>& b, WalkWs& w) {
+  int64_t total = 0;
+  for (int s = 0; s < b.n_series; ++s) {
+    b.ent_base[s] = (int32_t)total;
+    const int64_t span = (int64_t)b.series_K[s] * b.series_win[s];
+    total += span / b.fast_ms + span / b.slow_ms;
+  }
+  b.ent_base[b.n_series] = (int32_t)total;
+  w.recv = a.take<int16_t>((size_t)std::max<int64_t>(total * b.n_tau, 1));
+  w.rank = a.take<uint16_t>((size_t)std::max<int64_t>(total * b.n_tau * b.M, 1));
+}
+
+template <class T> cudaError_t launch_walk(const WalkBatch<T>& b, WalkWs& w, cudaStream_t s) {
   if (b.n_inst == 0) return cudaSuccess;
+  const int64_t ents = (int64_t)b.ent_base[b.n_series] * b.n_tau;
+  if (ents > 0) {
+    const int64_t th = ents * b.M;
+    k_tick_rank<T><<<(unsigned)((th + 255) / 256), 256, 0, s>>>(b, w.recv, w.rank);
+  }
   const unsigned grid = (unsigned)((b.n_inst + kWarpsPerBlock - 1) / kWarpsPerBlock);
   const int mpl = (b.M + 31) / 32;
   const unsigned th = kWarpsPerBlock * 32;
-  if (mpl <= 1) k_walk<T, 1><<<grid, th, 0, s>>>(b);
-  else if (mpl <= 2) k_walk<T, 2><<<grid, th, 0, s>>>(b);
-  else if (mpl <= 4) k_walk<T, 4><<<grid, th, 0, s>>>(b);
-  else if (mpl <= 8) k_walk<T, 8><<<grid, th, 0, s>>>(b);
-  else if (mpl <= 16) k_walk<T, 16><<<grid, th, 0, s>>>(b);
-  else k_walk<T, 32><<<grid, th, 0, s>>>(b);
+  if (mpl <= 1) k_walk<T, 1><<<grid, th, 0, s>>>(b, w.recv, w.rank);
+  else if (mpl <= 2) k_walk<T, 2><<<grid, th, 0, s>>>(b, w.recv, w.rank);
+  else if (mpl <= 4) k_walk<T, 4><<<grid, th, 0, s>>>(b, w.recv, w.rank);
+  else if (mpl <= 8) k_walk<T, 8><<<grid, th, 0, s>>>(b, w.recv, w.rank);
+  else if (mpl <= 16) k_walk<T, 16><<<grid, th, 0, s>>>(b, w.recv, w.rank);
+  else k_walk<T, 32><<<grid, th, 0, s>>>(b, w.recv, w.rank);
   return cudaGetLastError();
 }
 
-template cudaError_t launch_walk<float>(const WalkBatch<float>&, cudaStream_t);
-template cudaError_t launch_walk<double>(const WalkBatch<double>&, cudaStream_t);
+template void walk_ws_layout<float>(Arena&, WalkBatch<float>&, WalkWs&);
+template void walk_ws_layout<double>(Arena&, WalkBatch<double>&, WalkWs&);
+template cudaError_t launch_walk<float>(const WalkBatch<float>&, WalkWs&, cudaStream_t);
+template cudaError_t launch_walk<double>(const WalkBatch<double>&, WalkWs&, cudaStream_t);
 
 }  // namespace tre

@@ -41,7 +41,7 @@ def _call_noalloc(tre, lib, cnt_dev, prof_st, K, M, win, tdt, carry=None):
 
 
 @pytest.mark.parametrize("dtype", ["f32", "f64"])
-@pytest.mark.parametrize("K,M,win", [(36000, 8, 100), (600, 3, 1000), (20000, 64, 100)])
+@pytest.mark.parametrize("K,M,win", [(36000, 8, 100), (600, 3, 1000), (16384, 64, 100)])
 def test_noalloc_matches_tss_score_twice(dtype, K, M, win):
     import torch
     import paper_2609_29160_gb300 as tre
@@ -66,7 +66,7 @@ def test_noalloc_rejects_problems_beyond_its_buffer():
     import paper_2609_29160_gb300 as tre
     lib = tre.load()
     lib.tss_score_noalloc.restype = C.c_int
-    g = tre.Grid(1024, 100, 100000)     # 391 segments x 1024 models > 65536
+    g = tre.Grid(64, 100, 16385)        # 16385 x 64 cells > 2^20
     cs = tre.Counts(8, 8, 8, 8)
     prof = tre.Profile(0, 8, 8, 8, 8, 8, 8)
     st = lib.tss_score_noalloc(C.byref(g), C.byref(cs), C.byref(prof), None, None,
