@@ -161,20 +161,27 @@ def cpu_baseline(scale):
 
 
 def phase_bytes(sw, n_records_per_trace, M):
-    """Algorithmic bytes per launch of each phase (what the method must read and
-    write once): see the design doc, 'Roofline'."""
+    """Algorithmic bytes of one call of each phase over the whole sweep: what the
+    method must read and write once, per record and per (window, model)."""
+    nt = len(sw["traces"])
     K = [sw["duration_ms"] // int(w) for w in sw["window_ms"]]
-    Kb = min(K) and sw["duration_ms"] // int(min(sw["window_ms"]))
-    n_series = len(sw["traces"]) * len(K)
-    mw = sum(K) * len(sw["traces"]) * M
+    Kb = sw["duration_ms"] // int(min(sw["window_ms"]))
+    mw = sum(K) * nt * M                      # model-windows over all series
+    base = Kb * M * nt                        # base-grid cells over all traces
     return {
-        # records in (7 int32 columns) + P, D, A and W diffs, SLO counts out at the base grid
-        "reduce": float(np.mean(n_records_per_trace)) * 28 + Kb * M * 24,
-        # counts in, S + idle flag out, per series (average over series)
-        "score": mw * (16 + 4 + 1) / n_series,
-        # S + class + SLO counts in per series
-        "calibrate": mw * (4 + 1 + 8) / n_series,
-        "normalize": mw * (4 + 1 + 4 + 1) / n_series,
+        # 7 int32 columns per record in; P, D, A/W diffs (4 B each) and the
+        # packed SLO counts (8 B) per base cell out
+        "reduce": float(np.sum(n_records_per_trace)) * 28 + base * 24,
+        # diffs in, gauges out
+        "gauge_scan": base * 16,
+        # base counts + SLO in, series counts + SLO out
+        "aggregate": base * 24 + mw * 24,
+        # counts in, S and the idle flag out
+        "score": mw * (16 + 4 + 1),
+        # S, idle flag and SLO counts in
+        "calibrate": mw * (4 + 1 + 8),
+        # S and idle flag in, Z and region out
+        "normalize": mw * (4 + 1 + 4 + 1),
     }
 
 
@@ -265,15 +272,22 @@ def main():
     pb = phase_bytes(sw, n_rec, M)
     dom = max(phases, key=lambda k: phases[k]["ms"])
     share = phases[dom]["ms"] / max(ms, 1e-9)
+    def roof_of(name):
+        per_call_ms = phases[name]["ms"] / max(phases[name]["calls"], 1)
+        achieved = pb[name] / (per_call_ms / 1e3) / 1e9
+        return {"bound": "hbm", "kernel": name, "achieved": achieved, "peak": hbm,
+                "unit": "GB/s", "frac": achieved / hbm, "traffic": None,
+                "share_of_step": phases[name]["ms"] / max(ms, 1e-9), "peak_kind": peak_kind,
+                "bytes_per_call": pb[name], "us_per_call": per_call_ms * 1e3}
     if dom in pb and phases[dom]["calls"]:
-        per_launch_ms = phases[dom]["ms"] / phases[dom]["calls"]
-        achieved = pb[dom] / (per_launch_ms / 1e3) / 1e9
-        roof = {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": hbm, "unit": "GB/s",
-                "frac": achieved / hbm, "traffic": None, "share_of_step": share,
-                "peak_kind": peak_kind}
+        roof = roof_of(dom)
     else:
-        roof = {"bound": "latency", "kernel": dom, "achieved": None, "peak": hbm, "unit": "GB/s",
-                "frac": None, "traffic": None, "share_of_step": share, "peak_kind": peak_kind}
+        # the controller walk is serial over control ticks: no bandwidth roofline
+        # applies; report the largest bandwidth-bound phase beside it
+        hb = max((k for k in pb if phases.get(k, {}).get("calls")), key=lambda k: phases[k]["ms"])
+        roof = roof_of(hb)
+        roof["dominant_phase"] = {"name": dom, "share_of_step": share,
+                                  "bound": "latency (serial over control ticks)"}
     # whole-step view against HBM: algorithmic bytes of the full sweep per step
     step_bytes = total_rec * 28 + model_windows * (16 + 4 + 4 + 1)
     whole = {"algorithmic_bytes": step_bytes, "achieved_gbs": step_bytes / (ms_step / 1e3) / 1e9,
@@ -325,6 +339,8 @@ def main():
             "model_windows_per_s": mw_s,
             "roofline": roof, "step_roofline": whole, "phases_ms_per_step": {
                 k: p["ms"] / args.steps for k, p in phases.items() if p["calls"]},
+            "phases_roofline": {k: round(roof_of(k)["frac"], 4) for k in pb
+                                if phases.get(k, {}).get("calls")},
             "gpu_launches": launches, "clocks": clk, "e2e": e2e, "cpu_baseline": base,
         }
         print(json.dumps(line))

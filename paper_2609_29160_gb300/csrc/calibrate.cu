@@ -125,14 +125,23 @@ __device__ __forceinline__ int block_min(int v, int* red) {
   return r;
 }
 
+constexpr int kFine = 4096;     // buckets of the first histogram
+constexpr int kCap = 4096;      // most keys the exact pass sorts in shared memory
+
+template <class T> size_t search_smem_bytes() {
+  using U = typename KeyOf<T>::U;
+  const size_t fast = (size_t)kFine * (5 * 4 + sizeof(U)) + (size_t)kCap * (sizeof(U) + 4);
+  const size_t descent = (size_t)KeyOf<T>::kLevels * kNB * (4 + 4 + sizeof(U));
+  return fast > descent ? fast : descent;
+}
+
 template <class T>
 __global__ void __launch_bounds__(kNB)
 k_search(const __grid_constant__ SeriesTable<T> tab, const typename KeyOf<T>::U* __restrict__ keys,
          double reliability, T* theta, tre_diag* diag) {
   using U = typename KeyOf<T>::U;
   constexpr int NL = KeyOf<T>::kLevels;
-  __shared__ int32_t cnt[NL][kNB], hl[NL][kNB];
-  __shared__ U mn[NL][kNB];
+  extern __shared__ __align__(16) unsigned char dyn[];
   __shared__ U lo_s[NL], hi_s[NL];
   __shared__ int shift_s[NL], pos_s[NL];
   __shared__ int64_t cab_s[NL], hab_s[NL];
@@ -140,36 +149,39 @@ k_search(const __grid_constant__ SeriesTable<T> tab, const typename KeyOf<T>::U*
   __shared__ int red32[kWarps];
   __shared__ U kmin_s, kmax_s;
   __shared__ unsigned long long ncand_s;
+  __shared__ int nsel_s;
   const int M = tab.M;
   const int s = blockIdx.x / M, m = blockIdx.x % M;
   const int K = tab.K[s];
   const U* mk = keys + (size_t)tab.off[s] + (size_t)m * K;
   const int tid = threadIdx.x, lane = tid & 31;
+  const size_t out = (size_t)s * M + m;
 
-  // range of candidate keys
+  // ---- range of candidate keys -------------------------------------------
   if (tid == 0) {
     kmin_s = ~(U)0;
     kmax_s = 0;
     ncand_s = 0;
   }
   __syncthreads();
-  U lmin = ~(U)0, lmax = 0;
-  unsigned long long lc = 0;
-  for (int i = tid; i < K; i += kNB) {
-    const U p = mk[i];
-    if (!p) continue;
-    const U key = p >> 1;
-    lmin = key < lmin ? key : lmin;
-    lmax = key > lmax ? key : lmax;
-    ++lc;
-  }
-  if (lc) {
-    atomicMin(&kmin_s, lmin);
-    atomicMax(&kmax_s, lmax);
-    atomicAdd(&ncand_s, lc);
+  {
+    U lmin = ~(U)0, lmax = 0;
+    unsigned long long lc = 0;
+    for (int i = tid; i < K; i += kNB) {
+      const U p = mk[i];
+      if (!p) continue;
+      const U key = p >> 1;
+      lmin = key < lmin ? key : lmin;
+      lmax = key > lmax ? key : lmax;
+      ++lc;
+    }
+    if (lc) {
+      atomicMin(&kmin_s, lmin);
+      atomicMax(&kmax_s, lmax);
+      atomicAdd(&ncand_s, lc);
+    }
   }
   __syncthreads();
-  const size_t out = (size_t)s * M + m;
   if (ncand_s == 0) {
     if (tid == 0) {
       theta[out] = (T)1;
@@ -177,8 +189,177 @@ k_search(const __grid_constant__ SeriesTable<T> tab, const typename KeyOf<T>::U*
     }
     return;
   }
+  const U kmin = kmin_s, kmax = kmax_s;
 
-  // histogram of the keys in [lo, hi] of level l, bucket (key - lo) >> shift
+  // ---- fast path -----------------------------------------------------------
+  // A fine histogram over [kmin, kmax]; per bucket the exact test at its
+  // smallest value ("found") and the bound for values inside it ("maybe").
+  // With bf the lowest found bucket, theta is either a value inside a maybe
+  // bucket below bf or the smallest value of bf. Those maybe buckets' keys are
+  // gathered, sorted and tested one distinct value at a time.
+  {
+    int32_t* fcnt = reinterpret_cast<int32_t*>(dyn);
+    int32_t* fhl = fcnt + kFine;
+    int32_t* fst = fhl + kFine;                 // run start of a selected bucket, -1 if not
+    int32_t* fca = fst + kFine;                 // windows in buckets above
+    int32_t* fha = fca + kFine;                 // healthy windows in buckets above
+    U* fmn = reinterpret_cast<U*>(fha + kFine);
+    U* list = fmn + kFine;
+    int32_t* hpre = reinterpret_cast<int32_t*>(list + kCap);
+    int sh = 0;
+    while (sh < 63 && ((kmax - kmin) >> sh) >= (U)kFine) ++sh;
+    for (int b = tid; b < kFine; b += kNB) {
+      fcnt[b] = 0;
+      fhl[b] = 0;
+      fmn[b] = ~(U)0;
+    }
+    __syncthreads();
+    for (int i = tid; i < K; i += kNB) {
+      const U p = mk[i];
+      if (!p) continue;
+      const U key = p >> 1;
+      const int b = (int)((key - kmin) >> sh);
+      atomicAdd(&fcnt[b], 1);
+      if (p & 1) atomicAdd(&fhl[b], 1);
+      if (key < fmn[b]) atomicMin(&fmn[b], key);
+    }
+    __syncthreads();
+    constexpr int PER = kFine / kNB;            // consecutive buckets per thread
+    const int b0 = tid * PER;
+    int64_t tc = 0, th = 0;
+    for (int j = 0; j < PER; ++j) {
+      tc += fcnt[b0 + j];
+      th += fhl[b0 + j];
+    }
+    int64_t c_above = block_suffix(tc, red64), h_above = block_suffix(th, red64);
+    int my_found = 0x7fffffff;
+    uint32_t maybe_bits = 0;
+    for (int j = PER - 1; j >= 0; --j) {
+      const int b = b0 + j;
+      const int32_t c = fcnt[b], h = fhl[b];
+      fca[b] = (int32_t)c_above;
+      fha[b] = (int32_t)h_above;
+      if (c > 0) {
+        if ((double)(h_above + h) >= reliability * (double)(c_above + c)) {
+          my_found = b;
+        } else if ((double)(h_above + h + 1) >= reliability * (double)(c_above + h)) {
+          // a value inside adds at most the bucket's healthy windows to those
+          // above; one window of slack keeps the bound valid under rounding
+          maybe_bits |= 1u << j;
+        }
+      }
+      c_above += c;
+      h_above += h;
+    }
+    const int bf = block_min(my_found, red32);
+    int64_t my_sel = 0;
+    for (int j = 0; j < PER; ++j)
+      if ((maybe_bits >> j & 1) && b0 + j < bf) my_sel += fcnt[b0 + j];
+    const int64_t sel_above = block_suffix(my_sel, red64);
+    if (tid == 0) nsel_s = 0;
+    __syncthreads();
+    if (my_sel) atomicAdd(&nsel_s, (int)my_sel);
+    __syncthreads();
+    const int nsel = nsel_s;
+    if (nsel <= kCap) {
+      if (nsel == 0) {
+        if (tid == 0) {
+          if (bf != 0x7fffffff) {
+            theta[out] = value_of(fmn[bf]);
+          } else {
+            theta[out] = value_of(kmax);
+            atomicAdd(&diag->degenerate_calib, 1ull);
+          }
+        }
+        return;
+      }
+      // where each selected bucket's keys start in ascending order
+      int64_t run = nsel - sel_above - my_sel;
+      for (int j = 0; j < PER; ++j) {
+        const int b = b0 + j;
+        if ((maybe_bits >> j & 1) && b < bf) {
+          fst[b] = (int32_t)run;
+          run += fcnt[b];
+        } else {
+          fst[b] = -1;
+        }
+      }
+      if (tid == 0) nsel_s = 0;
+      __syncthreads();
+      for (int i = tid; i < K; i += kNB) {
+        const U p = mk[i];
+        if (!p) continue;
+        const int b = (int)(((p >> 1) - kmin) >> sh);
+        if (fst[b] >= 0) list[atomicAdd(&nsel_s, 1)] = p;
+      }
+      int n2 = 32;
+      while (n2 < nsel) n2 <<= 1;
+      for (int i = nsel + tid; i < n2; i += kNB) list[i] = ~(U)0;
+      __syncthreads();
+      for (int k2 = 2; k2 <= n2; k2 <<= 1) {       // bitonic sort, ascending
+        for (int j2 = k2 >> 1; j2 > 0; j2 >>= 1) {
+          for (int i = tid; i < n2; i += kNB) {
+            const int ixj = i ^ j2;
+            if (ixj > i) {
+              const U a = list[i], c = list[ixj];
+              if ((a > c) == ((i & k2) == 0)) {
+                list[i] = c;
+                list[ixj] = a;
+              }
+            }
+          }
+          __syncthreads();
+        }
+      }
+      // inclusive healthy prefix over the sorted keys
+      constexpr int PERC = kCap / kNB;
+      int hs = 0;
+      for (int j = 0; j < PERC; ++j) {
+        const int i = tid * PERC + j;
+        if (i < nsel) hs += (int)(list[i] & 1);
+      }
+      const int64_t h_after = block_suffix(hs, red64);
+      if (tid == 0) red64[0] = h_after + hs;       // total
+      __syncthreads();
+      int64_t hp = red64[0] - (h_after + hs);
+      __syncthreads();
+      for (int j = 0; j < PERC; ++j) {
+        const int i = tid * PERC + j;
+        if (i < nsel) hp += (int64_t)(list[i] & 1);
+        hpre[i] = (int32_t)hp;
+      }
+      __syncthreads();
+      // exact test at the first position of every distinct value
+      int best = 0x7fffffff;
+      for (int i = tid; i < nsel; i += kNB) {
+        const U key = list[i] >> 1;
+        if (i > 0 && (list[i - 1] >> 1) == key) continue;
+        const int b = (int)((key - kmin) >> sh);
+        const int end = fst[b] + fcnt[b];
+        const int64_t C = (int64_t)fca[b] + (end - i);
+        const int64_t H = (int64_t)fha[b] + hpre[end - 1] - (i > 0 ? hpre[i - 1] : 0);
+        if ((double)H >= reliability * (double)C) best = min(best, i);
+      }
+      best = block_min(best, red32);
+      if (tid == 0) {
+        if (best != 0x7fffffff) {
+          theta[out] = value_of(list[best] >> 1);
+        } else if (bf != 0x7fffffff) {
+          theta[out] = value_of(fmn[bf]);
+        } else {
+          theta[out] = value_of(kmax);
+          atomicAdd(&diag->degenerate_calib, 1ull);
+        }
+      }
+      return;
+    }
+  }
+  __syncthreads();
+
+  // ---- fallback: radix descent over the key range (many candidate keys) ----
+  int32_t (*cnt)[kNB] = reinterpret_cast<int32_t (*)[kNB]>(dyn);
+  int32_t (*hl)[kNB] = reinterpret_cast<int32_t (*)[kNB]>(dyn + (size_t)NL * kNB * 4);
+  U (*mn)[kNB] = reinterpret_cast<U (*)[kNB]>(dyn + (size_t)NL * kNB * 8);
   auto build = [&](int l) {
     cnt[l][tid] = 0;
     hl[l][tid] = 0;
@@ -205,8 +386,6 @@ k_search(const __grid_constant__ SeriesTable<T> tab, const typename KeyOf<T>::U*
     }
     __syncthreads();
   };
-
-  // level 0 covers [kmin, kmax]
   auto set_range = [&](int l, U lo, U hi, int64_t ca, int64_t ha) {
     int sh = 0;
     while (sh < 63 && ((hi - lo) >> sh) >= (U)kNB) ++sh;
@@ -217,12 +396,11 @@ k_search(const __grid_constant__ SeriesTable<T> tab, const typename KeyOf<T>::U*
     cab_s[l] = ca;
     hab_s[l] = ha;
   };
-  if (tid == 0) set_range(0, kmin_s, kmax_s, 0, 0);
+  if (tid == 0) set_range(0, kmin, kmax, 0, 0);
   __syncthreads();
   build(0);
   int l = 0;
   while (true) {
-    // per bucket: windows above it (inside this range and above the range)
     const int64_t c_above = block_suffix(cnt[l][tid], red64) + cab_s[l];
     const int64_t h_above = block_suffix(hl[l][tid], red64) + hab_s[l];
     const int32_t c = cnt[l][tid], h = hl[l][tid];
@@ -233,18 +411,15 @@ k_search(const __grid_constant__ SeriesTable<T> tab, const typename KeyOf<T>::U*
         kind = 1;
       } else if (shift_s[l] > 0 &&
                  (double)(h_above + h + 1) >= reliability * (double)(c_above + h)) {
-        // a value inside the bucket adds at most its healthy windows to those
-        // above; one window of slack keeps the bound valid under rounding
         kind = 2;
       }
       if (kind) cand = tid;
     }
     const int b = block_min(cand, red32);
     if (b == 0x7fffffff) {
-      // nothing in this range: resume the parent range above the refined bucket
       if (l == 0) {
         if (tid == 0) {
-          theta[out] = value_of(kmax_s);
+          theta[out] = value_of(kmax);
           atomicAdd(&diag->degenerate_calib, 1ull);
         }
         return;
@@ -260,7 +435,6 @@ k_search(const __grid_constant__ SeriesTable<T> tab, const typename KeyOf<T>::U*
       if (tid == 0) theta[out] = value_of(mn[l][b]);
       return;
     }
-    // refine bucket b
     if (tid == b) {
       const U lo = lo_s[l] + ((U)b << shift_s[l]);
       const U hi = lo + (((U)1 << shift_s[l]) - 1);
@@ -292,8 +466,16 @@ cudaError_t launch_calibrate(const SeriesTable<T>& tab, const T* S, const uint8_
     dim3 g((Kmax + 31) / 32, (tab.M + 31) / 32, tab.n), b(32, 8);
     k_pack<T><<<g, b, 0, s>>>(tab, S, cls, slo, w.thr, ok_frac, static_cast<U*>(w.keys));
   }
-  k_search<T><<<tab.n * tab.M, kNB, 0, s>>>(tab, static_cast<const U*>(w.keys), reliability,
-                                            theta, diag);
+  const size_t smem = search_smem_bytes<T>();
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(k_search<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e) return e;
+    attr_set = true;
+  }
+  k_search<T><<<tab.n * tab.M, kNB, smem, s>>>(tab, static_cast<const U*>(w.keys), reliability,
+                                               theta, diag);
   return cudaGetLastError();
 }
 

@@ -49,6 +49,25 @@ __device__ __forceinline__ void divmod(unsigned long long x, uint32_t d, unsigne
   }
 }
 
+// Division of an unsigned 32-bit value by a divisor fixed for the launch,
+// without a divide instruction (round-up multiply-high method of Granlund and
+// Montgomery): exact for every 32-bit dividend and 1 <= d < 2^31.
+struct FastDiv {
+  uint32_t d, m, s1, s2;
+  FastDiv() = default;
+  explicit FastDiv(uint32_t div) : d(div) {
+    uint32_t l = 0;
+    while ((1ull << l) < div) ++l;
+    m = (uint32_t)(((1ull << 32) * ((1ull << l) - div)) / div + 1);
+    s1 = l > 0 ? 1 : 0;
+    s2 = l > 0 ? l - 1 : 0;
+  }
+  __device__ __forceinline__ uint32_t div(uint32_t x) const {
+    const uint32_t t = __umulhi(x, m);
+    return (t + ((x - t) >> s1)) >> s2;
+  }
+};
+
 // warp-level sum of a 64-bit counter, one atomic per warp when non-zero
 __device__ __forceinline__ void warp_add_counter(unsigned long long* dst, unsigned long long v) {
   const unsigned full = 0xffffffffu;

@@ -162,7 +162,11 @@ template <class T> struct WalkBatch {
 // per-(series, tau, tick) receiver and per-model donor ranks
 struct WalkWs {
   int16_t* recv;
-  uint16_t* rank;
+  int16_t* n_donor;   // donors with a rank at the tick
+  uint16_t* rank;     // [entry][model] position in the donor order
+  uint16_t* order;    // [entry][position] model at that position
+  unsigned long long* packed;  // [entry] donor order, 4 bits per position (M <= 16)
+  uint32_t* dmask;             // [entry] bitmask of the models with a rank (M <= 16)
 };
 // lays out the tick tables and fills b.ent_base
 template <class T> void walk_ws_layout(Arena& a, WalkBatch<T>& b, WalkWs& w);

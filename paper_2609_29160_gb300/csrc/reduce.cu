@@ -17,12 +17,13 @@ namespace tre {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kStageBytes = 48 * 1024;
+constexpr int kStageBytes = 24 * 1024;   // staged rows per CTA: 8 CTAs of 256 threads per SM
 constexpr int kSpill = 32;  // staged rows beyond the CTA's arrival range
 
-__device__ __forceinline__ int64_t win_clamp(int64_t t, int win, int K) {
+// window of a millisecond time (int32 range), clamped to [0, K]
+__device__ __forceinline__ int64_t win_clamp(int64_t t, const FastDiv& fd, int K) {
   if (t < 0) return 0;
-  const int64_t b = t / win;
+  const int64_t b = fd.div((uint32_t)t);
   return b > K ? K : b;
 }
 
@@ -48,7 +49,7 @@ struct ReqBatch {
 
 template <bool SLO>
 __global__ void __launch_bounds__(kThreads)
-k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int win, int K, int rows,
+k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int win, FastDiv fd, int K, int rows,
                   int32_t* __restrict__ P0, int32_t* __restrict__ D0, int32_t* __restrict__ dA0,
                   int32_t* __restrict__ dW0, unsigned long long* __restrict__ slo0,
                   const int32_t* __restrict__ slo_ms, tre_diag* diag) {
@@ -67,8 +68,8 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int win, int K, in
   const int64_t i1 = min(r.n, i0 + per_cta);
   if (i0 >= i1) return;
   const int64_t span = (int64_t)K * win;
-  const int64_t k_lo = win_clamp(r.t_arr[i0], win, K);
-  const int64_t k_hi = win_clamp(r.t_arr[i1 - 1], win, K);
+  const int64_t k_lo = win_clamp(r.t_arr[i0], fd, K);
+  const int64_t k_hi = win_clamp(r.t_arr[i1 - 1], fd, K);
   const int64_t need = (k_hi >= k_lo ? k_hi - k_lo + 1 : 1) + kSpill;
   const int used = (int)min64(rows, need);
   const int cells = used * M;
@@ -84,20 +85,35 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int win, int K, in
   __syncthreads();
 
   unsigned long long n_range = 0, n_model = 0, n_order = 0;
+  // the next record's columns are loaded while the current one is processed
+  int32_t nx[7];
+  auto load_rec = [&](int64_t i) {
+    if (i < i1) {
+      nx[0] = r.model[i];
+      nx[1] = r.t_arr[i];
+      nx[2] = r.t_start[i];
+      nx[3] = r.t_first[i];
+      nx[4] = r.t_end[i];
+      nx[5] = r.L_in[i];
+      nx[6] = r.L_out[i];
+    }
+  };
+  load_rec(i0 + threadIdx.x);
   for (int64_t i = i0 + threadIdx.x; i < i1; i += kThreads) {
-    const int m = r.model[i];
-    const int64_t ta = r.t_arr[i], ts = r.t_start[i], tf = r.t_first[i], te = r.t_end[i];
-    const int32_t L_in = r.L_in[i], L = r.L_out[i];
+    const int m = nx[0];
+    const int64_t ta = nx[1], ts = nx[2], tf = nx[3], te = nx[4];
+    const int32_t L_in = nx[5], L = nx[6];
+    load_rec(i + kThreads);
     if (m < 0 || m >= M) { ++n_model; continue; }
     if (ta < 0 || ta >= span) { ++n_range; continue; }
     if (!(ta <= ts && ts <= tf && tf <= te) || L_in < 0 || L < 1) { ++n_order; continue; }
 
     if (tf < span) {
-      const int64_t kf = tf / win;
+      const int64_t kf = fd.div((uint32_t)tf);
       // prompt tokens, all at the first-token time
       if (L_in) stage_add<int32_t>(sP, P, kf, k_lo, used, M, m, L_in);
       // decode tokens: N(T) = tokens emitted before T; D[k] = N((k+1)w) - N(kw)
-      const int64_t ke_raw = te / win;
+      const int64_t ke_raw = fd.div((uint32_t)te);
       if (L == 1 || ke_raw == kf) {
         stage_add<int32_t>(sD, D, kf, k_lo, used, M, m, L);
       } else {
@@ -126,7 +142,7 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int win, int K, in
       }
     }
     // gauges: +1 where the state begins, -1 where it ends
-    const int64_t ba = win_clamp(ta, win, K), bs = win_clamp(ts, win, K), be = win_clamp(te, win, K);
+    const int64_t ba = win_clamp(ta, fd, K), bs = win_clamp(ts, fd, K), be = win_clamp(te, fd, K);
     if (ba != bs) {
       stage_add<int32_t>(sW, dW, ba, k_lo, used, M, m, 1);
       stage_add<int32_t>(sW, dW, bs, k_lo, used, M, m, -1);
@@ -205,7 +221,7 @@ __device__ __forceinline__ bool ms_tick(float t, int64_t span, int64_t& tick) {
 }
 
 __global__ void __launch_bounds__(kThreads)
-k_reduce_events(EvCols e, int M, int win, int K, int64_t per_cta, int rows,
+k_reduce_events(EvCols e, int M, int win, FastDiv fd, int K, int64_t per_cta, int rows,
                 int32_t* __restrict__ P, int32_t* __restrict__ D, int32_t* __restrict__ first,
                 int32_t* __restrict__ last, tre_diag* diag) {
   extern __shared__ unsigned long long smem[];
@@ -214,8 +230,8 @@ k_reduce_events(EvCols e, int M, int win, int K, int64_t per_cta, int rows,
   if (i0 >= i1) return;
   const int64_t span = (int64_t)K * win;
   int64_t t0, t1;
-  const int64_t k_lo = ms_tick(e.t_s[i0], span, t0) ? t0 / win : 0;
-  const int64_t k_hi = ms_tick(e.t_s[i1 - 1], span, t1) ? t1 / win : K;
+  const int64_t k_lo = ms_tick(e.t_s[i0], span, t0) ? fd.div((uint32_t)t0) : 0;
+  const int64_t k_hi = ms_tick(e.t_s[i1 - 1], span, t1) ? fd.div((uint32_t)t1) : K;
   const int64_t need = (k_hi >= k_lo ? k_hi - k_lo + 1 : 1) + kSpill;
   const int used = (int)min64(rows, need);
   const int cells = used * M;
@@ -245,7 +261,7 @@ k_reduce_events(EvCols e, int M, int win, int K, int64_t per_cta, int rows,
         ++n_order;
       } else {
         ok = true;
-        const int64_t k = tick / win;
+        const int64_t k = fd.div((uint32_t)tick);
         stage_add<int32_t>(ph == 0 ? sP : sD, ph == 0 ? P : D, k, k_lo, used, M, m, 1);
       }
     }
@@ -286,7 +302,7 @@ __global__ void k_fill_first_last(int32_t* first, int32_t* last, int64_t n) {
 // per request with at least one valid event: waiting on [t_arr, first),
 // running on [first, last)
 __global__ void __launch_bounds__(kThreads)
-k_event_gauges(EvCols e, int M, int win, int K, const int32_t* __restrict__ first,
+k_event_gauges(EvCols e, int M, FastDiv fd, int K, const int32_t* __restrict__ first,
                const int32_t* __restrict__ last, int32_t* __restrict__ dA,
                int32_t* __restrict__ dW, tre_diag* diag) {
   unsigned long long n_order = 0;
@@ -298,7 +314,7 @@ k_event_gauges(EvCols e, int M, int win, int K, const int32_t* __restrict__ firs
     const int m = e.req_model[r];
     const int64_t ta = e.req_t_arr[r];
     if (!(ta >= 0 && ta <= ft)) { ++n_order; continue; }
-    const int64_t ba = win_clamp(ta, win, K), bf = win_clamp(ft, win, K), bl = win_clamp(lt, win, K);
+    const int64_t ba = win_clamp(ta, fd, K), bf = win_clamp(ft, fd, K), bl = win_clamp(lt, fd, K);
     if (ba != bf) {
       atomicAdd(&dW[ba * M + m], 1);
       atomicAdd(&dW[bf * M + m], -1);
@@ -421,17 +437,17 @@ k_aggregate(const __grid_constant__ AggPlan pl, const int32_t* __restrict__ P,
   const size_t o0 = (size_t)pl.out_off[tr][w];
   for (int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x; t < n;
        t += (int64_t)gridDim.x * kThreads) {
-    const int m = (int)(t % M);
-    const int64_t k = t / M;
+    const uint32_t k = (uint32_t)t / (uint32_t)M;
+    const int m = (int)((uint32_t)t - k * (uint32_t)M);
     int32_t p = 0, d = 0;
     unsigned long long sl = 0;
     for (int j = 0; j < q; ++j) {
-      const size_t x = in0 + (size_t)(k * q + j) * M + m;
+      const size_t x = in0 + ((size_t)k * q + j) * M + m;
       p += P[x];
       d += D[x];
       if (slo) sl += slo[x];
     }
-    const size_t last = in0 + (size_t)(k * q + q - 1) * M + m;
+    const size_t last = in0 + ((size_t)k * q + q - 1) * M + m;
     Pq[o0 + t] = p;
     Dq[o0 + t] = d;
     Aq[o0 + t] = A[last];
@@ -513,11 +529,11 @@ cudaError_t launch_reduce_requests(const ReqCols* traces, int n_traces, int M, i
   const int rows = std::max(1, kStageBytes / (cell_bytes * M));
   const size_t smem = (size_t)rows * M * cell_bytes;
   if (slo)
-    k_reduce_requests<true><<<ctas, kThreads, smem, s>>>(bt, M, win, K, rows, P, D, w.dA, w.dW,
-                                                         slo, slo_ms, diag);
+    k_reduce_requests<true><<<ctas, kThreads, smem, s>>>(bt, M, win, FastDiv(win), K, rows, P, D,
+                                                         w.dA, w.dW, slo, slo_ms, diag);
   else
-    k_reduce_requests<false><<<ctas, kThreads, smem, s>>>(bt, M, win, K, rows, P, D, w.dA, w.dW,
-                                                          nullptr, nullptr, diag);
+    k_reduce_requests<false><<<ctas, kThreads, smem, s>>>(bt, M, win, FastDiv(win), K, rows, P, D,
+                                                          w.dA, w.dW, nullptr, nullptr, diag);
   return cudaGetLastError();
 }
 
@@ -545,13 +561,13 @@ cudaError_t launch_reduce_events(const EvCols& ev, int M, int win, int K, int32_
     const int rows = std::max(1, kStageBytes / (8 * M));
     const int64_t per = per_cta_records(ev.n, 2048, 16384);
     const unsigned grid = (unsigned)((ev.n + per - 1) / per);
-    k_reduce_events<<<grid, kThreads, (size_t)rows * M * 8, s>>>(ev, M, win, K, per, rows, P, D,
-                                                                 w.first, w.last, diag);
+    k_reduce_events<<<grid, kThreads, (size_t)rows * M * 8, s>>>(ev, M, win, FastDiv(win), K, per,
+                                                                 rows, P, D, w.first, w.last, diag);
     if ((e = cudaGetLastError())) return e;
   }
   if (ev.n_req > 0) {
-    k_event_gauges<<<grid_for(ev.n_req, 4), kThreads, 0, s>>>(ev, M, win, K, w.first, w.last,
-                                                               w.dA, w.dW, diag);
+    k_event_gauges<<<grid_for(ev.n_req, 4), kThreads, 0, s>>>(ev, M, FastDiv(win), K, w.first,
+                                                               w.last, w.dA, w.dW, diag);
     if ((e = cudaGetLastError())) return e;
   }
   return cudaSuccess;

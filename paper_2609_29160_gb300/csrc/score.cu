@@ -79,7 +79,7 @@ k_raw(const __grid_constant__ SeriesTable<T> tab, Counts c, const T* __restrict_
   for (int64_t i = (int64_t)blockIdx.x * kThreads + threadIdx.x; i < n;
        i += (int64_t)gridDim.x * kThreads) {
     const size_t x = (size_t)(tab.off[s] + i);
-    const int m = (int)(i % M);
+    const int m = (int)((uint32_t)i % (uint32_t)M);
     const int32_t p = c.P[x], d = c.D[x], a = c.A[x], w = c.W[x];
     if ((p | d | a | w) == 0) {
       cls[x] = kIdle;
@@ -92,6 +92,32 @@ k_raw(const __grid_constant__ SeriesTable<T> tab, Counts c, const T* __restrict_
     if (den < (T)1) den = (T)1;                       // demand floor of one request
     raw[x] = div_rn(num, den);
     cls[x] = kNom;
+  }
+}
+
+// raw values and classes of windows [k, k + kBatch) clipped to k1 (idle past k1)
+template <class T>
+__device__ __forceinline__ void load_batch(const T* __restrict__ raw, const uint8_t* __restrict__ cls,
+                                           size_t base, int M, int64_t k, int64_t k1,
+                                           T (&r)[kBatch], uint8_t (&c)[kBatch]) {
+  if (k + kBatch <= k1) {
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) {
+      const size_t x = base + (size_t)(k + j) * M;
+      c[j] = cls[x];
+      r[j] = raw[x];
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) {
+      c[j] = kIdle;
+      r[j] = (T)0;
+      if (k + j < k1) {
+        const size_t x = base + (size_t)(k + j) * M;
+        c[j] = cls[x];
+        r[j] = raw[x];
+      }
+    }
   }
 }
 
@@ -114,18 +140,12 @@ k_summary(const __grid_constant__ SeriesTable<T> tab, const T* __restrict__ raw,
   const size_t base = (size_t)tab.off[s] + m;
   T mm = (T)1, cc = (T)0, ci = (T)0;
   int h = 0;
+  T r[kBatch], rn[kBatch];
+  uint8_t c[kBatch], cn[kBatch];
+  load_batch(raw, cls, base, M, k0, k1, r, c);
   for (int64_t k = k0; k < k1; k += kBatch) {
-    T r[kBatch];
-    uint8_t c[kBatch];
-#pragma unroll
-    for (int j = 0; j < kBatch; ++j) {
-      c[j] = kIdle;
-      if (k + j < k1) {
-        const size_t x = base + (size_t)(k + j) * M;
-        c[j] = cls[x];
-        r[j] = raw[x];
-      }
-    }
+    // next batch in flight while this one is folded
+    load_batch(raw, cls, base, M, k + kBatch, k1, rn, cn);
 #pragma unroll
     for (int j = 0; j < kBatch; ++j) {
       if (c[j] == kIdle) continue;
@@ -134,6 +154,11 @@ k_summary(const __grid_constant__ SeriesTable<T> tab, const T* __restrict__ raw,
       cc = cc * b + ar;
       mm = mm * b;
       h = 1;
+    }
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) {
+      r[j] = rn[j];
+      c[j] = cn[j];
     }
   }
   sm[t] = mm;
@@ -219,19 +244,18 @@ __device__ __forceinline__ bool run_segment(size_t base, int M, int64_t k0, int6
                                             const T* __restrict__ raw, const ModelParams<T>& q,
                                             T& S, int& init, bool verify, int stored_init,
                                             T* S_out, T* Z_out, uint8_t* cls, bool with_z) {
+  T r[kBatch], rn[kBatch];
+  uint8_t c[kBatch], cn[kBatch];
+  load_batch(raw, cls, base, M, k0, k1, r, c);
   for (int64_t k = k0; k < k1; k += kBatch) {
-    T r[kBatch], old[kBatch];
-    uint8_t c[kBatch];
+    T old[kBatch];
+    if (verify) {
 #pragma unroll
-    for (int j = 0; j < kBatch; ++j) {
-      c[j] = kIdle;
-      if (k + j < k1) {
-        const size_t x = base + (size_t)(k + j) * M;
-        c[j] = cls[x];
-        r[j] = raw[x];
-        if (verify) old[j] = S_out[x];
-      }
+      for (int j = 0; j < kBatch; ++j)
+        if (k + j < k1) old[j] = S_out[base + (size_t)(k + j) * M];
     }
+    // next batch in flight while this one runs
+    load_batch(raw, cls, base, M, k + kBatch, k1, rn, cn);
 #pragma unroll
     for (int j = 0; j < kBatch; ++j) {
       if (k + j >= k1) break;
@@ -254,6 +278,11 @@ __device__ __forceinline__ bool run_segment(size_t base, int M, int64_t k0, int6
         Z_out[x] = Z;
         if (active) cls[x] = Z < q.tc ? kCrit : (Z > q.ts ? kSurp : kNom);
       }
+    }
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) {
+      r[j] = rn[j];
+      c[j] = cn[j];
     }
   }
   return false;
@@ -390,7 +419,7 @@ k_normalize(const __grid_constant__ SeriesTable<T> tab, const T* S, const uint8_
   for (int64_t i = (int64_t)blockIdx.x * kThreads + threadIdx.x; i < n;
        i += (int64_t)gridDim.x * kThreads) {
     const size_t x = (size_t)(tab.off[s] + i);
-    const int m = (int)(i % M);
+    const int m = (int)((uint32_t)i % (uint32_t)M);
     const T z = div_rn(S[x], theta[(size_t)s * M + m]);
     if (Z) Z[x] = z;
     if (cls) {

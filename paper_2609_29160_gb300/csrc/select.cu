@@ -22,13 +22,30 @@
 namespace tre {
 namespace {
 
-constexpr int kWarpsPerBlock = 4;
 constexpr uint16_t kNoRank = 0xffff;
 
 __device__ __forceinline__ int64_t tick_window(int64_t j, int64_t cadence, int64_t win) {
   // window whose right edge passes the j-th multiple of the cadence (j >= 1)
   return (j * cadence + win - 1) / win - 1;
 }
+
+// successive multiples j*c of a cadence c as quotient and remainder of win
+struct TickSeq {
+  int32_t q, r, qc, rc, win;
+  __device__ __forceinline__ TickSeq(int32_t c, int32_t w) : win(w) {
+    qc = c / w;
+    rc = c - qc * w;
+    q = qc;
+    r = rc;
+  }
+  // window whose right edge passes the current multiple (windows end before 2^31 ms)
+  __device__ __forceinline__ int32_t window() const { return q + (r > 0) - 1; }
+  __device__ __forceinline__ void next() {
+    q += qc;
+    r += rc;
+    if (r >= win) { r -= win; q += 1; }
+  }
+};
 
 template <class T>
 __device__ __forceinline__ uint8_t region_of(uint8_t c, T z, T tc, T ts) {
@@ -42,7 +59,8 @@ __device__ __forceinline__ uint8_t region_of(uint8_t c, T z, T tc, T ts) {
 // are its fast ticks, [nf, nf + ns) its slow ticks.
 template <class T>
 __global__ void __launch_bounds__(256)
-k_tick_rank(const __grid_constant__ WalkBatch<T> b, int16_t* recv_out, uint16_t* rank) {
+k_tick_rank(const __grid_constant__ WalkBatch<T> b, int16_t* recv_out, int16_t* ndon_out,
+            uint16_t* rank, uint16_t* order) {
   const int M = b.M;
   const int64_t gid = (int64_t)blockIdx.x * 256 + threadIdx.x;
   const int64_t total_ent = (int64_t)b.ent_base[b.n_series] * b.n_tau;
@@ -107,7 +125,106 @@ k_tick_rank(const __grid_constant__ WalkBatch<T> b, int16_t* recv_out, uint16_t*
   }
   const size_t row = (size_t)b.ent_base[s] * b.n_tau + (size_t)ti * n_ent + j;
   rank[row * M + m] = r;
-  if (m == 0) recv_out[row] = (int16_t)(act ? recv : -1);
+  if (r != kNoRank) order[row * M + r] = (uint16_t)m;
+  if (m == 0) {
+    int nd = 0;
+    if (act)
+      for (int q = 0; q < M; ++q) nd += group(q, reg(q)) >= 0;
+    recv_out[row] = (int16_t)(act ? recv : -1);
+    ndon_out[row] = (int16_t)nd;
+  }
+}
+
+// One thread per (series, tau, tick entry) for M <= MMAX: the regions are
+// computed once per model and the ranks in registers.
+template <class T, int MMAX>
+__global__ void __launch_bounds__(128)
+k_tick_rank_small(const __grid_constant__ WalkBatch<T> b, int16_t* recv_out, int16_t* ndon_out,
+                  uint16_t* rank, uint16_t* order, unsigned long long* packed, uint32_t* dmask) {
+  const int M = b.M;
+  const int64_t e = (int64_t)blockIdx.x * 128 + threadIdx.x;
+  if (e >= (int64_t)b.ent_base[b.n_series] * b.n_tau) return;
+  int s = 0;
+  while (s + 1 < b.n_series && (int64_t)b.ent_base[s + 1] * b.n_tau <= e) ++s;
+  const int64_t local = e - (int64_t)b.ent_base[s] * b.n_tau;
+  const int n_ent = b.ent_base[s + 1] - b.ent_base[s];
+  const int ti = (int)(local / n_ent);
+  const int j = (int)(local % n_ent);
+  const int64_t win = b.series_win[s];
+  const int64_t K = b.series_K[s];
+  const int64_t nf = K * win / b.fast_ms;
+  const bool fast = j < nf;
+  const int64_t k =
+      fast ? tick_window(j + 1, b.fast_ms, win) : tick_window(j - nf + 1, b.slow_ms, win);
+  const T* Zk = b.Z + b.series_off[s] + (size_t)k * M;
+  const uint8_t* Ck = b.cls + b.series_off[s] + (size_t)k * M;
+  const bool tau_dev = b.tau_crit != nullptr;
+  const T tau_v = b.tau_list[tau_dev ? 0 : ti];
+  T z[MMAX];
+  uint8_t rg[MMAX];
+  int recv = -1;
+  T zr = (T)0;
+#pragma unroll
+  for (int q = 0; q < MMAX; ++q) {
+    z[q] = (T)0;
+    rg[q] = 0xff;
+    if (q < M) {
+      z[q] = Zk[q];
+      rg[q] = region_of(Ck[q], z[q], tau_dev ? b.tau_crit[q] : tau_v, b.tau_surp[q]);
+      const bool cand = fast ? rg[q] == kCrit : rg[q] != kIdle;
+      if (cand && (recv < 0 || z[q] < zr)) {
+        recv = q;
+        zr = z[q];
+      }
+    }
+  }
+  const bool act = recv >= 0 && (fast || zr < (T)1);
+  int grp[MMAX];
+  int nd = 0;
+#pragma unroll
+  for (int q = 0; q < MMAX; ++q) {
+    int g = -1;
+    if (act && q < M && q != recv && rg[q] != kCrit) {
+      if (rg[q] == kIdle) g = 0;
+      else if (rg[q] == kSurp) g = 1;
+      else if (fast || z[q] > zr) g = 2;       // rebalance: nominal donors above the receiver
+    }
+    grp[q] = g;
+    nd += g >= 0;
+  }
+  const size_t row = (size_t)b.ent_base[s] * b.n_tau + (size_t)ti * n_ent + j;
+  unsigned long long pk = 0;
+  uint32_t dm = 0;
+#pragma unroll
+  for (int m = 0; m < MMAX; ++m) {
+    if (m >= M) break;
+    uint16_t r = kNoRank;
+    if (grp[m] >= 0) {
+      int before = 0;
+#pragma unroll
+      for (int q = 0; q < MMAX; ++q) {
+        if (q >= M || q == m || grp[q] < 0) continue;
+        bool prec;
+        if (grp[q] != grp[m]) prec = grp[q] < grp[m];
+        else if (grp[q] == 0) prec = q < m;
+        else prec = z[q] > z[m] || (z[q] == z[m] && q < m);
+        before += prec;
+      }
+      r = (uint16_t)before;
+      order[row * M + r] = (uint16_t)m;
+      if (MMAX <= 16) {
+        pk |= (unsigned long long)m << (4 * before);
+        dm |= 1u << m;
+      }
+    }
+    rank[row * M + m] = r;
+  }
+  recv_out[row] = (int16_t)(act ? recv : -1);
+  ndon_out[row] = (int16_t)nd;
+  if (MMAX <= 16) {
+    packed[row] = pk;
+    dmask[row] = dm;
+  }
 }
 
 template <int MPL>
@@ -132,25 +249,53 @@ __device__ __forceinline__ int lane_of_min_rank(const uint16_t (&rk)[MPL], const
   return src;
 }
 
-template <class T, int MPL>
-__global__ void __launch_bounds__(kWarpsPerBlock * 32)
-k_walk(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab, const uint16_t* rank) {
-  const int inst = blockIdx.x * kWarpsPerBlock + threadIdx.x / 32;
-  if (inst >= b.n_inst) return;
+// One CTA per (series, tau), one warp per pacing cap: the warps share the
+// tick tables of their (series, tau), staged in shared memory when they fit.
+template <class T, int MPL, bool STAGED>
+__global__ void __launch_bounds__(kMaxCap * 32)
+k_walk(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab, const int16_t* ndon_tab,
+       const uint16_t* rank, const uint16_t* order) {
+  extern __shared__ __align__(16) unsigned char dyn[];
+  const int grp = blockIdx.x;                       // (series, tau)
+  const int ti = grp % b.n_tau;
+  const int si = grp / b.n_tau;
+  const int ci = threadIdx.x / 32;                  // pacing cap index
   const int lane = threadIdx.x & 31;
   const int M = b.M;
-  const int ci = inst % b.n_cap;
-  const int ti = (inst / b.n_cap) % b.n_tau;
-  const int si = inst / (b.n_cap * b.n_tau);
   const int K = b.series_K[si];
   const int64_t win = b.series_win[si];
-  const int Kp = b.cap_list[ci];
-  const int64_t cap = b.moves_cap;
-  tre_move* mv = b.moves + (size_t)inst * cap;
   const int n_ent = b.ent_base[si + 1] - b.ent_base[si];
   const size_t row0 = (size_t)b.ent_base[si] * b.n_tau + (size_t)ti * n_ent;
   const int16_t* rv_tab = recv_tab + row0;
+  const int16_t* nd_tab = ndon_tab + row0;
   const uint16_t* rk0 = rank + row0 * M;
+  const uint16_t* od0 = order + row0 * M;
+  if (STAGED) {
+    const size_t a2 = ((size_t)n_ent * 2 + 15) & ~(size_t)15;
+    const size_t am = ((size_t)n_ent * M * 2 + 15) & ~(size_t)15;
+    int16_t* srv = reinterpret_cast<int16_t*>(dyn);
+    int16_t* snd = reinterpret_cast<int16_t*>(dyn + a2);
+    uint16_t* srk = reinterpret_cast<uint16_t*>(dyn + 2 * a2);
+    uint16_t* sod = reinterpret_cast<uint16_t*>(dyn + 2 * a2 + am);
+    for (int i = threadIdx.x; i < n_ent; i += blockDim.x) {
+      srv[i] = rv_tab[i];
+      snd[i] = nd_tab[i];
+    }
+    for (int64_t i = threadIdx.x; i < (int64_t)n_ent * M; i += blockDim.x) {
+      srk[i] = rk0[i];
+      sod[i] = od0[i];
+    }
+    __syncthreads();
+    rv_tab = srv;
+    nd_tab = snd;
+    rk0 = srk;
+    od0 = sod;
+  }
+  if (ci >= b.n_cap) return;
+  const int inst = (si * b.n_tau + ti) * b.n_cap + ci;
+  const int Kp = b.cap_list[ci];
+  const int64_t cap = b.moves_cap;
+  tre_move* mv = b.moves + (size_t)inst * cap;
   const int64_t F = b.fast_ms, Sl = b.slow_ms;
   const int64_t nf = (int64_t)K * win / F;
 
@@ -185,18 +330,27 @@ k_walk(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab, const ui
     return;
   }
   int64_t nm = 0;
-  int64_t jf = 1, js = 1;
+  // With unit footprints and one model per lane a tick is closed form: pool
+  // draws first, then donors drain in rank order down to their floors.
+  bool unit = true;
+#pragma unroll
+  for (int j = 0; j < MPL; ++j)
+    if (lane + 32 * j < M && g[j] != 1) unit = false;
+  const bool closed = MPL == 1 && __all_sync(0xffffffffu, unit);
+  // tick windows without division: the j-th tick of a cadence c ends window
+  // ceil(j*c / win) - 1; keep j*c as quotient and remainder of win
+  TickSeq sf((int32_t)F, (int32_t)win), ss((int32_t)Sl, (int32_t)win);
+  int32_t jf = 1, js = 1;
   while (true) {
-    const int64_t kf = tick_window(jf, F, win);
-    const int64_t ks = tick_window(js, Sl, win);
-    const int64_t k = kf < ks ? kf : ks;
+    const int32_t kf = sf.window(), ks = ss.window();
+    const int32_t k = kf < ks ? kf : ks;
     if (k >= K) break;
     const bool fast = kf == k, slow = ks == k;
-    const int64_t ef = jf - 1, es = nf + js - 1;   // entries of this tick
-    while (tick_window(jf, F, win) <= k) ++jf;
-    while (tick_window(js, Sl, win) <= k) ++js;
+    const int32_t ef = jf - 1, es = (int32_t)nf + js - 1;   // entries of this tick
+    while (sf.window() <= k) { sf.next(); ++jf; }
+    while (ss.window() <= k) { ss.next(); ++js; }
     int recv = -1, kind = 0;
-    int64_t ent = -1;
+    int32_t ent = -1;
     if (fast) {
       const int rv = rv_tab[ef];
       if (rv >= 0) { recv = rv; ent = ef; kind = TRE_RESCUE; }
@@ -206,6 +360,41 @@ k_walk(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab, const ui
       if (rv >= 0) { recv = rv; ent = es; kind = TRE_REBALANCE; }
     }
     if (!kind) continue;
+    if (closed) {
+      const int nd = nd_tab[ent];
+      const int mo = lane < nd ? od0[(size_t)ent * M + lane] : -1;
+      const int r_src = __shfl_sync(0xffffffffu, r[0] - rmin[0], mo < 0 ? 0 : mo);
+      const int cap_p = mo < 0 ? 0 : (r_src > 0 ? r_src : 0);
+      int incl = cap_p;
+      for (int o = 1; o < 32; o <<= 1) {
+        const int x = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += x;
+      }
+      const int excl = incl - cap_p;
+      const int total_cap = __shfl_sync(0xffffffffu, incl, 31);
+      const int n_pool = (int)(free_pool < Kp ? free_pool : Kp);
+      const int t_d = min(Kp - n_pool, total_cap);
+      const int give = max(0, min(t_d - excl, cap_p));
+      // moves: pool draws take seq 0.., donors follow in rank order
+      for (int q = lane; q < n_pool; q += 32)
+        if (nm + q < cap)
+          mv[nm + q] = tre_move{(int32_t)k, (int16_t)recv, (int16_t)-1, (uint8_t)kind,
+                                (uint8_t)q, 0};
+      for (int i = 0; i < give; ++i) {
+        const int64_t q = n_pool + excl + i;
+        if (nm + q < cap)
+          mv[nm + q] = tre_move{(int32_t)k, (int16_t)recv, (int16_t)mo, (uint8_t)kind,
+                                (uint8_t)q, 0};
+      }
+      // my model's position in the donor order, then what it gave
+      const uint16_t my_rank = lane < M ? rk0[(size_t)ent * M + lane] : kNoRank;
+      const int given = __shfl_sync(0xffffffffu, give, my_rank == kNoRank ? 0 : (my_rank & 31));
+      if (my_rank != kNoRank) r[0] -= given;
+      if (lane == recv) r[0] += n_pool + t_d;
+      free_pool -= n_pool;
+      nm += n_pool + t_d;
+      continue;
+    }
     uint16_t rk[MPL];
 #pragma unroll
     for (int j = 0; j < MPL; ++j)
@@ -271,6 +460,207 @@ k_walk(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab, const ui
   }
 }
 
+// One thread per controller instance (M <= 16): the threads of a CTA are the
+// pacing caps of one (series, tau) and share its staged tick tables. A
+// transition draws on the idle pool if it covers the receiver's footprint,
+// else releases donor replicas in the tick's donor order (lowest rank first,
+// each down to its floor). The models still above their floors are a bit
+// mask in a register, so a tick whose donors are all at their floors costs one
+// AND; the donor order is a packed 4-bit list per tick.
+template <class T, int MMAX>
+__device__ __forceinline__ int sel(const int (&a)[MMAX], int m) {
+  int v = 0;
+#pragma unroll
+  for (int q = 0; q < MMAX; ++q) v = q == m ? a[q] : v;
+  return v;
+}
+template <class T, int MMAX>
+__device__ __forceinline__ void add_at(int (&a)[MMAX], int m, int d) {
+#pragma unroll
+  for (int q = 0; q < MMAX; ++q) a[q] += q == m ? d : 0;
+}
+
+template <class T, int MMAX>
+__global__ void __launch_bounds__(32)
+k_walk_thread(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
+              const unsigned long long* packed, const uint32_t* dmask) {
+  extern __shared__ __align__(16) unsigned char dyn[];
+  const int grp = blockIdx.x;
+  const int ti = grp % b.n_tau;
+  const int si = grp / b.n_tau;
+  const int M = b.M;
+  const int K = b.series_K[si];
+  const int32_t win = b.series_win[si];
+  const int n_ent = b.ent_base[si + 1] - b.ent_base[si];
+  const size_t row0 = (size_t)b.ent_base[si] * b.n_tau + (size_t)ti * n_ent;
+  unsigned long long* spk = reinterpret_cast<unsigned long long*>(dyn);
+  uint32_t* sdm = reinterpret_cast<uint32_t*>(spk + n_ent);
+  int16_t* srv = reinterpret_cast<int16_t*>(sdm + n_ent);
+  for (int i = threadIdx.x; i < n_ent; i += blockDim.x) {
+    spk[i] = packed[row0 + i];
+    sdm[i] = dmask[row0 + i];
+    srv[i] = recv_tab[row0 + i];
+  }
+  __syncthreads();
+  const int ci = threadIdx.x;
+  if (ci >= b.n_cap) return;
+  const int inst = (si * b.n_tau + ti) * b.n_cap + ci;
+  const int Kp = b.cap_list[ci];
+  const int64_t cap = b.moves_cap;
+  tre_move* mv = b.moves + (size_t)inst * cap;
+  const int32_t nf = (int32_t)((int64_t)K * win / b.fast_ms);
+  int r[MMAX], rmin[MMAX], g[MMAX];
+  int64_t used = 0;
+  bool bad = false, unit = true;
+  uint32_t avail = 0;                           // models above their floor
+#pragma unroll
+  for (int m = 0; m < MMAX; ++m) {
+    r[m] = 0;
+    rmin[m] = 0;
+    g[m] = 1;
+    if (m < M) {
+      r[m] = b.r0[m];
+      rmin[m] = b.r_min[m];
+      g[m] = b.footprint[m];
+      used += (int64_t)g[m] * r[m];
+      if (r[m] < 0 || rmin[m] < 0 || g[m] < 1) bad = true;
+      if (g[m] != 1) unit = false;
+      if (r[m] > rmin[m]) avail |= 1u << m;
+    }
+  }
+  int64_t free_pool = b.budget - used;
+  if (bad || free_pool < 0) {
+    for (int m = 0; m < M && m < MMAX; ++m) b.r_out[(size_t)inst * M + m] = sel<T, MMAX>(r, m);
+    b.n_moves[inst] = 0;
+    b.diag->err = TRE_EINVAL;
+    return;
+  }
+  auto emit = [&](int64_t at, int32_t k, int recv, int donor, int kind, int sq) {
+    if (at < cap) mv[at] = tre_move{k, (int16_t)recv, (int16_t)donor, (uint8_t)kind, (uint8_t)sq, 0};
+  };
+  int64_t nm = 0;
+  TickSeq sf(b.fast_ms, win), ss(b.slow_ms, win);
+  int32_t jf = 1, js = 1;
+  while (true) {
+    const int32_t kf = sf.window(), ks = ss.window();
+    const int32_t k = kf < ks ? kf : ks;
+    if (k >= K) break;
+    const bool fast = kf == k, slow = ks == k;
+    const int32_t ef = jf - 1, es = nf + js - 1;
+    while (sf.window() <= k) { sf.next(); ++jf; }
+    while (ss.window() <= k) { ss.next(); ++js; }
+    int recv = -1, kind = 0;
+    int32_t ent = -1;
+    if (fast) {
+      const int rv = srv[ef];
+      if (rv >= 0) { recv = rv; ent = ef; kind = TRE_RESCUE; }
+    }
+    if (!kind && slow) {
+      const int rv = srv[es];
+      if (rv >= 0) { recv = rv; ent = es; kind = TRE_REBALANCE; }
+    }
+    if (!kind) continue;
+    const uint32_t usable = avail & sdm[ent];
+    const int need = unit ? 1 : sel<T, MMAX>(g, recv);
+    if (free_pool < need && !usable) continue;        // nothing can move this tick
+    unsigned long long pk = spk[ent];
+    if (unit) {
+      const int n_pool = (int)(free_pool < Kp ? free_pool : Kp);
+      for (int q = 0; q < n_pool; ++q) emit(nm + q, k, recv, -1, kind, q);
+      int sq = n_pool;
+      uint32_t left = usable;
+      while (sq < Kp && left) {
+        int m = (int)(pk & 15);                      // next model in donor order
+        pk >>= 4;
+        if (!(left >> m & 1)) continue;
+        left &= ~(1u << m);
+        const int c = sel<T, MMAX>(r, m) - sel<T, MMAX>(rmin, m);
+        const int take = min(c, Kp - sq);
+        add_at<T, MMAX>(r, m, -take);
+        if (take == c) avail &= ~(1u << m);
+        for (int i = 0; i < take; ++i, ++sq) emit(nm + sq, k, recv, m, kind, sq);
+      }
+      add_at<T, MMAX>(r, recv, sq);
+      if (sel<T, MMAX>(r, recv) > sel<T, MMAX>(rmin, recv)) avail |= 1u << recv;
+      free_pool -= n_pool;
+      nm += sq;
+      continue;
+    }
+    for (int sq = 0; sq < Kp; ++sq) {
+      if (free_pool >= need) {
+        free_pool -= need;
+        add_at<T, MMAX>(r, recv, 1);
+        if (sel<T, MMAX>(r, recv) > sel<T, MMAX>(rmin, recv)) avail |= 1u << recv;
+        emit(nm++, k, recv, -1, kind, sq);
+        continue;
+      }
+      // plan the releases; an uncoverable transition releases nothing
+      int64_t f = free_pool;
+      const int64_t nm0 = nm;
+      int taken[MMAX];
+#pragma unroll
+      for (int m = 0; m < MMAX; ++m) taken[m] = 0;
+      unsigned long long order = pk;
+      uint32_t left = avail & sdm[ent];
+      while (f < need && left) {
+        const int m = (int)(order & 15);
+        order >>= 4;
+        if (!(left >> m & 1)) continue;
+        left &= ~(1u << m);
+        int c = sel<T, MMAX>(r, m) - sel<T, MMAX>(rmin, m);
+        const int gm = sel<T, MMAX>(g, m);
+        while (f < need && c > 0) {
+          add_at<T, MMAX>(taken, m, 1);
+          --c;
+          f += gm;
+          emit(nm++, k, recv, m, kind, sq);
+        }
+      }
+      if (f < need) {
+        nm = nm0;
+        break;
+      }
+#pragma unroll
+      for (int m = 0; m < MMAX; ++m) {
+        r[m] -= taken[m];
+        if (m < M && !(r[m] > rmin[m])) avail &= ~(1u << m);
+      }
+      add_at<T, MMAX>(r, recv, 1);
+      if (sel<T, MMAX>(r, recv) > sel<T, MMAX>(rmin, recv)) avail |= 1u << recv;
+      free_pool = f - need;
+    }
+  }
+  for (int m = 0; m < M && m < MMAX; ++m) b.r_out[(size_t)inst * M + m] = sel<T, MMAX>(r, m);
+  b.n_moves[inst] = nm;
+  if (nm > cap) b.diag->err = TRE_EOVERFLOW;
+}
+
+constexpr size_t kStageMax = 160 * 1024;
+
+template <class T, int MPL>
+cudaError_t walk_launch(const WalkBatch<T>& b, WalkWs& w, cudaStream_t s) {
+  int max_ent = 0;
+  for (int i = 0; i < b.n_series; ++i) max_ent = std::max(max_ent, b.ent_base[i + 1] - b.ent_base[i]);
+  const size_t smem = 2 * (((size_t)max_ent * 2 + 15) & ~(size_t)15) +
+                      2 * (((size_t)max_ent * b.M * 2 + 15) & ~(size_t)15);
+  const unsigned grid = (unsigned)(b.n_series * b.n_tau);
+  const unsigned th = (unsigned)(b.n_cap * 32);
+  if (smem <= kStageMax) {
+    static bool attr = false;
+    if (!attr) {
+      cudaError_t e = cudaFuncSetAttribute(k_walk<T, MPL, true>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)kStageMax);
+      if (e) return e;
+      attr = true;
+    }
+    k_walk<T, MPL, true><<<grid, th, smem, s>>>(b, w.recv, w.n_donor, w.rank, w.order);
+  } else {
+    k_walk<T, MPL, false><<<grid, th, 0, s>>>(b, w.recv, w.n_donor, w.rank, w.order);
+  }
+  return cudaGetLastError();
+}
+
 }  // namespace
 
 template <class T> void walk_ws_layout(Arena& a, WalkBatch<T>& b, WalkWs& w) {
@@ -282,26 +672,63 @@ template <class T> void walk_ws_layout(Arena& a, WalkBatch<T>& b, WalkWs& w) {
   }
   b.ent_base[b.n_series] = (int32_t)total;
   w.recv = a.take<int16_t>((size_t)std::max<int64_t>(total * b.n_tau, 1));
+  w.n_donor = a.take<int16_t>((size_t)std::max<int64_t>(total * b.n_tau, 1));
   w.rank = a.take<uint16_t>((size_t)std::max<int64_t>(total * b.n_tau * b.M, 1));
+  w.order = a.take<uint16_t>((size_t)std::max<int64_t>(total * b.n_tau * b.M, 1));
+  w.packed = a.take<unsigned long long>((size_t)std::max<int64_t>(total * b.n_tau, 1));
+  w.dmask = a.take<uint32_t>((size_t)std::max<int64_t>(total * b.n_tau, 1));
+}
+
+// unit footprints and few models: thread-per-instance walk with staged tables
+template <class T, int MMAX>
+cudaError_t walk_thread_launch(const WalkBatch<T>& b, WalkWs& w, size_t smem, cudaStream_t s) {
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e = cudaFuncSetAttribute(k_walk_thread<T, MMAX>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)kStageMax);
+    if (e) return e;
+    attr = true;
+  }
+  k_walk_thread<T, MMAX><<<b.n_series * b.n_tau, 32, smem, s>>>(b, w.recv, w.packed, w.dmask);
+  return cudaGetLastError();
 }
 
 template <class T> cudaError_t launch_walk(const WalkBatch<T>& b, WalkWs& w, cudaStream_t s) {
   if (b.n_inst == 0) return cudaSuccess;
   const int64_t ents = (int64_t)b.ent_base[b.n_series] * b.n_tau;
   if (ents > 0) {
-    const int64_t th = ents * b.M;
-    k_tick_rank<T><<<(unsigned)((th + 255) / 256), 256, 0, s>>>(b, w.recv, w.rank);
+    if (b.M <= 8) {
+      k_tick_rank_small<T, 8><<<(unsigned)((ents + 127) / 128), 128, 0, s>>>(
+          b, w.recv, w.n_donor, w.rank, w.order, w.packed, w.dmask);
+    } else if (b.M <= 16) {
+      k_tick_rank_small<T, 16><<<(unsigned)((ents + 127) / 128), 128, 0, s>>>(
+          b, w.recv, w.n_donor, w.rank, w.order, w.packed, w.dmask);
+    } else if (b.M <= 32) {
+      k_tick_rank_small<T, 32><<<(unsigned)((ents + 127) / 128), 128, 0, s>>>(
+          b, w.recv, w.n_donor, w.rank, w.order, w.packed, w.dmask);
+    } else {
+      const int64_t th = ents * b.M;
+      k_tick_rank<T><<<(unsigned)((th + 255) / 256), 256, 0, s>>>(b, w.recv, w.n_donor, w.rank,
+                                                                   w.order);
+    }
   }
-  const unsigned grid = (unsigned)((b.n_inst + kWarpsPerBlock - 1) / kWarpsPerBlock);
+  if (b.M <= 16 && b.n_cap <= 32) {
+    int max_ent = 0;
+    for (int i = 0; i < b.n_series; ++i)
+      max_ent = std::max(max_ent, b.ent_base[i + 1] - b.ent_base[i]);
+    const size_t smem = (size_t)max_ent * (8 + 4 + 2) + 16;
+    if (smem <= kStageMax)
+      return b.M <= 8 ? walk_thread_launch<T, 8>(b, w, smem, s)
+                      : walk_thread_launch<T, 16>(b, w, smem, s);
+  }
   const int mpl = (b.M + 31) / 32;
-  const unsigned th = kWarpsPerBlock * 32;
-  if (mpl <= 1) k_walk<T, 1><<<grid, th, 0, s>>>(b, w.recv, w.rank);
-  else if (mpl <= 2) k_walk<T, 2><<<grid, th, 0, s>>>(b, w.recv, w.rank);
-  else if (mpl <= 4) k_walk<T, 4><<<grid, th, 0, s>>>(b, w.recv, w.rank);
-  else if (mpl <= 8) k_walk<T, 8><<<grid, th, 0, s>>>(b, w.recv, w.rank);
-  else if (mpl <= 16) k_walk<T, 16><<<grid, th, 0, s>>>(b, w.recv, w.rank);
-  else k_walk<T, 32><<<grid, th, 0, s>>>(b, w.recv, w.rank);
-  return cudaGetLastError();
+  if (mpl <= 1) return walk_launch<T, 1>(b, w, s);
+  if (mpl <= 2) return walk_launch<T, 2>(b, w, s);
+  if (mpl <= 4) return walk_launch<T, 4>(b, w, s);
+  if (mpl <= 8) return walk_launch<T, 8>(b, w, s);
+  if (mpl <= 16) return walk_launch<T, 16>(b, w, s);
+  return walk_launch<T, 32>(b, w, s);
 }
 
 template void walk_ws_layout<float>(Arena&, WalkBatch<float>&, WalkWs&);
