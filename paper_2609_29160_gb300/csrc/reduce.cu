@@ -17,7 +17,7 @@ namespace tre {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kStageBytes = 24 * 1024;   // staged rows per CTA: 8 CTAs of 256 threads per SM
+constexpr int kStageBytes = 32 * 1024;   // start-side staging per CTA
 constexpr int kSpill = 32;  // staged rows beyond the CTA's arrival range
 
 // window of a millisecond time (int32 range), clamped to [0, K]
@@ -47,12 +47,29 @@ struct ReqBatch {
   int32_t cta_base[kMaxTraces + 1];
 };
 
+// Targets of one record fall in two places: the arrival side (the waiting
+// gauge's +1 and the SLO counts at the arrival window) moves with the arrival
+// order of the records, the start side (waiting -1 and running +1 at the
+// start, prompt and decode tokens, running -1 at the end) with each model's
+// FCFS start order. A CTA stages the arrival side over the windows its records
+// arrive in, and the start side per model over a run of windows beginning at
+// that model's earliest start among the CTA's records. Targets outside both
+// go to global atomics.
+struct Stage {
+  int32_t *aW;                  // arrival side: [near_rows][M]
+  unsigned long long* aS;       // arrival side SLO counts: [near_rows][M]
+  int32_t *fP, *fD, *fA, *fW;   // start side: [M][far_rows]
+  int32_t* far_lo;              // [M]
+  int32_t* slo_lim;             // [M]
+};
+
 template <bool SLO>
 __global__ void __launch_bounds__(kThreads)
-k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int win, FastDiv fd, int K, int rows,
-                  int32_t* __restrict__ P0, int32_t* __restrict__ D0, int32_t* __restrict__ dA0,
-                  int32_t* __restrict__ dW0, unsigned long long* __restrict__ slo0,
-                  const int32_t* __restrict__ slo_ms, tre_diag* diag) {
+k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int win, FastDiv fd, int K,
+                  int near_rows, int far_rows, int32_t* __restrict__ P0, int32_t* __restrict__ D0,
+                  int32_t* __restrict__ dA0, int32_t* __restrict__ dW0,
+                  unsigned long long* __restrict__ slo0, const int32_t* __restrict__ slo_ms,
+                  tre_diag* diag) {
   extern __shared__ unsigned long long smem[];
   int t = 0;
   while (t + 1 < bt.n && bt.cta_base[t + 1] <= (int)blockIdx.x) ++t;
@@ -70,22 +87,52 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int win, FastDiv f
   const int64_t span = (int64_t)K * win;
   const int64_t k_lo = win_clamp(r.t_arr[i0], fd, K);
   const int64_t k_hi = win_clamp(r.t_arr[i1 - 1], fd, K);
-  const int64_t need = (k_hi >= k_lo ? k_hi - k_lo + 1 : 1) + kSpill;
-  const int used = (int)min64(rows, need);
-  const int cells = used * M;
-  unsigned long long* sS = smem;
-  int32_t* sP = reinterpret_cast<int32_t*>(smem + (SLO ? (size_t)rows * M : 0));
-  int32_t* sD = sP + (size_t)rows * M;
-  int32_t* sA = sD + (size_t)rows * M;
-  int32_t* sW = sA + (size_t)rows * M;
-  for (int c = threadIdx.x; c < cells; c += kThreads) {
-    sP[c] = 0; sD[c] = 0; sA[c] = 0; sW[c] = 0;
-    if (SLO) sS[c] = 0;
+  const int64_t need = (k_hi >= k_lo ? k_hi - k_lo + 1 : 1) + 1;
+  const int used = (int)min64(near_rows, need);
+  Stage st;
+  st.aS = smem;
+  st.aW = reinterpret_cast<int32_t*>(smem + (SLO ? (size_t)near_rows * M : 0));
+  st.fP = st.aW + (size_t)near_rows * M;
+  st.fD = st.fP + (size_t)far_rows * M;
+  st.fA = st.fD + (size_t)far_rows * M;
+  st.fW = st.fA + (size_t)far_rows * M;
+  st.far_lo = st.fW + (size_t)far_rows * M;
+  st.slo_lim = st.far_lo + M;
+  const int ncell = used * M, fcell = far_rows * M;
+  for (int c = threadIdx.x; c < ncell; c += kThreads) {
+    st.aW[c] = 0;
+    if (SLO) st.aS[c] = 0;
+  }
+  for (int c = threadIdx.x; c < fcell; c += kThreads) {
+    st.fP[c] = 0; st.fD[c] = 0; st.fA[c] = 0; st.fW[c] = 0;
+  }
+  for (int m = threadIdx.x; m < M; m += kThreads) {
+    st.far_lo[m] = 0x7fffffff;
+    if (SLO) st.slo_lim[m] = slo_ms[m];
+  }
+  __syncthreads();
+  // each model's earliest start window among this CTA's records
+  for (int64_t i = i0 + threadIdx.x; i < i1; i += kThreads) {
+    const int m = r.model[i];
+    const int32_t ts = r.t_start[i];
+    if (m >= 0 && m < M && ts >= 0) atomicMin(&st.far_lo[m], (int32_t)win_clamp(ts, fd, K));
   }
   __syncthreads();
 
+  // arrival-side target (waiting +1, SLO counts)
+  auto near_add = [&](auto* s_arr, auto* g_arr, int64_t k, int m, auto v) {
+    const int64_t rel = k - k_lo;
+    if (rel >= 0 && rel < used) atomicAdd(&s_arr[rel * M + m], v);
+    else atomicAdd(&g_arr[k * M + m], v);
+  };
+  // start-side target of model m
+  auto far_add = [&](int32_t* s_arr, int32_t* g_arr, int64_t k, int m, int32_t v) {
+    const int64_t rel = k - st.far_lo[m];
+    if (rel >= 0 && rel < far_rows) atomicAdd(&s_arr[m * far_rows + rel], v);
+    else atomicAdd(&g_arr[k * M + m], v);
+  };
+
   unsigned long long n_range = 0, n_model = 0, n_order = 0;
-  // the next record's columns are loaded while the current one is processed
   int32_t nx[7];
   auto load_rec = [&](int64_t i) {
     if (i < i1) {
@@ -108,67 +155,84 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int win, FastDiv f
     if (ta < 0 || ta >= span) { ++n_range; continue; }
     if (!(ta <= ts && ts <= tf && tf <= te) || L_in < 0 || L < 1) { ++n_order; continue; }
 
+    const int64_t ba = fd.div((uint32_t)ta);
+    const int64_t bs = win_clamp(ts, fd, K), be = win_clamp(te, fd, K);
+    if (ba != bs) {
+      near_add(st.aW, dW, ba, m, (int32_t)1);
+      far_add(st.fW, dW, bs, m, -1);
+    }
+    if (bs != be) {
+      far_add(st.fA, dA, bs, m, 1);
+      far_add(st.fA, dA, be, m, -1);
+    }
+    if (SLO) {
+      const unsigned long long met = (tf - ta <= (int64_t)st.slo_lim[m]) ? 1ull : 0ull;
+      near_add(st.aS, slo, ba, m, 1ull + (met << 32));
+    }
     if (tf < span) {
       const int64_t kf = fd.div((uint32_t)tf);
       // prompt tokens, all at the first-token time
-      if (L_in) stage_add<int32_t>(sP, P, kf, k_lo, used, M, m, L_in);
+      if (L_in) far_add(st.fP, P, kf, m, L_in);
       // decode tokens: N(T) = tokens emitted before T; D[k] = N((k+1)w) - N(kw)
       const int64_t ke_raw = fd.div((uint32_t)te);
       if (L == 1 || ke_raw == kf) {
-        stage_add<int32_t>(sD, D, kf, k_lo, used, M, m, L);
+        far_add(st.fD, D, kf, m, L);
       } else {
         const unsigned long long dur = (unsigned long long)(te - tf);
         const unsigned long long Lm1 = (unsigned long long)(L - 1);
-        const int64_t ke = min64(ke_raw, K - 1);
-        // N(T) = ceil((T - tf) * (L-1) / dur) for tf < T <= te, stepped by whole windows
-        unsigned long long q, rem, qs, rs;
+        unsigned long long q, rem;
+        // N at the first window boundary after tf: ceil((T - tf)(L-1)/dur)
         divmod((unsigned long long)((kf + 1) * win - tf) * Lm1, (uint32_t)dur, q, rem);
-        divmod((unsigned long long)win * Lm1, (uint32_t)dur, qs, rs);
-        unsigned long long prevN = 0;
-        for (int64_t k = kf; k <= ke; ++k) {
-          unsigned long long N;
-          if ((k + 1) * win > te) {
-            N = (unsigned long long)L;
-          } else {
-            N = q + (rem != 0);
-            q += qs;
-            rem += rs;
-            if (rem >= dur) { rem -= dur; q += 1; }
+        const int32_t n1 = (int32_t)(q + (rem != 0));
+        far_add(st.fD, D, kf, m, n1);
+        if (ke_raw == kf + 1) {
+          if (kf + 1 < K) far_add(st.fD, D, kf + 1, m, L - n1);
+        } else {
+          const int64_t ke = min64(ke_raw, K - 1);
+          unsigned long long qs, rs;
+          divmod((unsigned long long)win * Lm1, (uint32_t)dur, qs, rs);
+          q += qs;
+          rem += rs;
+          if (rem >= dur) { rem -= dur; q += 1; }
+          unsigned long long prevN = (unsigned long long)n1;
+          for (int64_t k = kf + 1; k <= ke; ++k) {
+            unsigned long long N;
+            if ((k + 1) * win > te) {
+              N = (unsigned long long)L;
+            } else {
+              N = q + (rem != 0);
+              q += qs;
+              rem += rs;
+              if (rem >= dur) { rem -= dur; q += 1; }
+            }
+            const int32_t cnt = (int32_t)(N - prevN);
+            if (cnt) far_add(st.fD, D, k, m, cnt);
+            prevN = N;
           }
-          const int32_t cnt = (int32_t)(N - prevN);
-          if (cnt) stage_add<int32_t>(sD, D, k, k_lo, used, M, m, cnt);
-          prevN = N;
         }
       }
     }
-    // gauges: +1 where the state begins, -1 where it ends
-    const int64_t ba = win_clamp(ta, fd, K), bs = win_clamp(ts, fd, K), be = win_clamp(te, fd, K);
-    if (ba != bs) {
-      stage_add<int32_t>(sW, dW, ba, k_lo, used, M, m, 1);
-      stage_add<int32_t>(sW, dW, bs, k_lo, used, M, m, -1);
-    }
-    if (bs != be) {
-      stage_add<int32_t>(sA, dA, bs, k_lo, used, M, m, 1);
-      stage_add<int32_t>(sA, dA, be, k_lo, used, M, m, -1);
-    }
-    if (SLO) {
-      const unsigned long long met = (tf - ta <= (int64_t)slo_ms[m]) ? 1ull : 0ull;
-      stage_add<unsigned long long>(sS, slo, ba, k_lo, used, M, m, 1ull + (met << 32));
-    }
   }
   __syncthreads();
-  for (int c = threadIdx.x; c < cells; c += kThreads) {
+  for (int c = threadIdx.x; c < ncell; c += kThreads) {
     const int64_t k = k_lo + c / M;
-    const int m = c % M;
+    const size_t g = (size_t)k * M + (c % M);
+    if (k < K && SLO && st.aS[c]) atomicAdd(&slo[g], st.aS[c]);
+    if (k <= K && st.aW[c]) atomicAdd(&dW[g], st.aW[c]);
+  }
+  for (int c = threadIdx.x; c < fcell; c += kThreads) {
+    const int m = c / far_rows;
+    const int lo = st.far_lo[m];
+    if (lo == 0x7fffffff) continue;
+    const int64_t k = (int64_t)lo + (c % far_rows);
     const size_t g = (size_t)k * M + m;
     if (k < K) {
-      if (sP[c]) atomicAdd(&P[g], sP[c]);
-      if (sD[c]) atomicAdd(&D[g], sD[c]);
-      if (SLO && sS[c]) atomicAdd(&slo[g], sS[c]);
+      if (st.fP[c]) atomicAdd(&P[g], st.fP[c]);
+      if (st.fD[c]) atomicAdd(&D[g], st.fD[c]);
     }
     if (k <= K) {
-      if (sA[c]) atomicAdd(&dA[g], sA[c]);
-      if (sW[c]) atomicAdd(&dW[g], sW[c]);
+      if (st.fA[c]) atomicAdd(&dA[g], st.fA[c]);
+      if (st.fW[c]) atomicAdd(&dW[g], st.fW[c]);
     }
   }
   warp_add_counter(&diag->dropped_range, n_range);
@@ -525,15 +589,34 @@ cudaError_t launch_reduce_requests(const ReqCols* traces, int n_traces, int M, i
   }
   bt.cta_base[n_traces] = ctas;
   if (ctas == 0) return cudaSuccess;
-  const int cell_bytes = 16 + (slo ? 8 : 0);
-  const int rows = std::max(1, kStageBytes / (cell_bytes * M));
-  const size_t smem = (size_t)rows * M * cell_bytes;
+  // arrival-side rows cover the CTA's arrival span; start-side rows per model
+  const int64_t per = bt.per_cta[0];
+  const int64_t near_cap = 48 * 1024 / ((4 + (slo ? 8 : 0)) * M);   // arrival-stage budget
+  const int near_rows = (int)std::max<int64_t>(
+      1, std::min<int64_t>(near_cap,
+                           (int64_t)(3.0 * per / std::max<int64_t>(total_n / n_traces, 1) * K) +
+                               34));   // 3x the mean arrival span
+  const int far_rows = std::max(8, std::min(512, (int)(kStageBytes / (16 * M))));
+  const size_t smem = (size_t)near_rows * M * (4 + (slo ? 8 : 0)) + (size_t)far_rows * M * 16 +
+                      (size_t)M * 8;
+  if (smem > 200 * 1024) return cudaErrorInvalidValue;
+  static bool attr = false;
+  if (!attr) {
+    cudaError_t e1 = cudaFuncSetAttribute(k_reduce_requests<true>,
+                                          cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+    cudaError_t e2 = cudaFuncSetAttribute(k_reduce_requests<false>,
+                                          cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+    if (e1 || e2) return e1 ? e1 : e2;
+    attr = true;
+  }
   if (slo)
-    k_reduce_requests<true><<<ctas, kThreads, smem, s>>>(bt, M, win, FastDiv(win), K, rows, P, D,
-                                                         w.dA, w.dW, slo, slo_ms, diag);
+    k_reduce_requests<true><<<ctas, kThreads, smem, s>>>(bt, M, win, FastDiv(win), K, near_rows,
+                                                         far_rows, P, D, w.dA, w.dW, slo, slo_ms,
+                                                         diag);
   else
-    k_reduce_requests<false><<<ctas, kThreads, smem, s>>>(bt, M, win, FastDiv(win), K, rows, P, D,
-                                                          w.dA, w.dW, nullptr, nullptr, diag);
+    k_reduce_requests<false><<<ctas, kThreads, smem, s>>>(bt, M, win, FastDiv(win), K, near_rows,
+                                                          far_rows, P, D, w.dA, w.dW, nullptr,
+                                                          nullptr, diag);
   return cudaGetLastError();
 }
 

@@ -635,6 +635,202 @@ k_walk_thread(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
   if (nm > cap) b.diag->err = TRE_EOVERFLOW;
 }
 
+// Jumping walk for nested cadences (slow_ms a multiple of fast_ms, so every
+// slow tick is a fast tick): the action of each tick (rescue entry, else
+// rebalance entry, else none) does not depend on the replica state, and the
+// state changes only when something moves. A tick can move something only if
+// the idle pool is non-empty or a model above its floor is a donor there; per
+// model, the next tick where it is a donor is precomputed, so the walk jumps
+// from one possible move to the next instead of visiting every tick.
+template <class T, int MMAX>
+__global__ void __launch_bounds__(32)
+k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
+            const unsigned long long* packed, const uint32_t* dmask) {
+  extern __shared__ __align__(16) unsigned char dyn[];
+  const int grp = blockIdx.x;
+  const int ti = grp % b.n_tau;
+  const int si = grp / b.n_tau;
+  const int M = b.M;
+  const int K = b.series_K[si];
+  const int64_t win = b.series_win[si];
+  const int n_ent = b.ent_base[si + 1] - b.ent_base[si];
+  const size_t row0 = (size_t)b.ent_base[si] * b.n_tau + (size_t)ti * n_ent;
+  const int nf = (int)((int64_t)K * win / b.fast_ms);   // fast ticks = all ticks
+  const int ratio = b.slow_ms / b.fast_ms;
+  // shared layout: per tick u < nf: action entry, kind, window; per entry:
+  // packed order and donor mask; per (model + any, tick): next acting tick
+  unsigned long long* spk = reinterpret_cast<unsigned long long*>(dyn);
+  uint32_t* sdm = reinterpret_cast<uint32_t*>(spk + n_ent);
+  int32_t* swin = reinterpret_cast<int32_t*>(sdm + n_ent);
+  int16_t* sent = reinterpret_cast<int16_t*>(swin + nf);
+  int16_t* srcv = sent + nf;
+  uint8_t* skind = reinterpret_cast<uint8_t*>(srcv + nf);
+  int16_t* snxt = reinterpret_cast<int16_t*>(skind + ((nf + 15) & ~15));  // [M + 1][nf + 1]
+  for (int i = threadIdx.x; i < n_ent; i += blockDim.x) {
+    spk[i] = packed[row0 + i];
+    sdm[i] = dmask[row0 + i];
+  }
+  for (int u = threadIdx.x; u < nf; u += blockDim.x) {
+    const int rf = recv_tab[row0 + u];
+    int e = -1, kd = 0, rv = -1;
+    if (rf >= 0) {
+      e = u; kd = TRE_RESCUE; rv = rf;
+    } else if ((u + 1) % ratio == 0) {
+      const int es = nf + (u + 1) / ratio - 1;
+      const int rs = recv_tab[row0 + es];
+      if (rs >= 0) { e = es; kd = TRE_REBALANCE; rv = rs; }
+    }
+    sent[u] = (int16_t)e;
+    srcv[u] = (int16_t)rv;
+    skind[u] = (uint8_t)kd;
+    swin[u] = (int32_t)tick_window(u + 1, b.fast_ms, win);
+  }
+  __syncthreads();
+  // next tick (>= u) where model m is a donor, and (row M) where any action is
+  for (int m = threadIdx.x; m <= M; m += blockDim.x) {
+    int16_t* col = snxt + (size_t)m * (nf + 1);
+    int nx = nf;
+    col[nf] = (int16_t)nf;
+    for (int u = nf - 1; u >= 0; --u) {
+      const int e = sent[u];
+      if (e >= 0 && (m == M || (sdm[e] >> m & 1))) nx = u;
+      col[u] = (int16_t)nx;
+    }
+  }
+  __syncthreads();
+  const int ci = threadIdx.x;
+  if (ci >= b.n_cap) return;
+  const int inst = (si * b.n_tau + ti) * b.n_cap + ci;
+  const int Kp = b.cap_list[ci];
+  const int64_t cap = b.moves_cap;
+  tre_move* mv = b.moves + (size_t)inst * cap;
+  int r[MMAX], rmin[MMAX], g[MMAX];
+  int64_t used = 0;
+  bool bad = false, unit = true;
+  uint32_t avail = 0;
+#pragma unroll
+  for (int m = 0; m < MMAX; ++m) {
+    r[m] = 0;
+    rmin[m] = 0;
+    g[m] = 1;
+    if (m < M) {
+      r[m] = b.r0[m];
+      rmin[m] = b.r_min[m];
+      g[m] = b.footprint[m];
+      used += (int64_t)g[m] * r[m];
+      if (r[m] < 0 || rmin[m] < 0 || g[m] < 1) bad = true;
+      if (g[m] != 1) unit = false;
+      if (r[m] > rmin[m]) avail |= 1u << m;
+    }
+  }
+  int64_t free_pool = b.budget - used;
+  if (bad || free_pool < 0) {
+    for (int m = 0; m < M && m < MMAX; ++m) b.r_out[(size_t)inst * M + m] = sel<T, MMAX>(r, m);
+    b.n_moves[inst] = 0;
+    b.diag->err = TRE_EINVAL;
+    return;
+  }
+  auto emit = [&](int64_t at, int32_t k, int recv, int donor, int kind, int sq) {
+    if (at < cap) mv[at] = tre_move{k, (int16_t)recv, (int16_t)donor, (uint8_t)kind, (uint8_t)sq, 0};
+  };
+  int64_t nm = 0;
+  int u = 0;
+  while (u < nf) {
+    // the next tick where something may move
+    int nxt;
+    if (free_pool > 0) {
+      nxt = snxt[(size_t)M * (nf + 1) + u];
+    } else {
+      nxt = nf;
+      uint32_t a = avail;
+      while (a) {
+        const int m = __ffs(a) - 1;
+        a &= a - 1;
+        nxt = min(nxt, (int)snxt[(size_t)m * (nf + 1) + u]);
+      }
+    }
+    if (nxt >= nf) break;
+    u = nxt;
+    const int ent = sent[u];
+    const int recv = srcv[u];
+    const int kind = skind[u];
+    const int32_t k = swin[u];
+    ++u;
+    if (ent < 0) continue;
+    const uint32_t usable = avail & sdm[ent];
+    const int need = unit ? 1 : sel<T, MMAX>(g, recv);
+    if (free_pool < need && !usable) continue;
+    unsigned long long pk = spk[ent];
+    if (unit) {
+      const int n_pool = (int)(free_pool < Kp ? free_pool : Kp);
+      for (int q = 0; q < n_pool; ++q) emit(nm + q, k, recv, -1, kind, q);
+      int sq = n_pool;
+      uint32_t left = usable;
+      while (sq < Kp && left) {
+        const int m = (int)(pk & 15);
+        pk >>= 4;
+        if (!(left >> m & 1)) continue;
+        left &= ~(1u << m);
+        const int c = sel<T, MMAX>(r, m) - sel<T, MMAX>(rmin, m);
+        const int take = min(c, Kp - sq);
+        add_at<T, MMAX>(r, m, -take);
+        if (take == c) avail &= ~(1u << m);
+        for (int i = 0; i < take; ++i, ++sq) emit(nm + sq, k, recv, m, kind, sq);
+      }
+      add_at<T, MMAX>(r, recv, sq);
+      if (sel<T, MMAX>(r, recv) > sel<T, MMAX>(rmin, recv)) avail |= 1u << recv;
+      free_pool -= n_pool;
+      nm += sq;
+      continue;
+    }
+    for (int sq = 0; sq < Kp; ++sq) {
+      if (free_pool >= need) {
+        free_pool -= need;
+        add_at<T, MMAX>(r, recv, 1);
+        if (sel<T, MMAX>(r, recv) > sel<T, MMAX>(rmin, recv)) avail |= 1u << recv;
+        emit(nm++, k, recv, -1, kind, sq);
+        continue;
+      }
+      int64_t f = free_pool;
+      const int64_t nm0 = nm;
+      int taken[MMAX];
+#pragma unroll
+      for (int m = 0; m < MMAX; ++m) taken[m] = 0;
+      unsigned long long order = pk;
+      uint32_t left = avail & sdm[ent];
+      while (f < need && left) {
+        const int m = (int)(order & 15);
+        order >>= 4;
+        if (!(left >> m & 1)) continue;
+        left &= ~(1u << m);
+        int c = sel<T, MMAX>(r, m) - sel<T, MMAX>(rmin, m);
+        const int gm = sel<T, MMAX>(g, m);
+        while (f < need && c > 0) {
+          add_at<T, MMAX>(taken, m, 1);
+          --c;
+          f += gm;
+          emit(nm++, k, recv, m, kind, sq);
+        }
+      }
+      if (f < need) {
+        nm = nm0;
+        break;
+      }
+#pragma unroll
+      for (int m = 0; m < MMAX; ++m) {
+        r[m] -= taken[m];
+        if (m < M && !(r[m] > rmin[m])) avail &= ~(1u << m);
+      }
+      add_at<T, MMAX>(r, recv, 1);
+      if (sel<T, MMAX>(r, recv) > sel<T, MMAX>(rmin, recv)) avail |= 1u << recv;
+      free_pool = f - need;
+    }
+  }
+  for (int m = 0; m < M && m < MMAX; ++m) b.r_out[(size_t)inst * M + m] = sel<T, MMAX>(r, m);
+  b.n_moves[inst] = nm;
+  if (nm > cap) b.diag->err = TRE_EOVERFLOW;
+}
+
 constexpr size_t kStageMax = 160 * 1024;
 
 template <class T, int MPL>
@@ -687,8 +883,30 @@ cudaError_t walk_thread_launch(const WalkBatch<T>& b, WalkWs& w, size_t smem, cu
     cudaError_t e = cudaFuncSetAttribute(k_walk_thread<T, MMAX>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)kStageMax);
-    if (e) return e;
+    cudaError_t e2 = cudaFuncSetAttribute(k_walk_jump<T, MMAX>,
+                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          (int)kStageMax);
+    if (e || e2) return e ? e : e2;
     attr = true;
+  }
+  // nested cadences with a fast tick not shorter than a window: jump between
+  // possible moves
+  if (b.slow_ms % b.fast_ms == 0 && b.fast_ms >= b.series_win[0]) {
+    bool ok = true;
+    size_t jsmem = 0;
+    for (int i = 0; i < b.n_series; ++i) {
+      if (b.fast_ms < b.series_win[i]) ok = false;
+      const int n_ent = b.ent_base[i + 1] - b.ent_base[i];
+      const int64_t nf = (int64_t)b.series_K[i] * b.series_win[i] / b.fast_ms;
+      if (nf >= 32767) ok = false;
+      const size_t need = (size_t)n_ent * 12 + (size_t)nf * (4 + 2 + 2) + ((nf + 15) & ~15) +
+                          (size_t)(b.M + 1) * (nf + 1) * 2 + 64;
+      jsmem = std::max(jsmem, need);
+    }
+    if (ok && jsmem <= kStageMax) {
+      k_walk_jump<T, MMAX><<<b.n_series * b.n_tau, 32, jsmem, s>>>(b, w.recv, w.packed, w.dmask);
+      return cudaGetLastError();
+    }
   }
   k_walk_thread<T, MMAX><<<b.n_series * b.n_tau, 32, smem, s>>>(b, w.recv, w.packed, w.dmask);
   return cudaGetLastError();
