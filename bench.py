@@ -222,16 +222,17 @@ def main():
     dev_traces = [{k: torch.as_tensor(v).cuda() for k, v in t.items()} for t in sw["traces"]]
     stream = torch.cuda.current_stream()
 
-    def step(traces, ws=None):
-        return tre.tre_sweep(traces, M, sw["duration_ms"], win, al, sw["tau_crit"],
-                             sw["pacing_cap"], sw["w_p"], sw["w_q"], sw["tau_surplus"],
-                             sw["slo_ttft_ms"], sw["budget"], sw["r0"], sw["r_min"],
-                             sw["footprint"], dtype="f32", moves_cap=moves_cap, ws=ws)
+    # the call is marshalled once; each step is one tre_sweep call on the stream
+    plan = tre.SweepPlan(dev_traces, M, sw["duration_ms"], win, al, sw["tau_crit"],
+                         sw["pacing_cap"], sw["w_p"], sw["w_q"], sw["tau_surplus"],
+                         sw["slo_ttft_ms"], sw["budget"], sw["r0"], sw["r_min"], sw["footprint"],
+                         dtype="f32", moves_cap=moves_cap)
 
-    out = step(dev_traces)
-    ws = out["ws"]
+    def step(traces=None, ws=None):
+        return plan.run(stream)
+
     for _ in range(args.warmup):
-        out = step(dev_traces, ws)
+        out = step()
     torch.cuda.synchronize()
 
     clocks = ClockSampler(local)
@@ -245,7 +246,7 @@ def main():
     clocks.mark(True)
     ev0.record(stream)
     for _ in range(args.steps):
-        out = step(dev_traces, ws)
+        out = step()
     ev1.record(stream)
     torch.cuda.synchronize()
     clocks.mark(False)
@@ -308,7 +309,7 @@ def main():
         for d, h in zip(dev_traces, host):
             for k in d:
                 d[k].copy_(h[k], non_blocking=True)
-        o = step(dev_traces, ws)
+        o = step()
         for k in res_host:
             res_host[k].copy_(o[k], non_blocking=True)
     e1.record(stream)

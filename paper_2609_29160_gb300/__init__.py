@@ -310,63 +310,88 @@ def tre_select_moves(Z, cls, profile, window_ms, budget, r0, r_min, footprint, f
     return mv, r, n, diag
 
 
+class SweepPlan:
+    """A tre_sweep call marshalled once: device parameter arrays, output
+    buffers, workspace and the C structs are built here, and run() issues the
+    one C call on a stream with no further host work. `traces`: list of dicts
+    of int32 CUDA tensors (kept referenced by the plan)."""
+
+    def __init__(self, traces, M, duration_ms, window_ms, alpha, tau_crit, pacing_cap, w_p, w_q,
+                 tau_surplus, slo_ttft_ms, budget, r0, r_min, footprint, fast_ms=5000,
+                 slow_ms=10000, dtype="f32", ok_frac=0.95, reliability=0.95, moves_cap=256,
+                 want_counts=False, want_S=False, diag=None, ws=None):
+        torch = _torch()
+        self.lib = load()
+        code, tdt = _dt(dtype)
+        win = np.asarray(window_ms, np.int32)
+        n_series = len(traces) * len(win)
+        self.K = [duration_ms // int(w) for w in win]
+        total = sum(self.K[i % len(win)] * M for i in range(n_series))
+        n_inst = n_series * len(tau_crit) * len(pacing_cap)
+        f = lambda v: torch.as_tensor(np.broadcast_to(np.asarray(v), (M,)).copy()).to(
+            device="cuda", dtype=tdt)
+        i32 = lambda v: torch.as_tensor(np.asarray(v, np.int32)).cuda()
+        k = {"w_p": f(w_p), "w_q": f(w_q), "ts": f(tau_surplus), "slo": i32(slo_ttft_ms),
+             "r0": i32(r0), "rmin": i32(r_min), "fp": i32(footprint)}
+        out = {"theta": torch.empty((n_series, M), dtype=tdt, device="cuda"),
+               "Z": torch.empty(total, dtype=tdt, device="cuda"),
+               "cls": torch.empty(total, dtype=torch.uint8, device="cuda"),
+               "moves": torch.zeros(n_inst * max(moves_cap, 1) * MOVE_DTYPE.itemsize,
+                                    dtype=torch.uint8, device="cuda"),
+               "n_moves": torch.zeros(n_inst, dtype=torch.int64, device="cuda"),
+               "r_final": torch.empty((n_inst, M), dtype=torch.int32, device="cuda")}
+        if want_counts:
+            for c in "PDAW":
+                out[c] = torch.empty(total, dtype=torch.int32, device="cuda")
+        if want_S:
+            out["S"] = torch.empty(total, dtype=tdt, device="cuda")
+        self._tr = (Requests * len(traces))(*[requests_struct(t) for t in traces])
+        self._wins = (C.c_int32 * len(win))(*[int(x) for x in win])
+        self._alph = (C.c_double * len(win))(*[float(a) for a in alpha])
+        self._taus = (C.c_double * len(tau_crit))(*[float(t) for t in tau_crit])
+        self._caps = (C.c_int32 * len(pacing_cap))(*[int(c) for c in pacing_cap])
+        ctrl = Ctrl(int(budget), k["rmin"].data_ptr(), k["fp"].data_ptr(), fast_ms, slow_ms, 0)
+        self.spec = SweepSpec(M, duration_ms, len(traces), self._tr, len(win), self._wins,
+                              self._alph, len(tau_crit), self._taus, len(pacing_cap), self._caps,
+                              code, k["w_p"].data_ptr(), k["w_q"].data_ptr(), k["ts"].data_ptr(),
+                              k["slo"].data_ptr(), ok_frac, reliability, ctrl, k["r0"].data_ptr())
+        self.sout = SweepOut(*[out[c].data_ptr() if c in out else None
+                               for c in ("P", "D", "A", "W", "S", "Z", "cls", "theta", "moves")],
+                             moves_cap, out["n_moves"].data_ptr(), out["r_final"].data_ptr())
+        size = C.c_size_t(0)
+        _check("tre_sweep", self.lib.tre_sweep(C.byref(self.spec), C.byref(self.sout), None,
+                                               C.byref(size), None, None))
+        if ws is None or ws.numel() < size.value:
+            ws = torch.empty(max(int(size.value), 256), dtype=torch.uint8, device="cuda")
+        self.diag = new_diag() if diag is None else diag
+        out.update(ws=ws, diag=self.diag, K=self.K)
+        self.out = out
+        self._keep = (k, traces)
+        self._ws_ptr = C.c_void_p(ws.data_ptr())
+        self._ws_n = C.c_size_t(ws.numel())
+        self._diag_ptr = C.c_void_p(self.diag.data_ptr())
+        self.n_inst, self.moves_cap = n_inst, moves_cap
+
+    def run(self, stream=None):
+        """Enqueue the sweep on `stream` (default: current torch stream); returns
+        the plan's output dict (the same tensors every call)."""
+        _check("tre_sweep", self.lib.tre_sweep(C.byref(self.spec), C.byref(self.sout),
+                                               self._ws_ptr, C.byref(self._ws_n), self._diag_ptr,
+                                               _stream(stream)))
+        return self.out
+
+
 def tre_sweep(traces, M, duration_ms, window_ms, alpha, tau_crit, pacing_cap, w_p, w_q,
               tau_surplus, slo_ttft_ms, budget, r0, r_min, footprint, fast_ms=5000,
               slow_ms=10000, dtype="f32", ok_frac=0.95, reliability=0.95, moves_cap=256,
               want_counts=False, want_S=False, diag=None, stream=None, ws=None):
-    """Batched open-loop sweep. `traces`: list of dicts of int32 CUDA tensors.
-    Returns a dict of CUDA tensors (theta, Z, cls, moves, n_moves, r_final, ...)."""
-    torch = _torch()
-    lib = load()
-    code, tdt = _dt(dtype)
-    win = np.asarray(window_ms, np.int32)
-    n_series = len(traces) * len(win)
-    K = [duration_ms // int(w) for w in win]
-    total = sum(K[i % len(win)] * M for i in range(n_series))
-    n_inst = n_series * len(tau_crit) * len(pacing_cap)
-    f = lambda v: torch.as_tensor(np.broadcast_to(np.asarray(v), (M,)).copy()).to(
-        device="cuda", dtype=tdt)
-    i32 = lambda v: torch.as_tensor(np.asarray(v, np.int32)).cuda()
-    keep = {"w_p": f(w_p), "w_q": f(w_q), "ts": f(tau_surplus), "slo": i32(slo_ttft_ms),
-            "r0": i32(r0), "rmin": i32(r_min), "fp": i32(footprint)}
-    out = {"theta": torch.empty((n_series, M), dtype=tdt, device="cuda"),
-           "Z": torch.empty(total, dtype=tdt, device="cuda"),
-           "cls": torch.empty(total, dtype=torch.uint8, device="cuda"),
-           "moves": torch.zeros(n_inst * max(moves_cap, 1) * MOVE_DTYPE.itemsize,
-                                dtype=torch.uint8, device="cuda"),
-           "n_moves": torch.zeros(n_inst, dtype=torch.int64, device="cuda"),
-           "r_final": torch.empty((n_inst, M), dtype=torch.int32, device="cuda")}
-    if want_counts:
-        for k in "PDAW":
-            out[k] = torch.empty(total, dtype=torch.int32, device="cuda")
-    if want_S:
-        out["S"] = torch.empty(total, dtype=tdt, device="cuda")
-    tr = (Requests * len(traces))(*[requests_struct(t) for t in traces])
-    wins = (C.c_int32 * len(win))(*[int(x) for x in win])
-    alph = (C.c_double * len(win))(*[float(a) for a in alpha])
-    taus = (C.c_double * len(tau_crit))(*[float(t) for t in tau_crit])
-    caps = (C.c_int32 * len(pacing_cap))(*[int(c) for c in pacing_cap])
-    ctrl = Ctrl(int(budget), keep["rmin"].data_ptr(), keep["fp"].data_ptr(), fast_ms, slow_ms, 0)
-    spec = SweepSpec(M, duration_ms, len(traces), tr, len(win), wins, alph, len(tau_crit), taus,
-                     len(pacing_cap), caps, code, keep["w_p"].data_ptr(), keep["w_q"].data_ptr(),
-                     keep["ts"].data_ptr(), keep["slo"].data_ptr(), ok_frac, reliability, ctrl,
-                     keep["r0"].data_ptr())
-    so = SweepOut(*[out[k].data_ptr() if k in out else None
-                    for k in ("P", "D", "A", "W", "S", "Z", "cls", "theta", "moves")],
-                  moves_cap, out["n_moves"].data_ptr(), out["r_final"].data_ptr())
-    diag = new_diag() if diag is None else diag
-    s = _stream(stream)
-    if ws is None:
-        ws = _workspace("tre_sweep", lambda w, n: lib.tre_sweep(C.byref(spec), C.byref(so), w, n,
-                                                                _ptr(diag), s))
-    else:
-        n = C.c_size_t(ws.numel())
-        _check("tre_sweep", lib.tre_sweep(C.byref(spec), C.byref(so), _ptr(ws), C.byref(n),
-                                          _ptr(diag), s))
-    out["ws"] = ws
-    out["diag"] = diag
-    out["K"] = K
-    out["_keep"] = (keep, tr)
+    """Batched open-loop sweep, one call. Returns a dict of CUDA tensors (theta,
+    Z, cls, moves, n_moves, r_final, ...) plus the workspace `ws` for reuse."""
+    plan = SweepPlan(traces, M, duration_ms, window_ms, alpha, tau_crit, pacing_cap, w_p, w_q,
+                     tau_surplus, slo_ttft_ms, budget, r0, r_min, footprint, fast_ms, slow_ms,
+                     dtype, ok_frac, reliability, moves_cap, want_counts, want_S, diag, ws)
+    out = dict(plan.run(stream))
+    out["_keep"] = plan
     return out
 
 
