@@ -17,7 +17,7 @@ namespace tre {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kStageBytes = 32 * 1024;   // start-side staging per CTA
+constexpr int kStageBytes = 32 * 1024;   // event staging per CTA
 constexpr int kSpill = 32;  // staged rows beyond the CTA's arrival range
 
 // window of a millisecond time (int32 range), clamped to [0, K]
@@ -40,11 +40,14 @@ __device__ __forceinline__ void stage_add(V* s, V* g, int64_t k, int64_t k_lo, i
 // batch of traces on one grid (CTAs [cta_base[t], cta_base[t+1]) take trace t)
 // --------------------------------------------------------------------------
 constexpr int kMaxTraces = 64;
+constexpr int kVec = 4;               // records per thread per pass
+constexpr int kMaxPerCta = 16384;     // bound that keeps the packed shared counters exact
 struct ReqBatch {
   int n;
   ReqCols cols[kMaxTraces];
   int64_t per_cta[kMaxTraces];
   int32_t cta_base[kMaxTraces + 1];
+  unsigned long long vec_ok;          // bit t: trace t's columns allow 16-byte loads
 };
 
 // Targets of one record fall in two places: the arrival side (the waiting
@@ -55,184 +58,272 @@ struct ReqBatch {
 // arrive in, and the start side per model over a run of windows beginning at
 // that model's earliest start among the CTA's records. Targets outside both
 // go to global atomics.
+//
+// Two counters share one 32-bit shared word where both stay small: a CTA
+// holds at most kMaxPerCta records, so the SLO pair (arrivals, met) packs as
+// arrivals + met * 2^16, and the running/waiting gauge deltas of one start
+// window pack as running + waiting * 2^16 (both signed, each bounded by the
+// CTA's record count; the low half is recovered by sign extension).
 struct Stage {
-  int32_t *aW;                  // arrival side: [near_rows][M]
-  unsigned long long* aS;       // arrival side SLO counts: [near_rows][M]
-  int32_t *fP, *fD, *fA, *fW;   // start side: [M][far_rows]
-  int32_t* far_lo;              // [M]
-  int32_t* slo_lim;             // [M]
+  int32_t* aW;        // arrival side, waiting +1: [near_rows][Mp]
+  uint32_t* aS;       // arrival side, packed SLO counts: [near_rows][Mp]
+  int32_t *fP, *fD;   // start side, tokens: [M][F + 1]
+  int32_t* fAW;       // start side, packed gauge deltas: [M][F + 1]
+  int32_t* far_lo;    // [M]
+  int32_t* slo_lim;   // [M]
 };
 
+__device__ __forceinline__ uint32_t ceil_div(unsigned long long x, uint32_t d) {
+  unsigned long long q, r;
+  divmod(x, d, q, r);
+  return (uint32_t)(q + (r != 0));
+}
+
 template <bool SLO>
-__global__ void __launch_bounds__(kThreads)
-k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int win, FastDiv fd, int K,
-                  int near_rows, int far_rows, int32_t* __restrict__ P0, int32_t* __restrict__ D0,
-                  int32_t* __restrict__ dA0, int32_t* __restrict__ dW0,
+__global__ void __launch_bounds__(kThreads, 4)
+k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win, FastDiv fd,
+                  int K, int near_rows, int lgF, int32_t* __restrict__ P0,
+                  int32_t* __restrict__ D0, int32_t* __restrict__ dA0, int32_t* __restrict__ dW0,
                   unsigned long long* __restrict__ slo0, const int32_t* __restrict__ slo_ms,
                   tre_diag* diag) {
   extern __shared__ unsigned long long smem[];
   int t = 0;
   while (t + 1 < bt.n && bt.cta_base[t + 1] <= (int)blockIdx.x) ++t;
   const ReqCols& r = bt.cols[t];
-  const int64_t per_cta = bt.per_cta[t];
+  const bool vec = (bt.vec_ok >> t) & 1ull;
   const size_t cells0 = (size_t)K * M, cells1 = (size_t)(K + 1) * M;
   int32_t* P = P0 + t * cells0;
   int32_t* D = D0 + t * cells0;
   int32_t* dA = dA0 + t * cells1;
   int32_t* dW = dW0 + t * cells1;
   unsigned long long* slo = SLO ? slo0 + t * cells0 : nullptr;
-  const int64_t i0 = (int64_t)(blockIdx.x - bt.cta_base[t]) * per_cta;
-  const int64_t i1 = min(r.n, i0 + per_cta);
-  if (i0 >= i1) return;
-  const int64_t span = (int64_t)K * win;
-  const int64_t k_lo = win_clamp(r.t_arr[i0], fd, K);
-  const int64_t k_hi = win_clamp(r.t_arr[i1 - 1], fd, K);
-  const int64_t need = (k_hi >= k_lo ? k_hi - k_lo + 1 : 1) + 1;
-  const int used = (int)min64(near_rows, need);
+  const int64_t i0 = (int64_t)(blockIdx.x - bt.cta_base[t]) * bt.per_cta[t];
+  const int n_loc = (int)min64(r.n - i0, bt.per_cta[t]);
+  if (n_loc <= 0) return;
+  const int Mp = 1 << lgMp, F = 1 << lgF, F1 = F + 1;
+  const uint32_t span = (uint32_t)K * (uint32_t)win;
+  const int a_first = r.t_arr[i0], a_last = r.t_arr[i0 + n_loc - 1];
+  const int k_lo = a_first < 0 ? 0 : (int)min(fd.div((uint32_t)a_first), (uint32_t)K);
+  const int k_hi = a_last < 0 ? 0 : (int)min(fd.div((uint32_t)a_last), (uint32_t)K);
+  const int used = min(near_rows, (k_hi >= k_lo ? k_hi - k_lo + 1 : 1) + 1);
   Stage st;
-  st.aS = smem;
-  st.aW = reinterpret_cast<int32_t*>(smem + (SLO ? (size_t)near_rows * M : 0));
-  st.fP = st.aW + (size_t)near_rows * M;
-  st.fD = st.fP + (size_t)far_rows * M;
-  st.fA = st.fD + (size_t)far_rows * M;
-  st.fW = st.fA + (size_t)far_rows * M;
-  st.far_lo = st.fW + (size_t)far_rows * M;
+  st.aW = reinterpret_cast<int32_t*>(smem);
+  st.aS = reinterpret_cast<uint32_t*>(st.aW + (size_t)near_rows * Mp);
+  st.fP = reinterpret_cast<int32_t*>(st.aS + (SLO ? (size_t)near_rows * Mp : 0));
+  st.fD = st.fP + (size_t)M * F1;
+  st.fAW = st.fD + (size_t)M * F1;
+  st.far_lo = st.fAW + (size_t)M * F1;
   st.slo_lim = st.far_lo + M;
-  const int ncell = used * M, fcell = far_rows * M;
+  const int ncell = used * Mp, fcell = M * F1;
   for (int c = threadIdx.x; c < ncell; c += kThreads) {
     st.aW[c] = 0;
     if (SLO) st.aS[c] = 0;
   }
-  for (int c = threadIdx.x; c < fcell; c += kThreads) {
-    st.fP[c] = 0; st.fD[c] = 0; st.fA[c] = 0; st.fW[c] = 0;
-  }
+  for (int c = threadIdx.x; c < fcell; c += kThreads) { st.fP[c] = 0; st.fD[c] = 0; st.fAW[c] = 0; }
   for (int m = threadIdx.x; m < M; m += kThreads) {
     st.far_lo[m] = 0x7fffffff;
     if (SLO) st.slo_lim[m] = slo_ms[m];
   }
   __syncthreads();
   // each model's earliest start window among this CTA's records
-  for (int64_t i = i0 + threadIdx.x; i < i1; i += kThreads) {
-    const int m = r.model[i];
-    const int32_t ts = r.t_start[i];
-    if (m >= 0 && m < M && ts >= 0) atomicMin(&st.far_lo[m], (int32_t)win_clamp(ts, fd, K));
+  for (int b = threadIdx.x * kVec; b < n_loc; b += kThreads * kVec) {
+    int mm[kVec], ss[kVec];
+    if (vec && b + kVec <= n_loc) {
+      const int4 a = *reinterpret_cast<const int4*>(r.model + i0 + b);
+      const int4 s = *reinterpret_cast<const int4*>(r.t_start + i0 + b);
+      mm[0] = a.x; mm[1] = a.y; mm[2] = a.z; mm[3] = a.w;
+      ss[0] = s.x; ss[1] = s.y; ss[2] = s.z; ss[3] = s.w;
+    } else {
+#pragma unroll
+      for (int u = 0; u < kVec; ++u) {
+        const bool in = b + u < n_loc;
+        mm[u] = in ? r.model[i0 + b + u] : -1;
+        ss[u] = in ? r.t_start[i0 + b + u] : -1;
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kVec; ++u)
+      if (mm[u] >= 0 && mm[u] < M && ss[u] >= 0)
+        atomicMin(&st.far_lo[mm[u]], (int)min(fd.div((uint32_t)ss[u]), (uint32_t)K));
   }
   __syncthreads();
 
-  // arrival-side target (waiting +1, SLO counts)
-  auto near_add = [&](auto* s_arr, auto* g_arr, int64_t k, int m, auto v) {
-    const int64_t rel = k - k_lo;
-    if (rel >= 0 && rel < used) atomicAdd(&s_arr[rel * M + m], v);
-    else atomicAdd(&g_arr[k * M + m], v);
+  // arrival-side target
+  auto near_idx = [&](int k, int m) -> int {
+    const unsigned rel = (unsigned)(k - k_lo);
+    return rel < (unsigned)used ? (int)(rel << lgMp) + m : -1;
   };
-  // start-side target of model m
-  auto far_add = [&](int32_t* s_arr, int32_t* g_arr, int64_t k, int m, int32_t v) {
-    const int64_t rel = k - st.far_lo[m];
-    if (rel >= 0 && rel < far_rows) atomicAdd(&s_arr[m * far_rows + rel], v);
-    else atomicAdd(&g_arr[k * M + m], v);
+  // start-side target of model m: shared cell index, or -1 when outside
+  auto far_idx = [&](int k, int m, int lo) -> int {
+    const unsigned rel = (unsigned)(k - lo);
+    return rel < (unsigned)F ? m * F1 + (int)rel : -1;
+  };
+  auto add_tok = [&](int32_t* s_arr, int32_t* g_arr, int k, int m, int lo, int32_t v) {
+    const int c = far_idx(k, m, lo);
+    if (c >= 0) atomicAdd(&s_arr[c], v);
+    else atomicAdd(&g_arr[(size_t)k * M + m], v);
+  };
+  auto add_aw = [&](int k, int m, int lo, int32_t a, int32_t w) {
+    const int c = far_idx(k, m, lo);
+    if (c >= 0) {
+      atomicAdd(&st.fAW[c], a + w * 65536);
+    } else {
+      if (a) atomicAdd(&dA[(size_t)k * M + m], a);
+      if (w) atomicAdd(&dW[(size_t)k * M + m], w);
+    }
   };
 
+  const unsigned full = 0xffffffffu;
+  const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
   unsigned long long n_range = 0, n_model = 0, n_order = 0;
-  int32_t nx[7];
-  auto load_rec = [&](int64_t i) {
-    if (i < i1) {
-      nx[0] = r.model[i];
-      nx[1] = r.t_arr[i];
-      nx[2] = r.t_start[i];
-      nx[3] = r.t_first[i];
-      nx[4] = r.t_end[i];
-      nx[5] = r.L_in[i];
-      nx[6] = r.L_out[i];
+  // warp-uniform passes: lane l of a pass takes records b + l*kVec + u
+  for (int wb = warp * 32 * kVec; wb < n_loc; wb += kThreads * kVec) {
+    const int b = wb + lane * kVec;
+    int v[7][kVec];
+    const int32_t* cols[7] = {r.model, r.t_arr, r.t_start, r.t_first, r.t_end, r.L_in, r.L_out};
+    if (vec && b + kVec <= n_loc) {
+#pragma unroll
+      for (int c = 0; c < 7; ++c) {
+        const int4 q = __ldcs(reinterpret_cast<const int4*>(cols[c] + i0 + b));
+        v[c][0] = q.x; v[c][1] = q.y; v[c][2] = q.z; v[c][3] = q.w;
+      }
+    } else {
+#pragma unroll
+      for (int u = 0; u < kVec; ++u) {
+        const bool in = b + u < n_loc;
+#pragma unroll
+        for (int c = 0; c < 7; ++c) v[c][u] = in ? cols[c][i0 + b + u] : 0;
+        if (!in) v[0][u] = -1;   // marks "no record" (not counted as a drop)
+      }
     }
-  };
-  load_rec(i0 + threadIdx.x);
-  for (int64_t i = i0 + threadIdx.x; i < i1; i += kThreads) {
-    const int m = nx[0];
-    const int64_t ta = nx[1], ts = nx[2], tf = nx[3], te = nx[4];
-    const int32_t L_in = nx[5], L = nx[6];
-    load_rec(i + kThreads);
-    if (m < 0 || m >= M) { ++n_model; continue; }
-    if (ta < 0 || ta >= span) { ++n_range; continue; }
-    if (!(ta <= ts && ts <= tf && tf <= te) || L_in < 0 || L < 1) { ++n_order; continue; }
-
-    const int64_t ba = fd.div((uint32_t)ta);
-    const int64_t bs = win_clamp(ts, fd, K), be = win_clamp(te, fd, K);
-    if (ba != bs) {
-      near_add(st.aW, dW, ba, m, (int32_t)1);
-      far_add(st.fW, dW, bs, m, -1);
-    }
-    if (bs != be) {
-      far_add(st.fA, dA, bs, m, 1);
-      far_add(st.fA, dA, be, m, -1);
-    }
-    if (SLO) {
-      const unsigned long long met = (tf - ta <= (int64_t)st.slo_lim[m]) ? 1ull : 0ull;
-      near_add(st.aS, slo, ba, m, 1ull + (met << 32));
-    }
-    if (tf < span) {
-      const int64_t kf = fd.div((uint32_t)tf);
-      // prompt tokens, all at the first-token time
-      if (L_in) far_add(st.fP, P, kf, m, L_in);
-      // decode tokens: N(T) = tokens emitted before T; D[k] = N((k+1)w) - N(kw)
-      const int64_t ke_raw = fd.div((uint32_t)te);
-      if (L == 1 || ke_raw == kf) {
-        far_add(st.fD, D, kf, m, L);
-      } else {
-        const unsigned long long dur = (unsigned long long)(te - tf);
-        const unsigned long long Lm1 = (unsigned long long)(L - 1);
-        unsigned long long q, rem;
-        // N at the first window boundary after tf: ceil((T - tf)(L-1)/dur)
-        divmod((unsigned long long)((kf + 1) * win - tf) * Lm1, (uint32_t)dur, q, rem);
-        const int32_t n1 = (int32_t)(q + (rem != 0));
-        far_add(st.fD, D, kf, m, n1);
-        if (ke_raw == kf + 1) {
-          if (kf + 1 < K) far_add(st.fD, D, kf + 1, m, L - n1);
-        } else {
-          const int64_t ke = min64(ke_raw, K - 1);
-          unsigned long long qs, rs;
-          divmod((unsigned long long)win * Lm1, (uint32_t)dur, qs, rs);
-          q += qs;
-          rem += rs;
-          if (rem >= dur) { rem -= dur; q += 1; }
-          unsigned long long prevN = (unsigned long long)n1;
-          for (int64_t k = kf + 1; k <= ke; ++k) {
-            unsigned long long N;
-            if ((k + 1) * win > te) {
-              N = (unsigned long long)L;
+#pragma unroll
+    for (int u = 0; u < kVec; ++u) {
+      const bool present = b + u < n_loc;
+      const int m = v[0][u], ta = v[1][u], ts = v[2][u], tf = v[3][u], te = v[4][u];
+      const int L_in = v[5][u], L = v[6][u];
+      bool ok = false;
+      if (present) {
+        if (m < 0 || m >= M) ++n_model;
+        else if (ta < 0 || (uint32_t)ta >= span) ++n_range;
+        else if (!(ta <= ts && ts <= tf && tf <= te) || L_in < 0 || L < 1) ++n_order;
+        else ok = true;
+      }
+      // decode windows after the first-token window that need a division each
+      bool lng = false;
+      int kf = 0, n1 = 0, pairs = 0;
+      if (ok) {
+        const int lo = st.far_lo[m];
+        const int ba = (int)fd.div((uint32_t)ta);
+        const int bs = (int)min(fd.div((uint32_t)ts), (uint32_t)K);
+        const int be_raw = (int)fd.div((uint32_t)te);
+        const int be = min(be_raw, K);
+        const int na = near_idx(ba, m);
+        if (ba != bs) {
+          if (na >= 0) atomicAdd(&st.aW[na], 1);
+          else atomicAdd(&dW[(size_t)ba * M + m], 1);
+        }
+        if (SLO) {
+          const uint32_t met = (tf - ta <= st.slo_lim[m]) ? 1u : 0u;
+          if (na >= 0) atomicAdd(&st.aS[na], 1u + (met << 16));
+          else atomicAdd(&slo[(size_t)ba * M + m], 1ull + ((unsigned long long)met << 32));
+        }
+        const int run = bs != be ? 1 : 0, wait = ba != bs ? -1 : 0;
+        if (run | wait) add_aw(bs, m, lo, run, wait);
+        if (run) add_aw(be, m, lo, -1, 0);
+        if ((uint32_t)tf < span) {
+          kf = (int)fd.div((uint32_t)tf);
+          if (L_in) add_tok(st.fP, P, kf, m, lo, L_in);
+          if (L == 1 || be_raw == kf) {
+            add_tok(st.fD, D, kf, m, lo, L);
+          } else {
+            // N(T) = tokens emitted before T = ceil((T - tf)(L-1)/dur)
+            n1 = (int)ceil_div((unsigned long long)((uint32_t)(kf + 1) * (uint32_t)win - (uint32_t)tf) *
+                                   (uint32_t)(L - 1),
+                               (uint32_t)(te - tf));
+            add_tok(st.fD, D, kf, m, lo, n1);
+            if (be_raw == kf + 1) {
+              if (kf + 1 < K) add_tok(st.fD, D, kf + 1, m, lo, L - n1);
             } else {
-              N = q + (rem != 0);
-              q += qs;
-              rem += rs;
-              if (rem >= dur) { rem -= dur; q += 1; }
+              pairs = min(be_raw, K - 1) - kf;   // windows kf+1 .. min(be, K-1)
+              lng = pairs > 0;
             }
-            const int32_t cnt = (int32_t)(N - prevN);
-            if (cnt) far_add(st.fD, D, k, m, cnt);
-            prevN = N;
           }
+        }
+      }
+      // Spread the remaining (record, window) pairs of the warp's long decodes
+      // over the lanes: pair p goes to lane p % 32 of chunk p / 32.
+      if (__any_sync(full, lng)) {
+        const int cnt = lng ? pairs : 0;
+        int incl = cnt;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int y = __shfl_up_sync(full, incl, o);
+          if (lane >= o) incl += y;
+        }
+        const int total = __shfl_sync(full, incl, 31);
+        int carry = 0;
+        for (int cb = 0; cb < total; cb += 32) {
+          const int p = cb + lane;
+          int o = 0;
+#pragma unroll
+          for (int s = 16; s; s >>= 1) {
+            const int y = __shfl_sync(full, incl, o + s - 1);
+            if (y <= p) o += s;
+          }
+          const int om = __shfl_sync(full, m, o), otf = __shfl_sync(full, tf, o);
+          const int ote = __shfl_sync(full, te, o), oL = __shfl_sync(full, L, o);
+          const int okf = __shfl_sync(full, kf, o), on1 = __shfl_sync(full, n1, o);
+          const int ostart = __shfl_sync(full, incl - cnt, o);
+          const bool act = p < total;
+          const int j = p - ostart;
+          const int k = okf + 1 + j;
+          uint32_t Nend = 0;
+          if (act) {
+            const uint32_t bend = (uint32_t)(k + 1) * (uint32_t)win;
+            Nend = bend > (uint32_t)ote
+                       ? (uint32_t)oL
+                       : ceil_div((unsigned long long)(bend - (uint32_t)otf) * (uint32_t)(oL - 1),
+                                  (uint32_t)(ote - otf));
+          }
+          const uint32_t prev = __shfl_up_sync(full, Nend, 1);
+          const uint32_t Nstart = j == 0 ? (uint32_t)on1 : (lane == 0 ? (uint32_t)carry : prev);
+          if (act && Nend != Nstart)
+            add_tok(st.fD, D, k, om, st.far_lo[om], (int32_t)(Nend - Nstart));
+          carry = (int)__shfl_sync(full, Nend, 31);
         }
       }
     }
   }
   __syncthreads();
   for (int c = threadIdx.x; c < ncell; c += kThreads) {
-    const int64_t k = k_lo + c / M;
-    const size_t g = (size_t)k * M + (c % M);
-    if (k < K && SLO && st.aS[c]) atomicAdd(&slo[g], st.aS[c]);
+    const int m = c & (Mp - 1);
+    if (m >= M) continue;
+    const int k = k_lo + (c >> lgMp);
+    const size_t g = (size_t)k * M + m;
+    if (SLO && k < K) {
+      const uint32_t s = st.aS[c];
+      if (s) atomicAdd(&slo[g], (unsigned long long)(s & 0xffffu) + ((unsigned long long)(s >> 16) << 32));
+    }
     if (k <= K && st.aW[c]) atomicAdd(&dW[g], st.aW[c]);
   }
-  for (int c = threadIdx.x; c < fcell; c += kThreads) {
-    const int m = c / far_rows;
+  for (int c = threadIdx.x; c < M * F; c += kThreads) {
+    const int m = c >> lgF;
     const int lo = st.far_lo[m];
     if (lo == 0x7fffffff) continue;
-    const int64_t k = (int64_t)lo + (c % far_rows);
+    const int k = lo + (c & (F - 1));
+    const int cell = m * F1 + (c & (F - 1));
     const size_t g = (size_t)k * M + m;
     if (k < K) {
-      if (st.fP[c]) atomicAdd(&P[g], st.fP[c]);
-      if (st.fD[c]) atomicAdd(&D[g], st.fD[c]);
+      if (st.fP[cell]) atomicAdd(&P[g], st.fP[cell]);
+      if (st.fD[cell]) atomicAdd(&D[g], st.fD[cell]);
     }
-    if (k <= K) {
-      if (st.fA[c]) atomicAdd(&dA[g], st.fA[c]);
-      if (st.fW[c]) atomicAdd(&dW[g], st.fW[c]);
+    const int32_t aw = st.fAW[cell];
+    if (k <= K && aw) {
+      const int32_t a = (int32_t)(int16_t)(aw & 0xffff);
+      const int32_t w = (aw - a) / 65536;
+      if (a) atomicAdd(&dA[g], a);
+      if (w) atomicAdd(&dW[g], w);
     }
   }
   warp_add_counter(&diag->dropped_range, n_range);
@@ -576,28 +667,40 @@ cudaError_t launch_reduce_requests(const ReqCols* traces, int n_traces, int M, i
   if (slo && (e = cudaMemsetAsync(slo, 0, cells * sizeof(unsigned long long), s))) return e;
   ReqBatch bt;
   bt.n = n_traces;
+  bt.vec_ok = 0;
   int64_t total_n = 0;
   for (int t = 0; t < n_traces; ++t) total_n += traces[t].n;
+  // records per CTA sized on the whole batch so the grid fills the GPU
+  const int64_t per = per_cta_records(std::max<int64_t>(total_n / n_traces, 1), 1024, 8192);
+  static_assert(8192 <= kMaxPerCta, "packed shared counters need <= kMaxPerCta records per CTA");
   int ctas = 0;
   for (int t = 0; t < n_traces; ++t) {
-    bt.cols[t] = traces[t];
-    // records per CTA sized on the whole batch so the grid fills the GPU
-    const int64_t per = per_cta_records(std::max<int64_t>(total_n / n_traces, 1), 1024, 8192);
+    const ReqCols& c = traces[t];
+    bt.cols[t] = c;
     bt.per_cta[t] = per;
     bt.cta_base[t] = ctas;
-    ctas += (int)((traces[t].n + per - 1) / per);
+    ctas += (int)((c.n + per - 1) / per);
+    const uintptr_t ptr_or = (uintptr_t)c.model | (uintptr_t)c.t_arr | (uintptr_t)c.t_start |
+                             (uintptr_t)c.t_first | (uintptr_t)c.t_end | (uintptr_t)c.L_in |
+                             (uintptr_t)c.L_out;
+    if ((ptr_or & 15u) == 0) bt.vec_ok |= 1ull << t;
   }
   bt.cta_base[n_traces] = ctas;
   if (ctas == 0) return cudaSuccess;
-  // arrival-side rows cover the CTA's arrival span; start-side rows per model
-  const int64_t per = bt.per_cta[0];
-  const int64_t near_cap = 48 * 1024 / ((4 + (slo ? 8 : 0)) * M);   // arrival-stage budget
+  // model rows padded to a power of two on the arrival side; start side runs
+  // of F (power of two) windows per model
+  int lgMp = 0;
+  while ((1 << lgMp) < M) ++lgMp;
+  const int Mp = 1 << lgMp;
+  const int64_t near_cap = 32 * 1024 / ((4 + (slo ? 4 : 0)) * Mp);   // arrival-stage budget
   const int near_rows = (int)std::max<int64_t>(
       1, std::min<int64_t>(near_cap,
                            (int64_t)(3.0 * per / std::max<int64_t>(total_n / n_traces, 1) * K) +
                                34));   // 3x the mean arrival span
-  const int far_rows = std::max(8, std::min(512, (int)(kStageBytes / (16 * M))));
-  const size_t smem = (size_t)near_rows * M * (4 + (slo ? 8 : 0)) + (size_t)far_rows * M * 16 +
+  int lgF = 3;
+  while (lgF < 8 && (size_t)12 * M * ((2 << lgF) + 1) <= 16 * 1024) ++lgF;
+  const int F = 1 << lgF;
+  const size_t smem = (size_t)near_rows * Mp * (4 + (slo ? 4 : 0)) + (size_t)12 * M * (F + 1) +
                       (size_t)M * 8;
   if (smem > 200 * 1024) return cudaErrorInvalidValue;
   static bool attr = false;
@@ -610,13 +713,13 @@ cudaError_t launch_reduce_requests(const ReqCols* traces, int n_traces, int M, i
     attr = true;
   }
   if (slo)
-    k_reduce_requests<true><<<ctas, kThreads, smem, s>>>(bt, M, win, FastDiv(win), K, near_rows,
-                                                         far_rows, P, D, w.dA, w.dW, slo, slo_ms,
-                                                         diag);
+    k_reduce_requests<true><<<ctas, kThreads, smem, s>>>(bt, M, lgMp, win, FastDiv(win), K,
+                                                         near_rows, lgF, P, D, w.dA, w.dW, slo,
+                                                         slo_ms, diag);
   else
-    k_reduce_requests<false><<<ctas, kThreads, smem, s>>>(bt, M, win, FastDiv(win), K, near_rows,
-                                                          far_rows, P, D, w.dA, w.dW, nullptr,
-                                                          nullptr, diag);
+    k_reduce_requests<false><<<ctas, kThreads, smem, s>>>(bt, M, lgMp, win, FastDiv(win), K,
+                                                          near_rows, lgF, P, D, w.dA, w.dW,
+                                                          nullptr, nullptr, diag);
   return cudaGetLastError();
 }
 

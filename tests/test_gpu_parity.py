@@ -85,6 +85,51 @@ def test_reduce_requests_adversarial(tre, seed, M, win, K):
     _check_reduce(tre, {k: v[perm] for k, v in req.items()}, M, win, K)
 
 
+def _sorted_long(rng, n, M, win, K):
+    """Arrival-sorted records (the order telemetry arrives in) with queue waits,
+    long decodes over many windows, very long outputs and some bad records."""
+    span = K * win
+    t_arr = np.sort(rng.integers(0, span + win, n))
+    wait = rng.integers(0, 40 * win, n) * (rng.random(n) < 0.7)
+    pre = rng.integers(0, 2 * win, n)
+    dec = np.where(rng.random(n) < 0.3, rng.integers(0, 60 * win, n), rng.integers(0, 2 * win, n))
+    L_out = np.where(rng.random(n) < 0.1, rng.integers(1, 100000, n), rng.integers(1, 400, n))
+    t_start = t_arr + wait
+    t_first = t_start + pre
+    t_end = np.where(L_out == 1, t_first, t_first + dec)
+    model = rng.integers(0, M, n)
+    model = np.where(rng.random(n) < 0.01, M, model)
+    return {"model": model.astype(np.int32), "t_arr_ms": t_arr.astype(np.int32),
+            "t_start_ms": t_start.astype(np.int32), "t_first_ms": t_first.astype(np.int32),
+            "t_end_ms": t_end.astype(np.int32),
+            "L_in": rng.integers(0, 5000, n).astype(np.int32), "L_out": L_out.astype(np.int32)}
+
+
+@pytest.mark.parametrize("seed,M,win,K,n", [(11, 8, 100, 3000, 60003), (12, 64, 50, 2000, 40001),
+                                            (13, 5, 1000, 400, 9999)])
+def test_reduce_requests_sorted_long_decodes(tre, seed, M, win, K, n):
+    rng = np.random.default_rng(seed)
+    _check_reduce(tre, _sorted_long(rng, n, M, win, K), M, win, K)
+
+
+def test_reduce_requests_unaligned_columns(tre):
+    """Columns that start 4 bytes past a 16-byte boundary take the scalar loads."""
+    import torch
+    rng = np.random.default_rng(21)
+    M, win, K = 8, 100, 1500
+    req = _sorted_long(rng, 30001, M, win, K)
+    P, D, A, W, drops = oracle.reduce_requests(req, M, win, K)
+    dev = {}
+    for k, v in req.items():
+        buf = torch.zeros(len(v) + 1, dtype=torch.int32, device="cuda")
+        buf[1:] = torch.as_tensor(v).cuda()
+        dev[k] = buf[1:]
+        assert dev[k].data_ptr() % 16 == 4
+    c = tre.tss_window_reduce(M, win, K, requests=dev)
+    for k, ref in zip("PDAW", (P, D, A, W)):
+        np.testing.assert_array_equal(_np(c[k]), ref, err_msg=k)
+
+
 def test_reduce_empty_and_zero_windows(tre):
     req = {k: np.zeros(0, np.int32) for k in REQ_KEYS}
     _check_reduce(tre, req, 4, 1000, 10)
