@@ -218,36 +218,57 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win,
         const int bs = (int)min(fd.div((uint32_t)ts), (uint32_t)K);
         const int be_raw = (int)fd.div((uint32_t)te);
         const int be = min(be_raw, K);
-        const int na = near_idx(ba, m);
-        if (ba != bs) {
-          if (na >= 0) atomicAdd(&st.aW[na], 1);
-          else atomicAdd(&dW[(size_t)ba * M + m], 1);
-        }
-        if (SLO) {
-          const uint32_t met = (tf - ta <= st.slo_lim[m]) ? 1u : 0u;
-          if (na >= 0) atomicAdd(&st.aS[na], 1u + (met << 16));
-          else atomicAdd(&slo[(size_t)ba * M + m], 1ull + ((unsigned long long)met << 32));
-        }
-        const int run = bs != be ? 1 : 0, wait = ba != bs ? -1 : 0;
-        if (run | wait) add_aw(bs, m, lo, run, wait);
-        if (run) add_aw(be, m, lo, -1, 0);
-        if ((uint32_t)tf < span) {
-          kf = (int)fd.div((uint32_t)tf);
-          if (L_in) add_tok(st.fP, P, kf, m, lo, L_in);
-          if (L == 1 || be_raw == kf) {
-            add_tok(st.fD, D, kf, m, lo, L);
+        const bool tok = (uint32_t)tf < span;
+        kf = tok ? (int)fd.div((uint32_t)tf) : 0;
+        // decode tokens of the first-token window (d0) and, for a decode that
+        // ends in the next window, of that window (d1); longer decodes leave
+        // their later windows to the warp-spread pass below
+        int d0 = L, d1 = 0;
+        if (tok && L != 1 && be_raw != kf) {
+          // N(T) = tokens emitted before T = ceil((T - tf)(L-1)/dur)
+          n1 = (int)ceil_div((unsigned long long)((uint32_t)(kf + 1) * (uint32_t)win -
+                                                  (uint32_t)tf) * (uint32_t)(L - 1),
+                             (uint32_t)(te - tf));
+          d0 = n1;
+          if (be_raw == kf + 1) {
+            d1 = L - n1;
           } else {
-            // N(T) = tokens emitted before T = ceil((T - tf)(L-1)/dur)
-            n1 = (int)ceil_div((unsigned long long)((uint32_t)(kf + 1) * (uint32_t)win - (uint32_t)tf) *
-                                   (uint32_t)(L - 1),
-                               (uint32_t)(te - tf));
-            add_tok(st.fD, D, kf, m, lo, n1);
-            if (be_raw == kf + 1) {
-              if (kf + 1 < K) add_tok(st.fD, D, kf + 1, m, lo, L - n1);
-            } else {
-              pairs = min(be_raw, K - 1) - kf;   // windows kf+1 .. min(be, K-1)
-              lng = pairs > 0;
-            }
+            pairs = min(be_raw, K - 1) - kf;   // windows kf+1 .. min(be, K-1)
+            lng = pairs > 0;
+          }
+        }
+        const int wait = ba != bs ? 1 : 0, run = bs != be ? 1 : 0;
+        const uint32_t met = SLO && (tf - ta <= st.slo_lim[m]) ? 1u : 0u;
+        const uint32_t rel_a = (uint32_t)(ba - k_lo);
+        // lo <= bs <= kf <= be: one test covers every start-side target
+        if (rel_a < (uint32_t)used && (uint32_t)(be - lo) < (uint32_t)F) {
+          const int na = (int)(rel_a << lgMp) + m;
+          const int fb = m * F1 - lo;
+          atomicAdd(&st.aW[na], wait);
+          if (SLO) atomicAdd(&st.aS[na], 1u + (met << 16));
+          atomicAdd(&st.fAW[fb + bs], run - wait * 65536);
+          if (run) atomicAdd(&st.fAW[fb + be], -1);
+          if (tok) {
+            if (L_in) atomicAdd(&st.fP[fb + kf], L_in);
+            atomicAdd(&st.fD[fb + kf], d0);
+            if (d1) atomicAdd(&st.fD[fb + kf + 1], d1);
+          }
+        } else {
+          const int na = near_idx(ba, m);
+          if (wait) {
+            if (na >= 0) atomicAdd(&st.aW[na], 1);
+            else atomicAdd(&dW[(size_t)ba * M + m], 1);
+          }
+          if (SLO) {
+            if (na >= 0) atomicAdd(&st.aS[na], 1u + (met << 16));
+            else atomicAdd(&slo[(size_t)ba * M + m], 1ull + ((unsigned long long)met << 32));
+          }
+          if (run | wait) add_aw(bs, m, lo, run, -wait);
+          if (run) add_aw(be, m, lo, -1, 0);
+          if (tok) {
+            if (L_in) add_tok(st.fP, P, kf, m, lo, L_in);
+            add_tok(st.fD, D, kf, m, lo, d0);
+            if (d1 && kf + 1 < K) add_tok(st.fD, D, kf + 1, m, lo, d1);
           }
         }
       }
@@ -622,10 +643,10 @@ int num_sms() {
   return n;
 }
 
-int64_t per_cta_records(int64_t n, int lo, int hi) {
+int64_t per_cta_records(int64_t n, int lo, int hi, int quantum = kThreads) {
   int64_t per = (n + (int64_t)num_sms() * 4 - 1) / ((int64_t)num_sms() * 4);
   per = std::max<int64_t>(lo, std::min<int64_t>(hi, per));
-  return (per + kThreads - 1) / kThreads * kThreads;
+  return (per + quantum - 1) / quantum * quantum;
 }
 
 unsigned grid_for(int64_t work, int per_thread = 1) {
@@ -671,7 +692,8 @@ cudaError_t launch_reduce_requests(const ReqCols* traces, int n_traces, int M, i
   int64_t total_n = 0;
   for (int t = 0; t < n_traces; ++t) total_n += traces[t].n;
   // records per CTA sized on the whole batch so the grid fills the GPU
-  const int64_t per = per_cta_records(std::max<int64_t>(total_n / n_traces, 1), 1024, 8192);
+  const int64_t per = per_cta_records(std::max<int64_t>(total_n / n_traces, 1), 1024, 8192,
+                                      kThreads * kVec);   // whole passes for every warp
   static_assert(8192 <= kMaxPerCta, "packed shared counters need <= kMaxPerCta records per CTA");
   int ctas = 0;
   for (int t = 0; t < n_traces; ++t) {
