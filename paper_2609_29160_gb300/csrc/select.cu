@@ -642,8 +642,17 @@ k_walk_thread(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
 // the idle pool is non-empty or a model above its floor is a donor there; per
 // model, the next tick where it is a donor is precomputed, so the walk jumps
 // from one possible move to the next instead of visiting every tick.
+// One tick's action as the walk reads it: donor order (4 bits a position),
+// donor mask, receiver (-1: nothing acts) and kind, in one 16-byte load.
+struct __align__(16) TickRec {
+  unsigned long long pk;
+  uint32_t dm;
+  int16_t recv;
+  uint8_t kind, pad;
+};
+
 template <class T, int MMAX>
-__global__ void __launch_bounds__(32)
+__global__ void __launch_bounds__(256, 1)
 k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
             const unsigned long long* packed, const uint32_t* dmask) {
   extern __shared__ __align__(16) unsigned char dyn[];
@@ -657,19 +666,14 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
   const size_t row0 = (size_t)b.ent_base[si] * b.n_tau + (size_t)ti * n_ent;
   const int nf = (int)((int64_t)K * win / b.fast_ms);   // fast ticks = all ticks
   const int ratio = b.slow_ms / b.fast_ms;
-  // shared layout: per tick u < nf: action entry, kind, window; per entry:
-  // packed order and donor mask; per (model + any, tick): next acting tick
-  unsigned long long* spk = reinterpret_cast<unsigned long long*>(dyn);
-  uint32_t* sdm = reinterpret_cast<uint32_t*>(spk + n_ent);
-  int32_t* swin = reinterpret_cast<int32_t*>(sdm + n_ent);
-  int16_t* sent = reinterpret_cast<int16_t*>(swin + nf);
-  int16_t* srcv = sent + nf;
-  uint8_t* skind = reinterpret_cast<uint8_t*>(srcv + nf);
-  int16_t* snxt = reinterpret_cast<int16_t*>(skind + ((nf + 15) & ~15));  // [M + 1][nf + 1]
-  for (int i = threadIdx.x; i < n_ent; i += blockDim.x) {
-    spk[i] = packed[row0 + i];
-    sdm[i] = dmask[row0 + i];
-  }
+  const unsigned full = 0xffffffffu;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, n_warps = blockDim.x >> 5;
+  // shared layout: per tick u < nf: action record and window; per
+  // (model + any, tick): next tick >= u where the model is a donor (row M:
+  // where anything acts)
+  TickRec* srec = reinterpret_cast<TickRec*>(dyn);
+  int32_t* swin = reinterpret_cast<int32_t*>(srec + nf);
+  int16_t* snxt = reinterpret_cast<int16_t*>(swin + ((nf + 3) & ~3));  // [M + 1][nf + 1]
   for (int u = threadIdx.x; u < nf; u += blockDim.x) {
     const int rf = recv_tab[row0 + u];
     int e = -1, kd = 0, rv = -1;
@@ -680,26 +684,42 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
       const int rs = recv_tab[row0 + es];
       if (rs >= 0) { e = es; kd = TRE_REBALANCE; rv = rs; }
     }
-    sent[u] = (int16_t)e;
-    srcv[u] = (int16_t)rv;
-    skind[u] = (uint8_t)kd;
+    TickRec t;
+    t.pk = e >= 0 ? packed[row0 + e] : 0ull;
+    t.dm = e >= 0 ? dmask[row0 + e] : 0u;
+    t.recv = (int16_t)rv;
+    t.kind = (uint8_t)kd;
+    t.pad = 0;
+    srec[u] = t;
     swin[u] = (int32_t)tick_window(u + 1, b.fast_ms, win);
   }
   __syncthreads();
-  // next tick (>= u) where model m is a donor, and (row M) where any action is
-  for (int m = threadIdx.x; m <= M; m += blockDim.x) {
+  // next-tick tables: a suffix minimum per row, 32 ticks per step
+  for (int m = warp; m <= M; m += n_warps) {
     int16_t* col = snxt + (size_t)m * (nf + 1);
-    int nx = nf;
-    col[nf] = (int16_t)nf;
-    for (int u = nf - 1; u >= 0; --u) {
-      const int e = sent[u];
-      if (e >= 0 && (m == M || (sdm[e] >> m & 1))) nx = u;
-      col[u] = (int16_t)nx;
+    if (lane == 0) col[nf] = (int16_t)nf;
+    int carry = nf;
+    for (int cb = (nf - 1) & ~31; cb >= 0; cb -= 32) {
+      const int u = cb + lane;
+      int v = nf;
+      if (u < nf) {
+        const TickRec& t = srec[u];
+        if (t.recv >= 0 && (m == M || (t.dm >> m & 1u))) v = u;
+      }
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_down_sync(full, v, o);
+        if (lane + o < 32) v = min(v, y);
+      }
+      v = min(v, carry);
+      if (u < nf) col[u] = (int16_t)v;
+      carry = __shfl_sync(full, v, 0);
     }
   }
   __syncthreads();
-  const int ci = threadIdx.x;
-  if (ci >= b.n_cap) return;
+  // one instance per warp, walked by its first lane
+  if (lane != 0) return;
+  for (int ci = warp; ci < b.n_cap; ci += n_warps) {
   const int inst = (si * b.n_tau + ti) * b.n_cap + ci;
   const int Kp = b.cap_list[ci];
   const int64_t cap = b.moves_cap;
@@ -728,7 +748,7 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
     for (int m = 0; m < M && m < MMAX; ++m) b.r_out[(size_t)inst * M + m] = sel<T, MMAX>(r, m);
     b.n_moves[inst] = 0;
     b.diag->err = TRE_EINVAL;
-    return;
+    continue;
   }
   auto emit = [&](int64_t at, int32_t k, int recv, int donor, int kind, int sq) {
     if (at < cap) mv[at] = tre_move{k, (int16_t)recv, (int16_t)donor, (uint8_t)kind, (uint8_t)sq, 0};
@@ -751,16 +771,16 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
     }
     if (nxt >= nf) break;
     u = nxt;
-    const int ent = sent[u];
-    const int recv = srcv[u];
-    const int kind = skind[u];
+    const TickRec tr = srec[u];
+    const int recv = tr.recv;
+    const int kind = tr.kind;
     const int32_t k = swin[u];
     ++u;
-    if (ent < 0) continue;
-    const uint32_t usable = avail & sdm[ent];
+    if (recv < 0) continue;
+    const uint32_t usable = avail & tr.dm;
     const int need = unit ? 1 : sel<T, MMAX>(g, recv);
     if (free_pool < need && !usable) continue;
-    unsigned long long pk = spk[ent];
+    unsigned long long pk = tr.pk;
     if (unit) {
       const int n_pool = (int)(free_pool < Kp ? free_pool : Kp);
       for (int q = 0; q < n_pool; ++q) emit(nm + q, k, recv, -1, kind, q);
@@ -797,7 +817,7 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
 #pragma unroll
       for (int m = 0; m < MMAX; ++m) taken[m] = 0;
       unsigned long long order = pk;
-      uint32_t left = avail & sdm[ent];
+      uint32_t left = avail & tr.dm;
       while (f < need && left) {
         const int m = (int)(order & 15);
         order >>= 4;
@@ -829,6 +849,7 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
   for (int m = 0; m < M && m < MMAX; ++m) b.r_out[(size_t)inst * M + m] = sel<T, MMAX>(r, m);
   b.n_moves[inst] = nm;
   if (nm > cap) b.diag->err = TRE_EOVERFLOW;
+  }
 }
 
 constexpr size_t kStageMax = 160 * 1024;
@@ -899,12 +920,14 @@ cudaError_t walk_thread_launch(const WalkBatch<T>& b, WalkWs& w, size_t smem, cu
       const int n_ent = b.ent_base[i + 1] - b.ent_base[i];
       const int64_t nf = (int64_t)b.series_K[i] * b.series_win[i] / b.fast_ms;
       if (nf >= 32767) ok = false;
-      const size_t need = (size_t)n_ent * 12 + (size_t)nf * (4 + 2 + 2) + ((nf + 15) & ~15) +
-                          (size_t)(b.M + 1) * (nf + 1) * 2 + 64;
+      const size_t need = (size_t)nf * sizeof(TickRec) + (size_t)((nf + 3) & ~3) * 4 +
+                          (size_t)(b.M + 1) * (nf + 1) * 2;
       jsmem = std::max(jsmem, need);
     }
     if (ok && jsmem <= kStageMax) {
-      k_walk_jump<T, MMAX><<<b.n_series * b.n_tau, 32, jsmem, s>>>(b, w.recv, w.packed, w.dmask);
+      const int warps = std::min(8, std::max(1, b.n_cap));
+      k_walk_jump<T, MMAX><<<b.n_series * b.n_tau, 32 * warps, jsmem, s>>>(b, w.recv, w.packed,
+                                                                           w.dmask);
       return cudaGetLastError();
     }
   }
