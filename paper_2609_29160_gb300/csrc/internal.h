@@ -85,7 +85,7 @@ template <class T> struct SeriesTable {
   int32_t K[kMaxSeries];
   int32_t win[kMaxSeries];
   T alpha[kMaxSeries];            // per series, used when the per-model alpha is null
-  int32_t seg_len[kMaxSeries];    // smoothing segment length of the series
+  int32_t seg_len[kMaxSeries];    // smoothing chunk length of the series
   int32_t seg_base[kMaxSeries + 1];  // prefix sum of segments per series
 };
 // fill seg_len / seg_base from K (returns the total segment count)
@@ -93,13 +93,11 @@ template <class T> int series_segments(SeriesTable<T>& t);
 
 // ---- score.cu -------------------------------------------------------------
 template <class T> struct ScoreWs {
-  T* raw;                      // Eq. 1 value per element (idle windows hold junk)
-  T *sum_m, *sum_c, *sum_ci;   // per-(segment, model) affine summaries
-  int32_t* sum_h;
-  T* start_S;                  // start state of the stored trajectory
+  T* raw;                      // Eq. 1 value per element (idle windows: a marker NaN)
+  T* start_S;                  // per (segment, model): state the stored run started from
   int32_t* start_init;
-  T *end_S, *end_S2;           // end states (double buffered)
-  int32_t *end_init, *end_init2;
+  T* end_S;                    // per (segment, model): state after the segment
+  int32_t* end_init;
   int cap_seg;                 // segments the arrays hold (per model)
 };
 template <class T> void score_ws_layout(Arena& a, int M, int64_t elems, int n_seg, ScoreWs<T>& w);

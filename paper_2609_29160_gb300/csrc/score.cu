@@ -5,18 +5,21 @@
 // smoothing S_k = alpha*raw_k + (1-alpha)*S_{k-1} is a sequential chain per
 // model; to spread it over the GPU and still return exactly the values of the
 // sequential definition (one rounding per operation, in order):
-//   1. each segment of windows computes its affine summary (approximate);
-//   2. a per-model scan of the summaries gives every segment an approximate
-//      start state;
-//   3. every segment runs the exact recurrence from that start;
-//   4. every segment re-runs from its predecessor's computed end until its new
-//      trajectory meets the stored one bit for bit (the recurrence is a
-//      contraction, so they meet after a short stretch; from there on every
-//      value is identical because each step depends only on the previous S);
-//   5. one thread per model walks the segment boundaries in order and repairs
-//      any segment whose start still differs from its predecessor's end.
-// After step 5 each segment's stored trajectory starts from the exact end of
-// the previous one, so the concatenation is the sequential result.
+//   1. the windows of each series are cut into chunks; one thread per (chunk,
+//      model) first runs the recurrence over the B windows before its chunk
+//      ("burn-in", started as if the series began there; B ~ 28 / -ln(1-alpha),
+//      so a start error shrinks by e^-28 before the chunk), records the state
+//      it reached, then runs its chunk from that state and stores the result;
+//   2. one thread per model walks the chunk boundaries in order: a chunk whose
+//      recorded burn-in state equals its predecessor's exact end state (bit
+//      for bit, with the same started/not-started flag) is exact, because
+//      every step depends only on the previous state; any other chunk is run
+//      again from the exact state until its new trajectory meets the stored
+//      one. A chunk whose burn-in reaches window 0 starts from the true initial
+//      state and is exact by construction.
+// The result is therefore the sequential one in every case; the in-order pass
+// only re-runs chunks when a burn-in did not converge (long idle stretches, a
+// tiny alpha), counted in tre_diag.ema_resolved.
 #include <algorithm>
 
 #include "common.cuh"
@@ -67,31 +70,87 @@ __device__ __forceinline__ ModelParams<T> load_params(const SeriesTable<T>& t, i
   return p;
 }
 
-// ---- pass 0: Eq. 1 for every (window, model); idle windows marked ---------
+// Eq. 1 values of idle windows carry this NaN pattern (arithmetic on the GPU
+// only produces the canonical NaN), so the smoothing pass reads one array.
+__device__ __forceinline__ float idle_raw(float) { return __uint_as_float(0xffc0deadu); }
+__device__ __forceinline__ double idle_raw(double) {
+  return __longlong_as_double((long long)0xfff8deaddeadbeefull);
+}
+__device__ __forceinline__ bool is_idle_raw(float r) { return __float_as_uint(r) == 0xffc0deadu; }
+__device__ __forceinline__ bool is_idle_raw(double r) {
+  return (unsigned long long)__double_as_longlong(r) == 0xfff8deaddeadbeefull;
+}
+
+// Walks the elements of all series of a table in one grid-stride loop:
+// element v of the concatenation maps to series s and local index v - vbase.
+template <class T> struct SeriesCursor {
+  int s = 0;
+  int64_t vbase = 0;
+  __device__ __forceinline__ void seek(const SeriesTable<T>& t, int64_t v) {
+    while (s + 1 < t.n && v >= vbase + (int64_t)t.K[s] * t.M) {
+      vbase += (int64_t)t.K[s] * t.M;
+      ++s;
+    }
+  }
+};
+
+__device__ __forceinline__ int model_of(int64_t local, const FastDiv& fm, int M) {
+  if (local <= 0xffffffffll) {
+    const uint32_t x = (uint32_t)local;
+    return (int)(x - fm.div(x) * (uint32_t)M);
+  }
+  return (int)(local % M);
+}
+
+// ---- pass 0: Eq. 1 for every (window, model) of every series ---------------
+constexpr int kEw = 4;   // elements per thread per pass (their loads issued together)
+
 template <class T>
 __global__ void __launch_bounds__(kThreads)
-k_raw(const __grid_constant__ SeriesTable<T> tab, Counts c, const T* __restrict__ w_p,
-      const T* __restrict__ w_q, T* __restrict__ raw, uint8_t* __restrict__ cls) {
-  const int s = blockIdx.y;
+k_raw(const __grid_constant__ SeriesTable<T> tab, int64_t total, FastDiv fm, Counts c,
+      const T* __restrict__ w_p, const T* __restrict__ w_q, T* __restrict__ raw,
+      uint8_t* __restrict__ cls) {
   const int M = tab.M;
-  const int64_t n = (int64_t)tab.K[s] * M;
-  const T dt = div_rn((T)tab.win[s], (T)1000);      // window length in seconds
-  for (int64_t i = (int64_t)blockIdx.x * kThreads + threadIdx.x; i < n;
-       i += (int64_t)gridDim.x * kThreads) {
-    const size_t x = (size_t)(tab.off[s] + i);
-    const int m = (int)((uint32_t)i % (uint32_t)M);
-    const int32_t p = c.P[x], d = c.D[x], a = c.A[x], w = c.W[x];
-    if ((p | d | a | w) == 0) {
-      cls[x] = kIdle;
-      continue;
+  SeriesCursor<T> cur;
+  const int64_t stride = (int64_t)gridDim.x * kThreads;
+  for (int64_t v0 = (int64_t)blockIdx.x * kThreads + threadIdx.x; v0 < total;
+       v0 += stride * kEw) {
+    size_t x[kEw];
+    int m[kEw], sr[kEw];
+    int32_t p[kEw], d[kEw], a[kEw], w[kEw];
+#pragma unroll
+    for (int u = 0; u < kEw; ++u) {
+      const int64_t v = v0 + u * stride;
+      sr[u] = -1;
+      if (v < total) {
+        cur.seek(tab, v);
+        sr[u] = cur.s;
+        const int64_t local = v - cur.vbase;
+        x[u] = (size_t)(tab.off[cur.s] + local);
+        m[u] = model_of(local, fm, M);
+        p[u] = c.P[x[u]];
+        d[u] = c.D[x[u]];
+        a[u] = c.A[x[u]];
+        w[u] = c.W[x[u]];
+      }
     }
-    const T r_pre = div_rn(from_i32<T>(p), dt);
-    const T r_dec = div_rn(from_i32<T>(d), dt);
-    const T num = add_rn(mul_rn(w_p[m], r_pre), r_dec);
-    T den = add_rn(from_i32<T>(a), mul_rn(w_q[m], from_i32<T>(w)));
-    if (den < (T)1) den = (T)1;                       // demand floor of one request
-    raw[x] = div_rn(num, den);
-    cls[x] = kNom;
+#pragma unroll
+    for (int u = 0; u < kEw; ++u) {
+      if (sr[u] < 0) continue;
+      if ((p[u] | d[u] | a[u] | w[u]) == 0) {
+        cls[x[u]] = kIdle;
+        raw[x[u]] = idle_raw((T)0);
+        continue;
+      }
+      const T dt = div_rn((T)tab.win[sr[u]], (T)1000);   // window length in seconds
+      const T r_pre = div_rn(from_i32<T>(p[u]), dt);
+      const T r_dec = div_rn(from_i32<T>(d[u]), dt);
+      const T num = add_rn(mul_rn(w_p[m[u]], r_pre), r_dec);
+      T den = add_rn(from_i32<T>(a[u]), mul_rn(w_q[m[u]], from_i32<T>(w[u])));
+      if (den < (T)1) den = (T)1;                       // demand floor of one request
+      raw[x[u]] = div_rn(num, den);
+      cls[x[u]] = kNom;
+    }
   }
 }
 
@@ -121,125 +180,12 @@ __device__ __forceinline__ void load_batch(const T* __restrict__ raw, const uint
   }
 }
 
-// ---- pass 1: affine summary of each segment -------------------------------
-template <class T>
-__global__ void __launch_bounds__(kThreads)
-k_summary(const __grid_constant__ SeriesTable<T> tab, const T* __restrict__ raw,
-          const uint8_t* __restrict__ cls, const T* __restrict__ alpha, T* sm, T* sc, T* sci,
-          int32_t* sh) {
-  const int M = tab.M;
-  const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
-  if (t >= (int64_t)tab.seg_base[tab.n] * M) return;
-  const int m = (int)(t % M);
-  const int seg = (int)(t / M);
-  const int s = series_of_seg(tab, seg);
-  const int L = tab.seg_len[s];
-  const int64_t k0 = (int64_t)(seg - tab.seg_base[s]) * L, k1 = min64(k0 + L, tab.K[s]);
-  const T a = alpha ? alpha[m] : tab.alpha[s];
-  const T b = sub_rn<T>((T)1, a);
-  const size_t base = (size_t)tab.off[s] + m;
-  T mm = (T)1, cc = (T)0, ci = (T)0;
-  int h = 0;
-  T r[kBatch], rn[kBatch];
-  uint8_t c[kBatch], cn[kBatch];
-  load_batch(raw, cls, base, M, k0, k1, r, c);
-  for (int64_t k = k0; k < k1; k += kBatch) {
-    // next batch in flight while this one is folded
-    load_batch(raw, cls, base, M, k + kBatch, k1, rn, cn);
-#pragma unroll
-    for (int j = 0; j < kBatch; ++j) {
-      if (c[j] == kIdle) continue;
-      const T ar = a * r[j];
-      ci = h ? ci * b + ar : r[j];
-      cc = cc * b + ar;
-      mm = mm * b;
-      h = 1;
-    }
-#pragma unroll
-    for (int j = 0; j < kBatch; ++j) {
-      r[j] = rn[j];
-      c[j] = cn[j];
-    }
-  }
-  sm[t] = mm;
-  sc[t] = cc;
-  sci[t] = ci;
-  sh[t] = h;
-}
-
-template <class T> struct Sum {
-  T m, c, ci;
-  int h;
-};
-
-template <class T> __device__ __forceinline__ Sum<T> combine(const Sum<T>& a, const Sum<T>& b) {
-  if (!b.h) return a;
-  if (!a.h) return b;
-  Sum<T> r;
-  r.m = a.m * b.m;
-  r.c = a.c * b.m + b.c;
-  r.ci = a.ci * b.m + b.c;
-  r.h = 1;
-  return r;
-}
-
-template <class T> __device__ __forceinline__ void apply(const Sum<T>& u, T& S, int& init) {
-  if (!u.h) return;
-  S = init ? u.m * S + u.c : u.ci;
-  init = 1;
-}
-
-// ---- pass 2: per-(series, model) exclusive scan -> approximate starts ------
-template <class T>
-__global__ void k_starts(const __grid_constant__ SeriesTable<T> tab, const T* sm, const T* sc,
-                         const T* sci, const int32_t* sh, const T* S_carry,
-                         const uint8_t* init_carry, T* start_S, int32_t* start_init) {
-  const int M = tab.M;
-  const int w = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
-  if (w >= tab.n * M) return;
-  const int s = w / M, m = w % M;
-  const int lane = threadIdx.x & 31;
-  const int n_seg = tab.seg_base[s + 1] - tab.seg_base[s];
-  const int per = (n_seg + 31) / 32;
-  const int s0 = lane * per, s1 = min(n_seg, s0 + per);
-  const size_t g0 = (size_t)tab.seg_base[s] * M + m;
-  Sum<T> agg{(T)1, (T)0, (T)0, 0};
-  for (int q = s0; q < s1; ++q) {
-    const size_t x = g0 + (size_t)q * M;
-    agg = combine(agg, Sum<T>{sm[x], sc[x], sci[x], sh[x]});
-  }
-  Sum<T> inc = agg;
-  for (int o = 1; o < 32; o <<= 1) {
-    Sum<T> v;
-    v.m = __shfl_up_sync(0xffffffffu, inc.m, o);
-    v.c = __shfl_up_sync(0xffffffffu, inc.c, o);
-    v.ci = __shfl_up_sync(0xffffffffu, inc.ci, o);
-    v.h = __shfl_up_sync(0xffffffffu, inc.h, o);
-    if (lane >= o) inc = combine(v, inc);
-  }
-  Sum<T> exc;
-  exc.m = __shfl_up_sync(0xffffffffu, inc.m, 1);
-  exc.c = __shfl_up_sync(0xffffffffu, inc.c, 1);
-  exc.ci = __shfl_up_sync(0xffffffffu, inc.ci, 1);
-  exc.h = __shfl_up_sync(0xffffffffu, inc.h, 1);
-  if (lane == 0) exc = Sum<T>{(T)1, (T)0, (T)0, 0};
-  int init = (init_carry && init_carry[m]) ? 1 : 0;
-  T S = init ? S_carry[m] : (T)0;
-  apply(exc, S, init);
-  for (int q = s0; q < s1; ++q) {
-    const size_t x = g0 + (size_t)q * M;
-    start_S[x] = S;
-    start_init[x] = init;
-    apply(Sum<T>{sm[x], sc[x], sci[x], sh[x]}, S, init);
-  }
-}
-
 // Run windows [k0, k1) of model m exactly from (S, init), writing S and, with
 // `with_z`, Z and the region (idle windows keep their class). With `verify`,
 // stop at the first window whose new S equals the stored one with the same
 // init state: from there the stored trajectory is the one this start produces.
 // Returns true if it stopped early.
-template <class T>
+template <class T, bool WRITE = true>
 __device__ __forceinline__ bool run_segment(size_t base, int M, int64_t k0, int64_t k1,
                                             const T* __restrict__ raw, const ModelParams<T>& q,
                                             T& S, int& init, bool verify, int stored_init,
@@ -270,6 +216,7 @@ __device__ __forceinline__ bool run_segment(size_t base, int M, int64_t k0, int6
         stored_init = 1;
       }
       if (verify && init == stored_init && same_bits(S, old[j])) return true;
+      if (!WRITE) continue;
       const size_t x = base + (size_t)(k + j) * M;
       const T Sv = init ? S : (T)0;
       S_out[x] = Sv;
@@ -288,14 +235,76 @@ __device__ __forceinline__ bool run_segment(size_t base, int M, int64_t k0, int6
   return false;
 }
 
-// ---- pass 3: run every segment from its approximate start -------------------
-template <class T>
-__global__ void __launch_bounds__(kThreads)
-k_run(const __grid_constant__ SeriesTable<T> tab, const T* __restrict__ raw, const T* alpha,
-      const T* theta, const T* tau_crit, const T* tau_surp, const T* start_S,
-      const int32_t* start_init, T* end_S, int32_t* end_init, T* S_out, T* Z_out, uint8_t* cls) {
+// ---- pass 1: burn-in and chunk run, one thread per (chunk, model) ----------
+// Each thread streams its model's windows through its own slots of a shared
+// memory ring with asynchronous copies (cp.async, kStages groups of kBlk
+// windows in flight), so the dependent chain reads shared memory while the
+// next windows are on their way.
+constexpr int kEmaThreads = 32;    // few chains in all: spread them over every SM
+constexpr int kBlk = 16;           // windows per copy group
+constexpr int kStages = 8;         // copy groups in flight
+constexpr int kRingStride = 64;    // chunk and burn-in lengths are multiples of this
+constexpr int kMaxBurn = 16384;    // burn-in cap (tiny alpha: the in-order pass repairs)
+
+template <int BYTES>
+__device__ __forceinline__ void cp_async(void* smem, const void* gmem) {
+  const unsigned sa = (unsigned)__cvta_generic_to_shared(smem);
+  asm volatile("cp.async.ca.shared.global [%0], [%1], %2;\n" ::"r"(sa), "l"(gmem), "n"(BYTES)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;\n" ::: "memory");
+}
+template <int N> __device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
+}
+
+// One group of kBlk windows of the chain, read from its ring stage. FULL: all
+// kBlk windows exist; STARTED: the chain has seen a non-idle window already
+// (then the step is branch-free); STORE: write S (and Z, regions with WITHZ).
+template <class T, bool FULL, bool STARTED, bool STORE, bool WITHZ>
+__device__ __forceinline__ void ema_group(const T* src, int n, const ModelParams<T>& q, T& S,
+                                          int& init, T*& sp, int M, T* S_out, T* Z_out,
+                                          uint8_t* cls) {
+  T r[kBlk];
+#pragma unroll
+  for (int j = 0; j < kBlk; ++j) r[j] = src[j * kEmaThreads];
+#pragma unroll
+  for (int j = 0; j < kBlk; ++j) {
+    if (!FULL && j >= n) break;
+    const bool idle = is_idle_raw(r[j]);
+    if (STARTED) {
+      const T nxt = add_rn(mul_rn(q.a, r[j]), mul_rn(q.b, S));
+      S = idle ? S : nxt;
+    } else if (!idle) {
+      S = init ? add_rn(mul_rn(q.a, r[j]), mul_rn(q.b, S)) : r[j];
+      init = 1;
+    }
+    if (STORE) {
+      const T Sv = (STARTED || init) ? S : (T)0;
+      *sp = Sv;
+      if (WITHZ) {
+        const size_t x = (size_t)(sp - S_out);
+        const T Z = div_rn(Sv, q.th);
+        Z_out[x] = Z;
+        if (!idle) cls[x] = Z < q.tc ? kCrit : (Z > q.ts ? kSurp : kNom);
+      }
+      sp += M;
+    }
+  }
+}
+
+template <class T, bool WITHZ>
+__global__ void __launch_bounds__(kEmaThreads)
+k_ema(const __grid_constant__ SeriesTable<T> tab, const T* __restrict__ raw, const T* alpha,
+      const T* theta, const T* tau_crit, const T* tau_surp, const T* S_carry,
+      const uint8_t* init_carry, T* __restrict__ b_S, int32_t* __restrict__ b_init,
+      T* __restrict__ e_S, int32_t* __restrict__ e_init, T* __restrict__ S_out,
+      T* __restrict__ Z_out, uint8_t* __restrict__ cls) {
+  __shared__ T ring[kStages * kBlk * kEmaThreads];
   const int M = tab.M;
-  const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+  const int lane = threadIdx.x;
+  const int64_t t = (int64_t)blockIdx.x * kEmaThreads + lane;
   if (t >= (int64_t)tab.seg_base[tab.n] * M) return;
   const int m = (int)(t % M);
   const int seg = (int)(t / M);
@@ -303,72 +312,160 @@ k_run(const __grid_constant__ SeriesTable<T> tab, const T* __restrict__ raw, con
   const ModelParams<T> q = load_params(tab, s, m, alpha, theta, tau_crit, tau_surp);
   const int L = tab.seg_len[s];
   const int64_t k0 = (int64_t)(seg - tab.seg_base[s]) * L, k1 = min64(k0 + L, tab.K[s]);
-  T S = start_S[t];
-  int init = start_init[t];
-  run_segment<T>((size_t)tab.off[s] + m, M, k0, k1, raw, q, S, init, false, 0, S_out, Z_out, cls,
-                 theta != nullptr);
-  end_S[t] = S;
-  end_init[t] = init;
-}
-
-// ---- pass 4: parallel verification from the predecessor's computed end ------
-template <class T>
-__global__ void __launch_bounds__(kThreads)
-k_verify(const __grid_constant__ SeriesTable<T> tab, const T* __restrict__ raw, const T* alpha,
-         const T* theta, const T* tau_crit, const T* tau_surp, T* start_S, int32_t* start_init,
-         const T* end_S, const int32_t* end_init, T* end_S2, int32_t* end_init2, T* S_out,
-         T* Z_out, uint8_t* cls, tre_diag* diag) {
-  const int M = tab.M;
-  const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
-  if (t >= (int64_t)tab.seg_base[tab.n] * M) return;
-  const int m = (int)(t % M);
-  const int seg = (int)(t / M);
-  const int s = series_of_seg(tab, seg);
-  T eS = end_S[t];
-  int eI = end_init[t];
-  if (seg > tab.seg_base[s]) {
-    const size_t p = t - M;
-    T S = end_S[p];
-    int init = end_init[p];
-    if (init != start_init[t] || !same_bits(S, start_S[t])) {
-      const ModelParams<T> q = load_params(tab, s, m, alpha, theta, tau_crit, tau_surp);
-      const int L = tab.seg_len[s];
-      const int64_t k0 = (int64_t)(seg - tab.seg_base[s]) * L, k1 = min64(k0 + L, tab.K[s]);
-      const int stored_init = start_init[t];
-      start_S[t] = S;
-      start_init[t] = init;
-      const bool met = run_segment<T>((size_t)tab.off[s] + m, M, k0, k1, raw, q, S, init, true,
-                                      stored_init, S_out, Z_out, cls, theta != nullptr);
-      if (!met) {
-        eS = S;
-        eI = init;
-      }
-      atomicAdd(&diag->ema_resolved, 1ull);
+  // burn-in length: (1 - alpha)^B <= e^-28, in whole ring strides
+  int B = kMaxBurn;
+  {
+    const float a = (float)q.a;
+    if (a >= 1.f) B = kRingStride;
+    else if (a > 0.f) {
+      const float x = 28.f / -log1pf(-a);
+      if (x < (float)kMaxBurn) B = (int)x + 1;
     }
+    B = (B + kRingStride - 1) / kRingStride * kRingStride;
   }
-  end_S2[t] = eS;
-  end_init2[t] = eI;
+  int64_t kb = k0 - B;
+  T S = (T)0;
+  int init = 0;
+  if (kb <= 0) {   // the burn-in reaches the series start: begin from the true state
+    kb = 0;
+    init = (init_carry && init_carry[m]) ? 1 : 0;
+    S = init ? S_carry[m] : (T)0;
+  }
+  const size_t base = (size_t)tab.off[s] + m;
+  const int n_grp = (int)((k1 - kb + kBlk - 1) / kBlk);
+  const int burn_grp = (int)((k0 - kb) / kBlk);
+  // group g holds windows kb + g*kBlk .. + kBlk-1 in stage g % kStages
+  const T* src_next = raw + base + (size_t)kb * M;
+  const size_t step = (size_t)M;
+  auto issue = [&](int g) {
+    if (g < n_grp) {
+      T* dst = ring + (size_t)(g % kStages) * kBlk * kEmaThreads + lane;
+      if (g + 1 < n_grp) {
+#pragma unroll
+        for (int j = 0; j < kBlk; ++j) {
+          cp_async<sizeof(T)>(dst + j * kEmaThreads, src_next);
+          src_next += step;
+        }
+      } else {
+        const int n = (int)(k1 - (kb + (int64_t)g * kBlk));
+#pragma unroll
+        for (int j = 0; j < kBlk; ++j)
+          if (j < n) {
+            cp_async<sizeof(T)>(dst + j * kEmaThreads, src_next);
+            src_next += step;
+          }
+      }
+    }
+    cp_async_commit();
+  };
+#pragma unroll
+  for (int g = 0; g < kStages - 1; ++g) issue(g);
+  T* sp = S_out + base + (size_t)k0 * M;
+  auto stage_of = [&](int g) { return ring + (size_t)(g % kStages) * kBlk * kEmaThreads + lane; };
+  int g = 0;
+  // burn-in: full groups, nothing stored
+  for (; g < burn_grp; ++g) {
+    issue(g + kStages - 1);
+    cp_async_wait<kStages - 1>();
+    if (init) ema_group<T, true, true, false, WITHZ>(stage_of(g), kBlk, q, S, init, sp, M, S_out, Z_out, cls);
+    else ema_group<T, true, false, false, WITHZ>(stage_of(g), kBlk, q, S, init, sp, M, S_out, Z_out, cls);
+  }
+  b_S[t] = S;
+  b_init[t] = init;
+  // the chunk: full groups, then the last (possibly partial) one
+  for (; g + 1 < n_grp; ++g) {
+    issue(g + kStages - 1);
+    cp_async_wait<kStages - 1>();
+    if (init) ema_group<T, true, true, true, WITHZ>(stage_of(g), kBlk, q, S, init, sp, M, S_out, Z_out, cls);
+    else ema_group<T, true, false, true, WITHZ>(stage_of(g), kBlk, q, S, init, sp, M, S_out, Z_out, cls);
+  }
+  cp_async_wait<0>();
+  {
+    const int n = (int)(k1 - (kb + (int64_t)g * kBlk));
+    ema_group<T, false, false, true, WITHZ>(stage_of(g), n, q, S, init, sp, M, S_out, Z_out, cls);
+  }
+  e_S[t] = S;
+  e_init[t] = init;
 }
 
-// ---- pass 5: in-order repair, one thread per (series, model) ---------------
+// ---- pass 2: boundary check and repair, one warp per (series, model) -------
+// Lanes check 32 chunk boundaries at a time. A chunk whose burn-in state
+// differs from its predecessor's end state is run again from that end until its
+// new trajectory meets the stored one; first as a dry run, so that a chunk is
+// rewritten only when every chunk before it keeps its end state. A chunk whose
+// re-run never meets its stored trajectory changes its end state, and from the
+// next chunk on the boundaries are walked in order by one lane.
 template <class T>
 __global__ void k_resolve(const __grid_constant__ SeriesTable<T> tab, const T* __restrict__ raw,
                           const T* alpha, const T* theta, const T* tau_crit, const T* tau_surp,
-                          const T* start_S, const int32_t* start_init, const T* end_S,
-                          const int32_t* end_init, T* S_out, T* Z_out, uint8_t* cls,
+                          const T* start_S, const int32_t* start_init, T* end_S,
+                          int32_t* end_init, T* S_out, T* Z_out, uint8_t* cls,
                           T* S_carry, uint8_t* init_carry, tre_diag* diag) {
   const int M = tab.M;
-  const int w = blockIdx.x * blockDim.x + threadIdx.x;
+  const int w = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
   if (w >= tab.n * M) return;
+  const int lane = threadIdx.x & 31;
   const int s = w / M, m = w % M;
   const int n_seg = tab.seg_base[s + 1] - tab.seg_base[s];
   if (n_seg == 0) return;
-  const ModelParams<T> q = load_params(tab, s, m, alpha, theta, tau_crit, tau_surp);
-  const int L = tab.seg_len[s];
   const size_t g0 = (size_t)tab.seg_base[s] * M + m;
-  T S = end_S[g0];
-  int init = end_init[g0];
-  for (int q0 = 1; q0 < n_seg; q0 += kBatch) {
+  const ModelParams<T> q = load_params(tab, s, m, alpha, theta, tau_crit, tau_surp);
+  const bool with_z = theta != nullptr;
+  const int L = tab.seg_len[s];
+  const size_t base = (size_t)tab.off[s] + m;
+  int first_bad = n_seg;   // the in-order walk starts here
+  for (int c0 = 1; c0 < n_seg; c0 += 32) {
+    const int c = c0 + lane;
+    bool bad = false, moved = false;
+    T pS = (T)0;
+    int pI = 0, sI = 0;
+    int64_t k0 = 0, k1 = 0;
+    if (c < n_seg) {
+      const size_t x = g0 + (size_t)c * M;
+      pS = end_S[x - M];
+      pI = end_init[x - M];
+      sI = start_init[x];
+      bad = sI != pI || !same_bits(start_S[x], pS);
+      k0 = (int64_t)c * L;
+      k1 = min64(k0 + L, tab.K[s]);
+    }
+    if (bad) {
+      T S = pS;
+      int init = pI;
+      moved = !run_segment<T, false>(base, M, k0, k1, raw, q, S, init, true, sI, S_out, Z_out,
+                                     cls, with_z);
+    }
+    const unsigned mv = __ballot_sync(0xffffffffu, moved);
+    const int lim = mv ? c0 + __ffs(mv) - 1 : n_seg;   // predecessors final up to here
+    if (bad && c <= lim) {
+      T S = pS;
+      int init = pI;
+      const bool met = run_segment<T>(base, M, k0, k1, raw, q, S, init, true, sI, S_out, Z_out,
+                                      cls, with_z);
+      if (!met) {
+        end_S[g0 + (size_t)c * M] = S;
+        end_init[g0 + (size_t)c * M] = init;
+      }
+      atomicAdd(&diag->ema_resolved, 1ull);
+    }
+    if (mv) {
+      first_bad = lim + 1;
+      break;
+    }
+  }
+  __syncwarp();
+  if (lane != 0) return;
+  const size_t last = g0 + (size_t)(min(first_bad, n_seg) - 1) * M;
+  T S = end_S[last];
+  int init = end_init[last];
+  if (first_bad >= n_seg) {
+    if (S_carry) {
+      S_carry[m] = S;
+      init_carry[m] = (uint8_t)init;
+    }
+    return;
+  }
+  for (int q0 = first_bad; q0 < n_seg; q0 += kBatch) {
     // load the boundary states of a batch of segments ahead of the checks
     T bS[kBatch], bE[kBatch];
     int bI[kBatch], bEI[kBatch];
@@ -410,25 +507,46 @@ __global__ void k_resolve(const __grid_constant__ SeriesTable<T> tab, const T* _
 // ---- Z and regions from S for every series ---------------------------------
 template <class T>
 __global__ void __launch_bounds__(kThreads)
-k_normalize(const __grid_constant__ SeriesTable<T> tab, const T* S, const uint8_t* idle_cls,
-            const T* theta, const T* tau_crit, T tau_crit_v, const T* tau_surp, T* Z,
-            uint8_t* cls) {
-  const int s = blockIdx.y;
+k_normalize(const __grid_constant__ SeriesTable<T> tab, int64_t total, FastDiv fm, const T* S,
+            const uint8_t* idle_cls, const T* theta, const T* tau_crit, T tau_crit_v,
+            const T* tau_surp, T* Z, uint8_t* cls) {
   const int M = tab.M;
-  const int64_t n = (int64_t)tab.K[s] * M;
-  for (int64_t i = (int64_t)blockIdx.x * kThreads + threadIdx.x; i < n;
-       i += (int64_t)gridDim.x * kThreads) {
-    const size_t x = (size_t)(tab.off[s] + i);
-    const int m = (int)((uint32_t)i % (uint32_t)M);
-    const T z = div_rn(S[x], theta[(size_t)s * M + m]);
-    if (Z) Z[x] = z;
-    if (cls) {
-      uint8_t c;
-      if (idle_cls[x] == kIdle) c = kIdle;
-      else if (z < (tau_crit ? tau_crit[m] : tau_crit_v)) c = kCrit;
-      else if (z > tau_surp[m]) c = kSurp;
-      else c = kNom;
-      cls[x] = c;
+  SeriesCursor<T> cur;
+  const int64_t stride = (int64_t)gridDim.x * kThreads;
+  for (int64_t v0 = (int64_t)blockIdx.x * kThreads + threadIdx.x; v0 < total;
+       v0 += stride * kEw) {
+    size_t x[kEw];
+    int m[kEw], sr[kEw];
+    T sv[kEw], th[kEw];
+    uint8_t ic[kEw];
+#pragma unroll
+    for (int u = 0; u < kEw; ++u) {
+      const int64_t v = v0 + u * stride;
+      sr[u] = -1;
+      if (v < total) {
+        cur.seek(tab, v);
+        sr[u] = cur.s;
+        const int64_t local = v - cur.vbase;
+        x[u] = (size_t)(tab.off[cur.s] + local);
+        m[u] = model_of(local, fm, M);
+        sv[u] = S[x[u]];
+        th[u] = theta[(size_t)cur.s * M + m[u]];
+        ic[u] = cls ? idle_cls[x[u]] : (uint8_t)0;
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kEw; ++u) {
+      if (sr[u] < 0) continue;
+      const T z = div_rn(sv[u], th[u]);
+      if (Z) Z[x[u]] = z;
+      if (cls) {
+        uint8_t c;
+        if (ic[u] == kIdle) c = kIdle;
+        else if (z < (tau_crit ? tau_crit[m[u]] : tau_crit_v)) c = kCrit;
+        else if (z > tau_surp[m[u]]) c = kSurp;
+        else c = kNom;
+        cls[x[u]] = c;
+      }
     }
   }
 }
@@ -455,15 +573,26 @@ __global__ void k_receiver(int M, int K, const T* Z, const uint8_t* cls, int32_t
   if (lane == 0) recv[k] = best;
 }
 
-template <class T> int64_t max_elems(const SeriesTable<T>& t) {
-  int64_t mx = 0;
-  for (int s = 0; s < t.n; ++s) mx = std::max<int64_t>(mx, (int64_t)t.K[s] * t.M);
-  return mx;
+template <class T> int64_t total_elems(const SeriesTable<T>& t) {
+  int64_t n = 0;
+  for (int s = 0; s < t.n; ++s) n += (int64_t)t.K[s] * t.M;
+  return n;
 }
 
 unsigned blocks_for(int64_t n, int cap) {
   int64_t b = (n + kThreads - 1) / kThreads;
   return (unsigned)std::max<int64_t>(1, std::min<int64_t>(b, cap));
+}
+
+int sm_count() {
+  static int n = 0;
+  if (!n) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1)
+      n = 148;
+  }
+  return n;
 }
 
 }  // namespace
@@ -472,14 +601,11 @@ template <class T> int series_segments(SeriesTable<T>& t) {
   int total = 0;
   for (int s = 0; s < t.n; ++s) {
     const int K = t.K[s];
-    // Two trajectories of the smoothing that start a few dozen ulps apart meet
-    // after about 4 / alpha windows; segments about twice that long let the
-    // verification pass meet the stored trajectory inside one segment.
-    const double a = (double)t.alpha[s];
-    int base = 64;
-    while (base < 512 && !(a > 0 && (double)base * a >= 8.0)) base *= 2;
-    int L = (K + 1023) / 1024;
-    L = L < base ? base : L;
+    // chunks of 256 windows (longer for very long series, to bound the count);
+    // a multiple of the smoothing pass's ring stride
+    int L = 256;
+    const int need = (K + 2047) / 2048;
+    if (need > L) L = (need + kRingStride - 1) / kRingStride * kRingStride;
     t.seg_len[s] = L;
     t.seg_base[s] = total;
     total += (K + L - 1) / L;
@@ -492,16 +618,10 @@ template <class T> void score_ws_layout(Arena& a, int M, int64_t elems, int n_se
   w.raw = a.take<T>((size_t)std::max<int64_t>(elems, 1));
   w.cap_seg = std::max(n_seg, 1);
   const size_t n = (size_t)w.cap_seg * M;
-  w.sum_m = a.take<T>(n);
-  w.sum_c = a.take<T>(n);
-  w.sum_ci = a.take<T>(n);
-  w.sum_h = a.take<int32_t>(n);
   w.start_S = a.take<T>(n);
   w.start_init = a.take<int32_t>(n);
   w.end_S = a.take<T>(n);
   w.end_init = a.take<int32_t>(n);
-  w.end_S2 = a.take<T>(n);
-  w.end_init2 = a.take<int32_t>(n);
 }
 
 template <class T>
@@ -513,24 +633,24 @@ cudaError_t launch_score(const SeriesTable<T>& tab, const int32_t* P, const int3
   const int M = tab.M;
   const int n_seg = tab.seg_base[tab.n];
   if (n_seg > w.cap_seg) return cudaErrorInvalidValue;
-  const int64_t mx = max_elems(tab);
-  if (mx == 0) return cudaSuccess;
+  const int64_t total = total_elems(tab);
+  if (total == 0) return cudaSuccess;
   const Counts c{P, D, A, W};
-  dim3 ge(blocks_for(mx, 2048), tab.n);
-  k_raw<T><<<ge, kThreads, 0, s>>>(tab, c, w_p, w_q, w.raw, cls);
+  k_raw<T><<<blocks_for(total, sm_count() * 8), kThreads, 0, s>>>(tab, total, FastDiv(M), c, w_p,
+                                                                  w_q, w.raw, cls);
   const int64_t segs = (int64_t)n_seg * M;
-  const unsigned g = (unsigned)((segs + kThreads - 1) / kThreads);
-  k_summary<T><<<g, kThreads, 0, s>>>(tab, w.raw, cls, alpha, w.sum_m, w.sum_c, w.sum_ci, w.sum_h);
+  const unsigned g = (unsigned)((segs + kEmaThreads - 1) / kEmaThreads);
+  if (theta)
+    k_ema<T, true><<<g, kEmaThreads, 0, s>>>(tab, w.raw, alpha, theta, tau_crit, tau_surp,
+                                             S_carry, init_carry, w.start_S, w.start_init,
+                                             w.end_S, w.end_init, S, Z, cls);
+  else
+    k_ema<T, false><<<g, kEmaThreads, 0, s>>>(tab, w.raw, alpha, theta, tau_crit, tau_surp,
+                                              S_carry, init_carry, w.start_S, w.start_init,
+                                              w.end_S, w.end_init, S, Z, cls);
   const int warps = tab.n * M;
-  k_starts<T><<<(warps + 3) / 4, 128, 0, s>>>(tab, w.sum_m, w.sum_c, w.sum_ci, w.sum_h, S_carry,
-                                              init_carry, w.start_S, w.start_init);
-  k_run<T><<<g, kThreads, 0, s>>>(tab, w.raw, alpha, theta, tau_crit, tau_surp, w.start_S,
-                                  w.start_init, w.end_S, w.end_init, S, Z, cls);
-  k_verify<T><<<g, kThreads, 0, s>>>(tab, w.raw, alpha, theta, tau_crit, tau_surp, w.start_S,
-                                     w.start_init, w.end_S, w.end_init, w.end_S2, w.end_init2, S,
-                                     Z, cls, diag);
-  k_resolve<T><<<(warps + 63) / 64, 64, 0, s>>>(tab, w.raw, alpha, theta, tau_crit, tau_surp,
-                                                w.start_S, w.start_init, w.end_S2, w.end_init2,
+  k_resolve<T><<<(warps + 1) / 2, 64, 0, s>>>(tab, w.raw, alpha, theta, tau_crit, tau_surp,
+                                                w.start_S, w.start_init, w.end_S, w.end_init,
                                                 S, Z, cls, S_carry, init_carry, diag);
   return cudaGetLastError();
 }
@@ -539,11 +659,10 @@ template <class T>
 cudaError_t launch_normalize(const SeriesTable<T>& tab, const T* S, const uint8_t* idle_cls,
                              const T* theta, const T* tau_crit, T tau_crit_v, const T* tau_surp,
                              T* Z, uint8_t* cls, cudaStream_t s) {
-  const int64_t mx = max_elems(tab);
-  if (mx == 0) return cudaSuccess;
-  dim3 g(blocks_for(mx, 1024), tab.n);
-  k_normalize<T><<<g, kThreads, 0, s>>>(tab, S, idle_cls, theta, tau_crit, tau_crit_v, tau_surp,
-                                        Z, cls);
+  const int64_t total = total_elems(tab);
+  if (total == 0) return cudaSuccess;
+  k_normalize<T><<<blocks_for(total, sm_count() * 8), kThreads, 0, s>>>(
+      tab, total, FastDiv(tab.M), S, idle_cls, theta, tau_crit, tau_crit_v, tau_surp, Z, cls);
   return cudaGetLastError();
 }
 
