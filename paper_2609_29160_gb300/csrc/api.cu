@@ -172,7 +172,7 @@ tre_status calibrate_typed(const tre_grid* g, const tre_requests* req, const tre
   ScoreWs<T> sw;
   score_ws_layout<T>(a, M, (int64_t)K * M, tab.seg_base[1], sw);
   CalibWs<T> cw;
-  calib_ws_layout<T>(a, (int64_t)K * M, cw);
+  calib_ws_layout<T>(a, (int64_t)K * M, M, cw);
   bool query;
   tre_status st = ws_check(a, ws, ws_bytes, query);
   if (st != TRE_OK || query) return st;
@@ -339,7 +339,7 @@ tre_status sweep_typed(const tre_sweep_spec* sp, const SweepPlan& pl, const tre_
   ScoreWs<T> sw;
   score_ws_layout<T>(a, M, (int64_t)tot, n_seg, sw);
   CalibWs<T> cw;
-  calib_ws_layout<T>(a, (int64_t)tot, cw);
+  calib_ws_layout<T>(a, (int64_t)tot, tab.n * M, cw);
   WalkBatch<T> b;
   std::memset(&b, 0, sizeof(b));
   b.M = M;

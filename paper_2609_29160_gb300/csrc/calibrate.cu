@@ -27,13 +27,13 @@ namespace tre {
 namespace {
 
 constexpr int kThrTable = 4096;
-constexpr int kNB = 512;            // buckets per level = threads per CTA
+constexpr int kNB = 1024;           // buckets per level = threads per CTA
 constexpr int kWarps = kNB / 32;
 
 template <class T> struct KeyOf;
 template <> struct KeyOf<float> {
   using U = uint32_t;
-  static constexpr int kLevels = 4;   // 31 key bits, >= 9 bits resolved per level
+  static constexpr int kLevels = 4;   // 31 key bits, >= 10 bits resolved per level
 };
 template <> struct KeyOf<double> {
   using U = unsigned long long;
@@ -45,9 +45,16 @@ __device__ __forceinline__ double value_of(unsigned long long k) {
   return __longlong_as_double((long long)k);
 }
 
-// thr[a] = smallest integer n with (double)n >= ok_frac * (double)a
-__global__ void k_thr(double ok_frac, int32_t* thr) {
+// thr[a] = smallest integer n with (double)n >= ok_frac * (double)a; also
+// resets the per-(series, model) candidate key ranges filled by k_pack
+template <class U>
+__global__ void k_thr(double ok_frac, int32_t* thr, int n_sm, U* kmin, U* kmax, uint32_t* ncand) {
   const int a = blockIdx.x * blockDim.x + threadIdx.x;
+  if (a < n_sm) {
+    kmin[a] = ~(U)0;
+    kmax[a] = 0;
+    ncand[a] = 0;
+  }
   if (a >= kThrTable) return;
   const double v = ok_frac * (double)a;
   int32_t t;
@@ -64,36 +71,87 @@ __device__ __forceinline__ bool healthy(uint32_t n_arr, uint32_t n_met, const in
 }
 
 // [K][M] S, class, packed SLO counts of every series -> [M][K] packed keys
-// (0 = not a calibration window) at the series' element offset
+// (0 = not a calibration window) at the series' element offset, plus each
+// (series, model)'s smallest and largest candidate key and candidate count.
+// A CTA transposes one tile of TK windows x TM models (TM = the model count
+// rounded up to a power of two, at most 32; TK * TM = 1024) through shared
+// memory; every thread of a CTA keeps to one model of the tile.
+constexpr int kPackThreads = 256;
+constexpr int kPackTile = 1024;
+struct PackPlan {
+  int lg_tm, tm, lg_tk, tk, m_tiles;
+  int tile_base[kMaxSeries + 1];   // prefix of tiles per series
+};
+
 template <class T>
-__global__ void k_pack(const __grid_constant__ SeriesTable<T> tab, const T* __restrict__ S,
-                       const uint8_t* __restrict__ cls, const unsigned long long* __restrict__ slo,
-                       const int32_t* __restrict__ thr, double ok_frac,
-                       typename KeyOf<T>::U* __restrict__ keys) {
+__global__ void __launch_bounds__(kPackThreads)
+k_pack(const __grid_constant__ SeriesTable<T> tab, const __grid_constant__ PackPlan pp,
+       const T* __restrict__ S, const uint8_t* __restrict__ cls,
+       const unsigned long long* __restrict__ slo, const int32_t* __restrict__ thr,
+       double ok_frac, typename KeyOf<T>::U* __restrict__ keys, typename KeyOf<T>::U* kmin_g,
+       typename KeyOf<T>::U* kmax_g, uint32_t* ncand_g) {
   using U = typename KeyOf<T>::U;
-  __shared__ U tile[32][33];
-  const int s = blockIdx.z;
+  __shared__ U tile[kPackTile + 32];
+  __shared__ U smin[32], smax[32];
+  __shared__ uint32_t scnt[32];
+  int s = 0;
+  while (s + 1 < tab.n && pp.tile_base[s + 1] <= (int)blockIdx.x) ++s;
   const int M = tab.M, K = tab.K[s];
-  const int k0 = blockIdx.x * 32, m0 = blockIdx.y * 32;
-  if (k0 >= K) return;
+  const int t_loc = blockIdx.x - pp.tile_base[s];
+  const int kt = pp.m_tiles == 1 ? t_loc : t_loc / pp.m_tiles;
+  const int k0 = kt * pp.tk, m0 = (t_loc - kt * pp.m_tiles) * pp.tm;
   const size_t off = (size_t)tab.off[s];
-  for (int j = threadIdx.y; j < 32; j += blockDim.y) {
-    const int k = k0 + j, m = m0 + threadIdx.x;
+  const int tid = threadIdx.x;
+  const int mm = tid & (pp.tm - 1);
+  const int m = m0 + mm;
+  if (tid < 32) {
+    smin[tid] = ~(U)0;
+    smax[tid] = 0;
+    scnt[tid] = 0;
+  }
+  U lmin = ~(U)0, lmax = 0;
+  uint32_t lc = 0;
+  const int TKp = pp.tk + 1;   // padded row of the transposed tile
+#pragma unroll
+  for (int j = 0; j < kPackTile / kPackThreads; ++j) {
+    const int e = tid + j * kPackThreads;
+    const int kk = e >> pp.lg_tm;
+    const int k = k0 + kk;
     U v = 0;
     if (k < K && m < M) {
       const size_t x = off + (size_t)k * M + m;
       const unsigned long long c = slo[x];
       const uint32_t n_arr = (uint32_t)c, n_met = (uint32_t)(c >> 32);
       const T sv = S[x];
-      if (cls[x] != kIdle && n_arr >= 1 && sv > (T)0)
-        v = ((U)key_of(sv) << 1) | (U)(healthy(n_arr, n_met, thr, ok_frac) ? 1 : 0);
+      if (cls[x] != kIdle && n_arr >= 1 && sv > (T)0) {
+        const U key = (U)key_of(sv);
+        v = (key << 1) | (U)(healthy(n_arr, n_met, thr, ok_frac) ? 1 : 0);
+        lmin = key < lmin ? key : lmin;
+        lmax = key > lmax ? key : lmax;
+        ++lc;
+      }
     }
-    tile[j][threadIdx.x] = v;
+    tile[mm * TKp + kk] = v;
   }
   __syncthreads();
-  for (int j = threadIdx.y; j < 32; j += blockDim.y) {
-    const int m = m0 + j, k = k0 + threadIdx.x;
-    if (m < M && k < K) keys[off + (size_t)m * K + k] = tile[threadIdx.x][j];
+  if (lc) {
+    atomicMin(&smin[mm], lmin);
+    atomicMax(&smax[mm], lmax);
+    atomicAdd(&scnt[mm], lc);
+  }
+#pragma unroll
+  for (int j = 0; j < kPackTile / kPackThreads; ++j) {
+    const int e = tid + j * kPackThreads;
+    const int r = e >> pp.lg_tk, kk = e & (pp.tk - 1);
+    const int mo = m0 + r, k = k0 + kk;
+    if (mo < M && k < K) keys[off + (size_t)mo * K + k] = tile[r * TKp + kk];
+  }
+  __syncthreads();
+  if (tid < pp.tm && m0 + tid < M && scnt[tid]) {
+    const size_t g = (size_t)s * M + m0 + tid;
+    atomicMin(&kmin_g[g], smin[tid]);
+    atomicMax(&kmax_g[g], smax[tid]);
+    atomicAdd(&ncand_g[g], scnt[tid]);
   }
 }
 
@@ -126,6 +184,7 @@ __device__ __forceinline__ int block_min(int v, int* red) {
 }
 
 constexpr int kFine = 4096;     // buckets of the first histogram
+constexpr int kUnroll = 8;      // keys per thread whose loads are issued together
 constexpr int kCap = 4096;      // most keys the exact pass sorts in shared memory
 
 template <class T> size_t search_smem_bytes() {
@@ -138,7 +197,8 @@ template <class T> size_t search_smem_bytes() {
 template <class T>
 __global__ void __launch_bounds__(kNB)
 k_search(const __grid_constant__ SeriesTable<T> tab, const typename KeyOf<T>::U* __restrict__ keys,
-         double reliability, T* theta, tre_diag* diag) {
+         const typename KeyOf<T>::U* kmin_g, const typename KeyOf<T>::U* kmax_g,
+         const uint32_t* ncand_g, double reliability, T* theta, tre_diag* diag) {
   using U = typename KeyOf<T>::U;
   constexpr int NL = KeyOf<T>::kLevels;
   extern __shared__ __align__(16) unsigned char dyn[];
@@ -147,8 +207,6 @@ k_search(const __grid_constant__ SeriesTable<T> tab, const typename KeyOf<T>::U*
   __shared__ int64_t cab_s[NL], hab_s[NL];
   __shared__ int64_t red64[kWarps];
   __shared__ int red32[kWarps];
-  __shared__ U kmin_s, kmax_s;
-  __shared__ unsigned long long ncand_s;
   __shared__ int nsel_s;
   const int M = tab.M;
   const int s = blockIdx.x / M, m = blockIdx.x % M;
@@ -157,39 +215,15 @@ k_search(const __grid_constant__ SeriesTable<T> tab, const typename KeyOf<T>::U*
   const int tid = threadIdx.x, lane = tid & 31;
   const size_t out = (size_t)s * M + m;
 
-  // ---- range of candidate keys -------------------------------------------
-  if (tid == 0) {
-    kmin_s = ~(U)0;
-    kmax_s = 0;
-    ncand_s = 0;
-  }
-  __syncthreads();
-  {
-    U lmin = ~(U)0, lmax = 0;
-    unsigned long long lc = 0;
-    for (int i = tid; i < K; i += kNB) {
-      const U p = mk[i];
-      if (!p) continue;
-      const U key = p >> 1;
-      lmin = key < lmin ? key : lmin;
-      lmax = key > lmax ? key : lmax;
-      ++lc;
-    }
-    if (lc) {
-      atomicMin(&kmin_s, lmin);
-      atomicMax(&kmax_s, lmax);
-      atomicAdd(&ncand_s, lc);
-    }
-  }
-  __syncthreads();
-  if (ncand_s == 0) {
+  // ---- range of candidate keys (from the packing pass) ---------------------
+  if (ncand_g[out] == 0) {
     if (tid == 0) {
       theta[out] = (T)1;
       atomicAdd(&diag->degenerate_calib, 1ull);
     }
     return;
   }
-  const U kmin = kmin_s, kmax = kmax_s;
+  const U kmin = kmin_g[out], kmax = kmax_g[out];
 
   // ---- fast path -----------------------------------------------------------
   // A fine histogram over [kmin, kmax]; per bucket the exact test at its
@@ -214,14 +248,23 @@ k_search(const __grid_constant__ SeriesTable<T> tab, const typename KeyOf<T>::U*
       fmn[b] = ~(U)0;
     }
     __syncthreads();
-    for (int i = tid; i < K; i += kNB) {
-      const U p = mk[i];
-      if (!p) continue;
-      const U key = p >> 1;
-      const int b = (int)((key - kmin) >> sh);
-      atomicAdd(&fcnt[b], 1);
-      if (p & 1) atomicAdd(&fhl[b], 1);
-      if (key < fmn[b]) atomicMin(&fmn[b], key);
+    for (int i0 = 0; i0 < K; i0 += kNB * kUnroll) {
+      U pv[kUnroll];
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const int i = i0 + u * kNB + tid;
+        pv[u] = i < K ? mk[i] : (U)0;
+      }
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const U p = pv[u];
+        if (!p) continue;
+        const U key = p >> 1;
+        const int b = (int)((key - kmin) >> sh);
+        atomicAdd(&fcnt[b], 1);
+        if (p & 1) atomicAdd(&fhl[b], 1);
+        if (key < fmn[b]) atomicMin(&fmn[b], key);
+      }
     }
     __syncthreads();
     constexpr int PER = kFine / kNB;            // consecutive buckets per thread
@@ -286,11 +329,20 @@ k_search(const __grid_constant__ SeriesTable<T> tab, const typename KeyOf<T>::U*
       }
       if (tid == 0) nsel_s = 0;
       __syncthreads();
-      for (int i = tid; i < K; i += kNB) {
-        const U p = mk[i];
-        if (!p) continue;
-        const int b = (int)(((p >> 1) - kmin) >> sh);
-        if (fst[b] >= 0) list[atomicAdd(&nsel_s, 1)] = p;
+      for (int i0 = 0; i0 < K; i0 += kNB * kUnroll) {
+        U pv[kUnroll];
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+          const int i = i0 + u * kNB + tid;
+          pv[u] = i < K ? mk[i] : (U)0;
+        }
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+          const U p = pv[u];
+          if (!p) continue;
+          const int b = (int)(((p >> 1) - kmin) >> sh);
+          if (fst[b] >= 0) list[atomicAdd(&nsel_s, 1)] = p;
+        }
       }
       int n2 = 32;
       while (n2 < nsel) n2 <<= 1;
@@ -449,9 +501,15 @@ k_search(const __grid_constant__ SeriesTable<T> tab, const typename KeyOf<T>::U*
 
 }  // namespace
 
-template <class T> void calib_ws_layout(Arena& a, int64_t elems, CalibWs<T>& w) {
-  w.keys = a.take<typename KeyOf<T>::U>((size_t)std::max<int64_t>(elems, 1));
+template <class T> void calib_ws_layout(Arena& a, int64_t elems, int n_sm, CalibWs<T>& w) {
+  using U = typename KeyOf<T>::U;
+  w.keys = a.take<U>((size_t)std::max<int64_t>(elems, 1));
   w.thr = a.take<int32_t>(kThrTable);
+  const size_t n = (size_t)std::max(n_sm, 1);
+  w.kmin = a.take<U>(n);
+  w.kmax = a.take<U>(n);
+  w.ncand = a.take<uint32_t>(n);
+  w.n_sm = n_sm;
 }
 
 template <class T>
@@ -459,13 +517,29 @@ cudaError_t launch_calibrate(const SeriesTable<T>& tab, const T* S, const uint8_
                              const unsigned long long* slo, double ok_frac, double reliability,
                              T* theta, CalibWs<T>& w, tre_diag* diag, cudaStream_t s) {
   using U = typename KeyOf<T>::U;
-  k_thr<<<kThrTable / 256, 256, 0, s>>>(ok_frac, w.thr);
-  int Kmax = 0;
-  for (int i = 0; i < tab.n; ++i) Kmax = std::max(Kmax, tab.K[i]);
-  if (Kmax > 0) {
-    dim3 g((Kmax + 31) / 32, (tab.M + 31) / 32, tab.n), b(32, 8);
-    k_pack<T><<<g, b, 0, s>>>(tab, S, cls, slo, w.thr, ok_frac, static_cast<U*>(w.keys));
+  const int n_sm = tab.n * tab.M;
+  if (n_sm > w.n_sm) return cudaErrorInvalidValue;
+  U* kmin = static_cast<U*>(w.kmin);
+  U* kmax = static_cast<U*>(w.kmax);
+  const int thr_n = std::max(kThrTable, n_sm);
+  k_thr<U><<<(thr_n + 255) / 256, 256, 0, s>>>(ok_frac, w.thr, n_sm, kmin, kmax, w.ncand);
+  PackPlan pp;
+  pp.lg_tm = 0;
+  while ((1 << pp.lg_tm) < tab.M && pp.lg_tm < 5) ++pp.lg_tm;
+  pp.tm = 1 << pp.lg_tm;
+  pp.lg_tk = 10 - pp.lg_tm;
+  pp.tk = 1 << pp.lg_tk;
+  static_assert(kPackTile == 1024, "tile of 2^10 elements");
+  pp.m_tiles = (tab.M + pp.tm - 1) / pp.tm;
+  int tiles = 0;
+  for (int i = 0; i < tab.n; ++i) {
+    pp.tile_base[i] = tiles;
+    tiles += (tab.K[i] + pp.tk - 1) / pp.tk * pp.m_tiles;
   }
+  pp.tile_base[tab.n] = tiles;
+  if (tiles > 0)
+    k_pack<T><<<tiles, kPackThreads, 0, s>>>(tab, pp, S, cls, slo, w.thr, ok_frac,
+                                             static_cast<U*>(w.keys), kmin, kmax, w.ncand);
   const size_t smem = search_smem_bytes<T>();
   static bool attr_set = false;
   if (!attr_set) {
@@ -474,13 +548,13 @@ cudaError_t launch_calibrate(const SeriesTable<T>& tab, const T* S, const uint8_
     if (e) return e;
     attr_set = true;
   }
-  k_search<T><<<tab.n * tab.M, kNB, smem, s>>>(tab, static_cast<const U*>(w.keys), reliability,
-                                               theta, diag);
+  k_search<T><<<tab.n * tab.M, kNB, smem, s>>>(tab, static_cast<const U*>(w.keys), kmin, kmax,
+                                               w.ncand, reliability, theta, diag);
   return cudaGetLastError();
 }
 
-template void calib_ws_layout<float>(Arena&, int64_t, CalibWs<float>&);
-template void calib_ws_layout<double>(Arena&, int64_t, CalibWs<double>&);
+template void calib_ws_layout<float>(Arena&, int64_t, int, CalibWs<float>&);
+template void calib_ws_layout<double>(Arena&, int64_t, int, CalibWs<double>&);
 template cudaError_t launch_calibrate<float>(const SeriesTable<float>&, const float*,
                                              const uint8_t*, const unsigned long long*, double,
                                              double, float*, CalibWs<float>&, tre_diag*,

@@ -125,8 +125,11 @@ cudaError_t launch_receiver(int M, int K, const T* Z, const uint8_t* cls, int32_
 template <class T> struct CalibWs {
   void* keys;                  // packed keys, same element offsets as the series
   int32_t* thr;                // healthy threshold table
+  void *kmin, *kmax;           // per (series, model): candidate key range
+  uint32_t* ncand;             // per (series, model): candidate count
+  int n_sm;                    // (series, model) pairs the range arrays hold
 };
-template <class T> void calib_ws_layout(Arena& a, int64_t elems, CalibWs<T>& w);
+template <class T> void calib_ws_layout(Arena& a, int64_t elems, int n_sm, CalibWs<T>& w);
 // theta[s*M + m] for every series of the table
 template <class T>
 cudaError_t launch_calibrate(const SeriesTable<T>& tab, const T* S, const uint8_t* cls,
