@@ -642,6 +642,28 @@ k_walk_thread(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
 // the idle pool is non-empty or a model above its floor is a donor there; per
 // model, the next tick where it is a donor is precomputed, so the walk jumps
 // from one possible move to the next instead of visiting every tick.
+// Smallest of a tick row's next-donor ticks over the models in `avail`: the
+// row holds MMAX 16-bit entries; models outside the mask are lifted to 0xffff
+// and the row is reduced with per-halfword minima.
+template <int MMAX>
+__device__ __forceinline__ int next_donor_tick(const uint16_t* row, uint32_t avail) {
+  const uint4* q = reinterpret_cast<const uint4*>(row);
+  uint32_t acc = 0xffffffffu;
+#pragma unroll
+  for (int h = 0; h < MMAX / 8; ++h) {
+    const uint4 w = q[h];
+    const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int m = h * 8 + 2 * i;
+      const uint32_t lift = ((avail >> m) & 1u ? 0u : 0xffffu) |
+                            ((avail >> (m + 1)) & 1u ? 0u : 0xffff0000u);
+      acc = __vminu2(acc, ws[i] | lift);
+    }
+  }
+  return (int)min(acc & 0xffffu, acc >> 16);
+}
+
 // One tick's action as the walk reads it: donor order (4 bits a position),
 // donor mask, receiver (-1: nothing acts) and kind, in one 16-byte load.
 struct __align__(16) TickRec {
@@ -668,12 +690,15 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
   const int ratio = b.slow_ms / b.fast_ms;
   const unsigned full = 0xffffffffu;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, n_warps = blockDim.x >> 5;
-  // shared layout: per tick u < nf: action record and window; per
-  // (model + any, tick): next tick >= u where the model is a donor (row M:
-  // where anything acts)
+  // shared layout: per tick u < nf: action record and window; per tick
+  // u <= nf: for every model the next tick >= u where it is a donor (one
+  // 2*MMAX-byte row per tick, so a row is read with 16-byte loads), and the
+  // next tick >= u where anything acts
   TickRec* srec = reinterpret_cast<TickRec*>(dyn);
   int32_t* swin = reinterpret_cast<int32_t*>(srec + nf);
-  int16_t* snxt = reinterpret_cast<int16_t*>(swin + ((nf + 3) & ~3));  // [M + 1][nf + 1]
+  uint16_t* snx = reinterpret_cast<uint16_t*>(swin + ((nf + 3) & ~3));   // [nf + 1][MMAX]
+  uint16_t* sany = snx + (size_t)(nf + 1) * MMAX;                          // [nf + 1]
+  __shared__ int s_cap[8][MMAX];   // unit footprints: replicas above the floor, per warp
   for (int u = threadIdx.x; u < nf; u += blockDim.x) {
     const int rf = recv_tab[row0 + u];
     int e = -1, kd = 0, rv = -1;
@@ -695,16 +720,22 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
   }
   __syncthreads();
   // next-tick tables: a suffix minimum per row, 32 ticks per step
-  for (int m = warp; m <= M; m += n_warps) {
-    int16_t* col = snxt + (size_t)m * (nf + 1);
-    if (lane == 0) col[nf] = (int16_t)nf;
+  for (int m = warp; m < MMAX + 1; m += n_warps) {
+    uint16_t* col = m < MMAX ? snx + m : sany;
+    const int cs = m < MMAX ? MMAX : 1;   // column stride
+    if (lane == 0) col[(size_t)nf * cs] = (uint16_t)nf;
+    if (m < MMAX && m >= M) {      // padding columns: never a donor
+      for (int u = lane; u < nf; u += 32) col[(size_t)u * cs] = (uint16_t)nf;
+      continue;
+    }
+    const int mm = m < MMAX ? m : M;   // model, or M for "anything acts"
     int carry = nf;
     for (int cb = (nf - 1) & ~31; cb >= 0; cb -= 32) {
       const int u = cb + lane;
       int v = nf;
       if (u < nf) {
         const TickRec& t = srec[u];
-        if (t.recv >= 0 && (m == M || (t.dm >> m & 1u))) v = u;
+        if (t.recv >= 0 && (mm == M || (t.dm >> mm & 1u))) v = u;
       }
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
@@ -712,7 +743,7 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
         if (lane + o < 32) v = min(v, y);
       }
       v = min(v, carry);
-      if (u < nf) col[u] = (int16_t)v;
+      if (u < nf) col[(size_t)u * cs] = (uint16_t)v;
       carry = __shfl_sync(full, v, 0);
     }
   }
@@ -755,20 +786,56 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
   };
   int64_t nm = 0;
   int u = 0;
+  if (unit) {
+    // unit footprints: a transition is one replica, so a tick moves up to
+    // K_p replicas from the pool, then from donors in order
+    int* scap = s_cap[warp];
+    for (int m = 0; m < M && m < MMAX; ++m) scap[m] = sel<T, MMAX>(r, m) - sel<T, MMAX>(rmin, m);
+    while (u < nf) {
+      const int nxt = free_pool > 0 ? (int)sany[u]
+                                    : next_donor_tick<MMAX>(snx + (size_t)u * MMAX, avail);
+      if (nxt >= nf) break;
+      u = nxt;
+      const TickRec tr = srec[u];
+      const int32_t k = swin[u];
+      ++u;
+      const int recv = tr.recv;
+      if (recv < 0) continue;
+      uint32_t left = avail & tr.dm;
+      if (free_pool <= 0 && !left) continue;
+      const int kind = tr.kind;
+      const int n_pool = free_pool < Kp ? (int)free_pool : Kp;
+      for (int q = 0; q < n_pool; ++q) emit(nm + q, k, recv, -1, kind, q);
+      int sq = n_pool;
+      unsigned long long pk = tr.pk;
+      while (sq < Kp && left) {
+        const int m = (int)(pk & 15);
+        pk >>= 4;
+        if (!(left >> m & 1)) continue;
+        left &= ~(1u << m);
+        const int c = scap[m];
+        const int take = min(c, Kp - sq);
+        scap[m] = c - take;
+        if (take == c) avail &= ~(1u << m);
+        for (int i = 0; i < take; ++i, ++sq) emit(nm + sq, k, recv, m, kind, sq);
+      }
+      const int cr = scap[recv] + sq;
+      scap[recv] = cr;
+      if (cr > 0) avail |= 1u << recv;
+      free_pool -= n_pool;
+      nm += sq;
+    }
+    for (int m = 0; m < M && m < MMAX; ++m)
+      b.r_out[(size_t)inst * M + m] = scap[m] + sel<T, MMAX>(rmin, m);
+    b.n_moves[inst] = nm;
+    if (nm > cap) b.diag->err = TRE_EOVERFLOW;
+    continue;
+  }
   while (u < nf) {
     // the next tick where something may move
     int nxt;
-    if (free_pool > 0) {
-      nxt = snxt[(size_t)M * (nf + 1) + u];
-    } else {
-      nxt = nf;
-      uint32_t a = avail;
-      while (a) {
-        const int m = __ffs(a) - 1;
-        a &= a - 1;
-        nxt = min(nxt, (int)snxt[(size_t)m * (nf + 1) + u]);
-      }
-    }
+    if (free_pool > 0) nxt = sany[u];
+    else nxt = next_donor_tick<MMAX>(snx + (size_t)u * MMAX, avail);
     if (nxt >= nf) break;
     u = nxt;
     const TickRec tr = srec[u];
@@ -921,7 +988,7 @@ cudaError_t walk_thread_launch(const WalkBatch<T>& b, WalkWs& w, size_t smem, cu
       const int64_t nf = (int64_t)b.series_K[i] * b.series_win[i] / b.fast_ms;
       if (nf >= 32767) ok = false;
       const size_t need = (size_t)nf * sizeof(TickRec) + (size_t)((nf + 3) & ~3) * 4 +
-                          (size_t)(b.M + 1) * (nf + 1) * 2;
+                          (size_t)(nf + 1) * MMAX * 2 + (size_t)(nf + 1) * 2;
       jsmem = std::max(jsmem, need);
     }
     if (ok && jsmem <= kStageMax) {
