@@ -3,6 +3,7 @@
 // caller; nothing here allocates.
 #include <algorithm>
 #include <cstring>
+#include <numeric>
 #include <vector>
 
 #include "internal.h"
@@ -318,13 +319,42 @@ tre_status sweep_typed(const tre_sweep_spec* sp, const SweepPlan& pl, const tre_
   for (int t = 0; t < NT; ++t)
     for (int w = 0; w < sp->n_win; ++w) ag.out_off[t][w] = pl.off[t * sp->n_win + w];
 
+  // Gauge scan and coarsening in one blocked pass when the ratios allow a
+  // short common block; the reduction then writes the base window length's
+  // counts in place (if it is one of the lengths).
+  GaugePlan gp;
+  std::memset(&gp, 0, sizeof(gp));
+  gp.n_traces = NT;
+  gp.n_win = sp->n_win;
+  gp.M = M;
+  gp.Kb = pl.Kb;
+  gp.base_w = -1;
+  int64_t lcm = 1;
+  for (int w = 0; w < sp->n_win; ++w) {
+    gp.q[w] = pl.q[w];
+    if (pl.q[w] == 1 && gp.base_w < 0) gp.base_w = w;
+    lcm = lcm / std::gcd<int64_t>(lcm, pl.q[w]) * pl.q[w];
+    if (lcm > 4096) break;
+  }
+  const bool fused = lcm <= 4096;
+  if (fused) {
+    gp.blk = (int)(lcm * std::max<int64_t>(1, (32 + lcm - 1) / lcm));
+    if (gp.blk < kGaugeMinBlk) gp.blk = (int)(lcm * ((kGaugeMinBlk + lcm - 1) / lcm));
+    gp.nblk = (pl.Kb + gp.blk - 1) / gp.blk;
+    for (int t = 0; t < NT; ++t) {
+      for (int w = 0; w < sp->n_win; ++w) gp.out_off[t][w] = pl.off[t * sp->n_win + w];
+      gp.in_off[t] = gp.base_w >= 0 ? gp.out_off[t][gp.base_w] : (int64_t)t * pl.Kb * M;
+    }
+  }
+  const bool in_place = fused && gp.base_w >= 0;
+
   Arena a(ws);
   const size_t nb = (size_t)pl.Kb * M * NT;
-  int32_t* Pb = a.take<int32_t>(nb);
-  int32_t* Db = a.take<int32_t>(nb);
-  int32_t* Ab = a.take<int32_t>(nb);
-  int32_t* Wb = a.take<int32_t>(nb);
-  unsigned long long* slob = a.take<unsigned long long>(nb);
+  int32_t* Pb = in_place ? nullptr : a.take<int32_t>(nb);
+  int32_t* Db = in_place ? nullptr : a.take<int32_t>(nb);
+  int32_t* Ab = fused ? nullptr : a.take<int32_t>(nb);
+  int32_t* Wb = fused ? nullptr : a.take<int32_t>(nb);
+  unsigned long long* slob = in_place ? nullptr : a.take<unsigned long long>(nb);
   ReduceWs rw;
   reduce_ws_layout(a, M, pl.Kb, NT, 0, rw);
   const size_t tot = (size_t)pl.total;
@@ -336,6 +366,11 @@ tre_status sweep_typed(const tre_sweep_spec* sp, const SweepPlan& pl, const tre_
   T* Z = out->Z ? static_cast<T*>(out->Z) : a.take<T>(tot);
   uint8_t* idle = a.take<uint8_t>(tot);
   unsigned long long* slo = a.take<unsigned long long>(tot);
+  if (in_place) {
+    Pb = P;
+    Db = D;
+    slob = slo;
+  }
   ScoreWs<T> sw;
   score_ws_layout<T>(a, M, (int64_t)tot, n_seg, sw);
   CalibWs<T> cw;
@@ -380,17 +415,30 @@ tre_status sweep_typed(const tre_sweep_spec* sp, const SweepPlan& pl, const tre_
   for (int t = 0; t < NT; ++t) cols[t] = cols_of(&sp->traces[t]);
   cudaError_t e;
   {
-    Scope sc(kReduce, 1, s);
+    Scope sc(kReduce, 2, s);
+    std::vector<int64_t> red_off(NT);
+    for (int t = 0; t < NT; ++t) red_off[t] = in_place ? gp.in_off[t] : (int64_t)t * pl.Kb * M;
     e = launch_reduce_requests(cols.data(), NT, M, pl.base_win, pl.Kb, Pb, Db, rw, slob,
-                               sp->slo_ttft_ms, diag, s);
+                               sp->slo_ttft_ms, diag, s, red_off.data());
   }
-  if (!e) {
-    Scope sc(kScan, 3, s);
-    e = launch_gauge_scan(M, pl.Kb, rw, Ab, Wb, s);
-  }
-  if (!e) {
-    Scope sc(kAggregate, 1, s);
-    e = launch_aggregate(ag, Pb, Db, Ab, Wb, slob, P, D, A, W, slo, s);
+  if (fused) {
+    if (!e) {
+      Scope sc(kScan, 2, s);
+      e = launch_gauge_prefix(gp, rw, s);
+    }
+    if (!e) {
+      Scope sc(kAggregate, 1, s);
+      e = launch_gauge_apply(gp, rw, Pb, Db, slob, P, D, A, W, slo, s);
+    }
+  } else {
+    if (!e) {
+      Scope sc(kScan, 3, s);
+      e = launch_gauge_scan(M, pl.Kb, rw, Ab, Wb, s);
+    }
+    if (!e) {
+      Scope sc(kAggregate, 1, s);
+      e = launch_aggregate(ag, Pb, Db, Ab, Wb, slob, P, D, A, W, slo, s);
+    }
   }
   if (!e) {
     Scope sc(kScore, 6, s);

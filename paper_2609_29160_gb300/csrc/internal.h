@@ -44,16 +44,20 @@ struct ReduceWs {
   int32_t *dA, *dW;
   int32_t *first, *last;       // events only, [n_req]
   int32_t *partA, *partW;
+  int64_t part_cap;            // partial entries per trace
   int n_traces;
 };
+constexpr int kGaugeMinBlk = 16;   // shortest row block of the fused gauge pass
 void reduce_ws_layout(Arena& a, int M, int K, int n_traces, int64_t n_req, ReduceWs& w);
 // Request records of n_traces traces (host array of column sets) on one grid;
 // trace t writes P, D (and the packed SLO counts when slo != null) at element
-// offset t*K*M. slo packs per-(window, model) arrivals (low 32 bits) and the
-// arrivals that met the TTFT bound (high 32 bits).
+// offset out_off[t] (host array; null: t*K*M). slo packs per-(window, model)
+// arrivals (low 32 bits) and the arrivals that met the TTFT bound (high 32
+// bits).
 cudaError_t launch_reduce_requests(const ReqCols* traces, int n_traces, int M, int win, int K,
                                    int32_t* P, int32_t* D, ReduceWs& w, unsigned long long* slo,
-                                   const int32_t* slo_ms, tre_diag* diag, cudaStream_t s);
+                                   const int32_t* slo_ms, tre_diag* diag, cudaStream_t s,
+                                   const int64_t* out_off = nullptr);
 cudaError_t launch_reduce_events(const EvCols& e, int M, int win, int K, int32_t* P, int32_t* D,
                                  ReduceWs& w, tre_diag* diag, cudaStream_t s);
 cudaError_t launch_slo_requests(const ReqCols& r, int M, int win, int K,
@@ -69,6 +73,24 @@ struct AggPlan {
   int32_t q[16], Kq[16];
   int64_t out_off[64][16];      // element offset of (trace, window length) in the outputs
 };
+// Gauge scan and coarsening in one pass over row blocks (sweeps): inputs are
+// the diff arrays in the reduction scratch and the base P, D, SLO counts at
+// in_off[trace]; the base window length (base_w >= 0) gets its gauges written
+// in place, every other length its counts and gauges at out_off.
+struct GaugePlan {
+  int n_traces, n_win, M, Kb;
+  int blk, nblk, base_w;
+  int32_t q[16];
+  int64_t out_off[64][16];
+  int64_t in_off[64];
+};
+// passes 1-2: block sums of the diffs and their exclusive prefixes
+cudaError_t launch_gauge_prefix(const GaugePlan& gp, ReduceWs& w, cudaStream_t s);
+// pass 3: base gauges and every coarser window length
+cudaError_t launch_gauge_apply(const GaugePlan& gp, ReduceWs& w, const int32_t* Pin,
+                               const int32_t* Din, const unsigned long long* sloin, int32_t* P,
+                               int32_t* D, int32_t* A, int32_t* W, unsigned long long* slo,
+                               cudaStream_t s);
 cudaError_t launch_aggregate(const AggPlan& plan, const int32_t* P, const int32_t* D,
                              const int32_t* A, const int32_t* W, const unsigned long long* slo,
                              int32_t* Pq, int32_t* Dq, int32_t* Aq, int32_t* Wq,

@@ -48,6 +48,7 @@ struct ReqBatch {
   int64_t per_cta[kMaxTraces];
   int32_t cta_base[kMaxTraces + 1];
   unsigned long long vec_ok;          // bit t: trace t's columns allow 16-byte loads
+  int64_t out_off[kMaxTraces];        // element offset of trace t's P, D, SLO counts
 };
 
 // Targets of one record fall in two places: the arrival side (the waiting
@@ -92,11 +93,11 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win,
   const ReqCols& r = bt.cols[t];
   const bool vec = (bt.vec_ok >> t) & 1ull;
   const size_t cells0 = (size_t)K * M, cells1 = (size_t)(K + 1) * M;
-  int32_t* P = P0 + t * cells0;
-  int32_t* D = D0 + t * cells0;
+  int32_t* P = P0 + bt.out_off[t];
+  int32_t* D = D0 + bt.out_off[t];
   int32_t* dA = dA0 + t * cells1;
   int32_t* dW = dW0 + t * cells1;
-  unsigned long long* slo = SLO ? slo0 + t * cells0 : nullptr;
+  unsigned long long* slo = SLO ? slo0 + bt.out_off[t] : nullptr;
   const int64_t i0 = (int64_t)(blockIdx.x - bt.cta_base[t]) * bt.per_cta[t];
   const int n_loc = (int)min64(r.n - i0, bt.per_cta[t]);
   if (n_loc <= 0) return;
@@ -632,6 +633,156 @@ k_aggregate(const __grid_constant__ AggPlan pl, const int32_t* __restrict__ P,
   }
 }
 
+// Clears a list of 32-bit word ranges in one launch (16-byte stores where a
+// range allows them).
+constexpr int kMaxZero = 3 * kMaxTraces + 2;
+struct ZeroList {
+  int n;
+  uint32_t* ptr[kMaxZero];
+  int64_t words[kMaxZero];
+};
+
+__global__ void __launch_bounds__(kThreads) k_zero(const __grid_constant__ ZeroList zl) {
+  const int64_t stride = (int64_t)gridDim.x * kThreads;
+  const int64_t tid = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+  for (int r = 0; r < zl.n; ++r) {
+    uint32_t* p = zl.ptr[r];
+    const int64_t n = zl.words[r];
+    // words before the first 16-byte boundary, then whole 16-byte groups, then the tail
+    const int64_t head = min64(n, (int64_t)((16 - ((uintptr_t)p & 15)) & 15) / 4);
+    if (tid < head) p[tid] = 0u;
+    uint4* q = reinterpret_cast<uint4*>(p + head);
+    const int64_t nq = (n - head) / 4;
+    for (int64_t i = tid; i < nq; i += stride) q[i] = make_uint4(0u, 0u, 0u, 0u);
+    const int64_t t0 = head + nq * 4;
+    if (tid < n - t0) p[t0 + tid] = 0u;
+  }
+}
+
+// ---- gauge scan fused with the exact coarsening (sweeps) --------------------
+// Base windows are cut into blocks of `blk` rows (a multiple of every window
+// length's ratio q, so no coarse window straddles two blocks). Pass 1 sums the
+// gauge diffs of every (trace, block, model); pass 2 turns those sums into
+// exclusive prefixes per (trace, model); pass 3 runs each block from its
+// prefix, writes the base gauges, and for every coarser window length adds the
+// counts over q base windows and reads the gauges at the last of them.
+__global__ void __launch_bounds__(kThreads)
+k_gauge_blocks(const __grid_constant__ GaugePlan gp, const int32_t* __restrict__ dA,
+               const int32_t* __restrict__ dW, int32_t* __restrict__ pA,
+               int32_t* __restrict__ pW) {
+  const int M = gp.M, Kb = gp.Kb;
+  const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+  if (t >= (int64_t)gp.n_traces * gp.nblk * M) return;
+  const int m = (int)(t % M);
+  const int64_t rest = t / M;
+  const int b = (int)(rest % gp.nblk), tr = (int)(rest / gp.nblk);
+  const int k0 = b * gp.blk, k1 = min(Kb, k0 + gp.blk);
+  const size_t base = (size_t)tr * (Kb + 1) * M + m;
+  int32_t a = 0, w = 0;
+#pragma unroll 4
+  for (int k = k0; k < k1; ++k) {
+    a += dA[base + (size_t)k * M];
+    w += dW[base + (size_t)k * M];
+  }
+  pA[t] = a;
+  pW[t] = w;
+}
+
+// exclusive scan of the block sums of one (trace, model) per CTA
+__global__ void __launch_bounds__(kThreads)
+k_gauge_block_scan(const __grid_constant__ GaugePlan gp, int32_t* __restrict__ pA,
+                   int32_t* __restrict__ pW) {
+  __shared__ int32_t wa[kThreads / 32], ww[kThreads / 32];
+  const int M = gp.M, nb = gp.nblk;
+  const int tr = blockIdx.x / M, m = blockIdx.x % M;
+  const size_t base = (size_t)tr * nb * M + m;
+  const int per = (nb + kThreads - 1) / kThreads;
+  const int b0 = threadIdx.x * per, b1 = min(nb, b0 + per);
+  int32_t sa = 0, sw = 0;
+  for (int b = b0; b < b1; ++b) {
+    sa += pA[base + (size_t)b * M];
+    sw += pW[base + (size_t)b * M];
+  }
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  int32_t ia = sa, iw = sw;
+  for (int o = 1; o < 32; o <<= 1) {
+    const int32_t xa = __shfl_up_sync(0xffffffffu, ia, o);
+    const int32_t xw = __shfl_up_sync(0xffffffffu, iw, o);
+    if (lane >= o) { ia += xa; iw += xw; }
+  }
+  if (lane == 31) { wa[wid] = ia; ww[wid] = iw; }
+  __syncthreads();
+  int32_t ea = ia - sa, ew = iw - sw;
+  for (int q = 0; q < wid; ++q) { ea += wa[q]; ew += ww[q]; }
+  for (int b = b0; b < b1; ++b) {
+    const size_t x = base + (size_t)b * M;
+    const int32_t va = pA[x], vw = pW[x];
+    pA[x] = ea;
+    pW[x] = ew;
+    ea += va;
+    ew += vw;
+  }
+}
+
+__global__ void __launch_bounds__(kThreads)
+k_gauge_apply(const __grid_constant__ GaugePlan gp, const int32_t* __restrict__ dA,
+              const int32_t* __restrict__ dW, const int32_t* __restrict__ pA,
+              const int32_t* __restrict__ pW, const int32_t* __restrict__ Pin,
+              const int32_t* __restrict__ Din, const unsigned long long* __restrict__ sloin,
+              int32_t* __restrict__ P, int32_t* __restrict__ D, int32_t* __restrict__ A,
+              int32_t* __restrict__ W, unsigned long long* __restrict__ slo) {
+  constexpr int NW = 16;
+  const int M = gp.M, Kb = gp.Kb;
+  const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+  if (t >= (int64_t)gp.n_traces * gp.nblk * M) return;
+  const int m = (int)(t % M);
+  const int64_t rest = t / M;
+  const int b = (int)(rest % gp.nblk), tr = (int)(rest / gp.nblk);
+  const int k0 = b * gp.blk, k1 = min(Kb, k0 + gp.blk);
+  const size_t dbase = (size_t)tr * (Kb + 1) * M + m;
+  const size_t ibase = (size_t)gp.in_off[tr] + m;
+  int32_t a = pA[t], w = pW[t];
+  int32_t ap[NW], ad[NW], cnt[NW], kq[NW];
+  unsigned long long as[NW];
+#pragma unroll
+  for (int j = 0; j < NW; ++j) {
+    ap[j] = 0; ad[j] = 0; as[j] = 0;
+    cnt[j] = j < gp.n_win ? gp.q[j] : 0;
+    kq[j] = j < gp.n_win ? k0 / gp.q[j] : 0;
+  }
+  for (int k = k0; k < k1; ++k) {
+    a += dA[dbase + (size_t)k * M];
+    w += dW[dbase + (size_t)k * M];
+    const size_t xi = ibase + (size_t)k * M;
+    const int32_t p = Pin[xi], d = Din[xi];
+    const unsigned long long sl = sloin ? sloin[xi] : 0ull;
+#pragma unroll
+    for (int j = 0; j < NW; ++j) {
+      if (j >= gp.n_win) break;
+      if (j == gp.base_w) {
+        const size_t o = (size_t)gp.out_off[tr][j] + (size_t)k * M + m;
+        A[o] = a;
+        W[o] = w;
+        continue;
+      }
+      ap[j] += p;
+      ad[j] += d;
+      as[j] += sl;
+      if (--cnt[j] == 0) {
+        const size_t o = (size_t)gp.out_off[tr][j] + (size_t)kq[j] * M + m;
+        P[o] = ap[j];
+        D[o] = ad[j];
+        A[o] = a;
+        W[o] = w;
+        if (slo) slo[o] = as[j];
+        ap[j] = 0; ad[j] = 0; as[j] = 0;
+        cnt[j] = gp.q[j];
+        ++kq[j];
+      }
+    }
+  }
+}
+
 int num_sms() {
   static int n = 0;
   if (!n) {
@@ -669,26 +820,41 @@ void reduce_ws_layout(Arena& a, int M, int K, int n_traces, int64_t n_req, Reduc
   w.first = n_req > 0 ? a.take<int32_t>((size_t)n_req) : nullptr;
   w.last = n_req > 0 ? a.take<int32_t>((size_t)n_req) : nullptr;
   const int L = scan_chunk_rows(K);
-  const int n_chunks = (K + L - 1) / L;
-  w.partA = a.take<int32_t>((size_t)std::max(n_chunks, 1) * M * n_traces);
-  w.partW = a.take<int32_t>((size_t)std::max(n_chunks, 1) * M * n_traces);
+  const int n_chunks = std::max((K + L - 1) / L, (K + kGaugeMinBlk - 1) / kGaugeMinBlk);
+  w.part_cap = (int64_t)std::max(n_chunks, 1) * M;
+  w.partA = a.take<int32_t>((size_t)w.part_cap * n_traces);
+  w.partW = a.take<int32_t>((size_t)w.part_cap * n_traces);
 }
 
 cudaError_t launch_reduce_requests(const ReqCols* traces, int n_traces, int M, int win, int K,
                                    int32_t* P, int32_t* D, ReduceWs& w, unsigned long long* slo,
-                                   const int32_t* slo_ms, tre_diag* diag, cudaStream_t s) {
+                                   const int32_t* slo_ms, tre_diag* diag, cudaStream_t s,
+                                   const int64_t* out_off) {
   if (n_traces < 1 || n_traces > kMaxTraces || n_traces > w.n_traces)
     return cudaErrorInvalidValue;
   const size_t cells = (size_t)K * M * n_traces;
-  cudaError_t e;
-  if ((e = cudaMemsetAsync(P, 0, cells * sizeof(int32_t), s))) return e;
-  if ((e = cudaMemsetAsync(D, 0, cells * sizeof(int32_t), s))) return e;
-  if ((e = cudaMemsetAsync(w.dA, 0, (cells + (size_t)M * n_traces) * sizeof(int32_t), s))) return e;
-  if ((e = cudaMemsetAsync(w.dW, 0, (cells + (size_t)M * n_traces) * sizeof(int32_t), s))) return e;
-  if (slo && (e = cudaMemsetAsync(slo, 0, cells * sizeof(unsigned long long), s))) return e;
   ReqBatch bt;
   bt.n = n_traces;
   bt.vec_ok = 0;
+  // every output the kernel adds into starts at zero: one clearing launch
+  ZeroList zl;
+  zl.n = 0;
+  for (int t = 0; t < n_traces; ++t) {
+    bt.out_off[t] = out_off ? out_off[t] : (int64_t)t * K * M;
+    zl.ptr[zl.n] = reinterpret_cast<uint32_t*>(P + bt.out_off[t]);
+    zl.words[zl.n++] = (int64_t)K * M;
+    zl.ptr[zl.n] = reinterpret_cast<uint32_t*>(D + bt.out_off[t]);
+    zl.words[zl.n++] = (int64_t)K * M;
+    if (slo) {
+      zl.ptr[zl.n] = reinterpret_cast<uint32_t*>(slo + bt.out_off[t]);
+      zl.words[zl.n++] = (int64_t)K * M * 2;
+    }
+  }
+  zl.ptr[zl.n] = reinterpret_cast<uint32_t*>(w.dA);
+  zl.words[zl.n++] = (int64_t)(cells + (size_t)M * n_traces);
+  zl.ptr[zl.n] = reinterpret_cast<uint32_t*>(w.dW);
+  zl.words[zl.n++] = (int64_t)(cells + (size_t)M * n_traces);
+  k_zero<<<num_sms() * 8, kThreads, 0, s>>>(zl);
   int64_t total_n = 0;
   for (int t = 0; t < n_traces; ++t) total_n += traces[t].n;
   // records per CTA sized on the whole batch so the grid fills the GPU
@@ -799,6 +965,27 @@ cudaError_t launch_gauge_scan(int M, int K, ReduceWs& w, int32_t* A, int32_t* W,
   k_scan_partials<<<g, kThreads, 0, s>>>(M, K, L, n_chunks, w.dA, w.dW, w.partA, w.partW);
   k_scan_chunks<<<dim3((M + 3) / 4, w.n_traces), 128, 0, s>>>(M, n_chunks, w.partA, w.partW);
   k_scan_apply<<<g, kThreads, 0, s>>>(M, K, L, n_chunks, w.dA, w.dW, w.partA, w.partW, A, W);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gauge_prefix(const GaugePlan& gp, ReduceWs& w, cudaStream_t s) {
+  if (gp.n_traces > w.n_traces || (int64_t)gp.nblk * gp.M > w.part_cap) return cudaErrorInvalidValue;
+  const int64_t n = (int64_t)gp.n_traces * gp.nblk * gp.M;
+  if (n == 0) return cudaSuccess;
+  k_gauge_blocks<<<(unsigned)((n + kThreads - 1) / kThreads), kThreads, 0, s>>>(gp, w.dA, w.dW,
+                                                                                w.partA, w.partW);
+  k_gauge_block_scan<<<gp.n_traces * gp.M, kThreads, 0, s>>>(gp, w.partA, w.partW);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gauge_apply(const GaugePlan& gp, ReduceWs& w, const int32_t* Pin,
+                               const int32_t* Din, const unsigned long long* sloin, int32_t* P,
+                               int32_t* D, int32_t* A, int32_t* W, unsigned long long* slo,
+                               cudaStream_t s) {
+  const int64_t n = (int64_t)gp.n_traces * gp.nblk * gp.M;
+  if (n == 0) return cudaSuccess;
+  k_gauge_apply<<<(unsigned)((n + kThreads - 1) / kThreads), kThreads, 0, s>>>(
+      gp, w.dA, w.dW, w.partA, w.partW, Pin, Din, sloin, P, D, A, W, slo);
   return cudaGetLastError();
 }
 
