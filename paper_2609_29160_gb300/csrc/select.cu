@@ -15,6 +15,7 @@
 // the replica counts in registers (models m = lane + 32*j) -- then only picks,
 // per released replica, the lowest-ranked model still above its floor.
 #include <algorithm>
+#include <cstddef>
 
 #include "common.cuh"
 #include "internal.h"
@@ -664,6 +665,22 @@ __device__ __forceinline__ int next_donor_tick(const uint16_t* row, uint32_t ava
   return (int)min(acc & 0xffffu, acc >> 16);
 }
 
+// One move record, written as three 32-bit words (window; receiver and donor;
+// kind and position in the tick) when it fits the caller's list.
+static_assert(sizeof(tre_move) == 12 && offsetof(tre_move, recv) == 4 &&
+                  offsetof(tre_move, donor) == 6 && offsetof(tre_move, kind) == 8 &&
+                  offsetof(tre_move, seq) == 9 && offsetof(tre_move, reserved) == 10,
+              "tre_move layout");
+__device__ __forceinline__ void put_move(tre_move* mv, int64_t at, int64_t cap, int32_t k,
+                                         int recv, int donor, int kind, int sq) {
+  if (at < cap) {
+    uint32_t* p = reinterpret_cast<uint32_t*>(mv + at);
+    p[0] = (uint32_t)k;
+    p[1] = (uint32_t)(uint16_t)recv | ((uint32_t)(uint16_t)donor << 16);
+    p[2] = (uint32_t)(uint8_t)kind | ((uint32_t)(uint8_t)sq << 8);
+  }
+}
+
 // One tick's action as the walk reads it: donor order (4 bits a position),
 // donor mask, receiver (-1: nothing acts) and kind, in one 16-byte load.
 struct __align__(16) TickRec {
@@ -791,9 +808,72 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
     // K_p replicas from the pool, then from donors in order
     int* scap = s_cap[warp];
     for (int m = 0; m < M && m < MMAX; ++m) scap[m] = sel<T, MMAX>(r, m) - sel<T, MMAX>(rmin, m);
+    // next-donor rows are masked by `avail` with these halfword lifts, rebuilt
+    // only when `avail` changes
+    uint32_t lw[MMAX / 2];
+    uint32_t lw_for = ~avail;
+    auto next_tick = [&](int uu) -> int {
+      if (free_pool > 0) return sany[uu];
+      if (lw_for != avail) {
+#pragma unroll
+        for (int i = 0; i < MMAX / 2; ++i)
+          lw[i] = ((avail >> (2 * i)) & 1u ? 0u : 0xffffu) |
+                  ((avail >> (2 * i + 1)) & 1u ? 0u : 0xffff0000u);
+        lw_for = avail;
+      }
+      const uint4* q = reinterpret_cast<const uint4*>(snx + (size_t)uu * MMAX);
+      uint32_t acc = 0xffffffffu;
+#pragma unroll
+      for (int h = 0; h < MMAX / 8; ++h) {
+        const uint4 w = q[h];
+        acc = __vminu2(acc, w.x | lw[4 * h]);
+        acc = __vminu2(acc, w.y | lw[4 * h + 1]);
+        acc = __vminu2(acc, w.z | lw[4 * h + 2]);
+        acc = __vminu2(acc, w.w | lw[4 * h + 3]);
+      }
+      return (int)min(acc & 0xffffu, acc >> 16);
+    };
+    if (Kp == 1 && MMAX == 8) {
+      // one transition per tick: every tick the jump lands on moves exactly
+      // one replica (it has a receiver, and a usable donor when the pool is
+      // empty), so the visit is straight-line code
+      int32_t nm1 = 0;
+      while (true) {
+        const int nxt = next_tick(u);
+        if (nxt >= nf) break;
+        u = nxt + 1;
+        const TickRec tr = srec[nxt];
+        const int32_t k = swin[nxt];
+        const int recv = tr.recv;
+        int donor = -1;
+        if (free_pool > 0) {
+          --free_pool;
+        } else {
+          const uint32_t left = avail & tr.dm;
+          const uint32_t tl = ((left & 0xFu) * 0x00204081u) & 0x01010101u;
+          const uint32_t th = (((left >> 4) & 0xFu) * 0x00204081u) & 0x01010101u;
+          const uint32_t pl = (uint32_t)tr.pk;
+          const int nd = __popc(tr.dm);
+          uint32_t f0 = __byte_perm(tl, th, pl & 0xFFFFu);
+          uint32_t f1 = __byte_perm(tl, th, pl >> 16);
+          if (nd < 4) f0 &= (1u << (8 * nd)) - 1u;
+          if (nd < 8) f1 &= nd <= 4 ? 0u : (1u << (8 * (nd - 4))) - 1u;
+          const int j = f0 ? (__ffs(f0) - 1) >> 3 : 4 + ((__ffs(f1) - 1) >> 3);
+          donor = (int)((pl >> (4 * j)) & 15u);
+          const int c = scap[donor] - 1;
+          scap[donor] = c;
+          if (c == 0) avail &= ~(1u << donor);
+        }
+        put_move(mv, nm1, cap, k, recv, donor, tr.kind, 0);
+        ++nm1;
+        scap[recv] += 1;
+        avail |= 1u << recv;
+      }
+      nm = nm1;
+      u = nf;
+    }
     while (u < nf) {
-      const int nxt = free_pool > 0 ? (int)sany[u]
-                                    : next_donor_tick<MMAX>(snx + (size_t)u * MMAX, avail);
+      const int nxt = next_tick(u);
       if (nxt >= nf) break;
       u = nxt;
       const TickRec tr = srec[u];
@@ -805,19 +885,50 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
       if (free_pool <= 0 && !left) continue;
       const int kind = tr.kind;
       const int n_pool = free_pool < Kp ? (int)free_pool : Kp;
-      for (int q = 0; q < n_pool; ++q) emit(nm + q, k, recv, -1, kind, q);
+      for (int q = 0; q < n_pool; ++q) put_move(mv, nm + q, cap, k, recv, -1, kind, q);
       int sq = n_pool;
       unsigned long long pk = tr.pk;
-      while (sq < Kp && left) {
-        const int m = (int)(pk & 15);
-        pk >>= 4;
-        if (!(left >> m & 1)) continue;
-        left &= ~(1u << m);
-        const int c = scap[m];
-        const int take = min(c, Kp - sq);
-        scap[m] = c - take;
-        if (take == c) avail &= ~(1u << m);
-        for (int i = 0; i < take; ++i, ++sq) emit(nm + sq, k, recv, m, kind, sq);
+      if (MMAX == 8) {
+        // usable donors by position in the order, one flag byte per position:
+        // spread the usable bits to bytes, then gather them by the order's
+        // model nibbles; positions past the tick's donor count are masked
+        const uint32_t tl = ((left & 0xFu) * 0x00204081u) & 0x01010101u;
+        const uint32_t th = (((left >> 4) & 0xFu) * 0x00204081u) & 0x01010101u;
+        const uint32_t pl = (uint32_t)pk;
+        const int nd = __popc(tr.dm);
+        uint32_t f0 = __byte_perm(tl, th, pl & 0xFFFFu);
+        uint32_t f1 = __byte_perm(tl, th, pl >> 16);
+        if (nd < 4) f0 &= (1u << (8 * nd)) - 1u;
+        if (nd < 8) f1 &= nd <= 4 ? 0u : (1u << (8 * (nd - 4))) - 1u;
+        while (sq < Kp && (f0 | f1)) {
+          int j;
+          if (f0) {
+            j = (__ffs(f0) - 1) >> 3;
+            f0 &= ~(0xFFu << (8 * j));
+          } else {
+            const int j1 = (__ffs(f1) - 1) >> 3;
+            f1 &= ~(0xFFu << (8 * j1));
+            j = 4 + j1;
+          }
+          const int m = (int)((pl >> (4 * j)) & 15u);
+          const int c = scap[m];
+          const int take = min(c, Kp - sq);
+          scap[m] = c - take;
+          if (take == c) avail &= ~(1u << m);
+          for (int i = 0; i < take; ++i, ++sq) put_move(mv, nm + sq, cap, k, recv, m, kind, sq);
+        }
+      } else {
+        while (sq < Kp && left) {
+          const int m = (int)(pk & 15);
+          pk >>= 4;
+          if (!(left >> m & 1)) continue;
+          left &= ~(1u << m);
+          const int c = scap[m];
+          const int take = min(c, Kp - sq);
+          scap[m] = c - take;
+          if (take == c) avail &= ~(1u << m);
+          for (int i = 0; i < take; ++i, ++sq) put_move(mv, nm + sq, cap, k, recv, m, kind, sq);
+        }
       }
       const int cr = scap[recv] + sq;
       scap[recv] = cr;
