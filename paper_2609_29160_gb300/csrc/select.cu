@@ -137,20 +137,22 @@ k_tick_rank(const __grid_constant__ WalkBatch<T> b, int16_t* recv_out, int16_t* 
 }
 
 // One thread per (series, tau, tick entry) for M <= MMAX: the regions are
-// computed once per model and the ranks in registers.
+// computed once per model and the ranks in registers; the per-model rank and
+// order tables are written only when the walk that follows reads them.
 template <class T, int MMAX>
 __global__ void __launch_bounds__(128)
 k_tick_rank_small(const __grid_constant__ WalkBatch<T> b, int16_t* recv_out, int16_t* ndon_out,
-                  uint16_t* rank, uint16_t* order, unsigned long long* packed, uint32_t* dmask) {
+                  uint16_t* rank, uint16_t* order, unsigned long long* packed, uint32_t* dmask,
+                  bool need_rank) {
   const int M = b.M;
   const int64_t e = (int64_t)blockIdx.x * 128 + threadIdx.x;
   if (e >= (int64_t)b.ent_base[b.n_series] * b.n_tau) return;
   int s = 0;
   while (s + 1 < b.n_series && (int64_t)b.ent_base[s + 1] * b.n_tau <= e) ++s;
-  const int64_t local = e - (int64_t)b.ent_base[s] * b.n_tau;
+  const int local = (int)(e - (int64_t)b.ent_base[s] * b.n_tau);
   const int n_ent = b.ent_base[s + 1] - b.ent_base[s];
-  const int ti = (int)(local / n_ent);
-  const int j = (int)(local % n_ent);
+  const int ti = local / n_ent;
+  const int j = local - ti * n_ent;
   const int64_t win = b.series_win[s];
   const int64_t K = b.series_K[s];
   const int64_t nf = K * win / b.fast_ms;
@@ -212,13 +214,13 @@ k_tick_rank_small(const __grid_constant__ WalkBatch<T> b, int16_t* recv_out, int
         before += prec;
       }
       r = (uint16_t)before;
-      order[row * M + r] = (uint16_t)m;
+      if (need_rank) order[row * M + r] = (uint16_t)m;
       if (MMAX <= 16) {
         pk |= (unsigned long long)m << (4 * before);
         dm |= 1u << m;
       }
     }
-    rank[row * M + m] = r;
+    if (need_rank) rank[row * M + m] = r;
   }
   recv_out[row] = (int16_t)(act ? recv : -1);
   ndon_out[row] = (int16_t)nd;
@@ -1116,31 +1118,32 @@ cudaError_t walk_thread_launch(const WalkBatch<T>& b, WalkWs& w, size_t smem, cu
 template <class T> cudaError_t launch_walk(const WalkBatch<T>& b, WalkWs& w, cudaStream_t s) {
   if (b.n_inst == 0) return cudaSuccess;
   const int64_t ents = (int64_t)b.ent_base[b.n_series] * b.n_tau;
+  // which walk runs decides whether the per-model rank tables are needed
+  int max_ent = 0;
+  for (int i = 0; i < b.n_series; ++i)
+    max_ent = std::max(max_ent, b.ent_base[i + 1] - b.ent_base[i]);
+  const size_t thread_smem = (size_t)max_ent * (8 + 4 + 2) + 16;
+  const bool thread_walk = b.M <= 16 && b.n_cap <= 32 && thread_smem <= kStageMax;
   if (ents > 0) {
+    const unsigned g = (unsigned)((ents + 127) / 128);
     if (b.M <= 8) {
-      k_tick_rank_small<T, 8><<<(unsigned)((ents + 127) / 128), 128, 0, s>>>(
-          b, w.recv, w.n_donor, w.rank, w.order, w.packed, w.dmask);
+      k_tick_rank_small<T, 8><<<g, 128, 0, s>>>(b, w.recv, w.n_donor, w.rank, w.order, w.packed,
+                                                w.dmask, !thread_walk);
     } else if (b.M <= 16) {
-      k_tick_rank_small<T, 16><<<(unsigned)((ents + 127) / 128), 128, 0, s>>>(
-          b, w.recv, w.n_donor, w.rank, w.order, w.packed, w.dmask);
+      k_tick_rank_small<T, 16><<<g, 128, 0, s>>>(b, w.recv, w.n_donor, w.rank, w.order,
+                                                 w.packed, w.dmask, !thread_walk);
     } else if (b.M <= 32) {
-      k_tick_rank_small<T, 32><<<(unsigned)((ents + 127) / 128), 128, 0, s>>>(
-          b, w.recv, w.n_donor, w.rank, w.order, w.packed, w.dmask);
+      k_tick_rank_small<T, 32><<<g, 128, 0, s>>>(b, w.recv, w.n_donor, w.rank, w.order,
+                                                 w.packed, w.dmask, true);
     } else {
       const int64_t th = ents * b.M;
       k_tick_rank<T><<<(unsigned)((th + 255) / 256), 256, 0, s>>>(b, w.recv, w.n_donor, w.rank,
                                                                    w.order);
     }
   }
-  if (b.M <= 16 && b.n_cap <= 32) {
-    int max_ent = 0;
-    for (int i = 0; i < b.n_series; ++i)
-      max_ent = std::max(max_ent, b.ent_base[i + 1] - b.ent_base[i]);
-    const size_t smem = (size_t)max_ent * (8 + 4 + 2) + 16;
-    if (smem <= kStageMax)
-      return b.M <= 8 ? walk_thread_launch<T, 8>(b, w, smem, s)
-                      : walk_thread_launch<T, 16>(b, w, smem, s);
-  }
+  if (thread_walk)
+    return b.M <= 8 ? walk_thread_launch<T, 8>(b, w, thread_smem, s)
+                    : walk_thread_launch<T, 16>(b, w, thread_smem, s);
   const int mpl = (b.M + 31) / 32;
   if (mpl <= 1) return walk_launch<T, 1>(b, w, s);
   if (mpl <= 2) return walk_launch<T, 2>(b, w, s);
