@@ -94,8 +94,7 @@ k_pack(const __grid_constant__ SeriesTable<T> tab, const __grid_constant__ PackP
   __shared__ U tile[kPackTile + 32];
   __shared__ U smin[32], smax[32];
   __shared__ uint32_t scnt[32];
-  int s = 0;
-  while (s + 1 < tab.n && pp.tile_base[s + 1] <= (int)blockIdx.x) ++s;
+  const int s = prefix_index(pp.tile_base, tab.n, blockIdx.x);
   const int M = tab.M, K = tab.K[s];
   const int t_loc = blockIdx.x - pp.tile_base[s];
   const int kt = pp.m_tiles == 1 ? t_loc : t_loc / pp.m_tiles;

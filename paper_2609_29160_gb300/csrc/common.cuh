@@ -68,6 +68,20 @@ struct FastDiv {
   }
 };
 
+// Largest i in [0, n) with base[i] * scale <= v, for a non-decreasing table
+// (prefix sums of per-series counts) with base[0] * scale <= v: a binary
+// search, so a lookup in a 64-entry kernel-parameter table costs six steps.
+__device__ __forceinline__ int prefix_index(const int32_t* base, int n, int64_t v,
+                                            int64_t scale = 1) {
+  int lo = 0, hi = n - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if ((int64_t)base[mid] * scale <= v) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
+}
+
 // warp-level sum of a 64-bit counter, one atomic per warp when non-zero
 __device__ __forceinline__ void warp_add_counter(unsigned long long* dst, unsigned long long v) {
   const unsigned full = 0xffffffffu;

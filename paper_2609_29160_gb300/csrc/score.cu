@@ -21,6 +21,7 @@
 // only re-runs chunks when a burn-in did not converge (long idle stretches, a
 // tiny alpha), counted in tre_diag.ema_resolved.
 #include <algorithm>
+#include <initializer_list>
 
 #include "common.cuh"
 #include "internal.h"
@@ -28,7 +29,6 @@
 namespace tre {
 namespace {
 
-constexpr int kThreads = 256;
 constexpr int kBatch = 16;  // windows loaded ahead in the sequential chains
 
 template <class T> __device__ __forceinline__ T sub_rn(T a, T b);
@@ -48,9 +48,7 @@ struct Counts {
 
 // series of a global segment index (the table has at most 64 entries)
 template <class T> __device__ __forceinline__ int series_of_seg(const SeriesTable<T>& t, int seg) {
-  int s = 0;
-  while (s + 1 < t.n && t.seg_base[s + 1] <= seg) ++s;
-  return s;
+  return prefix_index(t.seg_base, t.n, seg);
 }
 
 template <class T> struct ModelParams {
@@ -81,76 +79,83 @@ __device__ __forceinline__ bool is_idle_raw(double r) {
   return (unsigned long long)__double_as_longlong(r) == 0xfff8deaddeadbeefull;
 }
 
-// Walks the elements of all series of a table in one grid-stride loop:
-// element v of the concatenation maps to series s and local index v - vbase.
-template <class T> struct SeriesCursor {
-  int s = 0;
-  int64_t vbase = 0;
-  __device__ __forceinline__ void seek(const SeriesTable<T>& t, int64_t v) {
-    while (s + 1 < t.n && v >= vbase + (int64_t)t.K[s] * t.M) {
-      vbase += (int64_t)t.K[s] * t.M;
-      ++s;
-    }
-  }
+// ---- pass 0: Eq. 1 for every (window, model) of every series ---------------
+// Element-wise passes run over tiles of kTile consecutive elements of one
+// series; a thread takes four consecutive elements, with 16-byte loads and
+// stores when they are aligned (scalar ones otherwise), so that enough bytes
+// are in flight to cover memory latency.
+constexpr int kEwThreads = 256;
+constexpr int kTile = 4 * kEwThreads;
+struct TilePlan {
+  int tile_base[kMaxSeries + 1];   // prefix of tiles per series
 };
 
-__device__ __forceinline__ int model_of(int64_t local, const FastDiv& fm, int M) {
-  if (local <= 0xffffffffll) {
-    const uint32_t x = (uint32_t)local;
-    return (int)(x - fm.div(x) * (uint32_t)M);
-  }
-  return (int)(local % M);
+template <class T>
+__device__ __forceinline__ T raw_tss(int32_t p, int32_t d, int32_t a, int32_t w, T dt, T wp,
+                                     T wq) {
+  const T r_pre = div_rn(from_i32<T>(p), dt);
+  const T r_dec = div_rn(from_i32<T>(d), dt);
+  const T num = add_rn(mul_rn(wp, r_pre), r_dec);
+  T den = add_rn(from_i32<T>(a), mul_rn(wq, from_i32<T>(w)));
+  if (den < (T)1) den = (T)1;                       // demand floor of one request
+  return div_rn(num, den);
 }
 
-// ---- pass 0: Eq. 1 for every (window, model) of every series ---------------
-constexpr int kEw = 4;   // elements per thread per pass (their loads issued together)
-
 template <class T>
-__global__ void __launch_bounds__(kThreads)
-k_raw(const __grid_constant__ SeriesTable<T> tab, int64_t total, FastDiv fm, Counts c,
-      const T* __restrict__ w_p, const T* __restrict__ w_q, T* __restrict__ raw,
-      uint8_t* __restrict__ cls) {
+__global__ void __launch_bounds__(kEwThreads)
+k_raw(const __grid_constant__ SeriesTable<T> tab, const __grid_constant__ TilePlan tp, FastDiv fm,
+      bool vec, Counts c, const T* __restrict__ w_p, const T* __restrict__ w_q,
+      T* __restrict__ raw, uint8_t* __restrict__ cls) {
+  const int s = prefix_index(tp.tile_base, tab.n, blockIdx.x);
   const int M = tab.M;
-  SeriesCursor<T> cur;
-  const int64_t stride = (int64_t)gridDim.x * kThreads;
-  for (int64_t v0 = (int64_t)blockIdx.x * kThreads + threadIdx.x; v0 < total;
-       v0 += stride * kEw) {
-    size_t x[kEw];
-    int m[kEw], sr[kEw];
-    int32_t p[kEw], d[kEw], a[kEw], w[kEw];
+  const int64_t n = (int64_t)tab.K[s] * M;
+  const int64_t l0 = (int64_t)(blockIdx.x - tp.tile_base[s]) * kTile + 4 * threadIdx.x;
+  if (l0 >= n) return;
+  const size_t x0 = (size_t)(tab.off[s] + l0);
+  const T dt = div_rn((T)tab.win[s], (T)1000);      // window length in seconds
+  int32_t p[4], d[4], a[4], w[4];
+  const bool v4 = vec && l0 + 4 <= n;
+  if (v4) {
+    const int4 P4 = *reinterpret_cast<const int4*>(c.P + x0);
+    const int4 D4 = *reinterpret_cast<const int4*>(c.D + x0);
+    const int4 A4 = *reinterpret_cast<const int4*>(c.A + x0);
+    const int4 W4 = *reinterpret_cast<const int4*>(c.W + x0);
+    p[0] = P4.x; p[1] = P4.y; p[2] = P4.z; p[3] = P4.w;
+    d[0] = D4.x; d[1] = D4.y; d[2] = D4.z; d[3] = D4.w;
+    a[0] = A4.x; a[1] = A4.y; a[2] = A4.z; a[3] = A4.w;
+    w[0] = W4.x; w[1] = W4.y; w[2] = W4.z; w[3] = W4.w;
+  } else {
 #pragma unroll
-    for (int u = 0; u < kEw; ++u) {
-      const int64_t v = v0 + u * stride;
-      sr[u] = -1;
-      if (v < total) {
-        cur.seek(tab, v);
-        sr[u] = cur.s;
-        const int64_t local = v - cur.vbase;
-        x[u] = (size_t)(tab.off[cur.s] + local);
-        m[u] = model_of(local, fm, M);
-        p[u] = c.P[x[u]];
-        d[u] = c.D[x[u]];
-        a[u] = c.A[x[u]];
-        w[u] = c.W[x[u]];
-      }
+    for (int i = 0; i < 4; ++i) {
+      const bool in = l0 + i < n;
+      p[i] = in ? c.P[x0 + i] : 0;
+      d[i] = in ? c.D[x0 + i] : 0;
+      a[i] = in ? c.A[x0 + i] : 0;
+      w[i] = in ? c.W[x0 + i] : 0;
     }
+  }
+  int m = l0 <= 0xffffffffll ? (int)((uint32_t)l0 - fm.div((uint32_t)l0) * (uint32_t)M)
+                             : (int)(l0 % M);
+  T rv[4];
+  uint8_t cv[4];
 #pragma unroll
-    for (int u = 0; u < kEw; ++u) {
-      if (sr[u] < 0) continue;
-      if ((p[u] | d[u] | a[u] | w[u]) == 0) {
-        cls[x[u]] = kIdle;
-        raw[x[u]] = idle_raw((T)0);
-        continue;
+  for (int i = 0; i < 4; ++i) {
+    const bool idle = (p[i] | d[i] | a[i] | w[i]) == 0;
+    rv[i] = idle ? idle_raw((T)0) : raw_tss<T>(p[i], d[i], a[i], w[i], dt, w_p[m], w_q[m]);
+    cv[i] = idle ? kIdle : kNom;
+    if (++m == M) m = 0;
+  }
+  if (v4) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) raw[x0 + i] = rv[i];
+    *reinterpret_cast<uchar4*>(cls + x0) = make_uchar4(cv[0], cv[1], cv[2], cv[3]);
+  } else {
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      if (l0 + i < n) {
+        raw[x0 + i] = rv[i];
+        cls[x0 + i] = cv[i];
       }
-      const T dt = div_rn((T)tab.win[sr[u]], (T)1000);   // window length in seconds
-      const T r_pre = div_rn(from_i32<T>(p[u]), dt);
-      const T r_dec = div_rn(from_i32<T>(d[u]), dt);
-      const T num = add_rn(mul_rn(w_p[m[u]], r_pre), r_dec);
-      T den = add_rn(from_i32<T>(a[u]), mul_rn(w_q[m[u]], from_i32<T>(w[u])));
-      if (den < (T)1) den = (T)1;                       // demand floor of one request
-      raw[x[u]] = div_rn(num, den);
-      cls[x[u]] = kNom;
-    }
   }
 }
 
@@ -506,49 +511,55 @@ __global__ void k_resolve(const __grid_constant__ SeriesTable<T> tab, const T* _
 
 // ---- Z and regions from S for every series ---------------------------------
 template <class T>
-__global__ void __launch_bounds__(kThreads)
-k_normalize(const __grid_constant__ SeriesTable<T> tab, int64_t total, FastDiv fm, const T* S,
-            const uint8_t* idle_cls, const T* theta, const T* tau_crit, T tau_crit_v,
-            const T* tau_surp, T* Z, uint8_t* cls) {
+__global__ void __launch_bounds__(kEwThreads)
+k_normalize(const __grid_constant__ SeriesTable<T> tab, const __grid_constant__ TilePlan tp,
+            FastDiv fm, bool vec, const T* S, const uint8_t* idle_cls, const T* theta,
+            const T* tau_crit, T tau_crit_v, const T* tau_surp, T* Z, uint8_t* cls) {
+  const int s = prefix_index(tp.tile_base, tab.n, blockIdx.x);
   const int M = tab.M;
-  SeriesCursor<T> cur;
-  const int64_t stride = (int64_t)gridDim.x * kThreads;
-  for (int64_t v0 = (int64_t)blockIdx.x * kThreads + threadIdx.x; v0 < total;
-       v0 += stride * kEw) {
-    size_t x[kEw];
-    int m[kEw], sr[kEw];
-    T sv[kEw], th[kEw];
-    uint8_t ic[kEw];
+  const int64_t n = (int64_t)tab.K[s] * M;
+  const int64_t l0 = (int64_t)(blockIdx.x - tp.tile_base[s]) * kTile + 4 * threadIdx.x;
+  if (l0 >= n) return;
+  const size_t x0 = (size_t)(tab.off[s] + l0);
+  const bool v4 = vec && l0 + 4 <= n;
+  T sv[4];
+  uint8_t ic[4];
+  if (v4) {
 #pragma unroll
-    for (int u = 0; u < kEw; ++u) {
-      const int64_t v = v0 + u * stride;
-      sr[u] = -1;
-      if (v < total) {
-        cur.seek(tab, v);
-        sr[u] = cur.s;
-        const int64_t local = v - cur.vbase;
-        x[u] = (size_t)(tab.off[cur.s] + local);
-        m[u] = model_of(local, fm, M);
-        sv[u] = S[x[u]];
-        th[u] = theta[(size_t)cur.s * M + m[u]];
-        ic[u] = cls ? idle_cls[x[u]] : (uint8_t)0;
-      }
-    }
+    for (int i = 0; i < 4; ++i) sv[i] = S[x0 + i];
+    const uchar4 c4 = *reinterpret_cast<const uchar4*>(idle_cls + x0);
+    ic[0] = c4.x; ic[1] = c4.y; ic[2] = c4.z; ic[3] = c4.w;
+  } else {
 #pragma unroll
-    for (int u = 0; u < kEw; ++u) {
-      if (sr[u] < 0) continue;
-      const T z = div_rn(sv[u], th[u]);
-      if (Z) Z[x[u]] = z;
-      if (cls) {
-        uint8_t c;
-        if (ic[u] == kIdle) c = kIdle;
-        else if (z < (tau_crit ? tau_crit[m[u]] : tau_crit_v)) c = kCrit;
-        else if (z > tau_surp[m[u]]) c = kSurp;
-        else c = kNom;
-        cls[x[u]] = c;
-      }
+    for (int i = 0; i < 4; ++i) {
+      const bool in = l0 + i < n;
+      sv[i] = in ? S[x0 + i] : (T)0;
+      ic[i] = in ? idle_cls[x0 + i] : kIdle;
     }
   }
+  int m = l0 <= 0xffffffffll ? (int)((uint32_t)l0 - fm.div((uint32_t)l0) * (uint32_t)M)
+                             : (int)(l0 % M);
+  T zv[4];
+  uint8_t cv[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const T z = div_rn(sv[i], theta[(size_t)s * M + m]);
+    zv[i] = z;
+    uint8_t c;
+    if (ic[i] == kIdle) c = kIdle;
+    else if (z < (tau_crit ? tau_crit[m] : tau_crit_v)) c = kCrit;
+    else if (z > tau_surp[m]) c = kSurp;
+    else c = kNom;
+    cv[i] = c;
+    if (++m == M) m = 0;
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    if (!v4 && l0 + i >= n) break;
+    if (Z) Z[x0 + i] = zv[i];
+    if (cls && !v4) cls[x0 + i] = cv[i];
+  }
+  if (cls && v4) *reinterpret_cast<uchar4*>(cls + x0) = make_uchar4(cv[0], cv[1], cv[2], cv[3]);
 }
 
 // ---- Eq. 3 receiver per window: warp per window ----------------------------
@@ -573,25 +584,30 @@ __global__ void k_receiver(int M, int K, const T* Z, const uint8_t* cls, int32_t
   if (lane == 0) recv[k] = best;
 }
 
+template <class T> TilePlan tile_plan(const SeriesTable<T>& t, int& n_tiles) {
+  TilePlan tp;
+  n_tiles = 0;
+  for (int s = 0; s < t.n; ++s) {
+    tp.tile_base[s] = n_tiles;
+    n_tiles += (int)(((int64_t)t.K[s] * t.M + kTile - 1) / kTile);
+  }
+  tp.tile_base[t.n] = n_tiles;
+  return tp;
+}
+
+// 16-byte accesses need every series to start on a 4-element boundary and
+// the arrays on 16-byte ones
+template <class T> bool quad_aligned(const SeriesTable<T>& t, std::initializer_list<const void*> ps) {
+  for (int s = 0; s < t.n; ++s)
+    if (t.off[s] % 4) return false;
+  for (const void* p : ps)
+    if (p && ((uintptr_t)p % 16)) return false;
+  return true;
+}
+
 template <class T> int64_t total_elems(const SeriesTable<T>& t) {
   int64_t n = 0;
   for (int s = 0; s < t.n; ++s) n += (int64_t)t.K[s] * t.M;
-  return n;
-}
-
-unsigned blocks_for(int64_t n, int cap) {
-  int64_t b = (n + kThreads - 1) / kThreads;
-  return (unsigned)std::max<int64_t>(1, std::min<int64_t>(b, cap));
-}
-
-int sm_count() {
-  static int n = 0;
-  if (!n) {
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1)
-      n = 148;
-  }
   return n;
 }
 
@@ -636,8 +652,10 @@ cudaError_t launch_score(const SeriesTable<T>& tab, const int32_t* P, const int3
   const int64_t total = total_elems(tab);
   if (total == 0) return cudaSuccess;
   const Counts c{P, D, A, W};
-  k_raw<T><<<blocks_for(total, sm_count() * 8), kThreads, 0, s>>>(tab, total, FastDiv(M), c, w_p,
-                                                                  w_q, w.raw, cls);
+  int n_tiles = 0;
+  const TilePlan tp = tile_plan(tab, n_tiles);
+  const bool vec = quad_aligned(tab, {P, D, A, W, w.raw, cls});
+  k_raw<T><<<n_tiles, kEwThreads, 0, s>>>(tab, tp, FastDiv(M), vec, c, w_p, w_q, w.raw, cls);
   const int64_t segs = (int64_t)n_seg * M;
   const unsigned g = (unsigned)((segs + kEmaThreads - 1) / kEmaThreads);
   if (theta)
@@ -661,8 +679,11 @@ cudaError_t launch_normalize(const SeriesTable<T>& tab, const T* S, const uint8_
                              T* Z, uint8_t* cls, cudaStream_t s) {
   const int64_t total = total_elems(tab);
   if (total == 0) return cudaSuccess;
-  k_normalize<T><<<blocks_for(total, sm_count() * 8), kThreads, 0, s>>>(
-      tab, total, FastDiv(tab.M), S, idle_cls, theta, tau_crit, tau_crit_v, tau_surp, Z, cls);
+  int n_tiles = 0;
+  const TilePlan tp = tile_plan(tab, n_tiles);
+  const bool vec = quad_aligned(tab, {S, idle_cls, Z, cls});
+  k_normalize<T><<<n_tiles, kEwThreads, 0, s>>>(tab, tp, FastDiv(tab.M), vec, S, idle_cls, theta,
+                                                tau_crit, tau_crit_v, tau_surp, Z, cls);
   return cudaGetLastError();
 }
 

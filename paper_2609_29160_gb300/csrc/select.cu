@@ -68,8 +68,7 @@ k_tick_rank(const __grid_constant__ WalkBatch<T> b, int16_t* recv_out, int16_t* 
   if (gid >= total_ent * M) return;
   const int m = (int)(gid % M);
   const int64_t e = gid / M;                       // entry over (series, tau, tick)
-  int s = 0;
-  while (s + 1 < b.n_series && (int64_t)b.ent_base[s + 1] * b.n_tau <= e) ++s;
+  const int s = prefix_index(b.ent_base, b.n_series, e, b.n_tau);
   const int64_t local = e - (int64_t)b.ent_base[s] * b.n_tau;
   const int n_ent = b.ent_base[s + 1] - b.ent_base[s];
   const int ti = (int)(local / n_ent);
@@ -147,8 +146,7 @@ k_tick_rank_small(const __grid_constant__ WalkBatch<T> b, int16_t* recv_out, int
   const int M = b.M;
   const int64_t e = (int64_t)blockIdx.x * 128 + threadIdx.x;
   if (e >= (int64_t)b.ent_base[b.n_series] * b.n_tau) return;
-  int s = 0;
-  while (s + 1 < b.n_series && (int64_t)b.ent_base[s + 1] * b.n_tau <= e) ++s;
+  const int s = prefix_index(b.ent_base, b.n_series, e, b.n_tau);
   const int local = (int)(e - (int64_t)b.ent_base[s] * b.n_tau);
   const int n_ent = b.ent_base[s + 1] - b.ent_base[s];
   const int ti = local / n_ent;
