@@ -336,7 +336,7 @@ tre_status sweep_typed(const tre_sweep_spec* sp, const SweepPlan& pl, const tre_
     lcm = lcm / std::gcd<int64_t>(lcm, pl.q[w]) * pl.q[w];
     if (lcm > 4096) break;
   }
-  const bool fused = lcm <= 4096;
+  const bool fused = lcm <= 4096 && sp->n_win <= kGaugeMaxWin;
   if (fused) {
     gp.blk = (int)(lcm * std::max<int64_t>(1, (32 + lcm - 1) / lcm));
     if (gp.blk < kGaugeMinBlk) gp.blk = (int)(lcm * ((kGaugeMinBlk + lcm - 1) / lcm));

@@ -48,6 +48,7 @@ struct ReduceWs {
   int n_traces;
 };
 constexpr int kGaugeMinBlk = 16;   // shortest row block of the fused gauge pass
+constexpr int kGaugeMaxWin = 8;    // most window lengths the fused gauge pass takes
 void reduce_ws_layout(Arena& a, int M, int K, int n_traces, int64_t n_req, ReduceWs& w);
 // Request records of n_traces traces (host array of column sets) on one grid;
 // trace t writes P, D (and the packed SLO counts when slo != null) at element

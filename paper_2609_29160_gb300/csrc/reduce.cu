@@ -731,7 +731,8 @@ k_gauge_apply(const __grid_constant__ GaugePlan gp, const int32_t* __restrict__ 
               const int32_t* __restrict__ Din, const unsigned long long* __restrict__ sloin,
               int32_t* __restrict__ P, int32_t* __restrict__ D, int32_t* __restrict__ A,
               int32_t* __restrict__ W, unsigned long long* __restrict__ slo) {
-  constexpr int NW = 16;
+  constexpr int NW = kGaugeMaxWin;
+  constexpr int RB = 4;   // rows whose loads are issued together
   const int M = gp.M, Kb = gp.Kb;
   const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
   if (t >= (int64_t)gp.n_traces * gp.nblk * M) return;
@@ -750,34 +751,49 @@ k_gauge_apply(const __grid_constant__ GaugePlan gp, const int32_t* __restrict__ 
     cnt[j] = j < gp.n_win ? gp.q[j] : 0;
     kq[j] = j < gp.n_win ? k0 / gp.q[j] : 0;
   }
-  for (int k = k0; k < k1; ++k) {
-    a += dA[dbase + (size_t)k * M];
-    w += dW[dbase + (size_t)k * M];
-    const size_t xi = ibase + (size_t)k * M;
-    const int32_t p = Pin[xi], d = Din[xi];
-    const unsigned long long sl = sloin ? sloin[xi] : 0ull;
+  for (int kb = k0; kb < k1; kb += RB) {
+    int32_t va[RB], vw[RB], vp[RB], vd[RB];
+    unsigned long long vs[RB];
 #pragma unroll
-    for (int j = 0; j < NW; ++j) {
-      if (j >= gp.n_win) break;
-      if (j == gp.base_w) {
-        const size_t o = (size_t)gp.out_off[tr][j] + (size_t)k * M + m;
-        A[o] = a;
-        W[o] = w;
-        continue;
-      }
-      ap[j] += p;
-      ad[j] += d;
-      as[j] += sl;
-      if (--cnt[j] == 0) {
-        const size_t o = (size_t)gp.out_off[tr][j] + (size_t)kq[j] * M + m;
-        P[o] = ap[j];
-        D[o] = ad[j];
-        A[o] = a;
-        W[o] = w;
-        if (slo) slo[o] = as[j];
-        ap[j] = 0; ad[j] = 0; as[j] = 0;
-        cnt[j] = gp.q[j];
-        ++kq[j];
+    for (int r = 0; r < RB; ++r) {
+      const int k = kb + r;
+      const bool in = k < k1;
+      const size_t xd = dbase + (size_t)k * M, xi = ibase + (size_t)k * M;
+      va[r] = in ? dA[xd] : 0;
+      vw[r] = in ? dW[xd] : 0;
+      vp[r] = in ? Pin[xi] : 0;
+      vd[r] = in ? Din[xi] : 0;
+      vs[r] = in && sloin ? sloin[xi] : 0ull;
+    }
+#pragma unroll
+    for (int r = 0; r < RB; ++r) {
+      const int k = kb + r;
+      if (k >= k1) break;
+      a += va[r];
+      w += vw[r];
+#pragma unroll
+      for (int j = 0; j < NW; ++j) {
+        if (j >= gp.n_win) break;
+        if (j == gp.base_w) {
+          const size_t o = (size_t)gp.out_off[tr][j] + (size_t)k * M + m;
+          A[o] = a;
+          W[o] = w;
+          continue;
+        }
+        ap[j] += vp[r];
+        ad[j] += vd[r];
+        as[j] += vs[r];
+        if (--cnt[j] == 0) {
+          const size_t o = (size_t)gp.out_off[tr][j] + (size_t)kq[j] * M + m;
+          P[o] = ap[j];
+          D[o] = ad[j];
+          A[o] = a;
+          W[o] = w;
+          if (slo) slo[o] = as[j];
+          ap[j] = 0; ad[j] = 0; as[j] = 0;
+          cnt[j] = gp.q[j];
+          ++kq[j];
+        }
       }
     }
   }
