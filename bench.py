@@ -172,10 +172,11 @@ def phase_bytes(sw, n_records_per_trace, M):
         # 7 int32 columns per record in; P, D, A/W diffs (4 B each) and the
         # packed SLO counts (8 B) per base cell out
         "reduce": float(np.sum(n_records_per_trace)) * 28 + base * 24,
-        # diffs in, gauges out
-        "gauge_scan": base * 16,
-        # base counts + SLO in, series counts + SLO out
-        "aggregate": base * 24 + mw * 24,
+        # gauge diffs in (block sums and their prefixes)
+        "gauge_scan": base * 8,
+        # diffs, base counts and SLO in; base gauges and every coarser
+        # series' counts, gauges and SLO out
+        "aggregate": base * (8 + 16) + base * 8 + (mw - base) * 24,
         # counts in, S and the idle flag out
         "score": mw * (16 + 4 + 1),
         # S, idle flag and SLO counts in
