@@ -92,7 +92,7 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win,
   while (t + 1 < bt.n && bt.cta_base[t + 1] <= (int)blockIdx.x) ++t;
   const ReqCols& r = bt.cols[t];
   const bool vec = (bt.vec_ok >> t) & 1ull;
-  const size_t cells0 = (size_t)K * M, cells1 = (size_t)(K + 1) * M;
+  const size_t cells1 = (size_t)(K + 1) * M;
   int32_t* P = P0 + bt.out_off[t];
   int32_t* D = D0 + bt.out_off[t];
   int32_t* dA = dA0 + t * cells1;
@@ -633,30 +633,32 @@ k_aggregate(const __grid_constant__ AggPlan pl, const int32_t* __restrict__ P,
   }
 }
 
-// Clears a list of 32-bit word ranges in one launch (16-byte stores where a
-// range allows them).
+// Clears a list of 32-bit word ranges in one launch: every CTA clears one
+// chunk of kZeroChunk words of one range (16-byte stores where the range's
+// alignment allows them), the chunks of all ranges numbered back to back.
 constexpr int kMaxZero = 3 * kMaxTraces + 2;
+constexpr int kZeroChunk = kThreads * 16;   // words per CTA
 struct ZeroList {
   int n;
   uint32_t* ptr[kMaxZero];
   int64_t words[kMaxZero];
+  int32_t cta_base[kMaxZero + 1];
 };
 
 __global__ void __launch_bounds__(kThreads) k_zero(const __grid_constant__ ZeroList zl) {
-  const int64_t stride = (int64_t)gridDim.x * kThreads;
-  const int64_t tid = (int64_t)blockIdx.x * kThreads + threadIdx.x;
-  for (int r = 0; r < zl.n; ++r) {
-    uint32_t* p = zl.ptr[r];
-    const int64_t n = zl.words[r];
-    // words before the first 16-byte boundary, then whole 16-byte groups, then the tail
-    const int64_t head = min64(n, (int64_t)((16 - ((uintptr_t)p & 15)) & 15) / 4);
-    if (tid < head) p[tid] = 0u;
-    uint4* q = reinterpret_cast<uint4*>(p + head);
-    const int64_t nq = (n - head) / 4;
-    for (int64_t i = tid; i < nq; i += stride) q[i] = make_uint4(0u, 0u, 0u, 0u);
-    const int64_t t0 = head + nq * 4;
-    if (tid < n - t0) p[t0 + tid] = 0u;
-  }
+  const int r = prefix_index(zl.cta_base, zl.n, blockIdx.x);
+  uint32_t* p = zl.ptr[r];
+  const int64_t n = zl.words[r];
+  const int64_t w0 = (int64_t)(blockIdx.x - zl.cta_base[r]) * kZeroChunk;
+  const int64_t w1 = min64(n, w0 + kZeroChunk);
+  // words up to the first 16-byte boundary of the chunk, 16-byte groups, tail
+  const int64_t head = min64(w1 - w0, (int64_t)((16 - ((uintptr_t)(p + w0) & 15)) & 15) / 4);
+  if (threadIdx.x < head) p[w0 + threadIdx.x] = 0u;
+  uint4* q = reinterpret_cast<uint4*>(p + w0 + head);
+  const int64_t nq = (w1 - w0 - head) / 4;
+  for (int64_t i = threadIdx.x; i < nq; i += kThreads) q[i] = make_uint4(0u, 0u, 0u, 0u);
+  const int64_t t0 = w0 + head + nq * 4;
+  if (threadIdx.x < w1 - t0) p[t0 + threadIdx.x] = 0u;
 }
 
 // ---- gauge scan fused with the exact coarsening (sweeps) --------------------
@@ -870,7 +872,13 @@ cudaError_t launch_reduce_requests(const ReqCols* traces, int n_traces, int M, i
   zl.words[zl.n++] = (int64_t)(cells + (size_t)M * n_traces);
   zl.ptr[zl.n] = reinterpret_cast<uint32_t*>(w.dW);
   zl.words[zl.n++] = (int64_t)(cells + (size_t)M * n_traces);
-  k_zero<<<num_sms() * 8, kThreads, 0, s>>>(zl);
+  int zctas = 0;
+  for (int r = 0; r < zl.n; ++r) {
+    zl.cta_base[r] = zctas;
+    zctas += (int)((zl.words[r] + kZeroChunk - 1) / kZeroChunk);
+  }
+  zl.cta_base[zl.n] = zctas;
+  if (zctas > 0) k_zero<<<zctas, kThreads, 0, s>>>(zl);
   int64_t total_n = 0;
   for (int t = 0; t < n_traces; ++t) total_n += traces[t].n;
   // records per CTA sized on the whole batch so the grid fills the GPU
