@@ -160,6 +160,32 @@ def cpu_baseline(scale):
             "sample": f"1 of the 7 traces ({n_rec} records), all 4 window lengths, all 64 settings; {dt:.1f} s"}
 
 
+# DRAM traffic per call of a phase, from the committed ncu summary of its
+# kernels; used only while the kernel source is the one the counters were
+# taken on (the summary records its SHA-256)
+TRAFFIC_SUMMARIES = {"reduce": ("profiles/k_reduce_requests_sweep_7x1M.md",
+                                "paper_2609_29160_gb300/csrc/reduce.cu")}
+
+
+def captured_traffic(phase):
+    import hashlib
+    if phase not in TRAFFIC_SUMMARIES:
+        return None
+    summ, src = (os.path.join(ROOT, f) for f in TRAFFIC_SUMMARIES[phase])
+    try:
+        fields = {}
+        for line in open(summ):
+            if ":" in line and line.strip().startswith(("dram_bytes_per_call", "source_sha256")):
+                k, v = line.strip().strip("`-* ").split(":", 1)
+                fields[k.strip()] = v.strip().strip("`")
+        digest = hashlib.sha256(open(src, "rb").read()).hexdigest()
+        if fields.get("source_sha256") != digest:
+            return None
+        return float(fields["dram_bytes_per_call"])
+    except (OSError, KeyError, ValueError):
+        return None
+
+
 def phase_bytes(sw, n_records_per_trace, M):
     """Algorithmic bytes of one call of each phase over the whole sweep: what the
     method must read and write once, per record and per (window, model)."""
@@ -278,7 +304,7 @@ def main():
         per_call_ms = phases[name]["ms"] / max(phases[name]["calls"], 1)
         achieved = pb[name] / (per_call_ms / 1e3) / 1e9
         return {"bound": "hbm", "kernel": name, "achieved": achieved, "peak": hbm,
-                "unit": "GB/s", "frac": achieved / hbm, "traffic": None,
+                "unit": "GB/s", "frac": achieved / hbm, "traffic": captured_traffic(name),
                 "share_of_step": phases[name]["ms"] / max(ms, 1e-9), "peak_kind": peak_kind,
                 "bytes_per_call": pb[name], "us_per_call": per_call_ms * 1e3}
     if dom in pb and phases[dom]["calls"]:
