@@ -46,6 +46,25 @@ def parse():
     return ap.parse_args()
 
 
+def rank_seed0(rank):
+    """First trace seed of a rank's sweep: rank r sweeps traces 100 + 7r ..
+    106 + 7r, so the ranks' problems are disjoint (weak scaling)."""
+    return 100 + 7 * rank
+
+
+def over_ranks(dist, device, ms, units):
+    """Whole-job figures of a multi-rank run: the slowest rank's milliseconds
+    and the units (records, model-windows) summed over all ranks."""
+    import torch
+    t = torch.tensor([float(ms)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    if not units:
+        return float(t.item()), []
+    u = torch.tensor([float(x) for x in units], dtype=torch.float64, device=device)
+    dist.all_reduce(u, op=dist.ReduceOp.SUM)
+    return float(t.item()), [float(x) for x in u.tolist()]
+
+
 def alphas(windows):
     return [min(1.0, w / 5000.0) for w in windows]
 
@@ -236,7 +255,7 @@ def main():
     lib.tre_trace_collect.argtypes = [C.POINTER(Trace)]
 
     # each rank sweeps its own 7 traces (independent problems: weak scaling)
-    sw = tracegen.sweep_workload(scale=args.scale, seed0=100 + 7 * rank)
+    sw = tracegen.sweep_workload(scale=args.scale, seed0=rank_seed0(rank))
     M = sw["M"]
     win = sw["window_ms"]
     al = alphas(win)
@@ -284,13 +303,13 @@ def main():
     lib.tre_trace_collect(C.byref(tr))
     lib.tre_trace_enable(0)
     clk = clocks.stop()
+    job_rec, job_mw, job_inst = total_rec, model_windows, n_inst
     if world > 1:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+        ms, (job_rec, job_mw, job_inst) = over_ranks(dist, "cuda", ms,
+                                                     [total_rec, model_windows, n_inst])
     ms_step = ms / args.steps
-    value = total_rec * world * args.steps / (ms / 1e3)
-    mw_s = model_windows * world * args.steps / (ms / 1e3)
+    value = job_rec * args.steps / (ms / 1e3)
+    mw_s = job_mw * args.steps / (ms / 1e3)
     phases = {tr.name[i].decode(): {"ms": tr.ms[i], "calls": tr.calls[i],
                                     "launches": tr.launches[i]} for i in range(tr.n_phases)}
     launches = int(sum(p["launches"] for p in phases.values()))
@@ -343,10 +362,8 @@ def main():
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1) / args.e2e_steps
     if world > 1:
-        t = torch.tensor([e2e_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
-    e2e = {"value": total_rec * world / (e2e_ms / 1e3), "unit": UNIT,
+        e2e_ms, _ = over_ranks(dist, "cuda", e2e_ms, [])
+    e2e = {"value": job_rec / (e2e_ms / 1e3), "unit": UNIT,
            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
            "ms_per_step": e2e_ms}
 
@@ -359,9 +376,9 @@ def main():
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
             "data": "synthetic",
-            "config": {"workload": WORKLOAD, "records_per_step": total_rec * world,
-                       "model_windows_per_step": model_windows * world,
-                       "controller_instances": n_inst * world, "scale": args.scale,
+            "config": {"workload": WORKLOAD, "records_per_step": int(job_rec),
+                       "model_windows_per_step": int(job_mw),
+                       "controller_instances": int(job_inst), "scale": args.scale,
                        "l2": "inputs larger than L2 (7 x 28 B x ~1M records = 196 MB per step)",
                        "parallelism": f"independent sweeps per GPU x{world}"},
             "model_windows_per_s": mw_s,
