@@ -207,6 +207,7 @@ k_search(const __grid_constant__ SeriesTable<T> tab, const typename KeyOf<T>::U*
   __shared__ int64_t red64[kWarps];
   __shared__ int red32[kWarps];
   __shared__ int nsel_s;
+  __shared__ U bfmin_s;
   const int M = tab.M;
   const int s = blockIdx.x / M, m = blockIdx.x % M;
   const int K = tab.K[s];
@@ -241,12 +242,17 @@ k_search(const __grid_constant__ SeriesTable<T> tab, const typename KeyOf<T>::U*
     int32_t* hpre = reinterpret_cast<int32_t*>(list + kCap);
     int sh = 0;
     while (sh < 63 && ((kmax - kmin) >> sh) >= (U)kFine) ++sh;
+    (void)fmn;
     for (int b = tid; b < kFine; b += kNB) {
       fcnt[b] = 0;
       fhl[b] = 0;
-      fmn[b] = ~(U)0;
     }
+    if (tid == 0) bfmin_s = ~(U)0;
     __syncthreads();
+    // with fewer than 2^16 candidates, a bucket's count and healthy count
+    // share one 32-bit word (one atomic per key)
+    const bool packed = ncand_g[out] < 65536u;
+    uint32_t* fpk = reinterpret_cast<uint32_t*>(fcnt);
     for (int i0 = 0; i0 < K; i0 += kNB * kUnroll) {
       U pv[kUnroll];
 #pragma unroll
@@ -258,16 +264,25 @@ k_search(const __grid_constant__ SeriesTable<T> tab, const typename KeyOf<T>::U*
       for (int u = 0; u < kUnroll; ++u) {
         const U p = pv[u];
         if (!p) continue;
-        const U key = p >> 1;
-        const int b = (int)((key - kmin) >> sh);
-        atomicAdd(&fcnt[b], 1);
-        if (p & 1) atomicAdd(&fhl[b], 1);
-        if (key < fmn[b]) atomicMin(&fmn[b], key);
+        const int b = (int)(((p >> 1) - kmin) >> sh);
+        if (packed) {
+          atomicAdd(&fpk[b], 1u + ((uint32_t)(p & 1) << 16));
+        } else {
+          atomicAdd(&fcnt[b], 1);
+          if (p & 1) atomicAdd(&fhl[b], 1);
+        }
       }
     }
     __syncthreads();
     constexpr int PER = kFine / kNB;            // consecutive buckets per thread
     const int b0 = tid * PER;
+    if (packed) {
+      for (int j = 0; j < PER; ++j) {
+        const uint32_t v = fpk[b0 + j];
+        fcnt[b0 + j] = (int32_t)(v & 0xffffu);
+        fhl[b0 + j] = (int32_t)(v >> 16);
+      }
+    }
     int64_t tc = 0, th = 0;
     for (int j = 0; j < PER; ++j) {
       tc += fcnt[b0 + j];
@@ -303,11 +318,23 @@ k_search(const __grid_constant__ SeriesTable<T> tab, const typename KeyOf<T>::U*
     if (my_sel) atomicAdd(&nsel_s, (int)my_sel);
     __syncthreads();
     const int nsel = nsel_s;
+    // smallest key of the found bucket bf, by a pass over the keys (the gather
+    // pass below does it on the way when there are keys to gather)
+    auto bucket_min_pass = [&]() {
+      U lm = ~(U)0;
+      for (int i = tid; i < K; i += kNB) {
+        const U p = mk[i];
+        if (p && (int)(((p >> 1) - kmin) >> sh) == bf && (p >> 1) < lm) lm = p >> 1;
+      }
+      if (lm != ~(U)0) atomicMin(&bfmin_s, lm);
+      __syncthreads();
+    };
     if (nsel <= kCap) {
       if (nsel == 0) {
+        if (bf != 0x7fffffff) bucket_min_pass();
         if (tid == 0) {
           if (bf != 0x7fffffff) {
-            theta[out] = value_of(fmn[bf]);
+            theta[out] = value_of(bfmin_s);
           } else {
             theta[out] = value_of(kmax);
             atomicAdd(&diag->degenerate_calib, 1ull);
@@ -328,6 +355,7 @@ k_search(const __grid_constant__ SeriesTable<T> tab, const typename KeyOf<T>::U*
       }
       if (tid == 0) nsel_s = 0;
       __syncthreads();
+      U lmin = ~(U)0;
       for (int i0 = 0; i0 < K; i0 += kNB * kUnroll) {
         U pv[kUnroll];
 #pragma unroll
@@ -341,8 +369,10 @@ k_search(const __grid_constant__ SeriesTable<T> tab, const typename KeyOf<T>::U*
           if (!p) continue;
           const int b = (int)(((p >> 1) - kmin) >> sh);
           if (fst[b] >= 0) list[atomicAdd(&nsel_s, 1)] = p;
+          if (b == bf && (p >> 1) < lmin) lmin = p >> 1;
         }
       }
+      if (lmin != ~(U)0) atomicMin(&bfmin_s, lmin);
       int n2 = 32;
       while (n2 < nsel) n2 <<= 1;
       for (int i = nsel + tid; i < n2; i += kNB) list[i] = ~(U)0;
@@ -396,7 +426,7 @@ k_search(const __grid_constant__ SeriesTable<T> tab, const typename KeyOf<T>::U*
         if (best != 0x7fffffff) {
           theta[out] = value_of(list[best] >> 1);
         } else if (bf != 0x7fffffff) {
-          theta[out] = value_of(fmn[bf]);
+          theta[out] = value_of(bfmin_s);
         } else {
           theta[out] = value_of(kmax);
           atomicAdd(&diag->degenerate_calib, 1ull);
