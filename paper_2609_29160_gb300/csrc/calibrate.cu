@@ -184,11 +184,11 @@ __device__ __forceinline__ int block_min(int v, int* red) {
 
 constexpr int kFine = 4096;     // buckets of the first histogram
 constexpr int kUnroll = 8;      // keys per thread whose loads are issued together
-constexpr int kCap = 4096;      // most keys the exact pass sorts in shared memory
+constexpr int kCap = 2048;      // most keys the exact pass sorts in shared memory
 
 template <class T> size_t search_smem_bytes() {
   using U = typename KeyOf<T>::U;
-  const size_t fast = (size_t)kFine * (5 * 4 + sizeof(U)) + (size_t)kCap * (sizeof(U) + 4);
+  const size_t fast = (size_t)kFine * (5 * 4) + (size_t)kCap * (sizeof(U) + 4);
   const size_t descent = (size_t)KeyOf<T>::kLevels * kNB * (4 + 4 + sizeof(U));
   return fast > descent ? fast : descent;
 }
@@ -237,12 +237,10 @@ k_search(const __grid_constant__ SeriesTable<T> tab, const typename KeyOf<T>::U*
     int32_t* fst = fhl + kFine;                 // run start of a selected bucket, -1 if not
     int32_t* fca = fst + kFine;                 // windows in buckets above
     int32_t* fha = fca + kFine;                 // healthy windows in buckets above
-    U* fmn = reinterpret_cast<U*>(fha + kFine);
-    U* list = fmn + kFine;
+    U* list = reinterpret_cast<U*>(fha + kFine);
     int32_t* hpre = reinterpret_cast<int32_t*>(list + kCap);
     int sh = 0;
     while (sh < 63 && ((kmax - kmin) >> sh) >= (U)kFine) ++sh;
-    (void)fmn;
     for (int b = tid; b < kFine; b += kNB) {
       fcnt[b] = 0;
       fhl[b] = 0;
