@@ -111,24 +111,35 @@ k_pack(const __grid_constant__ SeriesTable<T> tab, const __grid_constant__ PackP
   U lmin = ~(U)0, lmax = 0;
   uint32_t lc = 0;
   const int TKp = pp.tk + 1;   // padded row of the transposed tile
+  constexpr int J = kPackTile / kPackThreads;
+  // every load of the thread's elements first, then the threshold lookups,
+  // then the keys: more requests in flight per thread
+  unsigned long long cj[J];
+  T sj[J];
+  uint8_t ij[J];
+  bool in[J];
 #pragma unroll
-  for (int j = 0; j < kPackTile / kPackThreads; ++j) {
-    const int e = tid + j * kPackThreads;
-    const int kk = e >> pp.lg_tm;
-    const int k = k0 + kk;
+  for (int j = 0; j < J; ++j) {
+    const int k = k0 + ((tid + j * kPackThreads) >> pp.lg_tm);
+    in[j] = k < K && m < M;
+    const size_t x = off + (size_t)k * M + m;
+    cj[j] = in[j] ? slo[x] : 0ull;
+    sj[j] = in[j] ? S[x] : (T)0;
+    ij[j] = in[j] ? cls[x] : kIdle;
+  }
+  bool hj[J];
+#pragma unroll
+  for (int j = 0; j < J; ++j) hj[j] = healthy((uint32_t)cj[j], (uint32_t)(cj[j] >> 32), thr, ok_frac);
+#pragma unroll
+  for (int j = 0; j < J; ++j) {
+    const int kk = (tid + j * kPackThreads) >> pp.lg_tm;
     U v = 0;
-    if (k < K && m < M) {
-      const size_t x = off + (size_t)k * M + m;
-      const unsigned long long c = slo[x];
-      const uint32_t n_arr = (uint32_t)c, n_met = (uint32_t)(c >> 32);
-      const T sv = S[x];
-      if (cls[x] != kIdle && n_arr >= 1 && sv > (T)0) {
-        const U key = (U)key_of(sv);
-        v = (key << 1) | (U)(healthy(n_arr, n_met, thr, ok_frac) ? 1 : 0);
-        lmin = key < lmin ? key : lmin;
-        lmax = key > lmax ? key : lmax;
-        ++lc;
-      }
+    if (in[j] && ij[j] != kIdle && (uint32_t)cj[j] >= 1 && sj[j] > (T)0) {
+      const U key = (U)key_of(sj[j]);
+      v = (key << 1) | (U)(hj[j] ? 1 : 0);
+      lmin = key < lmin ? key : lmin;
+      lmax = key > lmax ? key : lmax;
+      ++lc;
     }
     tile[mm * TKp + kk] = v;
   }
