@@ -191,12 +191,13 @@ def captured_traffic(phase):
     if phase not in TRAFFIC_SUMMARIES:
         return None
     summ, src = (os.path.join(ROOT, f) for f in TRAFFIC_SUMMARIES[phase])
+    import re
     try:
         fields = {}
         for line in open(summ):
-            if ":" in line and line.strip().startswith(("dram_bytes_per_call", "source_sha256")):
-                k, v = line.strip().strip("`-* ").split(":", 1)
-                fields[k.strip()] = v.strip().strip("`")
+            hit = re.match(r"^[-*\s]*(dram_bytes_per_call|source_sha256):\s*`?([0-9a-f]+)`?", line)
+            if hit:
+                fields[hit.group(1)] = hit.group(2)
         digest = hashlib.sha256(open(src, "rb").read()).hexdigest()
         if fields.get("source_sha256") != digest:
             return None
