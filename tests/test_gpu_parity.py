@@ -411,3 +411,23 @@ def test_sweep_small(tre):
     sw["pacing_cap"] = sw["pacing_cap"][::3]
     ref, out = _run_sweep_both(tre, sw, alpha, moves_cap=512)
     _compare_sweep(tre, sw, ref, out, 512)
+
+
+def test_reduce_requests_from_pinned_host_memory(tre):
+    """Record columns left in pinned host memory that the GPU addresses
+    directly give the same counts as device-resident columns."""
+    import os
+    import sys
+    import torch
+    sys.path.insert(0, os.path.dirname(os.path.dirname(os.path.abspath(__file__))))
+    import bench
+    rng = np.random.default_rng(31)
+    M, win, K = 8, 100, 1200
+    req = _sorted_long(rng, 20001, M, win, K)
+    host = {k: torch.as_tensor(v).pin_memory() for k, v in req.items()}
+    if not bench.host_mapped(host["model"].data_ptr()):
+        pytest.skip("pinned host memory is not mapped at the same address on this system")
+    ref = tre.tss_window_reduce(M, win, K, requests=_cuda(req))
+    got = tre.tss_window_reduce(M, win, K, requests=host)
+    for k in "PDAW":
+        assert torch.equal(got[k], ref[k]), k
