@@ -74,8 +74,9 @@ typedef struct {
 /* Request records, structure of arrays (int32, length n), in device memory or
  * in pinned host memory that the GPU addresses directly (cudaHostAlloc'd
  * memory under unified addressing; the kernels then read it over the host
- * link, with no separate copy). Columns on 16-byte boundaries are read 16
- * bytes at a time. Times in ms.
+ * link, with no separate copy; pageable host memory is refused with
+ * TRE_EINVAL). Columns on 16-byte boundaries are read 16 bytes at a time.
+ * Times in ms.
  * A record is valid when 0 <= model < n_models, 0 <= t_arr < n_windows*window_ms,
  * t_arr <= t_start <= t_first <= t_end, L_in >= 0 and L_out >= 1. Prompt tokens
  * count at t_first; decode token j is emitted at

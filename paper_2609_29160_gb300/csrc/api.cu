@@ -17,11 +17,27 @@ bool grid_ok(const tre_grid* g) {
          (int64_t)g->n_windows * g->window_ms < (int64_t)2147483647;
 }
 
+// A column the kernels may read: device memory, or host memory the GPU
+// addresses (pinned and mapped). Plain pageable host memory is refused here,
+// since a kernel reading it would fault. When the runtime cannot tell (no
+// device), the launch decides.
+bool gpu_addressable(const void* p) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return true;
+  }
+  return a.type != cudaMemoryTypeUnregistered;
+}
+
 bool req_ok(const tre_requests* r) {
   if (!r || r->n < 0) return false;
   if (r->n == 0) return true;
-  return r->model && r->t_arr_ms && r->t_start_ms && r->t_first_ms && r->t_end_ms && r->L_in &&
-         r->L_out;
+  const void* cols[7] = {r->model, r->t_arr_ms, r->t_start_ms, r->t_first_ms, r->t_end_ms,
+                         r->L_in, r->L_out};
+  for (const void* c : cols)
+    if (!c || !gpu_addressable(c)) return false;
+  return true;
 }
 
 bool ev_ok(const tre_events* e) {

@@ -80,7 +80,7 @@ __device__ __forceinline__ uint32_t ceil_div(unsigned long long x, uint32_t d) {
   return (uint32_t)(q + (r != 0));
 }
 
-template <bool SLO>
+template <bool SLO, bool COPY>
 __global__ void __launch_bounds__(kThreads, 4)
 k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win, FastDiv fd,
                   int K, int near_rows, int lgF, int32_t* __restrict__ P0,
@@ -103,12 +103,38 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win,
   if (n_loc <= 0) return;
   const int Mp = 1 << lgMp, F = 1 << lgF, F1 = F + 1;
   const uint32_t span = (uint32_t)K * (uint32_t)win;
-  const int a_first = r.t_arr[i0], a_last = r.t_arr[i0 + n_loc - 1];
+  // Columns of this CTA's records: read in place, or (COPY, for records in
+  // host memory) first copied once into shared memory so that no column is
+  // read twice over the host link.
+  const int32_t* gcol[7] = {r.model + i0, r.t_arr + i0, r.t_start + i0, r.t_first + i0,
+                            r.t_end + i0, r.L_in + i0, r.L_out + i0};
+  const int32_t* colp[7];
+  int32_t* recs = reinterpret_cast<int32_t*>(smem);
+  const int cap_rec = COPY ? (int)bt.per_cta[t] : 0;
+  if (COPY) {
+#pragma unroll
+    for (int c = 0; c < 7; ++c) {
+      int32_t* dst = recs + (size_t)c * cap_rec;
+      for (int i = threadIdx.x * 4; i < n_loc; i += kThreads * 4) {
+        if (vec && i + 4 <= n_loc) {
+          *reinterpret_cast<int4*>(dst + i) = *reinterpret_cast<const int4*>(gcol[c] + i);
+        } else {
+          for (int u = 0; u < 4 && i + u < n_loc; ++u) dst[i + u] = gcol[c][i + u];
+        }
+      }
+      colp[c] = dst;
+    }
+  } else {
+#pragma unroll
+    for (int c = 0; c < 7; ++c) colp[c] = gcol[c];
+  }
+  const bool vec4 = COPY || vec;
+  const int a_first = gcol[1][0], a_last = gcol[1][n_loc - 1];
   const int k_lo = a_first < 0 ? 0 : (int)min(fd.div((uint32_t)a_first), (uint32_t)K);
   const int k_hi = a_last < 0 ? 0 : (int)min(fd.div((uint32_t)a_last), (uint32_t)K);
   const int used = min(near_rows, (k_hi >= k_lo ? k_hi - k_lo + 1 : 1) + 1);
   Stage st;
-  st.aW = reinterpret_cast<int32_t*>(smem);
+  st.aW = reinterpret_cast<int32_t*>(smem + (size_t)cap_rec * 7 / 2);
   st.aS = reinterpret_cast<uint32_t*>(st.aW + (size_t)near_rows * Mp);
   st.fP = reinterpret_cast<int32_t*>(st.aS + (SLO ? (size_t)near_rows * Mp : 0));
   st.fD = st.fP + (size_t)M * F1;
@@ -129,17 +155,17 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win,
   // each model's earliest start window among this CTA's records
   for (int b = threadIdx.x * kVec; b < n_loc; b += kThreads * kVec) {
     int mm[kVec], ss[kVec];
-    if (vec && b + kVec <= n_loc) {
-      const int4 a = *reinterpret_cast<const int4*>(r.model + i0 + b);
-      const int4 s = *reinterpret_cast<const int4*>(r.t_start + i0 + b);
+    if (vec4 && b + kVec <= n_loc) {
+      const int4 a = *reinterpret_cast<const int4*>(colp[0] + b);
+      const int4 s = *reinterpret_cast<const int4*>(colp[2] + b);
       mm[0] = a.x; mm[1] = a.y; mm[2] = a.z; mm[3] = a.w;
       ss[0] = s.x; ss[1] = s.y; ss[2] = s.z; ss[3] = s.w;
     } else {
 #pragma unroll
       for (int u = 0; u < kVec; ++u) {
         const bool in = b + u < n_loc;
-        mm[u] = in ? r.model[i0 + b + u] : -1;
-        ss[u] = in ? r.t_start[i0 + b + u] : -1;
+        mm[u] = in ? colp[0][b + u] : -1;
+        ss[u] = in ? colp[2][b + u] : -1;
       }
     }
 #pragma unroll
@@ -182,11 +208,11 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win,
   for (int wb = warp * 32 * kVec; wb < n_loc; wb += kThreads * kVec) {
     const int b = wb + lane * kVec;
     int v[7][kVec];
-    const int32_t* cols[7] = {r.model, r.t_arr, r.t_start, r.t_first, r.t_end, r.L_in, r.L_out};
-    if (vec && b + kVec <= n_loc) {
+    if (vec4 && b + kVec <= n_loc) {
 #pragma unroll
       for (int c = 0; c < 7; ++c) {
-        const int4 q = __ldcs(reinterpret_cast<const int4*>(cols[c] + i0 + b));
+        const int4 q = COPY ? *reinterpret_cast<const int4*>(colp[c] + b)
+                            : __ldcs(reinterpret_cast<const int4*>(colp[c] + b));
         v[c][0] = q.x; v[c][1] = q.y; v[c][2] = q.z; v[c][3] = q.w;
       }
     } else {
@@ -194,7 +220,7 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win,
       for (int u = 0; u < kVec; ++u) {
         const bool in = b + u < n_loc;
 #pragma unroll
-        for (int c = 0; c < 7; ++c) v[c][u] = in ? cols[c][i0 + b + u] : 0;
+        for (int c = 0; c < 7; ++c) v[c][u] = in ? colp[c][b + u] : 0;
         if (!in) v[0][u] = -1;   // marks "no record" (not counted as a drop)
       }
     }
@@ -881,8 +907,18 @@ cudaError_t launch_reduce_requests(const ReqCols* traces, int n_traces, int M, i
   if (zctas > 0) k_zero<<<zctas, kThreads, 0, s>>>(zl);
   int64_t total_n = 0;
   for (int t = 0; t < n_traces; ++t) total_n += traces[t].n;
+  // records that live in host memory (pinned, mapped) are copied into shared
+  // memory once per CTA rather than read twice over the host link
+  bool copy_records = false;
+  for (int t = 0; t < n_traces; ++t) {
+    cudaPointerAttributes pa;
+    if (traces[t].n > 0 && cudaPointerGetAttributes(&pa, traces[t].model) == cudaSuccess &&
+        pa.type == cudaMemoryTypeHost)
+      copy_records = true;
+  }
   // records per CTA sized on the whole batch so the grid fills the GPU
-  const int64_t per = per_cta_records(std::max<int64_t>(total_n / n_traces, 1), 1024, 8192,
+  const int64_t per = per_cta_records(std::max<int64_t>(total_n / n_traces, 1), 1024,
+                                      copy_records ? 2048 : 8192,
                                       kThreads * kVec);   // whole passes for every warp
   static_assert(8192 <= kMaxPerCta, "packed shared counters need <= kMaxPerCta records per CTA");
   int ctas = 0;
@@ -912,26 +948,44 @@ cudaError_t launch_reduce_requests(const ReqCols* traces, int n_traces, int M, i
   int lgF = 3;
   while (lgF < 8 && (size_t)12 * M * ((2 << lgF) + 1) <= 16 * 1024) ++lgF;
   const int F = 1 << lgF;
-  const size_t smem = (size_t)near_rows * Mp * (4 + (slo ? 4 : 0)) + (size_t)12 * M * (F + 1) +
-                      (size_t)M * 8;
+  const size_t smem_stage = (size_t)near_rows * Mp * (4 + (slo ? 4 : 0)) +
+                            (size_t)12 * M * (F + 1) + (size_t)M * 8;
+  // records in host memory are copied into shared memory once per CTA
+  const size_t smem_copy = copy_records ? (size_t)per * 7 * 4 : 0;
+  const size_t smem = smem_stage + smem_copy;
   if (smem > 200 * 1024) return cudaErrorInvalidValue;
   static bool attr = false;
   if (!attr) {
-    cudaError_t e1 = cudaFuncSetAttribute(k_reduce_requests<true>,
-                                          cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
-    cudaError_t e2 = cudaFuncSetAttribute(k_reduce_requests<false>,
-                                          cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
-    if (e1 || e2) return e1 ? e1 : e2;
+    const cudaError_t es[4] = {
+        cudaFuncSetAttribute(k_reduce_requests<true, false>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024),
+        cudaFuncSetAttribute(k_reduce_requests<false, false>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024),
+        cudaFuncSetAttribute(k_reduce_requests<true, true>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024),
+        cudaFuncSetAttribute(k_reduce_requests<false, true>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024)};
+    for (cudaError_t e : es)
+      if (e) return e;
     attr = true;
   }
-  if (slo)
-    k_reduce_requests<true><<<ctas, kThreads, smem, s>>>(bt, M, lgMp, win, FastDiv(win), K,
-                                                         near_rows, lgF, P, D, w.dA, w.dW, slo,
-                                                         slo_ms, diag);
+  const FastDiv fd(win);
+  if (slo && copy_records)
+    k_reduce_requests<true, true><<<ctas, kThreads, smem, s>>>(bt, M, lgMp, win, fd, K,
+                                                               near_rows, lgF, P, D, w.dA, w.dW,
+                                                               slo, slo_ms, diag);
+  else if (slo)
+    k_reduce_requests<true, false><<<ctas, kThreads, smem, s>>>(bt, M, lgMp, win, fd, K,
+                                                                near_rows, lgF, P, D, w.dA, w.dW,
+                                                                slo, slo_ms, diag);
+  else if (copy_records)
+    k_reduce_requests<false, true><<<ctas, kThreads, smem, s>>>(bt, M, lgMp, win, fd, K,
+                                                                near_rows, lgF, P, D, w.dA, w.dW,
+                                                                nullptr, nullptr, diag);
   else
-    k_reduce_requests<false><<<ctas, kThreads, smem, s>>>(bt, M, lgMp, win, FastDiv(win), K,
-                                                          near_rows, lgF, P, D, w.dA, w.dW,
-                                                          nullptr, nullptr, diag);
+    k_reduce_requests<false, false><<<ctas, kThreads, smem, s>>>(bt, M, lgMp, win, fd, K,
+                                                                 near_rows, lgF, P, D, w.dA, w.dW,
+                                                                 nullptr, nullptr, diag);
   return cudaGetLastError();
 }
 

@@ -431,3 +431,19 @@ def test_reduce_requests_from_pinned_host_memory(tre):
     got = tre.tss_window_reduce(M, win, K, requests=host)
     for k in "PDAW":
         assert torch.equal(got[k], ref[k]), k
+
+
+def test_reduce_refuses_pageable_host_columns(tre):
+    """Record columns in ordinary (pageable) host memory would fault a kernel
+    reading them: the call refuses them before launching anything."""
+    import ctypes as C
+    import torch
+    cols = {k: torch.zeros(64, dtype=torch.int32) for k in REQ_KEYS}   # not pinned
+    lib = tre.load()
+    g = tre.Grid(4, 100, 10)
+    rq = tre.requests_struct(cols)
+    P, D, A, W = (torch.empty((10, 4), dtype=torch.int32, device="cuda") for _ in range(4))
+    out = tre.Counts(P.data_ptr(), D.data_ptr(), A.data_ptr(), W.data_ptr())
+    size = C.c_size_t(0)
+    st = lib.tss_window_reduce(C.byref(g), C.byref(rq), None, out, None, C.byref(size), None, None)
+    assert st == 1      # TRE_EINVAL
