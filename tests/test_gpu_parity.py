@@ -447,3 +447,72 @@ def test_reduce_refuses_pageable_host_columns(tre):
     size = C.c_size_t(0)
     st = lib.tss_window_reduce(C.byref(g), C.byref(rq), None, out, None, C.byref(size), None, None)
     assert st == 1      # TRE_EINVAL
+
+
+def test_sweep_f64(tre):
+    sw, alpha = _sweep_case(0.02, 2, 600.0)
+    sw["tau_crit"] = sw["tau_crit"][1::3]
+    sw["pacing_cap"] = sw["pacing_cap"][1::3]
+    ref, out = _run_sweep_both(tre, sw, alpha, moves_cap=512, dtype="f64")
+    _compare_sweep(tre, sw, ref, out, 512)
+
+
+def test_sweep_refuses_window_lengths_not_multiples_of_the_shortest(tre):
+    """Every window length must be a multiple of the shortest one (the grid
+    the records are reduced on); 200/300/600 ms is refused."""
+    sw, _ = _sweep_case(0.01, 1, 600.0)
+    sw["window_ms"] = np.array([200, 300, 600], dtype=np.int32)
+    alpha = [min(1.0, w / 5000.0) for w in sw["window_ms"]]
+    with pytest.raises(tre.TreError) as ei:
+        tre.tre_sweep([_cuda(t) for t in sw["traces"]], sw["M"], sw["duration_ms"],
+                      sw["window_ms"], alpha, sw["tau_crit"], sw["pacing_cap"], sw["w_p"],
+                      sw["w_q"], sw["tau_surplus"], sw["slo_ttft_ms"], sw["budget"], sw["r0"],
+                      sw["r_min"], sw["footprint"])
+    assert ei.value.code == 1
+
+
+def test_sweep_more_window_lengths_than_the_fused_pass_takes(tre):
+    """Nine window lengths: the gauge scan and the coarsening run as separate
+    passes."""
+    sw, _ = _sweep_case(0.01, 1, 600.0)
+    sw["window_ms"] = np.array([100, 200, 300, 400, 500, 600, 1000, 1200, 2000], dtype=np.int32)
+    alpha = [min(1.0, w / 5000.0) for w in sw["window_ms"]]
+    sw["tau_crit"] = sw["tau_crit"][::4]
+    sw["pacing_cap"] = sw["pacing_cap"][::4]
+    ref, out = _run_sweep_both(tre, sw, alpha, moves_cap=512)
+    _compare_sweep(tre, sw, ref, out, 512)
+
+
+def test_sweep_heterogeneous_footprints(tre):
+    """Models of different replica footprints: the walk's general transition
+    path (a receiver may need several donor releases)."""
+    sw, alpha = _sweep_case(0.02, 1, 600.0)
+    M = sw["M"]
+    sw["footprint"] = np.array([1, 2, 1, 3, 1, 2, 1, 1][:M], dtype=np.int32)
+    sw["budget"] = int((sw["footprint"] * sw["r0"]).sum()) + 3
+    sw["tau_crit"] = sw["tau_crit"][::2]
+    sw["pacing_cap"] = sw["pacing_cap"][::3]
+    ref, out = _run_sweep_both(tre, sw, alpha, moves_cap=512)
+    _compare_sweep(tre, sw, ref, out, 512)
+
+
+def test_sweep_twelve_models(tre):
+    """More than eight models: the walk's 16-model tables and donor scan."""
+    sw, alpha = _sweep_case(0.02, 1, 600.0)
+    rng = np.random.default_rng(5)
+    M0 = sw["M"]
+    for t in sw["traces"]:
+        t["model"] = np.where(rng.random(len(t["model"])) < 0.35, t["model"] + M0,
+                              t["model"]).astype(np.int32)
+        t["model"] = np.minimum(t["model"], 11).astype(np.int32)
+    M = 12
+    ext = lambda a: np.concatenate([np.asarray(a), np.asarray(a)])[:M]
+    sw["M"] = M
+    for k in ("w_p", "w_q", "tau_surplus", "slo_ttft_ms", "r0", "r_min", "footprint"):
+        if np.ndim(sw[k]):
+            sw[k] = ext(sw[k]).astype(np.asarray(sw[k]).dtype)
+    sw["budget"] = int(sw["r0"].sum()) + 2
+    sw["tau_crit"] = sw["tau_crit"][::3]
+    sw["pacing_cap"] = sw["pacing_cap"][::3]
+    ref, out = _run_sweep_both(tre, sw, alpha, moves_cap=512)
+    _compare_sweep(tre, sw, ref, out, 512)
