@@ -516,3 +516,28 @@ def test_sweep_twelve_models(tre):
     sw["pacing_cap"] = sw["pacing_cap"][::3]
     ref, out = _run_sweep_both(tre, sw, alpha, moves_cap=512)
     _compare_sweep(tre, sw, ref, out, 512)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f64"])
+def test_score_when_burn_ins_cannot_converge(tre, dtype):
+    """Smoothing that the chunk burn-ins cannot settle -- alpha 1e-4 (a capped
+    burn-in far shorter than 28/alpha), per-model alphas, a model idle for a
+    long stretch (burn-ins that see only idle windows) -- is repaired in
+    order to the exact sequential values; the repairs are counted."""
+    rng = np.random.default_rng(77)
+    K, M, win = 40000, 4, 100
+    cnt = _score_inputs(rng, K, M)
+    for k in cnt:
+        cnt[k][20000:30000, 3] = 0                # model 3 idle for a quarter of the series
+    npdt = np.float32 if dtype == "f32" else np.float64
+    prof = {"w_p": rng.uniform(0.1, 0.3, M), "w_q": rng.uniform(1.0, 3.0, M),
+            "alpha": np.array([1e-4, 0.02, 0.5, 0.003]), "theta": rng.uniform(5, 50, M),
+            "tau_crit": np.full(M, 0.8), "tau_surplus": np.full(M, 1.2)}
+    S, Z, cls, recv = oracle.score(cnt["P"], cnt["D"], cnt["A"], cnt["W"], prof, win, npdt)
+    diag = tre.new_diag()
+    out = tre.tss_score(_cuda(cnt), prof, win, dtype=dtype, diag=diag)
+    np.testing.assert_array_equal(_np(out["S"]), S)
+    np.testing.assert_array_equal(_np(out["Z"]), Z)
+    np.testing.assert_array_equal(_np(out["cls"]), cls)
+    np.testing.assert_array_equal(_np(out["recv"]), recv)
+    assert tre.read_diag(diag)["ema_resolved"] > 0
