@@ -151,6 +151,20 @@ def score(P, D, A, W, profile, window_ms, dtype=np.float64, carry=None):
     return S, Z, cls, recv
 
 
+def rank(Z, cls):
+    """Per window the Eq. 3 receiver (-1 if all idle) and its first 8 donors in
+    acquisition order (Sec. IV-B), -1 in unused slots. Returns (recv, order)."""
+    K, M = Z.shape
+    recv = np.zeros(K, np.int32)
+    order = np.zeros((K, 8), np.int32)
+    f = getattr(lib(), "orc_rank_" + _suffix(Z.dtype))
+    rc = f(C.c_int32(M), C.c_int32(K), _p(np.ascontiguousarray(Z)),
+           _p(np.ascontiguousarray(cls, np.uint8)), _p(recv), _p(order))
+    if rc:
+        raise ValueError("oracle: bad arguments")
+    return recv, order
+
+
 def calibrate(S, cls, n_arr, n_met, ok_frac=0.95, reliability=0.95):
     """theta per model (Sec. III-B). Returns (theta[M], n_degenerate)."""
     K, M = S.shape

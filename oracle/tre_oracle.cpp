@@ -368,6 +368,52 @@ struct Walk {
   }
 };
 
+// --------------------------------------------------------------------------
+// Per-window ranking (Eq. 3 receiver, Sec. IV-B acquisition order): the
+// receiver is the non-idle model of smallest Z (lowest index on ties), -1 if
+// every model is idle. Its donors, in the order they would be released: idle
+// models by index, then surplus models by Z descending, then nominal models
+// whose Z is above the receiver's, by Z descending (equal Z: lower index
+// first); never a critical model, never the receiver. The first 8 are
+// written, -1 in the slots left over (all of them without a receiver).
+// Regions come from cls (as scored with the profile's thresholds).
+// --------------------------------------------------------------------------
+template <class T>
+int rank_windows(int32_t M, int32_t K, const T* Z, const uint8_t* cls, int32_t* recv_out,
+                 int32_t* order_out) {
+  if (M < 1 || K < 0) return 1;
+  std::vector<int32_t> surp, nom;
+  for (int64_t k = 0; k < K; ++k) {
+    const T* z = Z + k * M;
+    const uint8_t* c = cls + k * M;
+    int32_t recv = -1;
+    for (int32_t m = 0; m < M; ++m)
+      if (c[m] != kIdle && (recv < 0 || z[m] < z[recv])) recv = m;
+    if (recv_out) recv_out[k] = recv;
+    if (!order_out) continue;
+    int32_t* o = order_out + k * 8;
+    for (int i = 0; i < 8; ++i) o[i] = -1;
+    if (recv < 0) continue;
+    std::vector<int32_t> order;
+    for (int32_t m = 0; m < M; ++m)
+      if (m != recv && c[m] == kIdle) order.push_back(m);
+    surp.clear();
+    nom.clear();
+    for (int32_t m = 0; m < M; ++m) {
+      if (m == recv) continue;
+      if (c[m] == kSurp) surp.push_back(m);
+      else if (c[m] == kNom && z[m] > z[recv]) nom.push_back(m);
+    }
+    auto by_z_desc = [&](int32_t a, int32_t b) { return z[a] > z[b] || (z[a] == z[b] && a < b); };
+    std::sort(surp.begin(), surp.end(), by_z_desc);
+    std::sort(nom.begin(), nom.end(), by_z_desc);
+    order.insert(order.end(), surp.begin(), surp.end());
+    order.insert(order.end(), nom.begin(), nom.end());
+    for (size_t i = 0; i < order.size() && i < 8; ++i) o[i] = order[i];
+  }
+  return 0;
+}
+
 template <class T>
 int select_moves(int32_t M, int32_t win, int32_t K, const T* Z, const uint8_t* cls,
                  const T* tau_crit, const T* tau_surplus, int64_t budget, const int32_t* r_min,
@@ -506,6 +552,15 @@ int orc_slo_counts_events(int32_t M, int32_t win, int32_t K, int64_t n_req,
 
 ORC_TYPED(f32, float)
 ORC_TYPED(f64, double)
+
+int orc_rank_f32(int32_t M, int32_t K, const float* Z, const uint8_t* cls, int32_t* recv,
+                 int32_t* order) {
+  return rank_windows<float>(M, K, Z, cls, recv, order);
+}
+int orc_rank_f64(int32_t M, int32_t K, const double* Z, const uint8_t* cls, int32_t* recv,
+                 int32_t* order) {
+  return rank_windows<double>(M, K, Z, cls, recv, order);
+}
 
 int orc_move_size(void) { return (int)sizeof(Move); }
 
