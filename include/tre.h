@@ -173,6 +173,26 @@ tre_status tss_score(const tre_grid* grid, const tre_counts* in, const tre_profi
                      tre_diag* diag, tre_stream stream);
 
 /*
+ * tss_rank -- per window, the Eq. 3 receiver and the donors it would draw on,
+ * in the order the controller releases them (Sec. IV-B): idle models by index,
+ * then surplus models by Z descending, then nominal models whose Z is above the
+ * receiver's, by Z descending; equal Z puts the lower index first; critical
+ * models and the receiver are never donors. The receiver is argmin Z over
+ * non-idle models, lowest index on ties, -1 if every model is idle (the same
+ * value as tss_score's recv_out). Replica floors, footprints and the idle pool
+ * are not applied here; tre_select_moves applies them on control ticks.
+ * Z (`dtype`) and cls (uint8) are [n_windows][n_models] in device memory, as
+ * tss_score writes them; Z must not be NaN where cls is not TRE_IDLE.
+ * recv_out: int32[n_windows]; donors_out: int32[n_windows][TRE_RANK_DONORS],
+ * the first TRE_RANK_DONORS donors of each window and -1 in the slots left
+ * over (every slot of a window without a receiver). Either may be NULL; Z and
+ * cls are required when one is not. Needs no workspace and touches no diag.
+ */
+#define TRE_RANK_DONORS 8
+tre_status tss_rank(const tre_grid* grid, tre_dtype dtype, const void* Z, const uint8_t* cls,
+                    int32_t* recv_out, int32_t* donors_out, tre_stream stream);
+
+/*
  * tss_calibrate -- healthy boundary theta (Sec. III-B: the lowest smoothed TSS at
  * which the SLO reliability target is still met). Calibration windows have at least
  * one arrival, are not idle and have S > 0. A window is healthy when at least

@@ -116,7 +116,9 @@ def load(build_if_missing: bool = True):
                                      P, P, C.c_int64, P, P, C.POINTER(C.c_size_t), P, P]
     lib.tre_sweep.argtypes = [C.POINTER(SweepSpec), C.POINTER(SweepOut), P,
                               C.POINTER(C.c_size_t), P, P]
-    for f in ("tss_window_reduce", "tss_score", "tss_calibrate", "tre_select_moves", "tre_sweep"):
+    lib.tss_rank.argtypes = [C.POINTER(Grid), C.c_int, P, P, P, P, P]
+    for f in ("tss_window_reduce", "tss_score", "tss_calibrate", "tre_select_moves", "tre_sweep",
+              "tss_rank"):
         getattr(lib, f).restype = C.c_int
     lib.tre_status_str.argtypes = [C.c_int]
     lib.tre_status_str.restype = C.c_char_p
@@ -257,6 +259,26 @@ def tss_score(counts, profile, window_ms, dtype="f32", carry=None, recv=True, di
         _ptr(carry["init"]) if carry else None, _ptr(S), _ptr(Z), _ptr(cls), _ptr(rv), ws, n,
         _ptr(diag), s))
     return {"S": S, "Z": Z, "cls": cls, "recv": rv}
+
+
+RANK_DONORS = 8
+
+
+def tss_rank(Z, cls, window_ms=1000, recv=True, donors=True, stream=None):
+    """Per window the Eq. 3 receiver and its first RANK_DONORS donors in release
+    order (Sec. IV-B). Z, cls: CUDA tensors [K, M]. Returns dict recv [K] int32
+    and donors [K, RANK_DONORS] int32 (-1 in unused slots)."""
+    torch = _torch()
+    lib = load()
+    K, M = Z.shape
+    code, _ = _dt(Z.dtype)
+    g = Grid(M, window_ms, K)
+    rv = torch.empty(K, dtype=torch.int32, device=Z.device) if recv else None
+    dn = torch.empty((K, RANK_DONORS), dtype=torch.int32, device=Z.device) if donors else None
+    Zc, cc = Z.contiguous(), cls.contiguous()
+    _check("tss_rank", lib.tss_rank(C.byref(g), code, _ptr(Zc), _ptr(cc), _ptr(rv), _ptr(dn),
+                                    _stream(stream)))
+    return {"recv": rv, "donors": dn}
 
 
 def tss_calibrate(counts, profile, window_ms, slo_ttft_ms, requests=None, events=None,

@@ -564,6 +564,20 @@ tre_status tss_score(const tre_grid* grid, const tre_counts* in, const tre_profi
                              ws, ws_bytes, diag, s);
 }
 
+tre_status tss_rank(const tre_grid* grid, tre_dtype dtype, const void* Z, const uint8_t* cls,
+                    int32_t* recv_out, int32_t* donors_out, tre_stream stream) {
+  if (!grid_ok(grid) || (dtype != TRE_F32 && dtype != TRE_F64)) return TRE_EINVAL;
+  if (grid->n_windows > 0 && (recv_out || donors_out) && (!Z || !cls)) return TRE_EINVAL;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const int M = grid->n_models, K = grid->n_windows;
+  Scope sc(kReceiver, 1, s);
+  return cuda_status(
+      dtype == TRE_F32
+          ? launch_rank<float>(M, K, static_cast<const float*>(Z), cls, recv_out, donors_out, s)
+          : launch_rank<double>(M, K, static_cast<const double*>(Z), cls, recv_out, donors_out,
+                                s));
+}
+
 tre_status tss_calibrate(const tre_grid* grid, const tre_requests* req, const tre_events* ev,
                          const tre_counts* in, const tre_profile* prof, const int32_t* slo_ttft_ms,
                          double ok_frac, double reliability, void* theta_out, void* ws,

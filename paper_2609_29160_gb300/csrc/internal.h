@@ -140,6 +140,11 @@ template <class T>
 cudaError_t launch_normalize(const SeriesTable<T>& tab, const T* S, const uint8_t* idle_cls,
                              const T* theta, const T* tau_crit, T tau_crit_v, const T* tau_surp,
                              T* Z, uint8_t* cls, cudaStream_t s);
+// donors listed per window by tss_rank
+constexpr int kRankDonors = 8;
+template <class T>
+cudaError_t launch_rank(int M, int K, const T* Z, const uint8_t* cls, int32_t* recv,
+                        int32_t* donors, cudaStream_t s);
 template <class T>
 cudaError_t launch_receiver(int M, int K, const T* Z, const uint8_t* cls, int32_t* recv,
                             cudaStream_t s);

@@ -584,6 +584,72 @@ __global__ void k_receiver(int M, int K, const T* Z, const uint8_t* cls, int32_t
   if (lane == 0) recv[k] = best;
 }
 
+// ---- per-window donor preference order (Sec. IV-B), warp per window ---------
+// Donor key: group (idle 0, surplus 1, nominal above the receiver 2), then Z
+// descending within surplus and nominal, then index. Keys are distinct, so the
+// r-th donor is the smallest key above the (r-1)-th: kRankDonors rounds of a
+// warp-wide minimum, each over the models whose key exceeds the last one.
+template <class T>
+__device__ __forceinline__ bool donor_key_less(int ga, T za, int ia, int gb, T zb, int ib) {
+  if (ga != gb) return ga < gb;
+  if (ga != 0 && za != zb) return za > zb;
+  return ia < ib;
+}
+
+template <class T>
+__global__ void k_rank(int M, int K, const T* Z, const uint8_t* cls, int32_t* recv,
+                       int32_t* donors) {
+  const int64_t k = (int64_t)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
+  if (k >= K) return;
+  const int lane = threadIdx.x & 31;
+  const T* z = Z + (size_t)k * M;
+  const uint8_t* c = cls + (size_t)k * M;
+  int best = -1;
+  T bz = (T)0;
+  for (int m = lane; m < M; m += 32) {
+    if (c[m] == kIdle) continue;
+    const T zm = z[m];
+    if (best < 0 || zm < bz) { best = m; bz = zm; }
+  }
+  for (int o = 16; o > 0; o >>= 1) {
+    const int ob = __shfl_xor_sync(0xffffffffu, best, o);
+    const T oz = __shfl_xor_sync(0xffffffffu, bz, o);
+    if (ob >= 0 && (best < 0 || oz < bz || (oz == bz && ob < best))) { best = ob; bz = oz; }
+  }
+  if (lane == 0 && recv) recv[k] = best;
+  if (!donors) return;
+  int32_t* out = donors + (size_t)k * kRankDonors;
+  int lg = -1, li = -1;
+  T lzv = (T)0;
+  int r = 0;
+  for (; best >= 0 && r < kRankDonors; ++r) {
+    int g = 3, i = -1;
+    T zv = (T)0;
+    for (int m = lane; m < M; m += 32) {
+      if (m == best) continue;
+      const uint8_t cm = c[m];
+      const T zm = z[m];
+      int gm;
+      if (cm == kIdle) gm = 0;
+      else if (cm == kSurp) gm = 1;
+      else if (cm == kNom && zm > bz) gm = 2;
+      else continue;
+      if (lg >= 0 && !donor_key_less(lg, lzv, li, gm, zm, m)) continue;
+      if (i < 0 || donor_key_less(gm, zm, m, g, zv, i)) { g = gm; zv = zm; i = m; }
+    }
+    for (int o = 16; o > 0; o >>= 1) {
+      const int og = __shfl_xor_sync(0xffffffffu, g, o);
+      const int oi = __shfl_xor_sync(0xffffffffu, i, o);
+      const T oz = __shfl_xor_sync(0xffffffffu, zv, o);
+      if (oi >= 0 && (i < 0 || donor_key_less(og, oz, oi, g, zv, i))) { g = og; zv = oz; i = oi; }
+    }
+    if (i < 0) break;
+    if (lane == 0) out[r] = i;
+    lg = g; lzv = zv; li = i;
+  }
+  if (lane >= r && lane < kRankDonors) out[lane] = -1;
+}
+
 template <class T> TilePlan tile_plan(const SeriesTable<T>& t, int& n_tiles) {
   TilePlan tp;
   n_tiles = 0;
@@ -695,6 +761,14 @@ cudaError_t launch_receiver(int M, int K, const T* Z, const uint8_t* cls, int32_
   return cudaGetLastError();
 }
 
+template <class T>
+cudaError_t launch_rank(int M, int K, const T* Z, const uint8_t* cls, int32_t* recv,
+                        int32_t* donors, cudaStream_t s) {
+  if (K == 0 || (!recv && !donors)) return cudaSuccess;
+  k_rank<T><<<(unsigned)((K + 7) / 8), 256, 0, s>>>(M, K, Z, cls, recv, donors);
+  return cudaGetLastError();
+}
+
 #define TRE_INST(T)                                                                               \
   template int series_segments<T>(SeriesTable<T>&);                                               \
   template void score_ws_layout<T>(Arena&, int, int64_t, int, ScoreWs<T>&);                       \
@@ -706,7 +780,9 @@ cudaError_t launch_receiver(int M, int K, const T* Z, const uint8_t* cls, int32_
                                            const T*, const T*, T, const T*, T*, uint8_t*,          \
                                            cudaStream_t);                                          \
   template cudaError_t launch_receiver<T>(int, int, const T*, const uint8_t*, int32_t*,            \
-                                          cudaStream_t);
+                                          cudaStream_t);                                          \
+  template cudaError_t launch_rank<T>(int, int, const T*, const uint8_t*, int32_t*, int32_t*,      \
+                                      cudaStream_t);
 TRE_INST(float)
 TRE_INST(double)
 

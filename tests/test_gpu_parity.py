@@ -259,6 +259,11 @@ def test_pipeline_requests(tre, dtype, name, scale):
     sc = tre.tss_score(c, dict(prof, theta=theta), win, dtype=dtype)
     for k in ("S", "Z", "cls", "recv"):
         np.testing.assert_array_equal(_np(sc[k]), o[k], err_msg=k)
+    rk = tre.tss_rank(sc["Z"], sc["cls"], win)
+    orv, odn = oracle.rank(o["Z"], o["cls"])
+    np.testing.assert_array_equal(_np(rk["recv"]), orv)
+    np.testing.assert_array_equal(_np(rk["recv"]), o["recv"])
+    np.testing.assert_array_equal(_np(rk["donors"]), odn)
     for cap in (1, 3):
         for tc in (0.6, 0.9):
             p2 = dict(prof, theta=theta, tau_crit=np.full(M, tc))
@@ -274,6 +279,41 @@ def test_pipeline_requests(tre, dtype, name, scale):
             ref = np.stack([om[f] for f in ("window", "recv", "donor", "kind", "seq")], 1) \
                 if n else np.zeros((0, 5))
             np.testing.assert_array_equal(got, ref)
+
+
+def _rank_case(rng, K, M, dtype):
+    """Z drawn from a few values (ties on Z), every region, idle runs, and
+    some all-idle windows."""
+    vals = np.array([0.25, 0.5, 0.75, 0.9, 1.0, 1.1, 1.3, 2.0, 3.5], dtype)
+    Z = rng.choice(vals, (K, M))
+    cls = rng.choice(np.array([0, 1, 2, 3], np.uint8), (K, M), p=[0.2, 0.4, 0.25, 0.15])
+    cls[rng.random(K) < 0.03] = 3
+    return np.ascontiguousarray(Z), np.ascontiguousarray(cls)
+
+
+@pytest.mark.parametrize("dtype", [np.float32, np.float64])
+@pytest.mark.parametrize("seed,K,M", [(31, 4099, 8), (32, 1037, 1), (33, 777, 5), (34, 513, 33),
+                                      (35, 129, 100), (36, 17, 1024)])
+def test_rank_matches_oracle(tre, dtype, seed, K, M):
+    rng = np.random.default_rng(seed)
+    Z, cls = _rank_case(rng, K, M, dtype)
+    orv, odn = oracle.rank(Z, cls)
+    g = tre.tss_rank(*_cuda({"Z": Z, "cls": cls}).values())
+    np.testing.assert_array_equal(_np(g["recv"]), orv)
+    np.testing.assert_array_equal(_np(g["donors"]), odn)
+    # either output alone gives the same values
+    only_r = tre.tss_rank(*_cuda({"Z": Z, "cls": cls}).values(), donors=False)
+    only_d = tre.tss_rank(*_cuda({"Z": Z, "cls": cls}).values(), recv=False)
+    assert only_r["donors"] is None and only_d["recv"] is None
+    np.testing.assert_array_equal(_np(only_r["recv"]), orv)
+    np.testing.assert_array_equal(_np(only_d["donors"]), odn)
+
+
+def test_rank_empty_grid(tre):
+    import torch
+    g = tre.tss_rank(torch.zeros((0, 4), dtype=torch.float32, device="cuda"),
+                     torch.zeros((0, 4), dtype=torch.uint8, device="cuda"))
+    assert g["recv"].numel() == 0 and g["donors"].shape == (0, 8)
 
 
 def test_calibrate_events(tre):

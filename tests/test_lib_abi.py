@@ -109,3 +109,16 @@ def test_select_and_sweep_argument_checks():
     wins2 = (C.c_int32 * 2)(500, 1000)
     spec.window_ms = wins2
     assert lib.tre_sweep(C.byref(spec), C.byref(so), None, C.byref(n), None, None) == 0
+
+
+def test_rank_argument_errors_are_reported_on_the_host():
+    lib = tre.load()
+    g = tre.Grid(4, 1000, 10)
+    out = C.c_void_p(16)        # never dereferenced: the checks fail first
+    assert lib.tss_rank(C.byref(g), 2, out, out, out, None, None) == 1    # unknown dtype
+    assert lib.tss_rank(C.byref(g), 0, None, out, out, None, None) == 1   # Z missing
+    assert lib.tss_rank(C.byref(g), 1, out, None, None, out, None) == 1   # cls missing
+    assert lib.tss_rank(None, 0, out, out, out, None, None) == 1
+    g0 = tre.Grid(4, 1000, 0)   # empty grid: nothing to enqueue
+    assert lib.tss_rank(C.byref(g0), 0, None, None, out, out, None) == 0
+
