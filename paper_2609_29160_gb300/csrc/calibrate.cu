@@ -83,6 +83,115 @@ struct PackPlan {
   int tile_base[kMaxSeries + 1];   // prefix of tiles per series
 };
 
+__device__ __forceinline__ uint32_t warp_min(uint32_t v) { return __reduce_min_sync(0xffffffffu, v); }
+__device__ __forceinline__ uint32_t warp_max(uint32_t v) { return __reduce_max_sync(0xffffffffu, v); }
+__device__ __forceinline__ unsigned long long warp_min(unsigned long long v) {
+  for (int o = 16; o > 0; o >>= 1) {
+    const unsigned long long y = __shfl_xor_sync(0xffffffffu, v, o);
+    v = y < v ? y : v;
+  }
+  return v;
+}
+__device__ __forceinline__ unsigned long long warp_max(unsigned long long v) {
+  for (int o = 16; o > 0; o >>= 1) {
+    const unsigned long long y = __shfl_xor_sync(0xffffffffu, v, o);
+    v = y > v ? y : v;
+  }
+  return v;
+}
+
+__device__ __forceinline__ void load4(const float* p, float (&v)[4]) {
+  const float4 q = *reinterpret_cast<const float4*>(p);
+  v[0] = q.x; v[1] = q.y; v[2] = q.z; v[3] = q.w;
+}
+__device__ __forceinline__ void load4(const double* p, double (&v)[4]) {
+  const double2 a = reinterpret_cast<const double2*>(p)[0];
+  const double2 b = reinterpret_cast<const double2*>(p)[1];
+  v[0] = a.x; v[1] = a.y; v[2] = b.x; v[3] = b.y;
+}
+
+// The same packing with 16-byte loads, for model counts that fill whole tile
+// rows (M a multiple of TM and of 4, 16-byte aligned arrays): a thread reads
+// four consecutive models of one window; the candidate range and count of a
+// tile row come from warp reductions over the transposed tile.
+template <class T>
+__global__ void __launch_bounds__(kPackThreads)
+k_pack_vec(const __grid_constant__ SeriesTable<T> tab, const __grid_constant__ PackPlan pp,
+           const T* __restrict__ S, const uint8_t* __restrict__ cls,
+           const unsigned long long* __restrict__ slo, const int32_t* __restrict__ thr,
+           double ok_frac, typename KeyOf<T>::U* __restrict__ keys,
+           typename KeyOf<T>::U* kmin_g, typename KeyOf<T>::U* kmax_g, uint32_t* ncand_g) {
+  using U = typename KeyOf<T>::U;
+  static_assert(kPackTile == 4 * kPackThreads, "four elements per thread");
+  __shared__ U tile[kPackTile + 32];
+  __shared__ U smin[32], smax[32];
+  __shared__ uint32_t scnt[32];
+  const int s = prefix_index(pp.tile_base, tab.n, blockIdx.x);
+  const int M = tab.M, K = tab.K[s];
+  const int t_loc = blockIdx.x - pp.tile_base[s];
+  const int kt = pp.m_tiles == 1 ? t_loc : t_loc / pp.m_tiles;
+  const int k0 = kt * pp.tk, m0 = (t_loc - kt * pp.m_tiles) * pp.tm;
+  const size_t off = (size_t)tab.off[s];
+  const int tid = threadIdx.x;
+  if (tid < 32) {
+    smin[tid] = ~(U)0;
+    smax[tid] = 0;
+    scnt[tid] = 0;
+  }
+  const int TKp = pp.tk + 1;
+  const int e4 = tid * 4;
+  const int kk = e4 >> pp.lg_tm, mm = e4 & (pp.tm - 1);
+  const int k = k0 + kk;
+  U v[4] = {0, 0, 0, 0};
+  if (k < K) {
+    const size_t x = off + (size_t)k * M + m0 + mm;
+    T sv[4];
+    load4(S + x, sv);
+    const uchar4 c4 = *reinterpret_cast<const uchar4*>(cls + x);
+    const ulonglong2 a = reinterpret_cast<const ulonglong2*>(slo + x)[0];
+    const ulonglong2 b = reinterpret_cast<const ulonglong2*>(slo + x)[1];
+    const unsigned long long cv[4] = {a.x, a.y, b.x, b.y};
+    const uint8_t iv[4] = {c4.x, c4.y, c4.z, c4.w};
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const uint32_t n_arr = (uint32_t)cv[u];
+      if (iv[u] != kIdle && n_arr >= 1 && sv[u] > (T)0) {
+        const bool h = healthy(n_arr, (uint32_t)(cv[u] >> 32), thr, ok_frac);
+        v[u] = ((U)key_of(sv[u]) << 1) | (U)(h ? 1 : 0);
+      }
+    }
+  }
+#pragma unroll
+  for (int u = 0; u < 4; ++u) tile[(mm + u) * TKp + kk] = v[u];
+  __syncthreads();
+  // tile rows are models: a warp's 32 consecutive elements share one row
+#pragma unroll
+  for (int j = 0; j < kPackTile / kPackThreads; ++j) {
+    const int e = tid + j * kPackThreads;
+    const int r = e >> pp.lg_tk, kr = e & (pp.tk - 1);
+    const int kg = k0 + kr;
+    const U w = tile[r * TKp + kr];
+    const bool in = kg < K;
+    if (in) keys[off + (size_t)(m0 + r) * K + kg] = w;
+    const bool cand = in && w != 0;
+    const U lo = warp_min(cand ? (U)(w >> 1) : ~(U)0);
+    const U hi = warp_max(cand ? (U)(w >> 1) : (U)0);
+    const uint32_t nc = __popc(__ballot_sync(0xffffffffu, cand));
+    if ((tid & 31) == 0 && nc) {
+      atomicMin(&smin[r], lo);
+      atomicMax(&smax[r], hi);
+      atomicAdd(&scnt[r], nc);
+    }
+  }
+  __syncthreads();
+  if (tid < pp.tm && scnt[tid]) {
+    const size_t g = (size_t)s * M + m0 + tid;
+    atomicMin(&kmin_g[g], smin[tid]);
+    atomicMax(&kmax_g[g], smax[tid]);
+    atomicAdd(&ncand_g[g], scnt[tid]);
+  }
+}
+
 template <class T>
 __global__ void __launch_bounds__(kPackThreads)
 k_pack(const __grid_constant__ SeriesTable<T> tab, const __grid_constant__ PackPlan pp,
@@ -575,7 +684,12 @@ cudaError_t launch_calibrate(const SeriesTable<T>& tab, const T* S, const uint8_
     tiles += (tab.K[i] + pp.tk - 1) / pp.tk * pp.m_tiles;
   }
   pp.tile_base[tab.n] = tiles;
-  if (tiles > 0)
+  const bool vec = tab.M % pp.tm == 0 && tab.M % 4 == 0 &&
+                   (((uintptr_t)S | (uintptr_t)cls | (uintptr_t)slo) & 15) == 0;
+  if (tiles > 0 && vec)
+    k_pack_vec<T><<<tiles, kPackThreads, 0, s>>>(tab, pp, S, cls, slo, w.thr, ok_frac,
+                                                 static_cast<U*>(w.keys), kmin, kmax, w.ncand);
+  else if (tiles > 0)
     k_pack<T><<<tiles, kPackThreads, 0, s>>>(tab, pp, S, cls, slo, w.thr, ok_frac,
                                              static_cast<U*>(w.keys), kmin, kmax, w.ncand);
   const size_t smem = search_smem_bytes<T>();
@@ -583,6 +697,10 @@ cudaError_t launch_calibrate(const SeriesTable<T>& tab, const T* S, const uint8_
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(k_search<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
+    // the largest carveout lets two searches share an SM where their tables fit
+    if (!e)
+      e = cudaFuncSetAttribute(k_search<T>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                               cudaSharedmemCarveoutMaxShared);
     if (e) return e;
     attr_set = true;
   }

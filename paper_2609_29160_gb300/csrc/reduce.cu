@@ -72,13 +72,16 @@ struct Stage {
   int32_t* fAW;       // start side, packed gauge deltas: [M][F + 1]
   int32_t* far_lo;    // [M]
   int32_t* slo_lim;   // [M]
+  int4* queue;        // long decodes of one warp pass: [warps][kQueue][2]
 };
 
-__device__ __forceinline__ uint32_t ceil_div(unsigned long long x, uint32_t d) {
-  unsigned long long q, r;
-  divmod(x, d, q, r);
-  return (uint32_t)(q + (r != 0));
-}
+// Long decodes (beyond the window after the first-token window) are queued per
+// warp pass -- at most one entry per record -- and then walked one record per
+// lane without a division per window: with y the emitted-token bound shifted
+// so that N(T) = floor(y / dur), moving one window boundary adds
+// win*(L-1) = Q*dur + R to y, so a window gets Q or Q + 1 tokens.
+constexpr int kQueue = 32 * kVec;
+
 
 template <bool SLO, bool COPY>
 __global__ void __launch_bounds__(kThreads, 4)
@@ -141,6 +144,9 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win,
   st.fAW = st.fD + (size_t)M * F1;
   st.far_lo = st.fAW + (size_t)M * F1;
   st.slo_lim = st.far_lo + M;
+  st.queue = reinterpret_cast<int4*>((reinterpret_cast<uintptr_t>(st.slo_lim + M) + 15) &
+                                     ~(uintptr_t)15) +
+             (size_t)(threadIdx.x >> 5) * kQueue * 2;
   const int ncell = used * Mp, fcell = M * F1;
   for (int c = threadIdx.x; c < ncell; c += kThreads) {
     st.aW[c] = 0;
@@ -207,6 +213,7 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win,
   // warp-uniform passes: lane l of a pass takes records b + l*kVec + u
   for (int wb = warp * 32 * kVec; wb < n_loc; wb += kThreads * kVec) {
     const int b = wb + lane * kVec;
+    int qn = 0;   // entries in the warp's queue this pass
     int v[7][kVec];
     if (vec4 && b + kVec <= n_loc) {
 #pragma unroll
@@ -236,9 +243,10 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win,
         else if (!(ta <= ts && ts <= tf && tf <= te) || L_in < 0 || L < 1) ++n_order;
         else ok = true;
       }
-      // decode windows after the first-token window that need a division each
+      // decode windows after the first-token window go to the warp's queue
       bool lng = false;
-      int kf = 0, n1 = 0, pairs = 0;
+      int kf = 0, be_q = 0;
+      uint32_t q1 = 0, r1 = 0;
       if (ok) {
         const int lo = st.far_lo[m];
         const int ba = (int)fd.div((uint32_t)ta);
@@ -247,22 +255,23 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win,
         const int be = min(be_raw, K);
         const bool tok = (uint32_t)tf < span;
         kf = tok ? (int)fd.div((uint32_t)tf) : 0;
+        be_q = be_raw;
         // decode tokens of the first-token window (d0) and, for a decode that
         // ends in the next window, of that window (d1); longer decodes leave
-        // their later windows to the warp-spread pass below
+        // their later windows to the queue walk below
         int d0 = L, d1 = 0;
         if (tok && L != 1 && be_raw != kf) {
           // N(T) = tokens emitted before T = ceil((T - tf)(L-1)/dur)
-          n1 = (int)ceil_div((unsigned long long)((uint32_t)(kf + 1) * (uint32_t)win -
-                                                  (uint32_t)tf) * (uint32_t)(L - 1),
-                             (uint32_t)(te - tf));
+          unsigned long long qq, rr;
+          divmod((unsigned long long)((uint32_t)(kf + 1) * (uint32_t)win - (uint32_t)tf) *
+                     (uint32_t)(L - 1),
+                 (uint32_t)(te - tf), qq, rr);
+          q1 = (uint32_t)qq;
+          r1 = (uint32_t)rr;
+          const int n1 = (int)(q1 + (r1 != 0));
           d0 = n1;
-          if (be_raw == kf + 1) {
-            d1 = L - n1;
-          } else {
-            pairs = min(be_raw, K - 1) - kf;   // windows kf+1 .. min(be, K-1)
-            lng = pairs > 0;
-          }
+          if (be_raw == kf + 1) d1 = L - n1;
+          else lng = kf + 1 < K;   // windows kf+1 .. min(be, K-1)
         }
         const int wait = ba != bs ? 1 : 0, run = bs != be ? 1 : 0;
         const uint32_t met = SLO && (tf - ta <= st.slo_lim[m]) ? 1u : 0u;
@@ -299,49 +308,53 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win,
           }
         }
       }
-      // Spread the remaining (record, window) pairs of the warp's long decodes
-      // over the lanes: pair p goes to lane p % 32 of chunk p / 32.
-      if (__any_sync(full, lng)) {
-        const int cnt = lng ? pairs : 0;
-        int incl = cnt;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-          const int y = __shfl_up_sync(full, incl, o);
-          if (lane >= o) incl += y;
+      const unsigned qb = __ballot_sync(full, lng);
+      if (lng) {
+        int4* e = st.queue + 2 * (qn + __popc(qb & ((1u << lane) - 1u)));
+        e[0] = make_int4(tf, te, L, m);
+        e[1] = make_int4(kf, (int)q1, (int)r1, be_q);
+      }
+      qn += __popc(qb);
+    }
+    // walk the pass's long decodes, one record per lane
+    __syncwarp();
+    for (int i = lane; i < qn; i += 32) {
+      const int4 e0 = st.queue[2 * i], e1 = st.queue[2 * i + 1];
+      const int m = e0.w, L = e0.z, kf = e1.x, be_raw = e1.w;
+      const uint32_t dur = (uint32_t)(e0.y - e0.x), q1 = (uint32_t)e1.y, r1 = (uint32_t)e1.z;
+      // y = x + dur - 1 at the end of window kf: N = floor(y / dur), rem = y mod dur
+      uint32_t n = q1 + (r1 != 0);
+      uint32_t rem = r1 ? r1 - 1 : dur - 1;
+      unsigned long long Q64, R64;
+      divmod((unsigned long long)(uint32_t)win * (uint32_t)(L - 1), dur, Q64, R64);
+      const uint32_t Q = (uint32_t)Q64, R = (uint32_t)R64;   // Q < L: dur > win here
+      const int lo = st.far_lo[m];
+      const int k_full = min(be_raw - 1, K - 1);   // windows ending at or before t_end
+      const int k_end = min(be_raw, K - 1);
+      if ((uint32_t)(k_end - lo) < (uint32_t)F) {
+        int32_t* fd_row = st.fD + m * F1 - lo;
+        for (int k = kf + 1; k <= k_full; ++k) {
+          const uint32_t t = rem + R;
+          const uint32_t c = t >= dur ? 1u : 0u;
+          rem = t - (c ? dur : 0u);
+          const uint32_t d = Q + c;
+          n += d;
+          if (d) atomicAdd(&fd_row[k], (int32_t)d);
         }
-        const int total = __shfl_sync(full, incl, 31);
-        int carry = 0;
-        for (int cb = 0; cb < total; cb += 32) {
-          const int p = cb + lane;
-          int o = 0;
-#pragma unroll
-          for (int s = 16; s; s >>= 1) {
-            const int y = __shfl_sync(full, incl, o + s - 1);
-            if (y <= p) o += s;
-          }
-          const int om = __shfl_sync(full, m, o), otf = __shfl_sync(full, tf, o);
-          const int ote = __shfl_sync(full, te, o), oL = __shfl_sync(full, L, o);
-          const int okf = __shfl_sync(full, kf, o), on1 = __shfl_sync(full, n1, o);
-          const int ostart = __shfl_sync(full, incl - cnt, o);
-          const bool act = p < total;
-          const int j = p - ostart;
-          const int k = okf + 1 + j;
-          uint32_t Nend = 0;
-          if (act) {
-            const uint32_t bend = (uint32_t)(k + 1) * (uint32_t)win;
-            Nend = bend > (uint32_t)ote
-                       ? (uint32_t)oL
-                       : ceil_div((unsigned long long)(bend - (uint32_t)otf) * (uint32_t)(oL - 1),
-                                  (uint32_t)(ote - otf));
-          }
-          const uint32_t prev = __shfl_up_sync(full, Nend, 1);
-          const uint32_t Nstart = j == 0 ? (uint32_t)on1 : (lane == 0 ? (uint32_t)carry : prev);
-          if (act && Nend != Nstart)
-            add_tok(st.fD, D, k, om, st.far_lo[om], (int32_t)(Nend - Nstart));
-          carry = (int)__shfl_sync(full, Nend, 31);
+        if (be_raw <= K - 1 && (uint32_t)L != n) atomicAdd(&fd_row[be_raw], (int32_t)(L - n));
+      } else {
+        for (int k = kf + 1; k <= k_full; ++k) {
+          const uint32_t t = rem + R;
+          const uint32_t c = t >= dur ? 1u : 0u;
+          rem = t - (c ? dur : 0u);
+          const uint32_t d = Q + c;
+          n += d;
+          if (d) add_tok(st.fD, D, k, m, lo, (int32_t)d);
         }
+        if (be_raw <= K - 1 && (uint32_t)L != n) add_tok(st.fD, D, be_raw, m, lo, (int32_t)(L - n));
       }
     }
+    __syncwarp();
   }
   __syncthreads();
   for (int c = threadIdx.x; c < ncell; c += kThreads) {
@@ -949,24 +962,28 @@ cudaError_t launch_reduce_requests(const ReqCols* traces, int n_traces, int M, i
   while (lgF < 8 && (size_t)12 * M * ((2 << lgF) + 1) <= 16 * 1024) ++lgF;
   const int F = 1 << lgF;
   const size_t smem_stage = (size_t)near_rows * Mp * (4 + (slo ? 4 : 0)) +
-                            (size_t)12 * M * (F + 1) + (size_t)M * 8;
+                            (size_t)12 * M * (F + 1) + (size_t)M * 8 + 16 +
+                            (size_t)(kThreads / 32) * kQueue * 2 * sizeof(int4);
   // records in host memory are copied into shared memory once per CTA
   const size_t smem_copy = copy_records ? (size_t)per * 7 * 4 : 0;
   const size_t smem = smem_stage + smem_copy;
   if (smem > 200 * 1024) return cudaErrorInvalidValue;
+  // the largest shared-memory carveout, so that four CTAs with their staging
+  // and queues share an SM
   static bool attr = false;
   if (!attr) {
-    const cudaError_t es[4] = {
-        cudaFuncSetAttribute(k_reduce_requests<true, false>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024),
-        cudaFuncSetAttribute(k_reduce_requests<false, false>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024),
-        cudaFuncSetAttribute(k_reduce_requests<true, true>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024),
-        cudaFuncSetAttribute(k_reduce_requests<false, true>,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024)};
-    for (cudaError_t e : es)
+    const void* fns[4] = {(const void*)k_reduce_requests<true, false>,
+                          (const void*)k_reduce_requests<false, false>,
+                          (const void*)k_reduce_requests<true, true>,
+                          (const void*)k_reduce_requests<false, true>};
+    for (const void* f : fns) {
+      cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           200 * 1024);
+      if (!e)
+        e = cudaFuncSetAttribute(f, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                 cudaSharedmemCarveoutMaxShared);
       if (e) return e;
+    }
     attr = true;
   }
   const FastDiv fd(win);

@@ -650,6 +650,61 @@ __global__ void k_rank(int M, int K, const T* Z, const uint8_t* cls, int32_t* re
   if (lane >= r && lane < kRankDonors) out[lane] = -1;
 }
 
+// Up to 16 models: one thread per window, the row in registers. A donor's
+// position is the number of donors with a smaller key; slot j takes the donor
+// whose position is j.
+template <class T, int MMAX>
+__global__ void __launch_bounds__(256)
+k_rank_small(int M, int K, const T* __restrict__ Z, const uint8_t* __restrict__ cls,
+             int32_t* __restrict__ recv, int32_t* __restrict__ donors) {
+  const int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (k >= K) return;
+  const T* z = Z + (size_t)k * M;
+  const uint8_t* c = cls + (size_t)k * M;
+  T zv[MMAX];
+  uint8_t cv[MMAX];
+#pragma unroll
+  for (int m = 0; m < MMAX; ++m) {
+    zv[m] = m < M ? z[m] : (T)0;
+    cv[m] = m < M ? c[m] : kIdle;
+  }
+  int best = -1;
+  T bz = (T)0;
+#pragma unroll
+  for (int m = 0; m < MMAX; ++m)
+    if (m < M && cv[m] != kIdle && (best < 0 || zv[m] < bz)) { best = m; bz = zv[m]; }
+  if (recv) recv[k] = best;
+  if (!donors) return;
+  int32_t* out = donors + (size_t)k * kRankDonors;
+  int g[MMAX];
+#pragma unroll
+  for (int m = 0; m < MMAX; ++m) {
+    int gm = 3;
+    if (m < M && m != best && best >= 0) {
+      if (cv[m] == kIdle) gm = 0;
+      else if (cv[m] == kSurp) gm = 1;
+      else if (cv[m] == kNom && zv[m] > bz) gm = 2;
+    }
+    g[m] = gm;
+  }
+  int pos[MMAX];
+#pragma unroll
+  for (int a = 0; a < MMAX; ++a) {
+    int r = 0;
+#pragma unroll
+    for (int b = 0; b < MMAX; ++b)
+      if (b != a && g[b] < 3 && donor_key_less(g[b], zv[b], b, g[a], zv[a], a)) ++r;
+    pos[a] = g[a] < 3 ? r : kRankDonors;
+  }
+#pragma unroll
+  for (int j = 0; j < kRankDonors; ++j) {
+    int d = -1;
+#pragma unroll
+    for (int a = 0; a < MMAX; ++a) d = pos[a] == j ? a : d;
+    out[j] = d;
+  }
+}
+
 template <class T> TilePlan tile_plan(const SeriesTable<T>& t, int& n_tiles) {
   TilePlan tp;
   n_tiles = 0;
@@ -765,7 +820,13 @@ template <class T>
 cudaError_t launch_rank(int M, int K, const T* Z, const uint8_t* cls, int32_t* recv,
                         int32_t* donors, cudaStream_t s) {
   if (K == 0 || (!recv && !donors)) return cudaSuccess;
-  k_rank<T><<<(unsigned)((K + 7) / 8), 256, 0, s>>>(M, K, Z, cls, recv, donors);
+  const unsigned thread_blocks = (unsigned)((K + 255) / 256);
+  if (M <= 8)
+    k_rank_small<T, 8><<<thread_blocks, 256, 0, s>>>(M, K, Z, cls, recv, donors);
+  else if (M <= 16)
+    k_rank_small<T, 16><<<thread_blocks, 256, 0, s>>>(M, K, Z, cls, recv, donors);
+  else
+    k_rank<T><<<(unsigned)((K + 7) / 8), 256, 0, s>>>(M, K, Z, cls, recv, donors);
   return cudaGetLastError();
 }
 

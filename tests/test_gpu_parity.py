@@ -292,8 +292,9 @@ def _rank_case(rng, K, M, dtype):
 
 
 @pytest.mark.parametrize("dtype", [np.float32, np.float64])
-@pytest.mark.parametrize("seed,K,M", [(31, 4099, 8), (32, 1037, 1), (33, 777, 5), (34, 513, 33),
-                                      (35, 129, 100), (36, 17, 1024)])
+@pytest.mark.parametrize("seed,K,M", [(31, 4099, 8), (32, 1037, 1), (33, 777, 5), (37, 301, 12),
+                                      (38, 2000, 16), (39, 99, 17), (34, 513, 33), (35, 129, 100),
+                                      (36, 17, 1024)])
 def test_rank_matches_oracle(tre, dtype, seed, K, M):
     rng = np.random.default_rng(seed)
     Z, cls = _rank_case(rng, K, M, dtype)
