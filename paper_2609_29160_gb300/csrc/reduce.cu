@@ -72,15 +72,15 @@ struct Stage {
   int32_t* fAW;       // start side, packed gauge deltas: [M][F + 1]
   int32_t* far_lo;    // [M]
   int32_t* slo_lim;   // [M]
-  int4* queue;        // long decodes of one warp pass: [warps][kQueue][2]
+  uint16_t* queue;    // long decodes of this warp: record indices in the CTA
 };
 
 // Long decodes (beyond the window after the first-token window) are queued per
-// warp pass -- at most one entry per record -- and then walked one record per
-// lane without a division per window: with y the emitted-token bound shifted
-// so that N(T) = floor(y / dur), moving one window boundary adds
-// win*(L-1) = Q*dur + R to y, so a window gets Q or Q + 1 tokens.
-constexpr int kQueue = 32 * kVec;
+// warp -- the record's index in the CTA, at most one entry per record -- and,
+// after the warp's last pass, walked one record per lane without a division
+// per window: with y the emitted-token bound shifted so that N(T) =
+// floor(y / dur), moving one window boundary adds win*(L-1) = Q*dur + R to y,
+// so a window gets Q or Q + 1 tokens.
 
 
 template <bool SLO, bool COPY>
@@ -144,9 +144,9 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win,
   st.fAW = st.fD + (size_t)M * F1;
   st.far_lo = st.fAW + (size_t)M * F1;
   st.slo_lim = st.far_lo + M;
-  st.queue = reinterpret_cast<int4*>((reinterpret_cast<uintptr_t>(st.slo_lim + M) + 15) &
-                                     ~(uintptr_t)15) +
-             (size_t)(threadIdx.x >> 5) * kQueue * 2;
+  st.queue = reinterpret_cast<uint16_t*>((reinterpret_cast<uintptr_t>(st.slo_lim + M) + 15) &
+                                         ~(uintptr_t)15) +
+             (size_t)(threadIdx.x >> 5) * (bt.per_cta[t] / (kThreads / 32));
   const int ncell = used * Mp, fcell = M * F1;
   for (int c = threadIdx.x; c < ncell; c += kThreads) {
     st.aW[c] = 0;
@@ -211,15 +211,19 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win,
   const int warp = threadIdx.x >> 5;
   unsigned long long n_range = 0, n_model = 0, n_order = 0;
   // warp-uniform passes: lane l of a pass takes records b + l*kVec + u
+  int qn = 0;   // entries in the warp's queue
   for (int wb = warp * 32 * kVec; wb < n_loc; wb += kThreads * kVec) {
     const int b = wb + lane * kVec;
-    int qn = 0;   // entries in the warp's queue this pass
     int v[7][kVec];
     if (vec4 && b + kVec <= n_loc) {
 #pragma unroll
       for (int c = 0; c < 7; ++c) {
+        // streaming loads, except the four columns the long-decode walk reads
+        // again (model, first-token and end times, output length)
+        const bool again = c == 0 || c == 3 || c == 4 || c == 6;
         const int4 q = COPY ? *reinterpret_cast<const int4*>(colp[c] + b)
-                            : __ldcs(reinterpret_cast<const int4*>(colp[c] + b));
+                       : again ? *reinterpret_cast<const int4*>(colp[c] + b)
+                               : __ldcs(reinterpret_cast<const int4*>(colp[c] + b));
         v[c][0] = q.x; v[c][1] = q.y; v[c][2] = q.z; v[c][3] = q.w;
       }
     } else {
@@ -245,8 +249,7 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win,
       }
       // decode windows after the first-token window go to the warp's queue
       bool lng = false;
-      int kf = 0, be_q = 0;
-      uint32_t q1 = 0, r1 = 0;
+      int kf = 0;
       if (ok) {
         const int lo = st.far_lo[m];
         const int ba = (int)fd.div((uint32_t)ta);
@@ -255,7 +258,6 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win,
         const int be = min(be_raw, K);
         const bool tok = (uint32_t)tf < span;
         kf = tok ? (int)fd.div((uint32_t)tf) : 0;
-        be_q = be_raw;
         // decode tokens of the first-token window (d0) and, for a decode that
         // ends in the next window, of that window (d1); longer decodes leave
         // their later windows to the queue walk below
@@ -266,9 +268,7 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win,
           divmod((unsigned long long)((uint32_t)(kf + 1) * (uint32_t)win - (uint32_t)tf) *
                      (uint32_t)(L - 1),
                  (uint32_t)(te - tf), qq, rr);
-          q1 = (uint32_t)qq;
-          r1 = (uint32_t)rr;
-          const int n1 = (int)(q1 + (r1 != 0));
+          const int n1 = (int)(qq + (rr != 0));
           d0 = n1;
           if (be_raw == kf + 1) d1 = L - n1;
           else lng = kf + 1 < K;   // windows kf+1 .. min(be, K-1)
@@ -309,19 +309,23 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win,
         }
       }
       const unsigned qb = __ballot_sync(full, lng);
-      if (lng) {
-        int4* e = st.queue + 2 * (qn + __popc(qb & ((1u << lane) - 1u)));
-        e[0] = make_int4(tf, te, L, m);
-        e[1] = make_int4(kf, (int)q1, (int)r1, be_q);
-      }
+      if (lng) st.queue[qn + __popc(qb & ((1u << lane) - 1u))] = (uint16_t)(b + u);
       qn += __popc(qb);
     }
-    // walk the pass's long decodes, one record per lane
-    __syncwarp();
-    for (int i = lane; i < qn; i += 32) {
-      const int4 e0 = st.queue[2 * i], e1 = st.queue[2 * i + 1];
-      const int m = e0.w, L = e0.z, kf = e1.x, be_raw = e1.w;
-      const uint32_t dur = (uint32_t)(e0.y - e0.x), q1 = (uint32_t)e1.y, r1 = (uint32_t)e1.z;
+  }
+  // walk the warp's long decodes, one record per lane
+  __syncwarp();
+  for (int i = lane; i < qn; i += 32) {
+    const int j = st.queue[i];
+    const int m = colp[0][j], tf = colp[3][j], te = colp[4][j], L = colp[6][j];
+    const int kf = (int)fd.div((uint32_t)tf), be_raw = (int)fd.div((uint32_t)te);
+    const uint32_t dur = (uint32_t)(te - tf);
+    unsigned long long qq, rr;
+    divmod((unsigned long long)((uint32_t)(kf + 1) * (uint32_t)win - (uint32_t)tf) *
+               (uint32_t)(L - 1),
+           dur, qq, rr);
+    const uint32_t q1 = (uint32_t)qq, r1 = (uint32_t)rr;
+    {
       // y = x + dur - 1 at the end of window kf: N = floor(y / dur), rem = y mod dur
       uint32_t n = q1 + (r1 != 0);
       uint32_t rem = r1 ? r1 - 1 : dur - 1;
@@ -354,7 +358,6 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win,
         if (be_raw <= K - 1 && (uint32_t)L != n) add_tok(st.fD, D, be_raw, m, lo, (int32_t)(L - n));
       }
     }
-    __syncwarp();
   }
   __syncthreads();
   for (int c = threadIdx.x; c < ncell; c += kThreads) {
@@ -963,7 +966,7 @@ cudaError_t launch_reduce_requests(const ReqCols* traces, int n_traces, int M, i
   const int F = 1 << lgF;
   const size_t smem_stage = (size_t)near_rows * Mp * (4 + (slo ? 4 : 0)) +
                             (size_t)12 * M * (F + 1) + (size_t)M * 8 + 16 +
-                            (size_t)(kThreads / 32) * kQueue * 2 * sizeof(int4);
+                            (size_t)per * sizeof(uint16_t);
   // records in host memory are copied into shared memory once per CTA
   const size_t smem_copy = copy_records ? (size_t)per * 7 * 4 : 0;
   const size_t smem = smem_stage + smem_copy;
