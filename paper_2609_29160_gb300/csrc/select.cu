@@ -135,10 +135,22 @@ k_tick_rank(const __grid_constant__ WalkBatch<T> b, int16_t* recv_out, int16_t* 
   }
 }
 
+__device__ __forceinline__ void load_quad(const float* p, float* v) {
+  const float4 q = *reinterpret_cast<const float4*>(p);
+  v[0] = q.x; v[1] = q.y; v[2] = q.z; v[3] = q.w;
+}
+__device__ __forceinline__ void load_quad(const double* p, double* v) {
+  const double2 a = reinterpret_cast<const double2*>(p)[0];
+  const double2 c = reinterpret_cast<const double2*>(p)[1];
+  v[0] = a.x; v[1] = a.y; v[2] = c.x; v[3] = c.y;
+}
+
 // One thread per (series, tau, tick entry) for M <= MMAX: the regions are
 // computed once per model and the ranks in registers; the per-model rank and
-// order tables are written only when the walk that follows reads them.
-template <class T, int MMAX>
+// order tables are written only when the walk that follows reads them. With
+// QUAD (M a multiple of 4, 16-byte aligned rows) a tick window's Z and class
+// rows are read four models per load.
+template <class T, int MMAX, bool QUAD>
 __global__ void __launch_bounds__(128)
 k_tick_rank_small(const __grid_constant__ WalkBatch<T> b, int16_t* recv_out, int16_t* ndon_out,
                   uint16_t* rank, uint16_t* order, unsigned long long* packed, uint32_t* dmask,
@@ -151,27 +163,42 @@ k_tick_rank_small(const __grid_constant__ WalkBatch<T> b, int16_t* recv_out, int
   const int n_ent = b.ent_base[s + 1] - b.ent_base[s];
   const int ti = local / n_ent;
   const int j = local - ti * n_ent;
-  const int64_t win = b.series_win[s];
-  const int64_t K = b.series_K[s];
-  const int64_t nf = K * win / b.fast_ms;
-  const bool fast = j < nf;
-  const int64_t k =
-      fast ? tick_window(j + 1, b.fast_ms, win) : tick_window(j - nf + 1, b.slow_ms, win);
+  // K * win < 2^31, so every tick time below fits 32 unsigned bits
+  const uint32_t win = (uint32_t)b.series_win[s];
+  const uint32_t nf = (uint32_t)b.series_K[s] * win / (uint32_t)b.fast_ms;
+  const bool fast = (uint32_t)j < nf;
+  const uint32_t tj = fast ? ((uint32_t)j + 1) * (uint32_t)b.fast_ms
+                           : ((uint32_t)j - nf + 1) * (uint32_t)b.slow_ms;
+  const uint32_t k = (tj + win - 1) / win - 1;   // window whose right edge passes tj
   const T* Zk = b.Z + b.series_off[s] + (size_t)k * M;
   const uint8_t* Ck = b.cls + b.series_off[s] + (size_t)k * M;
   const bool tau_dev = b.tau_crit != nullptr;
   const T tau_v = b.tau_list[tau_dev ? 0 : ti];
   T z[MMAX];
+  uint8_t cl[MMAX];
+  if (QUAD) {
+#pragma unroll
+    for (int q = 0; q < MMAX; q += 4) {
+      if (q < M) {
+        load_quad(Zk + q, z + q);
+        const uchar4 c4 = *reinterpret_cast<const uchar4*>(Ck + q);
+        cl[q] = c4.x; cl[q + 1] = c4.y; cl[q + 2] = c4.z; cl[q + 3] = c4.w;
+      }
+    }
+  }
   uint8_t rg[MMAX];
   int recv = -1;
   T zr = (T)0;
 #pragma unroll
   for (int q = 0; q < MMAX; ++q) {
-    z[q] = (T)0;
+    if (!QUAD || q >= M) z[q] = (T)0;
     rg[q] = 0xff;
     if (q < M) {
-      z[q] = Zk[q];
-      rg[q] = region_of(Ck[q], z[q], tau_dev ? b.tau_crit[q] : tau_v, b.tau_surp[q]);
+      if (!QUAD) {
+        z[q] = Zk[q];
+        cl[q] = Ck[q];
+      }
+      rg[q] = region_of(cl[q], z[q], tau_dev ? b.tau_crit[q] : tau_v, b.tau_surp[q]);
       const bool cand = fast ? rg[q] == kCrit : rg[q] != kIdle;
       if (cand && (recv < 0 || z[q] < zr)) {
         recv = q;
@@ -1124,15 +1151,22 @@ template <class T> cudaError_t launch_walk(const WalkBatch<T>& b, WalkWs& w, cud
   const bool thread_walk = b.M <= 16 && b.n_cap <= 32 && thread_smem <= kStageMax;
   if (ents > 0) {
     const unsigned g = (unsigned)((ents + 127) / 128);
-    if (b.M <= 8) {
-      k_tick_rank_small<T, 8><<<g, 128, 0, s>>>(b, w.recv, w.n_donor, w.rank, w.order, w.packed,
-                                                w.dmask, !thread_walk);
+    // rows start on 16-byte boundaries when M is a multiple of 4 (series
+    // offsets are multiples of M) and both arrays are 16-byte aligned
+    const bool quad =
+        b.M % 4 == 0 && (((uintptr_t)b.Z | (uintptr_t)b.cls) & 15) == 0;
+    if (b.M <= 8 && quad) {
+      k_tick_rank_small<T, 8, true><<<g, 128, 0, s>>>(b, w.recv, w.n_donor, w.rank, w.order,
+                                                      w.packed, w.dmask, !thread_walk);
+    } else if (b.M <= 8) {
+      k_tick_rank_small<T, 8, false><<<g, 128, 0, s>>>(b, w.recv, w.n_donor, w.rank, w.order,
+                                                       w.packed, w.dmask, !thread_walk);
     } else if (b.M <= 16) {
-      k_tick_rank_small<T, 16><<<g, 128, 0, s>>>(b, w.recv, w.n_donor, w.rank, w.order,
-                                                 w.packed, w.dmask, !thread_walk);
+      k_tick_rank_small<T, 16, false><<<g, 128, 0, s>>>(b, w.recv, w.n_donor, w.rank, w.order,
+                                                        w.packed, w.dmask, !thread_walk);
     } else if (b.M <= 32) {
-      k_tick_rank_small<T, 32><<<g, 128, 0, s>>>(b, w.recv, w.n_donor, w.rank, w.order,
-                                                 w.packed, w.dmask, true);
+      k_tick_rank_small<T, 32, false><<<g, 128, 0, s>>>(b, w.recv, w.n_donor, w.rank, w.order,
+                                                        w.packed, w.dmask, true);
     } else {
       const int64_t th = ents * b.M;
       k_tick_rank<T><<<(unsigned)((th + 255) / 256), 256, 0, s>>>(b, w.recv, w.n_donor, w.rank,
