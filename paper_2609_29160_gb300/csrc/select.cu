@@ -860,7 +860,47 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
       }
       return (int)min(acc & 0xffffu, acc >> 16);
     };
-    if (Kp == 1 && MMAX == 8) {
+    if (Kp == 1 && MMAX == 8 && b.budget <= 255) {
+      // as below, with the replicas above the floor packed one byte per model
+      // in a register (a model never holds more than the budget)
+      unsigned long long cp = 0;
+      for (int m = 0; m < M; ++m) cp |= (unsigned long long)scap[m] << (8 * m);
+      int32_t nm1 = 0;
+      while (true) {
+        const int nxt = next_tick(u);
+        if (nxt >= nf) break;
+        u = nxt + 1;
+        const TickRec tr = srec[nxt];
+        const int32_t k = swin[nxt];
+        const int recv = tr.recv;
+        int donor = -1;
+        if (free_pool > 0) {
+          --free_pool;
+        } else {
+          const uint32_t left = avail & tr.dm;
+          const uint32_t tl = ((left & 0xFu) * 0x00204081u) & 0x01010101u;
+          const uint32_t th = (((left >> 4) & 0xFu) * 0x00204081u) & 0x01010101u;
+          const uint32_t pl = (uint32_t)tr.pk;
+          const int nd = __popc(tr.dm);
+          uint32_t f0 = __byte_perm(tl, th, pl & 0xFFFFu);
+          uint32_t f1 = __byte_perm(tl, th, pl >> 16);
+          if (nd < 4) f0 &= (1u << (8 * nd)) - 1u;
+          if (nd < 8) f1 &= nd <= 4 ? 0u : (1u << (8 * (nd - 4))) - 1u;
+          const int j = f0 ? (__ffs(f0) - 1) >> 3 : 4 + ((__ffs(f1) - 1) >> 3);
+          donor = (int)((pl >> (4 * j)) & 15u);
+          cp -= 1ull << (8 * donor);
+          if (((cp >> (8 * donor)) & 0xFFull) == 0) avail &= ~(1u << donor);
+        }
+        put_move(mv, nm1, cap, k, recv, donor, tr.kind, 0);
+        ++nm1;
+        cp += 1ull << (8 * recv);
+        avail |= 1u << recv;
+      }
+      for (int m = 0; m < M; ++m) scap[m] = (int)((cp >> (8 * m)) & 0xFFull);
+      nm = nm1;
+      u = nf;
+    }
+    if (Kp == 1 && MMAX == 8 && u < nf) {
       // one transition per tick: every tick the jump lands on moves exactly
       // one replica (it has a receiver, and a usable donor when the pool is
       // empty), so the visit is straight-line code

@@ -400,6 +400,34 @@ def test_select_heterogeneous_footprints_and_overflow(tre):
     np.testing.assert_array_equal(_np(rf), orf)
 
 
+@pytest.mark.parametrize("M,r_each,extra", [(8, 20, 3), (8, 40, 5), (5, 60, 0), (7, 1, 1)])
+@pytest.mark.parametrize("cap", [1, 2])
+def test_select_unit_footprints_small_and_large_budgets(tre, M, r_each, extra, cap):
+    # budgets up to 255 keep every model's replicas in one byte; larger ones not
+    import torch
+    rng = np.random.default_rng(M * 100 + r_each)
+    K, win = 4000, 500
+    Z = rng.choice(np.array([0.3, 0.6, 0.85, 0.95, 1.0, 1.1, 1.3, 2.0]), (K, M)).astype(np.float32)
+    cls = np.where(rng.random((K, M)) < 0.1, oracle.IDLE, oracle.NOM).astype(np.uint8)
+    g = np.ones(M, np.int32)
+    r0 = np.full(M, r_each, np.int32)
+    r0[0] = 0
+    budget = int(r0.sum()) + extra
+    r_min = np.where(np.arange(M) % 3 == 1, 1, 0).astype(np.int32)
+    prof = {"w_p": 0.2, "w_q": 2.0, "alpha": 0.2, "theta": 1.0, "tau_crit": 0.8,
+            "tau_surplus": 1.2}
+    om, orf, _ = oracle.select_moves(Z, cls, 0.8, 1.2, win, budget, r0, r_min, g, 5000, 10000, cap)
+    Zc, Cc = torch.as_tensor(Z).cuda(), torch.as_tensor(cls).cuda()
+    mv, rf, n, diag = tre.tre_select_moves(Zc, Cc, prof, win, budget, r0, r_min, g,
+                                           pacing_cap=cap, moves_cap=len(om) + 5)
+    assert n == len(om) and n > 0
+    np.testing.assert_array_equal(_np(rf), orf)
+    got = np.stack([mv[f].astype(np.int32) for f in ("window", "recv", "donor", "kind", "seq")], 1)
+    ref = np.stack([om[f] for f in ("window", "recv", "donor", "kind", "seq")], 1)
+    np.testing.assert_array_equal(got, ref)
+    assert tre.read_diag(diag)["err"] == 0
+
+
 def _sweep_case(scale, n_traces, duration_s):
     sw = tracegen.sweep_workload(scale=scale, n_traces=n_traces, duration_s=duration_s)
     alpha = [min(1.0, w / 5000.0) for w in sw["window_ms"]]
