@@ -79,6 +79,19 @@ def reduce_requests(req, M, window_ms, K):
     return P, D, A, W, drops
 
 
+def occupancy_mean_requests(req, M, window_ms, K):
+    """Per-window request-milliseconds running (A_ms) and waiting (W_ms) inside
+    each window (time-averaged occupancy = these / window_ms). int64 [K, M]."""
+    cols = _req_cols(req)
+    A_ms, W_ms = np.zeros((K, M), np.int64), np.zeros((K, M), np.int64)
+    rc = lib().orc_occupancy_mean_requests(C.c_int32(M), C.c_int32(window_ms), C.c_int32(K),
+                                           C.c_int64(len(cols[0])), *[_p(c) for c in cols],
+                                           _p(A_ms), _p(W_ms))
+    if rc:
+        raise ValueError("oracle: bad arguments")
+    return A_ms, W_ms
+
+
 def slo_counts_requests(req, M, window_ms, K, slo_ttft_ms):
     cols = _req_cols(req)
     n_arr, n_met = np.zeros((K, M), np.int32), np.zeros((K, M), np.int32)
@@ -131,9 +144,11 @@ def _prof(profile, M, dtype):
             for k in ("w_p", "w_q", "alpha", "theta", "tau_crit", "tau_surplus")}
 
 
-def score(P, D, A, W, profile, window_ms, dtype=np.float64, carry=None):
+def score(P, D, A, W, profile, window_ms, dtype=np.float64, carry=None, occ_ms=None):
     """Eq. 1 raw TSS -> EMA -> Eq. 2 Z -> region. Returns (S, Z, cls, recv).
-    carry: optional dict {"S": [M], "init": [M] uint8} updated in place."""
+    carry: optional dict {"S": [M], "init": [M] uint8} updated in place.
+    occ_ms: optional (A_ms, W_ms) int64 -- time-averaged occupancy instead of
+    the sampled A, W."""
     K, M = P.shape
     pr = _prof(profile, M, dtype)
     S = np.zeros((K, M), dtype)
@@ -145,7 +160,10 @@ def score(P, D, A, W, profile, window_ms, dtype=np.float64, carry=None):
            *[_p(_i32(a)) for a in (P, D, A, W)],
            *[_p(pr[k]) for k in ("w_p", "w_q", "alpha", "theta", "tau_crit", "tau_surplus")],
            _p(carry["S"]) if carry else None, _p(carry["init"]) if carry else None,
-           _p(S), _p(Z), _p(cls), _p(recv))
+           _p(S), _p(Z), _p(cls), _p(recv),
+           *((_p(np.ascontiguousarray(occ_ms[0], np.int64)),
+              _p(np.ascontiguousarray(occ_ms[1], np.int64))) if occ_ms is not None
+             else (None, None)))
     if rc:
         raise ValueError("oracle: bad arguments")
     return S, Z, cls, recv

@@ -112,6 +112,40 @@ int reduce_requests(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t*
   return 0;
 }
 
+// Time-averaged occupancy of request records (the window-mean reading of the
+// running and waiting counts in Eq. 1, Sec. III-A; Sec. II-B speaks of an
+// average waiting queue): per (window, model) the request-milliseconds spent
+// running ([t_start, t_end)) and waiting ([t_arr, t_start)) inside the window.
+// The mean count is that sum divided by the window length. Records are taken
+// or skipped by the same rules as reduce_requests (nothing is counted here).
+int occupancy_mean_requests(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* model,
+                            const int32_t* t_arr, const int32_t* t_start,
+                            const int32_t* t_first, const int32_t* t_end, const int32_t* L_in,
+                            const int32_t* L_out, int64_t* A_ms, int64_t* W_ms) {
+  if (M < 1 || win < 1 || K < 0 || n < 0) return 1;
+  const int64_t span = (int64_t)K * win;
+  for (size_t x = 0; x < (size_t)K * M; ++x) A_ms[x] = W_ms[x] = 0;
+  // add the part of [a, e) inside every window it touches
+  auto add_span = [&](int64_t a, int64_t e, int64_t m, int64_t* out) {
+    if (e > span) e = span;
+    if (a >= e) return;
+    for (int64_t k = a / win; k * win < e; ++k) {
+      const int64_t lo = std::max(a, k * win), hi = std::min(e, (k + 1) * win);
+      out[(size_t)k * M + m] += hi - lo;
+    }
+  };
+  for (int64_t i = 0; i < n; ++i) {
+    const int64_t m = model[i];
+    if (m < 0 || m >= M) continue;
+    const int64_t ta = t_arr[i], ts = t_start[i], tf = t_first[i], te = t_end[i];
+    if (ta < 0 || ta >= span) continue;
+    if (!(ta <= ts && ts <= tf && tf <= te) || L_in[i] < 0 || L_out[i] < 1) continue;
+    add_span(ts, te, m, A_ms);
+    add_span(ta, ts, m, W_ms);
+  }
+  return 0;
+}
+
 // Calibration counts of request records: arrivals per (arrival window, model)
 // and how many of them met the TTFT bound of their model's SLO class.
 int slo_counts_requests(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* model,
@@ -206,12 +240,17 @@ int slo_counts_events(int32_t M, int32_t win, int32_t K, int64_t n_req, const in
 // S_carry / init_carry (may be null) hold the smoothing state across calls.
 // recv (may be null): per window, the Eq. 3 receiver argmin Z over non-idle
 // models (lowest index on ties), -1 if every model is idle.
+// A_ms / W_ms (both null or both given): the time-averaged occupancy in place
+// of the sampled A / W -- the mean counts A_ms / win and W_ms / win enter the
+// demand term, and a window is idle when P, D, A_ms and W_ms are all zero.
 // --------------------------------------------------------------------------
 template <class T>
 int score(int32_t M, int32_t win, int32_t K, const int32_t* P, const int32_t* D,
           const int32_t* A, const int32_t* W, const T* w_p, const T* w_q, const T* alpha,
           const T* theta, const T* tau_crit, const T* tau_surplus, T* S_carry,
-          uint8_t* init_carry, T* S_out, T* Z_out, uint8_t* cls_out, int32_t* recv) {
+          uint8_t* init_carry, T* S_out, T* Z_out, uint8_t* cls_out, int32_t* recv,
+          const int64_t* A_ms, const int64_t* W_ms) {
+  if ((A_ms == nullptr) != (W_ms == nullptr)) return 1;
   if (M < 1 || win < 1 || K < 0) return 1;
   const T dt = (T)win / (T)1000;                     // window length in seconds
   for (int64_t m = 0; m < M; ++m) {
@@ -222,14 +261,18 @@ int score(int32_t M, int32_t win, int32_t K, const int32_t* P, const int32_t* D,
     const T b = (T)1 - a;
     for (int64_t k = 0; k < K; ++k) {
       const size_t x = (size_t)k * M + m;
-      const bool idle = P[x] == 0 && D[x] == 0 && A[x] == 0 && W[x] == 0;
+      const bool idle = A_ms ? P[x] == 0 && D[x] == 0 && A_ms[x] == 0 && W_ms[x] == 0
+                             : P[x] == 0 && D[x] == 0 && A[x] == 0 && W[x] == 0;
       if (!idle) {
         const T r_pre = (T)P[x] / dt;                  // prefill token rate
         const T r_dec = (T)D[x] / dt;                  // decode token rate
         const T svc = w_p[m] * r_pre;
         const T num = svc + r_dec;
-        const T qw = w_q[m] * (T)W[x];
-        T den = (T)A[x] + qw;
+        // running and waiting counts: sampled, or window means
+        const T a_cnt = A_ms ? (T)A_ms[x] / (T)win : (T)A[x];
+        const T w_cnt = A_ms ? (T)W_ms[x] / (T)win : (T)W[x];
+        const T qw = w_q[m] * w_cnt;
+        T den = a_cnt + qw;
         if (den < (T)1) den = (T)1;                    // demand floor of one request
         const T raw = num / den;
         if (!init) {
@@ -504,6 +547,15 @@ int orc_reduce_requests(int32_t M, int32_t win, int32_t K, int64_t n, const int3
                          A, W, drops);
 }
 
+int orc_occupancy_mean_requests(int32_t M, int32_t win, int32_t K, int64_t n,
+                                const int32_t* model, const int32_t* t_arr,
+                                const int32_t* t_start, const int32_t* t_first,
+                                const int32_t* t_end, const int32_t* L_in, const int32_t* L_out,
+                                int64_t* A_ms, int64_t* W_ms) {
+  return occupancy_mean_requests(M, win, K, n, model, t_arr, t_start, t_first, t_end, L_in, L_out,
+                                 A_ms, W_ms);
+}
+
 int orc_slo_counts_requests(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* model,
                             const int32_t* t_arr, const int32_t* t_start, const int32_t* t_first,
                             const int32_t* t_end, const int32_t* L_in, const int32_t* L_out,
@@ -531,9 +583,10 @@ int orc_slo_counts_events(int32_t M, int32_t win, int32_t K, int64_t n_req,
   int orc_score_##SUF(int32_t M, int32_t win, int32_t K, const int32_t* P, const int32_t* D,      \
                       const int32_t* A, const int32_t* W, const T* w_p, const T* w_q,             \
                       const T* alpha, const T* theta, const T* tau_crit, const T* tau_surplus,    \
-                      T* S_carry, uint8_t* init_carry, T* S, T* Z, uint8_t* cls, int32_t* recv) { \
+                      T* S_carry, uint8_t* init_carry, T* S, T* Z, uint8_t* cls, int32_t* recv,   \
+                      const int64_t* A_ms, const int64_t* W_ms) {                                  \
     return score<T>(M, win, K, P, D, A, W, w_p, w_q, alpha, theta, tau_crit, tau_surplus,         \
-                    S_carry, init_carry, S, Z, cls, recv);                                         \
+                    S_carry, init_carry, S, Z, cls, recv, A_ms, W_ms);                             \
   }                                                                                                \
   int orc_calibrate_##SUF(int32_t M, int32_t K, const T* S, const uint8_t* cls,                   \
                           const int32_t* n_arr, const int32_t* n_met, double ok_frac,             \
