@@ -103,9 +103,19 @@ typedef struct {
 
 /* Per-window counts (device, int32, [n_windows][n_models] each):
  * P prompt tokens, D decode tokens, A running and W waiting requests read at
- * the last millisecond of the window. Counts wrap modulo 2^32. */
+ * the last millisecond of the window. Counts wrap modulo 2^32.
+ * A_ms, W_ms (device, int64, [n_windows][n_models]; both NULL or both set):
+ * the time-averaged occupancy -- request-milliseconds spent running
+ * ([t_start, t_end)) and waiting ([t_arr, t_start)) inside the window, so that
+ * A_ms / window_ms is the window's mean running count (Sec. III-A defines the
+ * counts at a time t; Sec. II-B speaks of an average waiting queue).
+ * tss_window_reduce fills them from request records when they are set (token
+ * events: TRE_EINVAL); tss_score, tss_score_noalloc and tss_calibrate then use
+ * the means A_ms / window_ms and W_ms / window_ms in Eq. 1's demand term in
+ * place of A and W, and a window is IDLE when P, D, A_ms and W_ms are zero. */
 typedef struct {
   int32_t *P, *D, *A, *W;
+  int64_t *A_ms, *W_ms;
 } tre_counts;
 
 /* Control profile (Sec. III-B, Sec. V-B): six scalars per model, device arrays

@@ -225,17 +225,22 @@ def select_moves(Z, cls, tau_crit, tau_surplus, window_ms, budget, r0, r_min, fo
 
 
 def pipeline_requests(req, M, window_ms, K, profile, slo_ttft_ms, dtype, ok_frac=0.95,
-                      reliability=0.95):
-    """Reduce -> score (S) -> calibrate theta -> score (Z, class, receiver)."""
+                      reliability=0.95, mean_occupancy=False):
+    """Reduce -> score (S) -> calibrate theta -> score (Z, class, receiver).
+    mean_occupancy: Eq. 1's running and waiting counts as window means."""
     P, D, A, W, drops = reduce_requests(req, M, window_ms, K)
+    occ = occupancy_mean_requests(req, M, window_ms, K) if mean_occupancy else None
     n_arr, n_met = slo_counts_requests(req, M, window_ms, K, slo_ttft_ms)
-    S, _, cls, _ = score(P, D, A, W, profile, window_ms, dtype)
+    S, _, cls, _ = score(P, D, A, W, profile, window_ms, dtype, occ_ms=occ)
     theta, deg = calibrate(S, cls, n_arr, n_met, ok_frac, reliability)
     prof = dict(profile)
     prof["theta"] = theta
-    S, Z, cls, recv = score(P, D, A, W, prof, window_ms, dtype)
-    return {"P": P, "D": D, "A": A, "W": W, "drops": drops, "n_arr": n_arr, "n_met": n_met,
-            "S": S, "Z": Z, "cls": cls, "recv": recv, "theta": theta, "degenerate": deg}
+    S, Z, cls, recv = score(P, D, A, W, prof, window_ms, dtype, occ_ms=occ)
+    out = {"P": P, "D": D, "A": A, "W": W, "drops": drops, "n_arr": n_arr, "n_met": n_met,
+           "S": S, "Z": Z, "cls": cls, "recv": recv, "theta": theta, "degenerate": deg}
+    if occ is not None:
+        out["A_ms"], out["W_ms"] = occ
+    return out
 
 
 def sweep(traces, M, duration_ms, window_ms_list, tau_crit_list, pacing_list, w_p, w_q,

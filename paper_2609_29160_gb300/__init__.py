@@ -45,7 +45,7 @@ class Events(C.Structure):
 
 
 class Counts(C.Structure):
-    _fields_ = [(k, C.c_void_p) for k in ("P", "D", "A", "W")]
+    _fields_ = [(k, C.c_void_p) for k in ("P", "D", "A", "W", "A_ms", "W_ms")]
 
 
 class Profile(C.Structure):
@@ -197,7 +197,8 @@ def events_struct(ev):
 
 
 def _counts(c):
-    return Counts(*[c[k].data_ptr() for k in ("P", "D", "A", "W")])
+    occ = [c[k].data_ptr() if c.get(k) is not None else None for k in ("A_ms", "W_ms")]
+    return Counts(*[c[k].data_ptr() for k in ("P", "D", "A", "W")], *occ)
 
 
 def _profile(prof, M, tdt, code):
@@ -219,14 +220,19 @@ def _profile(prof, M, tdt, code):
 # entry points
 # ---------------------------------------------------------------------------
 def tss_window_reduce(M, window_ms, K, requests=None, events=None, diag=None, stream=None,
-                      out=None):
+                      out=None, mean_occupancy=False):
     """Per-window P, D, A, W ([K][M] int32 CUDA tensors) from request records or
-    token events (dicts of CUDA tensors)."""
+    token events (dicts of CUDA tensors). With mean_occupancy (request records
+    only) also A_ms, W_ms: int64 request-milliseconds running / waiting per
+    window; a dict holding them makes tss_score use the window means."""
     torch = _torch()
     lib = load()
     g = Grid(M, window_ms, K)
     if out is None:
         out = {k: torch.empty((K, M), dtype=torch.int32, device="cuda") for k in "PDAW"}
+        if mean_occupancy:
+            for k in ("A_ms", "W_ms"):
+                out[k] = torch.empty((K, M), dtype=torch.int64, device="cuda")
     diag = new_diag() if diag is None else diag
     rq = requests_struct(requests) if requests is not None else None
     ev = events_struct(events) if events is not None else None

@@ -48,7 +48,9 @@ bool ev_ok(const tre_events* e) {
   return true;
 }
 
-bool counts_ok(const tre_counts* c) { return c && c->P && c->D && c->A && c->W; }
+bool counts_ok(const tre_counts* c) {
+  return c && c->P && c->D && c->A && c->W && (!c->A_ms) == (!c->W_ms);
+}
 
 bool prof_ok(const tre_profile* p, bool need_theta_tau) {
   if (!p || (p->dtype != TRE_F32 && p->dtype != TRE_F64)) return false;
@@ -165,7 +167,7 @@ tre_status score_typed(const tre_grid* g, const tre_counts* in, const tre_profil
                         static_cast<const T*>(p->theta), static_cast<const T*>(p->tau_crit),
                         static_cast<const T*>(p->tau_surplus), static_cast<T*>(S_carry),
                         init_carry, static_cast<T*>(S_out), static_cast<T*>(Z_out), cls_out, w,
-                        diag, s);
+                        diag, s, in->A_ms, in->W_ms);
   }
   if (!e && recv_out) {
     Scope sc(kReceiver, 1, s);
@@ -203,7 +205,8 @@ tre_status calibrate_typed(const tre_grid* g, const tre_requests* req, const tre
     Scope sc(kScore, 6, s);
     e = launch_score<T>(tab, in->P, in->D, in->A, in->W, static_cast<const T*>(p->w_p),
                         static_cast<const T*>(p->w_q), static_cast<const T*>(p->alpha), nullptr,
-                        nullptr, nullptr, nullptr, nullptr, S, nullptr, cls, sw, diag, s);
+                        nullptr, nullptr, nullptr, nullptr, S, nullptr, cls, sw, diag, s,
+                        in->A_ms, in->W_ms);
   }
   if (!e) {
     Scope sc(kCalibrate, 3, s);
@@ -525,6 +528,7 @@ tre_status tss_window_reduce(const tre_grid* grid, const tre_requests* req, cons
   if (!grid_ok(grid) || !ws_bytes || (!req) == (!ev)) return TRE_EINVAL;
   if (req ? !req_ok(req) : !ev_ok(ev)) return TRE_EINVAL;
   if (!counts_ok(&out)) return TRE_EINVAL;
+  if (out.A_ms && !req) return TRE_EINVAL;   // time-averaged occupancy: request records only
   if (ws && !diag) return TRE_EINVAL;
   const int M = grid->n_models, K = grid->n_windows;
   Arena a(ws);
@@ -545,6 +549,10 @@ tre_status tss_window_reduce(const tre_grid* grid, const tre_requests* req, cons
   if (!e) {
     Scope sc(kScan, 3, s);
     e = launch_gauge_scan(M, K, w, out.A, out.W, s);
+  }
+  if (!e && out.A_ms) {
+    Scope sc(kScan, 4, s);
+    e = launch_occupancy_mean(cols_of(req), M, grid->window_ms, K, w, out.A_ms, out.W_ms, s);
   }
   return cuda_status(e);
 }

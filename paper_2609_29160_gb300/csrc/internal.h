@@ -67,6 +67,11 @@ cudaError_t launch_slo_events(const EvCols& e, int M, int win, int K, unsigned l
                               const int32_t* slo_ms, cudaStream_t s);
 // inclusive scan of the diff arrays over windows -> A, W (trace t at t*K*M)
 cudaError_t launch_gauge_scan(int M, int K, ReduceWs& w, int32_t* A, int32_t* W, cudaStream_t s);
+// Time-averaged occupancy of one trace's request records: request-milliseconds
+// running and waiting per (window, model), int64 [K][M]; reuses the gauge
+// diff and partial arrays of w (call after the gauge scan of the same trace)
+cudaError_t launch_occupancy_mean(const ReqCols& r, int M, int win, int K, ReduceWs& w,
+                                  int64_t* A_ms, int64_t* W_ms, cudaStream_t s);
 // exact coarsening of every trace's base grid to every window length: counts
 // add over q base windows, gauges are read at the last base window
 struct AggPlan {
@@ -133,7 +138,8 @@ cudaError_t launch_score(const SeriesTable<T>& tab, const int32_t* P, const int3
                          const int32_t* A, const int32_t* W, const T* w_p, const T* w_q,
                          const T* alpha, const T* theta, const T* tau_crit, const T* tau_surp,
                          T* S_carry, uint8_t* init_carry, T* S, T* Z, uint8_t* cls,
-                         ScoreWs<T>& w, tre_diag* diag, cudaStream_t s);
+                         ScoreWs<T>& w, tre_diag* diag, cudaStream_t s,
+                         const int64_t* A_ms = nullptr, const int64_t* W_ms = nullptr);
 // Z = S / theta[series][m] and regions for every series (tau_crit device [M] or
 // one value for all)
 template <class T>

@@ -72,7 +72,7 @@ tre_status run(const tre_grid* g, const tre_counts* in, const tre_profile* p, vo
       static_cast<const T*>(p->w_q), static_cast<const T*>(p->alpha),
       static_cast<const T*>(p->theta), static_cast<const T*>(p->tau_crit),
       static_cast<const T*>(p->tau_surplus), static_cast<T*>(S_carry), init_carry,
-      static_cast<T*>(S_out), static_cast<T*>(Z_out), cls_out, w, diag, s);
+      static_cast<T*>(S_out), static_cast<T*>(Z_out), cls_out, w, diag, s, in->A_ms, in->W_ms);
   if (!e && recv_out)
     e = launch_receiver<T>(M, K, static_cast<const T*>(Z_out), cls_out, recv_out, s);
   return e == cudaSuccess ? TRE_OK : TRE_ECUDA;

@@ -1066,6 +1066,96 @@ cudaError_t launch_gauge_scan(int M, int K, ReduceWs& w, int32_t* A, int32_t* W,
   return cudaGetLastError();
 }
 
+// Time-averaged occupancy (the window-mean reading of Eq. 1's running and
+// waiting counts, Sec. III-A): the request-milliseconds that running
+// ([t_start, t_end)) and waiting ([t_arr, t_start)) requests spend inside each
+// window. A span adds its partial first and last windows directly (64-bit
+// atomics into the output) and marks the windows it covers completely in a
+// +1/-1 difference array; the prefix of that array times the window length is
+// added afterwards. Records are taken or skipped by the reduction's rules.
+__device__ __forceinline__ void occ_span(uint32_t a, uint32_t e, uint32_t span, int m, int M,
+                                         uint32_t win, const FastDiv& fd,
+                                         unsigned long long* __restrict__ part,
+                                         int32_t* __restrict__ full) {
+  if (e > span) e = span;
+  if (a >= e) return;
+  const uint32_t ka = fd.div(a), ke = fd.div(e - 1);
+  if (ka == ke) {
+    atomicAdd(&part[(size_t)ka * M + m], (unsigned long long)(e - a));
+    return;
+  }
+  atomicAdd(&part[(size_t)ka * M + m], (unsigned long long)((ka + 1) * win - a));
+  atomicAdd(&part[(size_t)ke * M + m], (unsigned long long)(e - ke * win));
+  if (ke > ka + 1) {
+    atomicAdd(&full[(size_t)(ka + 1) * M + m], 1);
+    atomicAdd(&full[(size_t)ke * M + m], -1);
+  }
+}
+
+__global__ void __launch_bounds__(kThreads)
+k_occ_spans(ReqCols r, int M, int win, FastDiv fd, int K, unsigned long long* __restrict__ pA,
+            unsigned long long* __restrict__ pW, int32_t* __restrict__ fA,
+            int32_t* __restrict__ fW) {
+  const uint32_t span = (uint32_t)K * (uint32_t)win;
+  for (int64_t i = (int64_t)blockIdx.x * kThreads + threadIdx.x; i < r.n;
+       i += (int64_t)gridDim.x * kThreads) {
+    const int m = r.model[i];
+    if (m < 0 || m >= M) continue;
+    const int ta = r.t_arr[i], ts = r.t_start[i], tf = r.t_first[i], te = r.t_end[i];
+    if (ta < 0 || (uint32_t)ta >= span) continue;
+    if (!(ta <= ts && ts <= tf && tf <= te) || r.L_in[i] < 0 || r.L_out[i] < 1) continue;
+    occ_span((uint32_t)ts, (uint32_t)te, span, m, M, (uint32_t)win, fd, pA, fA);
+    occ_span((uint32_t)ta, (uint32_t)ts, span, m, M, (uint32_t)win, fd, pW, fW);
+  }
+}
+
+// adds the full-window counts (chunk prefixes from the gauge scan's first
+// two passes) times the window length to the partial sums
+__global__ void __launch_bounds__(kThreads)
+k_occ_apply(int M, int K, int L, int n_chunks, int win, const int32_t* __restrict__ fA,
+            const int32_t* __restrict__ fW, const int32_t* __restrict__ pA,
+            const int32_t* __restrict__ pW, long long* __restrict__ A_ms,
+            long long* __restrict__ W_ms) {
+  const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+  if (t >= (int64_t)n_chunks * M) return;
+  const int m = (int)(t % M);
+  const int c = (int)(t / M);
+  const int64_t r0 = (int64_t)c * L, r1 = min64(r0 + L, K);
+  int32_t a = pA[t], w = pW[t];
+  for (int64_t k = r0; k < r1; ++k) {
+    a += fA[k * M + m];
+    w += fW[k * M + m];
+    A_ms[k * M + m] += (long long)a * win;
+    W_ms[k * M + m] += (long long)w * win;
+  }
+}
+
+cudaError_t launch_occupancy_mean(const ReqCols& r, int M, int win, int K, ReduceWs& w,
+                                  int64_t* A_ms, int64_t* W_ms, cudaStream_t s) {
+  if (K == 0) return cudaSuccess;
+  const size_t cells = (size_t)K * M, cells1 = (size_t)(K + 1) * M;
+  cudaError_t e = cudaMemsetAsync(A_ms, 0, cells * sizeof(int64_t), s);
+  if (!e) e = cudaMemsetAsync(W_ms, 0, cells * sizeof(int64_t), s);
+  if (!e) e = cudaMemsetAsync(w.dA, 0, cells1 * sizeof(int32_t), s);
+  if (!e) e = cudaMemsetAsync(w.dW, 0, cells1 * sizeof(int32_t), s);
+  if (e) return e;
+  if (r.n > 0)
+    k_occ_spans<<<grid_for(r.n, 4), kThreads, 0, s>>>(
+        r, M, win, FastDiv(win), K, reinterpret_cast<unsigned long long*>(A_ms),
+        reinterpret_cast<unsigned long long*>(W_ms), w.dA, w.dW);
+  const int L = scan_chunk_rows(K);
+  const int n_chunks = (K + L - 1) / L;
+  const int64_t segs = (int64_t)n_chunks * M;
+  const unsigned g = (unsigned)((segs + kThreads - 1) / kThreads);
+  k_scan_partials<<<dim3(g, 1), kThreads, 0, s>>>(M, K, L, n_chunks, w.dA, w.dW, w.partA,
+                                                  w.partW);
+  k_scan_chunks<<<dim3((M + 3) / 4, 1), 128, 0, s>>>(M, n_chunks, w.partA, w.partW);
+  k_occ_apply<<<g, kThreads, 0, s>>>(M, K, L, n_chunks, win, w.dA, w.dW, w.partA, w.partW,
+                                     reinterpret_cast<long long*>(A_ms),
+                                     reinterpret_cast<long long*>(W_ms));
+  return cudaGetLastError();
+}
+
 cudaError_t launch_gauge_prefix(const GaugePlan& gp, ReduceWs& w, cudaStream_t s) {
   if (gp.n_traces > w.n_traces || (int64_t)gp.nblk * gp.M > w.part_cap) return cudaErrorInvalidValue;
   const int64_t n = (int64_t)gp.n_traces * gp.nblk * gp.M;

@@ -44,7 +44,14 @@ __device__ __forceinline__ bool same_bits(double a, double b) {
 
 struct Counts {
   const int32_t *P, *D, *A, *W;
+  const int64_t *A_ms, *W_ms;   // time-averaged occupancy (request-ms per window) or null
 };
+
+template <class T> __device__ __forceinline__ T from_i64(long long v);
+template <> __device__ __forceinline__ float from_i64<float>(long long v) { return __ll2float_rn(v); }
+template <> __device__ __forceinline__ double from_i64<double>(long long v) {
+  return __ll2double_rn(v);
+}
 
 // series of a global segment index (the table has at most 64 entries)
 template <class T> __device__ __forceinline__ int series_of_seg(const SeriesTable<T>& t, int seg) {
@@ -101,7 +108,22 @@ __device__ __forceinline__ T raw_tss(int32_t p, int32_t d, int32_t a, int32_t w,
   return div_rn(num, den);
 }
 
+// Eq. 1 with the window means of the running and waiting counts: the
+// request-milliseconds inside the window divided by its length
 template <class T>
+__device__ __forceinline__ T raw_tss_mean(int32_t p, int32_t d, long long a_ms, long long w_ms,
+                                          T dt, T win, T wp, T wq) {
+  const T r_pre = div_rn(from_i32<T>(p), dt);
+  const T r_dec = div_rn(from_i32<T>(d), dt);
+  const T num = add_rn(mul_rn(wp, r_pre), r_dec);
+  const T a = div_rn(from_i64<T>(a_ms), win);
+  const T w = div_rn(from_i64<T>(w_ms), win);
+  T den = add_rn(a, mul_rn(wq, w));
+  if (den < (T)1) den = (T)1;                       // demand floor of one request
+  return div_rn(num, den);
+}
+
+template <class T, bool MEAN>
 __global__ void __launch_bounds__(kEwThreads)
 k_raw(const __grid_constant__ SeriesTable<T> tab, const __grid_constant__ TilePlan tp, FastDiv fm,
       bool vec, Counts c, const T* __restrict__ w_p, const T* __restrict__ w_q,
@@ -114,24 +136,40 @@ k_raw(const __grid_constant__ SeriesTable<T> tab, const __grid_constant__ TilePl
   const size_t x0 = (size_t)(tab.off[s] + l0);
   const T dt = div_rn((T)tab.win[s], (T)1000);      // window length in seconds
   int32_t p[4], d[4], a[4], w[4];
+  long long am[4], wm[4];
   const bool v4 = vec && l0 + 4 <= n;
   if (v4) {
     const int4 P4 = *reinterpret_cast<const int4*>(c.P + x0);
     const int4 D4 = *reinterpret_cast<const int4*>(c.D + x0);
-    const int4 A4 = *reinterpret_cast<const int4*>(c.A + x0);
-    const int4 W4 = *reinterpret_cast<const int4*>(c.W + x0);
     p[0] = P4.x; p[1] = P4.y; p[2] = P4.z; p[3] = P4.w;
     d[0] = D4.x; d[1] = D4.y; d[2] = D4.z; d[3] = D4.w;
-    a[0] = A4.x; a[1] = A4.y; a[2] = A4.z; a[3] = A4.w;
-    w[0] = W4.x; w[1] = W4.y; w[2] = W4.z; w[3] = W4.w;
+    if (MEAN) {
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const longlong2 A2 = reinterpret_cast<const longlong2*>(c.A_ms + x0)[h];
+        const longlong2 W2 = reinterpret_cast<const longlong2*>(c.W_ms + x0)[h];
+        am[2 * h] = A2.x; am[2 * h + 1] = A2.y;
+        wm[2 * h] = W2.x; wm[2 * h + 1] = W2.y;
+      }
+    } else {
+      const int4 A4 = *reinterpret_cast<const int4*>(c.A + x0);
+      const int4 W4 = *reinterpret_cast<const int4*>(c.W + x0);
+      a[0] = A4.x; a[1] = A4.y; a[2] = A4.z; a[3] = A4.w;
+      w[0] = W4.x; w[1] = W4.y; w[2] = W4.z; w[3] = W4.w;
+    }
   } else {
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       const bool in = l0 + i < n;
       p[i] = in ? c.P[x0 + i] : 0;
       d[i] = in ? c.D[x0 + i] : 0;
-      a[i] = in ? c.A[x0 + i] : 0;
-      w[i] = in ? c.W[x0 + i] : 0;
+      if (MEAN) {
+        am[i] = in ? c.A_ms[x0 + i] : 0;
+        wm[i] = in ? c.W_ms[x0 + i] : 0;
+      } else {
+        a[i] = in ? c.A[x0 + i] : 0;
+        w[i] = in ? c.W[x0 + i] : 0;
+      }
     }
   }
   int m = l0 <= 0xffffffffll ? (int)((uint32_t)l0 - fm.div((uint32_t)l0) * (uint32_t)M)
@@ -140,8 +178,15 @@ k_raw(const __grid_constant__ SeriesTable<T> tab, const __grid_constant__ TilePl
   uint8_t cv[4];
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
-    const bool idle = (p[i] | d[i] | a[i] | w[i]) == 0;
-    rv[i] = idle ? idle_raw((T)0) : raw_tss<T>(p[i], d[i], a[i], w[i], dt, w_p[m], w_q[m]);
+    bool idle;
+    if (MEAN) {
+      idle = (p[i] | d[i]) == 0 && (am[i] | wm[i]) == 0;
+      rv[i] = idle ? idle_raw((T)0)
+                   : raw_tss_mean<T>(p[i], d[i], am[i], wm[i], dt, (T)tab.win[s], w_p[m], w_q[m]);
+    } else {
+      idle = (p[i] | d[i] | a[i] | w[i]) == 0;
+      rv[i] = idle ? idle_raw((T)0) : raw_tss<T>(p[i], d[i], a[i], w[i], dt, w_p[m], w_q[m]);
+    }
     cv[i] = idle ? kIdle : kNom;
     if (++m == M) m = 0;
   }
@@ -766,17 +811,26 @@ cudaError_t launch_score(const SeriesTable<T>& tab, const int32_t* P, const int3
                          const int32_t* A, const int32_t* W, const T* w_p, const T* w_q,
                          const T* alpha, const T* theta, const T* tau_crit, const T* tau_surp,
                          T* S_carry, uint8_t* init_carry, T* S, T* Z, uint8_t* cls,
-                         ScoreWs<T>& w, tre_diag* diag, cudaStream_t s) {
+                         ScoreWs<T>& w, tre_diag* diag, cudaStream_t s, const int64_t* A_ms,
+                         const int64_t* W_ms) {
   const int M = tab.M;
   const int n_seg = tab.seg_base[tab.n];
   if (n_seg > w.cap_seg) return cudaErrorInvalidValue;
+  if ((A_ms == nullptr) != (W_ms == nullptr)) return cudaErrorInvalidValue;
   const int64_t total = total_elems(tab);
   if (total == 0) return cudaSuccess;
-  const Counts c{P, D, A, W};
+  const Counts c{P, D, A, W, A_ms, W_ms};
   int n_tiles = 0;
   const TilePlan tp = tile_plan(tab, n_tiles);
-  const bool vec = quad_aligned(tab, {P, D, A, W, w.raw, cls});
-  k_raw<T><<<n_tiles, kEwThreads, 0, s>>>(tab, tp, FastDiv(M), vec, c, w_p, w_q, w.raw, cls);
+  if (A_ms) {
+    const bool vec = quad_aligned(tab, {P, D, A_ms, W_ms, w.raw, cls});
+    k_raw<T, true><<<n_tiles, kEwThreads, 0, s>>>(tab, tp, FastDiv(M), vec, c, w_p, w_q, w.raw,
+                                                  cls);
+  } else {
+    const bool vec = quad_aligned(tab, {P, D, A, W, w.raw, cls});
+    k_raw<T, false><<<n_tiles, kEwThreads, 0, s>>>(tab, tp, FastDiv(M), vec, c, w_p, w_q, w.raw,
+                                                   cls);
+  }
   const int64_t segs = (int64_t)n_seg * M;
   const unsigned g = (unsigned)((segs + kEmaThreads - 1) / kEmaThreads);
   if (theta)
@@ -836,7 +890,8 @@ cudaError_t launch_rank(int M, int K, const T* Z, const uint8_t* cls, int32_t* r
   template cudaError_t launch_score<T>(const SeriesTable<T>&, const int32_t*, const int32_t*,      \
                                        const int32_t*, const int32_t*, const T*, const T*,         \
                                        const T*, const T*, const T*, const T*, T*, uint8_t*, T*,   \
-                                       T*, uint8_t*, ScoreWs<T>&, tre_diag*, cudaStream_t);        \
+                                       T*, uint8_t*, ScoreWs<T>&, tre_diag*, cudaStream_t,         \
+                                       const int64_t*, const int64_t*);                            \
   template cudaError_t launch_normalize<T>(const SeriesTable<T>&, const T*, const uint8_t*,        \
                                            const T*, const T*, T, const T*, T*, uint8_t*,          \
                                            cudaStream_t);                                          \

@@ -317,6 +317,70 @@ def test_rank_empty_grid(tre):
     assert g["recv"].numel() == 0 and g["donors"].shape == (0, 8)
 
 
+@pytest.mark.parametrize("name,scale", [("tiny", 1.0), ("mid", 0.05), ("hetero", 0.01)])
+def test_mean_occupancy_reduce_generated(tre, name, scale):
+    w = tracegen.workload(name, scale=scale)
+    M, win, K = w["M"], w["window_ms"], w["K"]
+    A_ms, W_ms = oracle.occupancy_mean_requests(w["requests"], M, win, K)
+    c = tre.tss_window_reduce(M, win, K, requests=_cuda(w["requests"]), mean_occupancy=True)
+    np.testing.assert_array_equal(_np(c["A_ms"]), A_ms)
+    np.testing.assert_array_equal(_np(c["W_ms"]), W_ms)
+    P, D, A, W, _ = oracle.reduce_requests(w["requests"], M, win, K)
+    for k, ref in zip("PDAW", (P, D, A, W)):
+        np.testing.assert_array_equal(_np(c[k]), ref, err_msg=k)
+
+
+@pytest.mark.parametrize("seed,M,win,K", [(41, 3, 1000, 50), (42, 8, 100, 700), (43, 17, 7, 333),
+                                          (44, 64, 250, 40), (45, 1, 1, 5000)])
+def test_mean_occupancy_reduce_adversarial(tre, seed, M, win, K):
+    rng = np.random.default_rng(seed)
+    req = _adversarial(rng, 20000, M, win, K)
+    A_ms, W_ms = oracle.occupancy_mean_requests(req, M, win, K)
+    diag = tre.new_diag()
+    c = tre.tss_window_reduce(M, win, K, requests=_cuda(req), diag=diag, mean_occupancy=True)
+    np.testing.assert_array_equal(_np(c["A_ms"]), A_ms)
+    np.testing.assert_array_equal(_np(c["W_ms"]), W_ms)
+    _, _, _, _, drops = oracle.reduce_requests(req, M, win, K)
+    d = tre.read_diag(diag)   # drops are counted once, by the reduction
+    assert [d["dropped_range"], d["dropped_model"], d["dropped_order"]] == drops.tolist()
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f64"])
+@pytest.mark.parametrize("name,scale", [("tiny", 1.0), ("mid", 0.05)])
+def test_mean_occupancy_pipeline(tre, dtype, name, scale):
+    w = tracegen.workload(name, scale=scale)
+    M, win, K = w["M"], w["window_ms"], w["K"]
+    npdt = np.float32 if dtype == "f32" else np.float64
+    prof = tracegen.default_profile(M, win)
+    o = oracle.pipeline_requests(w["requests"], M, win, K, prof, w["slo_ttft_ms"], npdt,
+                                 mean_occupancy=True)
+    req = _cuda(w["requests"])
+    c = tre.tss_window_reduce(M, win, K, requests=req, mean_occupancy=True)
+    diag = tre.new_diag()
+    theta = tre.tss_calibrate(c, prof, win, w["slo_ttft_ms"], requests=req, dtype=dtype,
+                              diag=diag)
+    np.testing.assert_array_equal(_np(theta), o["theta"])
+    sc = tre.tss_score(c, dict(prof, theta=theta), win, dtype=dtype)
+    for k in ("S", "Z", "cls", "recv"):
+        np.testing.assert_array_equal(_np(sc[k]), o[k], err_msg=k)
+    # the sampled gauges give a different score on this workload
+    plain = oracle.pipeline_requests(w["requests"], M, win, K, prof, w["slo_ttft_ms"], npdt)
+    assert not np.array_equal(plain["S"], o["S"])
+
+
+def test_mean_occupancy_empty_and_refusals(tre):
+    import torch
+    M, win, K = 4, 100, 30
+    empty = {k: torch.zeros(0, dtype=torch.int32, device="cuda") for k in REQ_KEYS}
+    c = tre.tss_window_reduce(M, win, K, requests=empty, mean_occupancy=True)
+    assert int(c["A_ms"].abs().sum()) == 0 and int(c["W_ms"].abs().sum()) == 0
+    # token events cannot give the time-averaged occupancy
+    w = _events_case(3)
+    with pytest.raises(tre.TreError):
+        tre.tss_window_reduce(w["M"], w["window_ms"], w["K"], events=_cuda(w["events"]),
+                              mean_occupancy=True)
+
+
 def test_calibrate_events(tre):
     w = _events_case(6)
     ev, M, win, K = w["events"], w["M"], w["window_ms"], w["K"]

@@ -122,3 +122,19 @@ def test_rank_argument_errors_are_reported_on_the_host():
     g0 = tre.Grid(4, 1000, 0)   # empty grid: nothing to enqueue
     assert lib.tss_rank(C.byref(g0), 0, None, None, out, out, None) == 0
 
+
+def test_mean_occupancy_arguments_are_checked_on_the_host():
+    lib = tre.load()
+    g = tre.Grid(3, 1000, 10)
+    n = C.c_size_t(0)
+    rq = tre.Requests(0)
+    ev = tre.Events(0)
+    one_sided = tre.Counts(1, 1, 1, 1, 1, None)          # A_ms without W_ms
+    assert lib.tss_window_reduce(C.byref(g), C.byref(rq), None, one_sided, None, C.byref(n),
+                                 None, None) == 1
+    both = tre.Counts(1, 1, 1, 1, 1, 1)
+    assert lib.tss_window_reduce(C.byref(g), None, C.byref(ev), both, None, C.byref(n), None,
+                                 None) == 1              # token events: no window means
+    assert lib.tss_window_reduce(C.byref(g), C.byref(rq), None, both, None, C.byref(n), None,
+                                 None) == 0              # workspace query
+
