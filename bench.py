@@ -197,6 +197,66 @@ def cpu_baseline(scale):
             "sample": f"1 of the 7 traces ({n_rec} records), all 4 window lengths, all 64 settings; {dt:.1f} s"}
 
 
+TRACE_PHASES = 10   # phases of tre_trace (the library header's count)
+
+
+def occupancy_cpu(scale):
+    """The oracle's time-averaged occupancy on one trace of the workload (1 core)."""
+    import oracle
+    sw = tracegen.sweep_workload(scale=scale, n_traces=1)
+    req = sw["traces"][0]
+    t0 = time.perf_counter()
+    oracle.occupancy_mean_requests(req, sw["M"], 100, sw["duration_ms"] // 100)
+    dt = time.perf_counter() - t0
+    n = len(req["model"])
+    return {"value": n / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"1 trace ({n} records) at the 100 ms grid; {dt:.2f} s"}
+
+
+def occupancy_measure(lib, Trace, dev_traces, M, duration_ms, hbm, peak_kind, reps=5):
+    """The time-averaged occupancy pass of tss_window_reduce (request-ms running
+    and waiting per window) on each trace of the workload at the 100 ms grid,
+    timed on the device by the library's phase events. The seven traces are
+    taken in turn (196 MB of records in all, more than L2), so a trace's columns
+    are not resident when it comes round again."""
+    import torch
+
+    import paper_2609_29160_gb300 as tre
+    win = 100
+    K = duration_ms // win
+    out = {k: torch.empty((K, M), dtype=torch.int32, device="cuda") for k in "PDAW"}
+    for k in ("A_ms", "W_ms"):
+        out[k] = torch.empty((K, M), dtype=torch.int64, device="cuda")
+    diag = tre.new_diag()
+    for t in dev_traces:
+        tre.tss_window_reduce(M, win, K, requests=t, out=out, diag=diag, mean_occupancy=True)
+    torch.cuda.synchronize()
+    lib.tre_trace_enable(1)
+    for _ in range(reps):
+        for t in dev_traces:
+            tre.tss_window_reduce(M, win, K, requests=t, out=out, diag=diag, mean_occupancy=True)
+    torch.cuda.synchronize()
+    tr = Trace()
+    lib.tre_trace_collect(C.byref(tr))
+    lib.tre_trace_enable(0)
+    ph = {tr.name[i].decode(): (tr.ms[i], tr.calls[i]) for i in range(tr.n_phases)}
+    n_rec = sum(int(t["model"].numel()) for t in dev_traces) / len(dev_traces)
+    occ_ms, occ_calls = ph["occupancy"]
+    red_ms, red_calls = ph["reduce"]
+    us = occ_ms / max(occ_calls, 1) * 1e3
+    # algorithmic bytes: the records' columns read once, the two int64 outputs
+    # written once
+    byts = n_rec * 28 + K * M * 16
+    achieved = byts / (us / 1e6) / 1e9
+    return {"row": "time-averaged running/waiting occupancy (request-ms per window)",
+            "window_ms": win, "records_per_call": int(n_rec), "model_windows_per_call": K * M,
+            "us_per_call": us, "sampled_reduce_us_per_call": red_ms / max(red_calls, 1) * 1e3,
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                         "frac": achieved / hbm, "peak_kind": peak_kind,
+                         "bytes_per_call": byts, "traffic": None},
+            "l2": "7 traces in turn, 196 MB of records"}
+
+
 # DRAM traffic per call of a phase, from the committed ncu summary of its
 # kernels; used only while the kernel source is the one the counters were
 # taken on (the summary records its SHA-256)
@@ -268,9 +328,11 @@ def main():
     lib = tre.load()
     lib.tre_trace_enable.argtypes = [C.c_int]
 
+    NP = TRACE_PHASES
+
     class Trace(C.Structure):
-        _fields_ = [("n_phases", C.c_int32), ("name", C.c_char_p * 9), ("ms", C.c_double * 9),
-                    ("calls", C.c_int64 * 9), ("launches", C.c_int64 * 9)]
+        _fields_ = [("n_phases", C.c_int32), ("name", C.c_char_p * NP), ("ms", C.c_double * NP),
+                    ("calls", C.c_int64 * NP), ("launches", C.c_int64 * NP)]
     lib.tre_trace_collect.argtypes = [C.POINTER(Trace)]
 
     # each rank sweeps its own 7 traces (independent problems: weak scaling)
@@ -464,9 +526,14 @@ def main():
            "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
            "ms_per_step": e2e_ms, "steps": n_e2e, "mode": mode}
 
+    # a widened step measured beside the sweep (not part of the timed step)
+    next_rows = {"occupancy_mean": occupancy_measure(lib, Trace, dev_traces, M,
+                                                     sw["duration_ms"], hbm, peak_kind)}
+
     base = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         base = cpu_baseline(args.scale)
+        next_rows["occupancy_mean"]["cpu_baseline"] = occupancy_cpu(args.scale)
     if rank == 0:
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
@@ -484,6 +551,7 @@ def main():
             "phases_roofline": {k: round(roof_of(k)["frac"], 4) for k in pb
                                 if phases.get(k, {}).get("calls")},
             "gpu_launches": launches, "clocks": clk, "e2e": e2e, "cpu_baseline": base,
+            "next_rows": next_rows,
         }
         print(json.dumps(line))
     if world > 1:

@@ -316,8 +316,9 @@ tre_status tre_sweep(const tre_sweep_spec* spec, const tre_sweep_out* out, void*
  * returns per-phase device milliseconds and kernel-launch counts accumulated
  * since tracing was enabled (or since the last collect), and starts over.
  * Phases: reduce, gauge_scan, aggregate, score, receiver, slo_counts,
- * calibrate, normalize, select. No counterpart in the paper (instrumentation). */
-#define TRE_TRACE_PHASES 9
+ * calibrate, normalize, select, occupancy (the time-averaged occupancy pass of
+ * tss_window_reduce). No counterpart in the paper (instrumentation). */
+#define TRE_TRACE_PHASES 10
 typedef struct {
   int32_t n_phases;
   const char* name[TRE_TRACE_PHASES];

@@ -86,10 +86,10 @@ tre_status cuda_status(cudaError_t e) { return e == cudaSuccess ? TRE_OK : TRE_E
 
 // ---- phase tracing ----------------------------------------------------------
 enum Phase { kReduce, kScan, kAggregate, kScore, kReceiver, kSlo, kCalibrate, kNormalize,
-             kSelect };
+             kSelect, kOccupancy };
 const char* const kPhaseName[TRE_TRACE_PHASES] = {"reduce", "gauge_scan", "aggregate", "score",
                                                   "receiver", "slo_counts", "calibrate",
-                                                  "normalize", "select"};
+                                                  "normalize", "select", "occupancy"};
 struct TraceRec {
   int phase, launches;
   cudaEvent_t a, b;
@@ -551,7 +551,7 @@ tre_status tss_window_reduce(const tre_grid* grid, const tre_requests* req, cons
     e = launch_gauge_scan(M, K, w, out.A, out.W, s);
   }
   if (!e && out.A_ms) {
-    Scope sc(kScan, 4, s);
+    Scope sc(kOccupancy, 3 + (req->n > 0), s);
     e = launch_occupancy_mean(cols_of(req), M, grid->window_ms, K, w, out.A_ms, out.W_ms, s);
   }
   return cuda_status(e);
