@@ -587,32 +587,43 @@ k_scan_partials(int M, int K, int L, int n_chunks, const int32_t* __restrict__ d
   pW[t] = w;
 }
 
-// exclusive scan over chunks, one warp per model (n_chunks <= 1024)
-__global__ void k_scan_chunks(int M, int n_chunks, int32_t* __restrict__ pA,
-                              int32_t* __restrict__ pW) {
-  const int m = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
-  if (m >= M) return;
+// exclusive scan over chunks, one CTA per model, one thread per chunk
+// (n_chunks <= 1024)
+__global__ void __launch_bounds__(1024)
+k_scan_chunks(int M, int n_chunks, int32_t* __restrict__ pA, int32_t* __restrict__ pW) {
+  __shared__ int32_t wa[32], ww[32];
+  const int m = blockIdx.x;
   pA += (size_t)blockIdx.y * n_chunks * M;
   pW += (size_t)blockIdx.y * n_chunks * M;
-  const int lane = threadIdx.x & 31;
-  const int per = (n_chunks + 31) / 32;
-  const int c0 = lane * per, c1 = min(n_chunks, c0 + per);
-  int32_t sa = 0, sw = 0;
-  for (int c = c0; c < c1; ++c) { sa += pA[(size_t)c * M + m]; sw += pW[(size_t)c * M + m]; }
-  int32_t ia = sa, iw = sw;
+  const int c = threadIdx.x, lane = c & 31, wid = c >> 5;
+  const int32_t va = c < n_chunks ? pA[(size_t)c * M + m] : 0;
+  const int32_t vw = c < n_chunks ? pW[(size_t)c * M + m] : 0;
+  int32_t ia = va, iw = vw;
+#pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
     const int32_t xa = __shfl_up_sync(0xffffffffu, ia, o);
     const int32_t xw = __shfl_up_sync(0xffffffffu, iw, o);
     if (lane >= o) { ia += xa; iw += xw; }
   }
-  int32_t ea = ia - sa, ew = iw - sw;
-  for (int c = c0; c < c1; ++c) {
-    const size_t x = (size_t)c * M + m;
-    const int32_t va = pA[x], vw = pW[x];
-    pA[x] = ea;
-    pW[x] = ew;
-    ea += va;
-    ew += vw;
+  if (lane == 31) { wa[wid] = ia; ww[wid] = iw; }
+  __syncthreads();
+  if (wid == 0) {
+    int32_t sa = lane < (int)(blockDim.x >> 5) ? wa[lane] : 0;
+    int32_t sw = lane < (int)(blockDim.x >> 5) ? ww[lane] : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int32_t xa = __shfl_up_sync(0xffffffffu, sa, o);
+      const int32_t xw = __shfl_up_sync(0xffffffffu, sw, o);
+      if (lane >= o) { sa += xa; sw += xw; }
+    }
+    wa[lane] = sa;   // inclusive over warps
+    ww[lane] = sw;
+  }
+  __syncthreads();
+  const int32_t base_a = wid ? wa[wid - 1] : 0, base_w = wid ? ww[wid - 1] : 0;
+  if (c < n_chunks) {
+    pA[(size_t)c * M + m] = base_a + ia - va;
+    pW[(size_t)c * M + m] = base_w + iw - vw;
   }
 }
 
@@ -1061,7 +1072,7 @@ cudaError_t launch_gauge_scan(int M, int K, ReduceWs& w, int32_t* A, int32_t* W,
   const int64_t segs = (int64_t)n_chunks * M;
   dim3 g((unsigned)((segs + kThreads - 1) / kThreads), w.n_traces);
   k_scan_partials<<<g, kThreads, 0, s>>>(M, K, L, n_chunks, w.dA, w.dW, w.partA, w.partW);
-  k_scan_chunks<<<dim3((M + 3) / 4, w.n_traces), 128, 0, s>>>(M, n_chunks, w.partA, w.partW);
+  k_scan_chunks<<<dim3(M, w.n_traces), 1024, 0, s>>>(M, n_chunks, w.partA, w.partW);
   k_scan_apply<<<g, kThreads, 0, s>>>(M, K, L, n_chunks, w.dA, w.dW, w.partA, w.partW, A, W);
   return cudaGetLastError();
 }
@@ -1070,42 +1081,177 @@ cudaError_t launch_gauge_scan(int M, int K, ReduceWs& w, int32_t* A, int32_t* W,
 // waiting counts, Sec. III-A): the request-milliseconds that running
 // ([t_start, t_end)) and waiting ([t_arr, t_start)) requests spend inside each
 // window. A span adds its partial first and last windows directly (64-bit
-// atomics into the output) and marks the windows it covers completely in a
-// +1/-1 difference array; the prefix of that array times the window length is
-// added afterwards. Records are taken or skipped by the reduction's rules.
-__device__ __forceinline__ void occ_span(uint32_t a, uint32_t e, uint32_t span, int m, int M,
-                                         uint32_t win, const FastDiv& fd,
-                                         unsigned long long* __restrict__ part,
-                                         int32_t* __restrict__ full) {
-  if (e > span) e = span;
-  if (a >= e) return;
-  const uint32_t ka = fd.div(a), ke = fd.div(e - 1);
-  if (ka == ke) {
-    atomicAdd(&part[(size_t)ka * M + m], (unsigned long long)(e - a));
-    return;
-  }
-  atomicAdd(&part[(size_t)ka * M + m], (unsigned long long)((ka + 1) * win - a));
-  atomicAdd(&part[(size_t)ke * M + m], (unsigned long long)(e - ke * win));
-  if (ke > ka + 1) {
-    atomicAdd(&full[(size_t)(ka + 1) * M + m], 1);
-    atomicAdd(&full[(size_t)ke * M + m], -1);
-  }
-}
-
+// sums) and marks the windows it covers completely in a +1/-1 difference
+// array; the prefix of that array times the window length is added
+// afterwards. Records are taken or skipped by the reduction's rules.
+// One CTA per chunk of consecutive records, staged in shared memory like the
+// token reduction: the waiting span's first window sits on the arrival side
+// (rows from the chunk's first arrival window), every other target near the
+// record's start (per model, a run of F windows from the earliest start among
+// the chunk's records). Targets outside both go to global atomics. Staged
+// partial sums are 32-bit (a chunk adds at most kOccPerCta * win to a cell,
+// staged only for win <= 2^20); the covered-window difference counts of
+// running and waiting share one word per start-side cell (each bounded by the
+// chunk's record count). Each thread reads four consecutive records per pass
+// with 16-byte loads when the columns allow it.
+constexpr int kOccPerCta = 2048;
 __global__ void __launch_bounds__(kThreads)
-k_occ_spans(ReqCols r, int M, int win, FastDiv fd, int K, unsigned long long* __restrict__ pA,
-            unsigned long long* __restrict__ pW, int32_t* __restrict__ fA,
-            int32_t* __restrict__ fW) {
+k_occ_staged(ReqCols r, bool vec, bool stage, int M, int lgMp, int win, FastDiv fd, int K,
+             int near_rows, int lgF, unsigned long long* __restrict__ pA,
+             unsigned long long* __restrict__ pW, int32_t* __restrict__ fA,
+             int32_t* __restrict__ fW) {
+  extern __shared__ uint32_t osm32[];
+  const int64_t i0 = (int64_t)blockIdx.x * kOccPerCta;
+  const int n_loc = (int)min64(r.n - i0, kOccPerCta);
+  if (n_loc <= 0) return;
+  const int Mp = 1 << lgMp, F = 1 << lgF;
   const uint32_t span = (uint32_t)K * (uint32_t)win;
-  for (int64_t i = (int64_t)blockIdx.x * kThreads + threadIdx.x; i < r.n;
-       i += (int64_t)gridDim.x * kThreads) {
-    const int m = r.model[i];
-    if (m < 0 || m >= M) continue;
-    const int ta = r.t_arr[i], ts = r.t_start[i], tf = r.t_first[i], te = r.t_end[i];
-    if (ta < 0 || (uint32_t)ta >= span) continue;
-    if (!(ta <= ts && ts <= tf && tf <= te) || r.L_in[i] < 0 || r.L_out[i] < 1) continue;
-    occ_span((uint32_t)ts, (uint32_t)te, span, m, M, (uint32_t)win, fd, pA, fA);
-    occ_span((uint32_t)ta, (uint32_t)ts, span, m, M, (uint32_t)win, fd, pW, fW);
+  const uint32_t uw = (uint32_t)win;
+  uint32_t* sWp = osm32;                                             // [near_rows][Mp]
+  int32_t* sWf = reinterpret_cast<int32_t*>(sWp + (size_t)near_rows * Mp);
+  uint32_t* sAp = reinterpret_cast<uint32_t*>(sWf + (size_t)near_rows * Mp);  // [M][F]
+  uint32_t* sWq = sAp + (size_t)M * F;                               // [M][F]
+  int32_t* sAWf = reinterpret_cast<int32_t*>(sWq + (size_t)M * F);   // [M][F]
+  int32_t* slo = sAWf + (size_t)M * F;                               // [M]
+  const int32_t* col[7] = {r.model + i0, r.t_arr + i0, r.t_start + i0, r.t_first + i0,
+                           r.t_end + i0, r.L_in + i0, r.L_out + i0};
+  const int a_first = col[1][0], a_last = col[1][n_loc - 1];
+  const int k_lo = a_first < 0 ? 0 : (int)min(fd.div((uint32_t)a_first), (uint32_t)K);
+  const int k_hi = a_last < 0 ? 0 : (int)min(fd.div((uint32_t)a_last), (uint32_t)K);
+  const int used = stage ? min(near_rows, (k_hi >= k_lo ? k_hi - k_lo + 1 : 1) + 1) : 0;
+  const int Fs = stage ? F : 0;
+  for (int c = threadIdx.x; c < used * Mp; c += kThreads) { sWp[c] = 0; sWf[c] = 0; }
+  for (int c = threadIdx.x; c < M * Fs; c += kThreads) { sAp[c] = 0; sWq[c] = 0; sAWf[c] = 0; }
+  for (int m = threadIdx.x; m < M; m += kThreads) slo[m] = 0x7fffffff;
+  __syncthreads();
+  // each model's earliest start-side window: the window before its first start
+  for (int b = threadIdx.x * kVec; b < n_loc; b += kThreads * kVec) {
+    int mm[kVec], ss[kVec];
+    if (vec && b + kVec <= n_loc) {
+      const int4 a = *reinterpret_cast<const int4*>(col[0] + b);
+      const int4 q = *reinterpret_cast<const int4*>(col[2] + b);
+      mm[0] = a.x; mm[1] = a.y; mm[2] = a.z; mm[3] = a.w;
+      ss[0] = q.x; ss[1] = q.y; ss[2] = q.z; ss[3] = q.w;
+    } else {
+#pragma unroll
+      for (int u = 0; u < kVec; ++u) {
+        const bool in = b + u < n_loc;
+        mm[u] = in ? col[0][b + u] : -1;
+        ss[u] = in ? col[2][b + u] : -1;
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kVec; ++u) {
+      if (mm[u] < 0 || mm[u] >= M || ss[u] < 0) continue;
+      const uint32_t s1 = min((uint32_t)ss[u], span);
+      atomicMin(&slo[mm[u]], s1 > 0 ? (int)fd.div(s1 - 1) : 0);
+    }
+  }
+  __syncthreads();
+  for (int b = threadIdx.x * kVec; b < n_loc; b += kThreads * kVec) {
+    int v[7][kVec];
+    if (vec && b + kVec <= n_loc) {
+#pragma unroll
+      for (int c = 0; c < 7; ++c) {
+        const int4 q = *reinterpret_cast<const int4*>(col[c] + b);
+        v[c][0] = q.x; v[c][1] = q.y; v[c][2] = q.z; v[c][3] = q.w;
+      }
+    } else {
+#pragma unroll
+      for (int u = 0; u < kVec; ++u) {
+        const bool in = b + u < n_loc;
+#pragma unroll
+        for (int c = 0; c < 7; ++c) v[c][u] = in ? col[c][b + u] : 0;
+        if (!in) v[0][u] = -1;
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kVec; ++u) {
+      const int m = v[0][u], ta = v[1][u], ts = v[2][u], tf = v[3][u], te = v[4][u];
+      if (m < 0 || m >= M) continue;
+      if (ta < 0 || (uint32_t)ta >= span) continue;
+      if (!(ta <= ts && ts <= tf && tf <= te) || v[5][u] < 0 || v[6][u] < 1) continue;
+      const int lo = slo[m];
+      auto near_part = [&](uint32_t k, uint32_t val) {
+        const uint32_t rel = k - (uint32_t)k_lo;
+        if (rel < (uint32_t)used) atomicAdd(&sWp[(rel << lgMp) + m], val);
+        else atomicAdd(&pW[(size_t)k * M + m], (unsigned long long)val);
+      };
+      auto near_full = [&](uint32_t k) {
+        const uint32_t rel = k - (uint32_t)k_lo;
+        if (rel < (uint32_t)used) atomicAdd(&sWf[(rel << lgMp) + m], 1);
+        else atomicAdd(&fW[(size_t)k * M + m], 1);
+      };
+      auto far_part = [&](uint32_t* st, unsigned long long* g, uint32_t k, uint32_t val) {
+        const uint32_t rel = k - (uint32_t)lo;
+        if (rel < (uint32_t)Fs) atomicAdd(&st[(m << lgF) + rel], val);
+        else atomicAdd(&g[(size_t)k * M + m], (unsigned long long)val);
+      };
+      auto far_full = [&](uint32_t k, int32_t a, int32_t w) {
+        const uint32_t rel = k - (uint32_t)lo;
+        if (rel < (uint32_t)Fs) {
+          atomicAdd(&sAWf[(m << lgF) + rel], a + w * 65536);
+        } else {
+          if (a) atomicAdd(&fA[(size_t)k * M + m], a);
+          if (w) atomicAdd(&fW[(size_t)k * M + m], w);
+        }
+      };
+      // waiting on [ta, ts)
+      const uint32_t ew = min((uint32_t)ts, span);
+      if ((uint32_t)ta < ew) {
+        const uint32_t ka = fd.div((uint32_t)ta), kw = fd.div(ew - 1);
+        if (ka == kw) {
+          near_part(ka, ew - (uint32_t)ta);
+        } else {
+          near_part(ka, (ka + 1) * uw - (uint32_t)ta);
+          far_part(sWq, pW, kw, ew - kw * uw);
+          if (kw > ka + 1) {
+            near_full(ka + 1);
+            far_full(kw, 0, -1);
+          }
+        }
+      }
+      // running on [ts, te)
+      const uint32_t er = min((uint32_t)te, span);
+      if ((uint32_t)ts < er) {
+        const uint32_t ks = fd.div((uint32_t)ts), ke = fd.div(er - 1);
+        if (ks == ke) {
+          far_part(sAp, pA, ks, er - (uint32_t)ts);
+        } else {
+          far_part(sAp, pA, ks, (ks + 1) * uw - (uint32_t)ts);
+          far_part(sAp, pA, ke, er - ke * uw);
+          if (ke > ks + 1) {
+            far_full(ks + 1, 1, 0);
+            far_full(ke, -1, 0);
+          }
+        }
+      }
+    }
+  }
+  __syncthreads();
+  for (int c = threadIdx.x; c < used * Mp; c += kThreads) {
+    const int m = c & (Mp - 1);
+    const int k = k_lo + (c >> lgMp);
+    if (m >= M || k >= K) continue;
+    if (sWp[c]) atomicAdd(&pW[(size_t)k * M + m], (unsigned long long)sWp[c]);
+    if (sWf[c]) atomicAdd(&fW[(size_t)k * M + m], sWf[c]);
+  }
+  for (int c = threadIdx.x; c < M * Fs; c += kThreads) {
+    const int m = c >> lgF;
+    const int lo = slo[m];
+    if (lo == 0x7fffffff) continue;
+    const int k = lo + (c & (F - 1));
+    if (k >= K) continue;
+    const size_t g = (size_t)k * M + m;
+    if (sAp[c]) atomicAdd(&pA[g], (unsigned long long)sAp[c]);
+    if (sWq[c]) atomicAdd(&pW[g], (unsigned long long)sWq[c]);
+    const int32_t aw = sAWf[c];
+    if (aw) {
+      const int32_t a = (int32_t)(int16_t)(aw & 0xffff);
+      const int32_t w = (aw - a) / 65536;
+      if (a) atomicAdd(&fA[g], a);
+      if (w) atomicAdd(&fW[g], w);
+    }
   }
 }
 
@@ -1122,11 +1268,29 @@ k_occ_apply(int M, int K, int L, int n_chunks, int win, const int32_t* __restric
   const int c = (int)(t / M);
   const int64_t r0 = (int64_t)c * L, r1 = min64(r0 + L, K);
   int32_t a = pA[t], w = pW[t];
-  for (int64_t k = r0; k < r1; ++k) {
-    a += fA[k * M + m];
-    w += fW[k * M + m];
-    A_ms[k * M + m] += (long long)a * win;
-    W_ms[k * M + m] += (long long)w * win;
+  constexpr int B = 8;
+  for (int64_t k0 = r0; k0 < r1; k0 += B) {
+    int32_t da[B], dw[B];
+    long long am[B], wm[B];
+#pragma unroll
+    for (int j = 0; j < B; ++j) {
+      const bool in = k0 + j < r1;
+      const int64_t x = (k0 + j) * M + m;
+      da[j] = in ? fA[x] : 0;
+      dw[j] = in ? fW[x] : 0;
+      am[j] = in ? A_ms[x] : 0;
+      wm[j] = in ? W_ms[x] : 0;
+    }
+#pragma unroll
+    for (int j = 0; j < B; ++j) {
+      a += da[j];
+      w += dw[j];
+      if (k0 + j < r1) {
+        const int64_t x = (k0 + j) * M + m;
+        A_ms[x] = am[j] + (long long)a * win;
+        W_ms[x] = wm[j] + (long long)w * win;
+      }
+    }
   }
 }
 
@@ -1139,17 +1303,45 @@ cudaError_t launch_occupancy_mean(const ReqCols& r, int M, int win, int K, Reduc
   if (!e) e = cudaMemsetAsync(w.dA, 0, cells1 * sizeof(int32_t), s);
   if (!e) e = cudaMemsetAsync(w.dW, 0, cells1 * sizeof(int32_t), s);
   if (e) return e;
-  if (r.n > 0)
-    k_occ_spans<<<grid_for(r.n, 4), kThreads, 0, s>>>(
-        r, M, win, FastDiv(win), K, reinterpret_cast<unsigned long long*>(A_ms),
-        reinterpret_cast<unsigned long long*>(W_ms), w.dA, w.dW);
+  if (r.n > 0) {
+    int lgMp = 0;
+    while ((1 << lgMp) < M) ++lgMp;
+    const int Mp = 1 << lgMp;
+    // arrival-side rows: 3x the mean arrival span of a chunk, within 16 KB
+    const int64_t near_cap = std::max<int64_t>(1, 16 * 1024 / (8 * Mp));
+    const int near_rows = (int)std::max<int64_t>(
+        1, std::min<int64_t>(near_cap, (int64_t)(3.0 * kOccPerCta / r.n * K) + 34));
+    // start-side run per model: the longest power of two within 24 KB
+    int lgF = 0;
+    while (lgF < 8 && (size_t)12 * M * (2u << lgF) <= 24 * 1024) ++lgF;
+    const size_t smem = (size_t)near_rows * Mp * 8 + (size_t)12 * M * (1u << lgF) +
+                        (size_t)4 * M;
+    const bool vec = ((uintptr_t)r.model | (uintptr_t)r.t_arr | (uintptr_t)r.t_start |
+                      (uintptr_t)r.t_first | (uintptr_t)r.t_end | (uintptr_t)r.L_in |
+                      (uintptr_t)r.L_out) % 16 == 0;
+    const bool stage = win <= (1 << 20);   // 32-bit staged sums cannot overflow
+    static bool attr = false;
+    if (!attr) {
+      e = cudaFuncSetAttribute(k_occ_staged, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               96 * 1024);
+      if (e) return e;
+      attr = true;
+    }
+    if (smem > 96 * 1024) return cudaErrorInvalidValue;
+    const unsigned ctas = (unsigned)((r.n + kOccPerCta - 1) / kOccPerCta);
+    k_occ_staged<<<ctas, kThreads, smem, s>>>(r, vec, stage, M, lgMp, win, FastDiv(win), K,
+                                              near_rows, lgF,
+                                              reinterpret_cast<unsigned long long*>(A_ms),
+                                              reinterpret_cast<unsigned long long*>(W_ms), w.dA,
+                                              w.dW);
+  }
   const int L = scan_chunk_rows(K);
   const int n_chunks = (K + L - 1) / L;
   const int64_t segs = (int64_t)n_chunks * M;
   const unsigned g = (unsigned)((segs + kThreads - 1) / kThreads);
   k_scan_partials<<<dim3(g, 1), kThreads, 0, s>>>(M, K, L, n_chunks, w.dA, w.dW, w.partA,
                                                   w.partW);
-  k_scan_chunks<<<dim3((M + 3) / 4, 1), 128, 0, s>>>(M, n_chunks, w.partA, w.partW);
+  k_scan_chunks<<<dim3(M, 1), 1024, 0, s>>>(M, n_chunks, w.partA, w.partW);
   k_occ_apply<<<g, kThreads, 0, s>>>(M, K, L, n_chunks, win, w.dA, w.dW, w.partA, w.partW,
                                      reinterpret_cast<long long*>(A_ms),
                                      reinterpret_cast<long long*>(W_ms));
