@@ -92,6 +92,18 @@ def occupancy_mean_requests(req, M, window_ms, K):
     return A_ms, W_ms
 
 
+def class_models(model, cls, M, n_classes):
+    """Model ids of (model, SLO class) pairs: model * n_classes + class, -1 if
+    either is out of range."""
+    model, cls = _i32(model), _i32(cls)
+    out = np.zeros(len(model), np.int32)
+    rc = lib().orc_class_models(C.c_int64(len(model)), _p(model), _p(cls), C.c_int32(M),
+                                C.c_int32(n_classes), _p(out))
+    if rc:
+        raise ValueError("oracle: bad arguments")
+    return out
+
+
 def slo_counts_requests(req, M, window_ms, K, slo_ttft_ms):
     cols = _req_cols(req)
     n_arr, n_met = np.zeros((K, M), np.int32), np.zeros((K, M), np.int32)

@@ -606,6 +606,19 @@ int orc_slo_counts_events(int32_t M, int32_t win, int32_t K, int64_t n_req,
 ORC_TYPED(f32, float)
 ORC_TYPED(f64, double)
 
+// Per-(model, SLO class) signal with a class per request (Sec. II-A gives
+// each model one class): every (model, class) pair becomes a model of its own,
+// id model * n_classes + class; ids outside the grid become -1.
+int orc_class_models(int64_t n, const int32_t* model, const int32_t* cls, int32_t M, int32_t C,
+                     int32_t* out) {
+  if (n < 0 || M < 1 || C < 1) return 1;
+  for (int64_t i = 0; i < n; ++i) {
+    const bool ok = model[i] >= 0 && model[i] < M && cls[i] >= 0 && cls[i] < C;
+    out[i] = ok ? model[i] * C + cls[i] : -1;
+  }
+  return 0;
+}
+
 int orc_rank_f32(int32_t M, int32_t K, const float* Z, const uint8_t* cls, int32_t* recv,
                  int32_t* order) {
   return rank_windows<float>(M, K, Z, cls, recv, order);
