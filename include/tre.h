@@ -203,6 +203,20 @@ tre_status tss_rank(const tre_grid* grid, tre_dtype dtype, const void* Z, const 
                     int32_t* recv_out, int32_t* donors_out, tre_stream stream);
 
 /*
+ * tss_class_models -- per-(model, SLO class) TSS with a class per request. The
+ * paper gives each model one SLO class (Sec. II-A); to keep the signal per
+ * (model, class) pair, every pair is treated as a model of its own:
+ * model_out[i] = model[i] * n_classes + cls[i], or -1 when model[i] is outside
+ * [0, n_models) or cls[i] outside [0, n_classes) (the reduction then drops the
+ * record as a bad model id). Pass model_out as the records' model column and
+ * n_models * n_classes as the grid's model count; slo_ttft_ms then holds one
+ * bound per pair. model, cls, model_out: device int32[n] (model_out may alias
+ * model). Limit: n_models * n_classes <= 1024. No workspace.
+ */
+tre_status tss_class_models(int64_t n, const int32_t* model, const int32_t* cls, int32_t n_models,
+                            int32_t n_classes, int32_t* model_out, tre_stream stream);
+
+/*
  * tss_calibrate -- healthy boundary theta (Sec. III-B: the lowest smoothed TSS at
  * which the SLO reliability target is still met). Calibration windows have at least
  * one arrival, are not idle and have S > 0. A window is healthy when at least

@@ -117,6 +117,8 @@ def load(build_if_missing: bool = True):
     lib.tre_sweep.argtypes = [C.POINTER(SweepSpec), C.POINTER(SweepOut), P,
                               C.POINTER(C.c_size_t), P, P]
     lib.tss_rank.argtypes = [C.POINTER(Grid), C.c_int, P, P, P, P, P]
+    lib.tss_class_models.argtypes = [C.c_int64, P, P, C.c_int32, C.c_int32, P, P]
+    lib.tss_class_models.restype = C.c_int
     for f in ("tss_window_reduce", "tss_score", "tss_calibrate", "tre_select_moves", "tre_sweep",
               "tss_rank"):
         getattr(lib, f).restype = C.c_int
@@ -265,6 +267,21 @@ def tss_score(counts, profile, window_ms, dtype="f32", carry=None, recv=True, di
         _ptr(carry["init"]) if carry else None, _ptr(S), _ptr(Z), _ptr(cls), _ptr(rv), ws, n,
         _ptr(diag), s))
     return {"S": S, "Z": Z, "cls": cls, "recv": rv}
+
+
+def tss_class_models(model, cls, n_models, n_classes, out=None, stream=None):
+    """Per-(model, SLO class) ids (model * n_classes + class, -1 when out of
+    range) as an int32 CUDA tensor, to pass as the records' model column with
+    n_models * n_classes models."""
+    torch = _torch()
+    lib = load()
+    n = int(model.numel())
+    if out is None:
+        out = torch.empty(n, dtype=torch.int32, device=model.device)
+    _check("tss_class_models", lib.tss_class_models(C.c_int64(n), _ptr(model), _ptr(cls),
+                                                    n_models, n_classes, _ptr(out),
+                                                    _stream(stream)))
+    return out
 
 
 RANK_DONORS = 8

@@ -381,6 +381,46 @@ def test_mean_occupancy_empty_and_refusals(tre):
                               mean_occupancy=True)
 
 
+def test_class_models_mapping(tre):
+    import torch
+    rng = np.random.default_rng(51)
+    n, M, n_cls = 100003, 8, 3
+    model = rng.integers(-2, M + 2, n).astype(np.int32)
+    cls = rng.integers(-1, n_cls + 1, n).astype(np.int32)
+    got = tre.tss_class_models(torch.as_tensor(model).cuda(), torch.as_tensor(cls).cuda(), M,
+                               n_cls)
+    np.testing.assert_array_equal(_np(got), oracle.class_models(model, cls, M, n_cls))
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f64"])
+def test_per_class_pipeline(tre, dtype):
+    # one SLO class per request: each (model, class) pair is scored as a model
+    w = tracegen.workload("mid", scale=0.05)
+    M, win, K = w["M"], w["window_ms"], w["K"]
+    n_cls = 3
+    rng = np.random.default_rng(52)
+    cls = rng.integers(0, n_cls, len(w["requests"]["model"])).astype(np.int32)
+    pair_model = oracle.class_models(w["requests"]["model"], cls, M, n_cls)
+    pair_req = dict(w["requests"], model=pair_model)
+    Mp = M * n_cls
+    slo = np.tile(np.array(tracegen.SLO_CLASSES_MS, np.int32), M)
+    npdt = np.float32 if dtype == "f32" else np.float64
+    prof = tracegen.default_profile(Mp, win)
+    o = oracle.pipeline_requests(pair_req, Mp, win, K, prof, slo, npdt)
+    req = _cuda(w["requests"])
+    import torch
+    req["model"] = tre.tss_class_models(req["model"], torch.as_tensor(cls).cuda(), M, n_cls)
+    np.testing.assert_array_equal(_np(req["model"]), pair_model)
+    c = tre.tss_window_reduce(Mp, win, K, requests=req)
+    for k in "PDAW":
+        np.testing.assert_array_equal(_np(c[k]), o[k], err_msg=k)
+    theta = tre.tss_calibrate(c, prof, win, slo, requests=req, dtype=dtype)
+    np.testing.assert_array_equal(_np(theta), o["theta"])
+    sc = tre.tss_score(c, dict(prof, theta=theta), win, dtype=dtype)
+    for k in ("S", "Z", "cls", "recv"):
+        np.testing.assert_array_equal(_np(sc[k]), o[k], err_msg=k)
+
+
 def test_calibrate_events(tre):
     w = _events_case(6)
     ev, M, win, K = w["events"], w["M"], w["window_ms"], w["K"]

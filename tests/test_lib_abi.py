@@ -138,3 +138,13 @@ def test_mean_occupancy_arguments_are_checked_on_the_host():
     assert lib.tss_window_reduce(C.byref(g), C.byref(rq), None, both, None, C.byref(n), None,
                                  None) == 0              # workspace query
 
+
+def test_class_models_arguments_are_checked_on_the_host():
+    lib = tre.load()
+    p = C.c_void_p(16)          # never dereferenced: the checks fail first
+    assert lib.tss_class_models(10, p, p, 0, 3, p, None) == 1      # no models
+    assert lib.tss_class_models(10, p, p, 8, 0, p, None) == 1      # no classes
+    assert lib.tss_class_models(10, p, p, 400, 3, p, None) == 1    # more than 1024 pairs
+    assert lib.tss_class_models(10, None, p, 8, 3, p, None) == 1
+    assert lib.tss_class_models(0, None, None, 8, 3, None, None) == 0
+
