@@ -182,15 +182,35 @@ def _workspace(fn, call):
     return ws
 
 
+def _need(t, dtype, n=None, what="array"):
+    """Checks a tensor argument before its pointer is handed to the library:
+    element type, contiguity and (when given) element count."""
+    torch = _torch()
+    want = getattr(torch, dtype)
+    if t.dtype != want:
+        raise ValueError(f"{what}: expected {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{what}: must be contiguous")
+    if n is not None and int(t.numel()) != n:
+        raise ValueError(f"{what}: expected {n} elements, got {int(t.numel())}")
+
+
 def requests_struct(req):
-    """tre_requests from a dict of int32 CUDA tensors (keeps no reference)."""
+    """tre_requests from a dict of int32 tensors, CUDA or pinned host (keeps no
+    reference)."""
     keys = ("model", "t_arr_ms", "t_start_ms", "t_first_ms", "t_end_ms", "L_in", "L_out")
     n = int(req["model"].numel())
+    for k in keys:
+        _need(req[k], "int32", n, k)
     return Requests(n, *[req[k].data_ptr() if n else None for k in keys])
 
 
 def events_struct(ev):
     n, nr = int(ev["model"].numel()), int(ev["req_model"].numel())
+    for k, dt, cnt in (("model", "int32", n), ("req", "int32", n), ("t_s", "float32", n),
+                       ("phase", "uint8", n), ("req_model", "int32", nr),
+                       ("req_t_arr_ms", "int32", nr), ("req_ttft_ms", "int32", nr)):
+        _need(ev[k], dt, cnt, k)
     return Events(n, ev["model"].data_ptr() if n else None, ev["req"].data_ptr() if n else None,
                   ev["t_s"].data_ptr() if n else None, ev["phase"].data_ptr() if n else None, nr,
                   ev["req_model"].data_ptr() if nr else None,
@@ -199,6 +219,12 @@ def events_struct(ev):
 
 
 def _counts(c):
+    n = int(c["P"].numel())
+    for k in ("P", "D", "A", "W"):
+        _need(c[k], "int32", n, k)
+    for k in ("A_ms", "W_ms"):
+        if c.get(k) is not None:
+            _need(c[k], "int64", n, k)
     occ = [c[k].data_ptr() if c.get(k) is not None else None for k in ("A_ms", "W_ms")]
     return Counts(*[c[k].data_ptr() for k in ("P", "D", "A", "W")], *occ)
 
@@ -276,8 +302,11 @@ def tss_class_models(model, cls, n_models, n_classes, out=None, stream=None):
     torch = _torch()
     lib = load()
     n = int(model.numel())
+    _need(model, "int32", None, "model")
+    _need(cls, "int32", n, "cls")
     if out is None:
         out = torch.empty(n, dtype=torch.int32, device=model.device)
+    _need(out, "int32", n, "out")
     _check("tss_class_models", lib.tss_class_models(C.c_int64(n), _ptr(model), _ptr(cls),
                                                     n_models, n_classes, _ptr(out),
                                                     _stream(stream)))
@@ -299,6 +328,7 @@ def tss_rank(Z, cls, window_ms=1000, recv=True, donors=True, stream=None):
     rv = torch.empty(K, dtype=torch.int32, device=Z.device) if recv else None
     dn = torch.empty((K, RANK_DONORS), dtype=torch.int32, device=Z.device) if donors else None
     Zc, cc = Z.contiguous(), cls.contiguous()
+    _need(cc, "uint8", K * M, "cls")
     _check("tss_rank", lib.tss_rank(C.byref(g), code, _ptr(Zc), _ptr(cc), _ptr(rv), _ptr(dn),
                                     _stream(stream)))
     return {"recv": rv, "donors": dn}

@@ -148,3 +148,21 @@ def test_class_models_arguments_are_checked_on_the_host():
     assert lib.tss_class_models(10, None, p, 8, 3, p, None) == 1
     assert lib.tss_class_models(0, None, None, 8, 3, None, None) == 0
 
+
+def test_binding_checks_tensor_arguments():
+    import torch
+    keys = ("model", "t_arr_ms", "t_start_ms", "t_first_ms", "t_end_ms", "L_in", "L_out")
+    good = {k: torch.zeros(5, dtype=torch.int32) for k in keys}
+    assert tre.requests_struct(good).n == 5
+    with pytest.raises(ValueError, match="int32"):
+        tre.requests_struct(dict(good, L_out=torch.zeros(5, dtype=torch.int64)))
+    with pytest.raises(ValueError, match="elements"):
+        tre.requests_struct(dict(good, t_end_ms=torch.zeros(4, dtype=torch.int32)))
+    with pytest.raises(ValueError, match="contiguous"):
+        tre.requests_struct(dict(good, t_arr_ms=torch.zeros(10, dtype=torch.int32)[::2]))
+    cnt = {k: torch.zeros((3, 2), dtype=torch.int32) for k in "PDAW"}
+    tre._counts(cnt)
+    with pytest.raises(ValueError, match="int64"):
+        tre._counts(dict(cnt, A_ms=torch.zeros((3, 2), dtype=torch.int32),
+                         W_ms=torch.zeros((3, 2), dtype=torch.int64)))
+
