@@ -457,34 +457,45 @@ int rank_windows(int32_t M, int32_t K, const T* Z, const uint8_t* cls, int32_t* 
   return 0;
 }
 
+// The controller of Sec. IV-B/IV-C, one control tick at a time: replica
+// state r (routable replicas per model), the idle pool, and the move list.
 template <class T>
-int select_moves(int32_t M, int32_t win, int32_t K, const T* Z, const uint8_t* cls,
-                 const T* tau_crit, const T* tau_surplus, int64_t budget, const int32_t* r_min,
-                 const int32_t* footprint, int32_t fast_ms, int32_t slow_ms, int32_t pacing_cap,
-                 int32_t* r_inout, Move* moves, int64_t cap, int64_t* n_moves) {
-  if (M < 1 || win < 1 || K < 0 || fast_ms < 1 || slow_ms < 1 || pacing_cap < 0) return 1;
-  std::vector<int64_t> r(M);
-  int64_t used = 0;
-  for (int32_t m = 0; m < M; ++m) {
-    if (r_inout[m] < 0 || footprint[m] < 1 || r_min[m] < 0) return 1;
-    r[m] = r_inout[m];
-    used += (int64_t)footprint[m] * r[m];
-  }
-  if (used > budget) return 1;
-  int64_t free_pool = budget - used;
+struct Controller {
+  int32_t M;
+  const T* tau_crit;
+  const T* tau_surplus;
+  const int32_t* r_min;
+  const int32_t* footprint;
+  int32_t pacing_cap;
+  std::vector<int64_t> r;
+  int64_t free_pool = 0;
+  Move* moves;
+  int64_t cap;
   int64_t nm = 0;
-  Walk<T> wk{M, nullptr, nullptr, tau_crit, tau_surplus, r_min, footprint};
-  auto emit = [&](int64_t k, int32_t recv, int32_t donor, int kind, int seq) {
+
+  // false on an inconsistent initial state (negative counts, footprints
+  // below one, more replicas than the budget holds)
+  bool init(int64_t budget, const int32_t* r0) {
+    r.assign(M, 0);
+    int64_t used = 0;
+    for (int32_t m = 0; m < M; ++m) {
+      if (r0[m] < 0 || footprint[m] < 1 || r_min[m] < 0) return false;
+      r[m] = r0[m];
+      used += (int64_t)footprint[m] * r[m];
+    }
+    if (used > budget) return false;
+    free_pool = budget - used;
+    return true;
+  }
+
+  void emit(int64_t k, int32_t recv, int32_t donor, int kind, int seq) {
     if (nm < cap) moves[nm] = Move{(int32_t)k, recv, donor, kind, seq};
     ++nm;
-  };
-  for (int64_t k = 0; k < K; ++k) {
-    const int64_t lo = k * (int64_t)win, hi = (k + 1) * (int64_t)win;
-    const bool fast = hi / fast_ms > lo / fast_ms;
-    const bool slow = hi / slow_ms > lo / slow_ms;
-    if (!fast && !slow) continue;
-    wk.Zk = Z + (size_t)k * M;
-    wk.ck = cls + (size_t)k * M;
+  }
+
+  // window k ends a fast and/or a slow tick; Zk, ck: that window's Z and class
+  void tick(int64_t k, const T* Zk, const uint8_t* ck, bool fast, bool slow) {
+    Walk<T> wk{M, Zk, ck, tau_crit, tau_surplus, r_min, footprint};
     int32_t recv = -1;
     int kind = 0;
     bool nom_above = false;
@@ -501,7 +512,7 @@ int select_moves(int32_t M, int32_t win, int32_t K, const T* Z, const uint8_t* c
         nom_above = true;
       }
     }
-    if (kind == 0) continue;
+    if (kind == 0) return;
     for (int32_t seq = 0; seq < pacing_cap; ++seq) {
       const int64_t need = footprint[recv];
       if (free_pool >= need) {                   // idle capacity first
@@ -530,9 +541,28 @@ int select_moves(int32_t M, int32_t win, int32_t K, const T* Z, const uint8_t* c
       for (int32_t d : rel) emit(k, recv, d, kind, seq);
     }
   }
-  for (int32_t m = 0; m < M; ++m) r_inout[m] = (int32_t)r[m];
-  *n_moves = nm;
-  return nm > cap ? 4 : 0;
+};
+
+// window k ends a tick of cadence c when a multiple of c falls in (k*win, (k+1)*win]
+inline bool ends_tick(int64_t k, int32_t win, int32_t c) {
+  return ((k + 1) * (int64_t)win) / c > (k * (int64_t)win) / c;
+}
+
+template <class T>
+int select_moves(int32_t M, int32_t win, int32_t K, const T* Z, const uint8_t* cls,
+                 const T* tau_crit, const T* tau_surplus, int64_t budget, const int32_t* r_min,
+                 const int32_t* footprint, int32_t fast_ms, int32_t slow_ms, int32_t pacing_cap,
+                 int32_t* r_inout, Move* moves, int64_t cap, int64_t* n_moves) {
+  if (M < 1 || win < 1 || K < 0 || fast_ms < 1 || slow_ms < 1 || pacing_cap < 0) return 1;
+  Controller<T> ctl{M, tau_crit, tau_surplus, r_min, footprint, pacing_cap, {}, 0, moves, cap};
+  if (!ctl.init(budget, r_inout)) return 1;
+  for (int64_t k = 0; k < K; ++k) {
+    const bool fast = ends_tick(k, win, fast_ms), slow = ends_tick(k, win, slow_ms);
+    if (fast || slow) ctl.tick(k, Z + (size_t)k * M, cls + (size_t)k * M, fast, slow);
+  }
+  for (int32_t m = 0; m < M; ++m) r_inout[m] = (int32_t)ctl.r[m];
+  *n_moves = ctl.nm;
+  return ctl.nm > cap ? 4 : 0;
 }
 
 }  // namespace
