@@ -236,6 +236,44 @@ def select_moves(Z, cls, tau_crit, tau_surplus, window_ms, budget, r0, r_min, fo
         return moves[: int(n[0])], rr, rc
 
 
+def closed_loop(lat, M, window_ms, K, profile, budget, r0, r_min, footprint, tau_crit,
+                tau_surplus, fast_ms=5000, slow_ms=10000, pacing_cap=1, dtype=np.float64,
+                cap=None):
+    """Closed-loop replay of latent requests (model, t_arr_ms, d_first_ms,
+    d_total_ms, L_in, L_out): the controller's moves change the servers, the
+    served requests make the telemetry it scores. profile holds w_p, w_q,
+    alpha, theta. Returns dict with the served records (t_start_ms, t_first_ms,
+    t_end_ms), moves, r_final, Z, cls."""
+    n = len(lat["model"])
+    pr = _prof(dict(profile, tau_crit=tau_crit, tau_surplus=tau_surplus), M, dtype)
+    out = {k: np.zeros(n, np.int32) for k in ("t_start_ms", "t_first_ms", "t_end_ms")}
+    Z = np.zeros((K, M), dtype)
+    cls = np.zeros((K, M), np.uint8)
+    r = np.zeros(M, np.int32)
+    cap = 1 << 16 if cap is None else cap
+    while True:
+        moves = np.zeros(cap, MOVE_DTYPE)
+        nm = np.zeros(1, np.int64)
+        f = getattr(lib(), "orc_closed_loop_" + _suffix(dtype))
+        rc = f(C.c_int32(M), C.c_int32(window_ms), C.c_int32(K), C.c_int64(n),
+               *[_p(_i32(lat[k])) for k in ("model", "t_arr_ms", "d_first_ms", "d_total_ms",
+                                            "L_in", "L_out")],
+               *[_p(pr[k]) for k in ("w_p", "w_q", "alpha", "theta", "tau_crit", "tau_surplus")],
+               C.c_int64(budget), _p(_i32(r0)), _p(_i32(r_min)), _p(_i32(footprint)),
+               C.c_int32(fast_ms), C.c_int32(slow_ms), C.c_int32(pacing_cap),
+               _p(out["t_start_ms"]), _p(out["t_first_ms"]), _p(out["t_end_ms"]), _p(r),
+               _p(moves), C.c_int64(cap), _p(nm), _p(Z), _p(cls))
+        if rc == 1:
+            raise ValueError("oracle: bad arguments")
+        if rc == 4:
+            cap = int(nm[0])
+            continue
+        break
+    rec = {"model": _i32(lat["model"]), "t_arr_ms": _i32(lat["t_arr_ms"]), **out,
+           "L_in": _i32(lat["L_in"]), "L_out": _i32(lat["L_out"])}
+    return {"records": rec, "moves": moves[: int(nm[0])], "r_final": r, "Z": Z, "cls": cls}
+
+
 def pipeline_requests(req, M, window_ms, K, profile, slo_ttft_ms, dtype, ok_frac=0.95,
                       reliability=0.95, mean_occupancy=False):
     """Reduce -> score (S) -> calibrate theta -> score (Z, class, receiver).

@@ -40,6 +40,8 @@
 #include <cmath>
 #include <cstdint>
 #include <cstring>
+#include <functional>
+#include <queue>
 #include <utility>
 #include <vector>
 
@@ -565,6 +567,117 @@ int select_moves(int32_t M, int32_t win, int32_t K, const T* Z, const uint8_t* c
   return ctl.nm > cap ? 4 : 0;
 }
 
+// --------------------------------------------------------------------------
+// Closed-loop replay: the controller's moves change the capacity that serves
+// the requests, and the telemetry it scores comes from the requests as they
+// are served. Readings:
+//  * each routable replica of a model is one server; a model's requests are
+//    served in input order (FCFS when sorted by arrival) by whichever server
+//    frees first; a request needs d_first ms to its first token and d_total
+//    ms to its last once started;
+//  * window k is processed at T = (k+1)*win: every request that starts before
+//    T is started first, then window k's telemetry (same attribution as
+//    reduce_requests) is scored (carry across windows) and, on a control
+//    tick, the controller acts with the replica counts as they are;
+//  * a replica added to a model is a server free at T; a replica taken from
+//    a model is the server that frees first (an idle one at once; a busy one
+//    finishes its request and is gone); no actuation delay;
+//  * a request not started by the end of the grid reports
+//    t_start = t_first = t_end = K*win; invalid latent records (model out of
+//    range, arrival outside [0, K*win), negative durations, d_first > d_total,
+//    L_in < 0, L_out < 1) are not served and report -1.
+// --------------------------------------------------------------------------
+template <class T>
+int closed_loop(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* model,
+                const int32_t* t_arr, const int32_t* d_first, const int32_t* d_total,
+                const int32_t* L_in, const int32_t* L_out, const T* w_p, const T* w_q,
+                const T* alpha, const T* theta, const T* tau_crit, const T* tau_surplus,
+                int64_t budget, const int32_t* r0, const int32_t* r_min, const int32_t* footprint,
+                int32_t fast_ms, int32_t slow_ms, int32_t pacing_cap, int32_t* t_start,
+                int32_t* t_first, int32_t* t_end, int32_t* r_out, Move* moves, int64_t cap,
+                int64_t* n_moves, T* Z_out, uint8_t* cls_out) {
+  if (M < 1 || win < 1 || K < 0 || n < 0 || fast_ms < 1 || slow_ms < 1 || pacing_cap < 0)
+    return 1;
+  const int64_t span = (int64_t)K * win;
+  Controller<T> ctl{M, tau_crit, tau_surplus, r_min, footprint, pacing_cap, {}, 0, moves, cap};
+  if (!ctl.init(budget, r0)) return 1;
+  using MinHeap = std::priority_queue<int64_t, std::vector<int64_t>, std::greater<int64_t>>;
+  std::vector<MinHeap> servers(M);
+  for (int32_t m = 0; m < M; ++m)
+    for (int64_t j = 0; j < ctl.r[m]; ++j) servers[m].push(0);
+  std::vector<std::vector<int64_t>> queue(M);
+  std::vector<size_t> head(M, 0);
+  std::vector<int64_t> arr_cnt((size_t)K * M, 0);     // arrivals per (window, model)
+  for (int64_t i = 0; i < n; ++i) {
+    t_start[i] = t_first[i] = t_end[i] = -1;
+    const int64_t m = model[i];
+    if (m < 0 || m >= M || t_arr[i] < 0 || t_arr[i] >= span) continue;
+    if (d_first[i] < 0 || d_total[i] < d_first[i] || L_in[i] < 0 || L_out[i] < 1) continue;
+    queue[m].push_back(i);
+    t_start[i] = t_first[i] = t_end[i] = (int32_t)span;   // until it starts
+    arr_cnt[(size_t)(t_arr[i] / win) * M + m] += 1;
+  }
+  // telemetry accumulated as requests start (windows at or after the current)
+  std::vector<uint32_t> P((size_t)K * M, 0), D((size_t)K * M, 0);
+  std::vector<int64_t> end_cnt((size_t)(K + 1) * M, 0);
+  std::vector<int64_t> cum_arr(M, 0), cum_start(M, 0), cum_end(M, 0);
+  std::vector<T> S_carry(M, (T)0), S_row(M), Z_row(M);
+  std::vector<uint8_t> init_carry(M, 0), cls_row(M);
+  std::vector<int32_t> Pk(M), Dk(M), Ak(M), Wk(M);
+  for (int64_t k = 0; k < K; ++k) {
+    const int64_t Tk = (k + 1) * (int64_t)win;
+    for (int32_t m = 0; m < M; ++m) {
+      while (head[m] < queue[m].size() && !servers[m].empty()) {
+        const int64_t i = queue[m][head[m]];
+        const int64_t st = std::max<int64_t>(t_arr[i], servers[m].top());
+        if (st >= Tk) break;
+        const int64_t tf = std::min<int64_t>(st + d_first[i], INT32_MAX);
+        const int64_t te = std::min<int64_t>(st + d_total[i], INT32_MAX);
+        servers[m].pop();
+        servers[m].push(st + d_total[i]);
+        ++head[m];
+        t_start[i] = (int32_t)st;
+        t_first[i] = (int32_t)tf;
+        t_end[i] = (int32_t)te;
+        cum_start[m] += 1;
+        // tokens and the end of the running span, as reduce_requests counts them
+        if (tf < span) P[(size_t)(tf / win) * M + m] += (uint32_t)L_in[i];
+        const int64_t L = L_out[i], dur = te - tf;
+        for (int64_t j = 0; j < L; ++j) {
+          const int64_t tj = (L == 1) ? tf : tf + (j * dur) / (L - 1);
+          if (tj < span) D[(size_t)(tj / win) * M + m] += 1u;
+        }
+        end_cnt[(size_t)win_of(te, win, K) * M + m] += 1;
+      }
+    }
+    for (int32_t m = 0; m < M; ++m) {
+      const size_t x = (size_t)k * M + m;
+      cum_arr[m] += arr_cnt[x];
+      cum_end[m] += end_cnt[x];
+      Pk[m] = (int32_t)P[x];
+      Dk[m] = (int32_t)D[x];
+      Ak[m] = (int32_t)(cum_start[m] - cum_end[m]);
+      Wk[m] = (int32_t)(cum_arr[m] - cum_start[m]);
+    }
+    score<T>(M, win, 1, Pk.data(), Dk.data(), Ak.data(), Wk.data(), w_p, w_q, alpha, theta,
+             tau_crit, tau_surplus, S_carry.data(), init_carry.data(), S_row.data(), Z_row.data(),
+             cls_row.data(), nullptr, nullptr, nullptr);
+    if (Z_out) std::copy(Z_row.begin(), Z_row.end(), Z_out + (size_t)k * M);
+    if (cls_out) std::copy(cls_row.begin(), cls_row.end(), cls_out + (size_t)k * M);
+    const bool fast = ends_tick(k, win, fast_ms), slow = ends_tick(k, win, slow_ms);
+    if (!fast && !slow) continue;
+    const std::vector<int64_t> before = ctl.r;
+    ctl.tick(k, Z_row.data(), cls_row.data(), fast, slow);
+    for (int32_t m = 0; m < M; ++m) {
+      for (int64_t j = before[m]; j < ctl.r[m]; ++j) servers[m].push(Tk);
+      for (int64_t j = ctl.r[m]; j < before[m]; ++j) servers[m].pop();
+    }
+  }
+  for (int32_t m = 0; m < M; ++m) r_out[m] = (int32_t)ctl.r[m];
+  *n_moves = ctl.nm;
+  return ctl.nm > cap ? 4 : 0;
+}
+
 }  // namespace
 
 extern "C" {
@@ -657,6 +770,23 @@ int orc_rank_f64(int32_t M, int32_t K, const double* Z, const uint8_t* cls, int3
                  int32_t* order) {
   return rank_windows<double>(M, K, Z, cls, recv, order);
 }
+
+#define ORC_CLOSED_LOOP(SUF, T)                                                                   \
+  int orc_closed_loop_##SUF(                                                                       \
+      int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* model, const int32_t* t_arr,    \
+      const int32_t* d_first, const int32_t* d_total, const int32_t* L_in, const int32_t* L_out,   \
+      const T* w_p, const T* w_q, const T* alpha, const T* theta, const T* tau_crit,               \
+      const T* tau_surplus, int64_t budget, const int32_t* r0, const int32_t* r_min,               \
+      const int32_t* footprint, int32_t fast_ms, int32_t slow_ms, int32_t pacing_cap,              \
+      int32_t* t_start, int32_t* t_first, int32_t* t_end, int32_t* r_out, Move* moves,             \
+      int64_t cap, int64_t* n_moves, T* Z_out, uint8_t* cls_out) {                                 \
+    return closed_loop<T>(M, win, K, n, model, t_arr, d_first, d_total, L_in, L_out, w_p, w_q,     \
+                          alpha, theta, tau_crit, tau_surplus, budget, r0, r_min, footprint,       \
+                          fast_ms, slow_ms, pacing_cap, t_start, t_first, t_end, r_out, moves,     \
+                          cap, n_moves, Z_out, cls_out);                                           \
+  }
+ORC_CLOSED_LOOP(f32, float)
+ORC_CLOSED_LOOP(f64, double)
 
 int orc_move_size(void) { return (int)sizeof(Move); }
 

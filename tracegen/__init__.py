@@ -145,8 +145,9 @@ def initial_replicas(spec: TraceSpec):
     return largest_remainder(load, spec.budget, floor=1)
 
 
-def gen_requests(spec: TraceSpec):
-    """Request records sorted by arrival. Returns dict of int32 columns + metadata."""
+def _draw(spec: TraceSpec):
+    """Per model: arrival times (s), prompt / output lengths, service times (s)
+    and prefill shares, from the spec's seeded generator; plus r0 and u."""
     rng = np.random.Generator(np.random.PCG64(spec.seed))
     M = spec.n_models
     scale = spec.n_target / _expected_count_unit(spec)
@@ -158,9 +159,7 @@ def gen_requests(spec: TraceSpec):
         u = spec.rho / max(lam[m] * spec.cost[m] * e_work[m] / r0[m] for m in range(M))
     else:
         u = spec.rho * r0.sum() / float((lam * spec.cost * e_work).sum())
-    cols = {k: [] for k in ("model", "t_arr_ms", "t_start_ms", "t_first_ms", "t_end_ms",
-                            "L_in", "L_out")}
-    arr_s = []
+    draws = []
     for m in range(M):
         rate, peak = _rate_fn(spec, m, scale)
         n_cand = rng.poisson(peak * spec.duration_s)
@@ -171,9 +170,67 @@ def gen_requests(spec: TraceSpec):
         L_in = _lengths(rng, spec.len_in[m][0], spec.len_in[m][1], n)
         L_out = _lengths(rng, spec.len_out[m][0], spec.len_out[m][1], n)
         svc = rng.exponential(u * spec.cost[m] * e_work[m], size=n)
-        start = _fcfs_starts(t, svc, int(r0[m]))
         pw = 0.2 * L_in
-        f = pw / (pw + L_out)
+        draws.append((t, L_in, L_out, svc, pw / (pw + L_out)))
+    return draws, r0, u
+
+
+def gen_latent(spec: TraceSpec):
+    """Inputs of a closed-loop replay, sorted by arrival: model, arrival (int ms),
+    L_in, L_out and the service a request needs once it starts -- whole
+    milliseconds to its first token (d_first) and to its last token (d_total;
+    equal to d_first when L_out = 1). Same draws as gen_requests."""
+    draws, r0, u = _draw(spec)
+    cols = {k: [] for k in ("model", "t_arr_ms", "d_first_ms", "d_total_ms", "L_in", "L_out")}
+    arr_s = []
+    for m, (t, L_in, L_out, svc, f) in enumerate(draws):
+        d_total = np.rint(svc * 1000.0).astype(np.int64)
+        d_first = np.minimum(np.rint(svc * f * 1000.0).astype(np.int64), d_total)
+        d_total = np.where(L_out == 1, d_first, d_total)
+        cols["model"].append(np.full(len(t), m, dtype=np.int32))
+        cols["t_arr_ms"].append(np.floor(t * 1000.0).astype(np.int64))
+        cols["d_first_ms"].append(d_first)
+        cols["d_total_ms"].append(d_total)
+        cols["L_in"].append(L_in)
+        cols["L_out"].append(L_out)
+        arr_s.append(t)
+    order = np.argsort(np.concatenate(arr_s), kind="stable")
+    out = {k: np.ascontiguousarray(np.concatenate(v)[order].astype(np.int32))
+           for k, v in cols.items()}
+    out["r0"] = r0
+    return out
+
+
+def fcfs_records(lat, M, r):
+    """Request records of latent requests served FCFS per model by r[m]
+    identical servers, all times in whole milliseconds (the open-loop queue)."""
+    n = len(lat["model"])
+    start = np.zeros(n, np.int64)
+    for m in range(M):
+        idx = np.flatnonzero(lat["model"] == m)
+        free = [0] * int(r[m])
+        heapq.heapify(free)
+        for i in idx:
+            a = int(lat["t_arr_ms"][i])
+            st = max(a, free[0])
+            start[i] = st
+            heapq.heapreplace(free, st + int(lat["d_total_ms"][i]))
+    return {"model": lat["model"].copy(), "t_arr_ms": lat["t_arr_ms"].copy(),
+            "t_start_ms": start.astype(np.int32),
+            "t_first_ms": (start + lat["d_first_ms"]).astype(np.int32),
+            "t_end_ms": (start + lat["d_total_ms"]).astype(np.int32),
+            "L_in": lat["L_in"].copy(), "L_out": lat["L_out"].copy()}
+
+
+def gen_requests(spec: TraceSpec):
+    """Request records sorted by arrival. Returns dict of int32 columns + metadata."""
+    draws, r0, u = _draw(spec)
+    cols = {k: [] for k in ("model", "t_arr_ms", "t_start_ms", "t_first_ms", "t_end_ms",
+                            "L_in", "L_out")}
+    arr_s = []
+    for m, (t, L_in, L_out, svc, f) in enumerate(draws):
+        n = len(t)
+        start = _fcfs_starts(t, svc, int(r0[m]))
         first = start + svc * f
         end = start + svc
         t_arr = np.floor(t * 1000.0).astype(np.int64)
