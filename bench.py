@@ -229,10 +229,11 @@ def cpu_baseline_parallel(scale, seed0):
     try:
         ctx = mp.get_context("spawn")
         with ctx.Pool(n_proc, initializer=_par_init, initargs=(scale, seed0)) as pool:
-            pool.map(_par_unit, [(0, 0)] * n_proc)          # workers up, traces generated
+            # bounded waits: a worker that dies must not stall the bench
+            pool.map_async(_par_unit, [(0, 0)] * n_proc).get(timeout=300)
             units = [(t, w) for t in range(7) for w in range(4)]
             t0 = time.perf_counter()
-            n_rec = sum(pool.map(_par_unit, units, chunksize=1))
+            n_rec = sum(pool.map_async(_par_unit, units, chunksize=1).get(timeout=300))
             dt = time.perf_counter() - t0
     except Exception as e:   # a baseline must not cost the bench line
         return {"error": f"{type(e).__name__}: {e}"}
