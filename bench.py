@@ -391,6 +391,11 @@ def main():
     K = [sw["duration_ms"] // int(w) for w in win]
     model_windows = sum(K) * len(sw["traces"]) * M
     n_inst = len(sw["traces"]) * len(win) * len(sw["tau_crit"]) * len(sw["pacing_cap"])
+    # prompt + output tokens of the step's records, and windows walked by all
+    # controller instances
+    tokens = int(sum(int(t["L_in"].astype(np.int64).sum() + t["L_out"].astype(np.int64).sum())
+                     for t in sw["traces"]))
+    inst_windows = len(sw["traces"]) * len(sw["tau_crit"]) * len(sw["pacing_cap"]) * sum(K)
     moves_cap = 512
     dev_traces = [{k: torch.as_tensor(v).cuda() for k, v in t.items()} for t in sw["traces"]]
     stream = torch.cuda.current_stream()
@@ -430,13 +435,16 @@ def main():
     lib.tre_trace_collect(C.byref(tr))
     lib.tre_trace_enable(0)
     clk = clocks.stop()
-    job_rec, job_mw, job_inst = total_rec, model_windows, n_inst
+    job_rec, job_mw, job_inst, job_tok, job_iw = (total_rec, model_windows, n_inst, tokens,
+                                                  inst_windows)
     if world > 1:
-        ms, (job_rec, job_mw, job_inst) = over_ranks(dist, "cuda", ms,
-                                                     [total_rec, model_windows, n_inst])
+        ms, (job_rec, job_mw, job_inst, job_tok, job_iw) = over_ranks(
+            dist, "cuda", ms, [total_rec, model_windows, n_inst, tokens, inst_windows])
     ms_step = ms / args.steps
     value = job_rec * args.steps / (ms / 1e3)
     mw_s = job_mw * args.steps / (ms / 1e3)
+    tok_s = job_tok * args.steps / (ms / 1e3)
+    iw_s = job_iw * args.steps / (ms / 1e3)
     phases = {tr.name[i].decode(): {"ms": tr.ms[i], "calls": tr.calls[i],
                                     "launches": tr.launches[i]} for i in range(tr.n_phases)}
     launches = int(sum(p["launches"] for p in phases.values()))
@@ -592,7 +600,8 @@ def main():
                        "controller_instances": int(job_inst), "scale": args.scale,
                        "l2": "inputs larger than L2 (7 x 28 B x ~1M records = 196 MB per step)",
                        "parallelism": f"independent sweeps per GPU x{world}"},
-            "model_windows_per_s": mw_s,
+            "model_windows_per_s": mw_s, "tokens_per_s": tok_s,
+            "instance_windows_per_s": iw_s,
             "roofline": roof, "step_roofline": whole, "phases_ms_per_step": {
                 k: p["ms"] / args.steps for k, p in phases.items() if p["calls"]},
             "phases_roofline": {k: round(roof_of(k)["frac"], 4) for k in pb
