@@ -274,6 +274,50 @@ def closed_loop(lat, M, window_ms, K, profile, budget, r0, r_min, footprint, tau
     return {"records": rec, "moves": moves[: int(nm[0])], "r_final": r, "Z": Z, "cls": cls}
 
 
+def slo_tpot_counts_requests(req, M, window_ms, K, tpot_ms):
+    """Per (arrival window, model): requests with L_out > 1 and how many met
+    (t_end - t_first) <= tpot_ms * (L_out - 1)."""
+    cols = _req_cols(req)
+    n_dec, n_met = np.zeros((K, M), np.int32), np.zeros((K, M), np.int32)
+    rc = lib().orc_slo_tpot_counts_requests(C.c_int32(M), C.c_int32(window_ms), C.c_int32(K),
+                                            C.c_int64(len(cols[0])), *[_p(c) for c in cols],
+                                            _p(_i32(tpot_ms)), _p(n_dec), _p(n_met))
+    if rc:
+        raise ValueError("oracle: bad arguments")
+    return n_dec, n_met
+
+
+def stage_gauges(req, M, window_ms, K):
+    """Running requests split at the first token, read at each window's last
+    millisecond: in prefill on [t_start, t_first) and decoding on
+    [t_first, t_end). Returns (A_prefill, A_decode)."""
+    A_p = reduce_requests(dict(req, t_end_ms=req["t_first_ms"]), M, window_ms, K)[2]
+    A_d = reduce_requests(dict(req, t_start_ms=req["t_first_ms"]), M, window_ms, K)[2]
+    return A_p, A_d
+
+
+def stage_pipeline(req, M, window_ms, K, profile, slo_ttft_ms, slo_tpot_ms, dtype,
+                   ok_frac=0.95, reliability=0.95):
+    """Stage-aware signal (separate prefill and decode states, Sec. VIII):
+    prefill TSS = (P/dt) / max(A_prefill + w_q*W, 1), calibrated on TTFT;
+    decode TSS = (D/dt) / max(A_decode, 1), calibrated on TPOT. Each stage is
+    smoothed, calibrated and normalised like the scalar signal."""
+    P, D, A, W, drops = reduce_requests(req, M, window_ms, K)
+    A_p, A_d = stage_gauges(req, M, window_ms, K)
+    zero = np.zeros_like(P)
+    n_arr, n_met = slo_counts_requests(req, M, window_ms, K, slo_ttft_ms)
+    n_dec, n_met_d = slo_tpot_counts_requests(req, M, window_ms, K, slo_tpot_ms)
+    out = {"A_prefill": A_p, "A_decode": A_d}
+    for stage, cnt, counts in (("prefill", (P, zero, A_p, W), (n_arr, n_met)),
+                               ("decode", (zero, D, A_d, zero), (n_dec, n_met_d))):
+        prof = dict(profile, w_p=1.0) if stage == "prefill" else dict(profile)
+        S, _, cls, _ = score(*cnt, prof, window_ms, dtype)
+        theta, deg = calibrate(S, cls, *counts, ok_frac, reliability)
+        S, Z, cls, _ = score(*cnt, dict(prof, theta=theta), window_ms, dtype)
+        out[stage] = {"S": S, "Z": Z, "cls": cls, "theta": theta, "degenerate": deg}
+    return out
+
+
 def pipeline_requests(req, M, window_ms, K, profile, slo_ttft_ms, dtype, ok_frac=0.95,
                       reliability=0.95, mean_occupancy=False):
     """Reduce -> score (S) -> calibrate theta -> score (Z, class, receiver).

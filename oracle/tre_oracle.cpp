@@ -170,6 +170,33 @@ int slo_counts_requests(int32_t M, int32_t win, int32_t K, int64_t n, const int3
   return 0;
 }
 
+// Decode-side SLO counts for a stage-aware signal (Sec. VIII: separate prefill
+// and decode states; Sec. III-A: decode determines TPOT): per (arrival window,
+// model) the requests with more than one output token and how many of them
+// met the model's TPOT bound, (t_end - t_first) <= tpot_ms * (L_out - 1)
+// (exact integer test). Records taken or skipped as in reduce_requests.
+int slo_tpot_counts_requests(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* model,
+                             const int32_t* t_arr, const int32_t* t_start,
+                             const int32_t* t_first, const int32_t* t_end, const int32_t* L_in,
+                             const int32_t* L_out, const int32_t* tpot_ms, int32_t* n_dec,
+                             int32_t* n_met) {
+  if (M < 1 || win < 1 || K < 0 || n < 0) return 1;
+  const int64_t span = (int64_t)K * win;
+  for (size_t x = 0; x < (size_t)K * M; ++x) n_dec[x] = n_met[x] = 0;
+  for (int64_t i = 0; i < n; ++i) {
+    const int64_t m = model[i];
+    if (m < 0 || m >= M) continue;
+    const int64_t ta = t_arr[i], ts = t_start[i], tf = t_first[i], te = t_end[i];
+    if (ta < 0 || ta >= span) continue;
+    if (!(ta <= ts && ts <= tf && tf <= te) || L_in[i] < 0 || L_out[i] < 1) continue;
+    if (L_out[i] < 2) continue;                      // no inter-token gap
+    const size_t x = (size_t)(ta / win) * M + m;
+    n_dec[x] += 1;
+    if (te - tf <= (int64_t)tpot_ms[m] * (L_out[i] - 1)) n_met[x] += 1;
+  }
+  return 0;
+}
+
 // --------------------------------------------------------------------------
 // Window reduction of token-level events (one record per emitted token).
 // --------------------------------------------------------------------------
@@ -697,6 +724,15 @@ int orc_occupancy_mean_requests(int32_t M, int32_t win, int32_t K, int64_t n,
                                 int64_t* A_ms, int64_t* W_ms) {
   return occupancy_mean_requests(M, win, K, n, model, t_arr, t_start, t_first, t_end, L_in, L_out,
                                  A_ms, W_ms);
+}
+
+int orc_slo_tpot_counts_requests(int32_t M, int32_t win, int32_t K, int64_t n,
+                                 const int32_t* model, const int32_t* t_arr,
+                                 const int32_t* t_start, const int32_t* t_first,
+                                 const int32_t* t_end, const int32_t* L_in, const int32_t* L_out,
+                                 const int32_t* tpot, int32_t* n_dec, int32_t* n_met) {
+  return slo_tpot_counts_requests(M, win, K, n, model, t_arr, t_start, t_first, t_end, L_in,
+                                  L_out, tpot, n_dec, n_met);
 }
 
 int orc_slo_counts_requests(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* model,
