@@ -501,6 +501,12 @@ struct Controller {
   Move* moves;
   int64_t cap;
   int64_t nm = 0;
+  // transitions of the last tick: receiver and the donor replicas it released
+  struct Transition {
+    int32_t recv;
+    std::vector<int32_t> donors;
+  };
+  std::vector<Transition> last;
 
   // false on an inconsistent initial state (negative counts, footprints
   // below one, more replicas than the budget holds)
@@ -524,6 +530,7 @@ struct Controller {
 
   // window k ends a fast and/or a slow tick; Zk, ck: that window's Z and class
   void tick(int64_t k, const T* Zk, const uint8_t* ck, bool fast, bool slow) {
+    last.clear();
     Walk<T> wk{M, Zk, ck, tau_crit, tau_surplus, r_min, footprint};
     int32_t recv = -1;
     int kind = 0;
@@ -548,6 +555,7 @@ struct Controller {
         free_pool -= need;
         r[recv] += 1;
         emit(k, recv, -1, kind, seq);
+        last.push_back({recv, {}});
         continue;
       }
       // release donors one replica at a time until the receiver's footprint
@@ -568,6 +576,7 @@ struct Controller {
       free_pool = f - need;
       r[recv] += 1;
       for (int32_t d : rel) emit(k, recv, d, kind, seq);
+      last.push_back({recv, rel});
     }
   }
 };
@@ -606,9 +615,15 @@ int select_moves(int32_t M, int32_t win, int32_t K, const T* Z, const uint8_t* c
 //    T is started first, then window k's telemetry (same attribution as
 //    reduce_requests) is scored (carry across windows) and, on a control
 //    tick, the controller acts with the replica counts as they are;
-//  * a replica added to a model is a server free at T; a replica taken from
-//    a model is the server that frees first (an idle one at once; a busy one
-//    finishes its request and is gone); no actuation delay;
+//  * a transition commits at its tick T (the controller's replica counts and
+//    pool change then); each donor replica it releases is the donor's server
+//    that frees first: it takes no request from T on, finishes the one it is
+//    serving (drain) and returns its GPU sleep_ms after that; the receiver's
+//    new replica starts waking when its GPU is free -- at T when the idle
+//    pool paid for it, else when the last of the transition's released
+//    donor replicas has returned its GPU -- and serves requests wake_ms
+//    later (Sec. VI-D measures sleep and wake; with both zero a drained
+//    donor's GPU passes straight to the receiver);
 //  * a request not started by the end of the grid reports
 //    t_start = t_first = t_end = K*win; invalid latent records (model out of
 //    range, arrival outside [0, K*win), negative durations, d_first > d_total,
@@ -620,10 +635,12 @@ int closed_loop(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* mod
                 const int32_t* L_in, const int32_t* L_out, const T* w_p, const T* w_q,
                 const T* alpha, const T* theta, const T* tau_crit, const T* tau_surplus,
                 int64_t budget, const int32_t* r0, const int32_t* r_min, const int32_t* footprint,
-                int32_t fast_ms, int32_t slow_ms, int32_t pacing_cap, int32_t* t_start,
-                int32_t* t_first, int32_t* t_end, int32_t* r_out, Move* moves, int64_t cap,
-                int64_t* n_moves, T* Z_out, uint8_t* cls_out) {
-  if (M < 1 || win < 1 || K < 0 || n < 0 || fast_ms < 1 || slow_ms < 1 || pacing_cap < 0)
+                int32_t fast_ms, int32_t slow_ms, int32_t pacing_cap, int32_t wake_ms,
+                int32_t sleep_ms, int32_t* t_start, int32_t* t_first, int32_t* t_end,
+                int32_t* r_out, Move* moves, int64_t cap, int64_t* n_moves, T* Z_out,
+                uint8_t* cls_out) {
+  if (M < 1 || win < 1 || K < 0 || n < 0 || fast_ms < 1 || slow_ms < 1 || pacing_cap < 0 ||
+      wake_ms < 0 || sleep_ms < 0)
     return 1;
   const int64_t span = (int64_t)K * win;
   Controller<T> ctl{M, tau_crit, tau_surplus, r_min, footprint, pacing_cap, {}, 0, moves, cap};
@@ -693,11 +710,15 @@ int closed_loop(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* mod
     if (cls_out) std::copy(cls_row.begin(), cls_row.end(), cls_out + (size_t)k * M);
     const bool fast = ends_tick(k, win, fast_ms), slow = ends_tick(k, win, slow_ms);
     if (!fast && !slow) continue;
-    const std::vector<int64_t> before = ctl.r;
     ctl.tick(k, Z_row.data(), cls_row.data(), fast, slow);
-    for (int32_t m = 0; m < M; ++m) {
-      for (int64_t j = before[m]; j < ctl.r[m]; ++j) servers[m].push(Tk);
-      for (int64_t j = ctl.r[m]; j < before[m]; ++j) servers[m].pop();
+    for (const auto& tr : ctl.last) {
+      int64_t gpu_free = Tk;                     // when the receiver's GPU is free
+      for (int32_t d : tr.donors) {
+        const int64_t drained = std::max<int64_t>(servers[d].top(), Tk);
+        servers[d].pop();
+        gpu_free = std::max<int64_t>(gpu_free, drained + sleep_ms);
+      }
+      servers[tr.recv].push(gpu_free + wake_ms);
     }
   }
   for (int32_t m = 0; m < M; ++m) r_out[m] = (int32_t)ctl.r[m];
@@ -814,12 +835,12 @@ int orc_rank_f64(int32_t M, int32_t K, const double* Z, const uint8_t* cls, int3
       const T* w_p, const T* w_q, const T* alpha, const T* theta, const T* tau_crit,               \
       const T* tau_surplus, int64_t budget, const int32_t* r0, const int32_t* r_min,               \
       const int32_t* footprint, int32_t fast_ms, int32_t slow_ms, int32_t pacing_cap,              \
-      int32_t* t_start, int32_t* t_first, int32_t* t_end, int32_t* r_out, Move* moves,             \
-      int64_t cap, int64_t* n_moves, T* Z_out, uint8_t* cls_out) {                                 \
+      int32_t wake_ms, int32_t sleep_ms, int32_t* t_start, int32_t* t_first, int32_t* t_end,       \
+      int32_t* r_out, Move* moves, int64_t cap, int64_t* n_moves, T* Z_out, uint8_t* cls_out) {    \
     return closed_loop<T>(M, win, K, n, model, t_arr, d_first, d_total, L_in, L_out, w_p, w_q,     \
                           alpha, theta, tau_crit, tau_surplus, budget, r0, r_min, footprint,       \
-                          fast_ms, slow_ms, pacing_cap, t_start, t_first, t_end, r_out, moves,     \
-                          cap, n_moves, Z_out, cls_out);                                           \
+                          fast_ms, slow_ms, pacing_cap, wake_ms, sleep_ms, t_start, t_first,       \
+                          t_end, r_out, moves, cap, n_moves, Z_out, cls_out);                      \
   }
 ORC_CLOSED_LOOP(f32, float)
 ORC_CLOSED_LOOP(f64, double)

@@ -8,9 +8,11 @@ acting on the capacity that serves the requests whose telemetry it scores).
   separately pinned batch functions gives the Z and classes the replay acted
   on, bit for bit, and the batch walk over them gives the replay's moves and
   final replicas -- so every decision used only telemetry complete at its tick;
-* the queue under changing capacity: a per-millisecond simulation (servers
-  added and removed at the tick times the moves give) starts every request at
-  the same millisecond;
+* the queue under changing capacity: a per-millisecond simulation (donor
+  servers taken and receiver servers given at the tick times the moves give,
+  with drain, sleep and wake delays) starts every request at the same
+  millisecond; with delays the decisions stay consistent with the served
+  records;
 * a hand-derived two-request case.
 """
 import numpy as np
@@ -70,30 +72,34 @@ def test_decisions_use_only_complete_telemetry(dtype, cap):
     np.testing.assert_array_equal(mv, o["moves"])
 
 
-def _per_ms_queue(lat, K, r0, moves):
-    """Start times by stepping through every millisecond: at a tick time the
-    capacity changes first (a new server is free at once; a removed one is the
-    server that frees first), then queued requests take free servers."""
+def _per_ms_queue(lat, K, r0, moves, wake=0, sleep=0):
+    """Start times by stepping through every millisecond. At a tick time each
+    transition first takes its released donor replicas (each the donor's
+    server that frees first; its GPU returns `sleep` ms after it drains), then
+    gives the receiver a server that frees `wake` ms after the GPU it needs is
+    free (at the tick when the idle pool paid for it). Then queued requests
+    take free servers."""
     span = K * WIN
-    delta = {}                       # tick time -> [(model, +1 / -1)]
-    transitions = set()
+    trans = {}                                   # (window, seq) -> [recv, donors]
     for mv in moves:
-        t = (int(mv["window"]) + 1) * WIN
-        if int(mv["donor"]) >= 0:    # each released donor replica
-            delta.setdefault(t, []).append((int(mv["donor"]), -1))
         key = (int(mv["window"]), int(mv["seq"]))
-        if key not in transitions:   # one receiver replica per transition
-            transitions.add(key)
-            delta.setdefault(t, []).append((int(mv["recv"]), +1))
+        t = trans.setdefault(key, [int(mv["recv"]), []])
+        if int(mv["donor"]) >= 0:
+            t[1].append(int(mv["donor"]))
+    at = {}
+    for (w, sq) in sorted(trans):
+        at.setdefault((w + 1) * WIN, []).append(trans[(w, sq)])
     busy = [[0] * int(r0[m]) for m in range(M)]
     queues = [list(np.flatnonzero(lat["model"] == m)) for m in range(M)]
     start = np.full(len(lat["model"]), span, np.int64)
     for t in range(span):
-        for m, d in delta.get(t, []):
-            if d > 0:
-                busy[m].append(t)
-            else:
-                busy[m].remove(min(busy[m]))
+        for recv, donors in at.get(t, []):
+            gpu = t
+            for d in donors:
+                b = min(busy[d])
+                busy[d].remove(b)
+                gpu = max(gpu, max(b, t) + sleep)
+            busy[recv].append(gpu + wake)
         for m in range(M):
             q = queues[m]
             while q and lat["t_arr_ms"][q[0]] <= t:
@@ -106,13 +112,34 @@ def _per_ms_queue(lat, K, r0, moves):
     return start
 
 
-def test_queue_under_changing_capacity_matches_per_millisecond_stepping():
+@pytest.mark.parametrize("wake,sleep", [(0, 0), (1310, 1870), (40, 0)])
+def test_queue_under_changing_capacity_matches_per_millisecond_stepping(wake, sleep):
     lat, K = _latent(0.002, 8, 240.0)
-    o = _run(lat, K, 2)
+    o = oracle.closed_loop(lat, M, WIN, K, _prof(np.full(M, 3.0)), 64, lat["r0"],
+                           np.ones(M, np.int32), np.ones(M, np.int32), 0.8, 1.2, pacing_cap=2,
+                           wake_ms=wake, sleep_ms=sleep)
     assert len(o["moves"]) > 0
     got = o["records"]["t_start_ms"]
-    want = _per_ms_queue(lat, K, lat["r0"], o["moves"])
+    want = _per_ms_queue(lat, K, lat["r0"], o["moves"], wake, sleep)
     np.testing.assert_array_equal(got, want)
+
+
+def test_actuation_delays_keep_decisions_consistent_with_the_served_records():
+    lat, K = _latent(0.01, 9, 900.0)
+    o = oracle.closed_loop(lat, M, WIN, K, _prof(np.full(M, 3.0)), 64, lat["r0"],
+                           np.ones(M, np.int32), np.ones(M, np.int32), 0.8, 1.2, pacing_cap=2,
+                           wake_ms=1310, sleep_ms=1870)
+    P, D, A, W, _ = oracle.reduce_requests(o["records"], M, WIN, K)
+    prof = dict(_prof(np.full(M, 3.0)), tau_crit=0.8, tau_surplus=1.2)
+    _, Z, cls, _ = oracle.score(P, D, A, W, prof, WIN, np.float64)
+    np.testing.assert_array_equal(Z, o["Z"])
+    mv, rf, _ = oracle.select_moves(Z, cls, 0.8, 1.2, WIN, 64, lat["r0"], np.ones(M),
+                                    np.ones(M), pacing_cap=2)
+    np.testing.assert_array_equal(mv, o["moves"])
+    # the delays hold capacity back: the served queue is not the immediate one
+    o0 = oracle.closed_loop(lat, M, WIN, K, _prof(np.full(M, 3.0)), 64, lat["r0"],
+                            np.ones(M, np.int32), np.ones(M, np.int32), 0.8, 1.2, pacing_cap=2)
+    assert not np.array_equal(o0["records"]["t_start_ms"], o["records"]["t_start_ms"])
 
 
 def test_hand_case():
