@@ -109,3 +109,77 @@ def test_walk_against_key_enumeration(w):
            for x in mv]
     assert got == want
     assert rf.tolist() == r_want
+
+
+@st.composite
+def calibration_cases(draw):
+    K = draw(st.integers(0, 25))
+    M = draw(st.integers(1, 3))
+    levels = [0.0, 0.25, 0.5, 1.0, 1.5, 2.0, 3.0]
+    S = np.array([[draw(st.sampled_from(levels)) for _ in range(M)] for _ in range(K)],
+                 np.float64).reshape(K, M)
+    cls = np.array([[draw(st.sampled_from([1, 1, 3])) for _ in range(M)] for _ in range(K)],
+                   np.uint8).reshape(K, M)
+    n_arr = np.array([[draw(st.integers(0, 6)) for _ in range(M)] for _ in range(K)],
+                     np.int32).reshape(K, M)
+    n_met = np.array([[draw(st.integers(0, int(a))) for a in row] for row in n_arr],
+                     np.int32).reshape(K, M)
+    ok_frac = draw(st.sampled_from([0.5, 0.95, 1.0]))
+    rho = draw(st.sampled_from([0.5, 0.8, 0.95, 1.0]))
+    return S, cls, n_arr, n_met, ok_frac, rho
+
+
+@settings(max_examples=200, deadline=None)
+@given(calibration_cases())
+def test_theta_against_brute_force(case):
+    from tests.test_oracle_calibrate import _brute_theta
+    S, cls, n_arr, n_met, ok_frac, rho = case
+    theta, deg = oracle.calibrate(S, cls, n_arr, n_met, ok_frac, rho)
+    want, wdeg = _brute_theta(S, cls, n_arr, n_met, ok_frac, rho)
+    np.testing.assert_array_equal(theta, want)
+    assert deg == wdeg
+
+
+@st.composite
+def latent_cases(draw):
+    M = draw(st.integers(1, 3))
+    K = draw(st.integers(1, 12))
+    n = draw(st.integers(0, 10))
+    rows = []
+    for _ in range(n):
+        d_total = draw(st.integers(0, 9000))
+        rows.append((draw(st.integers(0, M - 1)), draw(st.integers(0, K * 1000 - 1)),
+                     draw(st.integers(0, d_total)), d_total, draw(st.integers(0, 30)),
+                     draw(st.integers(1, 6))))
+    rows.sort(key=lambda r: r[1])
+    cols = list(zip(*rows)) if rows else [[]] * 6
+    lat = {k: np.array(v, np.int32) for k, v in zip(
+        ("model", "t_arr_ms", "d_first_ms", "d_total_ms", "L_in", "L_out"), cols)}
+    r0 = [draw(st.integers(0, 2)) for _ in range(M)]
+    budget = sum(r0) + draw(st.integers(0, 1))
+    Kp = draw(st.integers(0, 2))
+    wake = draw(st.sampled_from([0, 700]))
+    sleep = draw(st.sampled_from([0, 1200]))
+    theta = draw(st.sampled_from([0.5, 5.0, 50.0]))
+    return M, K, lat, r0, budget, Kp, wake, sleep, theta
+
+
+@settings(max_examples=60, deadline=None)
+@given(latent_cases())
+def test_closed_loop_against_batch_rescoring(case):
+    # decisions use only telemetry complete at their tick, with any delays
+    M, K, lat, r0, budget, Kp, wake, sleep, theta = case
+    prof = {"w_p": 0.2, "w_q": 2.0, "alpha": 0.5, "theta": np.full(M, theta)}
+    o = oracle.closed_loop(lat, M, 1000, K, prof, budget, r0, np.zeros(M, np.int32),
+                           np.ones(M, np.int32), 0.8, 1.2, pacing_cap=Kp, wake_ms=wake,
+                           sleep_ms=sleep)
+    P, D, A, W, drops = oracle.reduce_requests(o["records"], M, 1000, K)
+    assert drops.sum() == 0
+    _, Z, cls, _ = oracle.score(P, D, A, W, dict(prof, tau_crit=0.8, tau_surplus=1.2), 1000,
+                                np.float64)
+    np.testing.assert_array_equal(Z, o["Z"])
+    np.testing.assert_array_equal(cls, o["cls"])
+    mv, rf, _ = oracle.select_moves(Z, cls, 0.8, 1.2, 1000, budget, r0, np.zeros(M),
+                                    np.ones(M), pacing_cap=Kp)
+    np.testing.assert_array_equal(mv, o["moves"])
+    np.testing.assert_array_equal(rf, o["r_final"])
