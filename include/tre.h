@@ -9,9 +9,13 @@
  *   - raw Token Service Share (Eq. 1), its exponential smoothing (Sec. III-B),
  *     Z = TSS / theta (Eq. 2) and the critical / nominal / surplus regions,
  *   - the SLO calibration of the healthy boundary theta (Sec. III-B),
+ *   - the per-window Eq. 3 receiver and donor release order (Sec. IV-B),
  *   - the open-loop rescue / rebalance move selection with bounded pairwise
  *     transfer under a fixed replica budget (Sec. IV-B, Eq. 3, Sec. IV-C),
- *   - and a batched sweep of all of the above over many traces and settings.
+ *   - a batched sweep of all of the above over many traces and settings,
+ *   - and, beside the paper's signal: the time-averaged occupancy variant of
+ *     Eq. 1's demand term, per-(model, SLO class) scoring through pair ids,
+ *     and a scoring entry point that needs no workspace.
  *
  * Conventions (every entry point):
  *   - Array arguments are DEVICE pointers owned by the caller, unless a field
