@@ -334,6 +334,42 @@ def tss_rank(Z, cls, window_ms=1000, recv=True, donors=True, stream=None):
     return {"recv": rv, "donors": dn}
 
 
+def tss_stage_gauges(M, window_ms, K, requests, stream=None):
+    """Running requests split at the first token, read at each window's last
+    millisecond: (A_prefill, A_decode) int32 [K][M]. Two reductions of the same
+    columns, with t_first passed as t_end (prefill: [t_start, t_first)) and as
+    t_start (decode: [t_first, t_end)); only their running gauges are kept."""
+    pre = tss_window_reduce(M, window_ms, K, requests=dict(requests,
+                                                           t_end_ms=requests["t_first_ms"]),
+                            stream=stream)
+    dec = tss_window_reduce(M, window_ms, K, requests=dict(requests,
+                                                           t_start_ms=requests["t_first_ms"]),
+                            stream=stream)
+    return pre["A"], dec["A"]
+
+
+def stage_counts(counts, A_prefill, A_decode):
+    """Inputs of the two stage signals: prefill (P, no decode tokens, A_prefill,
+    W) and decode (no prompt tokens, D, A_decode, nothing waiting)."""
+    torch = _torch()
+    zero = torch.zeros_like(counts["P"])
+    return ({"P": counts["P"], "D": zero, "A": A_prefill, "W": counts["W"]},
+            {"P": zero, "D": counts["D"], "A": A_decode, "W": zero})
+
+
+def tss_stage_score(counts, A_prefill, A_decode, profile, window_ms, theta_prefill,
+                    theta_decode, dtype="f32", stream=None):
+    """Stage-aware signal: prefill TSS = (P/dt) / max(A_prefill + w_q W, 1) and
+    decode TSS = (D/dt) / max(A_decode, 1), each smoothed and normalised by its
+    own theta. Returns (prefill, decode) dicts as tss_score does."""
+    pre, dec = stage_counts(counts, A_prefill, A_decode)
+    p = tss_score(pre, dict(profile, w_p=1.0, theta=theta_prefill), window_ms, dtype=dtype,
+                  stream=stream)
+    d = tss_score(dec, dict(profile, theta=theta_decode), window_ms, dtype=dtype,
+                  stream=stream)
+    return p, d
+
+
 def tss_calibrate(counts, profile, window_ms, slo_ttft_ms, requests=None, events=None,
                   dtype="f32", ok_frac=0.95, reliability=0.95, diag=None, stream=None):
     """theta per model (CUDA tensor of dtype)."""

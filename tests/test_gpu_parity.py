@@ -421,6 +421,30 @@ def test_per_class_pipeline(tre, dtype):
         np.testing.assert_array_equal(_np(sc[k]), o[k], err_msg=k)
 
 
+@pytest.mark.parametrize("dtype", ["f32", "f64"])
+def test_stage_signal(tre, dtype):
+    w = tracegen.workload("mid", scale=0.02)
+    M, win, K = w["M"], w["window_ms"], w["K"]
+    npdt = np.float32 if dtype == "f32" else np.float64
+    prof = tracegen.default_profile(M, win)
+    tpot = np.full(M, 60, np.int32)
+    o = oracle.stage_pipeline(w["requests"], M, win, K, prof, w["slo_ttft_ms"], tpot, npdt)
+    req = _cuda(w["requests"])
+    A_p, A_d = tre.tss_stage_gauges(M, win, K, req)
+    np.testing.assert_array_equal(_np(A_p), o["A_prefill"])
+    np.testing.assert_array_equal(_np(A_d), o["A_decode"])
+    c = tre.tss_window_reduce(M, win, K, requests=req)
+    pre, _ = tre.stage_counts(c, A_p, A_d)
+    theta_p = tre.tss_calibrate(pre, dict(prof, w_p=1.0), win, w["slo_ttft_ms"], requests=req,
+                                dtype=dtype)
+    np.testing.assert_array_equal(_np(theta_p), o["prefill"]["theta"])
+    sp, sd = tre.tss_stage_score(c, A_p, A_d, prof, win, theta_p, o["decode"]["theta"],
+                                 dtype=dtype)
+    for k in ("S", "Z", "cls"):
+        np.testing.assert_array_equal(_np(sp[k]), o["prefill"][k], err_msg="prefill " + k)
+        np.testing.assert_array_equal(_np(sd[k]), o["decode"][k], err_msg="decode " + k)
+
+
 def test_calibrate_events(tre):
     w = _events_case(6)
     ev, M, win, K = w["events"], w["M"], w["window_ms"], w["K"]
