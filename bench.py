@@ -196,6 +196,21 @@ def run_reference(args):
         "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}))
 
 
+def host_cpu():
+    """The host's CPU model and core count, as lscpu reports them (for the CPU
+    baselines)."""
+    info = {"nproc": os.cpu_count()}
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            k, _, v = line.partition(":")
+            if k.strip() in ("Model name", "Architecture", "Vendor ID"):
+                info[k.strip().lower().replace(" ", "_")] = v.strip()
+    except Exception:
+        pass
+    return info
+
+
 def cpu_baseline(scale):
     import oracle
     sw = tracegen.sweep_workload(scale=scale, n_traces=1)
@@ -600,6 +615,7 @@ def main():
     base = base_par = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         base = cpu_baseline(args.scale)
+        base["host"] = host_cpu()
         next_rows["occupancy_mean"]["cpu_baseline"] = occupancy_cpu(args.scale)
         base_par = cpu_baseline_parallel(args.scale, rank_seed0(rank))
     if rank == 0:
