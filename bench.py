@@ -434,7 +434,7 @@ def main():
                          sw["slo_ttft_ms"], sw["budget"], sw["r0"], sw["r_min"], sw["footprint"],
                          dtype="f32", moves_cap=moves_cap)
 
-    def step(traces=None, ws=None):
+    def step():
         return plan.run(stream)
 
     for _ in range(args.warmup):
