@@ -556,6 +556,41 @@ def test_select_unit_footprints_small_and_large_budgets(tre, M, r_each, extra, c
     assert tre.read_diag(diag)["err"] == 0
 
 
+@pytest.mark.parametrize("cap", [1, 3])
+def test_select_and_rank_on_threshold_values_and_ties(tre, cap):
+    # Z exactly at tau_crit (0.8), tau_surplus (1.2) and the rebalance bound (1),
+    # with ties across models: every comparison is strict on both sides
+    import torch
+    rng = np.random.default_rng(61 + cap)
+    K, M, win = 3000, 6, 1000
+    Z = rng.choice(np.array([0.5, 0.8, 0.8, 1.0, 1.0, 1.2, 1.2, 1.5]), (K, M)).astype(np.float32)
+    cls = np.where(rng.random((K, M)) < 0.1, oracle.IDLE, oracle.NOM).astype(np.uint8)
+    r0 = np.array([3, 2, 2, 4, 1, 3], np.int32)
+    budget = int(r0.sum()) + 1
+    r_min = np.array([1, 0, 1, 0, 0, 1], np.int32)
+    g = np.ones(M, np.int32)
+    prof = {"w_p": 0.2, "w_q": 2.0, "alpha": 0.2, "theta": 1.0, "tau_crit": 0.8,
+            "tau_surplus": 1.2}
+    om, orf, _ = oracle.select_moves(Z, cls, 0.8, 1.2, win, budget, r0, r_min, g, 5000, 10000,
+                                     cap)
+    Zc, Cc = torch.as_tensor(Z).cuda(), torch.as_tensor(cls).cuda()
+    mv, rf, n, _ = tre.tre_select_moves(Zc, Cc, prof, win, budget, r0, r_min, g,
+                                        pacing_cap=cap, moves_cap=len(om) + 5)
+    assert n == len(om) and n > 0
+    np.testing.assert_array_equal(_np(rf), orf)
+    got = np.stack([mv[f].astype(np.int32) for f in ("window", "recv", "donor", "kind", "seq")], 1)
+    ref = np.stack([om[f] for f in ("window", "recv", "donor", "kind", "seq")], 1)
+    np.testing.assert_array_equal(got, ref)
+    # the per-window ranking on classes from the same thresholds
+    reg = np.where(cls == oracle.IDLE, oracle.IDLE,
+                   np.where(Z < np.float32(0.8), oracle.CRIT,
+                            np.where(Z > np.float32(1.2), oracle.SURP, oracle.NOM))).astype(np.uint8)
+    orv, odn = oracle.rank(Z, reg)
+    rk = tre.tss_rank(Zc, torch.as_tensor(reg).cuda(), win)
+    np.testing.assert_array_equal(_np(rk["recv"]), orv)
+    np.testing.assert_array_equal(_np(rk["donors"]), odn)
+
+
 def _sweep_case(scale, n_traces, duration_s):
     sw = tracegen.sweep_workload(scale=scale, n_traces=n_traces, duration_s=duration_s)
     alpha = [min(1.0, w / 5000.0) for w in sw["window_ms"]]
