@@ -592,7 +592,7 @@ int select_moves(int32_t M, int32_t win, int32_t K, const T* Z, const uint8_t* c
                  const int32_t* footprint, int32_t fast_ms, int32_t slow_ms, int32_t pacing_cap,
                  int32_t* r_inout, Move* moves, int64_t cap, int64_t* n_moves) {
   if (M < 1 || win < 1 || K < 0 || fast_ms < 1 || slow_ms < 1 || pacing_cap < 0) return 1;
-  Controller<T> ctl{M, tau_crit, tau_surplus, r_min, footprint, pacing_cap, {}, 0, moves, cap};
+  Controller<T> ctl{M, tau_crit, tau_surplus, r_min, footprint, pacing_cap, {}, 0, moves, cap, 0, {}};
   if (!ctl.init(budget, r_inout)) return 1;
   for (int64_t k = 0; k < K; ++k) {
     const bool fast = ends_tick(k, win, fast_ms), slow = ends_tick(k, win, slow_ms);
@@ -643,7 +643,7 @@ int closed_loop(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* mod
       wake_ms < 0 || sleep_ms < 0)
     return 1;
   const int64_t span = (int64_t)K * win;
-  Controller<T> ctl{M, tau_crit, tau_surplus, r_min, footprint, pacing_cap, {}, 0, moves, cap};
+  Controller<T> ctl{M, tau_crit, tau_surplus, r_min, footprint, pacing_cap, {}, 0, moves, cap, 0, {}};
   if (!ctl.init(budget, r0)) return 1;
   using MinHeap = std::priority_queue<int64_t, std::vector<int64_t>, std::greater<int64_t>>;
   std::vector<MinHeap> servers(M);
