@@ -131,6 +131,24 @@ def reduce_events(ev, M, window_ms, K):
     return P, D, A, W, drops
 
 
+def occupancy_mean_events(ev, M, window_ms, K):
+    """Time-averaged occupancy of token events: request-milliseconds running
+    (first to last valid event) and waiting (arrival to first event) per window.
+    int64 [K, M]."""
+    model, req = _i32(ev["model"]), _i32(ev["req"])
+    t_s = np.ascontiguousarray(ev["t_s"], dtype=np.float32)
+    phase = np.ascontiguousarray(ev["phase"], dtype=np.uint8)
+    rm, rta = _i32(ev["req_model"]), _i32(ev["req_t_arr_ms"])
+    A_ms, W_ms = np.zeros((K, M), np.int64), np.zeros((K, M), np.int64)
+    rc = lib().orc_occupancy_mean_events(C.c_int32(M), C.c_int32(window_ms), C.c_int32(K),
+                                         C.c_int64(len(model)), _p(model), _p(req), _p(t_s),
+                                         _p(phase), C.c_int64(len(rm)), _p(rm), _p(rta),
+                                         _p(A_ms), _p(W_ms))
+    if rc:
+        raise ValueError("oracle: bad arguments")
+    return A_ms, W_ms
+
+
 def slo_counts_events(ev, M, window_ms, K, slo_ttft_ms):
     rm, rta, rtt = _i32(ev["req_model"]), _i32(ev["req_t_arr_ms"]), _i32(ev["req_ttft_ms"])
     n_arr, n_met = np.zeros((K, M), np.int32), np.zeros((K, M), np.int32)

@@ -248,6 +248,46 @@ int reduce_events(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* m
   return 0;
 }
 
+// Time-averaged occupancy of token events: a request runs from its first to
+// its last valid event and waits from its arrival to its first event (the
+// spans reduce_events reads at each window's last millisecond); per (window,
+// model) the request-milliseconds of each span inside the window. Events and
+// requests are taken or skipped by reduce_events' rules (nothing is counted).
+int occupancy_mean_events(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* model,
+                          const int32_t* req, const float* t_s, const uint8_t* phase,
+                          int64_t n_req, const int32_t* req_model, const int32_t* req_t_arr,
+                          int64_t* A_ms, int64_t* W_ms) {
+  if (M < 1 || win < 1 || K < 0 || n < 0 || n_req < 0) return 1;
+  const int64_t span = (int64_t)K * win;
+  for (size_t x = 0; x < (size_t)K * M; ++x) A_ms[x] = W_ms[x] = 0;
+  std::vector<int64_t> first((size_t)n_req, INT64_MAX), last((size_t)n_req, -1);
+  for (int64_t i = 0; i < n; ++i) {
+    const int64_t m = model[i], r = req[i];
+    if (m < 0 || m >= M || r < 0 || r >= n_req || req_model[r] != m) continue;
+    const double ms = std::floor((double)t_s[i] * 1000.0);
+    if (!(ms >= 0.0 && ms < (double)span) || phase[i] > 1) continue;
+    const int64_t t = (int64_t)ms;
+    if (t < first[r]) first[r] = t;
+    if (t > last[r]) last[r] = t;
+  }
+  auto add_span = [&](int64_t a, int64_t e, int64_t m, int64_t* out) {
+    if (e > span) e = span;
+    if (a >= e) return;
+    for (int64_t k = a / win; k * win < e; ++k) {
+      const int64_t lo = std::max(a, k * win), hi = std::min(e, (k + 1) * win);
+      out[(size_t)k * M + m] += hi - lo;
+    }
+  };
+  for (int64_t r = 0; r < n_req; ++r) {
+    if (last[r] < 0) continue;
+    const int64_t m = req_model[r], ta = req_t_arr[r];
+    if (!(ta >= 0 && ta <= first[r])) continue;
+    add_span(first[r], last[r], m, A_ms);
+    add_span(ta, first[r], m, W_ms);
+  }
+  return 0;
+}
+
 int slo_counts_events(int32_t M, int32_t win, int32_t K, int64_t n_req, const int32_t* req_model,
                       const int32_t* req_t_arr, const int32_t* req_ttft,
                       const int32_t* slo_ttft_ms, int32_t* n_arr, int32_t* n_met) {
@@ -754,6 +794,14 @@ int orc_slo_tpot_counts_requests(int32_t M, int32_t win, int32_t K, int64_t n,
                                  const int32_t* tpot, int32_t* n_dec, int32_t* n_met) {
   return slo_tpot_counts_requests(M, win, K, n, model, t_arr, t_start, t_first, t_end, L_in,
                                   L_out, tpot, n_dec, n_met);
+}
+
+int orc_occupancy_mean_events(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* model,
+                              const int32_t* req, const float* t_s, const uint8_t* phase,
+                              int64_t n_req, const int32_t* req_model, const int32_t* req_t_arr,
+                              int64_t* A_ms, int64_t* W_ms) {
+  return occupancy_mean_events(M, win, K, n, model, req, t_s, phase, n_req, req_model, req_t_arr,
+                               A_ms, W_ms);
 }
 
 int orc_slo_counts_requests(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* model,

@@ -143,3 +143,45 @@ def test_dropped_records_add_nothing():
     assert drops.sum() == 30
     np.testing.assert_array_equal(np.stack(oracle.occupancy_mean_requests(both, M, win, K)),
                                   np.stack(oracle.occupancy_mean_requests(good, M, win, K)))
+
+
+def _events_case(seed, scale=0.002):
+    import tracegen
+    return tracegen.workload("stream", scale=scale, seed=seed)
+
+
+def test_events_one_millisecond_windows_equal_the_sampled_gauges():
+    # with 1 ms windows the window mean is the count at its only millisecond
+    w = _events_case(5)
+    ev, M = w["events"], w["M"]
+    K = 20000                                   # the first 20 s, 1 ms windows
+    _, _, A, W, _ = oracle.reduce_events(ev, M, 1, K)
+    A_ms, W_ms = oracle.occupancy_mean_events(ev, M, 1, K)
+    np.testing.assert_array_equal(A_ms, A)
+    np.testing.assert_array_equal(W_ms, W)
+
+
+def test_events_against_per_millisecond_membership():
+    w = _events_case(6)
+    ev, M = w["events"], w["M"]
+    win, K = 250, 60
+    span = win * K
+    A_ms, W_ms = oracle.occupancy_mean_events(ev, M, win, K)
+    # spans from the valid events of each request (numpy group min / max)
+    t = np.floor(ev["t_s"].astype(np.float64) * 1000.0)
+    ok = (t >= 0) & (t < span) & (ev["phase"] <= 1) & (ev["model"] == ev["req_model"][ev["req"]])
+    n_req = len(ev["req_model"])
+    first = np.full(n_req, np.iinfo(np.int64).max)
+    last = np.full(n_req, -1)
+    np.minimum.at(first, ev["req"][ok], t[ok].astype(np.int64))
+    np.maximum.at(last, ev["req"][ok], t[ok].astype(np.int64))
+    run = np.zeros((span, M), np.int64)
+    wait = np.zeros((span, M), np.int64)
+    for r in np.flatnonzero(last >= 0):
+        m, ta = ev["req_model"][r], ev["req_t_arr_ms"][r]
+        if not (0 <= ta <= first[r]):
+            continue
+        run[first[r]:last[r], m] += 1
+        wait[ta:min(first[r], span), m] += 1
+    np.testing.assert_array_equal(A_ms, run.reshape(K, win, M).sum(axis=1))
+    np.testing.assert_array_equal(W_ms, wait.reshape(K, win, M).sum(axis=1))
