@@ -270,7 +270,9 @@ tre_status tre_select_moves(const tre_grid* grid, const void* Z, const uint8_t* 
  * Limit: n_windows * n_models <= 1048576 (for example 36000 windows x 8 models
  * or 16384 x 64); larger problems return TRE_ENOMEM before anything is
  * enqueued. The first call on a device
- * looks up the buffer's device address (make it before any stream capture).
+ * looks up the buffer's device address (make it before any stream capture);
+ * the address is kept for the life of the process, so do not call this entry
+ * point on a device after cudaDeviceReset of that device.
  * All calls share the one buffer: calls whose GPU work overlaps in time (other
  * streams, other host threads) race on it and must be serialised by the
  * caller. Nothing in the buffer needs to start at zero; every call writes what

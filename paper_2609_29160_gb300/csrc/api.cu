@@ -12,10 +12,30 @@ using namespace tre;
 
 namespace {
 
-bool grid_ok(const tre_grid* g) {
-  return g && g->n_models >= 1 && g->n_models <= 1024 && g->window_ms >= 1 && g->n_windows >= 0 &&
-         (int64_t)g->n_windows * g->window_ms < (int64_t)2147483647;
-}
+// ---- phase tracing ----------------------------------------------------------
+const char* const kPhaseName[TRE_TRACE_PHASES] = {"reduce", "gauge_scan", "aggregate", "score",
+                                                  "receiver", "slo_counts", "calibrate",
+                                                  "normalize", "select", "occupancy"};
+struct TraceRec {
+  int phase, launches;
+  cudaEvent_t a, b;
+};
+struct Tracer {
+  bool on = false;
+  std::vector<cudaEvent_t> pool;
+  size_t used = 0;
+  std::vector<TraceRec> recs;
+  cudaEvent_t next() {
+    if (used == pool.size()) {
+      cudaEvent_t e;
+      if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+      pool.push_back(e);
+    }
+    return pool[used++];
+  }
+};
+Tracer g_trace;
+
 
 // A column the kernels may read: device memory, or host memory the GPU
 // addresses (pinned and mapped). Plain pageable host memory is refused here,
@@ -48,17 +68,6 @@ bool ev_ok(const tre_events* e) {
   return true;
 }
 
-bool counts_ok(const tre_counts* c) {
-  return c && c->P && c->D && c->A && c->W && (!c->A_ms) == (!c->W_ms);
-}
-
-bool prof_ok(const tre_profile* p, bool need_theta_tau) {
-  if (!p || (p->dtype != TRE_F32 && p->dtype != TRE_F64)) return false;
-  if (!(p->w_p && p->w_q && p->alpha)) return false;
-  if (need_theta_tau && !(p->theta && p->tau_crit && p->tau_surplus)) return false;
-  return true;
-}
-
 ReqCols cols_of(const tre_requests* r) {
   return ReqCols{r->model, r->t_arr_ms, r->t_start_ms, r->t_first_ms, r->t_end_ms, r->L_in,
                  r->L_out, r->n};
@@ -84,50 +93,43 @@ tre_status ws_check(const Arena& a, void* ws, size_t* ws_bytes, bool& query) {
 
 tre_status cuda_status(cudaError_t e) { return e == cudaSuccess ? TRE_OK : TRE_ECUDA; }
 
-// ---- phase tracing ----------------------------------------------------------
-enum Phase { kReduce, kScan, kAggregate, kScore, kReceiver, kSlo, kCalibrate, kNormalize,
-             kSelect, kOccupancy };
-const char* const kPhaseName[TRE_TRACE_PHASES] = {"reduce", "gauge_scan", "aggregate", "score",
-                                                  "receiver", "slo_counts", "calibrate",
-                                                  "normalize", "select", "occupancy"};
-struct TraceRec {
-  int phase, launches;
-  cudaEvent_t a, b;
-};
-struct Tracer {
-  bool on = false;
-  std::vector<cudaEvent_t> pool;
-  size_t used = 0;
-  std::vector<TraceRec> recs;
-  cudaEvent_t next() {
-    if (used == pool.size()) {
-      cudaEvent_t e;
-      if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
-      pool.push_back(e);
-    }
-    return pool[used++];
-  }
-};
-Tracer g_trace;
+}  // namespace
 
-// brackets the launches of one phase with events when tracing is on
-struct Scope {
-  TraceRec rec{};
-  cudaStream_t s;
-  bool live = false;
-  Scope(int phase, int launches, cudaStream_t st) : s(st) {
-    if (!g_trace.on) return;
-    rec.phase = phase;
-    rec.launches = launches;
-    rec.a = g_trace.next();
-    rec.b = g_trace.next();
-    if (!rec.a || !rec.b) return;
-    live = cudaEventRecord(rec.a, s) == cudaSuccess;
-  }
-  ~Scope() {
-    if (live && cudaEventRecord(rec.b, s) == cudaSuccess) g_trace.recs.push_back(rec);
-  }
-};
+namespace tre {
+
+bool grid_ok(const tre_grid* g) {
+  return g && g->n_models >= 1 && g->n_models <= 1024 && g->window_ms >= 1 && g->n_windows >= 0 &&
+         (int64_t)g->n_windows * g->window_ms < (int64_t)2147483647;
+}
+
+bool counts_ok(const tre_counts* c) {
+  return c && c->P && c->D && c->A && c->W && (!c->A_ms) == (!c->W_ms);
+}
+
+bool prof_ok(const tre_profile* p, bool need_theta_tau) {
+  if (!p || (p->dtype != TRE_F32 && p->dtype != TRE_F64)) return false;
+  if (!(p->w_p && p->w_q && p->alpha)) return false;
+  if (need_theta_tau && !(p->theta && p->tau_crit && p->tau_surplus)) return false;
+  return true;
+}
+
+Scope::Scope(int phase, int launches, cudaStream_t st) : s(st) {
+  if (!g_trace.on) return;
+  a = g_trace.next();
+  b = g_trace.next();
+  if (!a || !b) return;
+  ph = phase;
+  n = launches;
+  live = cudaEventRecord(a, s) == cudaSuccess;
+}
+
+Scope::~Scope() {
+  if (live && cudaEventRecord(b, s) == cudaSuccess) g_trace.recs.push_back(TraceRec{ph, n, a, b});
+}
+
+}  // namespace tre
+
+namespace {
 
 template <class T> T to_t(double v) { return (T)v; }
 

@@ -693,17 +693,9 @@ cudaError_t launch_calibrate(const SeriesTable<T>& tab, const T* S, const uint8_
     k_pack<T><<<tiles, kPackThreads, 0, s>>>(tab, pp, S, cls, slo, w.thr, ok_frac,
                                              static_cast<U*>(w.keys), kmin, kmax, w.ncand);
   const size_t smem = search_smem_bytes<T>();
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(k_search<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
-    // the largest carveout lets two searches share an SM where their tables fit
-    if (!e)
-      e = cudaFuncSetAttribute(k_search<T>, cudaFuncAttributePreferredSharedMemoryCarveout,
-                               cudaSharedmemCarveoutMaxShared);
-    if (e) return e;
-    attr_set = true;
-  }
+  // the largest carveout lets two searches share an SM where their tables fit
+  cudaError_t e = func_smem_once((const void*)k_search<T>, (int)smem, true);
+  if (e) return e;
   k_search<T><<<tab.n * tab.M, kNB, smem, s>>>(tab, static_cast<const U*>(w.keys), kmin, kmax,
                                                w.ncand, reliability, theta, diag);
   return cudaGetLastError();

@@ -36,6 +36,39 @@ struct EvCols {
   const int32_t *req_model, *req_t_arr, *req_ttft;
 };
 
+// ---- device.cu ------------------------------------------------------------
+// Launch state kept per GPU (the device current on the calling thread), safe to
+// call from several host threads.
+// SM count of the current device.
+int device_sm_count();
+// Raises fn's dynamic shared-memory limit to `bytes` (and, with max_carveout,
+// asks for the largest shared-memory carveout) once per (device, function).
+cudaError_t func_smem_once(const void* fn, int bytes, bool max_carveout);
+
+// ---- api.cu: argument checks shared by the entry points ---------------------
+bool grid_ok(const tre_grid* g);
+bool counts_ok(const tre_counts* c);
+bool prof_ok(const tre_profile* p, bool need_theta_tau);
+
+// ---- api.cu: phase tracing (tre_trace_enable / tre_trace_collect) -----------
+enum Phase { kReduce, kScan, kAggregate, kScore, kReceiver, kSlo, kCalibrate, kNormalize,
+             kSelect, kOccupancy };
+// While tracing is on, brackets the launches of one phase with a pair of
+// events recorded on the stream (constructed before, destroyed after them).
+class Scope {
+ public:
+  Scope(int phase, int launches, cudaStream_t st);
+  ~Scope();
+  Scope(const Scope&) = delete;
+  Scope& operator=(const Scope&) = delete;
+
+ private:
+  cudaStream_t s;
+  cudaEvent_t a = nullptr, b = nullptr;
+  int ph = 0, n = 0;
+  bool live = false;
+};
+
 // ---- reduce.cu ------------------------------------------------------------
 // Reduction scratch for a batch of traces on one grid: diff arrays
 // [trace][K+1][M] for the gauges, per-request first and last event ticks, scan

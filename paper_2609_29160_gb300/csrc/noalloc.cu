@@ -6,6 +6,7 @@
 #include <cuda_runtime.h>
 
 #include <cstring>
+#include <mutex>
 
 #include "internal.h"
 
@@ -27,13 +28,18 @@ static __device__ __align__(256) unsigned char g_score_scratch[kScratchBytes];
 
 constexpr int kMaxDevices = 256;
 void* g_scratch_addr[kMaxDevices];
+std::mutex g_scratch_mu;
 
 // Device address of the scratch for the current device, looked up once per
-// device (the first call on a device does this; make it before any stream
-// capture).
+// device with that device current (the first call on a device does this; make
+// it before any stream capture). Guarded for concurrent host threads. The
+// address belongs to the device's current context: cudaDeviceReset loads the
+// module anew and may move the buffer, so a process that resets a device must
+// not call tss_score_noalloc on it afterwards (tre.h says so).
 tre_status scratch_address(void** out) {
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return TRE_ECUDA;
+  std::lock_guard<std::mutex> lk(g_scratch_mu);
   if (!g_scratch_addr[dev]) {
     void* p = nullptr;
     if (cudaGetSymbolAddress(&p, g_score_scratch) != cudaSuccess || !p) return TRE_ECUDA;
@@ -67,14 +73,20 @@ tre_status run(const tre_grid* g, const tre_counts* in, const tre_profile* p, vo
   if (st != TRE_OK) return st;
   Arena a(base);
   score_ws_layout<T>(a, M, elems, n_seg, w);
-  cudaError_t e = launch_score<T>(
-      tab, in->P, in->D, in->A, in->W, static_cast<const T*>(p->w_p),
-      static_cast<const T*>(p->w_q), static_cast<const T*>(p->alpha),
-      static_cast<const T*>(p->theta), static_cast<const T*>(p->tau_crit),
-      static_cast<const T*>(p->tau_surplus), static_cast<T*>(S_carry), init_carry,
-      static_cast<T*>(S_out), static_cast<T*>(Z_out), cls_out, w, diag, s, in->A_ms, in->W_ms);
-  if (!e && recv_out)
+  cudaError_t e;
+  {
+    Scope sc(kScore, 6, s);
+    e = launch_score<T>(tab, in->P, in->D, in->A, in->W, static_cast<const T*>(p->w_p),
+                        static_cast<const T*>(p->w_q), static_cast<const T*>(p->alpha),
+                        static_cast<const T*>(p->theta), static_cast<const T*>(p->tau_crit),
+                        static_cast<const T*>(p->tau_surplus), static_cast<T*>(S_carry),
+                        init_carry, static_cast<T*>(S_out), static_cast<T*>(Z_out), cls_out, w,
+                        diag, s, in->A_ms, in->W_ms);
+  }
+  if (!e && recv_out) {
+    Scope sc(kReceiver, 1, s);
     e = launch_receiver<T>(M, K, static_cast<const T*>(Z_out), cls_out, recv_out, s);
+  }
   return e == cudaSuccess ? TRE_OK : TRE_ECUDA;
 }
 
@@ -85,14 +97,8 @@ extern "C" tre_status tss_score_noalloc(const tre_grid* grid, const tre_counts* 
                                         uint8_t* init_carry, void* S_out, void* Z_out,
                                         uint8_t* cls_out, int32_t* recv_out, tre_diag* diag,
                                         tre_stream stream) {
-  if (!grid || grid->n_models < 1 || grid->n_models > 1024 || grid->window_ms < 1 ||
-      grid->n_windows < 0 || (int64_t)grid->n_windows * grid->window_ms >= (int64_t)2147483647)
-    return TRE_EINVAL;
-  if (!in || !in->P || !in->D || !in->A || !in->W || !prof || !diag) return TRE_EINVAL;
-  if (prof->dtype != TRE_F32 && prof->dtype != TRE_F64) return TRE_EINVAL;
-  if (!prof->w_p || !prof->w_q || !prof->alpha || !prof->theta || !prof->tau_crit ||
-      !prof->tau_surplus)
-    return TRE_EINVAL;
+  // the same argument checks as tss_score (which additionally needs ws_bytes)
+  if (!grid_ok(grid) || !counts_ok(in) || !prof_ok(prof, true) || !diag) return TRE_EINVAL;
   if (!S_out || !Z_out || !cls_out || (!S_carry) != (!init_carry)) return TRE_EINVAL;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (prof->dtype == TRE_F32)

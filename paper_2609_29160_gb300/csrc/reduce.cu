@@ -854,16 +854,7 @@ k_gauge_apply(const __grid_constant__ GaugePlan gp, const int32_t* __restrict__ 
   }
 }
 
-int num_sms() {
-  static int n = 0;
-  if (!n) {
-    int dev = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-    if (n <= 0) n = 1;
-  }
-  return n;
-}
+int num_sms() { return device_sm_count(); }
 
 int64_t per_cta_records(int64_t n, int lo, int hi, int quantum = kThreads) {
   int64_t per = (n + (int64_t)num_sms() * 4 - 1) / ((int64_t)num_sms() * 4);
@@ -935,19 +926,54 @@ cudaError_t launch_reduce_requests(const ReqCols* traces, int n_traces, int M, i
   int64_t total_n = 0;
   for (int t = 0; t < n_traces; ++t) total_n += traces[t].n;
   // records that live in host memory (pinned, mapped) are copied into shared
-  // memory once per CTA rather than read twice over the host link
+  // memory once per CTA rather than read twice over the host link; any column
+  // in host memory selects the copying variant (it reads device columns too)
   bool copy_records = false;
   for (int t = 0; t < n_traces; ++t) {
-    cudaPointerAttributes pa;
-    if (traces[t].n > 0 && cudaPointerGetAttributes(&pa, traces[t].model) == cudaSuccess &&
-        pa.type == cudaMemoryTypeHost)
-      copy_records = true;
+    const ReqCols& c = traces[t];
+    if (c.n == 0) continue;
+    const void* cols[7] = {c.model, c.t_arr, c.t_start, c.t_first, c.t_end, c.L_in, c.L_out};
+    for (const void* p : cols) {
+      cudaPointerAttributes pa;
+      if (cudaPointerGetAttributes(&pa, p) != cudaSuccess) {
+        cudaGetLastError();
+        continue;
+      }
+      if (pa.type == cudaMemoryTypeHost) copy_records = true;
+    }
   }
-  // records per CTA sized on the whole batch so the grid fills the GPU
-  const int64_t per = per_cta_records(std::max<int64_t>(total_n / n_traces, 1), 1024,
-                                      copy_records ? 2048 : 8192,
-                                      kThreads * kVec);   // whole passes for every warp
+  const int64_t mean_n = std::max<int64_t>(total_n / n_traces, 1);
+  // model rows padded to a power of two on the arrival side; start side runs
+  // of F (power of two) windows per model
+  int lgMp = 0;
+  while ((1 << lgMp) < M) ++lgMp;
+  const int Mp = 1 << lgMp;
+  const int64_t near_cap = 32 * 1024 / ((4 + (slo ? 4 : 0)) * Mp);   // arrival-stage budget
+  int lgF = 3;
+  while (lgF < 8 && (size_t)12 * M * ((2 << lgF) + 1) <= 16 * 1024) ++lgF;
+  const int F = 1 << lgF;
+  // arrival-side rows (3x the mean arrival span of a CTA's records) and the
+  // shared memory a CTA of `p` records needs
+  auto rows_for = [&](int64_t p) {
+    return (int)std::max<int64_t>(
+        1, std::min<int64_t>(near_cap, (int64_t)(3.0 * p / mean_n * K) + 34));
+  };
+  auto smem_for = [&](int64_t p) {
+    const size_t stage = (size_t)rows_for(p) * Mp * (4 + (slo ? 4 : 0)) +
+                         (size_t)12 * M * (F + 1) + (size_t)M * 8 + 16 +
+                         (size_t)p * sizeof(uint16_t);
+    return stage + (copy_records ? (size_t)p * 7 * 4 : 0);
+  };
+  constexpr size_t kSmemMax = 200 * 1024;
+  // records per CTA sized on the whole batch so the grid fills the GPU, in
+  // whole passes of every warp; with copied records, fewer per CTA when many
+  // models leave less room beside the staging
+  int64_t per = per_cta_records(mean_n, 1024, copy_records ? 2048 : 8192, kThreads * kVec);
+  while (per > kThreads * kVec && smem_for(per) > kSmemMax) per -= kThreads * kVec;
   static_assert(8192 <= kMaxPerCta, "packed shared counters need <= kMaxPerCta records per CTA");
+  const int near_rows = rows_for(per);
+  const size_t smem = smem_for(per);
+  if (smem > kSmemMax) return cudaErrorInvalidValue;
   int ctas = 0;
   for (int t = 0; t < n_traces; ++t) {
     const ReqCols& c = traces[t];
@@ -962,43 +988,15 @@ cudaError_t launch_reduce_requests(const ReqCols* traces, int n_traces, int M, i
   }
   bt.cta_base[n_traces] = ctas;
   if (ctas == 0) return cudaSuccess;
-  // model rows padded to a power of two on the arrival side; start side runs
-  // of F (power of two) windows per model
-  int lgMp = 0;
-  while ((1 << lgMp) < M) ++lgMp;
-  const int Mp = 1 << lgMp;
-  const int64_t near_cap = 32 * 1024 / ((4 + (slo ? 4 : 0)) * Mp);   // arrival-stage budget
-  const int near_rows = (int)std::max<int64_t>(
-      1, std::min<int64_t>(near_cap,
-                           (int64_t)(3.0 * per / std::max<int64_t>(total_n / n_traces, 1) * K) +
-                               34));   // 3x the mean arrival span
-  int lgF = 3;
-  while (lgF < 8 && (size_t)12 * M * ((2 << lgF) + 1) <= 16 * 1024) ++lgF;
-  const int F = 1 << lgF;
-  const size_t smem_stage = (size_t)near_rows * Mp * (4 + (slo ? 4 : 0)) +
-                            (size_t)12 * M * (F + 1) + (size_t)M * 8 + 16 +
-                            (size_t)per * sizeof(uint16_t);
-  // records in host memory are copied into shared memory once per CTA
-  const size_t smem_copy = copy_records ? (size_t)per * 7 * 4 : 0;
-  const size_t smem = smem_stage + smem_copy;
-  if (smem > 200 * 1024) return cudaErrorInvalidValue;
   // the largest shared-memory carveout, so that four CTAs with their staging
   // and queues share an SM
-  static bool attr = false;
-  if (!attr) {
-    const void* fns[4] = {(const void*)k_reduce_requests<true, false>,
-                          (const void*)k_reduce_requests<false, false>,
-                          (const void*)k_reduce_requests<true, true>,
-                          (const void*)k_reduce_requests<false, true>};
-    for (const void* f : fns) {
-      cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           200 * 1024);
-      if (!e)
-        e = cudaFuncSetAttribute(f, cudaFuncAttributePreferredSharedMemoryCarveout,
-                                 cudaSharedmemCarveoutMaxShared);
-      if (e) return e;
-    }
-    attr = true;
+  const void* fns[4] = {(const void*)k_reduce_requests<true, false>,
+                        (const void*)k_reduce_requests<false, false>,
+                        (const void*)k_reduce_requests<true, true>,
+                        (const void*)k_reduce_requests<false, true>};
+  for (const void* f : fns) {
+    cudaError_t e = func_smem_once(f, 200 * 1024, true);
+    if (e) return e;
   }
   const FastDiv fd(win);
   if (slo && copy_records)
@@ -1320,13 +1318,8 @@ cudaError_t launch_occupancy_mean(const ReqCols& r, int M, int win, int K, Reduc
                       (uintptr_t)r.t_first | (uintptr_t)r.t_end | (uintptr_t)r.L_in |
                       (uintptr_t)r.L_out) % 16 == 0;
     const bool stage = win <= (1 << 20);   // 32-bit staged sums cannot overflow
-    static bool attr = false;
-    if (!attr) {
-      e = cudaFuncSetAttribute(k_occ_staged, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               96 * 1024);
-      if (e) return e;
-      attr = true;
-    }
+    e = func_smem_once((const void*)k_occ_staged, 96 * 1024, false);
+    if (e) return e;
     if (smem > 96 * 1024) return cudaErrorInvalidValue;
     const unsigned ctas = (unsigned)((r.n + kOccPerCta - 1) / kOccPerCta);
     k_occ_staged<<<ctas, kThreads, smem, s>>>(r, vec, stage, M, lgMp, win, FastDiv(win), K,

@@ -1108,14 +1108,8 @@ cudaError_t walk_launch(const WalkBatch<T>& b, WalkWs& w, cudaStream_t s) {
   const unsigned grid = (unsigned)(b.n_series * b.n_tau);
   const unsigned th = (unsigned)(b.n_cap * 32);
   if (smem <= kStageMax) {
-    static bool attr = false;
-    if (!attr) {
-      cudaError_t e = cudaFuncSetAttribute(k_walk<T, MPL, true>,
-                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           (int)kStageMax);
-      if (e) return e;
-      attr = true;
-    }
+    cudaError_t e = func_smem_once((const void*)k_walk<T, MPL, true>, (int)kStageMax, false);
+    if (e) return e;
     k_walk<T, MPL, true><<<grid, th, smem, s>>>(b, w.recv, w.n_donor, w.rank, w.order);
   } else {
     k_walk<T, MPL, false><<<grid, th, 0, s>>>(b, w.recv, w.n_donor, w.rank, w.order);
@@ -1144,17 +1138,9 @@ template <class T> void walk_ws_layout(Arena& a, WalkBatch<T>& b, WalkWs& w) {
 // unit footprints and few models: thread-per-instance walk with staged tables
 template <class T, int MMAX>
 cudaError_t walk_thread_launch(const WalkBatch<T>& b, WalkWs& w, size_t smem, cudaStream_t s) {
-  static bool attr = false;
-  if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(k_walk_thread<T, MMAX>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)kStageMax);
-    cudaError_t e2 = cudaFuncSetAttribute(k_walk_jump<T, MMAX>,
-                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                          (int)kStageMax);
-    if (e || e2) return e ? e : e2;
-    attr = true;
-  }
+  cudaError_t e = func_smem_once((const void*)k_walk_thread<T, MMAX>, (int)kStageMax, false);
+  if (!e) e = func_smem_once((const void*)k_walk_jump<T, MMAX>, (int)kStageMax, false);
+  if (e) return e;
   // nested cadences with a fast tick not shorter than a window: jump between
   // possible moves
   if (b.slow_ms % b.fast_ms == 0 && b.fast_ms >= b.series_win[0]) {

@@ -648,21 +648,56 @@ def test_sweep_small(tre):
 def test_reduce_requests_from_pinned_host_memory(tre):
     """Record columns left in pinned host memory that the GPU addresses
     directly give the same counts as device-resident columns."""
-    import os
-    import sys
     import torch
-    sys.path.insert(0, os.path.dirname(os.path.dirname(os.path.abspath(__file__))))
-    import bench
     rng = np.random.default_rng(31)
     M, win, K = 8, 100, 1200
     req = _sorted_long(rng, 20001, M, win, K)
     host = {k: torch.as_tensor(v).pin_memory() for k, v in req.items()}
-    if not bench.host_mapped(host["model"].data_ptr()):
-        pytest.skip("pinned host memory is not mapped at the same address on this system")
     ref = tre.tss_window_reduce(M, win, K, requests=_cuda(req))
     got = tre.tss_window_reduce(M, win, K, requests=host)
     for k in "PDAW":
         assert torch.equal(got[k], ref[k]), k
+
+
+@pytest.mark.parametrize("where", ["device", "pinned_host", "mixed"])
+def test_reduce_requests_1024_models(tre, where):
+    """The largest model count the library takes: the staging leaves less room
+    per CTA, and records read from host memory are copied into shared memory
+    beside it (fewer records per CTA). `mixed` leaves one column in host
+    memory."""
+    import torch
+    rng = np.random.default_rng(1024)
+    M, win, K = 1024, 100, 600
+    req = _adversarial(rng, 120000, M, win, K)
+    P, D, A, W, drops = oracle.reduce_requests(req, M, win, K)
+    if where == "device":
+        cols = _cuda(req)
+    elif where == "pinned_host":
+        cols = {k: torch.as_tensor(v).pin_memory() for k, v in req.items()}
+    else:
+        cols = _cuda(req)
+        cols["L_out"] = torch.as_tensor(req["L_out"]).pin_memory()
+    diag = tre.new_diag()
+    c = tre.tss_window_reduce(M, win, K, requests=cols, diag=diag)
+    for k, ref in zip("PDAW", (P, D, A, W)):
+        np.testing.assert_array_equal(_np(c[k]), ref, err_msg=k)
+    d = tre.read_diag(diag)
+    assert [d["dropped_range"], d["dropped_model"], d["dropped_order"]] == drops.tolist()
+
+
+def test_calibrate_1024_models(tre):
+    import torch
+    rng = np.random.default_rng(4)
+    M, win, K = 1024, 1000, 300
+    req = _adversarial(rng, 150000, M, win, K)
+    slo = rng.integers(200, 3000, M).astype(np.int32)
+    prof = {"w_p": 0.2, "w_q": 2.0, "alpha": 0.2, "theta": 1.0, "tau_crit": 0.8,
+            "tau_surplus": 1.2}
+    o = oracle.pipeline_requests(req, M, win, K, prof, slo, np.float32)
+    rc = _cuda(req)
+    c = tre.tss_window_reduce(M, win, K, requests=rc)
+    th = tre.tss_calibrate(c, prof, win, slo, requests=rc, dtype="f32")
+    np.testing.assert_array_equal(_np(th), o["theta"])
 
 
 def test_reduce_refuses_pageable_host_columns(tre):
