@@ -43,6 +43,8 @@ def parse():
     ap.add_argument("--scale", type=float, default=1.0, help="request-count scale (1.0 = full)")
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the single-trace workloads measured beside the sweep")
     return ap.parse_args()
 
 
@@ -97,15 +99,18 @@ def peaks():
 
 
 class ClockSampler:
-    """nvidia-smi clocks / throttle reasons sampled during the timed region."""
-    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    """nvidia-smi clocks / throttle reasons, sampled every 100 ms while the
+    sampler runs; window() keeps the samples taken between two marks (host wall
+    time, compared with nvidia-smi's own timestamps)."""
+    Q = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
          "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    NAMES = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
 
     def __init__(self, gpu):
         self.gpu = gpu
         self.proc = None
-        self.t0 = self.t1 = None
+        self.rows = []
 
     def start(self):
         try:
@@ -116,15 +121,14 @@ class ClockSampler:
         except Exception:
             self.proc = None
 
-    def mark(self, begin):
-        if begin:
-            self.t0 = time.time()
-        else:
-            self.t1 = time.time()
+    @staticmethod
+    def now():
+        import datetime
+        return datetime.datetime.now()
 
     def stop(self):
         if self.proc is None:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+            return
         time.sleep(0.15)
         self.proc.terminate()
         try:
@@ -132,21 +136,28 @@ class ClockSampler:
         except Exception:
             self.proc.kill()
             out = ""
-        rows = [r.split(", ") for r in out.strip().splitlines() if r.count(",") >= 8]
-        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
-        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        reasons = set()
-        for r in rows:
-            for i, n in enumerate(names):
-                if r[5 + i].strip().lower() == "active":
-                    reasons.add(n)
-        # samples are taken every 100 ms through warm-up and the timed loop; the
-        # loaded ones are those at or above the median of the run
-        load = [s for s in sm if s >= statistics.median(sm)] if sm else []
-        return {"sm_mhz": statistics.median(load) if load else None,
-                "sm_max_mhz": max(mx) if mx else None, "reasons": sorted(reasons),
-                "samples": len(sm)}
+        import datetime
+        for r in out.strip().splitlines():
+            f = [x.strip() for x in r.split(",")]
+            if len(f) < 10:
+                continue
+            try:
+                ts = datetime.datetime.strptime(f[0], "%Y/%m/%d %H:%M:%S.%f")
+                sm, mx = float(f[2]), float(f[3])
+            except ValueError:
+                continue
+            self.rows.append((ts, sm, mx, [n for i, n in enumerate(self.NAMES)
+                                           if f[6 + i].lower() == "active"]))
+
+    def window(self, t0, t1, what):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"],
+                    "samples": 0, "window": what}
+        rows = [r for r in self.rows if t0 <= r[0] <= t1]
+        reasons = sorted({n for r in rows for n in r[3]})
+        return {"sm_mhz": statistics.median([r[1] for r in rows]) if rows else None,
+                "sm_max_mhz": max(r[2] for r in rows) if rows else None,
+                "reasons": reasons, "samples": len(rows), "window": what}
 
 
 def _oracle_sweep(sw):
@@ -271,6 +282,229 @@ def cpu_baseline_parallel(scale, seed0):
                       f"{dt:.1f} s"}
 
 
+# ---------------------------------------------------------------------------
+# The single-trace workloads: one pass of the whole path per step
+# (tss_window_reduce -> tss_calibrate -> tss_score -> tre_select_moves).
+# ---------------------------------------------------------------------------
+CONFIGS = (
+    # (key, workload name, dtypes, timed steps, oracle sample: fraction of the
+    # trace's duration kept, from its start)
+    ("tiny_3_models_600s", "tiny", ("f64", "f32"), 50, 1.0),
+    ("mid_8_models_1M_requests_1h", "mid", ("f32", "f64"), 30, 1.0),
+    ("hetero_16_models_10M_requests_6h", "hetero", ("f32",), 20, 1.0 / 8),
+    ("stream_64_models_200M_token_events_24h", "stream", ("f32",), 10, 1.0 / 24),
+)
+
+
+def config_bytes(w, tsize):
+    """Algorithmic bytes of one pass: the telemetry read once (28 B per request
+    record, or 13 B per token event plus 12 B per request-table row) and, per
+    (window, model), the four counts, S and Z in the profile's type and the
+    region byte written once."""
+    KM = w["K"] * w["M"]
+    if "events" in w:
+        src = len(w["events"]["model"]) * 13 + len(w["events"]["req_model"]) * 12
+    else:
+        src = len(w["requests"]["model"]) * 28
+    return src + KM * (16 + 2 * tsize + 1)
+
+
+def cut_workload(w, frac):
+    """The first `frac` of a workload's duration: requests arriving (events
+    stamped) before the cut, on the windows before it."""
+    if frac >= 1.0:
+        return w
+    K = max(1, int(w["K"] * frac))
+    cut = K * w["window_ms"]
+    out = dict(w, K=K)
+    if "events" in w:
+        ev = w["events"]
+        keep = ev["t_s"].astype(np.float64) * 1000.0 < cut
+        out["events"] = {k: (v[keep] if len(v) == len(keep) and k in ("model", "req", "t_s",
+                                                                      "phase") else v)
+                         for k, v in ev.items()}
+    keep = w["requests"]["t_arr_ms"] < cut
+    out["requests"] = {k: v[keep] for k, v in w["requests"].items()}
+    return out
+
+
+def _oracle_path(w, dtype):
+    """The oracle's whole path for one trace (reduce, SLO counts, score,
+    calibrate, score, walk)."""
+    import oracle
+    M, win, K = w["M"], w["window_ms"], w["K"]
+    prof = tracegen.default_profile(M, win)
+    Z, cls = _oracle_models(w, dtype, prof)
+    oracle.select_moves(Z, cls, 0.8, 1.2, win, w["budget"], w["r0"], w["r_min"], w["footprint"],
+                        w["fast_ms"], w["slow_ms"], w["pacing_cap"])
+
+
+def _oracle_models(w, dtype, prof):
+    import oracle
+    M, win, K = w["M"], w["window_ms"], w["K"]
+    if "events" in w:
+        ev = w["events"]
+        P, D, A, W, _ = oracle.reduce_events(ev, M, win, K)
+        n_arr, n_met = oracle.slo_counts_events(ev, M, win, K, w["slo_ttft_ms"])
+        S, _, cls, _ = oracle.score(P, D, A, W, prof, win, dtype)
+        theta, _ = oracle.calibrate(S, cls, n_arr, n_met)
+        _, Z, cls, _ = oracle.score(P, D, A, W, dict(prof, theta=theta), win, dtype)
+        return Z, cls
+    o = oracle.pipeline_requests(w["requests"], M, win, K, prof, w["slo_ttft_ms"], dtype)
+    return o["Z"], o["cls"]
+
+
+def _model_slice(w, m):
+    """Model m's telemetry as a one-model workload (ids remapped to 0; token
+    events' request ids renumbered within the model)."""
+    one = {"M": 1, "window_ms": w["window_ms"], "K": w["K"],
+           "slo_ttft_ms": w["slo_ttft_ms"][m: m + 1]}
+    if "events" in w:
+        ev = w["events"]
+        rows = np.flatnonzero(ev["req_model"] == m)
+        keep = ev["model"] == m
+        req = np.searchsorted(rows, ev["req"][keep]).astype(np.int32)
+        one["events"] = {"model": np.zeros(int(keep.sum()), np.int32), "req": req,
+                         "t_s": ev["t_s"][keep], "phase": ev["phase"][keep],
+                         "req_model": np.zeros(len(rows), np.int32),
+                         "req_t_arr_ms": ev["req_t_arr_ms"][rows],
+                         "req_ttft_ms": ev["req_ttft_ms"][rows]}
+    else:
+        keep = w["requests"]["model"] == m
+        one["requests"] = {k: (np.zeros(int(keep.sum()), np.int32) if k == "model" else v[keep])
+                           for k, v in w["requests"].items()}
+    return one
+
+
+def _oracle_model_unit(args):
+    one, dtype = args
+    prof = tracegen.default_profile(1, one["window_ms"])
+    return _oracle_models(one, np.dtype(dtype).type, prof)
+
+
+def _noop(x):
+    return x
+
+
+def config_cpu(w, dtype, frac, pool):
+    """The oracle's rate on a bounded sample of a workload (the first `frac` of
+    its duration): single-threaded, and with its models as independent units
+    over the worker pool (reduce, calibrate and score per model) followed by
+    the walk."""
+    import oracle
+    sw = cut_workload(w, frac)
+    n = len(sw["events"]["model"]) if "events" in sw else len(sw["requests"]["model"])
+    npdt = np.float32 if dtype == "f32" else np.float64
+    t0 = time.perf_counter()
+    _oracle_path(sw, npdt)
+    dt1 = time.perf_counter() - t0
+    what = (f"first {sw['K'] * sw['window_ms'] / 1000:.0f} s of the trace ({n} "
+            f"{'token events' if 'events' in sw else 'request records'}, {sw['K']} windows)")
+    res = {"value": n / dt1, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": what,
+           "seconds": dt1}
+    if pool is not None:
+        try:
+            t0 = time.perf_counter()
+            parts = pool.map_async(_oracle_model_unit,
+                                   [(_model_slice(sw, m), np.dtype(npdt).name)
+                                    for m in range(sw["M"])], chunksize=1).get(timeout=600)
+            Z = np.stack([p[0][:, 0] for p in parts], 1)
+            cls = np.stack([p[1][:, 0] for p in parts], 1)
+            oracle.select_moves(Z, cls, 0.8, 1.2, sw["window_ms"], sw["budget"], sw["r0"],
+                                sw["r_min"], sw["footprint"], sw["fast_ms"], sw["slow_ms"],
+                                sw["pacing_cap"])
+            dtp = time.perf_counter() - t0
+            res["parallel"] = {"value": n / dtp, "unit": UNIT, "cores": pool._processes,
+                               "kind": "oracle", "seconds": dtp,
+                               "sample": what + f"; {sw['M']} per-model units over "
+                                                f"{pool._processes} processes, then the walk"}
+        except Exception as e:   # a baseline must not cost the bench line
+            res["parallel"] = {"error": f"{type(e).__name__}: {e}"}
+    return res
+
+
+def measure_configs(tre, lib, Trace, hbm, peak_kind, with_cpu):
+    """Device time of one pass of the whole path per workload and dtype, with
+    L2 flushed (a buffer of twice its size written) before every step and the
+    step alone between the CUDA events; phase times from the library's
+    events; the oracle's rates beside it."""
+    import multiprocessing as mp
+
+    import torch
+    pool = None
+    if with_cpu:
+        try:
+            pool = mp.get_context("spawn").Pool(max(1, os.cpu_count() or 1))
+            pool.map_async(_noop, range(pool._processes)).get(timeout=120)
+        except Exception:
+            pool = None
+    l2 = torch.cuda.get_device_properties(torch.cuda.current_device()).L2_cache_size
+    flush = torch.empty(2 * max(int(l2), 1 << 20), dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.current_stream()
+    out = {}
+    try:
+        for key, name, dtypes, steps, frac in CONFIGS:
+            w = tracegen.workload(name, scale=1.0)
+            dev = ({"events": {k: torch.as_tensor(v).cuda() for k, v in w["events"].items()}}
+                   if "events" in w else
+                   {"requests": {k: torch.as_tensor(v).cuda() for k, v in w["requests"].items()}})
+            prof = tracegen.default_profile(w["M"], w["window_ms"])
+            n_units = len(w["events"]["model"]) if "events" in w else len(w["requests"]["model"])
+            tokens = int(w["requests"]["L_in"].astype(np.int64).sum() +
+                         w["requests"]["L_out"].astype(np.int64).sum())
+            entry = {"records_or_events": n_units,
+                     "unit_kind": "token events" if "events" in w else "request records",
+                     "model_windows": w["K"] * w["M"], "tokens": tokens, "dtypes": {}}
+            for dt in dtypes:
+                plan = tre.PipelinePlan(w["M"], w["window_ms"], w["K"], prof, w["slo_ttft_ms"],
+                                        w["budget"], w["r0"], w["r_min"], w["footprint"],
+                                        dtype=dt, fast_ms=w["fast_ms"], slow_ms=w["slow_ms"],
+                                        pacing_cap=w["pacing_cap"], moves_cap=1 << 16, **dev)
+                for _ in range(3):
+                    plan.run(stream)
+                torch.cuda.synchronize()
+                lib.tre_trace_enable(1)
+                evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                       for _ in range(steps)]
+                for a, b in evs:
+                    flush.fill_(1)
+                    a.record(stream)
+                    plan.run(stream)
+                    b.record(stream)
+                torch.cuda.synchronize()
+                tr = Trace()
+                lib.tre_trace_collect(C.byref(tr))
+                lib.tre_trace_enable(0)
+                ms = sum(a.elapsed_time(b) for a, b in evs) / steps
+                tsize = 4 if dt == "f32" else 8
+                byts = config_bytes(w, tsize)
+                ph = {tr.name[i].decode(): tr.ms[i] / steps * 1e3 for i in range(tr.n_phases)
+                      if tr.calls[i]}
+                launches = int(sum(tr.launches[i] for i in range(tr.n_phases))) // steps
+                achieved = byts / (ms / 1e3) / 1e9
+                e = {"us_per_step": ms * 1e3, "steps": steps,
+                     "events_per_s": n_units / (ms / 1e3),
+                     "model_windows_per_s": w["K"] * w["M"] / (ms / 1e3),
+                     "tokens_per_s": tokens / (ms / 1e3), "n_moves": int(plan.n_moves.item()),
+                     "algorithmic_bytes": byts,
+                     "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm,
+                                  "unit": "GB/s", "frac": achieved / hbm,
+                                  "peak_kind": peak_kind},
+                     "phases_us_per_step": ph, "launches_per_step": launches,
+                     "l2": "flushed before every step (2x L2 written)"}
+                if with_cpu:
+                    e["cpu_baseline"] = config_cpu(w, dt, frac, pool)
+                entry["dtypes"][dt] = e
+                del plan
+            out[key] = entry
+            del dev, w
+            torch.cuda.empty_cache()
+    finally:
+        if pool is not None:
+            pool.terminate()
+    return out
+
+
 TRACE_PHASES = 10   # phases of tre_trace (the library header's count)
 
 
@@ -339,11 +573,15 @@ TRAFFIC_SUMMARIES = {"reduce": ("profiles/k_reduce_requests_sweep_7x1M.md",
 
 
 def captured_traffic(phase):
+    """DRAM bytes per call of a phase's kernel as one ncu capture measured them
+    (not measured in this run): taken from the committed capture summary, and
+    only while the kernel's source is the one the counters were taken on."""
     import hashlib
+    import re
     if phase not in TRAFFIC_SUMMARIES:
         return None
-    summ, src = (os.path.join(ROOT, f) for f in TRAFFIC_SUMMARIES[phase])
-    import re
+    rel_summ, rel_src = TRAFFIC_SUMMARIES[phase]
+    summ, src = os.path.join(ROOT, rel_summ), os.path.join(ROOT, rel_src)
     try:
         fields = {}
         for line in open(summ):
@@ -353,7 +591,7 @@ def captured_traffic(phase):
         digest = hashlib.sha256(open(src, "rb").read()).hexdigest()
         if fields.get("source_sha256") != digest:
             return None
-        return float(fields["dram_bytes_per_call"])
+        return {"dram_bytes_per_call": float(fields["dram_bytes_per_call"]), "summary": rel_summ}
     except (OSError, KeyError, ValueError):
         return None
 
@@ -449,20 +687,36 @@ def main():
         dist.barrier()
     torch.cuda.synchronize()
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    clocks.mark(True)
+    c0 = clocks.now()
     ev0.record(stream)
     for _ in range(args.steps):
         out = step()
     ev1.record(stream)
     torch.cuda.synchronize()
-    clocks.mark(False)
+    c1 = clocks.now()
     if world > 1:
         dist.barrier()
     ms = ev0.elapsed_time(ev1)
     tr = Trace()
     lib.tre_trace_collect(C.byref(tr))
     lib.tre_trace_enable(0)
-    clk = clocks.stop()
+    # the same step, back to back for at least 1.5 s right after the timed
+    # region: long enough for the 100 ms clock samples to see the kernels
+    n_sus = max(1, int(1500.0 / max(ms / args.steps, 1e-3)) + 1)
+    es0, es1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s0 = clocks.now()
+    es0.record(stream)
+    for _ in range(n_sus):
+        step()
+    es1.record(stream)
+    torch.cuda.synchronize()
+    s1 = clocks.now()
+    time.sleep(0.2)
+    clocks.stop()
+    clk = clocks.window(c0, s1, "timed region and the sustained loop of the same step after it")
+    clk["timed_region_samples"] = clocks.window(c0, c1, "")["samples"]
+    sustained = {"steps": n_sus, "ms_per_step": es0.elapsed_time(es1) / n_sus,
+                 "clocks": clocks.window(s0, s1, "sustained loop only")}
     job_rec, job_mw, job_inst, job_tok, job_iw = (total_rec, model_windows, n_inst, tokens,
                                                   inst_windows)
     if world > 1:
@@ -486,7 +740,8 @@ def main():
         per_call_ms = phases[name]["ms"] / max(phases[name]["calls"], 1)
         achieved = pb[name] / (per_call_ms / 1e3) / 1e9
         return {"bound": "hbm", "kernel": name, "achieved": achieved, "peak": hbm,
-                "unit": "GB/s", "frac": achieved / hbm, "traffic": captured_traffic(name),
+                "unit": "GB/s", "frac": achieved / hbm, "traffic": None,
+                "ncu_capture": captured_traffic(name),
                 "share_of_step": phases[name]["ms"] / max(ms, 1e-9), "peak_kind": peak_kind,
                 "bytes_per_call": pb[name], "us_per_call": per_call_ms * 1e3}
     if dom in pb and phases[dom]["calls"]:
@@ -612,6 +867,11 @@ def main():
     next_rows = {"occupancy_mean": occupancy_measure(lib, Trace, dev_traces, M,
                                                      sw["duration_ms"], hbm, peak_kind)}
 
+    configs = None
+    if rank == 0 and not args.no_configs:
+        configs = measure_configs(tre, lib, Trace, hbm, peak_kind,
+                                  with_cpu=world == 1 and not args.no_cpu_baseline)
+
     base = base_par = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         base = cpu_baseline(args.scale)
@@ -635,9 +895,10 @@ def main():
                 k: p["ms"] / args.steps for k, p in phases.items() if p["calls"]},
             "phases_roofline": {k: round(roof_of(k)["frac"], 4) for k in pb
                                 if phases.get(k, {}).get("calls")},
-            "gpu_launches": launches, "clocks": clk, "e2e": e2e, "cpu_baseline": base,
+            "gpu_launches": launches, "clocks": clk, "sustained": sustained, "e2e": e2e,
+            "cpu_baseline": base,
             "cpu_baseline_parallel": base_par,
-            "next_rows": next_rows,
+            "next_rows": next_rows, "configs": configs,
         }
         print(json.dumps(line))
     if world > 1:

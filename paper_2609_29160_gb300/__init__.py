@@ -512,3 +512,99 @@ def sweep_moves(out, n_inst, moves_cap):
     raw = raw.reshape(n_inst, max(moves_cap, 1))
     n = out["n_moves"].cpu().numpy()
     return [raw[i, : min(int(n[i]), moves_cap)] for i in range(n_inst)]
+
+
+class PipelinePlan:
+    """One trace's whole path marshalled once: tss_window_reduce ->
+    tss_calibrate -> tss_score -> tre_select_moves, on request records or token
+    events (dicts of int32/float32/uint8 CUDA tensors). Device parameter
+    arrays, outputs, one workspace (sized for the largest of the four calls,
+    which run in order on one stream) and the C structs are built here; run()
+    resets the controller's replicas to r0 and issues the four C calls with no
+    further host work."""
+
+    def __init__(self, M, window_ms, K, profile, slo_ttft_ms, budget, r0, r_min, footprint,
+                 requests=None, events=None, dtype="f32", fast_ms=5000, slow_ms=10000,
+                 pacing_cap=1, moves_cap=4096, ok_frac=0.95, reliability=0.95, diag=None):
+        torch = _torch()
+        self.lib = lib = load()
+        code, tdt = _dt(dtype)
+        self.g = Grid(M, window_ms, K)
+        self.rq = requests_struct(requests) if requests is not None else None
+        self.ev = events_struct(events) if events is not None else None
+        self._inputs = (requests, events)
+        c = {k: torch.empty((K, M), dtype=torch.int32, device="cuda") for k in "PDAW"}
+        self.cs = _counts(c)
+        prof = dict(profile)
+        self.theta = torch.empty(M, dtype=tdt, device="cuda")
+        prof["theta"] = self.theta
+        self.pst, self._prof = _profile(prof, M, tdt, code)
+        i32 = lambda a: (a if torch.is_tensor(a) else torch.as_tensor(np.asarray(a, np.int32))).to(
+            device="cuda", dtype=torch.int32).contiguous()
+        self.slo = i32(slo_ttft_ms)
+        self.r0, self.r = i32(r0), i32(r0).clone()
+        self._rmin, self._fp = i32(r_min), i32(footprint)
+        self.ctrl = Ctrl(int(budget), self._rmin.data_ptr(), self._fp.data_ptr(), fast_ms, slow_ms,
+                         pacing_cap)
+        self.S = torch.empty((K, M), dtype=tdt, device="cuda")
+        self.Z = torch.empty((K, M), dtype=tdt, device="cuda")
+        self.cls = torch.empty((K, M), dtype=torch.uint8, device="cuda")
+        self.recv = torch.empty(K, dtype=torch.int32, device="cuda")
+        self.moves = torch.zeros(max(moves_cap, 1) * MOVE_DTYPE.itemsize, dtype=torch.uint8,
+                                 device="cuda")
+        self.n_moves = torch.zeros(1, dtype=torch.int64, device="cuda")
+        self.moves_cap = moves_cap
+        self.diag = new_diag() if diag is None else diag
+        self.ok_frac, self.rel = float(ok_frac), float(reliability)
+        self.counts = c
+        # one workspace for the four calls
+        need = 0
+        for q in self._calls(None):
+            size = C.c_size_t(0)
+            _check(q[0], q[1](None, C.byref(size)))
+            need = max(need, int(size.value))
+        self.ws = torch.empty(max(need, 256), dtype=torch.uint8, device="cuda")
+        self._ws_n = C.c_size_t(self.ws.numel())
+
+    def _calls(self, stream):
+        lib, g, P = self.lib, self.g, C.c_void_p
+        rq = C.byref(self.rq) if self.rq is not None else None
+        ev = C.byref(self.ev) if self.ev is not None else None
+        dg = _ptr(self.diag)
+        return (
+            ("tss_window_reduce", lambda ws, n: lib.tss_window_reduce(
+                C.byref(g), rq, ev, self.cs, ws, n, dg, stream)),
+            ("tss_calibrate", lambda ws, n: lib.tss_calibrate(
+                C.byref(g), rq, ev, C.byref(self.cs), C.byref(self.pst), _ptr(self.slo),
+                C.c_double(self.ok_frac), C.c_double(self.rel), _ptr(self.theta), ws, n, dg,
+                stream)),
+            ("tss_score", lambda ws, n: lib.tss_score(
+                C.byref(g), C.byref(self.cs), C.byref(self.pst), None, None, _ptr(self.S),
+                _ptr(self.Z), _ptr(self.cls), _ptr(self.recv), ws, n, dg, stream)),
+            ("tre_select_moves", lambda ws, n: lib.tre_select_moves(
+                C.byref(g), _ptr(self.Z), _ptr(self.cls), C.byref(self.pst), C.byref(self.ctrl),
+                _ptr(self.r), _ptr(self.moves), C.c_int64(self.moves_cap), _ptr(self.n_moves),
+                ws, n, dg, stream)),
+        )
+
+    def run(self, stream=None):
+        """Enqueue the whole path on `stream` (default: current torch stream)."""
+        torch = _torch()
+        s = stream if stream is not None else torch.cuda.current_stream()
+        with torch.cuda.stream(s):
+            self.r.copy_(self.r0, non_blocking=True)
+        ws = C.c_void_p(self.ws.data_ptr())
+        for name, fn in self._calls(C.c_void_p(s.cuda_stream)):
+            _check(name, fn(ws, C.byref(self._ws_n)))
+        return self
+
+    def results(self):
+        """Host view of the last run: counts, theta, S, Z, cls, recv, moves, r_final."""
+        n = int(self.n_moves.item())
+        mv = np.frombuffer(self.moves.cpu().numpy().tobytes(),
+                           dtype=MOVE_DTYPE)[: min(n, self.moves_cap)]
+        out = {k: v.cpu().numpy() for k, v in self.counts.items()}
+        out.update(theta=self.theta.cpu().numpy(), S=self.S.cpu().numpy(), Z=self.Z.cpu().numpy(),
+                   cls=self.cls.cpu().numpy(), recv=self.recv.cpu().numpy(), moves=mv,
+                   n_moves=n, r_final=self.r.cpu().numpy())
+        return out
