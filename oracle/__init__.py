@@ -310,9 +310,15 @@ def slo_tpot_counts_requests(req, M, window_ms, K, tpot_ms):
 def stage_gauges(req, M, window_ms, K):
     """Running requests split at the first token, read at each window's last
     millisecond: in prefill on [t_start, t_first) and decoding on
-    [t_first, t_end). Returns (A_prefill, A_decode)."""
-    A_p = reduce_requests(dict(req, t_end_ms=req["t_first_ms"]), M, window_ms, K)[2]
-    A_d = reduce_requests(dict(req, t_start_ms=req["t_first_ms"]), M, window_ms, K)[2]
+    [t_first, t_end), among the records reduce_requests keeps. Returns
+    (A_prefill, A_decode)."""
+    cols = _req_cols(req)
+    A_p, A_d = np.zeros((K, M), np.int32), np.zeros((K, M), np.int32)
+    rc = lib().orc_stage_gauges_requests(C.c_int32(M), C.c_int32(window_ms), C.c_int32(K),
+                                         C.c_int64(len(cols[0])), *[_p(c) for c in cols],
+                                         _p(A_p), _p(A_d))
+    if rc:
+        raise ValueError("oracle: bad arguments")
     return A_p, A_d
 
 

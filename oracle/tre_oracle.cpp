@@ -170,6 +170,41 @@ int slo_counts_requests(int32_t M, int32_t win, int32_t K, int64_t n, const int3
   return 0;
 }
 
+// Running gauge split at the first token for a stage-aware signal (Sec. VIII:
+// separate prefill and decode states): among the records reduce_requests
+// keeps, a request is prefilling on [t_start, t_first) and decoding on
+// [t_first, t_end); both gauges are read at the last millisecond of each
+// window, by the same +1/-1 difference and running sum as A and W.
+int stage_gauges_requests(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* model,
+                          const int32_t* t_arr, const int32_t* t_start, const int32_t* t_first,
+                          const int32_t* t_end, const int32_t* L_in, const int32_t* L_out,
+                          int32_t* A_pre, int32_t* A_dec) {
+  if (M < 1 || win < 1 || K < 0 || n < 0) return 1;
+  const int64_t span = (int64_t)K * win;
+  std::vector<int64_t> dP((size_t)(K + 1) * M, 0), dD((size_t)(K + 1) * M, 0);
+  for (int64_t i = 0; i < n; ++i) {
+    const int64_t m = model[i];
+    if (m < 0 || m >= M) continue;
+    const int64_t ta = t_arr[i], ts = t_start[i], tf = t_first[i], te = t_end[i];
+    if (ta < 0 || ta >= span) continue;
+    if (!(ta <= ts && ts <= tf && tf <= te) || L_in[i] < 0 || L_out[i] < 1) continue;
+    dP[(size_t)win_of(ts, win, K) * M + m] += 1;
+    dP[(size_t)win_of(tf, win, K) * M + m] -= 1;
+    dD[(size_t)win_of(tf, win, K) * M + m] += 1;
+    dD[(size_t)win_of(te, win, K) * M + m] -= 1;
+  }
+  for (int64_t m = 0; m < M; ++m) {
+    int64_t a = 0, d = 0;
+    for (int64_t k = 0; k < K; ++k) {
+      a += dP[(size_t)k * M + m];
+      d += dD[(size_t)k * M + m];
+      A_pre[(size_t)k * M + m] = (int32_t)a;
+      A_dec[(size_t)k * M + m] = (int32_t)d;
+    }
+  }
+  return 0;
+}
+
 // Decode-side SLO counts for a stage-aware signal (Sec. VIII: separate prefill
 // and decode states; Sec. III-A: decode determines TPOT): per (arrival window,
 // model) the requests with more than one output token and how many of them
@@ -785,6 +820,15 @@ int orc_occupancy_mean_requests(int32_t M, int32_t win, int32_t K, int64_t n,
                                 int64_t* A_ms, int64_t* W_ms) {
   return occupancy_mean_requests(M, win, K, n, model, t_arr, t_start, t_first, t_end, L_in, L_out,
                                  A_ms, W_ms);
+}
+
+int orc_stage_gauges_requests(int32_t M, int32_t win, int32_t K, int64_t n,
+                              const int32_t* model, const int32_t* t_arr,
+                              const int32_t* t_start, const int32_t* t_first,
+                              const int32_t* t_end, const int32_t* L_in, const int32_t* L_out,
+                              int32_t* A_pre, int32_t* A_dec) {
+  return stage_gauges_requests(M, win, K, n, model, t_arr, t_start, t_first, t_end, L_in, L_out,
+                               A_pre, A_dec);
 }
 
 int orc_slo_tpot_counts_requests(int32_t M, int32_t win, int32_t K, int64_t n,

@@ -31,17 +31,44 @@ def _req(rng, n, M, win, K):
             "L_out": L_out.astype(np.int32)}
 
 
+def _malformed(rng, req, M, win, K):
+    """Some records the reduction drops: a start before the arrival, a first
+    token before the start, an end before the first token, a bad model id, an
+    arrival outside the grid, no output token."""
+    req = {k: v.copy() for k, v in req.items()}
+    n = len(req["model"])
+    pick = rng.choice(n, 6 * (n // 10), replace=False).reshape(6, -1)
+    req["t_start_ms"][pick[0]] = req["t_arr_ms"][pick[0]] - 1
+    req["t_first_ms"][pick[1]] = req["t_start_ms"][pick[1]] - 1
+    req["t_end_ms"][pick[2]] = req["t_first_ms"][pick[2]] - 1
+    req["model"][pick[3]] = M
+    req["t_arr_ms"][pick[4]] = K * win + 5
+    req["L_out"][pick[5]] = 0
+    return req
+
+
+def _kept(req, M, win, K):
+    m, ta, ts, tf, te = (req[k].astype(np.int64) for k in
+                         ("model", "t_arr_ms", "t_start_ms", "t_first_ms", "t_end_ms"))
+    return ((m >= 0) & (m < M) & (ta >= 0) & (ta < K * win) & (ta <= ts) & (ts <= tf) &
+            (tf <= te) & (req["L_in"] >= 0) & (req["L_out"] >= 1))
+
+
 @pytest.mark.parametrize("seed,M,win,K", [(0, 3, 7, 20), (1, 2, 50, 12), (2, 4, 1, 60)])
-def test_running_gauge_splits_at_the_first_token(seed, M, win, K):
+@pytest.mark.parametrize("malformed", [False, True])
+def test_running_gauge_splits_at_the_first_token(seed, M, win, K, malformed):
     rng = np.random.default_rng(seed)
     req = _req(rng, 80, M, win, K)
+    if malformed:
+        req = _malformed(rng, req, M, win, K)
     A_p, A_d = oracle.stage_gauges(req, M, win, K)
     A = oracle.reduce_requests(req, M, win, K)[2]
     np.testing.assert_array_equal(A_p + A_d, A)
+    kept = _kept(req, M, win, K)
     for k in range(K):
         t = (k + 1) * win - 1                                    # last millisecond
         for m in range(M):
-            sel = req["model"] == m
+            sel = (req["model"] == m) & kept
             ts, tf, te = req["t_start_ms"][sel], req["t_first_ms"][sel], req["t_end_ms"][sel]
             assert A_p[k, m] == int(((ts <= t) & (t < tf)).sum())
             assert A_d[k, m] == int(((tf <= t) & (t < te)).sum())
