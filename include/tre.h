@@ -113,8 +113,9 @@ typedef struct {
  * ([t_start, t_end)) and waiting ([t_arr, t_start)) inside the window, so that
  * A_ms / window_ms is the window's mean running count (Sec. III-A defines the
  * counts at a time t; Sec. II-B speaks of an average waiting queue).
- * tss_window_reduce fills them from request records when they are set (token
- * events: TRE_EINVAL); tss_score, tss_score_noalloc and tss_calibrate then use
+ * tss_window_reduce fills them when they are set, from request records or from
+ * token events (a request runs from its first to its last valid event and
+ * waits from t_arr to its first); tss_score, tss_score_noalloc and tss_calibrate then use
  * the means A_ms / window_ms and W_ms / window_ms in Eq. 1's demand term in
  * place of A and W, and a window is IDLE when P, D, A_ms and W_ms are zero. */
 typedef struct {
@@ -236,6 +237,55 @@ tre_status tss_calibrate(const tre_grid* grid, const tre_requests* req, const tr
                          const tre_counts* in, const tre_profile* prof, const int32_t* slo_ttft_ms,
                          double ok_frac, double reliability, void* theta_out, void* ws,
                          size_t* ws_bytes, tre_diag* diag, tre_stream stream);
+
+/*
+ * Stage-aware signal (Sec. VIII: separate prefill and decode states; Sec. III-A
+ * ties prefill to the time to first token and decode to the time per output
+ * token). Request records only; records are taken or skipped by
+ * tss_window_reduce's rules (drops are not counted again here).
+ *
+ * tss_stage_gauges -- the running gauge split at the first token, read at the
+ * last millisecond of each window: A_prefill counts requests on
+ * [t_start, t_first), A_decode on [t_first, t_end) (device int32
+ * [n_windows][n_models] each); the two sum to tss_window_reduce's A.
+ */
+tre_status tss_stage_gauges(const tre_grid* grid, const tre_requests* req, int32_t* A_prefill,
+                            int32_t* A_decode, void* ws, size_t* ws_bytes, tre_diag* diag,
+                            tre_stream stream);
+
+/*
+ * tss_stage_calibrate -- one healthy boundary per stage, by tss_calibrate's
+ * rule (Sec. III-B) on each stage's smoothed signal: the prefill signal
+ * (P/dt) / max(A_prefill + w_q*W, 1) against TTFT (t_first - t_arr <=
+ * slo_ttft_ms[m]) and the decode signal (D/dt) / max(A_decode, 1) against TPOT
+ * (a request with L_out > 1 meets it when t_end - t_first <=
+ * slo_tpot_ms[m] * (L_out - 1)), both counted at the arrival window. `in`
+ * supplies P, D and W of tss_window_reduce on the same records (A is not read;
+ * A_ms / W_ms must be NULL); w_q and alpha come from `prof`. theta_prefill,
+ * theta_decode: dtype[n_models] on the device.
+ */
+tre_status tss_stage_calibrate(const tre_grid* grid, const tre_requests* req,
+                               const tre_counts* in, const int32_t* A_prefill,
+                               const int32_t* A_decode, const tre_profile* prof,
+                               const int32_t* slo_ttft_ms, const int32_t* slo_tpot_ms,
+                               double ok_frac, double reliability, void* theta_prefill,
+                               void* theta_decode, void* ws, size_t* ws_bytes, tre_diag* diag,
+                               tre_stream stream);
+
+/*
+ * tss_stage_score -- both stage signals, each smoothed as tss_score smooths
+ * (alpha of `prof`), normalised by its own theta (Eq. 2) and classified with
+ * the profile's thresholds: prefill (P/dt) / max(A_prefill + w_q*W, 1) and
+ * decode (D/dt) / max(A_decode, 1). A stage window is IDLE when its tokens,
+ * its running gauge and (prefill) W are all zero. Outputs [n_windows][n_models]
+ * (S, Z in dtype, cls uint8), all required.
+ */
+tre_status tss_stage_score(const tre_grid* grid, const tre_counts* in, const int32_t* A_prefill,
+                           const int32_t* A_decode, const tre_profile* prof,
+                           const void* theta_prefill, const void* theta_decode, void* S_prefill,
+                           void* Z_prefill, uint8_t* cls_prefill, void* S_decode, void* Z_decode,
+                           uint8_t* cls_decode, void* ws, size_t* ws_bytes, tre_diag* diag,
+                           tre_stream stream);
 
 /*
  * tre_select_moves -- open-loop TRE controller over a scored trace (Sec. IV-B,

@@ -119,8 +119,15 @@ def load(build_if_missing: bool = True):
     lib.tss_rank.argtypes = [C.POINTER(Grid), C.c_int, P, P, P, P, P]
     lib.tss_class_models.argtypes = [C.c_int64, P, P, C.c_int32, C.c_int32, P, P]
     lib.tss_class_models.restype = C.c_int
+    lib.tss_stage_gauges.argtypes = [C.POINTER(Grid), C.POINTER(Requests), P, P, P,
+                                     C.POINTER(C.c_size_t), P, P]
+    lib.tss_stage_calibrate.argtypes = [C.POINTER(Grid), C.POINTER(Requests), C.POINTER(Counts),
+                                        P, P, C.POINTER(Profile), P, P, C.c_double, C.c_double,
+                                        P, P, P, C.POINTER(C.c_size_t), P, P]
+    lib.tss_stage_score.argtypes = [C.POINTER(Grid), C.POINTER(Counts), P, P, C.POINTER(Profile),
+                                    P, P, P, P, P, P, P, P, P, C.POINTER(C.c_size_t), P, P]
     for f in ("tss_window_reduce", "tss_score", "tss_calibrate", "tre_select_moves", "tre_sweep",
-              "tss_rank"):
+              "tss_rank", "tss_stage_gauges", "tss_stage_calibrate", "tss_stage_score"):
         getattr(lib, f).restype = C.c_int
     lib.tre_status_str.argtypes = [C.c_int]
     lib.tre_status_str.restype = C.c_char_p
@@ -250,9 +257,9 @@ def _profile(prof, M, tdt, code):
 def tss_window_reduce(M, window_ms, K, requests=None, events=None, diag=None, stream=None,
                       out=None, mean_occupancy=False):
     """Per-window P, D, A, W ([K][M] int32 CUDA tensors) from request records or
-    token events (dicts of CUDA tensors). With mean_occupancy (request records
-    only) also A_ms, W_ms: int64 request-milliseconds running / waiting per
-    window; a dict holding them makes tss_score use the window means."""
+    token events (dicts of CUDA tensors). With mean_occupancy also A_ms, W_ms:
+    int64 request-milliseconds running / waiting per window; a dict holding
+    them makes tss_score use the window means."""
     torch = _torch()
     lib = load()
     g = Grid(M, window_ms, K)
@@ -334,40 +341,77 @@ def tss_rank(Z, cls, window_ms=1000, recv=True, donors=True, stream=None):
     return {"recv": rv, "donors": dn}
 
 
-def tss_stage_gauges(M, window_ms, K, requests, stream=None):
+def tss_stage_gauges(M, window_ms, K, requests, diag=None, stream=None):
     """Running requests split at the first token, read at each window's last
-    millisecond: (A_prefill, A_decode) int32 [K][M]. Two reductions of the same
-    columns, with t_first passed as t_end (prefill: [t_start, t_first)) and as
-    t_start (decode: [t_first, t_end)); only their running gauges are kept."""
-    pre = tss_window_reduce(M, window_ms, K, requests=dict(requests,
-                                                           t_end_ms=requests["t_first_ms"]),
-                            stream=stream)
-    dec = tss_window_reduce(M, window_ms, K, requests=dict(requests,
-                                                           t_start_ms=requests["t_first_ms"]),
-                            stream=stream)
-    return pre["A"], dec["A"]
-
-
-def stage_counts(counts, A_prefill, A_decode):
-    """Inputs of the two stage signals: prefill (P, no decode tokens, A_prefill,
-    W) and decode (no prompt tokens, D, A_decode, nothing waiting)."""
+    millisecond: (A_prefill, A_decode) int32 [K][M] CUDA tensors."""
     torch = _torch()
-    zero = torch.zeros_like(counts["P"])
-    return ({"P": counts["P"], "D": zero, "A": A_prefill, "W": counts["W"]},
-            {"P": zero, "D": counts["D"], "A": A_decode, "W": zero})
+    lib = load()
+    g = Grid(M, window_ms, K)
+    A_p = torch.empty((K, M), dtype=torch.int32, device="cuda")
+    A_d = torch.empty((K, M), dtype=torch.int32, device="cuda")
+    diag = new_diag() if diag is None else diag
+    rq = requests_struct(requests)
+    s = _stream(stream)
+    _workspace("tss_stage_gauges", lambda ws, n: lib.tss_stage_gauges(
+        C.byref(g), C.byref(rq), _ptr(A_p), _ptr(A_d), ws, n, _ptr(diag), s))
+    return A_p, A_d
+
+
+def tss_stage_calibrate(counts, A_prefill, A_decode, profile, window_ms, slo_ttft_ms,
+                        slo_tpot_ms, requests, dtype="f32", ok_frac=0.95, reliability=0.95,
+                        diag=None, stream=None):
+    """theta of the prefill signal (against TTFT) and of the decode signal
+    (against TPOT): two CUDA tensors of dtype [M]."""
+    torch = _torch()
+    lib = load()
+    K, M = counts["P"].shape
+    code, tdt = _dt(dtype)
+    g = Grid(M, window_ms, K)
+    pst, keep = _profile(profile, M, tdt, code)
+    i32 = lambda a: (a if torch.is_tensor(a) else torch.as_tensor(np.asarray(a, np.int32))).to(
+        device="cuda", dtype=torch.int32).contiguous()
+    ttft, tpot = i32(slo_ttft_ms), i32(slo_tpot_ms)
+    for t, what in ((A_prefill, "A_prefill"), (A_decode, "A_decode")):
+        _need(t, "int32", K * M, what)
+    th_p = torch.empty(M, dtype=tdt, device="cuda")
+    th_d = torch.empty(M, dtype=tdt, device="cuda")
+    diag = new_diag() if diag is None else diag
+    rq = requests_struct(requests)
+    cs = _counts(counts)
+    s = _stream(stream)
+    _workspace("tss_stage_calibrate", lambda ws, n: lib.tss_stage_calibrate(
+        C.byref(g), C.byref(rq), C.byref(cs), _ptr(A_prefill), _ptr(A_decode), C.byref(pst),
+        _ptr(ttft), _ptr(tpot), C.c_double(ok_frac), C.c_double(reliability), _ptr(th_p),
+        _ptr(th_d), ws, n, _ptr(diag), s))
+    return th_p, th_d
 
 
 def tss_stage_score(counts, A_prefill, A_decode, profile, window_ms, theta_prefill,
-                    theta_decode, dtype="f32", stream=None):
+                    theta_decode, dtype="f32", diag=None, stream=None):
     """Stage-aware signal: prefill TSS = (P/dt) / max(A_prefill + w_q W, 1) and
     decode TSS = (D/dt) / max(A_decode, 1), each smoothed and normalised by its
-    own theta. Returns (prefill, decode) dicts as tss_score does."""
-    pre, dec = stage_counts(counts, A_prefill, A_decode)
-    p = tss_score(pre, dict(profile, w_p=1.0, theta=theta_prefill), window_ms, dtype=dtype,
-                  stream=stream)
-    d = tss_score(dec, dict(profile, theta=theta_decode), window_ms, dtype=dtype,
-                  stream=stream)
-    return p, d
+    own theta. Returns (prefill, decode) dicts of S, Z, cls."""
+    torch = _torch()
+    lib = load()
+    K, M = counts["P"].shape
+    code, tdt = _dt(dtype)
+    g = Grid(M, window_ms, K)
+    pst, keep = _profile(profile, M, tdt, code)
+    th = [(t if torch.is_tensor(t) else torch.as_tensor(np.asarray(t))).to(
+        device="cuda", dtype=tdt).contiguous() for t in (theta_prefill, theta_decode)]
+    for t, what in ((A_prefill, "A_prefill"), (A_decode, "A_decode")):
+        _need(t, "int32", K * M, what)
+    out = [{"S": torch.empty((K, M), dtype=tdt, device="cuda"),
+            "Z": torch.empty((K, M), dtype=tdt, device="cuda"),
+            "cls": torch.empty((K, M), dtype=torch.uint8, device="cuda")} for _ in range(2)]
+    diag = new_diag() if diag is None else diag
+    cs = _counts(counts)
+    s = _stream(stream)
+    _workspace("tss_stage_score", lambda ws, n: lib.tss_stage_score(
+        C.byref(g), C.byref(cs), _ptr(A_prefill), _ptr(A_decode), C.byref(pst), _ptr(th[0]),
+        _ptr(th[1]), _ptr(out[0]["S"]), _ptr(out[0]["Z"]), _ptr(out[0]["cls"]), _ptr(out[1]["S"]),
+        _ptr(out[1]["Z"]), _ptr(out[1]["cls"]), ws, n, _ptr(diag), s))
+    return out[0], out[1]
 
 
 def tss_calibrate(counts, profile, window_ms, slo_ttft_ms, requests=None, events=None,

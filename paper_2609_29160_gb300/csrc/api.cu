@@ -483,6 +483,107 @@ tre_status sweep_typed(const tre_sweep_spec* sp, const SweepPlan& pl, const tre_
 
 }  // namespace
 
+namespace {
+
+// ---- stage-aware signal (Sec. VIII) ----------------------------------------
+template <class T>
+tre_status stage_calibrate_typed(const tre_grid* g, const tre_requests* req, const tre_counts* in,
+                                 const int32_t* A_pre, const int32_t* A_dec,
+                                 const tre_profile* p, const int32_t* ttft_ms,
+                                 const int32_t* tpot_ms, double ok_frac, double rel,
+                                 void* th_pre, void* th_dec, void* ws, size_t* ws_bytes,
+                                 tre_diag* diag, cudaStream_t s) {
+  const int M = g->n_models, K = g->n_windows;
+  const size_t cells = (size_t)K * M;
+  SeriesTable<T> tab = single_series<T>(g);
+  Arena a(ws);
+  unsigned long long* ttft = a.take<unsigned long long>(cells);
+  unsigned long long* tpot = a.take<unsigned long long>(cells);
+  int32_t* zero = a.take<int32_t>(cells);
+  T* ones = a.take<T>((size_t)M);
+  T* S = a.take<T>(cells);
+  uint8_t* cls = a.take<uint8_t>(cells);
+  ScoreWs<T> sw;
+  score_ws_layout<T>(a, M, (int64_t)cells, tab.seg_base[1], sw);
+  CalibWs<T> cw;
+  calib_ws_layout<T>(a, (int64_t)cells, M, cw);
+  bool query;
+  tre_status st = ws_check(a, ws, ws_bytes, query);
+  if (st != TRE_OK || query) return st;
+  const T* w_p = static_cast<const T*>(p->w_p);
+  const T* w_q = static_cast<const T*>(p->w_q);
+  const T* alpha = static_cast<const T*>(p->alpha);
+  cudaError_t e;
+  {
+    Scope sc(kSlo, 1, s);
+    e = launch_stage_requests(cols_of(req), M, g->window_ms, K, nullptr, nullptr, ttft, tpot,
+                              ttft_ms, tpot_ms, s);
+  }
+  if (!e) e = cudaMemsetAsync(zero, 0, cells * sizeof(int32_t), s);
+  if (!e) e = launch_fill<T>(ones, M, (T)1, s);
+  // prefill: (P/dt) / max(A_prefill + w_q W, 1), calibrated on TTFT
+  if (!e) {
+    Scope sc(kScore, 6, s);
+    e = launch_score<T>(tab, in->P, zero, A_pre, in->W, ones, w_q, alpha, nullptr, nullptr,
+                        nullptr, nullptr, nullptr, S, nullptr, cls, sw, diag, s);
+  }
+  if (!e) {
+    Scope sc(kCalibrate, 3, s);
+    e = launch_calibrate<T>(tab, S, cls, ttft, ok_frac, rel, static_cast<T*>(th_pre), cw, diag, s);
+  }
+  // decode: (D/dt) / max(A_decode, 1), calibrated on TPOT
+  if (!e) {
+    Scope sc(kScore, 6, s);
+    e = launch_score<T>(tab, zero, in->D, A_dec, zero, w_p, w_q, alpha, nullptr, nullptr,
+                        nullptr, nullptr, nullptr, S, nullptr, cls, sw, diag, s);
+  }
+  if (!e) {
+    Scope sc(kCalibrate, 3, s);
+    e = launch_calibrate<T>(tab, S, cls, tpot, ok_frac, rel, static_cast<T*>(th_dec), cw, diag, s);
+  }
+  return cuda_status(e);
+}
+
+template <class T>
+tre_status stage_score_typed(const tre_grid* g, const tre_counts* in, const int32_t* A_pre,
+                             const int32_t* A_dec, const tre_profile* p, const void* th_pre,
+                             const void* th_dec, void* S_pre, void* Z_pre, uint8_t* cls_pre,
+                             void* S_dec, void* Z_dec, uint8_t* cls_dec, void* ws,
+                             size_t* ws_bytes, tre_diag* diag, cudaStream_t s) {
+  const int M = g->n_models, K = g->n_windows;
+  const size_t cells = (size_t)K * M;
+  SeriesTable<T> tab = single_series<T>(g);
+  Arena a(ws);
+  int32_t* zero = a.take<int32_t>(cells);
+  T* ones = a.take<T>((size_t)M);
+  ScoreWs<T> sw;
+  score_ws_layout<T>(a, M, (int64_t)cells, tab.seg_base[1], sw);
+  bool query;
+  tre_status st = ws_check(a, ws, ws_bytes, query);
+  if (st != TRE_OK || query) return st;
+  const T* w_q = static_cast<const T*>(p->w_q);
+  const T* alpha = static_cast<const T*>(p->alpha);
+  const T* tc = static_cast<const T*>(p->tau_crit);
+  const T* tsu = static_cast<const T*>(p->tau_surplus);
+  cudaError_t e = cudaMemsetAsync(zero, 0, cells * sizeof(int32_t), s);
+  if (!e) e = launch_fill<T>(ones, M, (T)1, s);
+  if (!e) {
+    Scope sc(kScore, 6, s);
+    e = launch_score<T>(tab, in->P, zero, A_pre, in->W, ones, w_q, alpha,
+                        static_cast<const T*>(th_pre), tc, tsu, nullptr, nullptr,
+                        static_cast<T*>(S_pre), static_cast<T*>(Z_pre), cls_pre, sw, diag, s);
+  }
+  if (!e) {
+    Scope sc(kScore, 6, s);
+    e = launch_score<T>(tab, zero, in->D, A_dec, zero, static_cast<const T*>(p->w_p), w_q,
+                        alpha, static_cast<const T*>(th_dec), tc, tsu, nullptr, nullptr,
+                        static_cast<T*>(S_dec), static_cast<T*>(Z_dec), cls_dec, sw, diag, s);
+  }
+  return cuda_status(e);
+}
+
+}  // namespace
+
 extern "C" {
 
 void tre_trace_enable(int on) {
@@ -530,7 +631,6 @@ tre_status tss_window_reduce(const tre_grid* grid, const tre_requests* req, cons
   if (!grid_ok(grid) || !ws_bytes || (!req) == (!ev)) return TRE_EINVAL;
   if (req ? !req_ok(req) : !ev_ok(ev)) return TRE_EINVAL;
   if (!counts_ok(&out)) return TRE_EINVAL;
-  if (out.A_ms && !req) return TRE_EINVAL;   // time-averaged occupancy: request records only
   if (ws && !diag) return TRE_EINVAL;
   const int M = grid->n_models, K = grid->n_windows;
   Arena a(ws);
@@ -553,8 +653,10 @@ tre_status tss_window_reduce(const tre_grid* grid, const tre_requests* req, cons
     e = launch_gauge_scan(M, K, w, out.A, out.W, s);
   }
   if (!e && out.A_ms) {
-    Scope sc(kOccupancy, 3 + (req->n > 0), s);
-    e = launch_occupancy_mean(cols_of(req), M, grid->window_ms, K, w, out.A_ms, out.W_ms, s);
+    Scope sc(kOccupancy, 3 + (req ? req->n > 0 : ev->n_req > 0), s);
+    e = req ? launch_occupancy_mean(cols_of(req), M, grid->window_ms, K, w, out.A_ms, out.W_ms, s)
+            : launch_occupancy_mean_events(cols_of(ev), M, grid->window_ms, K, w, out.A_ms,
+                                           out.W_ms, s);
   }
   return cuda_status(e);
 }
@@ -636,6 +738,81 @@ tre_status tre_sweep(const tre_sweep_spec* spec, const tre_sweep_out* out, void*
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (spec->dtype == TRE_F32) return sweep_typed<float>(spec, pl, out, ws, ws_bytes, diag, s);
   return sweep_typed<double>(spec, pl, out, ws, ws_bytes, diag, s);
+}
+
+tre_status tss_stage_gauges(const tre_grid* grid, const tre_requests* req, int32_t* A_prefill,
+                            int32_t* A_decode, void* ws, size_t* ws_bytes, tre_diag* diag,
+                            tre_stream stream) {
+  if (!grid_ok(grid) || !ws_bytes || !req_ok(req) || !A_prefill || !A_decode) return TRE_EINVAL;
+  if (ws && !diag) return TRE_EINVAL;
+  const int M = grid->n_models, K = grid->n_windows;
+  Arena a(ws);
+  ReduceWs w;
+  reduce_ws_layout(a, M, K, 1, 0, w);
+  bool query;
+  tre_status st = ws_check(a, ws, ws_bytes, query);
+  if (st != TRE_OK || query) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e;
+  {
+    // the prefill differences take the running slot and the decode ones the
+    // waiting slot of the gauge scan
+    Scope sc(kReduce, 1, s);
+    e = launch_stage_requests(cols_of(req), M, grid->window_ms, K, w.dA, w.dW, nullptr, nullptr,
+                              nullptr, nullptr, s);
+  }
+  if (!e) {
+    Scope sc(kScan, 3, s);
+    e = launch_gauge_scan(M, K, w, A_prefill, A_decode, s);
+  }
+  return cuda_status(e);
+}
+
+tre_status tss_stage_calibrate(const tre_grid* grid, const tre_requests* req,
+                               const tre_counts* in, const int32_t* A_prefill,
+                               const int32_t* A_decode, const tre_profile* prof,
+                               const int32_t* slo_ttft_ms, const int32_t* slo_tpot_ms,
+                               double ok_frac, double reliability, void* theta_prefill,
+                               void* theta_decode, void* ws, size_t* ws_bytes, tre_diag* diag,
+                               tre_stream stream) {
+  if (!grid_ok(grid) || !ws_bytes || !req_ok(req) || !counts_ok(in) || in->A_ms ||
+      !prof_ok(prof, false))
+    return TRE_EINVAL;
+  if (!A_prefill || !A_decode || !slo_ttft_ms || !slo_tpot_ms || !theta_prefill || !theta_decode)
+    return TRE_EINVAL;
+  if (ws && !diag) return TRE_EINVAL;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (prof->dtype == TRE_F32)
+    return stage_calibrate_typed<float>(grid, req, in, A_prefill, A_decode, prof, slo_ttft_ms,
+                                        slo_tpot_ms, ok_frac, reliability, theta_prefill,
+                                        theta_decode, ws, ws_bytes, diag, s);
+  return stage_calibrate_typed<double>(grid, req, in, A_prefill, A_decode, prof, slo_ttft_ms,
+                                       slo_tpot_ms, ok_frac, reliability, theta_prefill,
+                                       theta_decode, ws, ws_bytes, diag, s);
+}
+
+tre_status tss_stage_score(const tre_grid* grid, const tre_counts* in, const int32_t* A_prefill,
+                           const int32_t* A_decode, const tre_profile* prof,
+                           const void* theta_prefill, const void* theta_decode, void* S_prefill,
+                           void* Z_prefill, uint8_t* cls_prefill, void* S_decode, void* Z_decode,
+                           uint8_t* cls_decode, void* ws, size_t* ws_bytes, tre_diag* diag,
+                           tre_stream stream) {
+  if (!grid_ok(grid) || !ws_bytes || !counts_ok(in) || in->A_ms || !prof_ok(prof, false))
+    return TRE_EINVAL;
+  if (!prof->tau_crit || !prof->tau_surplus || !A_prefill || !A_decode || !theta_prefill ||
+      !theta_decode)
+    return TRE_EINVAL;
+  if (!S_prefill || !Z_prefill || !cls_prefill || !S_decode || !Z_decode || !cls_decode)
+    return TRE_EINVAL;
+  if (ws && !diag) return TRE_EINVAL;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (prof->dtype == TRE_F32)
+    return stage_score_typed<float>(grid, in, A_prefill, A_decode, prof, theta_prefill,
+                                    theta_decode, S_prefill, Z_prefill, cls_prefill, S_decode,
+                                    Z_decode, cls_decode, ws, ws_bytes, diag, s);
+  return stage_score_typed<double>(grid, in, A_prefill, A_decode, prof, theta_prefill,
+                                   theta_decode, S_prefill, Z_prefill, cls_prefill, S_decode,
+                                   Z_decode, cls_decode, ws, ws_bytes, diag, s);
 }
 
 }  // extern "C"

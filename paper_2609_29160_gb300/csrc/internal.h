@@ -105,6 +105,10 @@ cudaError_t launch_gauge_scan(int M, int K, ReduceWs& w, int32_t* A, int32_t* W,
 // diff and partial arrays of w (call after the gauge scan of the same trace)
 cudaError_t launch_occupancy_mean(const ReqCols& r, int M, int win, int K, ReduceWs& w,
                                   int64_t* A_ms, int64_t* W_ms, cudaStream_t s);
+// The same for token events: spans from the per-request first/last ticks the
+// event reduction left in w (call after launch_reduce_events and the gauge scan)
+cudaError_t launch_occupancy_mean_events(const EvCols& ev, int M, int win, int K, ReduceWs& w,
+                                         int64_t* A_ms, int64_t* W_ms, cudaStream_t s);
 // exact coarsening of every trace's base grid to every window length: counts
 // add over q base windows, gauges are read at the last base window
 struct AggPlan {
@@ -134,6 +138,19 @@ cudaError_t launch_aggregate(const AggPlan& plan, const int32_t* P, const int32_
                              const int32_t* A, const int32_t* W, const unsigned long long* slo,
                              int32_t* Pq, int32_t* Dq, int32_t* Aq, int32_t* Wq,
                              unsigned long long* sloq, cudaStream_t s);
+
+// ---- stage.cu -------------------------------------------------------------
+// One pass over request records kept by the reduction's rules: the +1/-1
+// window differences of the running gauge split at the first token (prefill
+// [t_start, t_first) into dPre, decode [t_first, t_end) into dDec, each
+// [K+1][M], cleared here; both null = skipped) and the packed TTFT and TPOT
+// calibration counts at the arrival window (count + met << 32, [K][M], cleared
+// here; both null = skipped).
+cudaError_t launch_stage_requests(const ReqCols& r, int M, int win, int K, int32_t* dPre,
+                                  int32_t* dDec, unsigned long long* ttft,
+                                  unsigned long long* tpot, const int32_t* ttft_ms,
+                                  const int32_t* tpot_ms, cudaStream_t s);
+template <class T> cudaError_t launch_fill(T* p, int64_t n, T v, cudaStream_t s);
 
 // ---- series tables ----------------------------------------------------------
 // A batch of series (one per (trace, window length) in a sweep, one for the

@@ -1292,6 +1292,63 @@ k_occ_apply(int M, int K, int L, int n_chunks, int win, const int32_t* __restric
   }
 }
 
+// Time-averaged occupancy of token events: per request with at least one
+// valid event (first/last tick from the event pass) and 0 <= t_arr <= first,
+// waiting on [t_arr, first) and running on [first, last), cut at the end of the
+// grid. One thread per request (the request table is small beside the event
+// stream): partial first and last windows are added to the 64-bit sums, the
+// windows a span covers completely are marked +1/-1 in the difference arrays.
+__global__ void __launch_bounds__(kThreads)
+k_occ_events(EvCols ev, int M, int win, FastDiv fd, int K, const int32_t* __restrict__ first,
+             const int32_t* __restrict__ last, unsigned long long* __restrict__ pA,
+             unsigned long long* __restrict__ pW, int32_t* __restrict__ fA,
+             int32_t* __restrict__ fW) {
+  const uint32_t span = (uint32_t)K * (uint32_t)win, uw = (uint32_t)win;
+  for (int64_t r = (int64_t)blockIdx.x * kThreads + threadIdx.x; r < ev.n_req;
+       r += (int64_t)gridDim.x * kThreads) {
+    const int32_t lt = last[r];
+    if (lt < 0) continue;
+    const int m = ev.req_model[r];
+    const int32_t ta = ev.req_t_arr[r], f = first[r];
+    if (m < 0 || m >= M || ta < 0 || ta > f) continue;
+    auto add_span = [&](uint32_t a, uint32_t e, unsigned long long* part, int32_t* full) {
+      e = min(e, span);
+      if (a >= e) return;
+      const uint32_t k0 = fd.div(a), k1 = fd.div(e - 1);
+      if (k0 == k1) {
+        atomicAdd(&part[(size_t)k0 * M + m], (unsigned long long)(e - a));
+        return;
+      }
+      atomicAdd(&part[(size_t)k0 * M + m], (unsigned long long)((k0 + 1) * uw - a));
+      atomicAdd(&part[(size_t)k1 * M + m], (unsigned long long)(e - k1 * uw));
+      if (k1 > k0 + 1) {
+        atomicAdd(&full[(size_t)(k0 + 1) * M + m], 1);
+        atomicAdd(&full[(size_t)k1 * M + m], -1);
+      }
+    };
+    add_span((uint32_t)ta, (uint32_t)f, pW, fW);
+    add_span((uint32_t)f, (uint32_t)lt, pA, fA);
+  }
+}
+
+// last step of both occupancy passes: the covered-window counts (inclusive
+// prefix of the difference arrays) times the window length added to the
+// partial sums
+cudaError_t occ_finish(int M, int win, int K, ReduceWs& w, int64_t* A_ms, int64_t* W_ms,
+                       cudaStream_t s) {
+  const int L = scan_chunk_rows(K);
+  const int n_chunks = (K + L - 1) / L;
+  const int64_t segs = (int64_t)n_chunks * M;
+  const unsigned g = (unsigned)((segs + kThreads - 1) / kThreads);
+  k_scan_partials<<<dim3(g, 1), kThreads, 0, s>>>(M, K, L, n_chunks, w.dA, w.dW, w.partA,
+                                                  w.partW);
+  k_scan_chunks<<<dim3(M, 1), 1024, 0, s>>>(M, n_chunks, w.partA, w.partW);
+  k_occ_apply<<<g, kThreads, 0, s>>>(M, K, L, n_chunks, win, w.dA, w.dW, w.partA, w.partW,
+                                     reinterpret_cast<long long*>(A_ms),
+                                     reinterpret_cast<long long*>(W_ms));
+  return cudaGetLastError();
+}
+
 cudaError_t launch_occupancy_mean(const ReqCols& r, int M, int win, int K, ReduceWs& w,
                                   int64_t* A_ms, int64_t* W_ms, cudaStream_t s) {
   if (K == 0) return cudaSuccess;
@@ -1328,17 +1385,26 @@ cudaError_t launch_occupancy_mean(const ReqCols& r, int M, int win, int K, Reduc
                                               reinterpret_cast<unsigned long long*>(W_ms), w.dA,
                                               w.dW);
   }
-  const int L = scan_chunk_rows(K);
-  const int n_chunks = (K + L - 1) / L;
-  const int64_t segs = (int64_t)n_chunks * M;
-  const unsigned g = (unsigned)((segs + kThreads - 1) / kThreads);
-  k_scan_partials<<<dim3(g, 1), kThreads, 0, s>>>(M, K, L, n_chunks, w.dA, w.dW, w.partA,
-                                                  w.partW);
-  k_scan_chunks<<<dim3(M, 1), 1024, 0, s>>>(M, n_chunks, w.partA, w.partW);
-  k_occ_apply<<<g, kThreads, 0, s>>>(M, K, L, n_chunks, win, w.dA, w.dW, w.partA, w.partW,
-                                     reinterpret_cast<long long*>(A_ms),
-                                     reinterpret_cast<long long*>(W_ms));
-  return cudaGetLastError();
+  return occ_finish(M, win, K, w, A_ms, W_ms, s);
+}
+
+cudaError_t launch_occupancy_mean_events(const EvCols& ev, int M, int win, int K, ReduceWs& w,
+                                         int64_t* A_ms, int64_t* W_ms, cudaStream_t s) {
+  if (K == 0) return cudaSuccess;
+  const size_t cells = (size_t)K * M, cells1 = (size_t)(K + 1) * M;
+  cudaError_t e = cudaMemsetAsync(A_ms, 0, cells * sizeof(int64_t), s);
+  if (!e) e = cudaMemsetAsync(W_ms, 0, cells * sizeof(int64_t), s);
+  if (!e) e = cudaMemsetAsync(w.dA, 0, cells1 * sizeof(int32_t), s);
+  if (!e) e = cudaMemsetAsync(w.dW, 0, cells1 * sizeof(int32_t), s);
+  if (e) return e;
+  if (ev.n_req > 0) {
+    k_occ_events<<<grid_for(ev.n_req, 4), kThreads, 0, s>>>(
+        ev, M, win, FastDiv(win), K, w.first, w.last,
+        reinterpret_cast<unsigned long long*>(A_ms), reinterpret_cast<unsigned long long*>(W_ms),
+        w.dA, w.dW);
+    if ((e = cudaGetLastError())) return e;
+  }
+  return occ_finish(M, win, K, w, A_ms, W_ms, s);
 }
 
 cudaError_t launch_gauge_prefix(const GaugePlan& gp, ReduceWs& w, cudaStream_t s) {

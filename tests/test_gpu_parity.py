@@ -374,11 +374,72 @@ def test_mean_occupancy_empty_and_refusals(tre):
     empty = {k: torch.zeros(0, dtype=torch.int32, device="cuda") for k in REQ_KEYS}
     c = tre.tss_window_reduce(M, win, K, requests=empty, mean_occupancy=True)
     assert int(c["A_ms"].abs().sum()) == 0 and int(c["W_ms"].abs().sum()) == 0
-    # token events cannot give the time-averaged occupancy
-    w = _events_case(3)
-    with pytest.raises(tre.TreError):
-        tre.tss_window_reduce(w["M"], w["window_ms"], w["K"], events=_cuda(w["events"]),
-                              mean_occupancy=True)
+    ev = {"model": torch.zeros(0, dtype=torch.int32, device="cuda"),
+          "req": torch.zeros(0, dtype=torch.int32, device="cuda"),
+          "t_s": torch.zeros(0, dtype=torch.float32, device="cuda"),
+          "phase": torch.zeros(0, dtype=torch.uint8, device="cuda"),
+          "req_model": torch.zeros(3, dtype=torch.int32, device="cuda"),
+          "req_t_arr_ms": torch.zeros(3, dtype=torch.int32, device="cuda"),
+          "req_ttft_ms": torch.zeros(3, dtype=torch.int32, device="cuda")}
+    c = tre.tss_window_reduce(M, win, K, events=ev, mean_occupancy=True)
+    assert int(c["A_ms"].abs().sum()) == 0 and int(c["W_ms"].abs().sum()) == 0
+
+
+def _corrupt_events(ev, rng, M):
+    ev = {k: v.copy() for k, v in ev.items()}
+    n = len(ev["model"])
+    idx = rng.choice(n, n // 50, replace=False)
+    q = len(idx) // 4
+    ev["t_s"][idx[:q]] = np.float32(-1.0)
+    ev["t_s"][idx[q: 2 * q]] = np.float32(np.nan)
+    ev["phase"][idx[2 * q: 3 * q]] = 7
+    ev["model"][idx[3 * q:]] = (ev["model"][idx[3 * q:]] + 1) % M
+    ev["req_t_arr_ms"][rng.choice(len(ev["req_model"]), 20)] = 10 ** 9
+    perm = rng.permutation(n)
+    for k in ("model", "req", "t_s", "phase"):
+        ev[k] = ev[k][perm]
+    return ev
+
+
+@pytest.mark.parametrize("seed,corrupt", [(7, False), (8, True)])
+def test_mean_occupancy_token_events(tre, seed, corrupt):
+    """Time-averaged occupancy from token events (running from a request's first
+    to its last valid event, waiting from its arrival to its first), on a
+    time-sorted stream and on a shuffled stream with corrupt events."""
+    w = _events_case(seed)
+    ev, M, win, K = w["events"], w["M"], w["window_ms"], w["K"]
+    if corrupt:
+        ev = _corrupt_events(ev, np.random.default_rng(seed), M)
+    A_ms, W_ms = oracle.occupancy_mean_events(ev, M, win, K)
+    c = tre.tss_window_reduce(M, win, K, events=_cuda(ev), mean_occupancy=True)
+    np.testing.assert_array_equal(_np(c["A_ms"]), A_ms)
+    np.testing.assert_array_equal(_np(c["W_ms"]), W_ms)
+    P, D, A, W, _ = oracle.reduce_events(ev, M, win, K)
+    for k, ref in zip("PDAW", (P, D, A, W)):
+        np.testing.assert_array_equal(_np(c[k]), ref, err_msg=k)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f64"])
+def test_mean_occupancy_token_events_pipeline(tre, dtype):
+    """Calibration and scoring with the event-form window means in Eq. 1's
+    demand term."""
+    w = _events_case(9)
+    ev, M, win, K = w["events"], w["M"], w["window_ms"], w["K"]
+    npdt = np.float32 if dtype == "f32" else np.float64
+    prof = tracegen.default_profile(M, win)
+    P, D, A, W, _ = oracle.reduce_events(ev, M, win, K)
+    occ = oracle.occupancy_mean_events(ev, M, win, K)
+    n_arr, n_met = oracle.slo_counts_events(ev, M, win, K, w["slo_ttft_ms"])
+    S, _, cls, _ = oracle.score(P, D, A, W, prof, win, npdt, occ_ms=occ)
+    theta, _ = oracle.calibrate(S, cls, n_arr, n_met)
+    S, Z, cls, recv = oracle.score(P, D, A, W, dict(prof, theta=theta), win, npdt, occ_ms=occ)
+    evc = _cuda(ev)
+    c = tre.tss_window_reduce(M, win, K, events=evc, mean_occupancy=True)
+    th = tre.tss_calibrate(c, prof, win, w["slo_ttft_ms"], events=evc, dtype=dtype)
+    np.testing.assert_array_equal(_np(th), theta)
+    sc = tre.tss_score(c, dict(prof, theta=th), win, dtype=dtype)
+    for k, ref in (("S", S), ("Z", Z), ("cls", cls), ("recv", recv)):
+        np.testing.assert_array_equal(_np(sc[k]), ref, err_msg=k)
 
 
 def test_class_models_mapping(tre):
@@ -434,15 +495,46 @@ def test_stage_signal(tre, dtype):
     np.testing.assert_array_equal(_np(A_p), o["A_prefill"])
     np.testing.assert_array_equal(_np(A_d), o["A_decode"])
     c = tre.tss_window_reduce(M, win, K, requests=req)
-    pre, _ = tre.stage_counts(c, A_p, A_d)
-    theta_p = tre.tss_calibrate(pre, dict(prof, w_p=1.0), win, w["slo_ttft_ms"], requests=req,
-                                dtype=dtype)
+    diag = tre.new_diag()
+    theta_p, theta_d = tre.tss_stage_calibrate(c, A_p, A_d, prof, win, w["slo_ttft_ms"], tpot,
+                                               req, dtype=dtype, diag=diag)
     np.testing.assert_array_equal(_np(theta_p), o["prefill"]["theta"])
-    sp, sd = tre.tss_stage_score(c, A_p, A_d, prof, win, theta_p, o["decode"]["theta"],
-                                 dtype=dtype)
+    np.testing.assert_array_equal(_np(theta_d), o["decode"]["theta"])
+    assert tre.read_diag(diag)["degenerate_calib"] == \
+        o["prefill"]["degenerate"] + o["decode"]["degenerate"]
+    sp, sd = tre.tss_stage_score(c, A_p, A_d, prof, win, theta_p, theta_d, dtype=dtype)
     for k in ("S", "Z", "cls"):
         np.testing.assert_array_equal(_np(sp[k]), o["prefill"][k], err_msg="prefill " + k)
         np.testing.assert_array_equal(_np(sd[k]), o["decode"][k], err_msg="decode " + k)
+
+
+@pytest.mark.parametrize("seed,M,win,K", [(41, 5, 1000, 120), (42, 64, 100, 900)])
+def test_stage_signal_adversarial(tre, seed, M, win, K):
+    """Records on window boundaries, one output token (no TPOT count), spans
+    past the grid, bad ids and order violations; TPOT bounds hit exactly."""
+    rng = np.random.default_rng(seed)
+    req = _adversarial(rng, 30000, M, win, K)
+    tpot = rng.integers(1, 40, M).astype(np.int32)
+    ok = (req["L_out"] > 1) & (rng.random(len(req["L_out"])) < 0.2)
+    te = req["t_first_ms"].astype(np.int64) + tpot[np.clip(req["model"], 0, M - 1)].astype(
+        np.int64) * (req["L_out"].astype(np.int64) - 1)
+    req["t_end_ms"] = np.where(ok & (te < 2 ** 31 - 1), te, req["t_end_ms"]).astype(np.int32)
+    slo = rng.integers(100, 3000, M).astype(np.int32)
+    prof = tracegen.default_profile(M, win)
+    for dtype, npdt in (("f32", np.float32), ("f64", np.float64)):
+        o = oracle.stage_pipeline(req, M, win, K, prof, slo, tpot, npdt)
+        rc = _cuda(req)
+        A_p, A_d = tre.tss_stage_gauges(M, win, K, rc)
+        np.testing.assert_array_equal(_np(A_p), o["A_prefill"])
+        np.testing.assert_array_equal(_np(A_d), o["A_decode"])
+        c = tre.tss_window_reduce(M, win, K, requests=rc)
+        th_p, th_d = tre.tss_stage_calibrate(c, A_p, A_d, prof, win, slo, tpot, rc, dtype=dtype)
+        np.testing.assert_array_equal(_np(th_p), o["prefill"]["theta"])
+        np.testing.assert_array_equal(_np(th_d), o["decode"]["theta"])
+        sp, sd = tre.tss_stage_score(c, A_p, A_d, prof, win, th_p, th_d, dtype=dtype)
+        for k in ("S", "Z", "cls"):
+            np.testing.assert_array_equal(_np(sp[k]), o["prefill"][k], err_msg="prefill " + k)
+            np.testing.assert_array_equal(_np(sd[k]), o["decode"][k], err_msg="decode " + k)
 
 
 def test_calibrate_events(tre):

@@ -134,7 +134,7 @@ def test_mean_occupancy_arguments_are_checked_on_the_host():
                                  None, None) == 1
     both = tre.Counts(1, 1, 1, 1, 1, 1)
     assert lib.tss_window_reduce(C.byref(g), None, C.byref(ev), both, None, C.byref(n), None,
-                                 None) == 1              # token events: no window means
+                                 None) == 0              # token events: workspace query
     assert lib.tss_window_reduce(C.byref(g), C.byref(rq), None, both, None, C.byref(n), None,
                                  None) == 0              # workspace query
 
@@ -166,3 +166,27 @@ def test_binding_checks_tensor_arguments():
         tre._counts(dict(cnt, A_ms=torch.zeros((3, 2), dtype=torch.int32),
                          W_ms=torch.zeros((3, 2), dtype=torch.int64)))
 
+
+
+def test_stage_arguments_are_checked_on_the_host():
+    lib = tre.load()
+    g = tre.Grid(3, 1000, 10)
+    n = C.c_size_t(0)
+    rq = tre.Requests(0)
+    p = C.c_void_p(16)          # never dereferenced: the checks fail first
+    assert lib.tss_stage_gauges(C.byref(g), C.byref(rq), p, None, None, C.byref(n), None,
+                                None) == 1              # A_decode missing
+    assert lib.tss_stage_gauges(C.byref(g), C.byref(rq), p, p, None, C.byref(n), None,
+                                None) == 0              # workspace query
+    cs = tre.Counts(16, 16, 16, 16, 16, 16)             # window means: not for stages
+    prof = tre.Profile(0, 16, 16, 16, 16, 16, 16)
+    assert lib.tss_stage_score(C.byref(g), C.byref(cs), p, p, C.byref(prof), p, p, p, p, p, p,
+                               p, p, None, C.byref(n), None, None) == 1
+    cs = tre.Counts(16, 16, 16, 16)
+    assert lib.tss_stage_score(C.byref(g), C.byref(cs), p, p, C.byref(prof), p, p, p, p, p, p,
+                               p, p, None, C.byref(n), None, None) == 0
+    assert lib.tss_stage_calibrate(C.byref(g), C.byref(rq), C.byref(cs), p, p, C.byref(prof), p,
+                                   None, 0.95, 0.95, p, p, None, C.byref(n), None,
+                                   None) == 1           # TPOT bounds missing
+    assert lib.tss_stage_calibrate(C.byref(g), C.byref(rq), C.byref(cs), p, p, C.byref(prof), p,
+                                   p, 0.95, 0.95, p, p, None, C.byref(n), None, None) == 0
