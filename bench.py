@@ -505,7 +505,7 @@ def measure_configs(tre, lib, Trace, hbm, peak_kind, with_cpu):
     return out
 
 
-TRACE_PHASES = 10   # phases of tre_trace (the library header's count)
+TRACE_PHASES = 11   # phases of tre_trace (the library header's count)
 
 
 def occupancy_cpu(scale):

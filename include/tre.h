@@ -379,6 +379,84 @@ typedef struct {
 tre_status tre_sweep(const tre_sweep_spec* spec, const tre_sweep_out* out, void* ws,
                      size_t* ws_bytes, tre_diag* diag, tre_stream stream);
 
+/*
+ * Closed-loop replay (Sec. IV-B: rescue and rebalance act on live capacity;
+ * Sec. IV-C: bounded transfer; Sec. VI-D: measured sleep and wake latencies).
+ * The controller's moves change the servers that serve the requests, and the
+ * telemetry it scores comes from the requests as they are served:
+ *  - each routable replica of a model is one server; a model's requests are
+ *    served in input order (FCFS when sorted by arrival) by whichever of its
+ *    servers frees first; once started a request needs d_first_ms to its first
+ *    token and d_total_ms to its last;
+ *  - window k is processed at T = (k+1)*window_ms: every request that can start
+ *    before T starts, then window k's telemetry (tss_window_reduce's token
+ *    attribution and gauges) is scored as tss_score scores it, with the
+ *    smoothing carried across windows, and on a control tick the controller of
+ *    tre_select_moves acts on the replica counts as they are;
+ *  - a transition commits at its tick; each donor replica it releases is the
+ *    donor's server that frees first: it takes no request from T on, finishes
+ *    the request it serves (drain) and returns its GPU sleep_ms later; the
+ *    receiver's new server starts waking when its GPU is free -- at T when the
+ *    idle pool paid, else when the transition's last released donor replica
+ *    has returned its GPU -- and serves wake_ms after that.
+ * A latent record is served when 0 <= model < n_models, 0 <= t_arr <
+ * n_windows*window_ms, 0 <= d_first <= d_total, L_in >= 0 and L_out >= 1.
+ */
+typedef struct {
+  int64_t n;                 /* < 2^31 */
+  const int32_t *model, *t_arr_ms, *d_first_ms, *d_total_ms, *L_in, *L_out;  /* device [n] */
+} tre_latent;
+
+/* Settings replayed side by side, instance i = t * n_cap + c. n_tau == 0: one
+ * threshold set, the profile's tau_crit per model; else tau_crit[t] (host) for
+ * every model. n_cap == 0: the control's pacing_cap; else pacing_cap[c] (host,
+ * 0..255). Limits: n_tau, n_cap <= 32. wake_ms, sleep_ms >= 0. */
+typedef struct {
+  int32_t n_tau;
+  const double* tau_crit;
+  int32_t n_cap;
+  const int32_t* pacing_cap;
+  int32_t wake_ms, sleep_ms;
+} tre_replay_spec;
+
+/* Replay outputs (device). Optional arrays may be NULL.
+ * t_start_ms, t_first_ms, t_end_ms: [n_inst][n] served times (all three or
+ *   none): K*window_ms for a request not started within the grid, -1 for a
+ *   record that is not served;
+ * Z (dtype), cls: [n_inst][n_windows][n_models] the signal the controller saw;
+ * moves [n_inst][moves_cap], n_moves [n_inst] (required; n_moves above
+ *   moves_cap sets diag.err = TRE_EOVERFLOW), r_final [n_inst][n_models]
+ *   (required);
+ * slo_met [n_inst][n_models]: served requests whose first token came within
+ *   slo_ttft_ms[m] of arrival, counting a request never started as getting it
+ *   at the end of the grid (needs slo_ttft_ms); served [n_inst][n_models]:
+ *   requests started within the grid. */
+typedef struct {
+  int32_t *t_start_ms, *t_first_ms, *t_end_ms;
+  void* Z;
+  uint8_t* cls;
+  tre_move* moves;
+  int64_t moves_cap;
+  int64_t* n_moves;
+  int32_t* r_final;
+  int64_t *slo_met, *served;
+} tre_replay_out;
+
+/*
+ * tre_replay -- the closed-loop replay of one latent trace for every setting of
+ * `spec` (NULL: one instance with the profile's thresholds, the control's
+ * pacing cap and no actuation delay). prof: w_p, w_q, alpha, theta, tau_crit,
+ * tau_surplus (device [n_models], all required); ctrl: budget (<= 65536),
+ * floors, footprints, cadences; r0: device int32[n_models] initial replicas.
+ * Limits: n_models <= 64. An inconsistent initial state (negative replicas or
+ * floors, footprints below one, more replicas than the budget holds) is found
+ * on the device: diag.err = TRE_EINVAL and nothing is replayed.
+ */
+tre_status tre_replay(const tre_grid* grid, const tre_latent* lat, const tre_profile* prof,
+                      const tre_ctrl* ctrl, const int32_t* r0, const tre_replay_spec* spec,
+                      const int32_t* slo_ttft_ms, const tre_replay_out* out, void* ws,
+                      size_t* ws_bytes, tre_diag* diag, tre_stream stream);
+
 /* Kernel-phase tracing (host side, not thread safe). While enabled, every
  * kernel phase an entry point enqueues is bracketed by a pair of CUDA events
  * recorded on the call's stream, so phases can be timed on the device inside
@@ -387,8 +465,9 @@ tre_status tre_sweep(const tre_sweep_spec* spec, const tre_sweep_out* out, void*
  * since tracing was enabled (or since the last collect), and starts over.
  * Phases: reduce, gauge_scan, aggregate, score, receiver, slo_counts,
  * calibrate, normalize, select, occupancy (the time-averaged occupancy pass of
- * tss_window_reduce). No counterpart in the paper (instrumentation). */
-#define TRE_TRACE_PHASES 10
+ * tss_window_reduce), replay (tre_replay). No counterpart in the paper
+ * (instrumentation). */
+#define TRE_TRACE_PHASES 11
 typedef struct {
   int32_t n_phases;
   const char* name[TRE_TRACE_PHASES];

@@ -80,6 +80,24 @@ class SweepOut(C.Structure):
         ("moves_cap", C.c_int64), ("n_moves", C.c_void_p), ("r_final", C.c_void_p)]
 
 
+class Latent(C.Structure):
+    _fields_ = [("n", C.c_int64)] + [(k, C.c_void_p) for k in (
+        "model", "t_arr_ms", "d_first_ms", "d_total_ms", "L_in", "L_out")]
+
+
+class ReplaySpec(C.Structure):
+    _fields_ = [("n_tau", C.c_int32), ("tau_crit", C.POINTER(C.c_double)), ("n_cap", C.c_int32),
+                ("pacing_cap", C.POINTER(C.c_int32)), ("wake_ms", C.c_int32),
+                ("sleep_ms", C.c_int32)]
+
+
+class ReplayOut(C.Structure):
+    _fields_ = [(k, C.c_void_p) for k in ("t_start_ms", "t_first_ms", "t_end_ms", "Z", "cls",
+                                          "moves")] + [
+        ("moves_cap", C.c_int64), ("n_moves", C.c_void_p), ("r_final", C.c_void_p),
+        ("slo_met", C.c_void_p), ("served", C.c_void_p)]
+
+
 MOVE_DTYPE = np.dtype([("window", np.int32), ("recv", np.int16), ("donor", np.int16),
                        ("kind", np.uint8), ("seq", np.uint8), ("reserved", np.uint16)])
 DIAG_BYTES = C.sizeof(Diag)
@@ -129,6 +147,10 @@ def load(build_if_missing: bool = True):
     for f in ("tss_window_reduce", "tss_score", "tss_calibrate", "tre_select_moves", "tre_sweep",
               "tss_rank", "tss_stage_gauges", "tss_stage_calibrate", "tss_stage_score"):
         getattr(lib, f).restype = C.c_int
+    lib.tre_replay.argtypes = [C.POINTER(Grid), C.POINTER(Latent), C.POINTER(Profile),
+                               C.POINTER(Ctrl), P, C.POINTER(ReplaySpec), P,
+                               C.POINTER(ReplayOut), P, C.POINTER(C.c_size_t), P, P]
+    lib.tre_replay.restype = C.c_int
     lib.tre_status_str.argtypes = [C.c_int]
     lib.tre_status_str.restype = C.c_char_p
     _lib = lib
@@ -652,3 +674,95 @@ class PipelinePlan:
                    cls=self.cls.cpu().numpy(), recv=self.recv.cpu().numpy(), moves=mv,
                    n_moves=n, r_final=self.r.cpu().numpy())
         return out
+
+
+LATENT_KEYS = ("model", "t_arr_ms", "d_first_ms", "d_total_ms", "L_in", "L_out")
+
+
+class ReplayPlan:
+    """A tre_replay call marshalled once: the closed-loop replay of one latent
+    trace (dict of int32 CUDA tensors, LATENT_KEYS) for every (rescue
+    threshold, pacing cap) setting. tau_list None: the profile's tau_crit;
+    cap_list None: pacing_cap. records / signal: also return the served
+    records and the Z / class rows each instance saw. run() issues the call."""
+
+    def __init__(self, latent, M, window_ms, K, profile, budget, r0, r_min, footprint,
+                 fast_ms=5000, slow_ms=10000, pacing_cap=1, tau_list=None, cap_list=None,
+                 wake_ms=0, sleep_ms=0, slo_ttft_ms=None, dtype="f64", records=False,
+                 signal=False, moves_cap=4096, diag=None):
+        torch = _torch()
+        self.lib = lib = load()
+        code, tdt = _dt(dtype)
+        n = int(latent["model"].numel())
+        for k in LATENT_KEYS:
+            _need(latent[k], "int32", n, k)
+        self._lat = latent
+        self.lat = Latent(n, *[latent[k].data_ptr() if n else None for k in LATENT_KEYS])
+        self.g = Grid(M, window_ms, K)
+        self.pst, self._prof = _profile(profile, M, tdt, code)
+        i32 = lambda a: (a if torch.is_tensor(a) else torch.as_tensor(np.asarray(a, np.int32))).to(
+            device="cuda", dtype=torch.int32).contiguous()
+        self._r0, self._rmin, self._fp = i32(r0), i32(r_min), i32(footprint)
+        self.ctrl = Ctrl(int(budget), self._rmin.data_ptr(), self._fp.data_ptr(), fast_ms, slow_ms,
+                         pacing_cap)
+        taus = [] if tau_list is None else [float(t) for t in tau_list]
+        caps = [] if cap_list is None else [int(c) for c in cap_list]
+        self._taus = (C.c_double * max(len(taus), 1))(*taus)
+        self._caps = (C.c_int32 * max(len(caps), 1))(*caps)
+        self.spec = ReplaySpec(len(taus), self._taus, len(caps), self._caps, wake_ms, sleep_ms)
+        self.n_inst = max(len(taus), 1) * max(len(caps), 1)
+        ni = self.n_inst
+        self.slo = i32(slo_ttft_ms) if slo_ttft_ms is not None else None
+        o = {"moves": torch.zeros(ni * max(moves_cap, 1) * MOVE_DTYPE.itemsize, dtype=torch.uint8,
+                                  device="cuda"),
+             "n_moves": torch.zeros(ni, dtype=torch.int64, device="cuda"),
+             "r_final": torch.zeros((ni, M), dtype=torch.int32, device="cuda"),
+             "served": torch.zeros((ni, M), dtype=torch.int64, device="cuda")}
+        if self.slo is not None:
+            o["slo_met"] = torch.zeros((ni, M), dtype=torch.int64, device="cuda")
+        if records:
+            for k in ("t_start_ms", "t_first_ms", "t_end_ms"):
+                o[k] = torch.empty((ni, n), dtype=torch.int32, device="cuda")
+        if signal:
+            o["Z"] = torch.empty((ni, K, M), dtype=tdt, device="cuda")
+            o["cls"] = torch.empty((ni, K, M), dtype=torch.uint8, device="cuda")
+        self.out = o
+        self.moves_cap = moves_cap
+        self.sout = ReplayOut(*[o[k].data_ptr() if k in o else None
+                                for k in ("t_start_ms", "t_first_ms", "t_end_ms", "Z", "cls",
+                                          "moves")],
+                              moves_cap, o["n_moves"].data_ptr(), o["r_final"].data_ptr(),
+                              o["slo_met"].data_ptr() if "slo_met" in o else None,
+                              o["served"].data_ptr())
+        self.diag = new_diag() if diag is None else diag
+        size = C.c_size_t(0)
+        _check("tre_replay", self._call(None, size, None))
+        self.ws = torch.empty(max(int(size.value), 256), dtype=torch.uint8, device="cuda")
+        self._ws_n = C.c_size_t(self.ws.numel())
+
+    def _call(self, ws, size, stream):
+        return self.lib.tre_replay(C.byref(self.g), C.byref(self.lat), C.byref(self.pst),
+                                   C.byref(self.ctrl), _ptr(self._r0), C.byref(self.spec),
+                                   _ptr(self.slo), C.byref(self.sout), ws, C.byref(size),
+                                   _ptr(self.diag), stream)
+
+    def run(self, stream=None):
+        """Enqueue the replay on `stream` (default: current torch stream)."""
+        _check("tre_replay", self._call(C.c_void_p(self.ws.data_ptr()), self._ws_n,
+                                        _stream(stream)))
+        return self.out
+
+    def moves(self):
+        """Host view of the move lists: one structured array per instance."""
+        raw = np.frombuffer(self.out["moves"].cpu().numpy().tobytes(), dtype=MOVE_DTYPE)
+        raw = raw.reshape(self.n_inst, max(self.moves_cap, 1))
+        n = self.out["n_moves"].cpu().numpy()
+        return [raw[i, : min(int(n[i]), self.moves_cap)] for i in range(self.n_inst)]
+
+
+def tre_replay(latent, M, window_ms, K, profile, budget, r0, r_min, footprint, **kw):
+    """Closed-loop replay, one call (see ReplayPlan). Returns (outputs dict of
+    CUDA tensors, list of host move arrays per instance, diag)."""
+    plan = ReplayPlan(latent, M, window_ms, K, profile, budget, r0, r_min, footprint, **kw)
+    out = plan.run()
+    return out, plan.moves(), plan.diag

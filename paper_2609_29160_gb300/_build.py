@@ -12,7 +12,8 @@ CSRC = os.path.join(HERE, "csrc")
 OUT_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT_DIR, "libtre.so")
 SOURCES = ["api.cu", "reduce.cu", "score.cu", "calibrate.cu", "select.cu", "noalloc.cu",
-           "classes.cu", "device.cu", "stage.cu"]
+           "classes.cu", "device.cu", "stage.cu",
+           "replay.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-fmad=false", "-Xcompiler", "-fPIC",
          "-I", os.path.join(ROOT, "include"), "-I", CSRC]

@@ -15,7 +15,8 @@ namespace {
 // ---- phase tracing ----------------------------------------------------------
 const char* const kPhaseName[TRE_TRACE_PHASES] = {"reduce", "gauge_scan", "aggregate", "score",
                                                   "receiver", "slo_counts", "calibrate",
-                                                  "normalize", "select", "occupancy"};
+                                                  "normalize", "select", "occupancy",
+                                                  "replay"};
 struct TraceRec {
   int phase, launches;
   cudaEvent_t a, b;
@@ -584,6 +585,67 @@ tre_status stage_score_typed(const tre_grid* g, const tre_counts* in, const int3
 
 }  // namespace
 
+namespace {
+
+// ---- tre_replay -------------------------------------------------------------
+template <class T>
+tre_status replay_typed(const tre_grid* g, const tre_latent* lat, const tre_profile* p,
+                        const tre_ctrl* c, const int32_t* r0, const tre_replay_spec* sp,
+                        const int32_t* slo_ms, const tre_replay_out* out, void* ws,
+                        size_t* ws_bytes, tre_diag* diag, cudaStream_t s) {
+  ReplayBatch<T> b;
+  std::memset(&b, 0, sizeof(b));
+  b.M = g->n_models;
+  b.win = g->window_ms;
+  b.K = g->n_windows;
+  const int n_tau = sp ? sp->n_tau : 0, n_cap = sp ? sp->n_cap : 0;
+  b.n_tau = n_tau;
+  b.n_cap = n_cap > 0 ? n_cap : 1;
+  for (int t = 0; t < n_tau; ++t) b.tau_list[t] = (T)sp->tau_crit[t];
+  for (int q = 0; q < b.n_cap; ++q) b.cap_list[q] = n_cap > 0 ? sp->pacing_cap[q] : c->pacing_cap;
+  b.n_inst = (n_tau > 0 ? n_tau : 1) * b.n_cap;
+  b.w_p = static_cast<const T*>(p->w_p);
+  b.w_q = static_cast<const T*>(p->w_q);
+  b.alpha = static_cast<const T*>(p->alpha);
+  b.theta = static_cast<const T*>(p->theta);
+  b.tau_crit = static_cast<const T*>(p->tau_crit);
+  b.tau_surp = static_cast<const T*>(p->tau_surplus);
+  b.budget = c->budget;
+  b.r0 = r0;
+  b.r_min = c->r_min;
+  b.footprint = c->footprint;
+  b.fast_ms = c->fast_ms;
+  b.slow_ms = c->slow_ms;
+  b.wake_ms = sp ? sp->wake_ms : 0;
+  b.sleep_ms = sp ? sp->sleep_ms : 0;
+  b.lat = ReplayLatent{lat->n, lat->model, lat->t_arr_ms, lat->d_first_ms, lat->d_total_ms,
+                       lat->L_in, lat->L_out};
+  b.slo_ms = slo_ms;
+  b.hcap = (int)c->budget;
+  b.o_ts = out->t_start_ms;
+  b.o_tf = out->t_first_ms;
+  b.o_te = out->t_end_ms;
+  b.Z = static_cast<T*>(out->Z);
+  b.cls = out->cls;
+  b.moves = out->moves;
+  b.moves_cap = out->moves_cap;
+  b.n_moves = out->n_moves;
+  b.r_final = out->r_final;
+  b.slo_met = out->slo_met;
+  b.served = out->served;
+  b.diag = diag;
+  Arena a(ws);
+  ReplayWs w;
+  replay_ws_layout<T>(a, b, w);
+  bool query;
+  tre_status st = ws_check(a, ws, ws_bytes, query);
+  if (st != TRE_OK || query) return st;
+  Scope sc(kReplay, 4, s);
+  return cuda_status(launch_replay<T>(b, w, s));
+}
+
+}  // namespace
+
 extern "C" {
 
 void tre_trace_enable(int on) {
@@ -813,6 +875,46 @@ tre_status tss_stage_score(const tre_grid* grid, const tre_counts* in, const int
   return stage_score_typed<double>(grid, in, A_prefill, A_decode, prof, theta_prefill,
                                    theta_decode, S_prefill, Z_prefill, cls_prefill, S_decode,
                                    Z_decode, cls_decode, ws, ws_bytes, diag, s);
+}
+
+tre_status tre_replay(const tre_grid* grid, const tre_latent* lat, const tre_profile* prof,
+                      const tre_ctrl* ctrl, const int32_t* r0, const tre_replay_spec* spec,
+                      const int32_t* slo_ttft_ms, const tre_replay_out* out, void* ws,
+                      size_t* ws_bytes, tre_diag* diag, tre_stream stream) {
+  if (!grid_ok(grid) || grid->n_models > 64 || !ws_bytes || !lat || lat->n < 0 || !ctrl || !r0 ||
+      !out)
+    return TRE_EINVAL;
+  if (lat->n > 0 && !(lat->model && lat->t_arr_ms && lat->d_first_ms && lat->d_total_ms &&
+                      lat->L_in && lat->L_out))
+    return TRE_EINVAL;
+  if (lat->n > 2147483647ll) return TRE_EINVAL;
+  if (!prof_ok(prof, true)) return TRE_EINVAL;
+  if (!ctrl->r_min || !ctrl->footprint || ctrl->fast_ms < 1 || ctrl->slow_ms < 1 ||
+      ctrl->budget < 0 || ctrl->budget > 65536)
+    return TRE_EINVAL;
+  if (spec) {
+    if (spec->n_tau < 0 || spec->n_tau > kMaxTau || (spec->n_tau > 0 && !spec->tau_crit))
+      return TRE_EINVAL;
+    if (spec->n_cap < 0 || spec->n_cap > kMaxCap || (spec->n_cap > 0 && !spec->pacing_cap))
+      return TRE_EINVAL;
+    for (int q = 0; q < spec->n_cap; ++q)
+      if (spec->pacing_cap[q] < 0 || spec->pacing_cap[q] > 255) return TRE_EINVAL;
+    if (spec->wake_ms < 0 || spec->sleep_ms < 0) return TRE_EINVAL;
+  }
+  if ((!spec || spec->n_cap == 0) && (ctrl->pacing_cap < 0 || ctrl->pacing_cap > 255))
+    return TRE_EINVAL;
+  if (!out->n_moves || !out->r_final || out->moves_cap < 0 || (out->moves_cap > 0 && !out->moves))
+    return TRE_EINVAL;
+  if ((!out->t_start_ms) != (!out->t_first_ms) || (!out->t_start_ms) != (!out->t_end_ms))
+    return TRE_EINVAL;
+  if ((!out->Z) != (!out->cls) || (out->slo_met && !slo_ttft_ms)) return TRE_EINVAL;
+  if (ws && !diag) return TRE_EINVAL;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (prof->dtype == TRE_F32)
+    return replay_typed<float>(grid, lat, prof, ctrl, r0, spec, slo_ttft_ms, out, ws, ws_bytes,
+                               diag, s);
+  return replay_typed<double>(grid, lat, prof, ctrl, r0, spec, slo_ttft_ms, out, ws, ws_bytes,
+                              diag, s);
 }
 
 }  // extern "C"

@@ -52,7 +52,7 @@ bool prof_ok(const tre_profile* p, bool need_theta_tau);
 
 // ---- api.cu: phase tracing (tre_trace_enable / tre_trace_collect) -----------
 enum Phase { kReduce, kScan, kAggregate, kScore, kReceiver, kSlo, kCalibrate, kNormalize,
-             kSelect, kOccupancy };
+             kSelect, kOccupancy, kReplay };
 // While tracing is on, brackets the launches of one phase with a pair of
 // events recorded on the stream (constructed before, destroyed after them).
 class Scope {
@@ -256,5 +256,54 @@ struct WalkWs {
 // lays out the tick tables and fills b.ent_base
 template <class T> void walk_ws_layout(Arena& a, WalkBatch<T>& b, WalkWs& w);
 template <class T> cudaError_t launch_walk(const WalkBatch<T>& b, WalkWs& w, cudaStream_t s);
+
+// ---- replay.cu ------------------------------------------------------------
+// Latent requests of a closed-loop replay (what a request needs once started).
+struct ReplayLatent {
+  int64_t n;
+  const int32_t *model, *t_arr, *d_first, *d_total, *L_in, *L_out;
+};
+// One controller instance per (rescue threshold, pacing cap); passed by value.
+template <class T> struct ReplayBatch {
+  int M, win, K, n_inst, n_tau, n_cap;
+  T tau_list[kMaxTau];             // used when n_tau > 0, else tau_crit per model
+  int32_t cap_list[kMaxCap];
+  const T *w_p, *w_q, *alpha, *theta, *tau_crit, *tau_surp;   // device [M]
+  int64_t budget;
+  const int32_t *r0, *r_min, *footprint;
+  int32_t fast_ms, slow_ms, wake_ms, sleep_ms;
+  ReplayLatent lat;
+  const int32_t* slo_ms;           // device [M] or null
+  // scratch
+  const int32_t* list;             // valid request indices grouped by model
+  const int32_t* base;             // [M + 1]
+  const int32_t* arr_cnt;          // [K][M] arrivals
+  uint32_t* acc;                   // per instance: P, D, ends, each [K + 1][M]
+  long long* gheap;                // per instance [M][hcap] when the heaps are global
+  int hcap;
+  int warps_per_cta;
+  int warp_bytes, heap_off;        // shared memory per warp, heap offset in it
+  // outputs
+  int32_t *o_ts, *o_tf, *o_te;     // [n_inst][n] or null
+  T* Z;                            // [n_inst][K][M] or null (with cls)
+  uint8_t* cls;
+  tre_move* moves;
+  int64_t moves_cap;
+  int64_t* n_moves;
+  int32_t* r_final;
+  int64_t *slo_met, *served;       // [n_inst][M] or null
+  tre_diag* diag;
+};
+struct ReplayWs {
+  int8_t* vm;
+  int32_t *arr_cnt, *n_valid, *base, *list;
+  uint32_t* acc;
+  long long* gheap;
+  bool shared_heaps;
+  int warps_per_cta;
+};
+// lays out the scratch and fills the batch's shared-memory plan
+template <class T> void replay_ws_layout(Arena& a, ReplayBatch<T>& b, ReplayWs& w);
+template <class T> cudaError_t launch_replay(ReplayBatch<T>& b, ReplayWs& w, cudaStream_t s);
 
 }  // namespace tre
