@@ -256,13 +256,15 @@ def select_moves(Z, cls, tau_crit, tau_surplus, window_ms, budget, r0, r_min, fo
 
 def closed_loop(lat, M, window_ms, K, profile, budget, r0, r_min, footprint, tau_crit,
                 tau_surplus, fast_ms=5000, slow_ms=10000, pacing_cap=1, dtype=np.float64,
-                cap=None, wake_ms=0, sleep_ms=0):
+                cap=None, wake_ms=0, sleep_ms=0, guard_ms=None):
     """Closed-loop replay of latent requests (model, t_arr_ms, d_first_ms,
     d_total_ms, L_in, L_out): the controller's moves change the servers, the
     served requests make the telemetry it scores. profile holds w_p, w_q,
     alpha, theta. wake_ms / sleep_ms: actuation delays of a receiver replica
-    and of a released donor replica (after it drains). Returns dict with the
-    served records (t_start_ms, t_first_ms, t_end_ms), moves, r_final, Z, cls."""
+    and of a released donor replica (after it drains). guard_ms: per-model
+    latency guard (a first token later than this after arrival breaches it),
+    None = no guard. Returns dict with the served records (t_start_ms,
+    t_first_ms, t_end_ms), moves, r_final, Z, cls."""
     n = len(lat["model"])
     pr = _prof(dict(profile, tau_crit=tau_crit, tau_surplus=tau_surplus), M, dtype)
     out = {k: np.zeros(n, np.int32) for k in ("t_start_ms", "t_first_ms", "t_end_ms")}
@@ -281,6 +283,7 @@ def closed_loop(lat, M, window_ms, K, profile, budget, r0, r_min, footprint, tau
                C.c_int64(budget), _p(_i32(r0)), _p(_i32(r_min)), _p(_i32(footprint)),
                C.c_int32(fast_ms), C.c_int32(slow_ms), C.c_int32(pacing_cap),
                C.c_int32(wake_ms), C.c_int32(sleep_ms),
+               _p(_i32(guard_ms)) if guard_ms is not None else None,
                _p(out["t_start_ms"]), _p(out["t_first_ms"]), _p(out["t_end_ms"]), _p(r),
                _p(moves), C.c_int64(cap), _p(nm), _p(Z), _p(cls))
         if rc == 1:

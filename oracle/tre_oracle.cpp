@@ -487,6 +487,7 @@ struct Walk {
   const T* tau_surplus;
   const int32_t* r_min;
   const int32_t* g;
+  const uint8_t* guard = nullptr;   // closed loop: donors whose latency guard is breached
 
   uint8_t region(int32_t m) const {
     if (ck[m] == kIdle) return kIdle;
@@ -498,16 +499,20 @@ struct Walk {
   // descending, then nominal by Z descending (nominal only above the
   // receiver's Z when `nom_above` is set); never critical, never the receiver,
   // never below the replica floor.
+  // A donor whose local latency guard is breached (closed loop only) is not
+  // released at this tick (Sec. IV-C donor-side release guard).
+  bool held(int32_t m) const { return guard && guard[m]; }
   int32_t pick_donor(const std::vector<int64_t>& r, int32_t recv, bool nom_above) const {
     for (int32_t m = 0; m < M; ++m)
-      if (m != recv && region(m) == kIdle && r[m] > r_min[m]) return m;
+      if (m != recv && region(m) == kIdle && r[m] > r_min[m] && !held(m)) return m;
     int32_t best = -1;
     for (int32_t m = 0; m < M; ++m)
-      if (m != recv && region(m) == kSurp && r[m] > r_min[m] && (best < 0 || Zk[m] > Zk[best]))
+      if (m != recv && region(m) == kSurp && r[m] > r_min[m] && !held(m) &&
+          (best < 0 || Zk[m] > Zk[best]))
         best = m;
     if (best >= 0) return best;
     for (int32_t m = 0; m < M; ++m) {
-      if (m == recv || region(m) != kNom || r[m] <= r_min[m]) continue;
+      if (m == recv || region(m) != kNom || r[m] <= r_min[m] || held(m)) continue;
       if (nom_above && !(Zk[m] > Zk[recv])) continue;
       if (best < 0 || Zk[m] > Zk[best]) best = m;
     }
@@ -603,19 +608,44 @@ struct Controller {
     ++nm;
   }
 
-  // window k ends a fast and/or a slow tick; Zk, ck: that window's Z and class
-  void tick(int64_t k, const T* Zk, const uint8_t* ck, bool fast, bool slow) {
+  // window k ends a fast and/or a slow tick; Zk, ck: that window's Z and class.
+  // Closed loop only (null / false in the open-loop walk): guard[m] set when
+  // model m breached its latency guard in the window, lost[m] when it has
+  // requests waiting and no routable replica, busy when a rebalance transfer
+  // is still in progress. Returns the kind of transition the tick made (0:
+  // none) -- a rescue deferred behind a rebalance in progress returns 0.
+  int tick(int64_t k, const T* Zk, const uint8_t* ck, bool fast, bool slow,
+           const uint8_t* guard = nullptr, const uint8_t* lost = nullptr, bool busy = false) {
     last.clear();
-    Walk<T> wk{M, Zk, ck, tau_crit, tau_surplus, r_min, footprint};
+    Walk<T> wk{M, Zk, ck, tau_crit, tau_surplus, r_min, footprint, guard};
     int32_t recv = -1;
     int kind = 0;
     bool nom_above = false;
-    if (fast) {                                  // rescue: lowest Z among critical models
-      for (int32_t m = 0; m < M; ++m)
-        if (wk.region(m) == kCrit && (recv < 0 || wk.Zk[m] < wk.Zk[recv])) recv = m;
-      if (recv >= 0) kind = kRescue;
+    if (fast) {
+      // rescue (Sec. IV-B): a hard latency-guard breach pre-empts every other
+      // event (the breaching model of lowest Z); otherwise the lowest Z among
+      // critical models and models that lost their routable capacity
+      bool hard = false;
+      if (guard)
+        for (int32_t m = 0; m < M; ++m)
+          if (guard[m] && (recv < 0 || wk.Zk[m] < wk.Zk[recv])) recv = m;
+      if (recv >= 0) {
+        hard = true;
+      } else {
+        for (int32_t m = 0; m < M; ++m) {
+          const bool want = wk.region(m) == kCrit || (lost && lost[m]);
+          if (want && (recv < 0 || wk.Zk[m] < wk.Zk[recv])) recv = m;
+        }
+      }
+      if (recv >= 0) {
+        // a rebalance transfer in progress is not pre-empted unless the
+        // receiver breaches a hard guard; the pending rescue still keeps the
+        // slow loop out of this tick
+        if (busy && !hard) return 0;
+        kind = kRescue;
+      }
     }
-    if (kind == 0 && slow) {                     // rebalance: Eq. 3 over non-idle models
+    if (kind == 0 && recv < 0 && slow) {         // rebalance: Eq. 3 over non-idle models
       for (int32_t m = 0; m < M; ++m)
         if (wk.region(m) != kIdle && (recv < 0 || wk.Zk[m] < wk.Zk[recv])) recv = m;
       if (recv >= 0 && wk.Zk[recv] < (T)1) {
@@ -623,7 +653,7 @@ struct Controller {
         nom_above = true;
       }
     }
-    if (kind == 0) return;
+    if (kind == 0) return 0;
     for (int32_t seq = 0; seq < pacing_cap; ++seq) {
       const int64_t need = footprint[recv];
       if (free_pool >= need) {                   // idle capacity first
@@ -653,6 +683,7 @@ struct Controller {
       for (int32_t d : rel) emit(k, recv, d, kind, seq);
       last.push_back({recv, rel});
     }
+    return kind;
   }
 };
 
@@ -711,9 +742,9 @@ int closed_loop(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* mod
                 const T* alpha, const T* theta, const T* tau_crit, const T* tau_surplus,
                 int64_t budget, const int32_t* r0, const int32_t* r_min, const int32_t* footprint,
                 int32_t fast_ms, int32_t slow_ms, int32_t pacing_cap, int32_t wake_ms,
-                int32_t sleep_ms, int32_t* t_start, int32_t* t_first, int32_t* t_end,
-                int32_t* r_out, Move* moves, int64_t cap, int64_t* n_moves, T* Z_out,
-                uint8_t* cls_out) {
+                int32_t sleep_ms, const int32_t* guard_ms, int32_t* t_start, int32_t* t_first,
+                int32_t* t_end, int32_t* r_out, Move* moves, int64_t cap, int64_t* n_moves,
+                T* Z_out, uint8_t* cls_out) {
   if (M < 1 || win < 1 || K < 0 || n < 0 || fast_ms < 1 || slow_ms < 1 || pacing_cap < 0 ||
       wake_ms < 0 || sleep_ms < 0)
     return 1;
@@ -743,6 +774,11 @@ int closed_loop(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* mod
   std::vector<T> S_carry(M, (T)0), S_row(M), Z_row(M);
   std::vector<uint8_t> init_carry(M, 0), cls_row(M);
   std::vector<int32_t> Pk(M), Dk(M), Ak(M), Wk(M);
+  // latency guard: first tokens per (window, model) later than the model's
+  // guard bound after arrival; the tick's guard and lost-capacity flags
+  std::vector<int64_t> late((size_t)K * M, 0);
+  std::vector<uint8_t> guard_row(M, 0), lost_row(M, 0);
+  int64_t reb_until = 0;                         // a rebalance transfer serves from here on
   for (int64_t k = 0; k < K; ++k) {
     const int64_t Tk = (k + 1) * (int64_t)win;
     for (int32_t m = 0; m < M; ++m) {
@@ -761,6 +797,7 @@ int closed_loop(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* mod
         cum_start[m] += 1;
         // tokens and the end of the running span, as reduce_requests counts them
         if (tf < span) P[(size_t)(tf / win) * M + m] += (uint32_t)L_in[i];
+        if (guard_ms && tf < span && tf - t_arr[i] > guard_ms[m]) late[(size_t)(tf / win) * M + m] += 1;
         const int64_t L = L_out[i], dur = te - tf;
         for (int64_t j = 0; j < L; ++j) {
           const int64_t tj = (L == 1) ? tf : tf + (j * dur) / (L - 1);
@@ -785,7 +822,13 @@ int closed_loop(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* mod
     if (cls_out) std::copy(cls_row.begin(), cls_row.end(), cls_out + (size_t)k * M);
     const bool fast = ends_tick(k, win, fast_ms), slow = ends_tick(k, win, slow_ms);
     if (!fast && !slow) continue;
-    ctl.tick(k, Z_row.data(), cls_row.data(), fast, slow);
+    for (int32_t m = 0; m < M; ++m) {
+      guard_row[m] = late[(size_t)k * M + m] > 0 ? 1 : 0;
+      lost_row[m] = ctl.r[m] == 0 && Wk[m] > 0 ? 1 : 0;
+    }
+    const int kind = ctl.tick(k, Z_row.data(), cls_row.data(), fast, slow,
+                              guard_ms ? guard_row.data() : nullptr, lost_row.data(),
+                              Tk < reb_until);
     for (const auto& tr : ctl.last) {
       int64_t gpu_free = Tk;                     // when the receiver's GPU is free
       for (int32_t d : tr.donors) {
@@ -794,6 +837,7 @@ int closed_loop(int32_t M, int32_t win, int32_t K, int64_t n, const int32_t* mod
         gpu_free = std::max<int64_t>(gpu_free, drained + sleep_ms);
       }
       servers[tr.recv].push(gpu_free + wake_ms);
+      if (kind == kRebalance) reb_until = std::max<int64_t>(reb_until, gpu_free + wake_ms);
     }
   }
   for (int32_t m = 0; m < M; ++m) r_out[m] = (int32_t)ctl.r[m];
@@ -927,12 +971,13 @@ int orc_rank_f64(int32_t M, int32_t K, const double* Z, const uint8_t* cls, int3
       const T* w_p, const T* w_q, const T* alpha, const T* theta, const T* tau_crit,               \
       const T* tau_surplus, int64_t budget, const int32_t* r0, const int32_t* r_min,               \
       const int32_t* footprint, int32_t fast_ms, int32_t slow_ms, int32_t pacing_cap,              \
-      int32_t wake_ms, int32_t sleep_ms, int32_t* t_start, int32_t* t_first, int32_t* t_end,       \
-      int32_t* r_out, Move* moves, int64_t cap, int64_t* n_moves, T* Z_out, uint8_t* cls_out) {    \
+      int32_t wake_ms, int32_t sleep_ms, const int32_t* guard_ms, int32_t* t_start,                \
+      int32_t* t_first, int32_t* t_end, int32_t* r_out, Move* moves, int64_t cap,                  \
+      int64_t* n_moves, T* Z_out, uint8_t* cls_out) {                                              \
     return closed_loop<T>(M, win, K, n, model, t_arr, d_first, d_total, L_in, L_out, w_p, w_q,     \
                           alpha, theta, tau_crit, tau_surplus, budget, r0, r_min, footprint,       \
-                          fast_ms, slow_ms, pacing_cap, wake_ms, sleep_ms, t_start, t_first,       \
-                          t_end, r_out, moves, cap, n_moves, Z_out, cls_out);                      \
+                          fast_ms, slow_ms, pacing_cap, wake_ms, sleep_ms, guard_ms, t_start,      \
+                          t_first, t_end, r_out, moves, cap, n_moves, Z_out, cls_out);             \
   }
 ORC_CLOSED_LOOP(f32, float)
 ORC_CLOSED_LOOP(f64, double)
