@@ -410,13 +410,24 @@ typedef struct {
 /* Settings replayed side by side, instance i = t * n_cap + c. n_tau == 0: one
  * threshold set, the profile's tau_crit per model; else tau_crit[t] (host) for
  * every model. n_cap == 0: the control's pacing_cap; else pacing_cap[c] (host,
- * 0..255). Limits: n_tau, n_cap <= 32. wake_ms, sleep_ms >= 0. */
+ * 0..255). Limits: n_tau, n_cap <= 32. wake_ms, sleep_ms >= 0.
+ * guard_ttft_ms (device int32[n_models], NULL = no guard): a model breaches its
+ * latency guard in window k when one of its requests got its first token in
+ * window k more than guard_ttft_ms[m] after arriving. At a fast tick a breach
+ * pre-empts every other rescue reason (receiver: the breaching model of lowest
+ * Z); otherwise rescue takes the lowest Z among critical models and models with
+ * requests waiting and no routable replica (lost capacity). A model whose guard
+ * is breached is not released as a donor at that tick (Sec. IV-C release
+ * guard). While a rebalance transfer is in progress (until its receiver's new
+ * server serves) a rescue without a breach is deferred, and the slow loop stays
+ * out of that tick (Sec. IV-B: the loops are mutually exclusive). */
 typedef struct {
   int32_t n_tau;
   const double* tau_crit;
   int32_t n_cap;
   const int32_t* pacing_cap;
   int32_t wake_ms, sleep_ms;
+  const int32_t* guard_ttft_ms;
 } tre_replay_spec;
 
 /* Replay outputs (device). Optional arrays may be NULL.

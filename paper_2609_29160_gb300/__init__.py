@@ -88,7 +88,7 @@ class Latent(C.Structure):
 class ReplaySpec(C.Structure):
     _fields_ = [("n_tau", C.c_int32), ("tau_crit", C.POINTER(C.c_double)), ("n_cap", C.c_int32),
                 ("pacing_cap", C.POINTER(C.c_int32)), ("wake_ms", C.c_int32),
-                ("sleep_ms", C.c_int32)]
+                ("sleep_ms", C.c_int32), ("guard_ttft_ms", C.c_void_p)]
 
 
 class ReplayOut(C.Structure):
@@ -683,13 +683,14 @@ class ReplayPlan:
     """A tre_replay call marshalled once: the closed-loop replay of one latent
     trace (dict of int32 CUDA tensors, LATENT_KEYS) for every (rescue
     threshold, pacing cap) setting. tau_list None: the profile's tau_crit;
-    cap_list None: pacing_cap. records / signal: also return the served
-    records and the Z / class rows each instance saw. run() issues the call."""
+    cap_list None: pacing_cap. guard_ttft_ms: per-model latency guard (None:
+    no guard). records / signal: also return the served records and the Z /
+    class rows each instance saw. run() issues the call."""
 
     def __init__(self, latent, M, window_ms, K, profile, budget, r0, r_min, footprint,
                  fast_ms=5000, slow_ms=10000, pacing_cap=1, tau_list=None, cap_list=None,
-                 wake_ms=0, sleep_ms=0, slo_ttft_ms=None, dtype="f64", records=False,
-                 signal=False, moves_cap=4096, diag=None):
+                 wake_ms=0, sleep_ms=0, slo_ttft_ms=None, guard_ttft_ms=None, dtype="f64",
+                 records=False, signal=False, moves_cap=4096, diag=None):
         torch = _torch()
         self.lib = lib = load()
         code, tdt = _dt(dtype)
@@ -709,7 +710,9 @@ class ReplayPlan:
         caps = [] if cap_list is None else [int(c) for c in cap_list]
         self._taus = (C.c_double * max(len(taus), 1))(*taus)
         self._caps = (C.c_int32 * max(len(caps), 1))(*caps)
-        self.spec = ReplaySpec(len(taus), self._taus, len(caps), self._caps, wake_ms, sleep_ms)
+        self._guard = i32(guard_ttft_ms) if guard_ttft_ms is not None else None
+        self.spec = ReplaySpec(len(taus), self._taus, len(caps), self._caps, wake_ms, sleep_ms,
+                               self._guard.data_ptr() if self._guard is not None else None)
         self.n_inst = max(len(taus), 1) * max(len(caps), 1)
         ni = self.n_inst
         self.slo = i32(slo_ttft_ms) if slo_ttft_ms is not None else None

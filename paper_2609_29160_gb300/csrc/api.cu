@@ -618,6 +618,7 @@ tre_status replay_typed(const tre_grid* g, const tre_latent* lat, const tre_prof
   b.slow_ms = c->slow_ms;
   b.wake_ms = sp ? sp->wake_ms : 0;
   b.sleep_ms = sp ? sp->sleep_ms : 0;
+  b.guard_ms = sp ? sp->guard_ttft_ms : nullptr;
   b.lat = ReplayLatent{lat->n, lat->model, lat->t_arr_ms, lat->d_first_ms, lat->d_total_ms,
                        lat->L_in, lat->L_out};
   b.slo_ms = slo_ms;

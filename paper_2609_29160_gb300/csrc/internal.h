@@ -274,11 +274,12 @@ template <class T> struct ReplayBatch {
   int32_t fast_ms, slow_ms, wake_ms, sleep_ms;
   ReplayLatent lat;
   const int32_t* slo_ms;           // device [M] or null
+  const int32_t* guard_ms;         // device [M] or null: latency guard per model
   // scratch
   const int32_t* list;             // valid request indices grouped by model
   const int32_t* base;             // [M + 1]
   const int32_t* arr_cnt;          // [K][M] arrivals
-  uint32_t* acc;                   // per instance: P, D, ends, each [K + 1][M]
+  uint32_t* acc;                   // per instance: P, D, ends, late first tokens, [K + 1][M] each
   long long* gheap;                // per instance [M][hcap] when the heaps are global
   int hcap;
   int warps_per_cta;

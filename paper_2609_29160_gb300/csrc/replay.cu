@@ -167,6 +167,7 @@ template <class T> struct Ctl {
   const ReplayBatch<T>& b;
   const T* z;
   const uint8_t* c;
+  const uint8_t* flag;   // bit 0: latency guard breached in the window; bit 1: lost capacity
   int32_t* r;
   T tc;            // the instance's rescue threshold (NaN: per model from the profile)
   __device__ T tcrit(int m) const { return tc == tc ? tc : b.tau_crit[m]; }
@@ -176,20 +177,23 @@ template <class T> struct Ctl {
     if (z[m] > b.tau_surp[m]) return TRE_SURP;
     return TRE_NOM;
   }
+  __device__ bool held(int m) const { return flag[m] & 1; }
   // donor preference: idle models (lowest index), then surplus by Z
   // descending, then nominal by Z descending (with nom_above only above the
-  // receiver's Z); never critical, never the receiver, never below the floor
+  // receiver's Z); never critical, never the receiver, never below the floor,
+  // never a donor whose latency guard is breached (its release is deferred)
   __device__ int pick(const int32_t* rr, int recv, bool nom_above) const {
     const int M = b.M;
     for (int m = 0; m < M; ++m)
-      if (m != recv && region(m) == TRE_IDLE && rr[m] > b.r_min[m]) return m;
+      if (m != recv && region(m) == TRE_IDLE && rr[m] > b.r_min[m] && !held(m)) return m;
     int best = -1;
     for (int m = 0; m < M; ++m)
-      if (m != recv && region(m) == TRE_SURP && rr[m] > b.r_min[m] && (best < 0 || z[m] > z[best]))
+      if (m != recv && region(m) == TRE_SURP && rr[m] > b.r_min[m] && !held(m) &&
+          (best < 0 || z[m] > z[best]))
         best = m;
     if (best >= 0) return best;
     for (int m = 0; m < M; ++m) {
-      if (m == recv || region(m) != TRE_NOM || rr[m] <= b.r_min[m]) continue;
+      if (m == recv || region(m) != TRE_NOM || rr[m] <= b.r_min[m] || held(m)) continue;
       if (nom_above && !(z[m] > z[recv])) continue;
       if (best < 0 || z[m] > z[best]) best = m;
     }
@@ -214,14 +218,16 @@ k_replay(const __grid_constant__ ReplayBatch<T> b) {
   int32_t* rr = r + M;
   int32_t* hs = rr + M;
   uint8_t* crow = reinterpret_cast<uint8_t*>(hs + M);
+  uint8_t* frow = crow + M;                     // guard / lost-capacity flags
   long long* heaps = SHEAP ? reinterpret_cast<long long*>(base + b.heap_off)
                            : b.gheap + (size_t)inst * M * b.hcap;
   const int ti = inst / b.n_cap, ci = inst % b.n_cap;
   const int pacing = b.cap_list[ci];
   const T tc = b.n_tau > 0 ? b.tau_list[ti] : (T)NAN;
-  uint32_t* Pacc = b.acc + (size_t)inst * 3 * (K + 1) * M;
+  uint32_t* Pacc = b.acc + (size_t)inst * 4 * (K + 1) * M;
   uint32_t* Dacc = Pacc + (size_t)(K + 1) * M;
   uint32_t* Eacc = Dacc + (size_t)(K + 1) * M;
+  uint32_t* Lacc = Eacc + (size_t)(K + 1) * M;  // first tokens later than the guard
   // initial replicas: one server free at t = 0 per replica
   long long used = 0;
   bool bad = false;
@@ -263,6 +269,7 @@ k_replay(const __grid_constant__ ReplayBatch<T> b) {
     init[j] = false;
   }
   long long free_pool = b.budget - used;        // lane 0's copy is the live one
+  long long reb_until = 0;                      // a rebalance transfer serves from here on
   int64_t nm = 0;
   __syncwarp();
   for (int k = 0; k < K; ++k) {
@@ -290,6 +297,8 @@ k_replay(const __grid_constant__ ReplayBatch<T> b) {
           b.o_te[x] = (int32_t)te;
         }
         if (b.slo_ms && tf - ta <= (long long)b.slo_ms[m]) ++met[j];
+        if (b.guard_ms && tf < span && tf - ta > (long long)b.guard_ms[m])
+          Lacc[(tf / win) * M + m] += 1u;
         if (tf < span) {
           const long long kf = tf / win, ke = min(te / win, (long long)K - 1);
           Pacc[kf * M + m] += (uint32_t)b.lat.L_in[i];
@@ -339,6 +348,9 @@ k_replay(const __grid_constant__ ReplayBatch<T> b) {
       else cl = TRE_NOM;
       zrow[m] = Z;
       crow[m] = cl;
+      // latency guard breached in the window; requests waiting with no
+      // routable replica (lost capacity)
+      frow[m] = (uint8_t)((b.guard_ms && Lacc[x] ? 1 : 0) | (r[m] == 0 && W > 0 ? 2 : 0));
       if (b.Z) {
         const size_t y = (size_t)inst * K * M + x;
         b.Z[y] = Z;
@@ -350,15 +362,31 @@ k_replay(const __grid_constant__ ReplayBatch<T> b) {
     __threadfence_block();
     __syncwarp();
     if (lane == 0) {
-      Ctl<T> ctl{b, zrow, crow, r, tc};
+      Ctl<T> ctl{b, zrow, crow, frow, r, tc};
       int recv = -1, kind = 0;
-      bool nom_above = false;
-      if (fast) {                                // rescue: lowest Z among critical models
+      bool nom_above = false, deferred = false;
+      if (fast) {
+        // rescue: a latency-guard breach pre-empts every other event (lowest
+        // Z among the breaching models); otherwise the lowest Z among critical
+        // models and models that lost their routable capacity. A rebalance
+        // transfer in progress defers a rescue without a breach; the pending
+        // rescue keeps the slow loop out of the tick.
+        bool hard = false;
         for (int m = 0; m < M; ++m)
-          if (ctl.region(m) == TRE_CRIT && (recv < 0 || zrow[m] < zrow[recv])) recv = m;
-        if (recv >= 0) kind = TRE_RESCUE;
+          if ((frow[m] & 1) && (recv < 0 || zrow[m] < zrow[recv])) recv = m;
+        if (recv >= 0) {
+          hard = true;
+        } else {
+          for (int m = 0; m < M; ++m)
+            if ((ctl.region(m) == TRE_CRIT || (frow[m] & 2)) && (recv < 0 || zrow[m] < zrow[recv]))
+              recv = m;
+        }
+        if (recv >= 0) {
+          if (Tk < reb_until && !hard) deferred = true;
+          else kind = TRE_RESCUE;
+        }
       }
-      if (kind == 0 && slow) {                   // rebalance: Eq. 3 over non-idle models
+      if (kind == 0 && recv < 0 && slow) {       // rebalance: Eq. 3 over non-idle models
         for (int m = 0; m < M; ++m)
           if (ctl.region(m) != TRE_IDLE && (recv < 0 || zrow[m] < zrow[recv])) recv = m;
         if (recv >= 0 && zrow[recv] < (T)1) {
@@ -379,6 +407,7 @@ k_replay(const __grid_constant__ ReplayBatch<T> b) {
         }
         ++nm;
       };
+      if (deferred) kind = 0;
       for (int seq = 0; kind && seq < pacing; ++seq) {
         const long long need = b.footprint[recv];
         Heap hr{heaps + (size_t)recv * b.hcap, hs[recv]};
@@ -388,6 +417,7 @@ k_replay(const __grid_constant__ ReplayBatch<T> b) {
           emit(recv, -1, seq);
           hr.push(Tk + b.wake_ms);
           hs[recv] = hr.n;
+          if (kind == TRE_REBALANCE) reb_until = max(reb_until, Tk + (long long)b.wake_ms);
           continue;
         }
         // dry run: can the eligible donors cover the receiver's footprint?
@@ -422,6 +452,7 @@ k_replay(const __grid_constant__ ReplayBatch<T> b) {
         r[recv] += 1;
         hr.push(gpu_free + b.wake_ms);
         hs[recv] = hr.n;
+        if (kind == TRE_REBALANCE) reb_until = max(reb_until, gpu_free + (long long)b.wake_ms);
       }
     }
     __threadfence_block();
@@ -451,7 +482,7 @@ constexpr size_t kReplaySmemMax = 160 * 1024;
 template <class T> int warp_base_bytes(int M) {
   size_t o = ((size_t)M * sizeof(T) + 15) & ~(size_t)15;   // Z row
   o += (size_t)M * 4 * 3;                                   // r, dry-run r, heap sizes
-  o += (size_t)M;                                           // class row
+  o += (size_t)M * 2;                                       // class and flag rows
   return (int)((o + 15) & ~(size_t)15);
 }
 
@@ -464,7 +495,7 @@ template <class T> void replay_ws_layout(Arena& a, ReplayBatch<T>& b, ReplayWs& 
   w.n_valid = a.take<int32_t>((size_t)M);
   w.base = a.take<int32_t>((size_t)M + 1);
   w.list = a.take<int32_t>((size_t)std::max<int64_t>(b.lat.n, 1));
-  w.acc = a.take<uint32_t>((size_t)b.n_inst * 3 * (K + 1) * M);
+  w.acc = a.take<uint32_t>((size_t)b.n_inst * 4 * (K + 1) * M);
   // warps per CTA: spread the instances over the SMs first
   const int sms = device_sm_count();
   int W = (int)std::min<int64_t>(8, std::max<int64_t>(1, (b.n_inst + sms - 1) / sms));
@@ -495,7 +526,7 @@ template <class T> cudaError_t launch_replay(ReplayBatch<T>& b, ReplayWs& w, cud
   const int M = b.M, K = b.K;
   cudaError_t e = cudaMemsetAsync(w.arr_cnt, 0, ((size_t)K * M + 1) * sizeof(int32_t), s);
   if (!e) e = cudaMemsetAsync(w.n_valid, 0, (size_t)M * sizeof(int32_t), s);
-  if (!e) e = cudaMemsetAsync(w.acc, 0, (size_t)b.n_inst * 3 * (K + 1) * M * sizeof(uint32_t), s);
+  if (!e) e = cudaMemsetAsync(w.acc, 0, (size_t)b.n_inst * 4 * (K + 1) * M * sizeof(uint32_t), s);
   if (e) return e;
   const int sms = device_sm_count();
   const unsigned g1 = (unsigned)std::max<int64_t>(

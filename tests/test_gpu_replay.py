@@ -50,7 +50,7 @@ def _counts(rec, lat, M, span, slo):
 
 
 def _check(tre, lat, M, win, K, prof, budget, r0, r_min, fp, dtype, settings, wake=0, sleep=0,
-           slo=None):
+           slo=None, guard=None):
     """settings: list of (tau_crit, pacing_cap) per instance, as the replay
     orders them (thresholds outer, caps inner)."""
     taus = sorted({t for t, _ in settings}, key=[t for t, _ in settings].index)
@@ -58,8 +58,8 @@ def _check(tre, lat, M, win, K, prof, budget, r0, r_min, fp, dtype, settings, wa
     slo = np.full(M, 1000, np.int32) if slo is None else slo
     out, moves, diag = tre.tre_replay(_cuda(lat), M, win, K, prof, budget, r0, r_min, fp,
                                       tau_list=taus, cap_list=caps, wake_ms=wake, sleep_ms=sleep,
-                                      slo_ttft_ms=slo, dtype=dtype, records=True, signal=True,
-                                      moves_cap=1 << 14)
+                                      slo_ttft_ms=slo, guard_ttft_ms=guard, dtype=dtype,
+                                      records=True, signal=True, moves_cap=1 << 14)
     npdt = np.float32 if dtype == "f32" else np.float64
     host = {k: v.cpu().numpy() for k, v in out.items() if k != "moves"}
     assert tre.read_diag(diag)["err"] == 0
@@ -67,7 +67,7 @@ def _check(tre, lat, M, win, K, prof, budget, r0, r_min, fp, dtype, settings, wa
     for i, (tau, cap) in enumerate((t, c) for t in taus for c in caps):
         ref = oracle.closed_loop(lat, M, win, K, prof, budget, r0, r_min, fp, tau,
                                  prof["tau_surplus"], pacing_cap=cap, dtype=npdt, wake_ms=wake,
-                                 sleep_ms=sleep)
+                                 sleep_ms=sleep, guard_ms=guard)
         for k in REC:
             np.testing.assert_array_equal(host[k][i], ref["records"][k], err_msg=f"{i} {k}")
         np.testing.assert_array_equal(host["Z"][i], ref["Z"], err_msg=f"{i} Z")
@@ -100,11 +100,26 @@ def test_replay_matches_oracle(tre, dtype, cap):
     assert (n > 10) == (cap > 0)
 
 
-@pytest.mark.parametrize("wake,sleep", [(1310, 1870), (0, 1870), (4000, 0)])
+@pytest.mark.parametrize("wake,sleep", [(1310, 1870), (0, 1870), (4000, 0), (4000, 3000)])
 def test_replay_with_actuation_delays(tre, wake, sleep):
+    """Delays longer than the rescue cadence also defer rescues behind
+    rebalance transfers in progress."""
     lat, M, budget = _mid_latent(0.01, 8, 900.0)
     n = _check(tre, lat, M, 1000, 900, _prof(M), budget, lat["r0"], np.ones(M, np.int32),
                np.ones(M, np.int32), "f64", [(0.8, 2)], wake=wake, sleep=sleep)
+    assert n > 10
+
+
+@pytest.mark.parametrize("dtype", ["f64", "f32"])
+@pytest.mark.parametrize("guard", [1500, 4000])
+def test_replay_with_latency_guards(tre, dtype, guard):
+    """Latency-guard breaches pre-empt rescue and hold donors; floors of zero
+    let models lose their last routable replica."""
+    lat, M, budget = _mid_latent(0.01, 13, 900.0)
+    r_min = np.array([1, 0, 1, 0, 1, 0, 1, 0], np.int32)
+    n = _check(tre, lat, M, 1000, 900, _prof(M), budget, lat["r0"], r_min, np.ones(M, np.int32),
+               dtype, [(0.7, 1), (0.8, 2)], wake=1310, sleep=1870,
+               guard=np.full(M, guard, np.int32))
     assert n > 10
 
 
@@ -115,7 +130,8 @@ def test_replay_batched_settings(tre):
     settings = [(t, c) for t in (0.5, 0.7, 0.8, 0.95) for c in (1, 2, 4)]
     slo = tracegen.slo_ttft_ms(M, 3)
     _check(tre, lat, M, 100, 6000, _prof(M), budget, lat["r0"], np.ones(M, np.int32),
-           np.ones(M, np.int32), "f32", settings, wake=1310, sleep=1870, slo=slo)
+           np.ones(M, np.int32), "f32", settings, wake=1310, sleep=1870, slo=slo,
+           guard=2 * slo)
 
 
 def test_replay_heterogeneous_footprints_and_pool(tre):
@@ -136,7 +152,8 @@ def test_replay_sixty_four_models_global_heaps(tre):
     M = spec.n_models
     prof = _prof(M, theta=2.0)
     _check(tre, lat, M, 100, 18000, prof, int(spec.budget), lat["r0"], np.ones(M, np.int32),
-           np.ones(M, np.int32), "f32", [(0.8, 1), (0.8, 2)], wake=1310, sleep=1870)
+           np.ones(M, np.int32), "f32", [(0.8, 1), (0.8, 2)], wake=1310, sleep=1870,
+           guard=np.full(M, 6000, np.int32))
 
 
 def test_replay_invalid_records_are_not_served(tre):
