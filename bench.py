@@ -43,6 +43,8 @@ def parse():
     ap.add_argument("--scale", type=float, default=1.0, help="request-count scale (1.0 = full)")
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-replay", action="store_true",
+                    help="skip the closed-loop replay measured beside the sweep")
     ap.add_argument("--no-configs", action="store_true",
                     help="skip the single-trace workloads measured beside the sweep")
     return ap.parse_args()
@@ -565,6 +567,104 @@ def occupancy_measure(lib, Trace, dev_traces, M, duration_ms, hbm, peak_kind, re
             "l2": "7 traces in turn, 196 MB of records"}
 
 
+# ---------------------------------------------------------------------------
+# Closed-loop replay of the sweep's traces (a widened row beside the sweep)
+# ---------------------------------------------------------------------------
+REPLAY_WAKE_MS, REPLAY_SLEEP_MS = 1310, 1870     # measured wake / sleep averages
+
+
+def replay_measure(lib, Trace, sw, theta, scale, rank, passes=2):
+    """tre_replay for every (trace, window length) of the sweep with all 64
+    (rescue threshold, pacing cap) settings each -- 1792 closed-loop controller
+    instances -- with the measured wake and sleep delays, a latency guard at
+    twice each model's TTFT bound, and theta as the open-loop sweep calibrated
+    it. Device time per pass over the 28 calls (the seven traces on seven
+    streams side by side, CUDA events around the pass), and the TTFT
+    attainment of the paper's rule (threshold 0.8, one transition per tick)
+    and of the best and worst settings per window length."""
+    import torch
+
+    import paper_2609_29160_gb300 as tre
+    M = sw["M"]
+    dur = sw["duration_ms"]
+    slo = np.asarray(sw["slo_ttft_ms"], np.int32)
+    taus, caps = [float(t) for t in sw["tau_crit"]], [int(c) for c in sw["pacing_cap"]]
+    plans, meta = [], []
+    n_tr = len(sw["traces"])
+    th = theta.cpu().numpy()
+    for ti in range(n_tr):
+        spec = tracegen.spec_mid(scale, rank_seed0(rank) + ti, dur / 1000.0)
+        lat = tracegen.gen_latent(spec)
+        dev = {k: torch.as_tensor(lat[k]).cuda() for k in tre.LATENT_KEYS}
+        for wi, win in enumerate(sw["window_ms"]):
+            win = int(win)
+            prof = {"w_p": sw["w_p"], "w_q": sw["w_q"], "alpha": min(1.0, win / 5000.0),
+                    "theta": th[ti * len(sw["window_ms"]) + wi], "tau_crit": 0.8,
+                    "tau_surplus": sw["tau_surplus"]}
+            plans.append(tre.ReplayPlan(dev, M, win, dur // win, prof, sw["budget"], lat["r0"],
+                                        sw["r_min"], sw["footprint"], tau_list=taus,
+                                        cap_list=caps, wake_ms=REPLAY_WAKE_MS,
+                                        sleep_ms=REPLAY_SLEEP_MS, slo_ttft_ms=slo,
+                                        guard_ttft_ms=2 * slo, dtype="f32", moves_cap=1024))
+            meta.append((ti, win, len(lat["model"]), dur // win))
+    # one stream per trace: a trace's four window lengths in turn, the traces
+    # side by side
+    main = torch.cuda.current_stream()
+    streams = [torch.cuda.Stream() for _ in range(n_tr)]
+
+    def one_pass():
+        ev = torch.cuda.Event()
+        ev.record(main)
+        done = []
+        for ti, st in enumerate(streams):
+            st.wait_event(ev)
+            for p, mt in zip(plans, meta):
+                if mt[0] == ti:
+                    p.run(st)
+            d = torch.cuda.Event()
+            d.record(st)
+            done.append(d)
+        for d in done:
+            main.wait_event(d)
+
+    one_pass()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(main)
+    for _ in range(passes):
+        one_pass()
+    e1.record(main)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / passes
+    n_inst = sum(p.n_inst for p in plans)
+    inst_windows = sum(p.n_inst * k for p, (_, _, _, k) in zip(plans, meta))
+    records = sum(n for (_, _, n, _) in meta)
+    att = {}
+    for win in sw["window_ms"]:
+        win = int(win)
+        met = np.zeros((len(taus) * len(caps),), np.float64)
+        tot = 0
+        for p, (ti, w, n, _) in zip(plans, meta):
+            if w != win:
+                continue
+            met += p.out["slo_met"].cpu().numpy().sum(axis=1)
+            tot += n
+        a = met / max(tot, 1)
+        rule = taus.index(0.8) * len(caps) + caps.index(1)
+        best = int(np.argmax(a))
+        att[str(win)] = {"paper_rule": float(a[rule]), "best": float(a[best]),
+                         "best_setting": {"tau_crit": taus[best // len(caps)],
+                                          "pacing_cap": caps[best % len(caps)]},
+                         "worst": float(a.min())}
+    return {"row": "closed-loop replay: 7 traces x 4 window lengths x 64 settings",
+            "instances": n_inst, "ms_per_pass": ms, "calls_per_pass": len(plans),
+            "instance_windows_per_s": inst_windows / (ms / 1e3),
+            "records_per_s": records * len(taus) * len(caps) / (ms / 1e3),
+            "wake_ms": REPLAY_WAKE_MS, "sleep_ms": REPLAY_SLEEP_MS,
+            "guard": "2 x TTFT bound", "ttft_attainment": att,
+            "bound": "latency (one warp per instance, serial over windows)"}
+
+
 # DRAM traffic per call of a phase, from the committed ncu summary of its
 # kernels; used only while the kernel source is the one the counters were
 # taken on (the summary records its SHA-256)
@@ -866,6 +966,9 @@ def main():
     # a widened step measured beside the sweep (not part of the timed step)
     next_rows = {"occupancy_mean": occupancy_measure(lib, Trace, dev_traces, M,
                                                      sw["duration_ms"], hbm, peak_kind)}
+    if not args.no_replay:
+        next_rows["closed_loop_replay"] = replay_measure(lib, Trace, sw, out["theta"],
+                                                         args.scale, rank)
 
     configs = None
     if rank == 0 and not args.no_configs:

@@ -277,6 +277,8 @@ template <class T> struct ReplayBatch {
   const int32_t* guard_ms;         // device [M] or null: latency guard per model
   // scratch
   const int32_t* list;             // valid request indices grouped by model
+  const int4* grp;                 // per grouped request: (t_arr, d_first, d_total, index),
+                                   // (L_in, L_out, -, -)
   const int32_t* base;             // [M + 1]
   const int32_t* arr_cnt;          // [K][M] arrivals
   uint32_t* acc;                   // per instance: P, D, ends, late first tokens, [K + 1][M] each
@@ -284,6 +286,9 @@ template <class T> struct ReplayBatch {
   int hcap;
   int warps_per_cta;
   int warp_bytes, heap_off;        // shared memory per warp, heap offset in it
+  int act_off, acap;               // decoding-request lists: offset, entries per model
+  int ring_off;                    // per-model window rings and pending far windows
+  int q_off;                       // per-model staged requests
   // outputs
   int32_t *o_ts, *o_tf, *o_te;     // [n_inst][n] or null
   T* Z;                            // [n_inst][K][M] or null (with cls)
@@ -298,6 +303,7 @@ template <class T> struct ReplayBatch {
 struct ReplayWs {
   int8_t* vm;
   int32_t *arr_cnt, *n_valid, *base, *list;
+  int4* grp;
   uint32_t* acc;
   long long* gheap;
   bool shared_heaps;

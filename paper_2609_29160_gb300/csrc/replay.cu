@@ -95,6 +95,20 @@ k_rp_fill(int64_t n, int M, const int8_t* __restrict__ vm, const int32_t* __rest
   }
 }
 
+// the model-grouped columns a lane walks: arrival, time to first and last
+// token, prompt and output lengths, in the grouped order
+__global__ void k_rp_gather(int64_t n_valid_total, ReplayLatent lat,
+                            const int32_t* __restrict__ list, const int32_t* __restrict__ base,
+                            int M, int4* __restrict__ g) {
+  const int64_t n = base[M];
+  for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < n;
+       p += (int64_t)gridDim.x * blockDim.x) {
+    const int32_t i = list[p];
+    g[2 * p] = make_int4(lat.t_arr[i], lat.d_first[i], lat.d_total[i], i);
+    g[2 * p + 1] = make_int4(lat.L_in[i], lat.L_out[i], 0, 0);
+  }
+}
+
 // served records start as "not started" (K*win) or "not served" (-1)
 __global__ void k_rp_init_records(int64_t n, int n_inst, int32_t span, const int8_t* __restrict__ vm,
                                   int32_t* ts, int32_t* tf, int32_t* te) {
@@ -154,9 +168,28 @@ __device__ __forceinline__ long long tokens_before(long long t, long long tf, lo
   if (t <= tf) return 0;
   if (t > te) return L;
   if (L == 1) return 1;
-  const long long num = (t - tf) * (L - 1), dur = te - tf;
-  return (num + dur - 1) / dur;
+  const unsigned long long num = (unsigned long long)(t - tf) * (unsigned long long)(L - 1);
+  const unsigned long long dur = (unsigned long long)(te - tf);
+  const unsigned long long y = num + dur - 1;
+  if ((y >> 32) == 0) return (long long)((uint32_t)y / (uint32_t)dur);   // 32-bit divide
+  return (long long)(y / dur);
 }
+
+// A request still emitting decode tokens after its first-token window: the
+// window from which it contributes, its last window (within the grid), its
+// last token time, output length and tokens counted so far. With
+// y = (T - tf)(L - 1) + dur - 1 the tokens before T are floor(y / dur) while
+// T <= te; moving T one window on adds win * (L - 1) = qd * dur + rd to y, so
+// the count is carried as a quotient and remainder without dividing.
+struct Decoding {
+  int32_t k_from, k_last, te, L, done;
+  int32_t q, r;            // floor and remainder of y / dur at T = k_from * win
+  int32_t qd, rd, dur;
+};
+// per-model window ring (power of two) and pending far-window list sizes; the
+// four counts a window collects
+constexpr int kRing = 64, kFar = 32, kQ = 32;
+enum { kP = 0, kD = 1, kEnd = 2, kLate = 3 };
 
 // window k ends a tick of cadence c when a multiple of c falls in (k*win, (k+1)*win]
 __device__ __forceinline__ bool ends_tick(long long k, int win, int c) {
@@ -202,7 +235,7 @@ template <class T> struct Ctl {
 };
 
 template <class T, int MPL, bool SHEAP>
-__global__ void __launch_bounds__(256)
+__global__ void __launch_bounds__(256, 1)
 k_replay(const __grid_constant__ ReplayBatch<T> b) {
   extern __shared__ unsigned long long rsm[];
   const int wid = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -221,13 +254,23 @@ k_replay(const __grid_constant__ ReplayBatch<T> b) {
   uint8_t* frow = crow + M;                     // guard / lost-capacity flags
   long long* heaps = SHEAP ? reinterpret_cast<long long*>(base + b.heap_off)
                            : b.gheap + (size_t)inst * M * b.hcap;
+  // per model, the requests still decoding past their first-token window
+  Decoding* act = reinterpret_cast<Decoding*>(base + b.act_off);
   const int ti = inst / b.n_cap, ci = inst % b.n_cap;
   const int pacing = b.cap_list[ci];
   const T tc = b.n_tau > 0 ? b.tau_list[ti] : (T)NAN;
-  uint32_t* Pacc = b.acc + (size_t)inst * 4 * (K + 1) * M;
-  uint32_t* Dacc = Pacc + (size_t)(K + 1) * M;
-  uint32_t* Eacc = Dacc + (size_t)(K + 1) * M;
-  uint32_t* Lacc = Eacc + (size_t)(K + 1) * M;  // first tokens later than the guard
+  // per-window prompt tokens, decode tokens, running-span ends and late first
+  // tokens beyond the ring, [4][K + 1][M]
+  uint32_t* Gacc = b.acc + (size_t)inst * 4 * (K + 1) * M;
+  uint32_t* ring = reinterpret_cast<uint32_t*>(base + b.ring_off);   // [4][M][kRing]
+  int32_t* farl = reinterpret_cast<int32_t*>(ring + (size_t)4 * M * kRing);  // [M][kFar]
+  // each model's next requests, staged from the grouped columns: grouped
+  // positions [qend - kQ, qend) sit in slot position % kQ; qhead mirrors the
+  // owning lane's cursor for the refill
+  int4* qbuf = reinterpret_cast<int4*>(base + b.q_off);              // [M][kQ][2]
+  int32_t* qhead = reinterpret_cast<int32_t*>(qbuf + (size_t)M * kQ * 2);
+  int32_t* qend = qhead + M;
+  for (int c = lane; c < 4 * M * kRing; c += 32) ring[c] = 0;
   // initial replicas: one server free at t = 0 per replica
   long long used = 0;
   bool bad = false;
@@ -255,7 +298,10 @@ k_replay(const __grid_constant__ ReplayBatch<T> b) {
     for (int q = 0; q < r[m]; ++q) heaps[(size_t)m * b.hcap + q] = 0;
   }
   // per-model state of this lane
-  int32_t head[MPL], end[MPL];
+  int32_t head[MPL], end[MPL], n_act[MPL], n_far[MPL];
+  bool far_all[MPL];
+  uint32_t arr_next[MPL];
+  T pw[MPL], pq[MPL], pa[MPL], pth[MPL], ptc[MPL], pts[MPL];   // the profile, per model
   long long cum_arr[MPL], cum_start[MPL], cum_end[MPL], met[MPL];
   T S[MPL];
   bool init[MPL];
@@ -264,6 +310,22 @@ k_replay(const __grid_constant__ ReplayBatch<T> b) {
     const int m = lane + 32 * j;
     head[j] = m < M ? b.base[m] : 0;
     end[j] = m < M ? b.base[m + 1] : 0;
+    n_act[j] = 0;
+    n_far[j] = 0;
+    far_all[j] = false;
+    arr_next[j] = m < M && K > 0 ? (uint32_t)b.arr_cnt[m] : 0u;
+    if (m < M) {
+      pw[j] = b.w_p[m];
+      pq[j] = b.w_q[m];
+      pa[j] = b.alpha[m];
+      pth[j] = b.theta[m];
+      ptc[j] = tc == tc ? tc : b.tau_crit[m];
+      pts[j] = b.tau_surp[m];
+    }
+    if (m < M) {
+      qhead[m] = head[j];
+      qend[m] = head[j];
+    }
     cum_arr[j] = cum_start[j] = cum_end[j] = met[j] = 0;
     S[j] = (T)0;
     init[j] = false;
@@ -274,19 +336,72 @@ k_replay(const __grid_constant__ ReplayBatch<T> b) {
   __syncwarp();
   for (int k = 0; k < K; ++k) {
     const long long Tk = (long long)(k + 1) * win;
+    // top up the staged requests of every model that has used half of them:
+    // the warp loads up to kQ of a model's next requests at once
+    for (int j = 0; j < MPL; ++j) {
+      const int m = lane + 32 * j;
+      const bool want = m < M && qend[m] < end[j] && qend[m] - head[j] < kQ / 2 &&
+                        head[j] < end[j];
+      unsigned need = __ballot_sync(0xffffffffu, want);
+      while (need) {
+        const int l = __ffs(need) - 1;
+        need &= need - 1;
+        const int mm = l + 32 * j;
+        const int h = __shfl_sync(0xffffffffu, head[j], l);
+        const int ne = __shfl_sync(0xffffffffu, end[j], l);
+        const int e = max(qend[mm], h);          // the owner may have read past them
+        const int upto = min(h + kQ, ne);
+        const int p = e + lane;
+        if (p < upto) {
+          int4* slot = qbuf + ((size_t)mm * kQ + (p & (kQ - 1))) * 2;
+          slot[0] = b.grp[2 * (size_t)p];
+          slot[1] = b.grp[2 * (size_t)p + 1];
+        }
+        __syncwarp();
+        if (lane == 0) qend[mm] = upto;
+        __syncwarp();
+      }
+    }
     for (int j = 0; j < MPL; ++j) {
       const int m = lane + 32 * j;
       if (m >= M) continue;
       Heap hp{heaps + (size_t)m * b.hcap, hs[m]};
+      Decoding* am = act + (size_t)m * b.acap;
+      int32_t* fl = farl + (size_t)m * kFar;
+      // per-window counts of this model: windows k .. k+kRing-1 in the shared
+      // ring, later ones in the instance's global accumulators (their windows
+      // listed, or every row reads them once the list has overflowed)
+      auto add = [&](int arr, long long kt, uint32_t v) {
+        if (kt - k < kRing) {
+          ring[((size_t)arr * M + m) * kRing + (kt & (kRing - 1))] += v;
+          return;
+        }
+        Gacc[(size_t)arr * (K + 1) * M + kt * M + m] += v;
+        if (far_all[j]) return;
+        for (int q = 0; q < n_far[j]; ++q)
+          if (fl[q] == (int32_t)kt) return;
+        if (n_far[j] < kFar) fl[n_far[j]++] = (int32_t)kt;
+        else far_all[j] = true;
+      };
       // start every request of the model that can start before T, in order
+      const int staged_end = qend[m];
       while (head[j] < end[j] && hp.n > 0) {
-        const int32_t i = b.list[head[j]];
-        const long long ta = b.lat.t_arr[i];
+        int4 c0, c1;
+        if (head[j] < staged_end) {
+          const int4* slot = qbuf + ((size_t)m * kQ + (head[j] & (kQ - 1))) * 2;
+          c0 = slot[0];
+          c1 = slot[1];
+        } else {                                 // beyond the staged ones
+          c0 = b.grp[2 * (size_t)head[j]];
+          c1 = b.grp[2 * (size_t)head[j] + 1];
+        }
+        const long long ta = c0.x;
         const long long st = max(ta, hp.h[0]);
         if (st >= Tk) break;
-        const long long dtot = b.lat.d_total[i];
-        const long long tf = min(st + (long long)b.lat.d_first[i], 2147483647ll);
+        const long long dtot = c0.z;
+        const long long tf = min(st + (long long)c0.y, 2147483647ll);
         const long long te = min(st + dtot, 2147483647ll);
+        const int32_t i = c0.w, L_in = c1.x, L_out = c1.y;
         hp.replace_top(st + dtot);
         ++head[j];
         ++cum_start[j];
@@ -297,35 +412,111 @@ k_replay(const __grid_constant__ ReplayBatch<T> b) {
           b.o_te[x] = (int32_t)te;
         }
         if (b.slo_ms && tf - ta <= (long long)b.slo_ms[m]) ++met[j];
-        if (b.guard_ms && tf < span && tf - ta > (long long)b.guard_ms[m])
-          Lacc[(tf / win) * M + m] += 1u;
+        bool ends_via_list = false;
         if (tf < span) {
-          const long long kf = tf / win, ke = min(te / win, (long long)K - 1);
-          Pacc[kf * M + m] += (uint32_t)b.lat.L_in[i];
-          const long long L = b.lat.L_out[i];
-          long long prev = tokens_before(kf * win, tf, te, L);
-          for (long long kk = kf; kk <= ke; ++kk) {
-            const long long nxt = tokens_before((kk + 1) * win, tf, te, L);
-            if (nxt != prev) Dacc[kk * M + m] += (uint32_t)(nxt - prev);
-            prev = nxt;
+          // times fit 31 bits: 32-bit divisions
+          const long long kf = (uint32_t)tf / (uint32_t)win;
+          const long long ke = min((long long)((uint32_t)te / (uint32_t)win), (long long)K - 1);
+          if (b.guard_ms && tf - ta > (long long)b.guard_ms[m]) add(kLate, kf, 1u);
+          add(kP, kf, (uint32_t)L_in);
+          const long long first = tokens_before((kf + 1) * win, tf, te, L_out);
+          if (first) add(kD, kf, (uint32_t)first);
+          if (ke > kf && L_out >= 2) {
+            if (n_act[j] < b.acap) {             // later windows: counted window by window
+              // here te >= (kf + 1) * win > tf and L_out >= 2 (else every token
+              // of the request falls in window kf)
+              const unsigned long long dur = (unsigned long long)(te - tf);
+              const unsigned long long y = (unsigned long long)((kf + 1) * win - tf) *
+                                               (unsigned long long)(L_out - 1) + dur - 1;
+              const unsigned long long step = (unsigned long long)win * (L_out - 1);
+              Decoding d;
+              d.k_from = (int32_t)kf + 1;
+              d.k_last = (int32_t)ke;
+              d.te = (int32_t)te;
+              d.L = L_out;
+              d.done = (int32_t)first;
+              d.q = (int32_t)(y / dur);
+              d.r = (int32_t)(y - (unsigned long long)d.q * dur);
+              // a step of more than L tokens ends the request in the next
+              // window, where the count is L: the clamp never shows
+              const unsigned long long qd = step / dur;
+              d.qd = (int32_t)min(qd, (unsigned long long)L_out + 1);
+              d.rd = (int32_t)(step - qd * dur);
+              d.dur = (int32_t)dur;
+              am[n_act[j]++] = d;
+              ends_via_list = true;
+            } else {                             // no room: add them all now
+              long long prev = first;
+              for (long long kk = kf + 1; kk <= ke; ++kk) {
+                const long long nxt = tokens_before((kk + 1) * win, tf, te, L_out);
+                if (nxt != prev) add(kD, kk, (uint32_t)(nxt - prev));
+                prev = nxt;
+              }
+            }
           }
         }
-        Eacc[min(te / win, (long long)K) * M + m] += 1u;
+        // the running span ends in window te / win (never read when te is
+        // past the grid); a listed request counts its end when it retires
+        if (!ends_via_list && te < span) add(kEnd, (uint32_t)te / (uint32_t)win, 1u);
       }
-      // window k's telemetry, scored with the carried smoothing state
+      qhead[m] = head[j];
+      // decode tokens of the requests still decoding, for window k, and the
+      // ends of those that retire in it
+      uint32_t d_live = 0, e_live = 0;
+      for (int q = 0; q < n_act[j];) {
+        Decoding& e = am[q];
+        if (e.k_from > k) {
+          ++q;
+          continue;
+        }
+        // y at the end of window k
+        e.q += e.qd;
+        e.r += e.rd;
+        if (e.r >= e.dur) {
+          e.r -= e.dur;
+          e.q += 1;
+        }
+        const int32_t nxt = (long long)(k + 1) * win > (long long)e.te ? e.L : e.q;
+        d_live += (uint32_t)(nxt - e.done);
+        e.done = nxt;
+        if (e.k_last <= k) {
+          if ((long long)e.te < span) ++e_live;
+          am[q] = am[--n_act[j]];
+        } else {
+          ++q;
+        }
+      }
+      // window k's counts: the ring slot (cleared for window k + kRing) plus
+      // any later-window contributions made before the ring reached it
+      uint32_t v[4];
+      bool far = far_all[j];
+      for (int q = 0; q < n_far[j]; ++q)
+        if (fl[q] == k) {
+          far = true;
+          fl[q] = fl[--n_far[j]];
+          break;
+        }
+#pragma unroll
+      for (int a = 0; a < 4; ++a) {
+        uint32_t* slot = &ring[((size_t)a * M + m) * kRing + (k & (kRing - 1))];
+        v[a] = *slot;
+        *slot = 0;
+        if (far) v[a] += Gacc[(size_t)a * (K + 1) * M + (size_t)k * M + m];
+      }
       const size_t x = (size_t)k * M + m;
-      cum_arr[j] += b.arr_cnt[x];
-      cum_end[j] += Eacc[x];
-      const int32_t P = (int32_t)Pacc[x], D = (int32_t)Dacc[x];
+      cum_arr[j] += arr_next[j];
+      if (k + 1 < K) arr_next[j] = b.arr_cnt[x + M];   // the next window's arrivals, early
+      cum_end[j] += v[kEnd] + e_live;
+      const int32_t P = (int32_t)v[kP], D = (int32_t)(v[kD] + d_live);
       const int32_t A = (int32_t)(cum_start[j] - cum_end[j]);
       const int32_t W = (int32_t)(cum_arr[j] - cum_start[j]);
       const bool idle = P == 0 && D == 0 && A == 0 && W == 0;
       if (!idle) {
         const T r_pre = (T)P / dt;
         const T r_dec = (T)D / dt;
-        const T svc = b.w_p[m] * r_pre;
+        const T svc = pw[j] * r_pre;
         const T num = svc + r_dec;
-        const T qw = b.w_q[m] * (T)W;
+        const T qw = pq[j] * (T)W;
         T den = (T)A + qw;
         if (den < (T)1) den = (T)1;
         const T raw = num / den;
@@ -333,24 +524,22 @@ k_replay(const __grid_constant__ ReplayBatch<T> b) {
           S[j] = raw;
           init[j] = true;
         } else {
-          const T a = b.alpha[m];
-          const T x1 = a * raw;
-          const T x2 = ((T)1 - a) * S[j];
+          const T x1 = pa[j] * raw;
+          const T x2 = ((T)1 - pa[j]) * S[j];
           S[j] = x1 + x2;
         }
       }
-      const T Z = S[j] / b.theta[m];
+      const T Z = S[j] / pth[j];
       uint8_t cl;
-      const T tcm = tc == tc ? tc : b.tau_crit[m];
       if (idle) cl = TRE_IDLE;
-      else if (Z < tcm) cl = TRE_CRIT;
-      else if (Z > b.tau_surp[m]) cl = TRE_SURP;
+      else if (Z < ptc[j]) cl = TRE_CRIT;
+      else if (Z > pts[j]) cl = TRE_SURP;
       else cl = TRE_NOM;
       zrow[m] = Z;
       crow[m] = cl;
       // latency guard breached in the window; requests waiting with no
       // routable replica (lost capacity)
-      frow[m] = (uint8_t)((b.guard_ms && Lacc[x] ? 1 : 0) | (r[m] == 0 && W > 0 ? 2 : 0));
+      frow[m] = (uint8_t)((b.guard_ms && v[kLate] ? 1 : 0) | (r[m] == 0 && W > 0 ? 2 : 0));
       if (b.Z) {
         const size_t y = (size_t)inst * K * M + x;
         b.Z[y] = Z;
@@ -465,7 +654,7 @@ k_replay(const __grid_constant__ ReplayBatch<T> b) {
     if (m >= M) continue;
     if (b.slo_ms) {
       for (int32_t q = head[j]; q < end[j]; ++q)
-        if (span - (long long)b.lat.t_arr[b.list[q]] <= (long long)b.slo_ms[m]) ++met[j];
+        if (span - (long long)b.grp[2 * q].x <= (long long)b.slo_ms[m]) ++met[j];
       if (b.slo_met) b.slo_met[(size_t)inst * M + m] = met[j];
     }
     if (b.served) b.served[(size_t)inst * M + m] = cum_start[j];
@@ -496,26 +685,43 @@ template <class T> void replay_ws_layout(Arena& a, ReplayBatch<T>& b, ReplayWs& 
   w.base = a.take<int32_t>((size_t)M + 1);
   w.list = a.take<int32_t>((size_t)std::max<int64_t>(b.lat.n, 1));
   w.acc = a.take<uint32_t>((size_t)b.n_inst * 4 * (K + 1) * M);
+  w.grp = a.take<int4>((size_t)std::max<int64_t>(b.lat.n, 1) * 2);
   // warps per CTA: spread the instances over the SMs first
   const int sms = device_sm_count();
   int W = (int)std::min<int64_t>(8, std::max<int64_t>(1, (b.n_inst + sms - 1) / sms));
+  auto a16 = [](size_t x) { return (x + 15) & ~(size_t)15; };
   const size_t wb = (size_t)warp_base_bytes<T>(M);
-  const size_t hb = (size_t)M * b.hcap * 8;
+  const size_t hb = a16((size_t)M * b.hcap * 8);
+  const size_t ring_bytes = a16((size_t)M * (4 * kRing + kFar) * 4);
+  const size_t q_bytes = a16((size_t)M * kQ * 32 + (size_t)M * 8);
+  // decoding requests per model: room for as many as the budget has replicas
+  // (more are added straight to the accumulators), at least 8
+  int acap = std::max(8, std::min(b.hcap, 256));
+  auto act_bytes = [&](int c) { return a16((size_t)M * c * sizeof(Decoding)); };
   w.shared_heaps = false;
   for (int tw = W; tw >= 1; tw >>= 1) {
-    if ((wb + hb) * tw <= kReplaySmemMax) {
+    if ((wb + hb + q_bytes + ring_bytes + act_bytes(8)) * tw <= kReplaySmemMax) {
       w.shared_heaps = true;
       W = tw;
       break;
     }
   }
+  const size_t fixed = wb + (w.shared_heaps ? hb : 0) + q_bytes + ring_bytes;
+  if (!w.shared_heaps) W = 1;
+  while (acap > 8 && (fixed + act_bytes(acap)) * W > kReplaySmemMax) acap >>= 1;
   w.warps_per_cta = W;
   b.warps_per_cta = W;
+  // per warp: base rows | heaps (when shared) | staged requests | rings | lists
   b.heap_off = (int)wb;
-  b.warp_bytes = (int)(w.shared_heaps ? wb + hb : wb);
+  b.q_off = (int)(wb + (w.shared_heaps ? hb : 0));
+  b.ring_off = (int)(b.q_off + q_bytes);
+  b.act_off = (int)(b.ring_off + ring_bytes);
+  b.acap = acap;
+  b.warp_bytes = (int)(fixed + act_bytes(acap));
   w.gheap = w.shared_heaps ? nullptr
                            : a.take<long long>((size_t)b.n_inst * M * b.hcap);
   b.list = w.list;
+  b.grp = w.grp;
   b.base = w.base;
   b.arr_cnt = w.arr_cnt;
   b.acc = w.acc;
@@ -533,6 +739,7 @@ template <class T> cudaError_t launch_replay(ReplayBatch<T>& b, ReplayWs& w, cud
       1, std::min<int64_t>((b.lat.n + 255) / 256, (int64_t)sms * 8));
   if (b.lat.n > 0) k_rp_valid<<<g1, 256, 0, s>>>(b.lat, M, b.win, K, w.vm, w.arr_cnt, w.n_valid);
   k_rp_fill<<<M, kFillThreads, 0, s>>>(b.lat.n, M, w.vm, w.n_valid, w.list, w.base);
+  if (b.lat.n > 0) k_rp_gather<<<g1, 256, 0, s>>>(b.lat.n, b.lat, w.list, w.base, M, w.grp);
   if ((e = cudaGetLastError())) return e;
   if (b.o_ts && b.lat.n > 0) {
     k_rp_init_records<<<(unsigned)sms * 8, 256, 0, s>>>(b.lat.n, b.n_inst, (int32_t)(K * b.win),
