@@ -68,10 +68,17 @@ def host_mapped(ptr):
     return rc == 0 and dptr.value == ptr
 
 
-def rank_seed0(rank):
-    """First trace seed of a rank's sweep: rank r sweeps traces 100 + 7r ..
-    106 + 7r, so the ranks' problems are disjoint (weak scaling)."""
-    return 100 + 7 * rank
+SWEEP_SEED0 = 100          # the sweep's traces are seeded 100 .. 106
+
+
+def idle_rank(dist, world, dev="cuda"):
+    """A rank with no trace of the sweep (more ranks than traces): it joins the
+    barriers and the whole-job reductions with nothing of its own."""
+    dist.barrier()
+    dist.barrier()
+    over_ranks(dist, dev, 0.0, [0, 0, 0, 0, 0])
+    over_ranks(dist, dev, 0.0, [])
+    dist.destroy_process_group()
 
 
 def over_ranks(dist, device, ms, units):
@@ -202,7 +209,7 @@ def run_reference(args):
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3,
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "higher_is_better": True, "scaling": "strong", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic", "config": {"workload": WORKLOAD, "sample": sample},
         "cpu_baseline": {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle",
                          "sample": sample},
@@ -593,7 +600,7 @@ def replay_measure(lib, Trace, sw, theta, scale, rank, passes=2):
     n_tr = len(sw["traces"])
     th = theta.cpu().numpy()
     for ti in range(n_tr):
-        spec = tracegen.spec_mid(scale, rank_seed0(rank) + ti, dur / 1000.0)
+        spec = tracegen.spec_mid(scale, sw["trace_seeds"][ti], dur / 1000.0)
         lat = tracegen.gen_latent(spec)
         dev = {k: torch.as_tensor(lat[k]).cuda() for k in tre.LATENT_KEYS}
         for wi, win in enumerate(sw["window_ms"]):
@@ -747,8 +754,16 @@ def main():
                     ("calls", C.c_int64 * NP), ("launches", C.c_int64 * NP)]
     lib.tre_trace_collect.argtypes = [C.POINTER(Trace)]
 
-    # each rank sweeps its own 7 traces (independent problems: weak scaling)
-    sw = tracegen.sweep_workload(scale=args.scale, seed0=rank_seed0(rank))
+    # the seven traces are independent problems: rank r sweeps traces
+    # t % world == r, so N ranks share one job (strong scaling); a rank
+    # without a trace only takes part in the collectives
+    from paper_2609_29160_gb300 import partition
+    sw = tracegen.sweep_workload(scale=args.scale, seed0=SWEEP_SEED0)
+    mine = partition.sweep_traces(len(sw["traces"]), rank, world)
+    sw["trace_seeds"] = [SWEEP_SEED0 + t for t in mine]
+    sw["traces"] = [sw["traces"][t] for t in mine]
+    if not mine:
+        return idle_rank(dist, world)
     M = sw["M"]
     win = sw["window_ms"]
     al = alphas(win)
@@ -786,17 +801,24 @@ def main():
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    # L2 is flushed (twice its size written) before every step, outside the
+    # step's pair of events: a rank's share of the records can be smaller than
+    # L2 when several ranks split the sweep
+    l2 = torch.cuda.get_device_properties(torch.cuda.current_device()).L2_cache_size
+    flush = torch.empty(2 * max(int(l2), 1 << 20), dtype=torch.uint8, device="cuda")
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(args.steps)]
     c0 = clocks.now()
-    ev0.record(stream)
-    for _ in range(args.steps):
+    for a, b in evs:
+        flush.fill_(1)
+        a.record(stream)
         out = step()
-    ev1.record(stream)
+        b.record(stream)
     torch.cuda.synchronize()
     c1 = clocks.now()
     if world > 1:
         dist.barrier()
-    ms = ev0.elapsed_time(ev1)
+    ms = sum(a.elapsed_time(b) for a, b in evs)
     tr = Trace()
     lib.tre_trace_collect(C.byref(tr))
     lib.tre_trace_enable(0)
@@ -980,18 +1002,21 @@ def main():
         base = cpu_baseline(args.scale)
         base["host"] = host_cpu()
         next_rows["occupancy_mean"]["cpu_baseline"] = occupancy_cpu(args.scale)
-        base_par = cpu_baseline_parallel(args.scale, rank_seed0(rank))
+        base_par = cpu_baseline_parallel(args.scale, SWEEP_SEED0)
     if rank == 0:
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "higher_is_better": True, "scaling": "strong", "vs_baseline": None, "dtype": "f32",
             "data": "synthetic",
             "config": {"workload": WORKLOAD, "records_per_step": int(job_rec),
                        "model_windows_per_step": int(job_mw),
                        "controller_instances": int(job_inst), "scale": args.scale,
-                       "l2": "inputs larger than L2 (7 x 28 B x ~1M records = 196 MB per step)",
-                       "parallelism": f"independent sweeps per GPU x{world}"},
+                       "l2": "flushed before every step (2x L2 written, outside the timed "
+                             "events); at one GPU the inputs are also larger than L2 "
+                             "(7 x 28 B x ~1M records = 196 MB)",
+                       "parallelism": f"the sweep's 7 traces split over {world} GPU(s) "
+                                      "(trace t on rank t % N)"},
             "model_windows_per_s": mw_s, "tokens_per_s": tok_s,
             "instance_windows_per_s": iw_s,
             "roofline": roof, "step_roofline": whole, "phases_ms_per_step": {

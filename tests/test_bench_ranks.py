@@ -1,5 +1,5 @@
-"""The multi-GPU bench path on the host: ranks sweep disjoint traces, and the
-whole-job figures are the slowest rank's time over the units of all ranks.
+"""The multi-GPU bench path on the host: ranks split the sweep's traces, and
+the whole-job figures are the slowest rank's time over the units of all ranks.
 Run as two gloo ranks on the CPU (no GPU, no NCCL)."""
 import os
 import socket
@@ -53,12 +53,46 @@ def test_over_ranks_two_gloo_ranks():
         assert ms_only == 6.0 and none == []
 
 
-def test_rank_workloads_are_disjoint():
+def test_ranks_split_the_sweep_traces():
+    """Every trace of the sweep goes to exactly one rank, for any rank count
+    (ranks beyond the trace count get none and only join the collectives)."""
     sys.path.insert(0, ROOT)
+    from paper_2609_29160_gb300 import partition
+    for world in (1, 2, 4, 7, 8):
+        got = sorted(t for r in range(world) for t in partition.sweep_traces(7, r, world))
+        assert got == list(range(7))
+        sizes = [len(partition.sweep_traces(7, r, world)) for r in range(world)]
+        assert max(sizes) - min(sizes) <= 1
+
+
+def _idle_worker(rank, world, port, q):
+    sys.path.insert(0, ROOT)
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
     import bench
-    import tracegen
-    s0, s1 = bench.rank_seed0(0), bench.rank_seed0(1)
-    assert not set(range(s0, s0 + 7)) & set(range(s1, s1 + 7))
-    a = tracegen.sweep_workload(scale=0.002, n_traces=2, seed0=s0)
-    b = tracegen.sweep_workload(scale=0.002, n_traces=2, seed0=s1)
-    assert not np.array_equal(a["traces"][0]["t_arr_ms"], b["traces"][0]["t_arr_ms"])
+    if rank == 1:
+        bench.idle_rank(dist, world, "cpu")      # the idle rank's side, on the CPU
+        q.put((rank, None, None))
+        return
+    dist.barrier()
+    dist.barrier()
+    ms, units = bench.over_ranks(dist, "cpu", 7.0, [10, 20, 30, 40, 50])
+    e2e, _ = bench.over_ranks(dist, "cpu", 9.0, [])
+    dist.destroy_process_group()
+    q.put((rank, (ms, units), e2e))
+
+
+def test_idle_rank_joins_the_collectives():
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_idle_worker, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    out = dict((r, (a, b)) for r, a, b in (q.get(timeout=120) for _ in procs))
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    (ms, units), e2e = out[0]
+    assert ms == 7.0 and units == [10.0, 20.0, 30.0, 40.0, 50.0] and e2e == 9.0
