@@ -43,6 +43,8 @@ def parse():
     ap.add_argument("--scale", type=float, default=1.0, help="request-count scale (1.0 = full)")
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-graph", action="store_true",
+                    help="issue the timed calls one by one instead of as one CUDA graph")
     ap.add_argument("--no-replay", action="store_true",
                     help="skip the closed-loop replay measured beside the sweep")
     ap.add_argument("--no-configs", action="store_true",
@@ -779,7 +781,9 @@ def main():
     inst_windows = len(sw["traces"]) * len(sw["tau_crit"]) * len(sw["pacing_cap"]) * sum(K)
     moves_cap = 512
     dev_traces = [{k: torch.as_tensor(v).cuda() for k, v in t.items()} for t in sw["traces"]]
-    stream = torch.cuda.current_stream()
+    torch.cuda.synchronize()
+    # a stream of its own: a CUDA graph cannot be captured on the default stream
+    stream = torch.cuda.Stream()
 
     # the call is marshalled once; each step is one tre_sweep call on the stream
     plan = tre.SweepPlan(dev_traces, M, sw["duration_ms"], win, al, sw["tau_crit"],
@@ -797,39 +801,93 @@ def main():
     clocks = ClockSampler(local)
     clocks.start()
     time.sleep(0.3)
-    lib.tre_trace_enable(1)
+    l2 = torch.cuda.get_device_properties(torch.cuda.current_device()).L2_cache_size
+    # Inputs larger than L2 (the whole sweep on one GPU: 196 MB) need no flush;
+    # the timed steps are then one CUDA graph of the K calls, replayed once.
+    # A rank holding less than that (several GPUs split the traces) flushes L2
+    # before every step (twice its size written), outside the step's events.
+    in_bytes = int(sum(v.numel() * v.element_size() for t in dev_traces for v in t.values()))
+    use_graph = in_bytes >= int(1.25 * l2) and not args.no_graph
+    graph = traced = None
+
+    def capture(trace_on):
+        lib.tre_trace_enable(1 if trace_on else 0)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream, capture_error_mode="relaxed"):
+            for _ in range(args.steps):
+                step()
+        with torch.cuda.stream(stream):
+            g.replay()                   # warm-up replay
+        torch.cuda.synchronize()
+        return g
+
+    if use_graph:
+        try:
+            # the timed graph carries no phase events; a second graph of the
+            # same calls with the library's phase events is replayed after it
+            graph = capture(False)
+            traced = capture(True)       # tracing stays on: its events are the phases'
+        except Exception as e:           # capture refused: time the calls one by one
+            graph = traced = None
+            graph_error = f"{type(e).__name__}: {e}"
+            lib.tre_trace_enable(0)
+    if graph is None:
+        lib.tre_trace_enable(1)
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
-    # L2 is flushed (twice its size written) before every step, outside the
-    # step's pair of events: a rank's share of the records can be smaller than
-    # L2 when several ranks split the sweep
-    l2 = torch.cuda.get_device_properties(torch.cuda.current_device()).L2_cache_size
-    flush = torch.empty(2 * max(int(l2), 1 << 20), dtype=torch.uint8, device="cuda")
-    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-           for _ in range(args.steps)]
     c0 = clocks.now()
-    for a, b in evs:
-        flush.fill_(1)
-        a.record(stream)
-        out = step()
-        b.record(stream)
-    torch.cuda.synchronize()
+    if graph is not None:
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ev0.record(stream)
+        with torch.cuda.stream(stream):
+            graph.replay()
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        ms = ev0.elapsed_time(ev1)
+    else:
+        flush = torch.empty(2 * max(int(l2), 1 << 20), dtype=torch.uint8, device="cuda")
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(args.steps)]
+        for a, b in evs:
+            with torch.cuda.stream(stream):
+                flush.fill_(1)
+            a.record(stream)
+            out = step()
+            b.record(stream)
+        torch.cuda.synchronize()
+        ms = sum(a.elapsed_time(b) for a, b in evs)
     c1 = clocks.now()
     if world > 1:
         dist.barrier()
-    ms = sum(a.elapsed_time(b) for a, b in evs)
+    if traced is not None:
+        with torch.cuda.stream(stream):
+            traced.replay()              # the phases of the same K calls
+        torch.cuda.synchronize()
     tr = Trace()
     lib.tre_trace_collect(C.byref(tr))
     lib.tre_trace_enable(0)
+    timing = {"launch": "one CUDA graph of the timed calls (phase times from a replay of a "
+                        "second graph of the same calls with the library's phase events)"
+              if graph is not None else "calls one by one, L2 flushed before each",
+              "input_bytes": in_bytes, "l2_bytes": int(l2)}
+    if use_graph and graph is None:
+        timing["graph_error"] = graph_error
     # the same step, back to back for at least 1.5 s right after the timed
     # region: long enough for the 100 ms clock samples to see the kernels
     n_sus = max(1, int(1500.0 / max(ms / args.steps, 1e-3)) + 1)
     es0, es1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     s0 = clocks.now()
     es0.record(stream)
-    for _ in range(n_sus):
-        step()
+    if graph is not None:
+        reps = max(1, n_sus // args.steps)
+        with torch.cuda.stream(stream):
+            for _ in range(reps):
+                graph.replay()
+        n_sus = reps * args.steps
+    else:
+        for _ in range(n_sus):
+            step()
     es1.record(stream)
     torch.cuda.synchronize()
     s1 = clocks.now()
@@ -1012,9 +1070,9 @@ def main():
             "config": {"workload": WORKLOAD, "records_per_step": int(job_rec),
                        "model_windows_per_step": int(job_mw),
                        "controller_instances": int(job_inst), "scale": args.scale,
-                       "l2": "flushed before every step (2x L2 written, outside the timed "
-                             "events); at one GPU the inputs are also larger than L2 "
-                             "(7 x 28 B x ~1M records = 196 MB)",
+                       "l2": "inputs larger than L2 (7 x 28 B x ~1M records = 196 MB) on one "
+                             "GPU; a rank with less flushes L2 before every step (2x L2 "
+                             "written, outside the timed events)",
                        "parallelism": f"the sweep's 7 traces split over {world} GPU(s) "
                                       "(trace t on rank t % N)"},
             "model_windows_per_s": mw_s, "tokens_per_s": tok_s,
@@ -1023,7 +1081,8 @@ def main():
                 k: p["ms"] / args.steps for k, p in phases.items() if p["calls"]},
             "phases_roofline": {k: round(roof_of(k)["frac"], 4) for k in pb
                                 if phases.get(k, {}).get("calls")},
-            "gpu_launches": launches, "clocks": clk, "sustained": sustained, "e2e": e2e,
+            "gpu_launches": launches, "clocks": clk, "sustained": sustained, "timing": timing,
+            "e2e": e2e,
             "cpu_baseline": base,
             "cpu_baseline_parallel": base_par,
             "next_rows": next_rows, "configs": configs,

@@ -476,8 +476,10 @@ tre_status tre_replay(const tre_grid* grid, const tre_latent* lat, const tre_pro
  * since tracing was enabled (or since the last collect), and starts over.
  * Phases: reduce, gauge_scan, aggregate, score, receiver, slo_counts,
  * calibrate, normalize, select, occupancy (the time-averaged occupancy pass of
- * tss_window_reduce), replay (tre_replay). No counterpart in the paper
- * (instrumentation). */
+ * tss_window_reduce), replay (tre_replay). Calls captured into a CUDA graph
+ * while tracing is on record their events as graph nodes: after a replay of
+ * the graph, tre_trace_collect returns that replay's phase times. No
+ * counterpart in the paper (instrumentation). */
 #define TRE_TRACE_PHASES 11
 typedef struct {
   int32_t n_phases;

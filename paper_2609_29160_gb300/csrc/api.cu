@@ -114,6 +114,19 @@ bool prof_ok(const tre_profile* p, bool need_theta_tau) {
   return true;
 }
 
+// An event recorded while the stream is being captured into a CUDA graph is
+// recorded as a graph node (the external flag), so a replay of the graph
+// records it and the phase can be timed from the replay.
+static cudaError_t record(cudaEvent_t e, cudaStream_t s) {
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(s, &cs) != cudaSuccess) {
+    cudaGetLastError();
+    cs = cudaStreamCaptureStatusNone;
+  }
+  return cs == cudaStreamCaptureStatusActive ? cudaEventRecordWithFlags(e, s, cudaEventRecordExternal)
+                                             : cudaEventRecord(e, s);
+}
+
 Scope::Scope(int phase, int launches, cudaStream_t st) : s(st) {
   if (!g_trace.on) return;
   a = g_trace.next();
@@ -121,11 +134,11 @@ Scope::Scope(int phase, int launches, cudaStream_t st) : s(st) {
   if (!a || !b) return;
   ph = phase;
   n = launches;
-  live = cudaEventRecord(a, s) == cudaSuccess;
+  live = record(a, s) == cudaSuccess;
 }
 
 Scope::~Scope() {
-  if (live && cudaEventRecord(b, s) == cudaSuccess) g_trace.recs.push_back(TraceRec{ph, n, a, b});
+  if (live && record(b, s) == cudaSuccess) g_trace.recs.push_back(TraceRec{ph, n, a, b});
 }
 
 }  // namespace tre
