@@ -252,6 +252,7 @@ struct WalkWs {
   uint16_t* order;    // [entry][position] model at that position
   unsigned long long* packed;  // [entry] donor order, 4 bits per position (M <= 16)
   uint32_t* dmask;             // [entry] bitmask of the models with a rank (M <= 16)
+  unsigned long long* dm64;    // [entry] the same for up to 64 models (warp walk)
 };
 // lays out the tick tables and fills b.ent_base
 template <class T> void walk_ws_layout(Arena& a, WalkBatch<T>& b, WalkWs& w);

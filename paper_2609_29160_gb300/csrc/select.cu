@@ -61,7 +61,7 @@ __device__ __forceinline__ uint8_t region_of(uint8_t c, T z, T tc, T ts) {
 template <class T>
 __global__ void __launch_bounds__(256)
 k_tick_rank(const __grid_constant__ WalkBatch<T> b, int16_t* recv_out, int16_t* ndon_out,
-            uint16_t* rank, uint16_t* order) {
+            uint16_t* rank, uint16_t* order, unsigned long long* dm64) {
   const int M = b.M;
   const int64_t gid = (int64_t)blockIdx.x * 256 + threadIdx.x;
   const int64_t total_ent = (int64_t)b.ent_base[b.n_series] * b.n_tau;
@@ -128,10 +128,16 @@ k_tick_rank(const __grid_constant__ WalkBatch<T> b, int16_t* recv_out, int16_t* 
   if (r != kNoRank) order[row * M + r] = (uint16_t)m;
   if (m == 0) {
     int nd = 0;
+    unsigned long long dm = 0;
     if (act)
-      for (int q = 0; q < M; ++q) nd += group(q, reg(q)) >= 0;
+      for (int q = 0; q < M; ++q)
+        if (group(q, reg(q)) >= 0) {
+          ++nd;
+          if (q < 64) dm |= 1ull << q;
+        }
     recv_out[row] = (int16_t)(act ? recv : -1);
     ndon_out[row] = (int16_t)nd;
+    if (dm64) dm64[row] = dm;                      // models that are donors at the tick
   }
 }
 
@@ -154,7 +160,7 @@ template <class T, int MMAX, bool QUAD>
 __global__ void __launch_bounds__(128)
 k_tick_rank_small(const __grid_constant__ WalkBatch<T> b, int16_t* recv_out, int16_t* ndon_out,
                   uint16_t* rank, uint16_t* order, unsigned long long* packed, uint32_t* dmask,
-                  bool need_rank) {
+                  bool need_rank, unsigned long long* dm64) {
   const int M = b.M;
   const int64_t e = (int64_t)blockIdx.x * 128 + threadIdx.x;
   if (e >= (int64_t)b.ent_base[b.n_series] * b.n_tau) return;
@@ -221,7 +227,7 @@ k_tick_rank_small(const __grid_constant__ WalkBatch<T> b, int16_t* recv_out, int
     nd += g >= 0;
   }
   const size_t row = (size_t)b.ent_base[s] * b.n_tau + (size_t)ti * n_ent + j;
-  unsigned long long pk = 0;
+  unsigned long long pk = 0, dmw = 0;
   uint32_t dm = 0;
 #pragma unroll
   for (int m = 0; m < MMAX; ++m) {
@@ -240,6 +246,7 @@ k_tick_rank_small(const __grid_constant__ WalkBatch<T> b, int16_t* recv_out, int
       }
       r = (uint16_t)before;
       if (need_rank) order[row * M + r] = (uint16_t)m;
+      dmw |= 1ull << m;
       if (MMAX <= 16) {
         pk |= (unsigned long long)m << (4 * before);
         dm |= 1u << m;
@@ -253,6 +260,7 @@ k_tick_rank_small(const __grid_constant__ WalkBatch<T> b, int16_t* recv_out, int
     packed[row] = pk;
     dmask[row] = dm;
   }
+  if (need_rank) dm64[row] = dmw;                  // for the warp walk
 }
 
 template <int MPL>
@@ -282,7 +290,7 @@ __device__ __forceinline__ int lane_of_min_rank(const uint16_t (&rk)[MPL], const
 template <class T, int MPL, bool STAGED>
 __global__ void __launch_bounds__(kMaxCap * 32)
 k_walk(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab, const int16_t* ndon_tab,
-       const uint16_t* rank, const uint16_t* order) {
+       const uint16_t* rank, const uint16_t* order, const unsigned long long* dm64) {
   extern __shared__ __align__(16) unsigned char dyn[];
   const int grp = blockIdx.x;                       // (series, tau)
   const int ti = grp % b.n_tau;
@@ -296,6 +304,7 @@ k_walk(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab, const in
   const size_t row0 = (size_t)b.ent_base[si] * b.n_tau + (size_t)ti * n_ent;
   const int16_t* rv_tab = recv_tab + row0;
   const int16_t* nd_tab = ndon_tab + row0;
+  const unsigned long long* dm_tab = dm64 + row0;
   const uint16_t* rk0 = rank + row0 * M;
   const uint16_t* od0 = order + row0 * M;
   if (STAGED) {
@@ -369,6 +378,29 @@ k_walk(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab, const in
   // ceil(j*c / win) - 1; keep j*c as quotient and remainder of win
   TickSeq sf((int32_t)F, (int32_t)win), ss((int32_t)Sl, (int32_t)win);
   int32_t jf = 1, js = 1;
+  // the receivers of the coming 32 fast and 32 slow ticks, one per lane: most
+  // ticks move nothing, and a tick then costs a shuffle instead of a load
+  int32_t fb0 = -64, sb0 = -64;                 // entries >= 0: the first access loads
+  int fbuf = -1, sbuf = -1;
+  auto rv_at = [&](int32_t e, int32_t& b0, int& buf) {
+    if ((uint32_t)(e - b0) >= 32u) {
+      b0 = e;
+      buf = e + lane < n_ent ? rv_tab[e + lane] : -1;
+    }
+    return __shfl_sync(0xffffffffu, buf, e - b0);
+  };
+  // the donor sets of the same ticks (models with a rank), for up to 64
+  // models: a tick whose receiver the pool cannot serve and whose donors all
+  // sit at their floors moves nothing, and costs no row load
+  int32_t fm0 = -64, sm0 = -64;
+  unsigned long long fmb = 0, smb = 0;
+  auto dm_at = [&](int32_t e, int32_t& b0, unsigned long long& buf) {
+    if ((uint32_t)(e - b0) >= 32u) {
+      b0 = e;
+      buf = e + lane < n_ent ? dm_tab[e + lane] : 0ull;
+    }
+    return __shfl_sync(0xffffffffu, buf, e - b0);
+  };
   while (true) {
     const int32_t kf = sf.window(), ks = ss.window();
     const int32_t k = kf < ks ? kf : ks;
@@ -380,14 +412,29 @@ k_walk(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab, const in
     int recv = -1, kind = 0;
     int32_t ent = -1;
     if (fast) {
-      const int rv = rv_tab[ef];
+      const int rv = rv_at(ef, fb0, fbuf);
       if (rv >= 0) { recv = rv; ent = ef; kind = TRE_RESCUE; }
     }
     if (!kind && slow) {
-      const int rv = rv_tab[es];
+      const int rv = rv_at(es, sb0, sbuf);
       if (rv >= 0) { recv = rv; ent = es; kind = TRE_REBALANCE; }
     }
     if (!kind) continue;
+    if (MPL <= 2) {
+      const unsigned long long donors =
+          ent < (int32_t)nf ? dm_at(ent, fm0, fmb) : dm_at(ent, sm0, smb);
+      unsigned long long above = 0;
+#pragma unroll
+      for (int j = 0; j < MPL; ++j)
+        above |= (unsigned long long)__ballot_sync(0xffffffffu, lane + 32 * j < M && r[j] > rmin[j])
+                 << (32 * j);
+      int g_rv = 0;
+#pragma unroll
+      for (int j = 0; j < MPL; ++j)
+        if (lane + 32 * j == recv) g_rv = g[j];
+      const int need_rv = __shfl_sync(0xffffffffu, g_rv, recv & 31);
+      if (free_pool < need_rv && !(donors & above)) continue;
+    }
     if (closed) {
       const int nd = nd_tab[ent];
       const int mo = lane < nd ? od0[(size_t)ent * M + lane] : -1;
@@ -720,7 +767,7 @@ struct __align__(16) TickRec {
 template <class T, int MMAX>
 __global__ void __launch_bounds__(256, 1)
 k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
-            const unsigned long long* packed, const uint32_t* dmask) {
+            const unsigned long long* packed, const uint32_t* dmask, bool store_win) {
   extern __shared__ __align__(16) unsigned char dyn[];
   const int grp = blockIdx.x;
   const int ti = grp % b.n_tau;
@@ -738,9 +785,15 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
   // u <= nf: for every model the next tick >= u where it is a donor (one
   // 2*MMAX-byte row per tick, so a row is read with 16-byte loads), and the
   // next tick >= u where anything acts
+  // (the window of each tick is staged when there is room, else recomputed
+  // at each visit)
   TickRec* srec = reinterpret_cast<TickRec*>(dyn);
   int32_t* swin = reinterpret_cast<int32_t*>(srec + nf);
-  uint16_t* snx = reinterpret_cast<uint16_t*>(swin + ((nf + 3) & ~3));   // [nf + 1][MMAX]
+  uint16_t* snx = store_win ? reinterpret_cast<uint16_t*>(swin + ((nf + 3) & ~3))
+                            : reinterpret_cast<uint16_t*>(swin);           // [nf + 1][MMAX]
+  auto tick_win = [&](int u) -> int32_t {
+    return store_win ? swin[u] : (int32_t)tick_window(u + 1, b.fast_ms, win);
+  };
   uint16_t* sany = snx + (size_t)(nf + 1) * MMAX;                          // [nf + 1]
   __shared__ int s_cap[8][MMAX];   // unit footprints: replicas above the floor, per warp
   for (int u = threadIdx.x; u < nf; u += blockDim.x) {
@@ -760,7 +813,7 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
     t.kind = (uint8_t)kd;
     t.pad = 0;
     srec[u] = t;
-    swin[u] = (int32_t)tick_window(u + 1, b.fast_ms, win);
+    if (store_win) swin[u] = (int32_t)tick_window(u + 1, b.fast_ms, win);
   }
   __syncthreads();
   // next-tick tables: a suffix minimum per row, 32 ticks per step
@@ -871,7 +924,7 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
         if (nxt >= nf) break;
         u = nxt + 1;
         const TickRec tr = srec[nxt];
-        const int32_t k = swin[nxt];
+        const int32_t k = tick_win(nxt);
         const int recv = tr.recv;
         int donor = -1;
         if (free_pool > 0) {
@@ -910,7 +963,7 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
         if (nxt >= nf) break;
         u = nxt + 1;
         const TickRec tr = srec[nxt];
-        const int32_t k = swin[nxt];
+        const int32_t k = tick_win(nxt);
         const int recv = tr.recv;
         int donor = -1;
         if (free_pool > 0) {
@@ -944,7 +997,7 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
       if (nxt >= nf) break;
       u = nxt;
       const TickRec tr = srec[u];
-      const int32_t k = swin[u];
+      const int32_t k = tick_win(u);
       ++u;
       const int recv = tr.recv;
       if (recv < 0) continue;
@@ -1019,7 +1072,7 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
     const TickRec tr = srec[u];
     const int recv = tr.recv;
     const int kind = tr.kind;
-    const int32_t k = swin[u];
+    const int32_t k = tick_win(u);
     ++u;
     if (recv < 0) continue;
     const uint32_t usable = avail & tr.dm;
@@ -1110,9 +1163,9 @@ cudaError_t walk_launch(const WalkBatch<T>& b, WalkWs& w, cudaStream_t s) {
   if (smem <= kStageMax) {
     cudaError_t e = func_smem_once((const void*)k_walk<T, MPL, true>, (int)kStageMax, false);
     if (e) return e;
-    k_walk<T, MPL, true><<<grid, th, smem, s>>>(b, w.recv, w.n_donor, w.rank, w.order);
+    k_walk<T, MPL, true><<<grid, th, smem, s>>>(b, w.recv, w.n_donor, w.rank, w.order, w.dm64);
   } else {
-    k_walk<T, MPL, false><<<grid, th, 0, s>>>(b, w.recv, w.n_donor, w.rank, w.order);
+    k_walk<T, MPL, false><<<grid, th, 0, s>>>(b, w.recv, w.n_donor, w.rank, w.order, w.dm64);
   }
   return cudaGetLastError();
 }
@@ -1133,34 +1186,48 @@ template <class T> void walk_ws_layout(Arena& a, WalkBatch<T>& b, WalkWs& w) {
   w.order = a.take<uint16_t>((size_t)std::max<int64_t>(total * b.n_tau * b.M, 1));
   w.packed = a.take<unsigned long long>((size_t)std::max<int64_t>(total * b.n_tau, 1));
   w.dmask = a.take<uint32_t>((size_t)std::max<int64_t>(total * b.n_tau, 1));
+  w.dm64 = a.take<unsigned long long>((size_t)std::max<int64_t>(total * b.n_tau, 1));
 }
 
 // unit footprints and few models: thread-per-instance walk with staged tables
 template <class T, int MMAX>
 cudaError_t walk_thread_launch(const WalkBatch<T>& b, WalkWs& w, size_t smem, cudaStream_t s) {
   cudaError_t e = func_smem_once((const void*)k_walk_thread<T, MMAX>, (int)kStageMax, false);
-  if (!e) e = func_smem_once((const void*)k_walk_jump<T, MMAX>, (int)kStageMax, false);
   if (e) return e;
   // nested cadences with a fast tick not shorter than a window: jump between
   // possible moves
   if (b.slow_ms % b.fast_ms == 0 && b.fast_ms >= b.series_win[0]) {
     bool ok = true;
-    size_t jsmem = 0;
+    size_t jsmem = 0, wsmem = 0;   // tables, and the staged tick windows
     for (int i = 0; i < b.n_series; ++i) {
       if (b.fast_ms < b.series_win[i]) ok = false;
-      const int n_ent = b.ent_base[i + 1] - b.ent_base[i];
       const int64_t nf = (int64_t)b.series_K[i] * b.series_win[i] / b.fast_ms;
       if (nf >= 32767) ok = false;
-      const size_t need = (size_t)nf * sizeof(TickRec) + (size_t)((nf + 3) & ~3) * 4 +
-                          (size_t)(nf + 1) * MMAX * 2 + (size_t)(nf + 1) * 2;
+      const size_t need = (size_t)nf * sizeof(TickRec) + (size_t)(nf + 1) * MMAX * 2 +
+                          (size_t)(nf + 1) * 2;
       jsmem = std::max(jsmem, need);
+      wsmem = std::max(wsmem, (size_t)((nf + 3) & ~3) * 4);
     }
-    if (ok && jsmem <= kStageMax) {
-      const int warps = std::min(8, std::max(1, b.n_cap));
-      k_walk_jump<T, MMAX><<<b.n_series * b.n_tau, 32 * warps, jsmem, s>>>(b, w.recv, w.packed,
-                                                                           w.dmask);
-      return cudaGetLastError();
+    // the largest dynamic shared memory a block may opt into, beside the
+    // kernel's static per-warp counts
+    int dev = 0, optin = 0;
+    if (cudaGetDevice(&dev) == cudaSuccess &&
+        cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) ==
+            cudaSuccess && optin > 4096) {
+      const size_t lim = (size_t)optin - 2048;
+      const bool store_win = jsmem + wsmem <= lim;
+      const size_t smem_j = store_win ? jsmem + wsmem : jsmem;
+      if (ok && smem_j <= lim) {
+        e = func_smem_once((const void*)k_walk_jump<T, MMAX>, (int)lim, false);
+        if (e) return e;
+        // eight warps build the tick tables; the first n_cap of them walk
+        const int warps = 8;
+        k_walk_jump<T, MMAX><<<b.n_series * b.n_tau, 32 * warps, smem_j, s>>>(
+            b, w.recv, w.packed, w.dmask, store_win);
+        return cudaGetLastError();
+      }
     }
+    cudaGetLastError();
   }
   k_walk_thread<T, MMAX><<<b.n_series * b.n_tau, 32, smem, s>>>(b, w.recv, w.packed, w.dmask);
   return cudaGetLastError();
@@ -1183,20 +1250,20 @@ template <class T> cudaError_t launch_walk(const WalkBatch<T>& b, WalkWs& w, cud
         b.M % 4 == 0 && (((uintptr_t)b.Z | (uintptr_t)b.cls) & 15) == 0;
     if (b.M <= 8 && quad) {
       k_tick_rank_small<T, 8, true><<<g, 128, 0, s>>>(b, w.recv, w.n_donor, w.rank, w.order,
-                                                      w.packed, w.dmask, !thread_walk);
+                                                      w.packed, w.dmask, !thread_walk, w.dm64);
     } else if (b.M <= 8) {
       k_tick_rank_small<T, 8, false><<<g, 128, 0, s>>>(b, w.recv, w.n_donor, w.rank, w.order,
-                                                       w.packed, w.dmask, !thread_walk);
+                                                       w.packed, w.dmask, !thread_walk, w.dm64);
     } else if (b.M <= 16) {
       k_tick_rank_small<T, 16, false><<<g, 128, 0, s>>>(b, w.recv, w.n_donor, w.rank, w.order,
-                                                        w.packed, w.dmask, !thread_walk);
+                                                        w.packed, w.dmask, !thread_walk, w.dm64);
     } else if (b.M <= 32) {
       k_tick_rank_small<T, 32, false><<<g, 128, 0, s>>>(b, w.recv, w.n_donor, w.rank, w.order,
-                                                        w.packed, w.dmask, true);
+                                                        w.packed, w.dmask, true, w.dm64);
     } else {
       const int64_t th = ents * b.M;
       k_tick_rank<T><<<(unsigned)((th + 255) / 256), 256, 0, s>>>(b, w.recv, w.n_donor, w.rank,
-                                                                   w.order);
+                                                                   w.order, w.dm64);
     }
   }
   if (thread_walk)

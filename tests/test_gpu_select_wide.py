@@ -158,3 +158,12 @@ def test_sweep_twenty_four_models(tre):
         np.testing.assert_array_equal(got, ref_m, err_msg=f"instance {i}")
         total += len(om)
     assert total > 0
+
+
+def test_jump_walk_long_series_sixteen_models(tre):
+    """Sixteen models over 43,200 windows of 500 ms (the code/chat workload's
+    shape): the jump walk's tables fill nearly all of a block's shared memory,
+    and the tick windows are recomputed at each visit instead of staged."""
+    Z, cls, g, r0, budget, r_min = _case(16, 43200, 16, idle=0.05)
+    for cap in (1, 2):
+        _check(tre, Z, cls, g, r0, budget, r_min, 500, cap)
