@@ -7,8 +7,9 @@
 // sequential definition (one rounding per operation, in order):
 //   1. the windows of each series are cut into chunks; one thread per (chunk,
 //      model) first runs the recurrence over the B windows before its chunk
-//      ("burn-in", started as if the series began there; B ~ 28 / -ln(1-alpha),
-//      so a start error shrinks by e^-28 before the chunk), records the state
+//      ("burn-in", started as if the series began there; B ~ c / -ln(1-alpha),
+//      so a start error shrinks by e^-c before the chunk: c = 28 for float, 45
+//      for double), records the state
 //      it reached, then runs its chunk from that state and stores the result;
 //   2. one thread per model walks the chunk boundaries in order: a chunk whose
 //      recorded burn-in state equals its predecessor's exact end state (bit
@@ -362,13 +363,17 @@ k_ema(const __grid_constant__ SeriesTable<T> tab, const T* __restrict__ raw, con
   const ModelParams<T> q = load_params(tab, s, m, alpha, theta, tau_crit, tau_surp);
   const int L = tab.seg_len[s];
   const int64_t k0 = (int64_t)(seg - tab.seg_base[s]) * L, k1 = min64(k0 + L, tab.K[s]);
-  // burn-in length: (1 - alpha)^B <= e^-28, in whole ring strides
+  // burn-in length: (1 - alpha)^B <= e^-c, in whole ring strides, with c well
+  // past the point where a start error falls below the type's last bit, so
+  // that the rounded trajectories have met (c = 28 for float's 6e-8 = e^-16.6,
+  // 45 for double's 1.1e-16 = e^-36.7)
   int B = kMaxBurn;
   {
     const float a = (float)q.a;
+    const float c = sizeof(T) == 4 ? 28.f : 45.f;
     if (a >= 1.f) B = kRingStride;
     else if (a > 0.f) {
-      const float x = 28.f / -log1pf(-a);
+      const float x = c / -log1pf(-a);
       if (x < (float)kMaxBurn) B = (int)x + 1;
     }
     B = (B + kRingStride - 1) / kRingStride * kRingStride;
