@@ -176,6 +176,7 @@ template <class T> struct ScoreWs {
   int32_t* start_init;
   T* end_S;                    // per (segment, model): state after the segment
   int32_t* end_init;
+  int32_t* active;             // per (segment, model): non-idle windows (long tables)
   int cap_seg;                 // segments the arrays hold (per model)
 };
 template <class T> void score_ws_layout(Arena& a, int M, int64_t elems, int n_seg, ScoreWs<T>& w);

@@ -286,6 +286,51 @@ __device__ __forceinline__ bool run_segment(size_t base, int M, int64_t k0, int6
   return false;
 }
 
+// ---- non-idle windows per (chunk, model) ----------------------------------
+// One CTA per chunk: its windows are consecutive rows of [K][M], read 16 bytes
+// at a time; idle windows are counted per model in shared memory.
+template <class T>
+__global__ void __launch_bounds__(256)
+k_active(const __grid_constant__ SeriesTable<T> tab, FastDiv fm, const uint8_t* __restrict__ cls,
+         int32_t* __restrict__ active) {
+  extern __shared__ int32_t s_idle[];
+  const int seg = blockIdx.x;
+  const int s = series_of_seg(tab, seg);
+  const int M = tab.M, L = tab.seg_len[s];
+  const int64_t k0 = (int64_t)(seg - tab.seg_base[s]) * L, k1 = min64(k0 + L, tab.K[s]);
+  for (int m = threadIdx.x; m < M; m += blockDim.x) s_idle[m] = 0;
+  __syncthreads();
+  const uint8_t* base = cls + tab.off[s] + (size_t)k0 * M;
+  const uint32_t n = (uint32_t)((k1 - k0) * M);
+  // bytes before the first 16-byte boundary, then whole 16-byte words, then the rest
+  const uint32_t head = min(n, (uint32_t)((16 - ((uintptr_t)base & 15)) & 15));
+  const uint32_t n16 = (n - head) / 16;
+  auto count = [&](uint32_t i, uint8_t v) {
+    if (v == kIdle) atomicAdd(&s_idle[i - fm.div(i) * (uint32_t)M], 1);
+  };
+  for (uint32_t i = threadIdx.x; i < head; i += blockDim.x) count(i, base[i]);
+  const uint4* q = reinterpret_cast<const uint4*>(base + head);
+  for (uint32_t w = threadIdx.x; w < n16; w += blockDim.x) {
+    const uint4 v = q[w];
+    const uint32_t ws[4] = {v.x, v.y, v.z, v.w};
+    // a word with no idle byte needs no per-byte work
+    bool any = false;
+#pragma unroll
+    for (int h = 0; h < 4; ++h) any |= __vcmpeq4(ws[h], kIdle * 0x01010101u) != 0;
+    if (!any) continue;
+    const uint32_t i0 = head + 16 * w;
+#pragma unroll
+    for (int h = 0; h < 4; ++h)
+#pragma unroll
+      for (int j = 0; j < 4; ++j) count(i0 + 4 * h + j, (uint8_t)(ws[h] >> (8 * j)));
+  }
+  for (uint32_t i = head + 16 * n16 + threadIdx.x; i < n; i += blockDim.x) count(i, base[i]);
+  __syncthreads();
+  const int rows = (int)(n / (uint32_t)M);
+  for (int m = threadIdx.x; m < M; m += blockDim.x)
+    active[(size_t)seg * M + m] = rows - s_idle[m];
+}
+
 // ---- pass 1: burn-in and chunk run, one thread per (chunk, model) ----------
 // Each thread streams its model's windows through its own slots of a shared
 // memory ring with asynchronous copies (cp.async, kStages groups of kBlk
@@ -296,6 +341,8 @@ constexpr int kBlk = 16;           // windows per copy group
 constexpr int kStages = 8;         // copy groups in flight
 constexpr int kRingStride = 64;    // chunk and burn-in lengths are multiples of this
 constexpr int kMaxBurn = 16384;    // burn-in cap (tiny alpha: the in-order pass repairs)
+constexpr int64_t kActiveMinCells = 1 << 22;   // series cells from which burn-ins skip idle chunks
+constexpr int64_t kEmaChains = 32768;         // (chunk, model) chains a long table is cut into
 
 template <int BYTES>
 __device__ __forceinline__ void cp_async(void* smem, const void* gmem) {
@@ -349,9 +396,9 @@ template <class T, bool WITHZ>
 __global__ void __launch_bounds__(kEmaThreads)
 k_ema(const __grid_constant__ SeriesTable<T> tab, const T* __restrict__ raw, const T* alpha,
       const T* theta, const T* tau_crit, const T* tau_surp, const T* S_carry,
-      const uint8_t* init_carry, T* __restrict__ b_S, int32_t* __restrict__ b_init,
-      T* __restrict__ e_S, int32_t* __restrict__ e_init, T* __restrict__ S_out,
-      T* __restrict__ Z_out, uint8_t* __restrict__ cls) {
+      const uint8_t* init_carry, const int32_t* __restrict__ active, T* __restrict__ b_S,
+      int32_t* __restrict__ b_init, T* __restrict__ e_S, int32_t* __restrict__ e_init,
+      T* __restrict__ S_out, T* __restrict__ Z_out, uint8_t* __restrict__ cls) {
   __shared__ T ring[kStages * kBlk * kEmaThreads];
   const int M = tab.M;
   const int lane = threadIdx.x;
@@ -363,10 +410,10 @@ k_ema(const __grid_constant__ SeriesTable<T> tab, const T* __restrict__ raw, con
   const ModelParams<T> q = load_params(tab, s, m, alpha, theta, tau_crit, tau_surp);
   const int L = tab.seg_len[s];
   const int64_t k0 = (int64_t)(seg - tab.seg_base[s]) * L, k1 = min64(k0 + L, tab.K[s]);
-  // burn-in length: (1 - alpha)^B <= e^-c, in whole ring strides, with c well
-  // past the point where a start error falls below the type's last bit, so
-  // that the rounded trajectories have met (c = 28 for float's 6e-8 = e^-16.6,
-  // 45 for double's 1.1e-16 = e^-36.7)
+  // burn-in length, in updates (non-idle windows): (1 - alpha)^B <= e^-c, in
+  // whole ring strides, with c well past the point where a start error falls
+  // below the type's last bit, so that the rounded trajectories have met
+  // (c = 28 for float's 6e-8 = e^-16.6, 45 for double's 1.1e-16 = e^-36.7)
   int B = kMaxBurn;
   {
     const float a = (float)q.a;
@@ -378,37 +425,95 @@ k_ema(const __grid_constant__ SeriesTable<T> tab, const T* __restrict__ raw, con
     }
     B = (B + kRingStride - 1) / kRingStride * kRingStride;
   }
-  int64_t kb = k0 - B;
+  // The burn-in runs over spans of windows [sp_lo, sp_hi), ascending. Without
+  // activity counts it is the one span [k0 - B, k0). With them (non-idle
+  // windows per chunk) it walks back over the preceding chunks until they hold
+  // B non-idle windows, leaving out chunks that are wholly idle: an idle window
+  // leaves the state as it is, so the trajectory is the same without them,
+  // and a burn-in across a long idle stretch still sees enough updates.
+  constexpr int kSpans = 8;
+  int64_t sp_lo[kSpans], sp_hi[kSpans];
+  int nsp = 0;
+  bool from_start = false;   // the burn-in covers every update since window 0
+  if (active == nullptr) {
+    int64_t kb = k0 - B;
+    if (kb <= 0) {
+      kb = 0;
+      from_start = true;
+    }
+    if (kb < k0) {
+      sp_lo[0] = kb;
+      sp_hi[0] = k0;
+      nsp = 1;
+    }
+  } else {
+    int64_t acc = 0;
+    int cb = seg - tab.seg_base[s];
+    const int32_t* act = active + (size_t)tab.seg_base[s] * M + m;
+    while (acc < B) {
+      if (cb == 0) {
+        from_start = true;
+        break;
+      }
+      --cb;
+      const int na = act[(size_t)cb * M];
+      if (na == 0) continue;
+      const int64_t hi = (int64_t)(cb + 1) * L;   // chunks before this one are whole
+      int64_t lo = (int64_t)cb * L;
+      if (na == L && acc + L > B)
+        lo = hi - (B - acc + kRingStride - 1) / kRingStride * kRingStride;
+      acc += na == L ? hi - lo : na;
+      if (nsp > 0 && sp_lo[nsp - 1] == hi) {
+        sp_lo[nsp - 1] = lo;
+      } else if (nsp < kSpans) {
+        sp_lo[nsp] = lo;
+        sp_hi[nsp] = hi;
+        ++nsp;
+      } else {
+        break;   // out of spans: a shorter burn-in, repaired by the in-order pass if short
+      }
+    }
+    for (int i = 0; i < nsp / 2; ++i) {
+      const int64_t l = sp_lo[i], h = sp_hi[i];
+      sp_lo[i] = sp_lo[nsp - 1 - i];
+      sp_hi[i] = sp_hi[nsp - 1 - i];
+      sp_lo[nsp - 1 - i] = l;
+      sp_hi[nsp - 1 - i] = h;
+    }
+  }
   T S = (T)0;
   int init = 0;
-  if (kb <= 0) {   // the burn-in reaches the series start: begin from the true state
-    kb = 0;
+  if (from_start) {   // begin from the true state
     init = (init_carry && init_carry[m]) ? 1 : 0;
     S = init ? S_carry[m] : (T)0;
   }
   const size_t base = (size_t)tab.off[s] + m;
-  const int n_grp = (int)((k1 - kb + kBlk - 1) / kBlk);
-  const int burn_grp = (int)((k0 - kb) / kBlk);
-  // group g holds windows kb + g*kBlk .. + kBlk-1 in stage g % kStages
-  const T* src_next = raw + base + (size_t)kb * M;
+  int burn_grp = 0;
+  for (int i = 0; i < nsp; ++i) burn_grp += (int)((sp_hi[i] - sp_lo[i]) / kBlk);
+  const int n_grp = burn_grp + (int)((k1 - k0 + kBlk - 1) / kBlk);
+  // groups are issued in order: the spans of the burn-in, then the chunk; a
+  // group never straddles two spans (span lengths are multiples of kBlk)
+  int cur = 0;
+  int64_t cur_k = nsp > 0 ? sp_lo[0] : k0, cur_end = nsp > 0 ? sp_hi[0] : k1;
   const size_t step = (size_t)M;
   auto issue = [&](int g) {
     if (g < n_grp) {
       T* dst = ring + (size_t)(g % kStages) * kBlk * kEmaThreads + lane;
-      if (g + 1 < n_grp) {
+      const T* src = raw + base + (size_t)cur_k * M;
+      const int64_t left = cur_end - cur_k;
+      if (left >= kBlk) {
 #pragma unroll
-        for (int j = 0; j < kBlk; ++j) {
-          cp_async<sizeof(T)>(dst + j * kEmaThreads, src_next);
-          src_next += step;
-        }
+        for (int j = 0; j < kBlk; ++j) cp_async<sizeof(T)>(dst + j * kEmaThreads, src + j * step);
       } else {
-        const int n = (int)(k1 - (kb + (int64_t)g * kBlk));
 #pragma unroll
         for (int j = 0; j < kBlk; ++j)
-          if (j < n) {
-            cp_async<sizeof(T)>(dst + j * kEmaThreads, src_next);
-            src_next += step;
-          }
+          if (j < left) cp_async<sizeof(T)>(dst + j * kEmaThreads, src + j * step);
+      }
+      cur_k += left < kBlk ? left : kBlk;
+      if (cur_k >= cur_end && cur < nsp) {
+        ++cur;
+        cur_k = cur < nsp ? sp_lo[cur] : k0;
+        cur_end = cur < nsp ? sp_hi[cur] : k1;
       }
     }
     cp_async_commit();
@@ -436,7 +541,7 @@ k_ema(const __grid_constant__ SeriesTable<T> tab, const T* __restrict__ raw, con
   }
   cp_async_wait<0>();
   {
-    const int n = (int)(k1 - (kb + (int64_t)g * kBlk));
+    const int n = (int)(k1 - (k0 + (int64_t)(g - burn_grp) * kBlk));
     ema_group<T, false, false, true, WITHZ>(stage_of(g), n, q, S, init, sp, M, S_out, Z_out, cls);
   }
   e_S[t] = S;
@@ -786,13 +891,17 @@ template <class T> int64_t total_elems(const SeriesTable<T>& t) {
 
 template <class T> int series_segments(SeriesTable<T>& t) {
   int total = 0;
+  int64_t cells = 0;
+  for (int s = 0; s < t.n; ++s) cells += (int64_t)t.K[s] * t.M;
   for (int s = 0; s < t.n; ++s) {
     const int K = t.K[s];
-    // chunks of 256 windows (longer for very long series, to bound the count);
-    // a multiple of the smoothing pass's ring stride
+    // chunks of 256 windows, longer for very long series (to bound the count)
+    // and for large tables: about kEmaChains chains keep the GPU busy, and
+    // longer chunks re-read fewer windows in their burn-ins; a multiple of the
+    // smoothing pass's ring stride
     int L = 256;
-    const int need = (K + 2047) / 2048;
-    if (need > L) L = (need + kRingStride - 1) / kRingStride * kRingStride;
+    int64_t need = std::max<int64_t>((K + 2047) / 2048, cells / kEmaChains);
+    if (need > L) L = (int)((need + kRingStride - 1) / kRingStride * kRingStride);
     t.seg_len[s] = L;
     t.seg_base[s] = total;
     total += (K + L - 1) / L;
@@ -809,6 +918,7 @@ template <class T> void score_ws_layout(Arena& a, int M, int64_t elems, int n_se
   w.start_init = a.take<int32_t>(n);
   w.end_S = a.take<T>(n);
   w.end_init = a.take<int32_t>(n);
+  w.active = a.take<int32_t>(n);
 }
 
 template <class T>
@@ -838,14 +948,22 @@ cudaError_t launch_score(const SeriesTable<T>& tab, const int32_t* P, const int3
   }
   const int64_t segs = (int64_t)n_seg * M;
   const unsigned g = (unsigned)((segs + kEmaThreads - 1) / kEmaThreads);
+  // activity counts for the burn-ins where the series are long enough that
+  // idle stretches would otherwise send chunks to the in-order pass, and the
+  // extra pass over the classes is small beside the smoothing
+  const int32_t* active = nullptr;
+  if (total >= kActiveMinCells) {
+    k_active<T><<<n_seg, 256, (size_t)M * sizeof(int32_t), s>>>(tab, FastDiv(M), cls, w.active);
+    active = w.active;
+  }
   if (theta)
     k_ema<T, true><<<g, kEmaThreads, 0, s>>>(tab, w.raw, alpha, theta, tau_crit, tau_surp,
-                                             S_carry, init_carry, w.start_S, w.start_init,
-                                             w.end_S, w.end_init, S, Z, cls);
+                                             S_carry, init_carry, active, w.start_S,
+                                             w.start_init, w.end_S, w.end_init, S, Z, cls);
   else
     k_ema<T, false><<<g, kEmaThreads, 0, s>>>(tab, w.raw, alpha, theta, tau_crit, tau_surp,
-                                              S_carry, init_carry, w.start_S, w.start_init,
-                                              w.end_S, w.end_init, S, Z, cls);
+                                              S_carry, init_carry, active, w.start_S,
+                                              w.start_init, w.end_S, w.end_init, S, Z, cls);
   const int warps = tab.n * M;
   k_resolve<T><<<(warps + 1) / 2, 64, 0, s>>>(tab, w.raw, alpha, theta, tau_crit, tau_surp,
                                                 w.start_S, w.start_init, w.end_S, w.end_init,

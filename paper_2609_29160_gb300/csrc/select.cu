@@ -401,40 +401,8 @@ k_walk(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab, const in
     }
     return __shfl_sync(0xffffffffu, buf, e - b0);
   };
-  while (true) {
-    const int32_t kf = sf.window(), ks = ss.window();
-    const int32_t k = kf < ks ? kf : ks;
-    if (k >= K) break;
-    const bool fast = kf == k, slow = ks == k;
-    const int32_t ef = jf - 1, es = (int32_t)nf + js - 1;   // entries of this tick
-    while (sf.window() <= k) { sf.next(); ++jf; }
-    while (ss.window() <= k) { ss.next(); ++js; }
-    int recv = -1, kind = 0;
-    int32_t ent = -1;
-    if (fast) {
-      const int rv = rv_at(ef, fb0, fbuf);
-      if (rv >= 0) { recv = rv; ent = ef; kind = TRE_RESCUE; }
-    }
-    if (!kind && slow) {
-      const int rv = rv_at(es, sb0, sbuf);
-      if (rv >= 0) { recv = rv; ent = es; kind = TRE_REBALANCE; }
-    }
-    if (!kind) continue;
-    if (MPL <= 2) {
-      const unsigned long long donors =
-          ent < (int32_t)nf ? dm_at(ent, fm0, fmb) : dm_at(ent, sm0, smb);
-      unsigned long long above = 0;
-#pragma unroll
-      for (int j = 0; j < MPL; ++j)
-        above |= (unsigned long long)__ballot_sync(0xffffffffu, lane + 32 * j < M && r[j] > rmin[j])
-                 << (32 * j);
-      int g_rv = 0;
-#pragma unroll
-      for (int j = 0; j < MPL; ++j)
-        if (lane + 32 * j == recv) g_rv = g[j];
-      const int need_rv = __shfl_sync(0xffffffffu, g_rv, recv & 31);
-      if (free_pool < need_rv && !(donors & above)) continue;
-    }
+  // the transitions of one tick: window k, receiver recv, table entry ent
+  auto act = [&](int32_t k, int recv, int kind, int32_t ent) {
     if (closed) {
       const int nd = nd_tab[ent];
       const int mo = lane < nd ? od0[(size_t)ent * M + lane] : -1;
@@ -468,7 +436,7 @@ k_walk(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab, const in
       if (lane == recv) r[0] += n_pool + t_d;
       free_pool -= n_pool;
       nm += n_pool + t_d;
-      continue;
+      return;
     }
     uint16_t rk[MPL];
 #pragma unroll
@@ -522,6 +490,98 @@ k_walk(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab, const in
         if (lane + 32 * j == recv) r[j] += 1;
       }
       free_pool = f - need;
+    }
+  };
+  // Nested cadences (the slow tick a multiple of the fast one, the fast tick
+  // at least a window): the ticks are the fast ticks u = 0 .. nf-1, and fast
+  // tick u also carries slow tick (u+1)/ratio when ratio divides u+1. The
+  // replica state only changes where a tick moves something, so 32 ticks are
+  // tested at once against the current state (a receiver, and either room in
+  // the pool for its footprint or a donor above its floor) and the walk jumps
+  // to the first that can act.
+  if (MPL <= 2 && F >= win && Sl % F == 0) {
+    const int64_t ratio = Sl / F;
+    int64_t u0 = 0;
+    while (u0 < nf) {
+      unsigned long long above = 0;
+#pragma unroll
+      for (int j = 0; j < MPL; ++j)
+        above |= (unsigned long long)__ballot_sync(0xffffffffu, lane + 32 * j < M && r[j] > rmin[j])
+                 << (32 * j);
+      const int64_t u = u0 + lane;
+      int rv = -1, kind = 0;
+      int32_t ent = -1;
+      unsigned long long dn = 0;
+      if (u < nf) {
+        const int32_t es = (int32_t)(nf + (u + 1) / ratio - 1);
+        const bool has_slow = (u + 1) % ratio == 0 && es < n_ent;
+        const int rf = rv_tab[u];
+        const int rs = has_slow ? rv_tab[es] : -1;
+        const unsigned long long df = dm_tab[u];
+        const unsigned long long ds = has_slow ? dm_tab[es] : 0ull;
+        if (rf >= 0) {
+          rv = rf; kind = TRE_RESCUE; ent = (int32_t)u; dn = df;
+        } else if (rs >= 0) {
+          rv = rs; kind = TRE_REBALANCE; ent = es; dn = ds;
+        }
+      }
+      // the receiver's footprint sits in lane rv % 32, slot rv / 32
+      int g_rv = 0;
+#pragma unroll
+      for (int j = 0; j < MPL; ++j) {
+        const int x = __shfl_sync(0xffffffffu, g[j], rv & 31);
+        if (rv >= 0 && (rv >> 5) == j) g_rv = x;
+      }
+      const bool can = rv >= 0 && (free_pool >= g_rv || (dn & above) != 0);
+      const unsigned hit = __ballot_sync(0xffffffffu, can);
+      if (!hit) {
+        u0 += 32;
+        continue;
+      }
+      const int src = __ffs(hit) - 1;
+      const int32_t e_t = __shfl_sync(0xffffffffu, ent, src);
+      const int rv_t = __shfl_sync(0xffffffffu, rv, src);
+      const int kd_t = __shfl_sync(0xffffffffu, kind, src);
+      const int64_t ut = u0 + src;
+      act((int32_t)tick_window(ut + 1, F, win), rv_t, kd_t, e_t);
+      u0 = ut + 1;
+    }
+  } else {
+    while (true) {
+      const int32_t kf = sf.window(), ks = ss.window();
+      const int32_t k = kf < ks ? kf : ks;
+      if (k >= K) break;
+      const bool fast = kf == k, slow = ks == k;
+      const int32_t ef = jf - 1, es = (int32_t)nf + js - 1;   // entries of this tick
+      while (sf.window() <= k) { sf.next(); ++jf; }
+      while (ss.window() <= k) { ss.next(); ++js; }
+      int recv = -1, kind = 0;
+      int32_t ent = -1;
+      if (fast) {
+        const int rv = rv_at(ef, fb0, fbuf);
+        if (rv >= 0) { recv = rv; ent = ef; kind = TRE_RESCUE; }
+      }
+      if (!kind && slow) {
+        const int rv = rv_at(es, sb0, sbuf);
+        if (rv >= 0) { recv = rv; ent = es; kind = TRE_REBALANCE; }
+      }
+      if (!kind) continue;
+      if (MPL <= 2) {
+        const unsigned long long donors =
+            ent < (int32_t)nf ? dm_at(ent, fm0, fmb) : dm_at(ent, sm0, smb);
+        unsigned long long above = 0;
+#pragma unroll
+        for (int j = 0; j < MPL; ++j)
+          above |= (unsigned long long)__ballot_sync(0xffffffffu, lane + 32 * j < M && r[j] > rmin[j])
+                   << (32 * j);
+        int g_rv = 0;
+#pragma unroll
+        for (int j = 0; j < MPL; ++j)
+          if (lane + 32 * j == recv) g_rv = g[j];
+        const int need_rv = __shfl_sync(0xffffffffu, g_rv, recv & 31);
+        if (free_pool < need_rv && !(donors & above)) continue;
+      }
+      act(k, recv, kind, ent);
     }
   }
 #pragma unroll

@@ -900,3 +900,48 @@ def test_score_when_burn_ins_cannot_converge(tre, dtype):
     np.testing.assert_array_equal(_np(out["cls"]), cls)
     np.testing.assert_array_equal(_np(out["recv"]), recv)
     assert tre.read_diag(diag)["ema_resolved"] > 0
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f64"])
+def test_score_long_table_idle_stretches(tre, dtype):
+    """A table long enough for the burn-ins that skip wholly idle chunks (at
+    least 2^22 cells) and for chunks longer than 256 windows (150,000 windows x
+    64 models: chunks of 320): models idle for stretches of 3,000 to 20,000
+    windows, a sparse model, one that never runs, per-model alphas down to
+    0.003, the series split in two calls with the carry between them -- bit
+    for bit the sequential values."""
+    import torch
+    rng = np.random.default_rng(2024)
+    K, M, win = 150000, 64, 100
+    cnt = _score_inputs(rng, K, M, idle_frac=0.02)
+    for m in range(0, M, 5):
+        a = int(rng.integers(0, K - 20000))
+        cnt_len = int(rng.integers(3000, 20000))
+        for k in cnt:
+            cnt[k][a:a + cnt_len, m] = 0
+    sparse = rng.random(K) < 0.7
+    for k in cnt:
+        cnt[k][sparse, 7] = 0
+        cnt[k][:, 9] = 0
+    npdt = np.float32 if dtype == "f32" else np.float64
+    alpha = rng.choice(np.array([0.02, 0.05, 0.003, 0.2]), M)
+    prof = {"w_p": rng.uniform(0.1, 0.3, M), "w_q": rng.uniform(1.0, 3.0, M),
+            "alpha": alpha, "theta": rng.uniform(5, 50, M),
+            "tau_crit": np.full(M, 0.8), "tau_surplus": np.full(M, 1.2)}
+    S, Z, cls, recv = oracle.score(cnt["P"], cnt["D"], cnt["A"], cnt["W"], prof, win, npdt)
+    diag = tre.new_diag()
+    out = tre.tss_score(_cuda(cnt), prof, win, dtype=dtype, diag=diag)
+    np.testing.assert_array_equal(_np(out["S"]), S)
+    np.testing.assert_array_equal(_np(out["Z"]), Z)
+    np.testing.assert_array_equal(_np(out["cls"]), cls)
+    np.testing.assert_array_equal(_np(out["recv"]), recv)
+    assert tre.read_diag(diag)["err"] == 0
+    tdt = torch.float32 if dtype == "f32" else torch.float64
+    carry = {"S": torch.zeros(M, dtype=tdt, device="cuda"),
+             "init": torch.zeros(M, dtype=torch.uint8, device="cuda")}
+    parts = []
+    for a, b in ((0, 140000), (140000, K)):
+        sub = _cuda({k: np.ascontiguousarray(v[a:b]) for k, v in cnt.items()})
+        parts.append(tre.tss_score(sub, prof, win, dtype=dtype, carry=carry))
+    np.testing.assert_array_equal(np.concatenate([_np(p["S"]) for p in parts]), S)
+    np.testing.assert_array_equal(np.concatenate([_np(p["cls"]) for p in parts]), cls)

@@ -167,3 +167,15 @@ def test_jump_walk_long_series_sixteen_models(tre):
     Z, cls, g, r0, budget, r_min = _case(16, 43200, 16, idle=0.05)
     for cap in (1, 2):
         _check(tre, Z, cls, g, r0, budget, r_min, 500, cap)
+
+
+@pytest.mark.parametrize("M", [24, 40])
+@pytest.mark.parametrize("fast_ms,slow_ms,win", [(3000, 10000, 1000), (500, 10000, 1000),
+                                                 (700, 2100, 100)])
+def test_warp_walk_cadences(tre, M, fast_ms, slow_ms, win):
+    """The warp walk for more than 16 models on cadences that are not nested
+    or a fast tick shorter than a window (every tick visited in order), and on
+    nested ones (32 ticks tested against the state at once)."""
+    Z, cls, g, r0, budget, r_min = _case(900 + M + fast_ms, 3000, M)
+    for cap in (1, 3):
+        _check(tre, Z, cls, g, r0, budget, r_min, win, cap, fast_ms, slow_ms)
