@@ -439,10 +439,21 @@ __device__ __forceinline__ bool ms_tick(float t, int64_t span, int64_t& tick) {
   return true;
 }
 
+// First and last valid tick of each request: the events of a CTA's slice (a
+// few seconds of a time-ordered stream) come from a few hundred requests,
+// each with many events, so the CTA keeps a shared-memory table of them (open
+// addressing on the request id, with the request's model cached beside it)
+// and flushes one min and one max per request; requests that find no slot
+// within kProbe probes go to global atomics directly.
+constexpr int kReqSlots = 1024;
+constexpr int kProbe = 32;
+constexpr int32_t kNoReq = -1;
+constexpr int32_t kModelUnread = -2;
+
 __global__ void __launch_bounds__(kThreads)
 k_reduce_events(EvCols e, int M, int win, FastDiv fd, int K, int64_t per_cta, int rows,
-                int32_t* __restrict__ P, int32_t* __restrict__ D, int32_t* __restrict__ first,
-                int32_t* __restrict__ last, tre_diag* diag) {
+                bool vec, int32_t* __restrict__ P, int32_t* __restrict__ D,
+                int32_t* __restrict__ first, int32_t* __restrict__ last, tre_diag* diag) {
   extern __shared__ unsigned long long smem[];
   const int64_t i0 = (int64_t)blockIdx.x * per_cta;
   const int64_t i1 = min(e.n, i0 + per_cta);
@@ -456,45 +467,82 @@ k_reduce_events(EvCols e, int M, int win, FastDiv fd, int K, int64_t per_cta, in
   const int cells = used * M;
   int32_t* sP = reinterpret_cast<int32_t*>(smem);
   int32_t* sD = sP + (size_t)rows * M;
+  int32_t* s_key = sD + (size_t)rows * M;
+  int32_t* s_first = s_key + kReqSlots;
+  int32_t* s_last = s_first + kReqSlots;
+  int32_t* s_model = s_last + kReqSlots;
   for (int c = threadIdx.x; c < cells; c += kThreads) { sP[c] = 0; sD[c] = 0; }
+  for (int c = threadIdx.x; c < kReqSlots; c += kThreads) {
+    s_key[c] = kNoReq;
+    s_first[c] = 0x7fffffff;
+    s_last[c] = -1;
+    s_model[c] = kModelUnread;
+  }
   __syncthreads();
 
-  const unsigned full = 0xffffffffu;
-  const int lane = threadIdx.x & 31;
   unsigned long long n_range = 0, n_model = 0, n_order = 0;
-  for (int64_t base = i0; base < i1; base += kThreads) {
-    const int64_t i = base + threadIdx.x;
-    bool ok = false;
-    int64_t tick = 0;
-    int rq = 0;
-    if (i < i1) {
-      const int m = e.model[i];
-      rq = e.req[i];
-      const float ts = e.t_s[i];
-      const uint8_t ph = e.phase[i];
-      if (m < 0 || m >= M || rq < 0 || rq >= e.n_req || e.req_model[rq] != m) {
-        ++n_model;
-      } else if (!ms_tick(ts, span, tick)) {
-        ++n_range;
-      } else if (ph > 1) {
-        ++n_order;
-      } else {
-        ok = true;
-        const int64_t k = fd.div((uint32_t)tick);
-        stage_add<int32_t>(ph == 0 ? sP : sD, ph == 0 ? P : D, k, k_lo, used, M, m, 1);
+  auto one = [&](int m, int rq, float ts, uint8_t ph) {
+    if (m < 0 || m >= M || rq < 0 || rq >= e.n_req) {
+      ++n_model;
+      return;
+    }
+    // the request's slot (or -1: none free within kProbe probes)
+    int slot = -1;
+    {
+      uint32_t h = ((uint32_t)rq * 0x9E3779B1u) >> (32 - 10);
+      for (int p = 0; p < kProbe; ++p, h = (h + 1) & (kReqSlots - 1)) {
+        const int32_t k = s_key[h];
+        if (k == rq) { slot = (int)h; break; }
+        if (k == kNoReq) {
+          const int32_t prev = atomicCAS(&s_key[h], kNoReq, rq);
+          if (prev == kNoReq || prev == rq) { slot = (int)h; break; }
+        }
       }
     }
-    // first / last tick per request, one atomic per run of equal request ids
-    const unsigned active = __ballot_sync(full, ok);
-    if (ok) {
-      const unsigned grp = __match_any_sync(active, rq);
-      const int t32 = (int)tick;
-      const int mn = __reduce_min_sync(grp, t32);
-      const int mx = __reduce_max_sync(grp, t32);
-      if (lane == __ffs(grp) - 1) {
-        atomicMin(&first[rq], mn);
-        atomicMax(&last[rq], mx);
+    int rm = slot >= 0 ? s_model[slot] : kModelUnread;
+    if (rm == kModelUnread) {
+      rm = e.req_model[rq];
+      if (slot >= 0) s_model[slot] = rm;
+    }
+    int64_t tick = 0;
+    if (rm != m) {
+      ++n_model;
+    } else if (!ms_tick(ts, span, tick)) {
+      ++n_range;
+    } else if (ph > 1) {
+      ++n_order;
+    } else {
+      const int64_t k = fd.div((uint32_t)tick);
+      stage_add<int32_t>(ph == 0 ? sP : sD, ph == 0 ? P : D, k, k_lo, used, M, m, 1);
+      if (slot >= 0) {
+        atomicMin(&s_first[slot], (int)tick);
+        atomicMax(&s_last[slot], (int)tick);
+      } else {
+        atomicMin(&first[rq], (int)tick);
+        atomicMax(&last[rq], (int)tick);
       }
+    }
+  };
+  // four consecutive events per thread and pass, with 16-byte loads of the
+  // columns when they are aligned, so that enough bytes are in flight
+  for (int64_t b = i0 + 4 * threadIdx.x; b < i1; b += 4 * kThreads) {
+    int mm[4], rr[4];
+    float tt[4];
+    uint8_t pp[4];
+    if (vec && b + 4 <= i1) {
+      const int4 a4 = *reinterpret_cast<const int4*>(e.model + b);
+      const int4 q4 = *reinterpret_cast<const int4*>(e.req + b);
+      const float4 t4 = *reinterpret_cast<const float4*>(e.t_s + b);
+      const uchar4 p4 = *reinterpret_cast<const uchar4*>(e.phase + b);
+      mm[0] = a4.x; mm[1] = a4.y; mm[2] = a4.z; mm[3] = a4.w;
+      rr[0] = q4.x; rr[1] = q4.y; rr[2] = q4.z; rr[3] = q4.w;
+      tt[0] = t4.x; tt[1] = t4.y; tt[2] = t4.z; tt[3] = t4.w;
+      pp[0] = p4.x; pp[1] = p4.y; pp[2] = p4.z; pp[3] = p4.w;
+#pragma unroll
+      for (int u = 0; u < 4; ++u) one(mm[u], rr[u], tt[u], pp[u]);
+    } else {
+      for (int u = 0; u < 4 && b + u < i1; ++u)
+        one(e.model[b + u], e.req[b + u], e.t_s[b + u], e.phase[b + u]);
     }
   }
   __syncthreads();
@@ -504,6 +552,12 @@ k_reduce_events(EvCols e, int M, int win, FastDiv fd, int K, int64_t per_cta, in
     const size_t g = (size_t)k * M + (c % M);
     if (sP[c]) atomicAdd(&P[g], sP[c]);
     if (sD[c]) atomicAdd(&D[g], sD[c]);
+  }
+  for (int c = threadIdx.x; c < kReqSlots; c += kThreads) {
+    const int rq = s_key[c];
+    if (rq == kNoReq || s_last[c] < 0) continue;
+    atomicMin(&first[rq], s_first[c]);
+    atomicMax(&last[rq], s_last[c]);
   }
   warp_add_counter(&diag->dropped_range, n_range);
   warp_add_counter(&diag->dropped_model, n_model);
@@ -1042,8 +1096,11 @@ cudaError_t launch_reduce_events(const EvCols& ev, int M, int win, int K, int32_
     const int rows = std::max(1, kStageBytes / (8 * M));
     const int64_t per = per_cta_records(ev.n, 2048, 16384);
     const unsigned grid = (unsigned)((ev.n + per - 1) / per);
-    k_reduce_events<<<grid, kThreads, (size_t)rows * M * 8, s>>>(ev, M, win, FastDiv(win), K, per,
-                                                                 rows, P, D, w.first, w.last, diag);
+    // per is a multiple of four, so every CTA's first event keeps the alignment
+    const bool vec = ((((uintptr_t)ev.model | (uintptr_t)ev.req | (uintptr_t)ev.t_s) & 15) |
+                      ((uintptr_t)ev.phase & 3)) == 0;
+    k_reduce_events<<<grid, kThreads, (size_t)rows * M * 8 + (size_t)kReqSlots * 16, s>>>(
+        ev, M, win, FastDiv(win), K, per, rows, vec, P, D, w.first, w.last, diag);
     if ((e = cudaGetLastError())) return e;
   }
   if (ev.n_req > 0) {
