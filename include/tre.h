@@ -232,11 +232,32 @@ tre_status tss_class_models(int64_t n, const int32_t* model, const int32_t* cls,
  * counted in diag.degenerate_calib). S uses w_p, w_q, alpha of `prof` (theta
  * and thresholds are ignored). Exactly one of req / ev non-NULL; `in` holds the
  * counts of the same telemetry. theta_out: dtype[n_models] on the device.
+ * S_out (dtype) and cls_out (uint8), [n_windows][n_models] on the device, may
+ * be NULL; when given they receive the smoothed series the boundary was taken
+ * from (the S tss_score returns for the same counts and profile) and the idle
+ * classes (TRE_IDLE for idle windows, TRE_NOM otherwise), which tss_normalize
+ * turns into Z and regions without smoothing the series again.
  */
 tre_status tss_calibrate(const tre_grid* grid, const tre_requests* req, const tre_events* ev,
                          const tre_counts* in, const tre_profile* prof, const int32_t* slo_ttft_ms,
-                         double ok_frac, double reliability, void* theta_out, void* ws,
-                         size_t* ws_bytes, tre_diag* diag, tre_stream stream);
+                         double ok_frac, double reliability, void* theta_out, void* S_out,
+                         uint8_t* cls_out, void* ws, size_t* ws_bytes, tre_diag* diag,
+                         tre_stream stream);
+
+/*
+ * tss_normalize -- Z = S / theta (Eq. 2), the regions (Sec. IV-A: critical
+ * below tau_crit, surplus above tau_surplus, idle windows stay idle) and the
+ * Eq. 3 receiver, for a series smoothed already (tss_calibrate's S_out and
+ * cls_out): with them it returns exactly tss_score's Z, cls and recv. S
+ * (dtype) and idle_cls (uint8, TRE_IDLE marks idle windows) are
+ * [n_windows][n_models] on the device; prof supplies theta, tau_crit and
+ * tau_surplus (w_p, w_q, alpha are not read). Z_out (dtype) and cls_out
+ * (uint8, may be idle_cls itself) are [n_windows][n_models]; recv_out
+ * (int32[n_windows]) may be NULL. Needs no workspace and touches no diag.
+ */
+tre_status tss_normalize(const tre_grid* grid, const tre_profile* prof, const void* S,
+                         const uint8_t* idle_cls, void* Z_out, uint8_t* cls_out,
+                         int32_t* recv_out, tre_stream stream);
 
 /*
  * Stage-aware signal (Sec. VIII: separate prefill and decode states; Sec. III-A

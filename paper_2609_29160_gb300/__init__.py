@@ -129,7 +129,8 @@ def load(build_if_missing: bool = True):
                               P, P, P, C.POINTER(C.c_size_t), P, P]
     lib.tss_calibrate.argtypes = [C.POINTER(Grid), C.POINTER(Requests), C.POINTER(Events),
                                   C.POINTER(Counts), C.POINTER(Profile), P, C.c_double,
-                                  C.c_double, P, P, C.POINTER(C.c_size_t), P, P]
+                                  C.c_double, P, P, P, P, C.POINTER(C.c_size_t), P, P]
+    lib.tss_normalize.argtypes = [C.POINTER(Grid), C.POINTER(Profile), P, P, P, P, P, P]
     lib.tre_select_moves.argtypes = [C.POINTER(Grid), P, P, C.POINTER(Profile), C.POINTER(Ctrl),
                                      P, P, C.c_int64, P, P, C.POINTER(C.c_size_t), P, P]
     lib.tre_sweep.argtypes = [C.POINTER(SweepSpec), C.POINTER(SweepOut), P,
@@ -145,7 +146,8 @@ def load(build_if_missing: bool = True):
     lib.tss_stage_score.argtypes = [C.POINTER(Grid), C.POINTER(Counts), P, P, C.POINTER(Profile),
                                     P, P, P, P, P, P, P, P, P, C.POINTER(C.c_size_t), P, P]
     for f in ("tss_window_reduce", "tss_score", "tss_calibrate", "tre_select_moves", "tre_sweep",
-              "tss_rank", "tss_stage_gauges", "tss_stage_calibrate", "tss_stage_score"):
+              "tss_rank", "tss_stage_gauges", "tss_stage_calibrate", "tss_stage_score",
+              "tss_normalize"):
         getattr(lib, f).restype = C.c_int
     lib.tre_replay.argtypes = [C.POINTER(Grid), C.POINTER(Latent), C.POINTER(Profile),
                                C.POINTER(Ctrl), P, C.POINTER(ReplaySpec), P,
@@ -437,8 +439,11 @@ def tss_stage_score(counts, A_prefill, A_decode, profile, window_ms, theta_prefi
 
 
 def tss_calibrate(counts, profile, window_ms, slo_ttft_ms, requests=None, events=None,
-                  dtype="f32", ok_frac=0.95, reliability=0.95, diag=None, stream=None):
-    """theta per model (CUDA tensor of dtype)."""
+                  dtype="f32", ok_frac=0.95, reliability=0.95, diag=None, stream=None,
+                  S_out=None, cls_out=None):
+    """theta per model (CUDA tensor of dtype). S_out / cls_out ([K][M] CUDA
+    tensors of dtype / uint8), when given, receive the smoothed series and the
+    idle classes the boundary was taken from."""
     torch = _torch()
     lib = load()
     K, M = counts["P"].shape
@@ -455,9 +460,28 @@ def tss_calibrate(counts, profile, window_ms, slo_ttft_ms, requests=None, events
     s = _stream(stream)
     _workspace("tss_calibrate", lambda ws, n: lib.tss_calibrate(
         C.byref(g), C.byref(rq) if rq else None, C.byref(ev) if ev else None, C.byref(cs),
-        C.byref(pst), _ptr(slo), C.c_double(ok_frac), C.c_double(reliability), _ptr(theta), ws,
-        n, _ptr(diag), s))
+        C.byref(pst), _ptr(slo), C.c_double(ok_frac), C.c_double(reliability), _ptr(theta),
+        _ptr(S_out), _ptr(cls_out), ws, n, _ptr(diag), s))
     return theta
+
+
+def tss_normalize(S, idle_cls, profile, window_ms, recv=True, Z_out=None, cls_out=None,
+                  stream=None):
+    """Eq. 2 and the regions (and the Eq. 3 receiver) of a smoothed series:
+    returns dict Z, cls (and recv), as tss_score does for the same S."""
+    torch = _torch()
+    lib = load()
+    K, M = S.shape
+    code, tdt = _dt(S.dtype)
+    _need(idle_cls, "uint8", K * M, "idle_cls")
+    g = Grid(M, window_ms, K)
+    pst, keep = _profile(profile, M, tdt, code)
+    Z = torch.empty((K, M), dtype=tdt, device="cuda") if Z_out is None else Z_out
+    cls = torch.empty((K, M), dtype=torch.uint8, device="cuda") if cls_out is None else cls_out
+    rv = torch.empty(K, dtype=torch.int32, device="cuda") if recv else None
+    _check("tss_normalize", lib.tss_normalize(C.byref(g), C.byref(pst), _ptr(S), _ptr(idle_cls),
+                                              _ptr(Z), _ptr(cls), _ptr(rv), _stream(stream)))
+    return {"Z": Z, "cls": cls, "recv": rv}
 
 
 def tre_select_moves(Z, cls, profile, window_ms, budget, r0, r_min, footprint, fast_ms=5000,
@@ -582,12 +606,12 @@ def sweep_moves(out, n_inst, moves_cap):
 
 class PipelinePlan:
     """One trace's whole path marshalled once: tss_window_reduce ->
-    tss_calibrate -> tss_score -> tre_select_moves, on request records or token
-    events (dicts of int32/float32/uint8 CUDA tensors). Device parameter
-    arrays, outputs, one workspace (sized for the largest of the four calls,
-    which run in order on one stream) and the C structs are built here; run()
-    resets the controller's replicas to r0 and issues the four C calls with no
-    further host work."""
+    tss_calibrate (which also returns the smoothed series) -> tss_normalize ->
+    tre_select_moves, on request records or token events (dicts of
+    int32/float32/uint8 CUDA tensors). Device parameter arrays, outputs, one
+    workspace (sized for the largest of the calls, which run in order on one
+    stream) and the C structs are built here; run() resets the controller's
+    replicas to r0 and issues the four C calls with no further host work."""
 
     def __init__(self, M, window_ms, K, profile, slo_ttft_ms, budget, r0, r_min, footprint,
                  requests=None, events=None, dtype="f32", fast_ms=5000, slow_ms=10000,
@@ -642,11 +666,12 @@ class PipelinePlan:
                 C.byref(g), rq, ev, self.cs, ws, n, dg, stream)),
             ("tss_calibrate", lambda ws, n: lib.tss_calibrate(
                 C.byref(g), rq, ev, C.byref(self.cs), C.byref(self.pst), _ptr(self.slo),
-                C.c_double(self.ok_frac), C.c_double(self.rel), _ptr(self.theta), ws, n, dg,
-                stream)),
-            ("tss_score", lambda ws, n: lib.tss_score(
-                C.byref(g), C.byref(self.cs), C.byref(self.pst), None, None, _ptr(self.S),
-                _ptr(self.Z), _ptr(self.cls), _ptr(self.recv), ws, n, dg, stream)),
+                C.c_double(self.ok_frac), C.c_double(self.rel), _ptr(self.theta), _ptr(self.S),
+                _ptr(self.cls), ws, n, dg, stream)),
+            # Z and regions from the series calibrate smoothed (no workspace)
+            ("tss_normalize", lambda ws, n: lib.tss_normalize(
+                C.byref(g), C.byref(self.pst), _ptr(self.S), _ptr(self.cls), _ptr(self.Z),
+                _ptr(self.cls), _ptr(self.recv), stream) if ws is not None else 0),
             ("tre_select_moves", lambda ws, n: lib.tre_select_moves(
                 C.byref(g), _ptr(self.Z), _ptr(self.cls), C.byref(self.pst), C.byref(self.ctrl),
                 _ptr(self.r), _ptr(self.moves), C.c_int64(self.moves_cap), _ptr(self.n_moves),

@@ -196,14 +196,18 @@ tre_status score_typed(const tre_grid* g, const tre_counts* in, const tre_profil
 template <class T>
 tre_status calibrate_typed(const tre_grid* g, const tre_requests* req, const tre_events* ev,
                            const tre_counts* in, const tre_profile* p, const int32_t* slo_ms,
-                           double ok_frac, double rel, void* theta, void* ws, size_t* ws_bytes,
-                           tre_diag* diag, cudaStream_t s) {
+                           double ok_frac, double rel, void* theta, void* S_out,
+                           uint8_t* cls_out, void* ws, size_t* ws_bytes, tre_diag* diag,
+                           cudaStream_t s) {
   const int M = g->n_models, K = g->n_windows;
   SeriesTable<T> tab = single_series<T>(g);
   Arena a(ws);
   unsigned long long* slo = a.take<unsigned long long>((size_t)K * M);
-  T* S = a.take<T>((size_t)K * M);
-  uint8_t* cls = a.take<uint8_t>((size_t)K * M);
+  T* S_ws = a.take<T>((size_t)K * M);
+  uint8_t* cls_ws = a.take<uint8_t>((size_t)K * M);
+  // the smoothed series and idle classes go to the caller's arrays when given
+  T* S = S_out ? static_cast<T*>(S_out) : S_ws;
+  uint8_t* cls = cls_out ? cls_out : cls_ws;
   ScoreWs<T> sw;
   score_ws_layout<T>(a, M, (int64_t)K * M, tab.seg_base[1], sw);
   CalibWs<T> cw;
@@ -768,8 +772,9 @@ tre_status tss_rank(const tre_grid* grid, tre_dtype dtype, const void* Z, const 
 
 tre_status tss_calibrate(const tre_grid* grid, const tre_requests* req, const tre_events* ev,
                          const tre_counts* in, const tre_profile* prof, const int32_t* slo_ttft_ms,
-                         double ok_frac, double reliability, void* theta_out, void* ws,
-                         size_t* ws_bytes, tre_diag* diag, tre_stream stream) {
+                         double ok_frac, double reliability, void* theta_out, void* S_out,
+                         uint8_t* cls_out, void* ws, size_t* ws_bytes, tre_diag* diag,
+                         tre_stream stream) {
   if (!grid_ok(grid) || !ws_bytes || (!req) == (!ev) || !counts_ok(in) || !prof_ok(prof, false))
     return TRE_EINVAL;
   if (req ? !req_ok(req) : !ev_ok(ev)) return TRE_EINVAL;
@@ -778,9 +783,51 @@ tre_status tss_calibrate(const tre_grid* grid, const tre_requests* req, const tr
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (prof->dtype == TRE_F32)
     return calibrate_typed<float>(grid, req, ev, in, prof, slo_ttft_ms, ok_frac, reliability,
-                                  theta_out, ws, ws_bytes, diag, s);
+                                  theta_out, S_out, cls_out, ws, ws_bytes, diag, s);
   return calibrate_typed<double>(grid, req, ev, in, prof, slo_ttft_ms, ok_frac, reliability,
-                                 theta_out, ws, ws_bytes, diag, s);
+                                 theta_out, S_out, cls_out, ws, ws_bytes, diag, s);
+}
+
+tre_status tss_normalize(const tre_grid* grid, const tre_profile* prof, const void* S,
+                         const uint8_t* idle_cls, void* Z_out, uint8_t* cls_out,
+                         int32_t* recv_out, tre_stream stream) {
+  if (!grid_ok(grid) || !prof_ok(prof, true)) return TRE_EINVAL;
+  if (grid->n_windows > 0 && (!S || !idle_cls || !Z_out || !cls_out)) return TRE_EINVAL;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const int M = grid->n_models, K = grid->n_windows;
+  if (K == 0) return TRE_OK;
+  cudaError_t e;
+  if (prof->dtype == TRE_F32) {
+    const SeriesTable<float> tab = single_series<float>(grid);
+    {
+      Scope sc(kNormalize, 1, s);
+      e = launch_normalize<float>(tab, static_cast<const float*>(S), idle_cls,
+                                  static_cast<const float*>(prof->theta),
+                                  static_cast<const float*>(prof->tau_crit), 0.f,
+                                  static_cast<const float*>(prof->tau_surplus),
+                                  static_cast<float*>(Z_out), cls_out, s);
+    }
+    if (!e && recv_out) {
+      Scope sc(kReceiver, 1, s);
+      e = launch_receiver<float>(M, K, static_cast<const float*>(Z_out), cls_out, recv_out, s);
+    }
+  } else {
+    const SeriesTable<double> tab = single_series<double>(grid);
+    {
+      Scope sc(kNormalize, 1, s);
+      e = launch_normalize<double>(tab, static_cast<const double*>(S), idle_cls,
+                                   static_cast<const double*>(prof->theta),
+                                   static_cast<const double*>(prof->tau_crit), 0.0,
+                                   static_cast<const double*>(prof->tau_surplus),
+                                   static_cast<double*>(Z_out), cls_out, s);
+    }
+    if (!e && recv_out) {
+      Scope sc(kReceiver, 1, s);
+      e = launch_receiver<double>(M, K, static_cast<const double*>(Z_out), cls_out, recv_out,
+                                  s);
+    }
+  }
+  return cuda_status(e);
 }
 
 tre_status tre_select_moves(const tre_grid* grid, const void* Z, const uint8_t* cls,

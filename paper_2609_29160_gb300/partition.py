@@ -127,12 +127,16 @@ def block_signal(tre, block, window_ms, K, profile, slo_ttft_ms, dtype="f32", st
     profile and SLO bounds are the block's models' ([m1 - m0])."""
     M = int(len(slo_ttft_ms))
     kw = {k: v for k, v in block.items()}
+    import torch
     c = tre.tss_window_reduce(M, window_ms, K, stream=stream, **kw)
+    S = torch.empty((K, M), dtype=torch.float32 if dtype == "f32" else torch.float64,
+                    device="cuda")
+    cls = torch.empty((K, M), dtype=torch.uint8, device="cuda")
     theta = tre.tss_calibrate(c, profile, window_ms, slo_ttft_ms, dtype=dtype, stream=stream,
-                              **kw)
-    sc = tre.tss_score(c, dict(profile, theta=theta), window_ms, dtype=dtype, recv=False,
-                       stream=stream)
-    return {"counts": c, "theta": theta, "Z": sc["Z"], "cls": sc["cls"], "S": sc["S"]}
+                              S_out=S, cls_out=cls, **kw)
+    sc = tre.tss_normalize(S, cls, dict(profile, theta=theta), window_ms, recv=False,
+                           cls_out=cls, stream=stream)
+    return {"counts": c, "theta": theta, "Z": sc["Z"], "cls": sc["cls"], "S": S}
 
 
 def walk_on_ticks(tre, Z_ticks, cls_ticks, profile, window_ms, fast_ms, slow_ms, budget, r0,

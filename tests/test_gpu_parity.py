@@ -945,3 +945,33 @@ def test_score_long_table_idle_stretches(tre, dtype):
         parts.append(tre.tss_score(sub, prof, win, dtype=dtype, carry=carry))
     np.testing.assert_array_equal(np.concatenate([_np(p["S"]) for p in parts]), S)
     np.testing.assert_array_equal(np.concatenate([_np(p["cls"]) for p in parts]), cls)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "f64"])
+@pytest.mark.parametrize("name,scale", [("tiny", 1.0), ("hetero", 0.005)])
+def test_calibrate_series_then_normalize(tre, dtype, name, scale):
+    """tss_calibrate's smoothed series and idle classes, turned into Z, regions
+    and receivers by tss_normalize (in place on the classes), equal the
+    oracle's S, Z, cls and recv -- the path the pipeline takes instead of
+    smoothing the series a second time."""
+    import torch
+    w = tracegen.workload(name, scale=scale)
+    M, win, K = w["M"], w["window_ms"], w["K"]
+    npdt = np.float32 if dtype == "f32" else np.float64
+    prof = tracegen.default_profile(M, win)
+    o = oracle.pipeline_requests(w["requests"], M, win, K, prof, w["slo_ttft_ms"], npdt)
+    req = _cuda(w["requests"])
+    c = tre.tss_window_reduce(M, win, K, requests=req)
+    S = torch.empty((K, M), dtype=torch.float32 if dtype == "f32" else torch.float64,
+                    device="cuda")
+    cls = torch.empty((K, M), dtype=torch.uint8, device="cuda")
+    theta = tre.tss_calibrate(c, prof, win, w["slo_ttft_ms"], requests=req, dtype=dtype,
+                              S_out=S, cls_out=cls)
+    np.testing.assert_array_equal(_np(theta), o["theta"])
+    np.testing.assert_array_equal(_np(S), o["S"])
+    assert set(np.unique(_np(cls))) <= {oracle.IDLE, oracle.NOM}
+    np.testing.assert_array_equal(_np(cls) == oracle.IDLE, o["cls"] == oracle.IDLE)
+    out = tre.tss_normalize(S, cls, dict(prof, theta=theta), win, cls_out=cls)
+    np.testing.assert_array_equal(_np(out["Z"]), o["Z"])
+    np.testing.assert_array_equal(_np(out["cls"]), o["cls"])
+    np.testing.assert_array_equal(_np(out["recv"]), o["recv"])

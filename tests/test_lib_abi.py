@@ -190,3 +190,20 @@ def test_stage_arguments_are_checked_on_the_host():
                                    None) == 1           # TPOT bounds missing
     assert lib.tss_stage_calibrate(C.byref(g), C.byref(rq), C.byref(cs), p, p, C.byref(prof), p,
                                    p, 0.95, 0.95, p, p, None, C.byref(n), None, None) == 0
+
+
+def test_normalize_argument_checks():
+    """tss_normalize refuses a profile without theta or thresholds and missing
+    arrays, and an empty grid is a no-op; none of these touches the device."""
+    lib = tre.load()
+    g = tre.Grid(4, 100, 1000)
+    full = tre.Profile(0, 8, 8, 8, 8, 8, 8)
+    no_theta = tre.Profile(0, 8, 8, 8, None, 8, 8)
+    assert lib.tss_normalize(C.byref(g), C.byref(no_theta), 8, 8, 8, 8, None, None) == 1
+    assert lib.tss_normalize(C.byref(g), C.byref(full), None, 8, 8, 8, None, None) == 1
+    assert lib.tss_normalize(C.byref(g), C.byref(full), 8, 8, 8, None, None, None) == 1
+    bad_dtype = tre.Profile(7, 8, 8, 8, 8, 8, 8)
+    assert lib.tss_normalize(C.byref(g), C.byref(bad_dtype), 8, 8, 8, 8, None, None) == 1
+    empty = tre.Grid(4, 100, 0)
+    assert lib.tss_normalize(C.byref(empty), C.byref(full), None, None, None, None, None,
+                             None) == 0
