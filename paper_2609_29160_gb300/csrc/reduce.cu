@@ -395,19 +395,66 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win,
   warp_add_counter(&diag->dropped_order, n_order);
 }
 
-// SLO counts alone (for calibration from records whose counts exist already)
+// SLO counts alone (for calibration from records whose counts exist already).
+// Records sorted by arrival put a CTA's slice into a short run of arrival
+// windows: the CTA adds into a shared copy of those rows, two 16-bit counts
+// (arrivals, met) per 32-bit word (a slice holds at most kSloPer records), and
+// flushes them once; records outside the run (unsorted input) go to global
+// atomics.
+constexpr int kSloPer = 4096;
 __global__ void __launch_bounds__(kThreads)
-k_slo_requests(ReqCols r, int M, int win, int K, unsigned long long* __restrict__ slo,
-               const int32_t* __restrict__ slo_ms) {
-  const int64_t span = (int64_t)K * win;
-  for (int64_t i = (int64_t)blockIdx.x * kThreads + threadIdx.x; i < r.n;
-       i += (int64_t)gridDim.x * kThreads) {
-    const int m = r.model[i];
-    const int64_t ta = r.t_arr[i], ts = r.t_start[i], tf = r.t_first[i], te = r.t_end[i];
-    if (m < 0 || m >= M || ta < 0 || ta >= span) continue;
-    if (!(ta <= ts && ts <= tf && tf <= te) || r.L_in[i] < 0 || r.L_out[i] < 1) continue;
-    const unsigned long long met = (tf - ta <= (int64_t)slo_ms[m]) ? 1ull : 0ull;
-    atomicAdd(&slo[(size_t)(ta / win) * M + m], 1ull + (met << 32));
+k_slo_requests(ReqCols r, int M, int win, FastDiv fd, int K, int rows, bool vec,
+               unsigned long long* __restrict__ slo, const int32_t* __restrict__ slo_ms) {
+  extern __shared__ uint32_t s_slo[];   // [rows][M]
+  const int64_t i0 = (int64_t)blockIdx.x * kSloPer;
+  const int n_loc = (int)min64(r.n - i0, (int64_t)kSloPer);
+  if (n_loc <= 0) return;
+  const uint32_t span = (uint32_t)K * (uint32_t)win;
+  const int a_first = r.t_arr[i0];
+  const int k_lo = (a_first < 0 || (uint32_t)a_first >= span) ? 0 : (int)fd.div((uint32_t)a_first);
+  const int used = min(rows, K - k_lo);
+  for (int c = threadIdx.x; c < used * M; c += kThreads) s_slo[c] = 0;
+  __syncthreads();
+  // every column of four consecutive records is loaded before any test, so
+  // that the loads are in flight together
+  const int32_t* col[7] = {r.model + i0, r.t_arr + i0, r.t_start + i0, r.t_first + i0,
+                           r.t_end + i0, r.L_in + i0, r.L_out + i0};
+  for (int b = 4 * threadIdx.x; b < n_loc; b += 4 * kThreads) {
+    int v[7][4];
+    if (vec && b + 4 <= n_loc) {
+#pragma unroll
+      for (int c = 0; c < 7; ++c) {
+        const int4 q = __ldcs(reinterpret_cast<const int4*>(col[c] + b));
+        v[c][0] = q.x; v[c][1] = q.y; v[c][2] = q.z; v[c][3] = q.w;
+      }
+    } else {
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const bool in = b + u < n_loc;
+#pragma unroll
+        for (int c = 0; c < 7; ++c) v[c][u] = in ? col[c][b + u] : 0;
+        if (!in) v[0][u] = -1;
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int m = v[0][u], ta = v[1][u], ts = v[2][u], tf = v[3][u], te = v[4][u];
+      const bool ok = m >= 0 && m < M && ta >= 0 && (uint32_t)ta < span && ta <= ts && ts <= tf &&
+                      tf <= te && v[5][u] >= 0 && v[6][u] >= 1;
+      if (!ok) continue;
+      const uint32_t met = (int64_t)tf - ta <= (int64_t)slo_ms[m] ? 1u : 0u;
+      const int k = (int)fd.div((uint32_t)ta);
+      const uint32_t rel = (uint32_t)(k - k_lo);
+      if (rel < (uint32_t)used) atomicAdd(&s_slo[rel * M + m], 1u + (met << 16));
+      else atomicAdd(&slo[(size_t)k * M + m], 1ull + ((unsigned long long)met << 32));
+    }
+  }
+  __syncthreads();
+  for (int c = threadIdx.x; c < used * M; c += kThreads) {
+    const uint32_t v = s_slo[c];
+    if (v)
+      atomicAdd(&slo[(size_t)k_lo * M + c],
+                (unsigned long long)(v & 0xffffu) + ((unsigned long long)(v >> 16) << 32));
   }
 }
 
@@ -1076,7 +1123,17 @@ cudaError_t launch_slo_requests(const ReqCols& r, int M, int win, int K,
                                 unsigned long long* slo, const int32_t* slo_ms, cudaStream_t s) {
   cudaError_t e = cudaMemsetAsync(slo, 0, (size_t)K * M * sizeof(unsigned long long), s);
   if (e || r.n == 0) return e;
-  k_slo_requests<<<grid_for(r.n, 4), kThreads, 0, s>>>(r, M, win, K, slo, slo_ms);
+  // arrival rows staged per CTA: the mean arrival span of a slice, three times
+  // over, plus a margin, within 32 KB
+  const int64_t mean_rows = (int64_t)kSloPer * K / std::max<int64_t>(r.n, 1);
+  const int rows = (int)std::max<int64_t>(1, std::min<int64_t>(3 * mean_rows + 34,
+                                                               32 * 1024 / (4 * M)));
+  const unsigned grid = (unsigned)((r.n + kSloPer - 1) / kSloPer);
+  const bool vec = (((uintptr_t)r.model | (uintptr_t)r.t_arr | (uintptr_t)r.t_start |
+                     (uintptr_t)r.t_first | (uintptr_t)r.t_end | (uintptr_t)r.L_in |
+                     (uintptr_t)r.L_out) & 15) == 0;
+  k_slo_requests<<<grid, kThreads, (size_t)rows * M * 4, s>>>(r, M, win, FastDiv(win), K, rows,
+                                                              vec, slo, slo_ms);
   return cudaGetLastError();
 }
 

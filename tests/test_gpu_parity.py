@@ -588,6 +588,18 @@ def test_calibrate_adversarial_ties(tre, dtype):
                                ok_frac=0.95, reliability=rho, diag=diag)
         np.testing.assert_array_equal(_np(th), theta)
         assert tre.read_diag(diag)["degenerate_calib"] == deg
+    # the same records shuffled (arrival windows no longer in runs), and with
+    # records out of range at the head of every slice of 4096: the same theta
+    perm = rng.permutation(len(req["model"]))
+    shuf = {k: v[perm] for k, v in req.items()}
+    heads = np.arange(0, len(perm), 4096)
+    shuf["t_arr_ms"][heads] = K * win + 5
+    n_arr, n_met = oracle.slo_counts_requests(shuf, M, win, K, slo)
+    theta, deg = oracle.calibrate(S, cls, n_arr, n_met, 0.95, 0.95)
+    for order in (shuf, {k: v[np.argsort(shuf["t_arr_ms"], kind="stable")] for k, v in shuf.items()}):
+        th = tre.tss_calibrate(_cuda(cnt), prof, win, slo, requests=_cuda(order), dtype=dtype,
+                               ok_frac=0.95, reliability=0.95)
+        np.testing.assert_array_equal(_np(th), theta)
 
 
 def test_select_heterogeneous_footprints_and_overflow(tre):
