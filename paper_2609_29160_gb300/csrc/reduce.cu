@@ -42,6 +42,7 @@ __device__ __forceinline__ void stage_add(V* s, V* g, int64_t k, int64_t k_lo, i
 constexpr int kMaxTraces = 64;
 constexpr int kVec = 4;               // records per thread per pass
 constexpr int kMaxPerCta = 16384;     // bound that keeps the packed shared counters exact
+constexpr int kFarScan = 1024;        // records that place a CTA's start-side rows
 struct ReqBatch {
   int n;
   ReqCols cols[kMaxTraces];
@@ -158,8 +159,12 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win,
     if (SLO) st.slo_lim[m] = slo_ms[m];
   }
   __syncthreads();
-  // each model's earliest start window among this CTA's records
-  for (int b = threadIdx.x * kVec; b < n_loc; b += kThreads * kVec) {
+  // each model's earliest start window among the CTA's first kFarScan
+  // records: records come in arrival order and each model starts its requests
+  // in arrival order (first come, first served), so its earliest starts are
+  // among its first records; a record that starts before this window takes
+  // the global path (the tests below check both ends)
+  for (int b = threadIdx.x * kVec; b < min(n_loc, kFarScan); b += kThreads * kVec) {
     int mm[kVec], ss[kVec];
     if (vec4 && b + kVec <= n_loc) {
       const int4 a = *reinterpret_cast<const int4*>(colp[0] + b);
@@ -276,8 +281,8 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win,
         const int wait = ba != bs ? 1 : 0, run = bs != be ? 1 : 0;
         const uint32_t met = SLO && (tf - ta <= st.slo_lim[m]) ? 1u : 0u;
         const uint32_t rel_a = (uint32_t)(ba - k_lo);
-        // lo <= bs <= kf <= be: one test covers every start-side target
-        if (rel_a < (uint32_t)used && (uint32_t)(be - lo) < (uint32_t)F) {
+        // bs <= kf <= be: the two ends bound every start-side target
+        if (rel_a < (uint32_t)used && (uint32_t)(be - lo) < (uint32_t)F && bs >= lo) {
           const int na = (int)(rel_a << lgMp) + m;
           const int fb = m * F1 - lo;
           atomicAdd(&st.aW[na], wait);
@@ -335,7 +340,7 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win,
       const int lo = st.far_lo[m];
       const int k_full = min(be_raw - 1, K - 1);   // windows ending at or before t_end
       const int k_end = min(be_raw, K - 1);
-      if ((uint32_t)(k_end - lo) < (uint32_t)F) {
+      if ((uint32_t)(k_end - lo) < (uint32_t)F && kf + 1 >= lo) {
         int32_t* fd_row = st.fD + m * F1 - lo;
         for (int k = kf + 1; k <= k_full; ++k) {
           const uint32_t t = rem + R;

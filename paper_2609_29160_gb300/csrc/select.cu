@@ -151,37 +151,33 @@ __device__ __forceinline__ void load_quad(const double* p, double* v) {
   v[0] = a.x; v[1] = a.y; v[2] = c.x; v[3] = c.y;
 }
 
-// One thread per (series, tau, tick entry) for M <= MMAX: the regions are
-// computed once per model and the ranks in registers; the per-model rank and
-// order tables are written only when the walk that follows reads them. With
-// QUAD (M a multiple of 4, 16-byte aligned rows) a tick window's Z and class
+// The action of one control tick of (series s, tau ti) at window k, for
+// M <= MMAX: regions from the window's Z and class rows; the receiver (rescue:
+// lowest Z among critical models; rebalance: lowest Z among non-idle models,
+// acting only below Z = 1; lowest index on ties; -1 when the tick does
+// nothing); each model's rank in the donor order (kNoRank when not a donor),
+// the donor order packed four bits a position (M <= 16), the donor mask and
+// the donor count. With QUAD (M a multiple of 4, 16-byte aligned rows) the
 // rows are read four models per load.
 template <class T, int MMAX, bool QUAD>
-__global__ void __launch_bounds__(128)
-k_tick_rank_small(const __grid_constant__ WalkBatch<T> b, int16_t* recv_out, int16_t* ndon_out,
-                  uint16_t* rank, uint16_t* order, unsigned long long* packed, uint32_t* dmask,
-                  bool need_rank, unsigned long long* dm64) {
+struct TickAction {
+  int recv, nd;
+  unsigned long long pk, dmw;
+  uint32_t dm;
+  uint16_t rk[MMAX];
+};
+
+template <class T, int MMAX, bool QUAD>
+__device__ __forceinline__ void tick_row(const WalkBatch<T>& b, int s, uint32_t k, T (&z)[MMAX],
+                                         uint8_t (&cl)[MMAX]) {
   const int M = b.M;
-  const int64_t e = (int64_t)blockIdx.x * 128 + threadIdx.x;
-  if (e >= (int64_t)b.ent_base[b.n_series] * b.n_tau) return;
-  const int s = prefix_index(b.ent_base, b.n_series, e, b.n_tau);
-  const int local = (int)(e - (int64_t)b.ent_base[s] * b.n_tau);
-  const int n_ent = b.ent_base[s + 1] - b.ent_base[s];
-  const int ti = local / n_ent;
-  const int j = local - ti * n_ent;
-  // K * win < 2^31, so every tick time below fits 32 unsigned bits
-  const uint32_t win = (uint32_t)b.series_win[s];
-  const uint32_t nf = (uint32_t)b.series_K[s] * win / (uint32_t)b.fast_ms;
-  const bool fast = (uint32_t)j < nf;
-  const uint32_t tj = fast ? ((uint32_t)j + 1) * (uint32_t)b.fast_ms
-                           : ((uint32_t)j - nf + 1) * (uint32_t)b.slow_ms;
-  const uint32_t k = (tj + win - 1) / win - 1;   // window whose right edge passes tj
   const T* Zk = b.Z + b.series_off[s] + (size_t)k * M;
   const uint8_t* Ck = b.cls + b.series_off[s] + (size_t)k * M;
-  const bool tau_dev = b.tau_crit != nullptr;
-  const T tau_v = b.tau_list[tau_dev ? 0 : ti];
-  T z[MMAX];
-  uint8_t cl[MMAX];
+#pragma unroll
+  for (int q = 0; q < MMAX; ++q) {
+    z[q] = (T)0;
+    cl[q] = kIdle;
+  }
   if (QUAD) {
 #pragma unroll
     for (int q = 0; q < MMAX; q += 4) {
@@ -191,19 +187,30 @@ k_tick_rank_small(const __grid_constant__ WalkBatch<T> b, int16_t* recv_out, int
         cl[q] = c4.x; cl[q + 1] = c4.y; cl[q + 2] = c4.z; cl[q + 3] = c4.w;
       }
     }
+  } else {
+#pragma unroll
+    for (int q = 0; q < MMAX; ++q)
+      if (q < M) {
+        z[q] = Zk[q];
+        cl[q] = Ck[q];
+      }
   }
+}
+
+template <class T, int MMAX, bool QUAD>
+__device__ __forceinline__ void tick_action(const WalkBatch<T>& b, int ti, bool fast,
+                                            const T (&z)[MMAX], const uint8_t (&cl)[MMAX],
+                                            TickAction<T, MMAX, QUAD>& out) {
+  const int M = b.M;
+  const bool tau_dev = b.tau_crit != nullptr;
+  const T tau_v = b.tau_list[tau_dev ? 0 : ti];
   uint8_t rg[MMAX];
   int recv = -1;
   T zr = (T)0;
 #pragma unroll
   for (int q = 0; q < MMAX; ++q) {
-    if (!QUAD || q >= M) z[q] = (T)0;
     rg[q] = 0xff;
     if (q < M) {
-      if (!QUAD) {
-        z[q] = Zk[q];
-        cl[q] = Ck[q];
-      }
       rg[q] = region_of(cl[q], z[q], tau_dev ? b.tau_crit[q] : tau_v, b.tau_surp[q]);
       const bool cand = fast ? rg[q] == kCrit : rg[q] != kIdle;
       if (cand && (recv < 0 || z[q] < zr)) {
@@ -226,14 +233,12 @@ k_tick_rank_small(const __grid_constant__ WalkBatch<T> b, int16_t* recv_out, int
     grp[q] = g;
     nd += g >= 0;
   }
-  const size_t row = (size_t)b.ent_base[s] * b.n_tau + (size_t)ti * n_ent + j;
   unsigned long long pk = 0, dmw = 0;
   uint32_t dm = 0;
 #pragma unroll
   for (int m = 0; m < MMAX; ++m) {
-    if (m >= M) break;
     uint16_t r = kNoRank;
-    if (grp[m] >= 0) {
+    if (m < M && grp[m] >= 0) {
       int before = 0;
 #pragma unroll
       for (int q = 0; q < MMAX; ++q) {
@@ -245,22 +250,65 @@ k_tick_rank_small(const __grid_constant__ WalkBatch<T> b, int16_t* recv_out, int
         before += prec;
       }
       r = (uint16_t)before;
-      if (need_rank) order[row * M + r] = (uint16_t)m;
       dmw |= 1ull << m;
       if (MMAX <= 16) {
         pk |= (unsigned long long)m << (4 * before);
         dm |= 1u << m;
       }
     }
-    if (need_rank) rank[row * M + m] = r;
+    out.rk[m] = r;
   }
-  recv_out[row] = (int16_t)(act ? recv : -1);
-  ndon_out[row] = (int16_t)nd;
+  out.recv = act ? recv : -1;
+  out.nd = nd;
+  out.pk = pk;
+  out.dm = dm;
+  out.dmw = dmw;
+}
+
+// One thread per (series, tau, tick entry) for M <= MMAX: the regions are
+// computed once per model and the ranks in registers; the per-model rank and
+// order tables are written only when the walk that follows reads them.
+template <class T, int MMAX, bool QUAD>
+__global__ void __launch_bounds__(128)
+k_tick_rank_small(const __grid_constant__ WalkBatch<T> b, int16_t* recv_out, int16_t* ndon_out,
+                  uint16_t* rank, uint16_t* order, unsigned long long* packed, uint32_t* dmask,
+                  bool need_rank, unsigned long long* dm64) {
+  const int M = b.M;
+  const int64_t e = (int64_t)blockIdx.x * 128 + threadIdx.x;
+  if (e >= (int64_t)b.ent_base[b.n_series] * b.n_tau) return;
+  const int s = prefix_index(b.ent_base, b.n_series, e, b.n_tau);
+  const int local = (int)(e - (int64_t)b.ent_base[s] * b.n_tau);
+  const int n_ent = b.ent_base[s + 1] - b.ent_base[s];
+  const int ti = local / n_ent;
+  const int j = local - ti * n_ent;
+  // K * win < 2^31, so every tick time below fits 32 unsigned bits
+  const uint32_t win = (uint32_t)b.series_win[s];
+  const uint32_t nf = (uint32_t)b.series_K[s] * win / (uint32_t)b.fast_ms;
+  const bool fast = (uint32_t)j < nf;
+  const uint32_t tj = fast ? ((uint32_t)j + 1) * (uint32_t)b.fast_ms
+                           : ((uint32_t)j - nf + 1) * (uint32_t)b.slow_ms;
+  const uint32_t k = (tj + win - 1) / win - 1;   // window whose right edge passes tj
+  T z[MMAX];
+  uint8_t cl[MMAX];
+  tick_row<T, MMAX, QUAD>(b, s, k, z, cl);
+  TickAction<T, MMAX, QUAD> a;
+  tick_action<T, MMAX, QUAD>(b, ti, fast, z, cl, a);
+  const size_t row = (size_t)b.ent_base[s] * b.n_tau + (size_t)ti * n_ent + j;
+  if (need_rank) {
+#pragma unroll
+    for (int m = 0; m < MMAX; ++m) {
+      if (m >= M) break;
+      rank[row * M + m] = a.rk[m];
+      if (a.rk[m] != kNoRank) order[row * M + a.rk[m]] = (uint16_t)m;
+    }
+    dm64[row] = a.dmw;                             // for the warp walk
+  }
+  recv_out[row] = (int16_t)a.recv;
+  ndon_out[row] = (int16_t)a.nd;
   if (MMAX <= 16) {
-    packed[row] = pk;
-    dmask[row] = dm;
+    packed[row] = a.pk;
+    dmask[row] = a.dm;
   }
-  if (need_rank) dm64[row] = dmw;                  // for the warp walk
 }
 
 template <int MPL>
@@ -824,7 +872,11 @@ struct __align__(16) TickRec {
   uint8_t kind, pad;
 };
 
-template <class T, int MMAX>
+// RANK: the CTA of a (series, tau) finds its ticks' actions itself from the Z
+// and class rows (tick_action) while it builds the tables -- one launch, for
+// batches with a CTA per SM or more; otherwise it reads them from the tick
+// tables k_tick_rank_small wrote (the ranking then spreads over many CTAs).
+template <class T, int MMAX, bool RANK, bool QUAD>
 __global__ void __launch_bounds__(256, 1)
 k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
             const unsigned long long* packed, const uint32_t* dmask, bool store_win) {
@@ -857,18 +909,39 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
   uint16_t* sany = snx + (size_t)(nf + 1) * MMAX;                          // [nf + 1]
   __shared__ int s_cap[8][MMAX];   // unit footprints: replicas above the floor, per warp
   for (int u = threadIdx.x; u < nf; u += blockDim.x) {
-    const int rf = recv_tab[row0 + u];
-    int e = -1, kd = 0, rv = -1;
-    if (rf >= 0) {
-      e = u; kd = TRE_RESCUE; rv = rf;
-    } else if ((u + 1) % ratio == 0) {
-      const int es = nf + (u + 1) / ratio - 1;
-      const int rs = recv_tab[row0 + es];
-      if (rs >= 0) { e = es; kd = TRE_REBALANCE; rv = rs; }
+    int kd = 0, rv = -1;
+    unsigned long long pk = 0;
+    uint32_t dm = 0;
+    if (!RANK) {
+      const int rf = recv_tab[row0 + u];
+      int e = -1;
+      if (rf >= 0) {
+        e = u; kd = TRE_RESCUE; rv = rf;
+      } else if ((u + 1) % ratio == 0) {
+        const int es = nf + (u + 1) / ratio - 1;
+        const int rs = recv_tab[row0 + es];
+        if (rs >= 0) { e = es; kd = TRE_REBALANCE; rv = rs; }
+      }
+      pk = e >= 0 ? packed[row0 + e] : 0ull;
+      dm = e >= 0 ? dmask[row0 + e] : 0u;
+    } else {
+      // a slow tick falls on the window of the fast tick it coincides with;
+      // a rescue at a tick takes precedence over its rebalance
+      T z[MMAX];
+      uint8_t cl[MMAX];
+      tick_row<T, MMAX, QUAD>(b, si, (uint32_t)tick_window(u + 1, b.fast_ms, win), z, cl);
+      TickAction<T, MMAX, QUAD> a;
+      tick_action<T, MMAX, QUAD>(b, ti, true, z, cl, a);
+      if (a.recv >= 0) {
+        kd = TRE_RESCUE; rv = a.recv; pk = a.pk; dm = a.dm;
+      } else if ((u + 1) % ratio == 0) {
+        tick_action<T, MMAX, QUAD>(b, ti, false, z, cl, a);
+        if (a.recv >= 0) { kd = TRE_REBALANCE; rv = a.recv; pk = a.pk; dm = a.dm; }
+      }
     }
     TickRec t;
-    t.pk = e >= 0 ? packed[row0 + e] : 0ull;
-    t.dm = e >= 0 ? dmask[row0 + e] : 0u;
+    t.pk = pk;
+    t.dm = dm;
     t.recv = (int16_t)rv;
     t.kind = (uint8_t)kd;
     t.pad = 0;
@@ -1250,45 +1323,60 @@ template <class T> void walk_ws_layout(Arena& a, WalkBatch<T>& b, WalkWs& w) {
 }
 
 // unit footprints and few models: thread-per-instance walk with staged tables
+// Whether the jump walk applies (nested cadences, a fast tick not shorter
+// than a window, tick tables within the opt-in shared-memory limit) and its
+// shared memory: the tables, with or without the staged tick windows.
+struct JumpPlan {
+  bool ok, store_win;
+  size_t smem, lim;
+};
+template <class T, int MMAX> JumpPlan jump_plan(const WalkBatch<T>& b) {
+  JumpPlan p{false, false, 0, 0};
+  if (b.slow_ms % b.fast_ms != 0 || b.fast_ms < b.series_win[0]) return p;
+  bool ok = true;
+  size_t jsmem = 0, wsmem = 0;
+  for (int i = 0; i < b.n_series; ++i) {
+    if (b.fast_ms < b.series_win[i]) ok = false;
+    const int64_t nf = (int64_t)b.series_K[i] * b.series_win[i] / b.fast_ms;
+    if (nf >= 32767) ok = false;
+    const size_t need = (size_t)nf * sizeof(TickRec) + (size_t)(nf + 1) * MMAX * 2 +
+                        (size_t)(nf + 1) * 2;
+    jsmem = std::max(jsmem, need);
+    wsmem = std::max(wsmem, (size_t)((nf + 3) & ~3) * 4);
+  }
+  // the largest dynamic shared memory a block may opt into, beside the
+  // kernel's static per-warp counts
+  int dev = 0, optin = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) !=
+          cudaSuccess || optin <= 4096) {
+    cudaGetLastError();
+    return p;
+  }
+  p.lim = (size_t)optin - 2048;
+  p.store_win = jsmem + wsmem <= p.lim;
+  p.smem = p.store_win ? jsmem + wsmem : jsmem;
+  p.ok = ok && p.smem <= p.lim;
+  return p;
+}
+
+// The jump walk; RANK: it ranks its own ticks (one launch for the selection).
+template <class T, int MMAX, bool RANK, bool QUAD>
+cudaError_t jump_launch(const WalkBatch<T>& b, const WalkWs& w, const JumpPlan& p,
+                        cudaStream_t s) {
+  cudaError_t e =
+      func_smem_once((const void*)k_walk_jump<T, MMAX, RANK, QUAD>, (int)p.lim, false);
+  if (e) return e;
+  // eight warps build the tables; the first n_cap of them walk
+  k_walk_jump<T, MMAX, RANK, QUAD><<<b.n_series * b.n_tau, 256, p.smem, s>>>(
+      b, w.recv, w.packed, w.dmask, p.store_win);
+  return cudaGetLastError();
+}
+
 template <class T, int MMAX>
 cudaError_t walk_thread_launch(const WalkBatch<T>& b, WalkWs& w, size_t smem, cudaStream_t s) {
   cudaError_t e = func_smem_once((const void*)k_walk_thread<T, MMAX>, (int)kStageMax, false);
   if (e) return e;
-  // nested cadences with a fast tick not shorter than a window: jump between
-  // possible moves
-  if (b.slow_ms % b.fast_ms == 0 && b.fast_ms >= b.series_win[0]) {
-    bool ok = true;
-    size_t jsmem = 0, wsmem = 0;   // tables, and the staged tick windows
-    for (int i = 0; i < b.n_series; ++i) {
-      if (b.fast_ms < b.series_win[i]) ok = false;
-      const int64_t nf = (int64_t)b.series_K[i] * b.series_win[i] / b.fast_ms;
-      if (nf >= 32767) ok = false;
-      const size_t need = (size_t)nf * sizeof(TickRec) + (size_t)(nf + 1) * MMAX * 2 +
-                          (size_t)(nf + 1) * 2;
-      jsmem = std::max(jsmem, need);
-      wsmem = std::max(wsmem, (size_t)((nf + 3) & ~3) * 4);
-    }
-    // the largest dynamic shared memory a block may opt into, beside the
-    // kernel's static per-warp counts
-    int dev = 0, optin = 0;
-    if (cudaGetDevice(&dev) == cudaSuccess &&
-        cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) ==
-            cudaSuccess && optin > 4096) {
-      const size_t lim = (size_t)optin - 2048;
-      const bool store_win = jsmem + wsmem <= lim;
-      const size_t smem_j = store_win ? jsmem + wsmem : jsmem;
-      if (ok && smem_j <= lim) {
-        e = func_smem_once((const void*)k_walk_jump<T, MMAX>, (int)lim, false);
-        if (e) return e;
-        // eight warps build the tick tables; the first n_cap of them walk
-        const int warps = 8;
-        k_walk_jump<T, MMAX><<<b.n_series * b.n_tau, 32 * warps, smem_j, s>>>(
-            b, w.recv, w.packed, w.dmask, store_win);
-        return cudaGetLastError();
-      }
-    }
-    cudaGetLastError();
-  }
   k_walk_thread<T, MMAX><<<b.n_series * b.n_tau, 32, smem, s>>>(b, w.recv, w.packed, w.dmask);
   return cudaGetLastError();
 }
@@ -1302,6 +1390,17 @@ template <class T> cudaError_t launch_walk(const WalkBatch<T>& b, WalkWs& w, cud
     max_ent = std::max(max_ent, b.ent_base[i + 1] - b.ent_base[i]);
   const size_t thread_smem = (size_t)max_ent * (8 + 4 + 2) + 16;
   const bool thread_walk = b.M <= 16 && b.n_cap <= 32 && thread_smem <= kStageMax;
+  const bool quad = b.M % 4 == 0 && (((uintptr_t)b.Z | (uintptr_t)b.cls) & 15) == 0;
+  JumpPlan jp{false, false, 0, 0};
+  if (thread_walk && ents > 0) jp = b.M <= 8 ? jump_plan<T, 8>(b) : jump_plan<T, 16>(b);
+  // with a CTA per SM or more, the jump walk ranks its own ticks: one launch
+  if (jp.ok && b.n_series * b.n_tau >= device_sm_count()) {
+    if (b.M <= 8)
+      return quad ? jump_launch<T, 8, true, true>(b, w, jp, s)
+                  : jump_launch<T, 8, true, false>(b, w, jp, s);
+    return quad ? jump_launch<T, 16, true, true>(b, w, jp, s)
+                : jump_launch<T, 16, true, false>(b, w, jp, s);
+  }
   if (ents > 0) {
     const unsigned g = (unsigned)((ents + 127) / 128);
     // rows start on 16-byte boundaries when M is a multiple of 4 (series
@@ -1326,6 +1425,9 @@ template <class T> cudaError_t launch_walk(const WalkBatch<T>& b, WalkWs& w, cud
                                                                    w.order, w.dm64);
     }
   }
+  if (jp.ok)
+    return b.M <= 8 ? jump_launch<T, 8, false, false>(b, w, jp, s)
+                    : jump_launch<T, 16, false, false>(b, w, jp, s);
   if (thread_walk)
     return b.M <= 8 ? walk_thread_launch<T, 8>(b, w, thread_smem, s)
                     : walk_thread_launch<T, 16>(b, w, thread_smem, s);

@@ -749,6 +749,17 @@ def test_sweep_small(tre):
     _compare_sweep(tre, sw, ref, out, 512)
 
 
+@pytest.mark.parametrize("dtype", ["f32", "f64"])
+def test_sweep_many_series_rank_in_walk(tre, dtype):
+    """Five traces x 4 window lengths x 8 rescue thresholds: at least one
+    (series, threshold) block per SM, so the jump walk ranks its own ticks
+    from the Z and class rows (one launch) instead of reading tick tables."""
+    sw, alpha = _sweep_case(0.02, 5, 600.0)
+    sw["pacing_cap"] = sw["pacing_cap"][::4]
+    ref, out = _run_sweep_both(tre, sw, alpha, moves_cap=512, dtype=dtype)
+    _compare_sweep(tre, sw, ref, out, 512)
+
+
 def test_reduce_requests_from_pinned_host_memory(tre):
     """Record columns left in pinned host memory that the GPU addresses
     directly give the same counts as device-resident columns."""
