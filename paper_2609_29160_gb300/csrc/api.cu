@@ -377,8 +377,10 @@ tre_status sweep_typed(const tre_sweep_spec* sp, const SweepPlan& pl, const tre_
   }
   const bool fused = lcm <= 4096 && sp->n_win <= kGaugeMaxWin;
   if (fused) {
-    gp.blk = (int)(lcm * std::max<int64_t>(1, (32 + lcm - 1) / lcm));
-    if (gp.blk < kGaugeMinBlk) gp.blk = (int)(lcm * ((kGaugeMinBlk + lcm - 1) / lcm));
+    // the shortest row block that holds whole coarse windows of every length
+    // and at least kGaugeMinBlk rows: more (trace, block, model) threads keep
+    // more loads in flight
+    gp.blk = (int)(lcm * ((kGaugeMinBlk + lcm - 1) / lcm));
     gp.nblk = (pl.Kb + gp.blk - 1) / gp.blk;
     for (int t = 0; t < NT; ++t) {
       for (int w = 0; w < sp->n_win; ++w) gp.out_off[t][w] = pl.off[t * sp->n_win + w];

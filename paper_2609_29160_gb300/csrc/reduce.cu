@@ -671,6 +671,7 @@ k_slo_events(EvCols e, int M, int win, int K, unsigned long long* __restrict__ s
 // Segment = (chunk of rows, model); adjacent threads take adjacent models so
 // each row is read coalesced.
 // --------------------------------------------------------------------------
+constexpr int kScanBatch = 16;
 __global__ void __launch_bounds__(kThreads)
 k_scan_partials(int M, int K, int L, int n_chunks, const int32_t* __restrict__ dA,
                 const int32_t* __restrict__ dW, int32_t* __restrict__ pA,
@@ -685,7 +686,22 @@ k_scan_partials(int M, int K, int L, int n_chunks, const int32_t* __restrict__ d
   const int c = (int)(t / M);
   const int64_t r0 = (int64_t)c * L, r1 = min64(r0 + L, K);
   int32_t a = 0, w = 0;
-  for (int64_t k = r0; k < r1; ++k) {
+  int64_t k = r0;
+  // kScanBatch rows' loads issued together, so that enough bytes are in flight
+  for (; k + kScanBatch <= r1; k += kScanBatch) {
+    int32_t xa[kScanBatch], xw[kScanBatch];
+#pragma unroll
+    for (int j = 0; j < kScanBatch; ++j) {
+      xa[j] = dA[(k + j) * M + m];
+      xw[j] = dW[(k + j) * M + m];
+    }
+#pragma unroll
+    for (int j = 0; j < kScanBatch; ++j) {
+      a += xa[j];
+      w += xw[j];
+    }
+  }
+  for (; k < r1; ++k) {
     a += dA[k * M + m];
     w += dW[k * M + m];
   }
@@ -749,7 +765,23 @@ k_scan_apply(int M, int K, int L, int n_chunks, const int32_t* __restrict__ dA,
   const int c = (int)(t / M);
   const int64_t r0 = (int64_t)c * L, r1 = min64(r0 + L, K);
   int32_t a = pA[t], w = pW[t];
-  for (int64_t k = r0; k < r1; ++k) {
+  int64_t k = r0;
+  for (; k + kScanBatch <= r1; k += kScanBatch) {
+    int32_t xa[kScanBatch], xw[kScanBatch];
+#pragma unroll
+    for (int j = 0; j < kScanBatch; ++j) {
+      xa[j] = dA[(k + j) * M + m];
+      xw[j] = dW[(k + j) * M + m];
+    }
+#pragma unroll
+    for (int j = 0; j < kScanBatch; ++j) {
+      a += xa[j];
+      w += xw[j];
+      A[(k + j) * M + m] = a;
+      W[(k + j) * M + m] = w;
+    }
+  }
+  for (; k < r1; ++k) {
     a += dA[k * M + m];
     w += dW[k * M + m];
     A[k * M + m] = a;
