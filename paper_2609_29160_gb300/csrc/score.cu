@@ -719,24 +719,57 @@ k_normalize(const __grid_constant__ SeriesTable<T> tab, const __grid_constant__ 
 
 // ---- Eq. 3 receiver per window: warp per window ----------------------------
 template <class T>
-__global__ void k_receiver(int M, int K, const T* Z, const uint8_t* cls, int32_t* recv) {
-  const int64_t k = (int64_t)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
+__device__ __forceinline__ void load_quad_z(const T* p, T (&v)[4]);
+template <> __device__ __forceinline__ void load_quad_z<float>(const float* p, float (&v)[4]) {
+  const float4 q = *reinterpret_cast<const float4*>(p);
+  v[0] = q.x; v[1] = q.y; v[2] = q.z; v[3] = q.w;
+}
+template <> __device__ __forceinline__ void load_quad_z<double>(const double* p, double (&v)[4]) {
+  const double2 a = reinterpret_cast<const double2*>(p)[0];
+  const double2 c = reinterpret_cast<const double2*>(p)[1];
+  v[0] = a.x; v[1] = a.y; v[2] = c.x; v[3] = c.y;
+}
+
+// Eq. 3 receiver per window: argmin Z over non-idle models, lowest index on
+// ties (the first minimum in index order), -1 when every model is idle. One
+// thread per window; with QUAD (M a multiple of 4, 16-byte aligned rows) a
+// row is read four models per load, several loads in flight.
+template <class T, bool QUAD>
+__global__ void __launch_bounds__(256)
+k_receiver(int M, int K, const T* __restrict__ Z, const uint8_t* __restrict__ cls,
+           int32_t* __restrict__ recv) {
+  const int64_t k = (int64_t)blockIdx.x * 256 + threadIdx.x;
   if (k >= K) return;
-  const int lane = threadIdx.x & 31;
+  const T* z = Z + (size_t)k * M;
+  const uint8_t* c = cls + (size_t)k * M;
   int best = -1;
   T bz = (T)0;
-  for (int m = lane; m < M; m += 32) {
-    const size_t x = (size_t)k * M + m;
-    if (cls[x] == kIdle) continue;
-    const T z = Z[x];
-    if (best < 0 || z < bz) { best = m; bz = z; }
+  if (QUAD) {
+#pragma unroll 4
+    for (int m0 = 0; m0 < M; m0 += 4) {
+      T zv[4];
+      load_quad_z<T>(z + m0, zv);
+      const uchar4 c4 = *reinterpret_cast<const uchar4*>(c + m0);
+      const uint8_t cv[4] = {c4.x, c4.y, c4.z, c4.w};
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        if (cv[i] != kIdle && (best < 0 || zv[i] < bz)) {
+          best = m0 + i;
+          bz = zv[i];
+        }
+    }
+  } else {
+#pragma unroll 4
+    for (int m = 0; m < M; ++m) {
+      const uint8_t cv = c[m];
+      const T zv = z[m];
+      if (cv != kIdle && (best < 0 || zv < bz)) {
+        best = m;
+        bz = zv;
+      }
+    }
   }
-  for (int o = 16; o > 0; o >>= 1) {
-    const int ob = __shfl_down_sync(0xffffffffu, best, o);
-    const T oz = __shfl_down_sync(0xffffffffu, bz, o);
-    if (ob >= 0 && (best < 0 || oz < bz || (oz == bz && ob < best))) { best = ob; bz = oz; }
-  }
-  if (lane == 0) recv[k] = best;
+  recv[k] = best;
 }
 
 // ---- per-window donor preference order (Sec. IV-B), warp per window ---------
@@ -989,7 +1022,11 @@ template <class T>
 cudaError_t launch_receiver(int M, int K, const T* Z, const uint8_t* cls, int32_t* recv,
                             cudaStream_t s) {
   if (K == 0) return cudaSuccess;
-  k_receiver<T><<<(unsigned)((K + 7) / 8), 256, 0, s>>>(M, K, Z, cls, recv);
+  const unsigned g = (unsigned)((K + 255) / 256);
+  if (M % 4 == 0 && (((uintptr_t)Z | (uintptr_t)cls) & 15) == 0)
+    k_receiver<T, true><<<g, 256, 0, s>>>(M, K, Z, cls, recv);
+  else
+    k_receiver<T, false><<<g, 256, 0, s>>>(M, K, Z, cls, recv);
   return cudaGetLastError();
 }
 
