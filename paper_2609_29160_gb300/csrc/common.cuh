@@ -55,7 +55,7 @@ __device__ __forceinline__ void divmod(unsigned long long x, uint32_t d, unsigne
 struct FastDiv {
   uint32_t d, m, s1, s2;
   FastDiv() = default;
-  explicit FastDiv(uint32_t div) : d(div) {
+  __host__ __device__ explicit FastDiv(uint32_t div) : d(div) {
     uint32_t l = 0;
     while ((1ull << l) < div) ++l;
     m = (uint32_t)(((1ull << 32) * ((1ull << l) - div)) / div + 1);

@@ -891,7 +891,6 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
   const size_t row0 = (size_t)b.ent_base[si] * b.n_tau + (size_t)ti * n_ent;
   const int nf = (int)((int64_t)K * win / b.fast_ms);   // fast ticks = all ticks
   const int ratio = b.slow_ms / b.fast_ms;
-  const unsigned full = 0xffffffffu;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, n_warps = blockDim.x >> 5;
   // shared layout: per tick u < nf: action record and window; per tick
   // u <= nf: for every model the next tick >= u where it is a donor (one
@@ -903,33 +902,43 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
   int32_t* swin = reinterpret_cast<int32_t*>(srec + nf);
   uint16_t* snx = store_win ? reinterpret_cast<uint16_t*>(swin + ((nf + 3) & ~3))
                             : reinterpret_cast<uint16_t*>(swin);           // [nf + 1][MMAX]
+  // window of fast tick u, ceil((u + 1) * fast / win) - 1, without a divide
+  // instruction (the tick times stay below 2^31 ms)
+  const FastDiv fwin((uint32_t)win);
+  auto tick_of = [&](int u) -> int32_t {
+    return (int32_t)fwin.div((uint32_t)(u + 1) * (uint32_t)b.fast_ms + (uint32_t)win - 1u) - 1;
+  };
   auto tick_win = [&](int u) -> int32_t {
-    return store_win ? swin[u] : (int32_t)tick_window(u + 1, b.fast_ms, win);
+    return store_win ? swin[u] : tick_of(u);
   };
   uint16_t* sany = snx + (size_t)(nf + 1) * MMAX;                          // [nf + 1]
   __shared__ int s_cap[8][MMAX];   // unit footprints: replicas above the floor, per warp
+#pragma unroll 4
   for (int u = threadIdx.x; u < nf; u += blockDim.x) {
     int kd = 0, rv = -1;
     unsigned long long pk = 0;
     uint32_t dm = 0;
     if (!RANK) {
+      // both entries' loads issued before either is used
+      const bool has_slow = (u + 1) % ratio == 0;
+      const int es = nf + (u + 1) / ratio - 1;
       const int rf = recv_tab[row0 + u];
-      int e = -1;
+      const unsigned long long pf = packed[row0 + u];
+      const uint32_t df = dmask[row0 + u];
+      const int rs = has_slow ? recv_tab[row0 + es] : -1;
+      const unsigned long long ps = has_slow ? packed[row0 + es] : 0ull;
+      const uint32_t ds = has_slow ? dmask[row0 + es] : 0u;
       if (rf >= 0) {
-        e = u; kd = TRE_RESCUE; rv = rf;
-      } else if ((u + 1) % ratio == 0) {
-        const int es = nf + (u + 1) / ratio - 1;
-        const int rs = recv_tab[row0 + es];
-        if (rs >= 0) { e = es; kd = TRE_REBALANCE; rv = rs; }
+        kd = TRE_RESCUE; rv = rf; pk = pf; dm = df;
+      } else if (rs >= 0) {
+        kd = TRE_REBALANCE; rv = rs; pk = ps; dm = ds;
       }
-      pk = e >= 0 ? packed[row0 + e] : 0ull;
-      dm = e >= 0 ? dmask[row0 + e] : 0u;
     } else {
       // a slow tick falls on the window of the fast tick it coincides with;
       // a rescue at a tick takes precedence over its rebalance
       T z[MMAX];
       uint8_t cl[MMAX];
-      tick_row<T, MMAX, QUAD>(b, si, (uint32_t)tick_window(u + 1, b.fast_ms, win), z, cl);
+      tick_row<T, MMAX, QUAD>(b, si, (uint32_t)tick_of(u), z, cl);
       TickAction<T, MMAX, QUAD> a;
       tick_action<T, MMAX, QUAD>(b, ti, true, z, cl, a);
       if (a.recv >= 0) {
@@ -946,35 +955,45 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
     t.kind = (uint8_t)kd;
     t.pad = 0;
     srec[u] = t;
-    if (store_win) swin[u] = (int32_t)tick_window(u + 1, b.fast_ms, win);
+    if (store_win) swin[u] = tick_of(u);
   }
   __syncthreads();
-  // next-tick tables: a suffix minimum per row, 32 ticks per step
-  for (int m = warp; m < MMAX + 1; m += n_warps) {
-    uint16_t* col = m < MMAX ? snx + m : sany;
-    const int cs = m < MMAX ? MMAX : 1;   // column stride
-    if (lane == 0) col[(size_t)nf * cs] = (uint16_t)nf;
-    if (m < MMAX && m >= M) {      // padding columns: never a donor
-      for (int u = lane; u < nf; u += 32) col[(size_t)u * cs] = (uint16_t)nf;
-      continue;
-    }
-    const int mm = m < MMAX ? m : M;   // model, or M for "anything acts"
-    int carry = nf;
-    for (int cb = (nf - 1) & ~31; cb >= 0; cb -= 32) {
-      const int u = cb + lane;
-      int v = nf;
-      if (u < nf) {
-        const TickRec& t = srec[u];
-        if (t.recv >= 0 && (mm == M || (t.dm >> mm & 1u))) v = u;
+  // next-tick tables, a suffix minimum per column (MMAX models, then "any"):
+  // the CTA's threads split each column into segments of consecutive ticks;
+  // each finds its segment's first acting tick, then writes its segment
+  // backwards from the first acting tick of the segments after it
+  constexpr int NC = MMAX + 1;
+  const int n_seg = (int)blockDim.x / NC;              // segments per column
+  const int seg_len = (nf + n_seg - 1) / n_seg;
+  __shared__ int s_first[256];                         // [NC][n_seg]
+  const int my_c = threadIdx.x / n_seg, my_s = threadIdx.x % n_seg;
+  const bool has_seg = my_c < NC;
+  auto acts = [&](int u, int c) -> bool {
+    const TickRec& t = srec[u];
+    if (t.recv < 0) return false;
+    if (c == MMAX) return true;                        // anything acts
+    return c < M && (t.dm >> c & 1u);                  // padding columns never give
+  };
+  const int u_lo = my_s * seg_len, u_hi = min(nf, u_lo + seg_len);
+  if (has_seg) {
+    int f = nf;
+    for (int u = u_lo; u < u_hi; ++u)
+      if (acts(u, my_c)) {
+        f = u;
+        break;
       }
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const int y = __shfl_down_sync(full, v, o);
-        if (lane + o < 32) v = min(v, y);
-      }
-      v = min(v, carry);
-      if (u < nf) col[(size_t)u * cs] = (uint16_t)v;
-      carry = __shfl_sync(full, v, 0);
+    s_first[threadIdx.x] = f;
+  }
+  __syncthreads();
+  if (has_seg) {
+    uint16_t* col = my_c < MMAX ? snx + my_c : sany;
+    const int cs = my_c < MMAX ? MMAX : 1;             // column stride
+    int v = nf;
+    for (int j = my_s + 1; j < n_seg; ++j) v = min(v, s_first[my_c * n_seg + j]);
+    if (my_s == n_seg - 1) col[(size_t)nf * cs] = (uint16_t)nf;
+    for (int u = u_hi - 1; u >= u_lo; --u) {
+      if (acts(u, my_c)) v = u;
+      col[(size_t)u * cs] = (uint16_t)v;
     }
   }
   __syncthreads();
@@ -1083,6 +1102,52 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
         avail |= 1u << recv;
       }
       for (int m = 0; m < M; ++m) scap[m] = (int)((cp >> (8 * m)) & 0xFFull);
+      nm = nm1;
+      u = nf;
+    }
+    if (Kp == 1 && MMAX == 16 && b.budget <= 255) {
+      // as above for up to 16 models: the replicas above the floor packed a
+      // byte per model in two registers, and the donor the first model of
+      // the tick's order that can still give (the jump only lands on ticks
+      // that have one when the pool is empty)
+      unsigned long long c0 = 0ull, c1 = 0ull;
+      for (int m = 0; m < M; ++m) {
+        const unsigned long long v = (unsigned long long)scap[m] << (8 * (m & 7));
+        if (m < 8) c0 |= v; else c1 |= v;
+      }
+      int32_t nm1 = 0;
+      while (true) {
+        const int nxt = next_tick(u);
+        if (nxt >= nf) break;
+        u = nxt + 1;
+        const TickRec tr = srec[nxt];
+        const int32_t k = tick_win(nxt);
+        const int recv = tr.recv;
+        int donor = -1;
+        if (free_pool > 0) {
+          --free_pool;
+        } else {
+          const uint32_t left = avail & tr.dm;
+          unsigned long long pk = tr.pk;
+          int d = (int)(pk & 15u);
+          for (int p = 1; p < MMAX && !((left >> d) & 1u); ++p) {
+            pk >>= 4;
+            d = (int)(pk & 15u);
+          }
+          donor = d;
+          const int sh = 8 * (d & 7);
+          const unsigned long long c = (d < 8 ? c0 : c1) - (1ull << sh);
+          if (d < 8) c0 = c; else c1 = c;
+          if (((c >> sh) & 0xFFull) == 0) avail &= ~(1u << d);
+        }
+        put_move(mv, nm1, cap, k, recv, donor, tr.kind, 0);
+        ++nm1;
+        if (recv < 8) c0 += 1ull << (8 * recv);
+        else c1 += 1ull << (8 * (recv - 8));
+        avail |= 1u << recv;
+      }
+      for (int m = 0; m < M; ++m)
+        scap[m] = (int)(((m < 8 ? c0 : c1) >> (8 * (m & 7))) & 0xFFull);
       nm = nm1;
       u = nf;
     }
