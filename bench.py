@@ -919,9 +919,13 @@ def main():
     def roof_of(name):
         per_call_ms = phases[name]["ms"] / max(phases[name]["calls"], 1)
         achieved = pb[name] / (per_call_ms / 1e3) / 1e9
+        cap = captured_traffic(name)
+        # traffic: DRAM bytes per call from the one ncu capture of this kernel
+        # source (null once the source has changed since the capture)
         return {"bound": "hbm", "kernel": name, "achieved": achieved, "peak": hbm,
-                "unit": "GB/s", "frac": achieved / hbm, "traffic": None,
-                "ncu_capture": captured_traffic(name),
+                "unit": "GB/s", "frac": achieved / hbm,
+                "traffic": cap["dram_bytes_per_call"] if cap else None,
+                "ncu_capture": cap,
                 "share_of_step": phases[name]["ms"] / max(ms, 1e-9), "peak_kind": peak_kind,
                 "bytes_per_call": pb[name], "us_per_call": per_call_ms * 1e3}
     if dom in pb and phases[dom]["calls"]:

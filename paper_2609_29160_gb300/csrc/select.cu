@@ -549,29 +549,47 @@ k_walk(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab, const in
   // to the first that can act.
   if (MPL <= 2 && F >= win && Sl % F == 0) {
     const int64_t ratio = Sl / F;
-    int64_t u0 = 0;
-    while (u0 < nf) {
+    // tick windows by multiply-high division (tick times stay below 2^31 ms)
+    const FastDiv fwin((uint32_t)win);
+    // the table entries of 32 consecutive fast ticks, one per lane: receivers
+    // and donor masks of the tick and of the slow tick it carries
+    struct Ent {
+      int rf, rs;
+      unsigned long long df, ds;
+    };
+    // entry of the slow tick carried by fast tick u
+    auto slow_ent = [&](int64_t u) { return (int32_t)(nf + (u + 1) / ratio - 1); };
+    auto load = [&](int64_t base, Ent& e) {
+      const int64_t u = base + lane;
+      const int32_t es = slow_ent(u);
+      const bool in = u < nf;
+      const bool has_slow = in && (u + 1) % ratio == 0 && es < n_ent;
+      e.rf = in ? rv_tab[u] : -1;
+      e.df = in ? dm_tab[u] : 0ull;
+      e.rs = has_slow ? rv_tab[es] : -1;
+      e.ds = has_slow ? dm_tab[es] : 0ull;
+    };
+    // the next group's entries are loaded while the current group is tested
+    // and acted on; after a tick acts, the rest of its group is tested again
+    // against the new state without loading anything
+    Ent cur, nxt;
+    int64_t base = 0;
+    int start = 0;   // lanes of the current group before it are done
+    load(0, cur);
+    load(32, nxt);
+    while (base < nf) {
       unsigned long long above = 0;
 #pragma unroll
       for (int j = 0; j < MPL; ++j)
         above |= (unsigned long long)__ballot_sync(0xffffffffu, lane + 32 * j < M && r[j] > rmin[j])
                  << (32 * j);
-      const int64_t u = u0 + lane;
       int rv = -1, kind = 0;
       int32_t ent = -1;
       unsigned long long dn = 0;
-      if (u < nf) {
-        const int32_t es = (int32_t)(nf + (u + 1) / ratio - 1);
-        const bool has_slow = (u + 1) % ratio == 0 && es < n_ent;
-        const int rf = rv_tab[u];
-        const int rs = has_slow ? rv_tab[es] : -1;
-        const unsigned long long df = dm_tab[u];
-        const unsigned long long ds = has_slow ? dm_tab[es] : 0ull;
-        if (rf >= 0) {
-          rv = rf; kind = TRE_RESCUE; ent = (int32_t)u; dn = df;
-        } else if (rs >= 0) {
-          rv = rs; kind = TRE_REBALANCE; ent = es; dn = ds;
-        }
+      if (cur.rf >= 0) {
+        rv = cur.rf; kind = TRE_RESCUE; ent = (int32_t)(base + lane); dn = cur.df;
+      } else if (cur.rs >= 0) {
+        rv = cur.rs; kind = TRE_REBALANCE; ent = slow_ent(base + lane); dn = cur.ds;
       }
       // the receiver's footprint sits in lane rv % 32, slot rv / 32
       int g_rv = 0;
@@ -580,19 +598,26 @@ k_walk(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab, const in
         const int x = __shfl_sync(0xffffffffu, g[j], rv & 31);
         if (rv >= 0 && (rv >> 5) == j) g_rv = x;
       }
-      const bool can = rv >= 0 && (free_pool >= g_rv || (dn & above) != 0);
+      const bool can = lane >= start && rv >= 0 && (free_pool >= g_rv || (dn & above) != 0);
       const unsigned hit = __ballot_sync(0xffffffffu, can);
-      if (!hit) {
-        u0 += 32;
-        continue;
+      int next_start = 32;
+      if (hit) {
+        const int src = __ffs(hit) - 1;
+        const int32_t e_t = __shfl_sync(0xffffffffu, ent, src);
+        const int rv_t = __shfl_sync(0xffffffffu, rv, src);
+        const int kd_t = __shfl_sync(0xffffffffu, kind, src);
+        act((int32_t)fwin.div((uint32_t)(base + src + 1) * (uint32_t)F + (uint32_t)win - 1u) - 1,
+            rv_t, kd_t, e_t);
+        next_start = src + 1;
       }
-      const int src = __ffs(hit) - 1;
-      const int32_t e_t = __shfl_sync(0xffffffffu, ent, src);
-      const int rv_t = __shfl_sync(0xffffffffu, rv, src);
-      const int kd_t = __shfl_sync(0xffffffffu, kind, src);
-      const int64_t ut = u0 + src;
-      act((int32_t)tick_window(ut + 1, F, win), rv_t, kd_t, e_t);
-      u0 = ut + 1;
+      if (next_start < 32) {
+        start = next_start;
+      } else {
+        base += 32;
+        cur = nxt;
+        load(base + 32, nxt);
+        start = 0;
+      }
     }
   } else {
     while (true) {
