@@ -92,308 +92,314 @@ k_reduce_requests(const __grid_constant__ ReqBatch bt, int M, int lgMp, int win,
                   unsigned long long* __restrict__ slo0, const int32_t* __restrict__ slo_ms,
                   tre_diag* diag) {
   extern __shared__ unsigned long long smem[];
-  int t = 0;
-  while (t + 1 < bt.n && bt.cta_base[t + 1] <= (int)blockIdx.x) ++t;
-  const ReqCols& r = bt.cols[t];
-  const bool vec = (bt.vec_ok >> t) & 1ull;
-  const size_t cells1 = (size_t)(K + 1) * M;
-  int32_t* P = P0 + bt.out_off[t];
-  int32_t* D = D0 + bt.out_off[t];
-  int32_t* dA = dA0 + t * cells1;
-  int32_t* dW = dW0 + t * cells1;
-  unsigned long long* slo = SLO ? slo0 + bt.out_off[t] : nullptr;
-  const int64_t i0 = (int64_t)(blockIdx.x - bt.cta_base[t]) * bt.per_cta[t];
-  const int n_loc = (int)min64(r.n - i0, bt.per_cta[t]);
-  if (n_loc <= 0) return;
-  const int Mp = 1 << lgMp, F = 1 << lgF, F1 = F + 1;
-  const uint32_t span = (uint32_t)K * (uint32_t)win;
-  // Columns of this CTA's records: read in place, or (COPY, for records in
-  // host memory) first copied once into shared memory so that no column is
-  // read twice over the host link.
-  const int32_t* gcol[7] = {r.model + i0, r.t_arr + i0, r.t_start + i0, r.t_first + i0,
-                            r.t_end + i0, r.L_in + i0, r.L_out + i0};
-  const int32_t* colp[7];
-  int32_t* recs = reinterpret_cast<int32_t*>(smem);
-  const int cap_rec = COPY ? (int)bt.per_cta[t] : 0;
-  if (COPY) {
-#pragma unroll
-    for (int c = 0; c < 7; ++c) {
-      int32_t* dst = recs + (size_t)c * cap_rec;
-      for (int i = threadIdx.x * 4; i < n_loc; i += kThreads * 4) {
-        if (vec && i + 4 <= n_loc) {
-          *reinterpret_cast<int4*>(dst + i) = *reinterpret_cast<const int4*>(gcol[c] + i);
-        } else {
-          for (int u = 0; u < 4 && i + u < n_loc; ++u) dst[i + u] = gcol[c][i + u];
-        }
-      }
-      colp[c] = dst;
-    }
-  } else {
-#pragma unroll
-    for (int c = 0; c < 7; ++c) colp[c] = gcol[c];
-  }
-  const bool vec4 = COPY || vec;
-  const int a_first = gcol[1][0], a_last = gcol[1][n_loc - 1];
-  const int k_lo = a_first < 0 ? 0 : (int)min(fd.div((uint32_t)a_first), (uint32_t)K);
-  const int k_hi = a_last < 0 ? 0 : (int)min(fd.div((uint32_t)a_last), (uint32_t)K);
-  const int used = min(near_rows, (k_hi >= k_lo ? k_hi - k_lo + 1 : 1) + 1);
-  Stage st;
-  st.aW = reinterpret_cast<int32_t*>(smem + (size_t)cap_rec * 7 / 2);
-  st.aS = reinterpret_cast<uint32_t*>(st.aW + (size_t)near_rows * Mp);
-  st.fP = reinterpret_cast<int32_t*>(st.aS + (SLO ? (size_t)near_rows * Mp : 0));
-  st.fD = st.fP + (size_t)M * F1;
-  st.fAW = st.fD + (size_t)M * F1;
-  st.far_lo = st.fAW + (size_t)M * F1;
-  st.slo_lim = st.far_lo + M;
-  st.queue = reinterpret_cast<uint16_t*>((reinterpret_cast<uintptr_t>(st.slo_lim + M) + 15) &
-                                         ~(uintptr_t)15) +
-             (size_t)(threadIdx.x >> 5) * (bt.per_cta[t] / (kThreads / 32));
-  const int ncell = used * Mp, fcell = M * F1;
-  for (int c = threadIdx.x; c < ncell; c += kThreads) {
-    st.aW[c] = 0;
-    if (SLO) st.aS[c] = 0;
-  }
-  for (int c = threadIdx.x; c < fcell; c += kThreads) { st.fP[c] = 0; st.fD[c] = 0; st.fAW[c] = 0; }
-  for (int m = threadIdx.x; m < M; m += kThreads) {
-    st.far_lo[m] = 0x7fffffff;
-    if (SLO) st.slo_lim[m] = slo_ms[m];
-  }
-  __syncthreads();
-  // each model's earliest start window among the CTA's first kFarScan
-  // records: records come in arrival order and each model starts its requests
-  // in arrival order (first come, first served), so its earliest starts are
-  // among its first records; a record that starts before this window takes
-  // the global path (the tests below check both ends)
-  for (int b = threadIdx.x * kVec; b < min(n_loc, kFarScan); b += kThreads * kVec) {
-    int mm[kVec], ss[kVec];
-    if (vec4 && b + kVec <= n_loc) {
-      const int4 a = *reinterpret_cast<const int4*>(colp[0] + b);
-      const int4 s = *reinterpret_cast<const int4*>(colp[2] + b);
-      mm[0] = a.x; mm[1] = a.y; mm[2] = a.z; mm[3] = a.w;
-      ss[0] = s.x; ss[1] = s.y; ss[2] = s.z; ss[3] = s.w;
-    } else {
-#pragma unroll
-      for (int u = 0; u < kVec; ++u) {
-        const bool in = b + u < n_loc;
-        mm[u] = in ? colp[0][b + u] : -1;
-        ss[u] = in ? colp[2][b + u] : -1;
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < kVec; ++u)
-      if (mm[u] >= 0 && mm[u] < M && ss[u] >= 0)
-        atomicMin(&st.far_lo[mm[u]], (int)min(fd.div((uint32_t)ss[u]), (uint32_t)K));
-  }
-  __syncthreads();
-
-  // arrival-side target
-  auto near_idx = [&](int k, int m) -> int {
-    const unsigned rel = (unsigned)(k - k_lo);
-    return rel < (unsigned)used ? (int)(rel << lgMp) + m : -1;
-  };
-  // start-side target of model m: shared cell index, or -1 when outside
-  auto far_idx = [&](int k, int m, int lo) -> int {
-    const unsigned rel = (unsigned)(k - lo);
-    return rel < (unsigned)F ? m * F1 + (int)rel : -1;
-  };
-  auto add_tok = [&](int32_t* s_arr, int32_t* g_arr, int k, int m, int lo, int32_t v) {
-    const int c = far_idx(k, m, lo);
-    if (c >= 0) atomicAdd(&s_arr[c], v);
-    else atomicAdd(&g_arr[(size_t)k * M + m], v);
-  };
-  auto add_aw = [&](int k, int m, int lo, int32_t a, int32_t w) {
-    const int c = far_idx(k, m, lo);
-    if (c >= 0) {
-      atomicAdd(&st.fAW[c], a + w * 65536);
-    } else {
-      if (a) atomicAdd(&dA[(size_t)k * M + m], a);
-      if (w) atomicAdd(&dW[(size_t)k * M + m], w);
-    }
-  };
-
-  const unsigned full = 0xffffffffu;
-  const int lane = threadIdx.x & 31;
-  const int warp = threadIdx.x >> 5;
   unsigned long long n_range = 0, n_model = 0, n_order = 0;
-  // warp-uniform passes: lane l of a pass takes records b + l*kVec + u
-  int qn = 0;   // entries in the warp's queue
-  for (int wb = warp * 32 * kVec; wb < n_loc; wb += kThreads * kVec) {
-    const int b = wb + lane * kVec;
-    int v[7][kVec];
-    if (vec4 && b + kVec <= n_loc) {
+  // a CTA takes slices blockIdx.x, blockIdx.x + gridDim.x, ...: one slice when
+  // the grid holds them all; a smaller grid leaves SMs to other streams' work
+  // (records read over the host link keep fewer SMs busy just as well)
+  for (int vb = blockIdx.x; vb < bt.cta_base[bt.n]; vb += gridDim.x) {
+    int t = 0;
+    while (t + 1 < bt.n && bt.cta_base[t + 1] <= vb) ++t;
+    const ReqCols& r = bt.cols[t];
+    const bool vec = (bt.vec_ok >> t) & 1ull;
+    const size_t cells1 = (size_t)(K + 1) * M;
+    int32_t* P = P0 + bt.out_off[t];
+    int32_t* D = D0 + bt.out_off[t];
+    int32_t* dA = dA0 + t * cells1;
+    int32_t* dW = dW0 + t * cells1;
+    unsigned long long* slo = SLO ? slo0 + bt.out_off[t] : nullptr;
+    const int64_t i0 = (int64_t)(vb - bt.cta_base[t]) * bt.per_cta[t];
+    const int n_loc = (int)min64(r.n - i0, bt.per_cta[t]);
+    if (n_loc <= 0) continue;
+    const int Mp = 1 << lgMp, F = 1 << lgF, F1 = F + 1;
+    const uint32_t span = (uint32_t)K * (uint32_t)win;
+    // Columns of this CTA's records: read in place, or (COPY, for records in
+    // host memory) first copied once into shared memory so that no column is
+    // read twice over the host link.
+    const int32_t* gcol[7] = {r.model + i0, r.t_arr + i0, r.t_start + i0, r.t_first + i0,
+                              r.t_end + i0, r.L_in + i0, r.L_out + i0};
+    const int32_t* colp[7];
+    int32_t* recs = reinterpret_cast<int32_t*>(smem);
+    const int cap_rec = COPY ? (int)bt.per_cta[t] : 0;
+    if (COPY) {
 #pragma unroll
       for (int c = 0; c < 7; ++c) {
-        // streaming loads, except the four columns the long-decode walk reads
-        // again (model, first-token and end times, output length)
-        const bool again = c == 0 || c == 3 || c == 4 || c == 6;
-        const int4 q = COPY ? *reinterpret_cast<const int4*>(colp[c] + b)
-                       : again ? *reinterpret_cast<const int4*>(colp[c] + b)
-                               : __ldcs(reinterpret_cast<const int4*>(colp[c] + b));
-        v[c][0] = q.x; v[c][1] = q.y; v[c][2] = q.z; v[c][3] = q.w;
+        int32_t* dst = recs + (size_t)c * cap_rec;
+        for (int i = threadIdx.x * 4; i < n_loc; i += kThreads * 4) {
+          if (vec && i + 4 <= n_loc) {
+            *reinterpret_cast<int4*>(dst + i) = *reinterpret_cast<const int4*>(gcol[c] + i);
+          } else {
+            for (int u = 0; u < 4 && i + u < n_loc; ++u) dst[i + u] = gcol[c][i + u];
+          }
+        }
+        colp[c] = dst;
       }
     } else {
 #pragma unroll
-      for (int u = 0; u < kVec; ++u) {
-        const bool in = b + u < n_loc;
-#pragma unroll
-        for (int c = 0; c < 7; ++c) v[c][u] = in ? colp[c][b + u] : 0;
-        if (!in) v[0][u] = -1;   // marks "no record" (not counted as a drop)
-      }
+      for (int c = 0; c < 7; ++c) colp[c] = gcol[c];
     }
-#pragma unroll
-    for (int u = 0; u < kVec; ++u) {
-      const bool present = b + u < n_loc;
-      const int m = v[0][u], ta = v[1][u], ts = v[2][u], tf = v[3][u], te = v[4][u];
-      const int L_in = v[5][u], L = v[6][u];
-      bool ok = false;
-      if (present) {
-        if (m < 0 || m >= M) ++n_model;
-        else if (ta < 0 || (uint32_t)ta >= span) ++n_range;
-        else if (!(ta <= ts && ts <= tf && tf <= te) || L_in < 0 || L < 1) ++n_order;
-        else ok = true;
-      }
-      // decode windows after the first-token window go to the warp's queue
-      bool lng = false;
-      int kf = 0;
-      if (ok) {
-        const int lo = st.far_lo[m];
-        const int ba = (int)fd.div((uint32_t)ta);
-        const int bs = (int)min(fd.div((uint32_t)ts), (uint32_t)K);
-        const int be_raw = (int)fd.div((uint32_t)te);
-        const int be = min(be_raw, K);
-        const bool tok = (uint32_t)tf < span;
-        kf = tok ? (int)fd.div((uint32_t)tf) : 0;
-        // decode tokens of the first-token window (d0) and, for a decode that
-        // ends in the next window, of that window (d1); longer decodes leave
-        // their later windows to the queue walk below
-        int d0 = L, d1 = 0;
-        if (tok && L != 1 && be_raw != kf) {
-          // N(T) = tokens emitted before T = ceil((T - tf)(L-1)/dur)
-          unsigned long long qq, rr;
-          divmod((unsigned long long)((uint32_t)(kf + 1) * (uint32_t)win - (uint32_t)tf) *
-                     (uint32_t)(L - 1),
-                 (uint32_t)(te - tf), qq, rr);
-          const int n1 = (int)(qq + (rr != 0));
-          d0 = n1;
-          if (be_raw == kf + 1) d1 = L - n1;
-          else lng = kf + 1 < K;   // windows kf+1 .. min(be, K-1)
-        }
-        const int wait = ba != bs ? 1 : 0, run = bs != be ? 1 : 0;
-        const uint32_t met = SLO && (tf - ta <= st.slo_lim[m]) ? 1u : 0u;
-        const uint32_t rel_a = (uint32_t)(ba - k_lo);
-        // bs <= kf <= be: the two ends bound every start-side target
-        if (rel_a < (uint32_t)used && (uint32_t)(be - lo) < (uint32_t)F && bs >= lo) {
-          const int na = (int)(rel_a << lgMp) + m;
-          const int fb = m * F1 - lo;
-          atomicAdd(&st.aW[na], wait);
-          if (SLO) atomicAdd(&st.aS[na], 1u + (met << 16));
-          atomicAdd(&st.fAW[fb + bs], run - wait * 65536);
-          if (run) atomicAdd(&st.fAW[fb + be], -1);
-          if (tok) {
-            if (L_in) atomicAdd(&st.fP[fb + kf], L_in);
-            atomicAdd(&st.fD[fb + kf], d0);
-            if (d1) atomicAdd(&st.fD[fb + kf + 1], d1);
-          }
-        } else {
-          const int na = near_idx(ba, m);
-          if (wait) {
-            if (na >= 0) atomicAdd(&st.aW[na], 1);
-            else atomicAdd(&dW[(size_t)ba * M + m], 1);
-          }
-          if (SLO) {
-            if (na >= 0) atomicAdd(&st.aS[na], 1u + (met << 16));
-            else atomicAdd(&slo[(size_t)ba * M + m], 1ull + ((unsigned long long)met << 32));
-          }
-          if (run | wait) add_aw(bs, m, lo, run, -wait);
-          if (run) add_aw(be, m, lo, -1, 0);
-          if (tok) {
-            if (L_in) add_tok(st.fP, P, kf, m, lo, L_in);
-            add_tok(st.fD, D, kf, m, lo, d0);
-            if (d1 && kf + 1 < K) add_tok(st.fD, D, kf + 1, m, lo, d1);
-          }
-        }
-      }
-      const unsigned qb = __ballot_sync(full, lng);
-      if (lng) st.queue[qn + __popc(qb & ((1u << lane) - 1u))] = (uint16_t)(b + u);
-      qn += __popc(qb);
+    const bool vec4 = COPY || vec;
+    const int a_first = gcol[1][0], a_last = gcol[1][n_loc - 1];
+    const int k_lo = a_first < 0 ? 0 : (int)min(fd.div((uint32_t)a_first), (uint32_t)K);
+    const int k_hi = a_last < 0 ? 0 : (int)min(fd.div((uint32_t)a_last), (uint32_t)K);
+    const int used = min(near_rows, (k_hi >= k_lo ? k_hi - k_lo + 1 : 1) + 1);
+    Stage st;
+    st.aW = reinterpret_cast<int32_t*>(smem + (size_t)cap_rec * 7 / 2);
+    st.aS = reinterpret_cast<uint32_t*>(st.aW + (size_t)near_rows * Mp);
+    st.fP = reinterpret_cast<int32_t*>(st.aS + (SLO ? (size_t)near_rows * Mp : 0));
+    st.fD = st.fP + (size_t)M * F1;
+    st.fAW = st.fD + (size_t)M * F1;
+    st.far_lo = st.fAW + (size_t)M * F1;
+    st.slo_lim = st.far_lo + M;
+    st.queue = reinterpret_cast<uint16_t*>((reinterpret_cast<uintptr_t>(st.slo_lim + M) + 15) &
+                                           ~(uintptr_t)15) +
+               (size_t)(threadIdx.x >> 5) * (bt.per_cta[t] / (kThreads / 32));
+    const int ncell = used * Mp, fcell = M * F1;
+    for (int c = threadIdx.x; c < ncell; c += kThreads) {
+      st.aW[c] = 0;
+      if (SLO) st.aS[c] = 0;
     }
-  }
-  // walk the warp's long decodes, one record per lane
-  __syncwarp();
-  for (int i = lane; i < qn; i += 32) {
-    const int j = st.queue[i];
-    const int m = colp[0][j], tf = colp[3][j], te = colp[4][j], L = colp[6][j];
-    const int kf = (int)fd.div((uint32_t)tf), be_raw = (int)fd.div((uint32_t)te);
-    const uint32_t dur = (uint32_t)(te - tf);
-    unsigned long long qq, rr;
-    divmod((unsigned long long)((uint32_t)(kf + 1) * (uint32_t)win - (uint32_t)tf) *
-               (uint32_t)(L - 1),
-           dur, qq, rr);
-    const uint32_t q1 = (uint32_t)qq, r1 = (uint32_t)rr;
-    {
-      // y = x + dur - 1 at the end of window kf: N = floor(y / dur), rem = y mod dur
-      uint32_t n = q1 + (r1 != 0);
-      uint32_t rem = r1 ? r1 - 1 : dur - 1;
-      unsigned long long Q64, R64;
-      divmod((unsigned long long)(uint32_t)win * (uint32_t)(L - 1), dur, Q64, R64);
-      const uint32_t Q = (uint32_t)Q64, R = (uint32_t)R64;   // Q < L: dur > win here
-      const int lo = st.far_lo[m];
-      const int k_full = min(be_raw - 1, K - 1);   // windows ending at or before t_end
-      const int k_end = min(be_raw, K - 1);
-      if ((uint32_t)(k_end - lo) < (uint32_t)F && kf + 1 >= lo) {
-        int32_t* fd_row = st.fD + m * F1 - lo;
-        for (int k = kf + 1; k <= k_full; ++k) {
-          const uint32_t t = rem + R;
-          const uint32_t c = t >= dur ? 1u : 0u;
-          rem = t - (c ? dur : 0u);
-          const uint32_t d = Q + c;
-          n += d;
-          if (d) atomicAdd(&fd_row[k], (int32_t)d);
-        }
-        if (be_raw <= K - 1 && (uint32_t)L != n) atomicAdd(&fd_row[be_raw], (int32_t)(L - n));
+    for (int c = threadIdx.x; c < fcell; c += kThreads) { st.fP[c] = 0; st.fD[c] = 0; st.fAW[c] = 0; }
+    for (int m = threadIdx.x; m < M; m += kThreads) {
+      st.far_lo[m] = 0x7fffffff;
+      if (SLO) st.slo_lim[m] = slo_ms[m];
+    }
+    __syncthreads();
+    // each model's earliest start window among the CTA's first kFarScan
+    // records: records come in arrival order and each model starts its requests
+    // in arrival order (first come, first served), so its earliest starts are
+    // among its first records; a record that starts before this window takes
+    // the global path (the tests below check both ends)
+    for (int b = threadIdx.x * kVec; b < min(n_loc, kFarScan); b += kThreads * kVec) {
+      int mm[kVec], ss[kVec];
+      if (vec4 && b + kVec <= n_loc) {
+        const int4 a = *reinterpret_cast<const int4*>(colp[0] + b);
+        const int4 s = *reinterpret_cast<const int4*>(colp[2] + b);
+        mm[0] = a.x; mm[1] = a.y; mm[2] = a.z; mm[3] = a.w;
+        ss[0] = s.x; ss[1] = s.y; ss[2] = s.z; ss[3] = s.w;
       } else {
-        for (int k = kf + 1; k <= k_full; ++k) {
-          const uint32_t t = rem + R;
-          const uint32_t c = t >= dur ? 1u : 0u;
-          rem = t - (c ? dur : 0u);
-          const uint32_t d = Q + c;
-          n += d;
-          if (d) add_tok(st.fD, D, k, m, lo, (int32_t)d);
+#pragma unroll
+        for (int u = 0; u < kVec; ++u) {
+          const bool in = b + u < n_loc;
+          mm[u] = in ? colp[0][b + u] : -1;
+          ss[u] = in ? colp[2][b + u] : -1;
         }
-        if (be_raw <= K - 1 && (uint32_t)L != n) add_tok(st.fD, D, be_raw, m, lo, (int32_t)(L - n));
+      }
+#pragma unroll
+      for (int u = 0; u < kVec; ++u)
+        if (mm[u] >= 0 && mm[u] < M && ss[u] >= 0)
+          atomicMin(&st.far_lo[mm[u]], (int)min(fd.div((uint32_t)ss[u]), (uint32_t)K));
+    }
+    __syncthreads();
+
+    // arrival-side target
+    auto near_idx = [&](int k, int m) -> int {
+      const unsigned rel = (unsigned)(k - k_lo);
+      return rel < (unsigned)used ? (int)(rel << lgMp) + m : -1;
+    };
+    // start-side target of model m: shared cell index, or -1 when outside
+    auto far_idx = [&](int k, int m, int lo) -> int {
+      const unsigned rel = (unsigned)(k - lo);
+      return rel < (unsigned)F ? m * F1 + (int)rel : -1;
+    };
+    auto add_tok = [&](int32_t* s_arr, int32_t* g_arr, int k, int m, int lo, int32_t v) {
+      const int c = far_idx(k, m, lo);
+      if (c >= 0) atomicAdd(&s_arr[c], v);
+      else atomicAdd(&g_arr[(size_t)k * M + m], v);
+    };
+    auto add_aw = [&](int k, int m, int lo, int32_t a, int32_t w) {
+      const int c = far_idx(k, m, lo);
+      if (c >= 0) {
+        atomicAdd(&st.fAW[c], a + w * 65536);
+      } else {
+        if (a) atomicAdd(&dA[(size_t)k * M + m], a);
+        if (w) atomicAdd(&dW[(size_t)k * M + m], w);
+      }
+    };
+
+    const unsigned full = 0xffffffffu;
+    const int lane = threadIdx.x & 31;
+    const int warp = threadIdx.x >> 5;
+    // warp-uniform passes: lane l of a pass takes records b + l*kVec + u
+    int qn = 0;   // entries in the warp's queue
+    for (int wb = warp * 32 * kVec; wb < n_loc; wb += kThreads * kVec) {
+      const int b = wb + lane * kVec;
+      int v[7][kVec];
+      if (vec4 && b + kVec <= n_loc) {
+#pragma unroll
+        for (int c = 0; c < 7; ++c) {
+          // streaming loads, except the four columns the long-decode walk reads
+          // again (model, first-token and end times, output length)
+          const bool again = c == 0 || c == 3 || c == 4 || c == 6;
+          const int4 q = COPY ? *reinterpret_cast<const int4*>(colp[c] + b)
+                         : again ? *reinterpret_cast<const int4*>(colp[c] + b)
+                                 : __ldcs(reinterpret_cast<const int4*>(colp[c] + b));
+          v[c][0] = q.x; v[c][1] = q.y; v[c][2] = q.z; v[c][3] = q.w;
+        }
+      } else {
+#pragma unroll
+        for (int u = 0; u < kVec; ++u) {
+          const bool in = b + u < n_loc;
+#pragma unroll
+          for (int c = 0; c < 7; ++c) v[c][u] = in ? colp[c][b + u] : 0;
+          if (!in) v[0][u] = -1;   // marks "no record" (not counted as a drop)
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kVec; ++u) {
+        const bool present = b + u < n_loc;
+        const int m = v[0][u], ta = v[1][u], ts = v[2][u], tf = v[3][u], te = v[4][u];
+        const int L_in = v[5][u], L = v[6][u];
+        bool ok = false;
+        if (present) {
+          if (m < 0 || m >= M) ++n_model;
+          else if (ta < 0 || (uint32_t)ta >= span) ++n_range;
+          else if (!(ta <= ts && ts <= tf && tf <= te) || L_in < 0 || L < 1) ++n_order;
+          else ok = true;
+        }
+        // decode windows after the first-token window go to the warp's queue
+        bool lng = false;
+        int kf = 0;
+        if (ok) {
+          const int lo = st.far_lo[m];
+          const int ba = (int)fd.div((uint32_t)ta);
+          const int bs = (int)min(fd.div((uint32_t)ts), (uint32_t)K);
+          const int be_raw = (int)fd.div((uint32_t)te);
+          const int be = min(be_raw, K);
+          const bool tok = (uint32_t)tf < span;
+          kf = tok ? (int)fd.div((uint32_t)tf) : 0;
+          // decode tokens of the first-token window (d0) and, for a decode that
+          // ends in the next window, of that window (d1); longer decodes leave
+          // their later windows to the queue walk below
+          int d0 = L, d1 = 0;
+          if (tok && L != 1 && be_raw != kf) {
+            // N(T) = tokens emitted before T = ceil((T - tf)(L-1)/dur)
+            unsigned long long qq, rr;
+            divmod((unsigned long long)((uint32_t)(kf + 1) * (uint32_t)win - (uint32_t)tf) *
+                       (uint32_t)(L - 1),
+                   (uint32_t)(te - tf), qq, rr);
+            const int n1 = (int)(qq + (rr != 0));
+            d0 = n1;
+            if (be_raw == kf + 1) d1 = L - n1;
+            else lng = kf + 1 < K;   // windows kf+1 .. min(be, K-1)
+          }
+          const int wait = ba != bs ? 1 : 0, run = bs != be ? 1 : 0;
+          const uint32_t met = SLO && (tf - ta <= st.slo_lim[m]) ? 1u : 0u;
+          const uint32_t rel_a = (uint32_t)(ba - k_lo);
+          // bs <= kf <= be: the two ends bound every start-side target
+          if (rel_a < (uint32_t)used && (uint32_t)(be - lo) < (uint32_t)F && bs >= lo) {
+            const int na = (int)(rel_a << lgMp) + m;
+            const int fb = m * F1 - lo;
+            atomicAdd(&st.aW[na], wait);
+            if (SLO) atomicAdd(&st.aS[na], 1u + (met << 16));
+            atomicAdd(&st.fAW[fb + bs], run - wait * 65536);
+            if (run) atomicAdd(&st.fAW[fb + be], -1);
+            if (tok) {
+              if (L_in) atomicAdd(&st.fP[fb + kf], L_in);
+              atomicAdd(&st.fD[fb + kf], d0);
+              if (d1) atomicAdd(&st.fD[fb + kf + 1], d1);
+            }
+          } else {
+            const int na = near_idx(ba, m);
+            if (wait) {
+              if (na >= 0) atomicAdd(&st.aW[na], 1);
+              else atomicAdd(&dW[(size_t)ba * M + m], 1);
+            }
+            if (SLO) {
+              if (na >= 0) atomicAdd(&st.aS[na], 1u + (met << 16));
+              else atomicAdd(&slo[(size_t)ba * M + m], 1ull + ((unsigned long long)met << 32));
+            }
+            if (run | wait) add_aw(bs, m, lo, run, -wait);
+            if (run) add_aw(be, m, lo, -1, 0);
+            if (tok) {
+              if (L_in) add_tok(st.fP, P, kf, m, lo, L_in);
+              add_tok(st.fD, D, kf, m, lo, d0);
+              if (d1 && kf + 1 < K) add_tok(st.fD, D, kf + 1, m, lo, d1);
+            }
+          }
+        }
+        const unsigned qb = __ballot_sync(full, lng);
+        if (lng) st.queue[qn + __popc(qb & ((1u << lane) - 1u))] = (uint16_t)(b + u);
+        qn += __popc(qb);
       }
     }
-  }
-  __syncthreads();
-  for (int c = threadIdx.x; c < ncell; c += kThreads) {
-    const int m = c & (Mp - 1);
-    if (m >= M) continue;
-    const int k = k_lo + (c >> lgMp);
-    const size_t g = (size_t)k * M + m;
-    if (SLO && k < K) {
-      const uint32_t s = st.aS[c];
-      if (s) atomicAdd(&slo[g], (unsigned long long)(s & 0xffffu) + ((unsigned long long)(s >> 16) << 32));
+    // walk the warp's long decodes, one record per lane
+    __syncwarp();
+    for (int i = lane; i < qn; i += 32) {
+      const int j = st.queue[i];
+      const int m = colp[0][j], tf = colp[3][j], te = colp[4][j], L = colp[6][j];
+      const int kf = (int)fd.div((uint32_t)tf), be_raw = (int)fd.div((uint32_t)te);
+      const uint32_t dur = (uint32_t)(te - tf);
+      unsigned long long qq, rr;
+      divmod((unsigned long long)((uint32_t)(kf + 1) * (uint32_t)win - (uint32_t)tf) *
+                 (uint32_t)(L - 1),
+             dur, qq, rr);
+      const uint32_t q1 = (uint32_t)qq, r1 = (uint32_t)rr;
+      {
+        // y = x + dur - 1 at the end of window kf: N = floor(y / dur), rem = y mod dur
+        uint32_t n = q1 + (r1 != 0);
+        uint32_t rem = r1 ? r1 - 1 : dur - 1;
+        unsigned long long Q64, R64;
+        divmod((unsigned long long)(uint32_t)win * (uint32_t)(L - 1), dur, Q64, R64);
+        const uint32_t Q = (uint32_t)Q64, R = (uint32_t)R64;   // Q < L: dur > win here
+        const int lo = st.far_lo[m];
+        const int k_full = min(be_raw - 1, K - 1);   // windows ending at or before t_end
+        const int k_end = min(be_raw, K - 1);
+        if ((uint32_t)(k_end - lo) < (uint32_t)F && kf + 1 >= lo) {
+          int32_t* fd_row = st.fD + m * F1 - lo;
+          for (int k = kf + 1; k <= k_full; ++k) {
+            const uint32_t t = rem + R;
+            const uint32_t c = t >= dur ? 1u : 0u;
+            rem = t - (c ? dur : 0u);
+            const uint32_t d = Q + c;
+            n += d;
+            if (d) atomicAdd(&fd_row[k], (int32_t)d);
+          }
+          if (be_raw <= K - 1 && (uint32_t)L != n) atomicAdd(&fd_row[be_raw], (int32_t)(L - n));
+        } else {
+          for (int k = kf + 1; k <= k_full; ++k) {
+            const uint32_t t = rem + R;
+            const uint32_t c = t >= dur ? 1u : 0u;
+            rem = t - (c ? dur : 0u);
+            const uint32_t d = Q + c;
+            n += d;
+            if (d) add_tok(st.fD, D, k, m, lo, (int32_t)d);
+          }
+          if (be_raw <= K - 1 && (uint32_t)L != n) add_tok(st.fD, D, be_raw, m, lo, (int32_t)(L - n));
+        }
+      }
     }
-    if (k <= K && st.aW[c]) atomicAdd(&dW[g], st.aW[c]);
-  }
-  for (int c = threadIdx.x; c < M * F; c += kThreads) {
-    const int m = c >> lgF;
-    const int lo = st.far_lo[m];
-    if (lo == 0x7fffffff) continue;
-    const int k = lo + (c & (F - 1));
-    const int cell = m * F1 + (c & (F - 1));
-    const size_t g = (size_t)k * M + m;
-    if (k < K) {
-      if (st.fP[cell]) atomicAdd(&P[g], st.fP[cell]);
-      if (st.fD[cell]) atomicAdd(&D[g], st.fD[cell]);
+    __syncthreads();
+    for (int c = threadIdx.x; c < ncell; c += kThreads) {
+      const int m = c & (Mp - 1);
+      if (m >= M) continue;
+      const int k = k_lo + (c >> lgMp);
+      const size_t g = (size_t)k * M + m;
+      if (SLO && k < K) {
+        const uint32_t s = st.aS[c];
+        if (s) atomicAdd(&slo[g], (unsigned long long)(s & 0xffffu) + ((unsigned long long)(s >> 16) << 32));
+      }
+      if (k <= K && st.aW[c]) atomicAdd(&dW[g], st.aW[c]);
     }
-    const int32_t aw = st.fAW[cell];
-    if (k <= K && aw) {
-      const int32_t a = (int32_t)(int16_t)(aw & 0xffff);
-      const int32_t w = (aw - a) / 65536;
-      if (a) atomicAdd(&dA[g], a);
-      if (w) atomicAdd(&dW[g], w);
+    for (int c = threadIdx.x; c < M * F; c += kThreads) {
+      const int m = c >> lgF;
+      const int lo = st.far_lo[m];
+      if (lo == 0x7fffffff) continue;
+      const int k = lo + (c & (F - 1));
+      const int cell = m * F1 + (c & (F - 1));
+      const size_t g = (size_t)k * M + m;
+      if (k < K) {
+        if (st.fP[cell]) atomicAdd(&P[g], st.fP[cell]);
+        if (st.fD[cell]) atomicAdd(&D[g], st.fD[cell]);
+      }
+      const int32_t aw = st.fAW[cell];
+      if (k <= K && aw) {
+        const int32_t a = (int32_t)(int16_t)(aw & 0xffff);
+        const int32_t w = (aw - a) / 65536;
+        if (a) atomicAdd(&dA[g], a);
+        if (w) atomicAdd(&dW[g], w);
+      }
     }
+    __syncthreads();   // the next slice reuses the shared memory
   }
   warp_add_counter(&diag->dropped_range, n_range);
   warp_add_counter(&diag->dropped_model, n_model);
@@ -1137,20 +1143,28 @@ cudaError_t launch_reduce_requests(const ReqCols* traces, int n_traces, int M, i
     if (e) return e;
   }
   const FastDiv fd(win);
+  // Records read over the host link: one CTA per slice would hold every SM for
+  // the length of the transfer. CTAs on two thirds of the SMs (two each) still
+  // keep the link busy -- a CTA spends most of a slice copying it in -- and
+  // leave the other SMs to work on other streams, such as the later phases of
+  // the step before.
+  const unsigned grid = copy_records
+                            ? (unsigned)std::min(ctas, 2 * std::max(1, device_sm_count() * 2 / 3))
+                            : (unsigned)ctas;
   if (slo && copy_records)
-    k_reduce_requests<true, true><<<ctas, kThreads, smem, s>>>(bt, M, lgMp, win, fd, K,
+    k_reduce_requests<true, true><<<grid, kThreads, smem, s>>>(bt, M, lgMp, win, fd, K,
                                                                near_rows, lgF, P, D, w.dA, w.dW,
                                                                slo, slo_ms, diag);
   else if (slo)
-    k_reduce_requests<true, false><<<ctas, kThreads, smem, s>>>(bt, M, lgMp, win, fd, K,
+    k_reduce_requests<true, false><<<grid, kThreads, smem, s>>>(bt, M, lgMp, win, fd, K,
                                                                 near_rows, lgF, P, D, w.dA, w.dW,
                                                                 slo, slo_ms, diag);
   else if (copy_records)
-    k_reduce_requests<false, true><<<ctas, kThreads, smem, s>>>(bt, M, lgMp, win, fd, K,
+    k_reduce_requests<false, true><<<grid, kThreads, smem, s>>>(bt, M, lgMp, win, fd, K,
                                                                 near_rows, lgF, P, D, w.dA, w.dW,
                                                                 nullptr, nullptr, diag);
   else
-    k_reduce_requests<false, false><<<ctas, kThreads, smem, s>>>(bt, M, lgMp, win, fd, K,
+    k_reduce_requests<false, false><<<grid, kThreads, smem, s>>>(bt, M, lgMp, win, fd, K,
                                                                  near_rows, lgF, P, D, w.dA, w.dW,
                                                                  nullptr, nullptr, diag);
   return cudaGetLastError();
