@@ -177,7 +177,7 @@ tre_status score_typed(const tre_grid* g, const tre_counts* in, const tre_profil
   if (st != TRE_OK || query) return st;
   cudaError_t e;
   {
-    Scope sc(kScore, 6, s);
+    Scope sc(kScore, score_launches(tab), s);
     e = launch_score<T>(tab, in->P, in->D, in->A, in->W, static_cast<const T*>(p->w_p),
                         static_cast<const T*>(p->w_q), static_cast<const T*>(p->alpha),
                         static_cast<const T*>(p->theta), static_cast<const T*>(p->tau_crit),
@@ -222,7 +222,7 @@ tre_status calibrate_typed(const tre_grid* g, const tre_requests* req, const tre
             : launch_slo_events(cols_of(ev), M, g->window_ms, K, slo, slo_ms, s);
   }
   if (!e) {
-    Scope sc(kScore, 6, s);
+    Scope sc(kScore, score_launches(tab), s);
     e = launch_score<T>(tab, in->P, in->D, in->A, in->W, static_cast<const T*>(p->w_p),
                         static_cast<const T*>(p->w_q), static_cast<const T*>(p->alpha), nullptr,
                         nullptr, nullptr, nullptr, nullptr, S, nullptr, cls, sw, diag, s,
@@ -274,7 +274,10 @@ tre_status select_typed(const tre_grid* g, const void* Z, const uint8_t* cls,
   tre_status st = ws_check(a, ws, ws_bytes, query);
   if (st != TRE_OK || query) return st;
   Scope sc(kSelect, 2, s);
-  return cuda_status(launch_walk<T>(b, w, s));
+  int n_launch = 0;
+  const cudaError_t e = launch_walk<T>(b, w, s, &n_launch);
+  sc.set_launches(n_launch);
+  return cuda_status(e);
 }
 
 // ---- tre_sweep --------------------------------------------------------------
@@ -482,7 +485,7 @@ tre_status sweep_typed(const tre_sweep_spec* sp, const SweepPlan& pl, const tre_
     }
   }
   if (!e) {
-    Scope sc(kScore, 6, s);
+    Scope sc(kScore, score_launches(tab), s);
     e = launch_score<T>(tab, P, D, A, W, static_cast<const T*>(sp->w_p),
                         static_cast<const T*>(sp->w_q), nullptr, nullptr, nullptr, nullptr,
                         nullptr, nullptr, S, nullptr, idle, sw, diag, s);
@@ -498,7 +501,10 @@ tre_status sweep_typed(const tre_sweep_spec* sp, const SweepPlan& pl, const tre_
   }
   if (e) return TRE_ECUDA;
   Scope sc(kSelect, 2, s);
-  return cuda_status(launch_walk<T>(b, wk, s));
+  int n_launch = 0;
+  const cudaError_t e2 = launch_walk<T>(b, wk, s, &n_launch);
+  sc.set_launches(n_launch);
+  return cuda_status(e2);
 }
 
 }  // namespace
@@ -543,7 +549,7 @@ tre_status stage_calibrate_typed(const tre_grid* g, const tre_requests* req, con
   if (!e) e = launch_fill<T>(ones, M, (T)1, s);
   // prefill: (P/dt) / max(A_prefill + w_q W, 1), calibrated on TTFT
   if (!e) {
-    Scope sc(kScore, 6, s);
+    Scope sc(kScore, score_launches(tab), s);
     e = launch_score<T>(tab, in->P, zero, A_pre, in->W, ones, w_q, alpha, nullptr, nullptr,
                         nullptr, nullptr, nullptr, S, nullptr, cls, sw, diag, s);
   }
@@ -553,7 +559,7 @@ tre_status stage_calibrate_typed(const tre_grid* g, const tre_requests* req, con
   }
   // decode: (D/dt) / max(A_decode, 1), calibrated on TPOT
   if (!e) {
-    Scope sc(kScore, 6, s);
+    Scope sc(kScore, score_launches(tab), s);
     e = launch_score<T>(tab, zero, in->D, A_dec, zero, w_p, w_q, alpha, nullptr, nullptr,
                         nullptr, nullptr, nullptr, S, nullptr, cls, sw, diag, s);
   }
@@ -588,13 +594,13 @@ tre_status stage_score_typed(const tre_grid* g, const tre_counts* in, const int3
   cudaError_t e = cudaMemsetAsync(zero, 0, cells * sizeof(int32_t), s);
   if (!e) e = launch_fill<T>(ones, M, (T)1, s);
   if (!e) {
-    Scope sc(kScore, 6, s);
+    Scope sc(kScore, score_launches(tab), s);
     e = launch_score<T>(tab, in->P, zero, A_pre, in->W, ones, w_q, alpha,
                         static_cast<const T*>(th_pre), tc, tsu, nullptr, nullptr,
                         static_cast<T*>(S_pre), static_cast<T*>(Z_pre), cls_pre, sw, diag, s);
   }
   if (!e) {
-    Scope sc(kScore, 6, s);
+    Scope sc(kScore, score_launches(tab), s);
     e = launch_score<T>(tab, zero, in->D, A_dec, zero, static_cast<const T*>(p->w_p), w_q,
                         alpha, static_cast<const T*>(th_dec), tc, tsu, nullptr, nullptr,
                         static_cast<T*>(S_dec), static_cast<T*>(Z_dec), cls_dec, sw, diag, s);
@@ -724,7 +730,7 @@ tre_status tss_window_reduce(const tre_grid* grid, const tre_requests* req, cons
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   cudaError_t e;
   {
-    Scope sc(kReduce, req ? 1 : 3, s);
+    Scope sc(kReduce, req ? 2 : 3, s);   // clearing + reduction; or three event passes
     const ReqCols rc = req ? cols_of(req) : ReqCols{};
     e = req ? launch_reduce_requests(&rc, 1, M, grid->window_ms, K, out.P, out.D, w, nullptr,
                                      nullptr, diag, s)

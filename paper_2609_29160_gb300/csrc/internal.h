@@ -61,6 +61,7 @@ class Scope {
   ~Scope();
   Scope(const Scope&) = delete;
   Scope& operator=(const Scope&) = delete;
+  void set_launches(int launches) { n = launches; }
 
  private:
   cudaStream_t s;
@@ -184,6 +185,8 @@ template <class T> void score_ws_layout(Arena& a, int M, int64_t elems, int n_se
 // of the table. Profile arrays are device [M]; alpha may be null (then the
 // table's per-series value is used); theta null = S only (cls = IDLE / NOM).
 // The carries (device [M], may be null) apply to a one-series table.
+// kernels one launch_score call issues (for the phase trace)
+template <class T> int score_launches(const SeriesTable<T>& tab);
 template <class T>
 cudaError_t launch_score(const SeriesTable<T>& tab, const int32_t* P, const int32_t* D,
                          const int32_t* A, const int32_t* W, const T* w_p, const T* w_q,
@@ -257,7 +260,9 @@ struct WalkWs {
 };
 // lays out the tick tables and fills b.ent_base
 template <class T> void walk_ws_layout(Arena& a, WalkBatch<T>& b, WalkWs& w);
-template <class T> cudaError_t launch_walk(const WalkBatch<T>& b, WalkWs& w, cudaStream_t s);
+// *launches (may be null): kernels it issued
+template <class T> cudaError_t launch_walk(const WalkBatch<T>& b, WalkWs& w, cudaStream_t s,
+                                          int* launches = nullptr);
 
 // ---- replay.cu ------------------------------------------------------------
 // Latent requests of a closed-loop replay (what a request needs once started).

@@ -75,7 +75,7 @@ tre_status run(const tre_grid* g, const tre_counts* in, const tre_profile* p, vo
   score_ws_layout<T>(a, M, elems, n_seg, w);
   cudaError_t e;
   {
-    Scope sc(kScore, 6, s);
+    Scope sc(kScore, score_launches(tab), s);
     e = launch_score<T>(tab, in->P, in->D, in->A, in->W, static_cast<const T*>(p->w_p),
                         static_cast<const T*>(p->w_q), static_cast<const T*>(p->alpha),
                         static_cast<const T*>(p->theta), static_cast<const T*>(p->tau_crit),

@@ -954,6 +954,10 @@ template <class T> void score_ws_layout(Arena& a, int M, int64_t elems, int n_se
   w.active = a.take<int32_t>(n);
 }
 
+template <class T> int score_launches(const SeriesTable<T>& tab) {
+  return (total_elems(tab) >= kActiveMinCells ? 1 : 0) + 3;
+}
+
 template <class T>
 cudaError_t launch_score(const SeriesTable<T>& tab, const int32_t* P, const int32_t* D,
                          const int32_t* A, const int32_t* W, const T* w_p, const T* w_q,
@@ -1046,6 +1050,7 @@ cudaError_t launch_rank(int M, int K, const T* Z, const uint8_t* cls, int32_t* r
 
 #define TRE_INST(T)                                                                               \
   template int series_segments<T>(SeriesTable<T>&);                                               \
+  template int score_launches<T>(const SeriesTable<T>&);                                          \
   template void score_ws_layout<T>(Arena&, int, int64_t, int, ScoreWs<T>&);                       \
   template cudaError_t launch_score<T>(const SeriesTable<T>&, const int32_t*, const int32_t*,      \
                                        const int32_t*, const int32_t*, const T*, const T*,         \

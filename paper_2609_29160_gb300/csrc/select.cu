@@ -1471,7 +1471,9 @@ cudaError_t walk_thread_launch(const WalkBatch<T>& b, WalkWs& w, size_t smem, cu
   return cudaGetLastError();
 }
 
-template <class T> cudaError_t launch_walk(const WalkBatch<T>& b, WalkWs& w, cudaStream_t s) {
+template <class T>
+cudaError_t launch_walk(const WalkBatch<T>& b, WalkWs& w, cudaStream_t s, int* launches) {
+  if (launches) *launches = 0;
   if (b.n_inst == 0) return cudaSuccess;
   const int64_t ents = (int64_t)b.ent_base[b.n_series] * b.n_tau;
   // which walk runs decides whether the per-model rank tables are needed
@@ -1480,23 +1482,24 @@ template <class T> cudaError_t launch_walk(const WalkBatch<T>& b, WalkWs& w, cud
     max_ent = std::max(max_ent, b.ent_base[i + 1] - b.ent_base[i]);
   const size_t thread_smem = (size_t)max_ent * (8 + 4 + 2) + 16;
   const bool thread_walk = b.M <= 16 && b.n_cap <= 32 && thread_smem <= kStageMax;
+  // rows start on 16-byte boundaries when M is a multiple of 4 (series
+  // offsets are multiples of M) and both arrays are 16-byte aligned
   const bool quad = b.M % 4 == 0 && (((uintptr_t)b.Z | (uintptr_t)b.cls) & 15) == 0;
   JumpPlan jp{false, false, 0, 0};
   if (thread_walk && ents > 0) jp = b.M <= 8 ? jump_plan<T, 8>(b) : jump_plan<T, 16>(b);
   // with a CTA per SM or more, the jump walk ranks its own ticks: one launch
   if (jp.ok && b.n_series * b.n_tau >= device_sm_count()) {
+    if (launches) *launches = 1;
     if (b.M <= 8)
       return quad ? jump_launch<T, 8, true, true>(b, w, jp, s)
                   : jump_launch<T, 8, true, false>(b, w, jp, s);
     return quad ? jump_launch<T, 16, true, true>(b, w, jp, s)
                 : jump_launch<T, 16, true, false>(b, w, jp, s);
   }
+  // the tick ranking, then the walk
+  if (launches) *launches = (ents > 0 ? 1 : 0) + 1;
   if (ents > 0) {
     const unsigned g = (unsigned)((ents + 127) / 128);
-    // rows start on 16-byte boundaries when M is a multiple of 4 (series
-    // offsets are multiples of M) and both arrays are 16-byte aligned
-    const bool quad =
-        b.M % 4 == 0 && (((uintptr_t)b.Z | (uintptr_t)b.cls) & 15) == 0;
     if (b.M <= 8 && quad) {
       k_tick_rank_small<T, 8, true><<<g, 128, 0, s>>>(b, w.recv, w.n_donor, w.rank, w.order,
                                                       w.packed, w.dmask, !thread_walk, w.dm64);
@@ -1532,7 +1535,7 @@ template <class T> cudaError_t launch_walk(const WalkBatch<T>& b, WalkWs& w, cud
 
 template void walk_ws_layout<float>(Arena&, WalkBatch<float>&, WalkWs&);
 template void walk_ws_layout<double>(Arena&, WalkBatch<double>&, WalkWs&);
-template cudaError_t launch_walk<float>(const WalkBatch<float>&, WalkWs&, cudaStream_t);
-template cudaError_t launch_walk<double>(const WalkBatch<double>&, WalkWs&, cudaStream_t);
+template cudaError_t launch_walk<float>(const WalkBatch<float>&, WalkWs&, cudaStream_t, int*);
+template cudaError_t launch_walk<double>(const WalkBatch<double>&, WalkWs&, cudaStream_t, int*);
 
 }  // namespace tre
