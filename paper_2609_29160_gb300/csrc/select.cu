@@ -989,7 +989,10 @@ k_walk_jump(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab,
   // backwards from the first acting tick of the segments after it
   constexpr int NC = MMAX + 1;
   const int n_seg = (int)blockDim.x / NC;              // segments per column
-  const int seg_len = (nf + n_seg - 1) / n_seg;
+  // a segment length of 1 mod 8 puts the segments' tick records (16 bytes, so
+  // 8 to a bank cycle) of one step on different banks
+  int seg_len = (nf + n_seg - 1) / n_seg;
+  seg_len += (9 - seg_len % 8) % 8;
   __shared__ int s_first[256];                         // [NC][n_seg]
   const int my_c = threadIdx.x / n_seg, my_s = threadIdx.x % n_seg;
   const bool has_seg = my_c < NC;
