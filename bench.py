@@ -295,7 +295,7 @@ def cpu_baseline_parallel(scale, seed0):
 
 # ---------------------------------------------------------------------------
 # The single-trace workloads: one pass of the whole path per step
-# (tss_window_reduce -> tss_calibrate -> tss_score -> tre_select_moves).
+# (tss_window_reduce -> tss_calibrate -> tss_normalize -> tre_select_moves).
 # ---------------------------------------------------------------------------
 CONFIGS = (
     # (key, workload name, dtypes, timed steps, oracle sample: fraction of the

@@ -1,5 +1,5 @@
 """GPU parity at the workloads' full sizes, in the launch configuration the
-benchmark times (one marshalled pass of reduce -> calibrate -> score -> select
+benchmark times (one marshalled pass of reduce -> calibrate -> normalize -> select
 per trace, and the batched sweep), against the oracle on the same seeded
 inputs, bit for bit: counts and drops, theta, S, Z, regions, receivers, moves
 and final replicas.
