@@ -923,6 +923,9 @@ k_gauge_block_scan(const __grid_constant__ GaugePlan gp, int32_t* __restrict__ p
   }
 }
 
+// NW: the most window lengths the launch serves (their running sums live in
+// registers; four cover the sweep's usual lengths with fewer registers)
+template <int NW>
 __global__ void __launch_bounds__(kThreads)
 k_gauge_apply(const __grid_constant__ GaugePlan gp, const int32_t* __restrict__ dA,
               const int32_t* __restrict__ dW, const int32_t* __restrict__ pA,
@@ -930,7 +933,6 @@ k_gauge_apply(const __grid_constant__ GaugePlan gp, const int32_t* __restrict__ 
               const int32_t* __restrict__ Din, const unsigned long long* __restrict__ sloin,
               int32_t* __restrict__ P, int32_t* __restrict__ D, int32_t* __restrict__ A,
               int32_t* __restrict__ W, unsigned long long* __restrict__ slo) {
-  constexpr int NW = kGaugeMaxWin;
   constexpr int RB = 4;   // rows whose loads are issued together
   const int M = gp.M, Kb = gp.Kb;
   const int64_t t = (int64_t)blockIdx.x * kThreads + threadIdx.x;
@@ -1588,8 +1590,13 @@ cudaError_t launch_gauge_apply(const GaugePlan& gp, ReduceWs& w, const int32_t* 
                                cudaStream_t s) {
   const int64_t n = (int64_t)gp.n_traces * gp.nblk * gp.M;
   if (n == 0) return cudaSuccess;
-  k_gauge_apply<<<(unsigned)((n + kThreads - 1) / kThreads), kThreads, 0, s>>>(
-      gp, w.dA, w.dW, w.partA, w.partW, Pin, Din, sloin, P, D, A, W, slo);
+  const unsigned g = (unsigned)((n + kThreads - 1) / kThreads);
+  if (gp.n_win <= 4)
+    k_gauge_apply<4><<<g, kThreads, 0, s>>>(gp, w.dA, w.dW, w.partA, w.partW, Pin, Din, sloin,
+                                            P, D, A, W, slo);
+  else
+    k_gauge_apply<kGaugeMaxWin><<<g, kThreads, 0, s>>>(gp, w.dA, w.dW, w.partA, w.partW, Pin, Din,
+                                                       sloin, P, D, A, W, slo);
   return cudaGetLastError();
 }
 
