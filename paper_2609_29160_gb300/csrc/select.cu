@@ -333,17 +333,20 @@ __device__ __forceinline__ int lane_of_min_rank(const uint16_t (&rk)[MPL], const
   return src;
 }
 
-// One CTA per (series, tau), one warp per pacing cap: the warps share the
-// tick tables of their (series, tau), staged in shared memory when they fit.
+// One CTA per (series, tau) and group of up to kCapWarps pacing caps, one warp
+// per cap: the warps share the tick tables of their (series, tau), staged in
+// shared memory when they fit. (Eight warps a CTA leave each thread the
+// registers the walk's state needs.)
+constexpr int kCapWarps = 8;
 template <class T, int MPL, bool STAGED>
-__global__ void __launch_bounds__(kMaxCap * 32)
+__global__ void __launch_bounds__(kCapWarps * 32)
 k_walk(const __grid_constant__ WalkBatch<T> b, const int16_t* recv_tab, const int16_t* ndon_tab,
        const uint16_t* rank, const uint16_t* order, const unsigned long long* dm64) {
   extern __shared__ __align__(16) unsigned char dyn[];
   const int grp = blockIdx.x;                       // (series, tau)
   const int ti = grp % b.n_tau;
   const int si = grp / b.n_tau;
-  const int ci = threadIdx.x / 32;                  // pacing cap index
+  const int ci = blockIdx.y * kCapWarps + threadIdx.x / 32;   // pacing cap index
   const int lane = threadIdx.x & 31;
   const int M = b.M;
   const int K = b.series_K[si];
@@ -1384,8 +1387,9 @@ cudaError_t walk_launch(const WalkBatch<T>& b, WalkWs& w, cudaStream_t s) {
   for (int i = 0; i < b.n_series; ++i) max_ent = std::max(max_ent, b.ent_base[i + 1] - b.ent_base[i]);
   const size_t smem = 2 * (((size_t)max_ent * 2 + 15) & ~(size_t)15) +
                       2 * (((size_t)max_ent * b.M * 2 + 15) & ~(size_t)15);
-  const unsigned grid = (unsigned)(b.n_series * b.n_tau);
-  const unsigned th = (unsigned)(b.n_cap * 32);
+  const dim3 grid((unsigned)(b.n_series * b.n_tau),
+                  (unsigned)((b.n_cap + kCapWarps - 1) / kCapWarps));
+  const unsigned th = (unsigned)(std::min(b.n_cap, kCapWarps) * 32);
   if (smem <= kStageMax) {
     cudaError_t e = func_smem_once((const void*)k_walk<T, MPL, true>, (int)kStageMax, false);
     if (e) return e;

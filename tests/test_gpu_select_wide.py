@@ -115,9 +115,11 @@ def test_pacing_cap_above_thirty_two(tre, M):
     _check(tre, Z, cls, g, r0, budget, r_min, 1000, 40)
 
 
-def test_sweep_twenty_four_models(tre):
+@pytest.mark.parametrize("caps", [None, list(range(1, 13))])
+def test_sweep_twenty_four_models(tre, caps):
     """The sweep's walk launch with more than 16 models: one warp per
-    (trace, window length, rescue threshold, pacing cap) instance."""
+    (trace, window length, rescue threshold, pacing cap) instance, eight
+    caps to a block (twelve caps: two blocks per (series, threshold))."""
     import tracegen
     sw = tracegen.sweep_workload(scale=0.02, n_traces=1, duration_s=600.0)
     rng = np.random.default_rng(8)
@@ -131,7 +133,8 @@ def test_sweep_twenty_four_models(tre):
             sw[k] = ext(sw[k]).astype(np.asarray(sw[k]).dtype)
     sw["budget"] = int(sw["r0"].sum()) + 2
     sw["tau_crit"] = sw["tau_crit"][::3]
-    sw["pacing_cap"] = sw["pacing_cap"][::3]
+    sw["pacing_cap"] = (sw["pacing_cap"][::3] if caps is None
+                        else np.asarray(caps, dtype=np.asarray(sw["pacing_cap"]).dtype))
     alpha = [min(1.0, w / 5000.0) for w in sw["window_ms"]]
     import torch
     ref = oracle.sweep(sw["traces"], M, sw["duration_ms"], sw["window_ms"], sw["tau_crit"],
